@@ -1,0 +1,215 @@
+/*
+ * msd.h - C ABI of the GB300 (sm_103a) hot path of Multimodal Speculative
+ * Decoding (MSD, arXiv 2505.14260): one greedy draft -> verify -> accept ->
+ * compact decode step of a LLaVA-style decoder.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ * - All pointers named *_dev are device pointers on the device that was
+ *   current when msd_create ran; *_host pointers are host memory. Sizes are
+ *   element counts unless stated otherwise.
+ * - Weight matrices are [out, in] row-major (in contiguous), in the dtype of
+ *   msd_config.dtype; norm gains are [hidden] vectors of the same dtype.
+ *   Weights are BORROWED: the caller keeps them alive and unchanged for the
+ *   lifetime of the context.
+ * - The context OWNS its KV caches, tree scratch and activations (allocated
+ *   once in msd_create; no call allocates afterwards).
+ * - Output buffers are caller-owned device memory.
+ * - Every call is asynchronous on `stream` (a cudaStream_t, 0 = legacy default
+ *   stream). Argument, shape and capacity errors are returned synchronously
+ *   before anything is launched. Device-detected errors (bounded waits that
+ *   timed out, failed in-kernel range checks) set a device status word; the
+ *   first call that observes it returns MSD_ERR_DEVICE.
+ * - One context is used from one host thread and one stream at a time.
+ * - Token ids are int32 in [0, vocab). Trees are stored per request with a
+ *   fixed stride of N = msd_config.tree_nodes nodes; node 0 is the root.
+ *
+ * Notation (paper): L = tokens in the target KV cache (positions 0..L-1); the
+ * root token x_L sits at position L; N tree nodes including the root; depth D
+ * (number of draft passes); top-k k.
+ */
+#ifndef MSD_H
+#define MSD_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef struct msd_ctx msd_ctx;
+
+typedef enum {
+    MSD_OK = 0,
+    MSD_ERR_INVALID = -1,   /* bad argument, shape or state */
+    MSD_ERR_CAPACITY = -2,  /* a request would exceed max_seq */
+    MSD_ERR_OOM = -3,       /* device allocation failed in msd_create */
+    MSD_ERR_CUDA = -4,      /* a CUDA runtime call failed */
+    MSD_ERR_DEVICE = -5     /* the device status word was set by a kernel */
+} msd_status;
+
+enum { MSD_F32 = 0, MSD_BF16 = 1 };
+
+/* Model and capacity. The target is a pre-norm LLaMA-style decoder (the LLM of
+ * LLaVA-1.5, Sec. 3.1); the draft model is one decoder layer of the same shape
+ * plus the fc projection f_down of Eq. 4 (Sec. 3.2). */
+typedef struct {
+    int32_t n_layers, hidden, n_heads, head_dim, ffn, vocab;
+    float rms_eps, rope_base;
+    int32_t dtype;          /* MSD_F32 or MSD_BF16: weights, KV cache, GEMM operands */
+    int32_t max_batch;      /* B: requests decoded together */
+    int32_t max_seq;        /* cache capacity per request, in positions */
+    int32_t tree_nodes;     /* N, including the root; 1 <= N <= 256 */
+    int32_t tree_depth;     /* D >= 1: draft passes per step */
+    int32_t topk;           /* k >= 1; k + (D-1)k^2 >= N-1 */
+} msd_config;
+
+/* One decoder layer: RMSNorm gains [H]; wq, wk, wv, wo [H,H];
+ * w_gate, w_up [F,H]; w_down [H,F]. */
+typedef struct {
+    const void *attn_norm, *wq, *wk, *wv, *wo, *mlp_norm, *w_gate, *w_up, *w_down;
+} msd_layer;
+
+/* All weights (device pointers). `layers` is a HOST array of n_layers entries
+ * (copied by msd_create). embed and lm_head are [V,H] (untied); draft_fc is the
+ * [H, 2H] f_down of Eq. 4, applied to Concat(h, e) in that order. */
+typedef struct {
+    const void *embed;
+    const msd_layer *layers;
+    const void *final_norm;
+    const void *lm_head;
+    msd_layer draft;
+    const void *draft_fc;
+} msd_weights;
+
+/* A token tree, device memory, per request b at stride N:
+ * tokens[b*N+i], parent[b*N+i] (-1 for the root, else < i), depth[b*N+i],
+ * mask[(b*N+i)*W + w] with W = ceil(N/64): bit j%64 of word j/64 is set iff
+ * node j is an ancestor of node i or j == i. n_nodes[b] (nullable: all N) is the
+ * number of valid nodes of request b. */
+typedef struct {
+    int32_t *tokens, *parent, *depth;
+    uint64_t *mask;
+    int32_t *n_nodes;
+} msd_tree;
+
+/* Optional record of the draft passes (device, all nullable), for parity checks.
+ * Pass p = 0 is the root slot (one row per request, row 0 used); passes
+ * p = 1..D-1 have k rows per request (the expanded frontier, best first).
+ *   logits    [B][D][k][V] fp32  draft LM-head logits of each row
+ *   topk_ids  [B][D][k][k] int32 top-k token ids of each row (ties: lower id)
+ *   topk_logp [B][D][k][k] fp32  their log-probabilities                   */
+typedef struct {
+    float *logits;
+    int32_t *topk_ids;
+    float *topk_logp;
+} msd_draft_record;
+
+/* Device-side view of the context state, for tests and tooling. Layouts:
+ *   target_kv  [n_layers][2][B][n_heads][max_seq][head_dim]   (K then V, K after RoPE)
+ *   draft_kv   [2][B][n_heads][max_seq][head_dim]
+ *   seq_len    int32 [B]  L of each request
+ *   n_pending  int32 [B]  draft rows still to be caught up (draft cache = L - n_pending)
+ *   root       int32 [B]  current root token x_L                                  */
+typedef struct {
+    void *target_kv, *draft_kv;
+    int32_t *seq_len, *n_pending, *root;
+    int64_t elem_bytes;
+} msd_state_view;
+
+/* Creates a context on the current device: validates the configuration,
+ * copies the weight pointer table, allocates caches and scratch.
+ * Errors: MSD_ERR_INVALID (bad config or null weight), MSD_ERR_OOM. */
+msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out);
+
+/* Frees everything the context owns. Safe on NULL. */
+msd_status msd_destroy(msd_ctx *ctx);
+
+/* Prefill (Sec. 3.1, Eq. 1-3; draft input of Eq. 7). For each request b <
+ * batch: ids_dev[b*ids_stride + i], i < seq_len_host[b], is the interleaved
+ * prompt, with -1 marking a visual slot; visual slots consume rows of
+ * vis_dev ([rows][H], model dtype) in order starting at row vis_off_host[b].
+ * Runs the target over the prompt (filling its KV cache), writes the root token
+ * x_L = argmax of the last position's logits to root_out_dev[b], and builds the
+ * draft cache over positions 0..L-2 with f = e at visual positions and
+ * f = f_down(Concat(h, e_next)) at text positions (Eq. 7).
+ * Errors: MSD_ERR_INVALID (batch out of range, empty prompt, prompt not ending
+ * in a text token), MSD_ERR_CAPACITY (L + 1 + N > max_seq). Resets all state. */
+msd_status msd_prefill(msd_ctx *ctx, int32_t batch, const int32_t *seq_len_host,
+                       const int32_t *ids_dev, int32_t ids_stride,
+                       const void *vis_dev, const int64_t *vis_off_host,
+                       int32_t *root_out_dev, void *stream);
+
+/* Draft tree (Sec. 3.2 feature-level draft phase, Eq. 4-5, with the MSD input
+ * of Eq. 7). Pass 1 catches the draft cache up over the positions accepted by
+ * the last step (root slot last) and gives the depth-1 candidates (top-k of the
+ * root slot's distribution); passes 2..D expand the k best frontier nodes with
+ * top-k children each, score = sum of log-probabilities; the N-1 best
+ * candidates form the tree (index 1 + rank; ties: higher score, lower depth,
+ * earlier creation). Writes the tree to *out (caller-owned device arrays of
+ * the layout above; n_nodes, if given, is set to N). rec is nullable. */
+msd_status msd_draft_tree(msd_ctx *ctx, const msd_tree *out,
+                          const msd_draft_record *rec, void *stream);
+
+/* Verify (Sec. 3.2 verification phase): one target forward over all tree
+ * tokens, node i at position L + depth(i), attending to the whole prefix and to
+ * its ancestors and itself. `tree` is the drafted tree or any caller-planted
+ * tree with tokens[b*N] == the current root. Writes the target argmax of every
+ * node to argmax_dev[b*N+i] (ties: lower id) and, if logits_dev is not NULL,
+ * the fp32 logits [B][N][V]. Tree K/V are kept in context scratch for
+ * msd_accept_compact. */
+msd_status msd_verify(msd_ctx *ctx, const msd_tree *tree, int32_t *argmax_dev,
+                      float *logits_dev, void *stream);
+
+/* Accept and compact (Eq. 6 at temperature 0, and the rule that rejected
+ * drafts are discarded): from the root, follow the child whose token equals the
+ * target argmax at the current node; path_dev[b*(D+1)+j] (j <= a, rest -1),
+ * accept_len_dev[b] = a, bonus_dev[b] = argmax at the last accepted node. The
+ * K/V of path[j] move to cache position L+j; L <- L + a + 1; the bonus becomes
+ * the new root. index_map_dev (nullable) [b*(D+1)+j] = L_old + j for j <= a,
+ * else -1. `tree` and `argmax_dev` must be those of the preceding msd_verify. */
+msd_status msd_accept_compact(msd_ctx *ctx, const msd_tree *tree,
+                              const int32_t *argmax_dev, int32_t *path_dev,
+                              int32_t *accept_len_dev, int32_t *bonus_dev,
+                              int32_t *index_map_dev, void *stream);
+
+/* Building block used by every projection of the step (Sec. 3.1 decoder
+ * layers, Eq. 4 f_down, Eq. 5 LM head), exposed for tests and kernel timing:
+ * y[i][j] (= or, if accumulate != 0, +=) sum_t x[i][t] * w[j][t] for i < m,
+ * j < o, t < k. x [m][ldx] and w [o][k] are in the context dtype (bf16 rows
+ * 16-byte aligned: ldx and k multiples of 8), y [m][ldy] is fp32; all device.
+ * bf16 runs on the tcgen05 tensor-core GEMM, fp32 on the CUDA-core GEMM.
+ * Errors: MSD_ERR_INVALID on null pointers, non-positive sizes or bad strides. */
+msd_status msd_linear(msd_ctx *ctx, const void *x_dev, int32_t ldx, int32_t m, int32_t k,
+                      const void *w_dev, int32_t o, float *y_dev, int32_t ldy,
+                      int32_t accumulate, void *stream);
+
+/* Profiling counters (tracing subsystem). kernel_launches counts every kernel
+ * the library has launched in this process. While profiling is enabled on a
+ * context, each tensor-core GEMM launch (bf16 contexts) is bracketed by CUDA
+ * events on its own stream; msd_profile_read synchronises on them and returns
+ * the number of timed launches, their summed durations, and their algorithmic
+ * bytes (every weight element once + activations read + fp32 output written,
+ * read too when accumulating), then starts a new window. */
+typedef struct {
+    int64_t kernel_launches;
+    int64_t gemm_launches;
+    double gemm_ms;
+    double gemm_bytes;
+    double gemm_weight_bytes;
+} msd_profile;
+
+msd_status msd_profile_enable(msd_ctx *ctx, int32_t on);
+msd_status msd_profile_read(msd_ctx *ctx, msd_profile *out);
+
+/* Device pointers of the context state (see msd_state_view). */
+msd_status msd_state(msd_ctx *ctx, msd_state_view *out);
+
+/* Text of the last error on this context ("" if none). Never NULL. */
+const char *msd_last_error(const msd_ctx *ctx);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* MSD_H */

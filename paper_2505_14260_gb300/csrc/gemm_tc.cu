@@ -1,0 +1,513 @@
+// bf16 GEMM for the decode step on the sm_103a tensor cores.
+//
+// Decode GEMMs multiply a few token rows (M = 7 .. 960) by large weight
+// matrices, so they stream weights from HBM. The kernel swaps operands: a
+// 128-row weight tile is the MMA's A operand (M = 128) and the token rows are
+// its B operand (N = 16 .. 256), so the accumulator D^T[128 weight rows][N
+// tokens] sits in TMEM, one weight row per TMEM lane.
+//
+// Per CTA (128 threads):
+//   warp 0 lane 0  TMA producer: 128x64 weight tile + Nx64 token tile per
+//                  stage, 128-byte swizzle, completion on a full[] mbarrier
+//   warp 1         allocates TMEM; lane 0 issues tcgen05.mma (K = 16 per
+//                  instruction, 4 per stage) and frees stages via
+//                  tcgen05.commit -> empty[]
+//   all 4 warps    epilogue: tcgen05.ld of their 32 TMEM lanes, fp32 store
+//                  or accumulate into Y (coalesced along the output dim)
+// Split-K: when there are too few weight tiles to cover the SMs, K is split;
+// every split writes its fp32 partial to a workspace and the last CTA to
+// finish a tile (atomic counter) sums the partials in split order, so results
+// are deterministic, and resets the counter. No CTA waits on another.
+// Every mbarrier wait is bounded (2 s of %globaltimer); on timeout the CTA
+// sets the device status word and winds down.
+#include <cuda.h>
+#include <cudaTypedefs.h>
+
+#include <cstdio>
+#include <cstring>
+#include <unordered_map>
+#include <vector>
+
+#include "gemm_tc.h"
+
+namespace msd {
+
+namespace {
+
+constexpr int BM = 128;          // weight rows per tile (MMA M)
+constexpr int BK = 64;           // K per stage: one 128-byte swizzle row of bf16
+constexpr int THREADS = 128;
+constexpr int MAX_STAGES = 8;
+constexpr uint32_t A_BYTES = BM * BK * 2;          // 16 KB
+constexpr unsigned long long TIMEOUT_NS = 2000000000ull;
+constexpr size_t WS_BYTES = 64ull << 20;
+constexpr int N_COUNTERS = 16384;
+
+struct TcParams {
+    int n_seg;
+    int seg_tiles[3];
+    int seg_rows[3];
+    int seg_out[3];
+    int M, kblocks, splits, kb_per_split, BN, n_tiles_n, stages, tmem_cols;
+    float *Y;
+    int ldy, epi;
+    float *ws;
+    int *counters;
+    int *status;
+};
+
+__device__ __forceinline__ uint32_t smem_u32(const void *p) {
+    return (uint32_t)__cvta_generic_to_shared(p);
+}
+
+__device__ __forceinline__ unsigned long long gtimer() {
+    unsigned long long t;
+    asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+    return t;
+}
+
+__device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+
+__device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n.reg .pred p;\n"
+        "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "selp.b32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait for the phase with the given parity to complete.
+__device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag, int *status) {
+    if (mbar_try(bar, parity)) return true;
+    const unsigned long long t0 = gtimer();
+    while (true) {
+        if (mbar_try(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (gtimer() - t0 > TIMEOUT_NS) {
+            *abort_flag = 1;
+            set_status(status, ST_TIMEOUT);
+            return false;
+        }
+    }
+}
+
+__device__ __forceinline__ void mbar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes)
+                 : "memory");
+}
+
+__device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                            uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(map), "r"(x), "r"(y), "r"(bar)
+        : "memory");
+}
+
+// Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row
+// core-matrix groups 1024 bytes apart, sm100 descriptor version 1.
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)1 << 16) |
+           ((uint64_t)(1024 >> 4) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
+}
+
+// Instruction descriptor, kind::f16: fp32 accumulate, bf16 A and B, both
+// K-major, N = BN, M = 128.
+__device__ __forceinline__ uint32_t instr_desc(int BN) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
+           ((uint32_t)(BM >> 4) << 24);
+}
+
+__device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc,
+                                         uint32_t accumulate) {
+    asm volatile(
+        "{\n.reg .pred p;\n"
+        "setp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile(
+        "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
+__global__ void __launch_bounds__(THREADS, 1)
+    gemm_tc_kernel(const __grid_constant__ CUtensorMap mw0, const __grid_constant__ CUtensorMap mw1,
+                   const __grid_constant__ CUtensorMap mw2, const __grid_constant__ CUtensorMap mx,
+                   const TcParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t bars[2 * MAX_STAGES + 1];
+    __shared__ uint32_t tmem_base;
+    __shared__ volatile int abort_flag;
+    __shared__ int is_last;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int tile = blockIdx.x, seg = 0;
+    while (seg < p.n_seg - 1 && tile >= p.seg_tiles[seg]) {
+        tile -= p.seg_tiles[seg];
+        ++seg;
+    }
+    const CUtensorMap *mw = seg == 0 ? &mw0 : (seg == 1 ? &mw1 : &mw2);
+    const int row0 = tile * BM;
+    const int ntile = blockIdx.y, n0 = ntile * p.BN;
+    const int split = blockIdx.z;
+    const int kb0 = split * p.kb_per_split;
+    const int kb1 = min(p.kblocks, kb0 + p.kb_per_split);
+    const int nk = kb1 - kb0;
+    const int stages = p.stages;
+    const uint32_t b_bytes = (uint32_t)p.BN * BK * 2;
+
+    const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+    const uint32_t a_base = sbase, b_base = sbase + stages * A_BYTES;
+    const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[MAX_STAGES]);
+    const uint32_t done = smem_u32(&bars[2 * MAX_STAGES]);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < stages; ++s) {
+            mbar_init(full0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        mbar_init(done, 1);
+        abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(mw) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(&tmem_base)),
+                     "r"(p.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            int issued = 0;
+            for (int i = 0; i < nk; ++i) {
+                const int s = i % stages;
+                const uint32_t ph = (uint32_t)(i / stages) & 1u;
+                if (!mbar_wait(empty0 + 8 * s, ph ^ 1u, &abort_flag, p.status)) break;
+                mbar_expect_tx(full0 + 8 * s, A_BYTES + b_bytes);
+                tma_load_2d(a_base + s * A_BYTES, mw, (kb0 + i) * BK, row0, full0 + 8 * s);
+                tma_load_2d(b_base + s * b_bytes, &mx, (kb0 + i) * BK, n0, full0 + 8 * s);
+                issued = i + 1;
+            }
+            if (abort_flag) {
+                // let the copies still in flight land before the CTA exits
+                volatile int never = 0;
+                for (int i = (issued > stages ? issued - stages : 0); i < issued; ++i)
+                    mbar_wait(full0 + 8 * (i % stages), (uint32_t)(i / stages) & 1u, &never,
+                              p.status);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        if (lane == 0) {
+            const uint32_t idesc = instr_desc(p.BN);
+            for (int i = 0; i < nk; ++i) {
+                const int s = i % stages;
+                const uint32_t ph = (uint32_t)(i / stages) & 1u;
+                if (!mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status)) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint64_t ad = smem_desc(a_base + s * A_BYTES);
+                const uint64_t bd = smem_desc(b_base + s * b_bytes);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)
+                    mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (i | kk) != 0);
+                mma_commit(empty0 + 8 * s);
+            }
+            mma_commit(done);   // arrives once every MMA issued above has completed
+        }
+        __syncwarp();
+    }
+
+    // ---- epilogue -----------------------------------------------------------
+    const bool ok = mbar_wait(done, 0, &abort_flag, p.status) && !abort_flag;
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const int row = warp * 32 + lane;
+    const int o_local = row0 + row;
+    const bool row_ok = o_local < p.seg_rows[seg];
+    const int o = p.seg_out[seg] + o_local;
+    const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
+    const int M = p.M;
+
+    if (p.splits == 1) {
+        for (int c0 = 0; c0 < p.BN; c0 += 16) {
+            uint32_t r[16];
+            tmem_ld16(taddr + c0, r);
+            if (ok && row_ok) {
+#pragma unroll
+                for (int j = 0; j < 16; ++j) {
+                    const int m = n0 + c0 + j;
+                    if (m < M) {
+                        float *y = p.Y + (size_t)m * p.ldy + o;
+                        const float v = __uint_as_float(r[j]);
+                        *y = p.epi == EPI_ADD ? *y + v : v;
+                    }
+                }
+            }
+        }
+    } else {
+        const int tile_id = blockIdx.x * p.n_tiles_n + ntile;
+        const size_t tile_elems = (size_t)p.BN * BM;
+        float *part = p.ws + ((size_t)tile_id * p.splits + split) * tile_elems;
+        for (int c0 = 0; c0 < p.BN; c0 += 16) {
+            uint32_t r[16];
+            tmem_ld16(taddr + c0, r);
+#pragma unroll
+            for (int j = 0; j < 16; ++j) part[(size_t)(c0 + j) * BM + row] = __uint_as_float(r[j]);
+        }
+        __threadfence();
+        __syncthreads();
+        if (threadIdx.x == 0) {
+            const int prev = atomicAdd(&p.counters[tile_id], 1);
+            is_last = prev == p.splits - 1;
+        }
+        __syncthreads();
+        if (is_last) {
+            __threadfence();
+            const float *tb = p.ws + (size_t)tile_id * p.splits * tile_elems;
+            for (int c = 0; c < p.BN; ++c) {
+                const int m = n0 + c;
+                if (m >= M) break;
+                float v = 0.f;
+                for (int s = 0; s < p.splits; ++s)
+                    v += __ldcg(tb + (size_t)s * tile_elems + (size_t)c * BM + row);
+                if (ok && row_ok) {
+                    float *y = p.Y + (size_t)m * p.ldy + o;
+                    *y = p.epi == EPI_ADD ? *y + v : v;
+                }
+            }
+            if (threadIdx.x == 0) p.counters[tile_id] = 0;
+        }
+    }
+
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(p.tmem_cols)
+                     : "memory");
+    }
+}
+
+struct MapKey {
+    const void *ptr;
+    long rows, cols, ld, box_rows;
+    bool operator==(const MapKey &o) const {
+        return ptr == o.ptr && rows == o.rows && cols == o.cols && ld == o.ld &&
+               box_rows == o.box_rows;
+    }
+};
+struct MapKeyHash {
+    size_t operator()(const MapKey &k) const {
+        size_t h = std::hash<const void *>()(k.ptr);
+        h ^= std::hash<long>()(k.rows * 1315423911L + k.cols * 2654435761L + k.ld * 97 + k.box_rows);
+        return h;
+    }
+};
+
+}  // namespace
+
+struct GemmPlan {
+    float *ws = nullptr;
+    int *counters = nullptr;
+    int num_sms = 148;
+    PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
+    std::unordered_map<MapKey, CUtensorMap, MapKeyHash> maps;
+    bool smem_set = false;
+    bool profile = false;
+    std::vector<cudaEvent_t> ev;
+    size_t ev_used = 0;
+    double prof_bytes = 0.0, prof_wbytes = 0.0;
+};
+
+bool gemm_plan_create(GemmPlan **out, int, int, int, int) {
+    GemmPlan *p = new GemmPlan();
+    int dev = 0;
+    cudaGetDevice(&dev);
+    cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev);
+    cudaDriverEntryPointQueryResult q;
+    void *fn = nullptr;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
+                                         &q) != cudaSuccess ||
+        q != cudaDriverEntryPointSuccess || !fn) {
+        delete p;
+        return false;
+    }
+    p->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    if (cudaMalloc(&p->ws, WS_BYTES) != cudaSuccess ||
+        cudaMalloc(&p->counters, sizeof(int) * N_COUNTERS) != cudaSuccess) {
+        gemm_plan_destroy(p);
+        return false;
+    }
+    cudaMemset(p->counters, 0, sizeof(int) * N_COUNTERS);
+    *out = p;
+    return true;
+}
+
+void gemm_plan_destroy(GemmPlan *p) {
+    if (!p) return;
+    if (p->ws) cudaFree(p->ws);
+    if (p->counters) cudaFree(p->counters);
+    for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
+    delete p;
+}
+
+void gemm_profile_enable(GemmPlan *p, bool on) {
+    p->profile = on;
+    p->ev_used = 0;
+    p->prof_bytes = p->prof_wbytes = 0.0;
+}
+
+GemmProfile gemm_profile_read(GemmPlan *p) {
+    GemmProfile r{0, 0.0, p->prof_bytes, p->prof_wbytes};
+    for (size_t i = 0; i + 1 < p->ev_used; i += 2) {
+        float ms = 0.f;
+        cudaEventSynchronize(p->ev[i + 1]);
+        if (cudaEventElapsedTime(&ms, p->ev[i], p->ev[i + 1]) == cudaSuccess) r.ms += ms;
+        r.launches += 1;
+    }
+    p->ev_used = 0;
+    p->prof_bytes = p->prof_wbytes = 0.0;
+    return r;
+}
+
+static const CUtensorMap *get_map(GemmPlan *p, const void *ptr, long rows, long cols, long ld,
+                                  long box_rows, int *status) {
+    MapKey key{ptr, rows, cols, ld, box_rows};
+    auto it = p->maps.find(key);
+    if (it != p->maps.end()) return &it->second;
+    CUtensorMap m;
+    memset(&m, 0, sizeof m);
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    CUresult r = p->encode(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims,
+                           strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+                           CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                           CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+    if (r != CUDA_SUCCESS) {
+        fprintf(stderr, "msd: cuTensorMapEncodeTiled failed (%d) rows=%ld cols=%ld ld=%ld\n", (int)r,
+                rows, cols, ld);
+        return nullptr;
+    }
+    return &p->maps.emplace(key, m).first->second;
+}
+
+void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
+               int ldy, int epi, int *status, cudaStream_t s) {
+    if (M <= 0 || O <= 0) return;
+    TcParams tp;
+    memset(&tp, 0, sizeof tp);
+    tp.n_seg = W.nseg;
+    int tiles = 0, out_off = 0;
+    for (int i = 0; i < W.nseg; ++i) {
+        tp.seg_rows[i] = W.rows[i];
+        tp.seg_tiles[i] = (W.rows[i] + BM - 1) / BM;
+        tp.seg_out[i] = out_off;
+        out_off += W.rows[i];
+        tiles += tp.seg_tiles[i];
+    }
+    const int nt = (M + 255) / 256;
+    int BN = (M + nt - 1) / nt;
+    BN = ((BN + 15) / 16) * 16;
+    const int kblocks = (K + BK - 1) / BK;
+    const uint32_t stage_bytes = A_BYTES + (uint32_t)BN * BK * 2;
+    int ctas_per_sm = BN <= 128 ? 2 : 1;
+    int stages = (int)((ctas_per_sm == 2 ? 100u * 1024u : 200u * 1024u) / stage_bytes);
+    stages = stages < 2 ? 2 : (stages > MAX_STAGES ? MAX_STAGES : stages);
+    const size_t smem = 1024 + (size_t)stages * stage_bytes;
+
+    // split-K: fewest waves x k-blocks per CTA, plus a small reduction cost
+    const long base = (long)tiles * nt;
+    const long slots = (long)p->num_sms * ctas_per_sm;
+    const size_t tile_bytes = (size_t)BN * BM * sizeof(float);
+    int best_s = 1;
+    double best = 1e30;
+    for (int sp = 1; sp <= 16 && sp <= kblocks; ++sp) {
+        const int kps = (kblocks + sp - 1) / sp;
+        const int se = (kblocks + kps - 1) / kps;
+        if (se > 1 && ((size_t)base * se * tile_bytes > WS_BYTES || base > N_COUNTERS)) continue;
+        const long waves = (base * se + slots - 1) / slots;
+        const double cost = (double)waves * kps + (se > 1 ? 2.0 : 0.0);
+        if (cost < best - 1e-9) { best = cost; best_s = se; }
+    }
+    const int kps = (kblocks + best_s - 1) / best_s;
+    tp.splits = (kblocks + kps - 1) / kps;
+    tp.kb_per_split = kps;
+    tp.M = M;
+    tp.kblocks = kblocks;
+    tp.BN = BN;
+    tp.n_tiles_n = nt;
+    tp.stages = stages;
+    tp.tmem_cols = BN <= 32 ? 32 : (BN <= 64 ? 64 : (BN <= 128 ? 128 : 256));
+    tp.Y = Y;
+    tp.ldy = ldy;
+    tp.epi = epi;
+    tp.ws = p->ws;
+    tp.counters = p->counters;
+    tp.status = status;
+
+    const CUtensorMap *mw[3] = {nullptr, nullptr, nullptr};
+    for (int i = 0; i < W.nseg; ++i) {
+        mw[i] = get_map(p, W.w[i], W.rows[i], K, K, BM, status);
+        if (!mw[i]) return;
+    }
+    for (int i = W.nseg; i < 3; ++i) mw[i] = mw[0];
+    const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
+    if (!mx) return;
+    if (!p->smem_set) {
+        cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             200 * 1024 + 1024);
+        p->smem_set = true;
+    }
+    dim3 grid(tiles, nt, tp.splits);
+    const bool prof = p->profile;
+    if (prof) {
+        while (p->ev.size() < p->ev_used + 2) {
+            cudaEvent_t e;
+            cudaEventCreate(&e);
+            p->ev.push_back(e);
+        }
+        cudaEventRecord(p->ev[p->ev_used], s);
+    }
+    gemm_tc_kernel<<<grid, THREADS, smem, s>>>(*mw[0], *mw[1], *mw[2], *mx, tp);
+    note_launch();
+    if (prof) {
+        cudaEventRecord(p->ev[p->ev_used + 1], s);
+        p->ev_used += 2;
+        const double wb = (double)O * K * 2.0;
+        p->prof_wbytes += wb;
+        p->prof_bytes += wb + (double)M * K * 2.0 + (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
+    }
+}
+
+}  // namespace msd

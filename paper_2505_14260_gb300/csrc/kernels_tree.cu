@@ -1,0 +1,508 @@
+// Integer side of the MSD step: draft-row set-up, the draft-tree builder
+// (Sec. 3.2 tree drafting), verify set-up, greedy acceptance (Eq. 6 at T = 0)
+// and KV compaction (rejected drafts are discarded, Sec. 3.2).
+#include "kernels_tree.h"
+
+namespace msd {
+
+// ---------------------------------------------------------------------------
+// Pass 1 (catch-up): rows r = b*D1 + j for the pending positions of request b.
+// Input f = f_down(Concat(h, e_next)) (Eq. 4); the concatenated row is built
+// here and the GEMM applies f_down. K/V go to the draft cache at their
+// positions; each row attends causally to the cache.
+// ---------------------------------------------------------------------------
+template <typename T>
+__global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int *__restrict__ n_pend,
+                                     const T *__restrict__ pend_h, const int *__restrict__ pend_next,
+                                     const T *__restrict__ E, int H, int D1, int V,
+                                     T *__restrict__ xfc, RowDesc *__restrict__ rows, int *status) {
+    const int r = blockIdx.x, b = r / D1, j = r - b * D1;
+    const int L = seq_len[b], P = n_pend[b];
+    const bool valid = j < P;
+    const int pos = L - P + j;
+    if (threadIdx.x == 0) {
+        RowDesc d;
+        d.req = b;
+        d.pos = valid ? pos : 0;
+        d.plen = valid ? pos + 1 : 1;
+        d.dst = valid ? pos : -1;
+        rows[r] = d;
+    }
+    int tok = valid ? pend_next[b * D1 + j] : 0;
+    if (tok < 0 || tok >= V) {
+        if (threadIdx.x == 0) set_status(status, ST_BAD_TOKEN);
+        tok = 0;
+    }
+    T *dst = xfc + (size_t)r * 2 * H;
+    const T *hsrc = pend_h + (size_t)(b * D1 + j) * H;
+    const T *esrc = E + (size_t)tok * H;
+    for (int c = threadIdx.x; c < H; c += blockDim.x) {
+        dst[c] = valid ? hsrc[c] : from_f<T>(0.f);
+        dst[H + c] = esrc[c];
+    }
+}
+
+// h_hat of the root slot = draft output of the last pending row.
+template <typename T>
+__global__ void root_gather_kernel(const float *__restrict__ x, const int *__restrict__ n_pend, int D1,
+                                   int H, float *__restrict__ hhat_root, T *__restrict__ xr) {
+    const int b = blockIdx.x;
+    const int r = b * D1 + max(n_pend[b] - 1, 0);
+    for (int c = threadIdx.x; c < H; c += blockDim.x) {
+        const float v = x[(size_t)r * H + c];
+        hhat_root[(size_t)b * H + c] = v;
+        xr[(size_t)b * H + c] = from_f<T>(v);
+    }
+}
+
+// Store h_hat of a tree pass's rows by slot, and a T copy for the LM head.
+template <typename T>
+__global__ void hhat_store_kernel(const float *__restrict__ x, const RowDesc *__restrict__ rows,
+                                  int Td, int H, float *__restrict__ hhat_slot, T *__restrict__ xb) {
+    const int r = blockIdx.x;
+    const RowDesc d = rows[r];
+    for (int c = threadIdx.x; c < H; c += blockDim.x) {
+        const float v = x[(size_t)r * H + c];
+        hhat_slot[((size_t)d.req * Td + d.dst) * H + c] = v;
+        xb[(size_t)r * H + c] = from_f<T>(v);
+    }
+}
+
+// Assemble the draft-pass row of frontier candidate c at row j, slot `slot`:
+// input Concat(h_hat of its parent, e of its token), position L-1+depth.
+template <typename T>
+__device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int c, int depth,
+                                  const float *parent_h, int slot, const uint64_t *parent_mask) {
+    const int H = a.H, k = a.k, Wd = a.Wd;
+    const int L = a.seq_len[b];
+    const int r = b * k + j;
+    if (threadIdx.x == 0) {
+        RowDesc d;
+        d.req = b;
+        d.pos = L - 1 + depth;
+        d.plen = L;
+        d.dst = slot;
+        a.rows[r] = d;
+        for (int w = 0; w < Wd; ++w) {
+            uint64_t m = parent_mask ? parent_mask[w] : 0ull;
+            if (w == slot / 64) m |= 1ull << (slot % 64);
+            a.slot_mask[((size_t)b * a.Td + slot) * Wd + w] = m;
+            a.row_mask[(size_t)r * Wd + w] = m;
+        }
+    }
+    int tok = a.cand_tok[(size_t)b * a.C + c];
+    if (tok < 0 || tok >= a.V) tok = 0;
+    T *dst = a.xfc + (size_t)r * 2 * H;
+    const T *e = a.E + (size_t)tok * H;
+    for (int q = threadIdx.x; q < H; q += blockDim.x) {
+        dst[q] = from_f<T>(parent_h[q]);
+        dst[H + q] = e[q];
+    }
+}
+
+// Depth-1 candidates from the root slot's top-k; frontier = all of them, best
+// first; emit the rows of pass 2.
+template <typename T>
+__global__ void tree_init_kernel(DraftArgs<T> a) {
+    const int b = blockIdx.x, k = a.k;
+    __shared__ float sc[TREE_MAXK];
+    for (int t = threadIdx.x; t < k; t += blockDim.x) {
+        const size_t c = (size_t)b * a.C + t;
+        a.cand_tok[c] = a.ids[(size_t)b * k + t];
+        a.cand_par[c] = -1;
+        a.cand_depth[c] = 1;
+        const float s = a.logp[(size_t)b * k + t];
+        a.cand_score[c] = s;
+        sc[t] = s;
+    }
+    __syncthreads();
+    for (int t = threadIdx.x; t < k; t += blockDim.x) {
+        int rank = 0;
+        for (int u = 0; u < k; ++u) rank += better(sc[u], u, sc[t], t);
+        a.frontier[(size_t)b * k + rank] = t;
+    }
+    __syncthreads();
+    if (a.D < 2) return;
+    for (int j = 0; j < k; ++j) {
+        const int c = a.frontier[(size_t)b * k + j];
+        emit_frontier_row(a, b, j, c, 1, a.hhat_root + (size_t)b * a.H, j, nullptr);
+    }
+}
+
+// After pass d (2..D): add the k*k children of the pass rows, then (d < D) pick
+// the k best of them as the next frontier and emit the rows of pass d+1.
+template <typename T>
+__global__ void tree_step_kernel(DraftArgs<T> a, int d) {
+    extern __shared__ float smem[];
+    const int b = blockIdx.x, k = a.k, kk = k * k;
+    const int base = k + (d - 2) * kk;
+    float *sc = smem;                                 // [kk]
+    int *newf = reinterpret_cast<int *>(smem + kk);   // [k]
+    for (int e = threadIdx.x; e < kk; e += blockDim.x) {
+        const int j = e / k, t = e - j * k;
+        const int p = a.frontier[(size_t)b * k + j];
+        const size_t c = (size_t)b * a.C + base + e;
+        const size_t src = ((size_t)b * k + j) * k + t;
+        a.cand_tok[c] = a.ids[src];
+        a.cand_par[c] = p;
+        a.cand_depth[c] = d;
+        const float s = __fadd_rn(a.cand_score[(size_t)b * a.C + p], a.logp[src]);
+        a.cand_score[c] = s;
+        sc[e] = s;
+    }
+    __syncthreads();
+    if (d >= a.D) return;
+    for (int e = threadIdx.x; e < kk; e += blockDim.x) {
+        int rank = 0;
+        for (int u = 0; u < kk; ++u) rank += better(sc[u], u, sc[e], e);
+        if (rank < k) newf[rank] = base + e;
+    }
+    __syncthreads();
+    for (int j = threadIdx.x; j < k; j += blockDim.x) a.frontier[(size_t)b * k + j] = newf[j];
+    __syncthreads();
+    for (int j = 0; j < k; ++j) {
+        const int c = newf[j];
+        const int jp = (c - base) / k;                   // parent's row in pass d
+        const int sp = (d - 2) * k + jp;                 // parent's slot
+        const int slot = (d - 1) * k + j;
+        emit_frontier_row(a, b, j, c, d, a.hhat_slot + ((size_t)b * a.Td + sp) * a.H, slot,
+                          a.slot_mask + ((size_t)b * a.Td + sp) * a.Wd);
+        __syncthreads();
+    }
+}
+
+// Final tree: the N-1 best candidates (score desc, creation asc), tree index
+// 1 + rank; parents, depths and ancestor masks; the root is node 0.
+__global__ void tree_finalize_kernel(TreeOut t, const int *__restrict__ cand_tok,
+                                     const int *__restrict__ cand_par, const int *__restrict__ cand_depth,
+                                     const float *__restrict__ cand_score, int *__restrict__ node_of,
+                                     const int *__restrict__ root, int C, int N, int *status) {
+    extern __shared__ float ssc[];   // [C]
+    const int b = blockIdx.x, W = (N + 63) / 64;
+    const size_t cb = (size_t)b * C;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) ssc[c] = cand_score[cb + c];
+    __syncthreads();
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        int rank = 0;
+        const float s = ssc[c];
+        for (int u = 0; u < C; ++u) rank += better(ssc[u], u, s, c);
+        node_of[cb + c] = rank < N - 1 ? 1 + rank : -1;
+    }
+    __syncthreads();
+    const size_t nb = (size_t)b * N;
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        const int i = node_of[cb + c];
+        if (i < 0) continue;
+        t.tokens[nb + i] = cand_tok[cb + c];
+        t.depth[nb + i] = cand_depth[cb + c];
+        const int p = cand_par[cb + c];
+        int pi = p < 0 ? 0 : node_of[cb + p];
+        if (pi < 0 || pi >= i) { set_status(status, ST_BAD_TREE); pi = 0; }
+        t.parent[nb + i] = pi;
+        for (int w = 0; w < W; ++w) t.mask[(nb + i) * W + w] = 0ull;
+        // ancestors-or-self: walk the candidate chain, then the root
+        int cur = c, node = i;
+        while (true) {
+            t.mask[(nb + i) * W + node / 64] |= 1ull << (node % 64);
+            if (cur < 0) break;
+            const int pc = cand_par[cb + cur];
+            node = pc < 0 ? 0 : node_of[cb + pc];
+            if (node < 0) break;
+            cur = pc;
+        }
+    }
+    if (threadIdx.x == 0) {
+        t.tokens[nb] = root[b];
+        t.parent[nb] = -1;
+        t.depth[nb] = 0;
+        for (int w = 0; w < W; ++w) t.mask[nb * W + w] = w == 0 ? 1ull : 0ull;
+        if (t.n_nodes) t.n_nodes[b] = N;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Verify set-up: row r = b*N + i at position L + depth(i), sees the prefix
+// [0, L) and the tree nodes of its mask (restricted to valid nodes).
+// ---------------------------------------------------------------------------
+__global__ void verify_setup_kernel(TreeIn t, const int *__restrict__ seq_len,
+                                    const int *__restrict__ root, int B, int N, int V,
+                                    RowDesc *__restrict__ rows, int *__restrict__ src,
+                                    uint64_t *__restrict__ vmask, int *status) {
+    const int r = blockIdx.x * blockDim.x + threadIdx.x;
+    if (r >= B * N) return;
+    const int b = r / N, i = r - b * N, W = (N + 63) / 64;
+    const int n = t.n_nodes ? t.n_nodes[b] : N;
+    const bool valid = i < n;
+    const int L = seq_len[b];
+    int tok = valid ? t.tokens[r] : 0;
+    if (tok < 0 || tok >= V) { set_status(status, ST_BAD_TOKEN); tok = 0; }
+    int depth = valid ? t.depth[r] : 0;
+    if (valid) {
+        const int p = t.parent[r];
+        bool ok = i == 0 ? (p == -1 && depth == 0 && tok == root[b])
+                         : (p >= 0 && p < i && depth == t.depth[b * N + p] + 1);
+        if (!ok) { set_status(status, ST_BAD_TREE); depth = depth < 0 ? 0 : depth; }
+    }
+    RowDesc d;
+    d.req = b;
+    d.pos = L + depth;
+    d.plen = L;
+    d.dst = i;
+    rows[r] = d;
+    src[r] = tok;
+    for (int w = 0; w < W; ++w) {
+        uint64_t m = 0;
+        if (valid) {
+            m = t.mask[(size_t)r * W + w];
+            const int lo = w * 64;
+            if (n - lo < 64) m &= n - lo <= 0 ? 0ull : ((1ull << (n - lo)) - 1ull);
+        } else if (w == i / 64) {
+            m = 1ull << (i % 64);
+        }
+        vmask[(size_t)r * W + w] = m;
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Greedy acceptance (Eq. 6 at T = 0): one warp per request walks from the root
+// to the child whose token is the target argmax of the current node.
+// ---------------------------------------------------------------------------
+__global__ void accept_kernel(TreeIn t, const int *__restrict__ argmax, int N, int D,
+                              int *__restrict__ seq_len, int *__restrict__ n_pend,
+                              int *__restrict__ root, int *__restrict__ pend_next,
+                              int *__restrict__ acc_path, int *__restrict__ acc_L0,
+                              int *__restrict__ acc_a, int *__restrict__ path_out,
+                              int *__restrict__ accept_len_out, int *__restrict__ bonus_out,
+                              int *__restrict__ index_map_out) {
+    const int b = blockIdx.x, lane = threadIdx.x, D1 = D + 1;
+    const size_t nb = (size_t)b * N;
+    const int n = t.n_nodes ? t.n_nodes[b] : N;
+    __shared__ int path[TREE_MAXD + 1];
+    int cur = 0, a = 0;
+    if (lane == 0) path[0] = 0;
+    while (a < D) {
+        const int want = argmax[nb + cur];
+        int found = 0x7fffffff;
+        for (int c = 1 + lane; c < n; c += 32)
+            if (t.parent[nb + c] == cur && t.tokens[nb + c] == want) found = min(found, c);
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) found = min(found, __shfl_xor_sync(0xffffffffu, found, o));
+        if (found == 0x7fffffff) break;
+        cur = found;
+        ++a;
+        if (lane == 0) path[a] = cur;
+    }
+    __syncwarp();
+    const int bonus = argmax[nb + cur];
+    const int L0 = seq_len[b];
+    for (int j = lane; j < D1; j += 32) {
+        const int pj = j <= a ? path[j] : -1;
+        acc_path[b * D1 + j] = pj;
+        if (path_out) path_out[b * D1 + j] = pj;
+        if (index_map_out) index_map_out[b * D1 + j] = j <= a ? L0 + j : -1;
+        if (j <= a) pend_next[b * D1 + j] = j < a ? t.tokens[nb + path[j + 1]] : bonus;
+    }
+    if (lane == 0) {
+        acc_L0[b] = L0;
+        acc_a[b] = a;
+        if (accept_len_out) accept_len_out[b] = a;
+        if (bonus_out) bonus_out[b] = bonus;
+        n_pend[b] = a + 1;
+        seq_len[b] = L0 + a + 1;
+        root[b] = bonus;
+    }
+}
+
+// K/V of accepted node path[j] -> cache position L0 + j, all layers and heads.
+// grid (n_layers*2*nh, B); 16-byte vector copies.
+__global__ void compact_kv_kernel(const uint4 *__restrict__ tree_kv, uint4 *__restrict__ cache,
+                                  const int *__restrict__ acc_path, const int *__restrict__ acc_L0,
+                                  const int *__restrict__ acc_a, int B, int nh, int N, int S,
+                                  int D1, int vec_per_row, int *status) {
+    const int lkh = blockIdx.x, b = blockIdx.y;
+    const int h = lkh % nh, lk = lkh / nh;           // lk = layer*2 + kv
+    const int a = acc_a[b], L0 = acc_L0[b];
+    if (L0 + a >= S) {
+        if (threadIdx.x == 0) set_status(status, ST_RANGE);
+        return;
+    }
+    const size_t tb = ((size_t)(lk * B + b) * nh + h) * N;
+    const size_t cb = ((size_t)(lk * B + b) * nh + h) * S;
+    const int total = (a + 1) * vec_per_row;
+    for (int idx = threadIdx.x; idx < total; idx += blockDim.x) {
+        const int j = idx / vec_per_row, v = idx - j * vec_per_row;
+        const int node = acc_path[b * D1 + j];
+        cache[(cb + L0 + j) * vec_per_row + v] = tree_kv[(tb + node) * vec_per_row + v];
+    }
+}
+
+// Pending draft rows: target features h of the accepted nodes.
+template <typename T>
+__global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ acc_path,
+                              const int *__restrict__ acc_a, int N, int D1, int H,
+                              T *__restrict__ pend_h) {
+    const int b = blockIdx.x / D1, j = blockIdx.x - b * D1;
+    if (j > acc_a[b]) return;
+    const int node = acc_path[b * D1 + j];
+    const T *s = hT + ((size_t)b * N + node) * H;
+    T *d = pend_h + ((size_t)b * D1 + j) * H;
+    for (int c = threadIdx.x; c < H; c += blockDim.x) d[c] = s[c];
+}
+
+// ---------------------------------------------------------------------------
+// Prefill helpers
+// ---------------------------------------------------------------------------
+// Decoupled draft input (Eq. 7): visual rows take the raw embedding.
+template <typename T>
+__global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict__ emb,
+                                     const int *__restrict__ src, int H) {
+    const int r = blockIdx.x;
+    if (src[r] >= 0) return;
+    for (int c = threadIdx.x; c < H; c += blockDim.x)
+        x[(size_t)r * H + c] = to_f(emb[(size_t)r * H + c]);
+}
+
+// Concat(h_i, e_{i+1}) rows for the draft prefill (text positions; visual rows
+// are overwritten after f_down by select_visual_kernel).
+template <typename T>
+__global__ void concat_next_kernel(const T *__restrict__ h, const T *__restrict__ emb, int H,
+                                   T *__restrict__ xfc) {
+    const int r = blockIdx.x;
+    for (int c = threadIdx.x; c < H; c += blockDim.x) {
+        xfc[(size_t)r * 2 * H + c] = h[(size_t)r * H + c];
+        xfc[(size_t)r * 2 * H + H + c] = emb[(size_t)(r + 1) * H + c];
+    }
+}
+
+template <typename T>
+__global__ void prefill_finish_kernel(const int *__restrict__ argmax1, const T *__restrict__ h_last,
+                                      int b, int L, int D1, int H, int *__restrict__ seq_len,
+                                      int *__restrict__ n_pend, int *__restrict__ root,
+                                      int *__restrict__ pend_next, T *__restrict__ pend_h,
+                                      int *__restrict__ root_out) {
+    const int x = argmax1[0];
+    if (threadIdx.x == 0) {
+        seq_len[b] = L;
+        n_pend[b] = 1;
+        root[b] = x;
+        pend_next[b * D1] = x;
+        if (root_out) root_out[b] = x;
+    }
+    for (int c = threadIdx.x; c < H; c += blockDim.x) pend_h[(size_t)b * D1 * H + c] = h_last[c];
+}
+
+// ---------------------------------------------------------------------------
+// Launchers
+// ---------------------------------------------------------------------------
+template <typename T>
+void launch_catchup_setup(const int *seq_len, const int *n_pend, const T *pend_h,
+                          const int *pend_next, const T *E, int B, int H, int D1, int V, T *xfc,
+                          RowDesc *rows, int *status, cudaStream_t s) {
+    catchup_setup_kernel<T><<<B * D1, 256, 0, s>>>(seq_len, n_pend, pend_h, pend_next, E, H, D1,
+                                                   V, xfc, rows, status); note_launch();
+}
+
+template <typename T>
+void launch_root_gather(const float *x, const int *n_pend, int B, int D1, int H, float *hhat_root,
+                        T *xr, cudaStream_t s) {
+    root_gather_kernel<T><<<B, 256, 0, s>>>(x, n_pend, D1, H, hhat_root, xr); note_launch();
+}
+
+template <typename T>
+void launch_hhat_store(const float *x, const RowDesc *rows, int R, int Td, int H,
+                       float *hhat_slot, T *xb, cudaStream_t s) {
+    hhat_store_kernel<T><<<R, 256, 0, s>>>(x, rows, Td, H, hhat_slot, xb); note_launch();
+}
+
+template <typename T>
+void launch_tree_init(const DraftArgs<T> &a, int B, cudaStream_t s) {
+    tree_init_kernel<T><<<B, 256, 0, s>>>(a); note_launch();
+}
+
+template <typename T>
+void launch_tree_step(const DraftArgs<T> &a, int B, int d, cudaStream_t s) {
+    const size_t sm = (size_t)a.k * a.k * sizeof(float) + (size_t)a.k * sizeof(int);
+    tree_step_kernel<T><<<B, 256, sm, s>>>(a, d); note_launch();
+}
+
+void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand_par,
+                          const int *cand_depth, const float *cand_score, int *node_of,
+                          const int *root, int B, int C, int N, int *status, cudaStream_t s) {
+    tree_finalize_kernel<<<B, 512, (size_t)C * sizeof(float), s>>>(
+        t, cand_tok, cand_par, cand_depth, cand_score, node_of, root, C, N, status); note_launch();
+}
+
+void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, int B, int N,
+                         int V, RowDesc *rows, int *src, uint64_t *vmask, int *status,
+                         cudaStream_t s) {
+    const int R = B * N;
+    verify_setup_kernel<<<(R + 127) / 128, 128, 0, s>>>(t, seq_len, root, B, N, V, rows, src,
+                                                          vmask, status); note_launch();
+}
+
+void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int *seq_len,
+                   int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
+                   int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,
+                   cudaStream_t s) {
+    accept_kernel<<<B, 32, 0, s>>>(t, argmax, N, D, seq_len, n_pend, root, pend_next, acc_path,
+                                   acc_L0, acc_a, path_out, accept_len_out, bonus_out,
+                                   index_map_out); note_launch();
+}
+
+void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, const int *acc_L0,
+                       const int *acc_a, int n_layers, int B, int nh, int N, int S, int D1,
+                       int row_bytes, int *status, cudaStream_t s) {
+    dim3 grid(n_layers * 2 * nh, B);
+    compact_kv_kernel<<<grid, 128, 0, s>>>(static_cast<const uint4 *>(tree_kv),
+                                           static_cast<uint4 *>(cache), acc_path, acc_L0, acc_a,
+                                           B, nh, N, S, D1, row_bytes / 16, status); note_launch();
+}
+
+template <typename T>
+void launch_pend_h(const T *hT, const int *acc_path, const int *acc_a, int B, int N, int D1,
+                   int H, T *pend_h, cudaStream_t s) {
+    pend_h_kernel<T><<<B * D1, 256, 0, s>>>(hT, acc_path, acc_a, N, D1, H, pend_h); note_launch();
+}
+
+template <typename T>
+void launch_select_visual(float *x, const T *emb, const int *src, int R, int H, cudaStream_t s) {
+    if (R <= 0) return;
+    select_visual_kernel<T><<<R, 256, 0, s>>>(x, emb, src, H); note_launch();
+}
+
+template <typename T>
+void launch_concat_next(const T *h, const T *emb, int R, int H, T *xfc, cudaStream_t s) {
+    if (R <= 0) return;
+    concat_next_kernel<T><<<R, 256, 0, s>>>(h, emb, H, xfc); note_launch();
+}
+
+template <typename T>
+void launch_prefill_finish(const int *argmax1, const T *h_last, int b, int L, int D1, int H,
+                           int *seq_len, int *n_pend, int *root, int *pend_next, T *pend_h,
+                           int *root_out, cudaStream_t s) {
+    prefill_finish_kernel<T><<<1, 256, 0, s>>>(argmax1, h_last, b, L, D1, H, seq_len, n_pend,
+                                               root, pend_next, pend_h, root_out); note_launch();
+}
+
+#define MSD_INST(T)                                                                             \
+    template void launch_catchup_setup<T>(const int *, const int *, const T *, const int *,     \
+                                          const T *, int, int, int, int, T *, RowDesc *, int *, \
+                                          cudaStream_t);                                        \
+    template void launch_root_gather<T>(const float *, const int *, int, int, int, float *, T *, \
+                                        cudaStream_t);                                          \
+    template void launch_hhat_store<T>(const float *, const RowDesc *, int, int, int, float *,  \
+                                       T *, cudaStream_t);                                      \
+    template void launch_tree_init<T>(const DraftArgs<T> &, int, cudaStream_t);                 \
+    template void launch_tree_step<T>(const DraftArgs<T> &, int, int, cudaStream_t);            \
+    template void launch_pend_h<T>(const T *, const int *, const int *, int, int, int, int, T *, \
+                                   cudaStream_t);                                               \
+    template void launch_select_visual<T>(float *, const T *, const int *, int, int,            \
+                                          cudaStream_t);                                        \
+    template void launch_concat_next<T>(const T *, const T *, int, int, T *, cudaStream_t);     \
+    template void launch_prefill_finish<T>(const int *, const T *, int, int, int, int, int *,   \
+                                           int *, int *, int *, T *, int *, cudaStream_t);
+MSD_INST(float)
+MSD_INST(bf16)
+#undef MSD_INST
+
+}  // namespace msd

@@ -1,0 +1,82 @@
+// Launchers of the integer-side kernels (tree building, acceptance,
+// compaction) and the draft/verify row set-up.
+#pragma once
+
+#include "kernels.h"
+
+namespace msd {
+
+constexpr int TREE_MAXK = 16;   // top-k limit (also the top-k kernel's limit)
+constexpr int TREE_MAXD = 64;   // depth limit
+
+// Draft-tree builder state and outputs of one draft pass (device pointers).
+template <typename T>
+struct DraftArgs {
+    const int *ids;             // top-k ids of the pass rows [rows][k]
+    const float *logp;          // their log-probabilities
+    int k, D, C, H, V, Td, Wd;  // C = k + (D-1)k^2 candidates, Td = (D-1)k slots
+    int *cand_tok, *cand_par, *cand_depth;   // [B][C]
+    float *cand_score;                       // [B][C]
+    int *frontier;                           // [B][k] candidate ids, best first
+    const float *hhat_root;                  // [B][H]
+    const float *hhat_slot;                  // [B][Td][H]
+    const T *E;
+    const int *seq_len;
+    T *xfc;                     // next pass input rows [B*k][2H]
+    RowDesc *rows;              // next pass row descriptors [B*k]
+    uint64_t *slot_mask;        // [B][Td][Wd]
+    uint64_t *row_mask;         // [B*k][Wd]
+};
+
+struct TreeOut {
+    int *tokens, *parent, *depth;
+    uint64_t *mask;
+    int *n_nodes;
+};
+
+struct TreeIn {
+    const int *tokens, *parent, *depth;
+    const uint64_t *mask;
+    const int *n_nodes;
+};
+
+template <typename T>
+void launch_catchup_setup(const int *seq_len, const int *n_pend, const T *pend_h,
+                          const int *pend_next, const T *E, int B, int H, int D1, int V, T *xfc,
+                          RowDesc *rows, int *status, cudaStream_t s);
+template <typename T>
+void launch_root_gather(const float *x, const int *n_pend, int B, int D1, int H, float *hhat_root,
+                        T *xr, cudaStream_t s);
+template <typename T>
+void launch_hhat_store(const float *x, const RowDesc *rows, int R, int Td, int H,
+                       float *hhat_slot, T *xb, cudaStream_t s);
+template <typename T>
+void launch_tree_init(const DraftArgs<T> &a, int B, cudaStream_t s);
+template <typename T>
+void launch_tree_step(const DraftArgs<T> &a, int B, int d, cudaStream_t s);
+void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand_par,
+                          const int *cand_depth, const float *cand_score, int *node_of,
+                          const int *root, int B, int C, int N, int *status, cudaStream_t s);
+void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, int B, int N,
+                         int V, RowDesc *rows, int *src, uint64_t *vmask, int *status,
+                         cudaStream_t s);
+void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int *seq_len,
+                   int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
+                   int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,
+                   cudaStream_t s);
+void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, const int *acc_L0,
+                       const int *acc_a, int n_layers, int B, int nh, int N, int S, int D1,
+                       int row_bytes, int *status, cudaStream_t s);
+template <typename T>
+void launch_pend_h(const T *hT, const int *acc_path, const int *acc_a, int B, int N, int D1,
+                   int H, T *pend_h, cudaStream_t s);
+template <typename T>
+void launch_select_visual(float *x, const T *emb, const int *src, int R, int H, cudaStream_t s);
+template <typename T>
+void launch_concat_next(const T *h, const T *emb, int R, int H, T *xfc, cudaStream_t s);
+template <typename T>
+void launch_prefill_finish(const int *argmax1, const T *h_last, int b, int L, int D1, int H,
+                           int *seq_len, int *n_pend, int *root, int *pend_next, T *pend_h,
+                           int *root_out, cudaStream_t s);
+
+}  // namespace msd

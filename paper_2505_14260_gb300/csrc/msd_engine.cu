@@ -1,0 +1,667 @@
+// Step engine and C ABI of the MSD hot path (include/msd.h).
+//
+// Orchestrates the kernels of one decode step on one stream:
+//   msd_draft_tree     catch-up pass + D-1 tree passes of the one-layer draft
+//                      model (Sec. 3.2, Eq. 4-5) with the decoupled input (Eq. 7)
+//   msd_verify         one tree-masked target forward (Sec. 3.2, verification)
+//   msd_accept_compact greedy acceptance (Eq. 6 at T = 0) + KV compaction
+// Every size a kernel needs at run time (L, accepted length, pending rows) is
+// read by the kernels from device state, so a step needs no host round trip.
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <string>
+#include <vector>
+
+#include "msd.h"
+#include "kernels.h"
+#include "kernels_tree.h"
+#include "gemm_tc.h"
+
+using namespace msd;
+
+struct msd_ctx {
+    msd_config cfg;
+    msd_weights w;
+    std::vector<msd_layer> layers;
+    int dev = 0;
+    size_t esz = 0;
+    int B, S, N, D, D1, k, H, F, V, nh, hd, NL, W, C, Td, Wd, Rmax, chunk, Rlog;
+
+    void *target_kv = nullptr, *draft_kv = nullptr, *tree_kv = nullptr, *dtree_kv = nullptr;
+    int *seq_len = nullptr, *n_pend = nullptr, *root = nullptr, *pend_next = nullptr;
+    void *pend_h = nullptr;
+    float *x = nullptr, *qkv = nullptr, *gu = nullptr, *logits = nullptr;
+    void *xn = nullptr, *q = nullptr, *attn = nullptr, *act = nullptr, *xfc = nullptr, *xr = nullptr;
+    int *argmax_tmp = nullptr;
+    RowDesc *rows = nullptr;
+    int *src = nullptr;
+    uint64_t *vmask = nullptr;
+    int *cand_tok = nullptr, *cand_par = nullptr, *cand_depth = nullptr, *frontier = nullptr,
+        *node_of = nullptr;
+    float *cand_score = nullptr, *hhat_root = nullptr, *hhat_slot = nullptr;
+    uint64_t *slot_mask = nullptr, *row_mask = nullptr;
+    int *topk_ids = nullptr;
+    float *topk_logp = nullptr;
+    void *hT = nullptr;
+    int *acc_path = nullptr, *acc_L0 = nullptr, *acc_a = nullptr;
+    float2 *rope_tab = nullptr;
+    void *h_all = nullptr, *emb_all = nullptr;
+    int *status = nullptr;
+    int *status_host = nullptr;
+    cudaEvent_t status_ev = nullptr;
+    bool status_pending = false;
+    GemmPlan *gplan = nullptr;
+    std::vector<void *> allocs;
+    std::vector<long> L_bound;
+    bool prefilled = false;
+    std::string err;
+};
+
+namespace {
+
+msd_status fail(msd_ctx *c, msd_status st, const std::string &msg) {
+    if (c) c->err = msg;
+    return st;
+}
+
+#define CU(call)                                                                          \
+    do {                                                                                  \
+        cudaError_t e_ = (call);                                                          \
+        if (e_ != cudaSuccess)                                                            \
+            return fail(c, MSD_ERR_CUDA, std::string(#call) + ": " + cudaGetErrorString(e_)); \
+    } while (0)
+
+template <typename P>
+bool dalloc(msd_ctx *c, P **p, size_t bytes) {
+    void *v = nullptr;
+    if (bytes == 0) bytes = 16;
+    if (cudaMalloc(&v, bytes) != cudaSuccess) return false;
+    cudaMemset(v, 0, bytes);
+    c->allocs.push_back(v);
+    *p = static_cast<P *>(v);
+    return true;
+}
+
+// The device status word of earlier calls, observed without blocking.
+msd_status check_status(msd_ctx *c) {
+    if (c->status_pending && cudaEventQuery(c->status_ev) == cudaSuccess) {
+        c->status_pending = false;
+        if (*c->status_host != 0) {
+            char buf[96];
+            snprintf(buf, sizeof buf, "device status word set (code %d)", *c->status_host);
+            return fail(c, MSD_ERR_DEVICE, buf);
+        }
+    }
+    return MSD_OK;
+}
+
+msd_status post_status(msd_ctx *c, cudaStream_t s) {
+    CU(cudaGetLastError());
+    CU(cudaMemcpyAsync(c->status_host, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
+    CU(cudaEventRecord(c->status_ev, s));
+    c->status_pending = true;
+    return MSD_OK;
+}
+
+size_t kv_layer_elems(const msd_ctx *c, int slots) {
+    return (size_t)c->B * c->nh * slots * c->hd;
+}
+
+template <typename T>
+T *tkv(const msd_ctx *c, void *base, int layer, int kv, int slots) {
+    return static_cast<T *>(base) + ((size_t)layer * 2 + kv) * kv_layer_elems(c, slots);
+}
+
+// Y (=|+=) X W^T on the dtype's GEMM: tcgen05 tensor cores for bf16, the
+// CUDA-core kernel for fp32.
+template <typename T>
+void gemm(msd_ctx *c, const T *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
+          int ldy, int epi, cudaStream_t s);
+
+template <>
+void gemm<float>(msd_ctx *c, const float *X, int ldx, int M, int K, const GemmW &W, int O,
+                 float *Y, int ldy, int epi, cudaStream_t s) {
+    launch_gemm_simt<float>(X, ldx, M, K, W, O, Y, ldy, epi, s);
+}
+
+template <>
+void gemm<bf16>(msd_ctx *c, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
+                float *Y, int ldy, int epi, cudaStream_t s) {
+    gemm_bf16(c->gplan, X, ldx, M, K, W, O, Y, ldy, epi, c->status, s);
+}
+
+// One pre-norm decoder layer over R rows (target or draft).
+template <typename T>
+void run_layer(msd_ctx *c, const msd_layer &lw, int R, const RowDesc *rows, T *kdst, T *vdst,
+               int dst_slots, const T *ck, const T *cv, int cslots, const T *tk, const T *tv,
+               int tslots, const uint64_t *mask, int mw, cudaStream_t s) {
+    const int H = c->H, F = c->F;
+    const float eps = c->cfg.rms_eps;
+    launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.attn_norm), R, H, eps,
+                      static_cast<T *>(c->xn), s);
+    GemmW wqkv = {{lw.wq, lw.wk, lw.wv}, {H, H, H}, 3};
+    gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wqkv, 3 * H, c->qkv, 3 * H, EPI_STORE, s);
+    launch_rope_kv<T>(c->qkv, rows, R, c->nh, c->hd, c->rope_tab, c->S, static_cast<T *>(c->q),
+                      kdst, vdst, dst_slots, c->status, s);
+    AttnArgs<T> a;
+    a.q = static_cast<const T *>(c->q);
+    a.rows = rows;
+    a.R = R;
+    a.cache_k = ck;
+    a.cache_v = cv;
+    a.cache_slots = cslots;
+    a.tree_k = tk;
+    a.tree_v = tv;
+    a.tree_slots = tslots;
+    a.mask = mask;
+    a.mask_words = mw;
+    a.nh = c->nh;
+    a.hd = c->hd;
+    a.scale = 1.0f / sqrtf((float)c->hd);
+    a.out = static_cast<T *>(c->attn);
+    launch_attention<T>(a, s);
+    GemmW wo = {{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1};
+    gemm<T>(c, static_cast<const T *>(c->attn), H, R, H, wo, H, c->x, H, EPI_ADD, s);
+    launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.mlp_norm), R, H, eps,
+                      static_cast<T *>(c->xn), s);
+    GemmW wgu = {{lw.w_gate, lw.w_up, nullptr}, {F, F, 0}, 2};
+    gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wgu, 2 * F, c->gu, 2 * F, EPI_STORE, s);
+    launch_swiglu<T>(c->gu, R, F, static_cast<T *>(c->act), s);
+    GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1};
+    gemm<T>(c, static_cast<const T *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD, s);
+}
+
+GemmW one(const void *w, int rows) { return GemmW{{w, nullptr, nullptr}, {rows, 0, 0}, 1}; }
+
+// ---------------------------------------------------------------------------
+// Prefill
+// ---------------------------------------------------------------------------
+template <typename T>
+msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, const int32_t *ids_dev,
+                        int ids_stride, const void *vis_dev, const int64_t *vis_off_host,
+                        int32_t *root_out, cudaStream_t s) {
+    const int H = c->H, V = c->V, D1 = c->D1;
+    const T *E = static_cast<const T *>(c->w.embed);
+    const T *vis = static_cast<const T *>(vis_dev);
+    CU(cudaMemsetAsync(c->seq_len, 0, sizeof(int) * c->B, s));
+    CU(cudaMemsetAsync(c->n_pend, 0, sizeof(int) * c->B, s));
+    for (int b = 0; b < c->B; ++b) c->L_bound[b] = 0;
+    std::vector<int> ids, src;
+    std::vector<RowDesc> rd;
+    for (int b = 0; b < batch; ++b) {
+        const int L = seq_len_host[b];
+        ids.resize(L);
+        CU(cudaMemcpy(ids.data(), ids_dev + (size_t)b * ids_stride, sizeof(int) * L,
+                      cudaMemcpyDeviceToHost));
+        if (ids[L - 1] < 0) return fail(c, MSD_ERR_INVALID, "a prompt must end with a text token");
+        src.resize(L);
+        long vrow = vis_off_host ? vis_off_host[b] : 0;
+        int n_vis = 0;
+        for (int i = 0; i < L; ++i) {
+            if (ids[i] >= V || ids[i] < -1) return fail(c, MSD_ERR_INVALID, "token id out of range");
+            if (ids[i] >= 0) src[i] = ids[i];
+            else { src[i] = (int)(-1 - (vrow + n_vis)); ++n_vis; }
+        }
+        if (n_vis > 0 && !vis) return fail(c, MSD_ERR_INVALID, "visual slots but no visual rows");
+        CU(cudaMemcpyAsync(c->src, src.data(), sizeof(int) * L, cudaMemcpyHostToDevice, s));
+        // target over the prompt, causal, in chunks
+        for (int r0 = 0; r0 < L; r0 += c->chunk) {
+            const int n = std::min(c->chunk, L - r0);
+            rd.resize(n);
+            for (int i = 0; i < n; ++i) rd[i] = RowDesc{b, r0 + i, r0 + i + 1, r0 + i};
+            CU(cudaMemcpyAsync(c->rows, rd.data(), sizeof(RowDesc) * n, cudaMemcpyHostToDevice, s));
+            launch_embed_rows<T>(E, vis, c->src + r0, n, H, c->x,
+                                 static_cast<T *>(c->emb_all) + (size_t)r0 * H, V, c->status, s);
+            for (int l = 0; l < c->NL; ++l) {
+                T *K = tkv<T>(c, c->target_kv, l, 0, c->S), *Vv = tkv<T>(c, c->target_kv, l, 1, c->S);
+                run_layer<T>(c, c->layers[l], n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr,
+                             nullptr, 0, nullptr, 0, s);
+            }
+            launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), n, H, c->cfg.rms_eps,
+                              static_cast<T *>(c->h_all) + (size_t)r0 * H, s);
+            CU(cudaStreamSynchronize(s));   // rd/src host vectors are reused
+        }
+        const T *h_last = static_cast<const T *>(c->h_all) + (size_t)(L - 1) * H;
+        gemm<T>(c, h_last, H, 1, H, one(c->w.lm_head, V), V, c->logits, V, EPI_STORE, s);
+        launch_argmax(c->logits, 1, V, c->argmax_tmp, s);
+        // draft cache over positions 0 .. L-2 with the decoupled input (Eq. 7)
+        for (int r0 = 0; r0 < L - 1; r0 += c->chunk) {
+            const int n = std::min(c->chunk, L - 1 - r0);
+            rd.resize(n);
+            for (int i = 0; i < n; ++i) rd[i] = RowDesc{b, r0 + i, r0 + i + 1, r0 + i};
+            CU(cudaMemcpyAsync(c->rows, rd.data(), sizeof(RowDesc) * n, cudaMemcpyHostToDevice, s));
+            launch_concat_next<T>(static_cast<const T *>(c->h_all) + (size_t)r0 * H,
+                                  static_cast<const T *>(c->emb_all) + (size_t)r0 * H, n, H,
+                                  static_cast<T *>(c->xfc), s);
+            gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, n, 2 * H, one(c->w.draft_fc, H), H,
+                    c->x, H, EPI_STORE, s);
+            launch_select_visual<T>(c->x, static_cast<const T *>(c->emb_all) + (size_t)r0 * H,
+                                    c->src + r0, n, H, s);
+            T *K = tkv<T>(c, c->draft_kv, 0, 0, c->S), *Vv = tkv<T>(c, c->draft_kv, 0, 1, c->S);
+            run_layer<T>(c, c->w.draft, n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr, nullptr, 0,
+                         nullptr, 0, s);
+            CU(cudaStreamSynchronize(s));
+        }
+        launch_prefill_finish<T>(c->argmax_tmp, h_last, b, L, D1, H, c->seq_len, c->n_pend, c->root,
+                                 c->pend_next, static_cast<T *>(c->pend_h), root_out, s);
+        c->L_bound[b] = L;
+    }
+    c->prefilled = true;
+    return post_status(c, s);
+}
+
+// ---------------------------------------------------------------------------
+// Draft tree
+// ---------------------------------------------------------------------------
+template <typename T>
+DraftArgs<T> draft_args(msd_ctx *c) {
+    DraftArgs<T> a;
+    a.ids = c->topk_ids;
+    a.logp = c->topk_logp;
+    a.k = c->k; a.D = c->D; a.C = c->C; a.H = c->H; a.V = c->V; a.Td = c->Td; a.Wd = c->Wd;
+    a.cand_tok = c->cand_tok; a.cand_par = c->cand_par; a.cand_depth = c->cand_depth;
+    a.cand_score = c->cand_score; a.frontier = c->frontier;
+    a.hhat_root = c->hhat_root; a.hhat_slot = c->hhat_slot;
+    a.E = static_cast<const T *>(c->w.embed);
+    a.seq_len = c->seq_len;
+    a.xfc = static_cast<T *>(c->xfc);
+    a.rows = c->rows;
+    a.slot_mask = c->slot_mask;
+    a.row_mask = c->row_mask;
+    return a;
+}
+
+msd_status record_pass(msd_ctx *c, const msd_draft_record *rec, int pass, int rows_per_req,
+                       cudaStream_t s) {
+    if (!rec) return MSD_OK;
+    const int B = c->B, D = c->D, k = c->k, V = c->V;
+    if (rec->logits)
+        CU(cudaMemcpy2DAsync(rec->logits + (size_t)pass * k * V, sizeof(float) * D * k * V,
+                             c->logits, sizeof(float) * rows_per_req * V,
+                             sizeof(float) * rows_per_req * V, B, cudaMemcpyDeviceToDevice, s));
+    if (rec->topk_ids)
+        CU(cudaMemcpy2DAsync(rec->topk_ids + (size_t)pass * k * k, sizeof(int) * D * k * k,
+                             c->topk_ids, sizeof(int) * rows_per_req * k,
+                             sizeof(int) * rows_per_req * k, B, cudaMemcpyDeviceToDevice, s));
+    if (rec->topk_logp)
+        CU(cudaMemcpy2DAsync(rec->topk_logp + (size_t)pass * k * k, sizeof(float) * D * k * k,
+                             c->topk_logp, sizeof(float) * rows_per_req * k,
+                             sizeof(float) * rows_per_req * k, B, cudaMemcpyDeviceToDevice, s));
+    return MSD_OK;
+}
+
+template <typename T>
+msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *rec,
+                      cudaStream_t s) {
+    const int B = c->B, H = c->H, V = c->V, k = c->k, D1 = c->D1, S = c->S;
+    const T *E = static_cast<const T *>(c->w.embed);
+    T *dK = tkv<T>(c, c->draft_kv, 0, 0, S), *dV = tkv<T>(c, c->draft_kv, 0, 1, S);
+    T *tK = tkv<T>(c, c->dtree_kv, 0, 0, c->Td), *tV = tkv<T>(c, c->dtree_kv, 0, 1, c->Td);
+    // pass 1: catch-up rows + root slot
+    const int R1 = B * D1;
+    launch_catchup_setup<T>(c->seq_len, c->n_pend, static_cast<const T *>(c->pend_h), c->pend_next,
+                            E, B, H, D1, V, static_cast<T *>(c->xfc), c->rows, c->status, s);
+    gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, R1, 2 * H, one(c->w.draft_fc, H), H, c->x, H,
+            EPI_STORE, s);
+    run_layer<T>(c, c->w.draft, R1, c->rows, dK, dV, S, dK, dV, S, nullptr, nullptr, 0, nullptr, 0,
+                 s);
+    launch_root_gather<T>(c->x, c->n_pend, B, D1, H, c->hhat_root, static_cast<T *>(c->xr), s);
+    gemm<T>(c, static_cast<const T *>(c->xr), H, B, H, one(c->w.lm_head, V), V, c->logits, V,
+            EPI_STORE, s);
+    launch_topk_logp(c->logits, B, V, k, c->topk_ids, c->topk_logp, s);
+    msd_status st = record_pass(c, rec, 0, 1, s);
+    if (st != MSD_OK) return st;
+    DraftArgs<T> a = draft_args<T>(c);
+    launch_tree_init<T>(a, B, s);
+    // passes 2..D: expand the frontier
+    const int Rk = B * k;
+    for (int d = 2; d <= c->D; ++d) {
+        gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, Rk, 2 * H, one(c->w.draft_fc, H), H,
+                c->x, H, EPI_STORE, s);
+        run_layer<T>(c, c->w.draft, Rk, c->rows, tK, tV, c->Td, dK, dV, S, tK, tV, c->Td,
+                     c->row_mask, c->Wd, s);
+        launch_hhat_store<T>(c->x, c->rows, Rk, c->Td, H, c->hhat_slot, static_cast<T *>(c->xr), s);
+        gemm<T>(c, static_cast<const T *>(c->xr), H, Rk, H, one(c->w.lm_head, V), V, c->logits, V,
+                EPI_STORE, s);
+        launch_topk_logp(c->logits, Rk, V, k, c->topk_ids, c->topk_logp, s);
+        st = record_pass(c, rec, d - 1, k, s);
+        if (st != MSD_OK) return st;
+        launch_tree_step<T>(a, B, d, s);
+    }
+    TreeOut t{out->tokens, out->parent, out->depth, out->mask, out->n_nodes};
+    launch_tree_finalize(t, c->cand_tok, c->cand_par, c->cand_depth, c->cand_score, c->node_of,
+                         c->root, B, c->C, c->N, c->status, s);
+    return post_status(c, s);
+}
+
+// ---------------------------------------------------------------------------
+// Verify
+// ---------------------------------------------------------------------------
+template <typename T>
+msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, float *logits_dev,
+                       cudaStream_t s) {
+    const int B = c->B, N = c->N, H = c->H, V = c->V, R = B * N;
+    TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
+    launch_verify_setup(t, c->seq_len, c->root, B, N, V, c->rows, c->src, c->vmask, c->status, s);
+    launch_embed_rows<T>(static_cast<const T *>(c->w.embed), nullptr, c->src, R, H, c->x, nullptr,
+                         V, c->status, s);
+    for (int l = 0; l < c->NL; ++l) {
+        T *K = tkv<T>(c, c->target_kv, l, 0, c->S), *Vv = tkv<T>(c, c->target_kv, l, 1, c->S);
+        T *tK = tkv<T>(c, c->tree_kv, l, 0, N), *tV = tkv<T>(c, c->tree_kv, l, 1, N);
+        run_layer<T>(c, c->layers[l], R, c->rows, tK, tV, N, K, Vv, c->S, tK, tV, N, c->vmask, c->W,
+                     s);
+    }
+    launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), R, H, c->cfg.rms_eps,
+                      static_cast<T *>(c->hT), s);
+    float *lg = logits_dev ? logits_dev : c->logits;
+    gemm<T>(c, static_cast<const T *>(c->hT), H, R, H, one(c->w.lm_head, V), V, lg, V, EPI_STORE,
+            s);
+    launch_argmax(lg, R, V, argmax_dev, s);
+    return post_status(c, s);
+}
+
+template <typename T>
+msd_status accept_impl(msd_ctx *c, const msd_tree *tree, const int32_t *argmax, int32_t *path,
+                       int32_t *alen, int32_t *bonus, int32_t *imap, cudaStream_t s) {
+    TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
+    launch_accept(t, argmax, c->B, c->N, c->D, c->seq_len, c->n_pend, c->root, c->pend_next,
+                  c->acc_path, c->acc_L0, c->acc_a, path, alen, bonus, imap, s);
+    launch_compact_kv(c->tree_kv, c->target_kv, c->acc_path, c->acc_L0, c->acc_a, c->NL, c->B, c->nh,
+                      c->N, c->S, c->D1, (int)(c->hd * c->esz), c->status, s);
+    launch_pend_h<T>(static_cast<const T *>(c->hT), c->acc_path, c->acc_a, c->B, c->N, c->D1, c->H,
+                     static_cast<T *>(c->pend_h), s);
+    for (int b = 0; b < c->B; ++b) c->L_bound[b] += c->D1;
+    return post_status(c, s);
+}
+
+// A step writes at most positions L .. L+D (tree K/V land at L+depth only in
+// scratch), so L + D + 1 <= max_seq keeps every write in bounds. The host
+// keeps an upper bound of L and reads the true value only when the bound
+// says it may be too large.
+msd_status check_capacity(msd_ctx *c) {
+    bool tight = false;
+    for (int b = 0; b < c->B; ++b)
+        if (c->L_bound[b] + c->D + 1 > c->S) tight = true;
+    if (!tight) return MSD_OK;
+    std::vector<int> L(c->B);
+    CU(cudaDeviceSynchronize());
+    CU(cudaMemcpy(L.data(), c->seq_len, sizeof(int) * c->B, cudaMemcpyDeviceToHost));
+    for (int b = 0; b < c->B; ++b) {
+        c->L_bound[b] = L[b];
+        if (L[b] + c->D + 1 > c->S) return fail(c, MSD_ERR_CAPACITY, "request would exceed max_seq");
+    }
+    return MSD_OK;
+}
+
+msd_status validate_config(const msd_config *g) {
+    if (!g) return MSD_ERR_INVALID;
+    if (g->n_layers < 1 || g->hidden < 1 || g->n_heads < 1 || g->ffn < 1 || g->vocab < 2)
+        return MSD_ERR_INVALID;
+    if (g->head_dim != 64 && g->head_dim != 128) return MSD_ERR_INVALID;
+    if (g->n_heads * g->head_dim != g->hidden) return MSD_ERR_INVALID;
+    if (g->hidden % 64 || g->ffn % 16) return MSD_ERR_INVALID;
+    if (g->dtype != MSD_F32 && g->dtype != MSD_BF16) return MSD_ERR_INVALID;
+    if (g->max_batch < 1 || g->max_seq < 2) return MSD_ERR_INVALID;
+    if (g->tree_nodes < 1 || g->tree_nodes > 256) return MSD_ERR_INVALID;
+    if (g->tree_depth < 1 || g->tree_depth > TREE_MAXD) return MSD_ERR_INVALID;
+    if (g->topk < 1 || g->topk > TREE_MAXK || g->topk > g->vocab) return MSD_ERR_INVALID;
+    const long cand = g->topk + (long)(g->tree_depth - 1) * g->topk * g->topk;
+    if (cand < g->tree_nodes - 1) return MSD_ERR_INVALID;
+    return MSD_OK;
+}
+
+}  // namespace
+
+// ---------------------------------------------------------------------------
+// C ABI
+// ---------------------------------------------------------------------------
+extern "C" {
+
+msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out) {
+    if (!out) return MSD_ERR_INVALID;
+    *out = nullptr;
+    if (validate_config(cfg) != MSD_OK || !w || !w->layers) return MSD_ERR_INVALID;
+    const void *need[] = {w->embed, w->final_norm, w->lm_head, w->draft_fc, w->draft.attn_norm,
+                          w->draft.wq, w->draft.wk, w->draft.wv, w->draft.wo, w->draft.mlp_norm,
+                          w->draft.w_gate, w->draft.w_up, w->draft.w_down};
+    for (const void *p : need)
+        if (!p) return MSD_ERR_INVALID;
+    for (int l = 0; l < cfg->n_layers; ++l) {
+        const msd_layer &L = w->layers[l];
+        const void *lp[] = {L.attn_norm, L.wq, L.wk, L.wv, L.wo, L.mlp_norm, L.w_gate, L.w_up, L.w_down};
+        for (const void *p : lp)
+            if (!p) return MSD_ERR_INVALID;
+    }
+    msd_ctx *c = new msd_ctx();
+    c->cfg = *cfg;
+    c->w = *w;
+    c->layers.assign(w->layers, w->layers + cfg->n_layers);
+    c->w.layers = c->layers.data();
+    cudaGetDevice(&c->dev);
+    c->esz = cfg->dtype == MSD_BF16 ? 2 : 4;
+    c->B = cfg->max_batch; c->S = cfg->max_seq; c->N = cfg->tree_nodes; c->D = cfg->tree_depth;
+    c->D1 = c->D + 1; c->k = cfg->topk; c->H = cfg->hidden; c->F = cfg->ffn; c->V = cfg->vocab;
+    c->nh = cfg->n_heads; c->hd = cfg->head_dim; c->NL = cfg->n_layers;
+    c->W = (c->N + 63) / 64;
+    c->C = c->k + (c->D - 1) * c->k * c->k;
+    c->Td = std::max(1, (c->D - 1) * c->k);
+    c->Wd = (c->Td + 63) / 64;
+    c->chunk = std::min(c->S, 1024);
+    c->Rmax = std::max(std::max(c->B * c->N, c->B * c->D1), std::max(c->B * c->k, c->chunk));
+    c->Rlog = std::max(std::max(c->B * c->N, c->B * c->k), 1);
+    c->L_bound.assign(c->B, 0);
+    const size_t e = c->esz, H = c->H, F = c->F, R = c->Rmax;
+    bool ok = true;
+    ok &= dalloc(c, &c->target_kv, (size_t)c->NL * 2 * kv_layer_elems(c, c->S) * e);
+    ok &= dalloc(c, &c->draft_kv, 2 * kv_layer_elems(c, c->S) * e);
+    ok &= dalloc(c, &c->tree_kv, (size_t)c->NL * 2 * kv_layer_elems(c, c->N) * e);
+    ok &= dalloc(c, &c->dtree_kv, 2 * kv_layer_elems(c, c->Td) * e);
+    ok &= dalloc(c, &c->seq_len, sizeof(int) * c->B);
+    ok &= dalloc(c, &c->n_pend, sizeof(int) * c->B);
+    ok &= dalloc(c, &c->root, sizeof(int) * c->B);
+    ok &= dalloc(c, &c->pend_next, sizeof(int) * c->B * c->D1);
+    ok &= dalloc(c, &c->pend_h, (size_t)c->B * c->D1 * H * e);
+    ok &= dalloc(c, &c->x, R * H * 4);
+    ok &= dalloc(c, &c->xn, R * H * e);
+    ok &= dalloc(c, &c->qkv, R * 3 * H * 4);
+    ok &= dalloc(c, &c->q, R * H * e);
+    ok &= dalloc(c, &c->attn, R * H * e);
+    ok &= dalloc(c, &c->gu, R * 2 * F * 4);
+    ok &= dalloc(c, &c->act, R * F * e);
+    ok &= dalloc(c, &c->xfc, R * 2 * H * e);
+    ok &= dalloc(c, &c->xr, R * H * e);
+    ok &= dalloc(c, &c->logits, (size_t)c->Rlog * c->V * 4);
+    ok &= dalloc(c, &c->argmax_tmp, sizeof(int) * 4);
+    ok &= dalloc(c, &c->rows, sizeof(RowDesc) * R);
+    ok &= dalloc(c, &c->src, sizeof(int) * std::max<size_t>(R, c->S));
+    ok &= dalloc(c, &c->vmask, sizeof(uint64_t) * c->B * c->N * c->W);
+    ok &= dalloc(c, &c->cand_tok, sizeof(int) * c->B * c->C);
+    ok &= dalloc(c, &c->cand_par, sizeof(int) * c->B * c->C);
+    ok &= dalloc(c, &c->cand_depth, sizeof(int) * c->B * c->C);
+    ok &= dalloc(c, &c->cand_score, sizeof(float) * c->B * c->C);
+    ok &= dalloc(c, &c->node_of, sizeof(int) * c->B * c->C);
+    ok &= dalloc(c, &c->frontier, sizeof(int) * c->B * c->k);
+    ok &= dalloc(c, &c->hhat_root, sizeof(float) * c->B * H);
+    ok &= dalloc(c, &c->hhat_slot, sizeof(float) * c->B * c->Td * H);
+    ok &= dalloc(c, &c->slot_mask, sizeof(uint64_t) * c->B * c->Td * c->Wd);
+    ok &= dalloc(c, &c->row_mask, sizeof(uint64_t) * c->B * c->k * c->Wd);
+    ok &= dalloc(c, &c->topk_ids, sizeof(int) * c->Rlog * c->k);
+    ok &= dalloc(c, &c->topk_logp, sizeof(float) * c->Rlog * c->k);
+    ok &= dalloc(c, &c->hT, (size_t)c->B * c->N * H * e);
+    ok &= dalloc(c, &c->acc_path, sizeof(int) * c->B * c->D1);
+    ok &= dalloc(c, &c->acc_L0, sizeof(int) * c->B);
+    ok &= dalloc(c, &c->acc_a, sizeof(int) * c->B);
+    ok &= dalloc(c, &c->rope_tab, sizeof(float2) * (size_t)c->S * (c->hd / 2));
+    ok &= dalloc(c, &c->h_all, (size_t)c->S * H * e);
+    ok &= dalloc(c, &c->emb_all, (size_t)c->S * H * e);
+    ok &= dalloc(c, &c->status, sizeof(int));
+    if (ok) ok = cudaMallocHost(&c->status_host, sizeof(int)) == cudaSuccess;
+    if (ok) ok = cudaEventCreateWithFlags(&c->status_ev, cudaEventDisableTiming) == cudaSuccess;
+    if (ok && cfg->dtype == MSD_BF16) ok = gemm_plan_create(&c->gplan, c->Rmax, c->H, c->F, c->V);
+    if (!ok) {
+        msd_destroy(c);
+        cudaGetLastError();
+        return MSD_ERR_OOM;
+    }
+    *c->status_host = 0;
+    // RoPE table: (cos, sin) of pos * base^(-2i/hd), computed in double.
+    std::vector<float2> tab((size_t)c->S * (c->hd / 2));
+    for (int p = 0; p < c->S; ++p)
+        for (int i = 0; i < c->hd / 2; ++i) {
+            const double th = std::pow((double)cfg->rope_base, -2.0 * i / c->hd);
+            const double ang = (double)p * th;
+            tab[(size_t)p * (c->hd / 2) + i] = make_float2((float)std::cos(ang), (float)std::sin(ang));
+        }
+    if (cudaMemcpy(c->rope_tab, tab.data(), sizeof(float2) * tab.size(), cudaMemcpyHostToDevice) !=
+            cudaSuccess ||
+        cudaDeviceSynchronize() != cudaSuccess) {
+        msd_destroy(c);
+        return MSD_ERR_CUDA;
+    }
+    *out = c;
+    return MSD_OK;
+}
+
+msd_status msd_destroy(msd_ctx *c) {
+    if (!c) return MSD_OK;
+    cudaDeviceSynchronize();
+    for (void *p : c->allocs) cudaFree(p);
+    if (c->status_host) cudaFreeHost(c->status_host);
+    if (c->status_ev) cudaEventDestroy(c->status_ev);
+    if (c->gplan) gemm_plan_destroy(c->gplan);
+    delete c;
+    return MSD_OK;
+}
+
+msd_status msd_prefill(msd_ctx *c, int32_t batch, const int32_t *seq_len_host,
+                       const int32_t *ids_dev, int32_t ids_stride, const void *vis_dev,
+                       const int64_t *vis_off_host, int32_t *root_out_dev, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (batch < 1 || batch > c->B || !seq_len_host || !ids_dev)
+        return fail(c, MSD_ERR_INVALID, "bad batch or null argument");
+    if (batch != c->B) return fail(c, MSD_ERR_INVALID, "batch must equal max_batch");
+    for (int b = 0; b < batch; ++b) {
+        if (seq_len_host[b] < 1) return fail(c, MSD_ERR_INVALID, "empty prompt");
+        if (seq_len_host[b] > ids_stride) return fail(c, MSD_ERR_INVALID, "prompt longer than ids_stride");
+        if ((long)seq_len_host[b] + c->D + 1 > c->S) return fail(c, MSD_ERR_CAPACITY, "prompt exceeds max_seq");
+    }
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (c->cfg.dtype == MSD_BF16)
+        return prefill_impl<bf16>(c, batch, seq_len_host, ids_dev, ids_stride, vis_dev, vis_off_host,
+                                  root_out_dev, s);
+    return prefill_impl<float>(c, batch, seq_len_host, ids_dev, ids_stride, vis_dev, vis_off_host,
+                               root_out_dev, s);
+}
+
+static bool tree_ok(const msd_tree *t) {
+    return t && t->tokens && t->parent && t->depth && t->mask;
+}
+
+msd_status msd_draft_tree(msd_ctx *c, const msd_tree *out, const msd_draft_record *rec,
+                          void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!tree_ok(out)) return fail(c, MSD_ERR_INVALID, "null tree array");
+    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    st = check_capacity(c);
+    if (st != MSD_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (c->cfg.dtype == MSD_BF16) return draft_impl<bf16>(c, out, rec, s);
+    return draft_impl<float>(c, out, rec, s);
+}
+
+msd_status msd_verify(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, float *logits_dev,
+                      void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!tree_ok(tree) || !argmax_dev) return fail(c, MSD_ERR_INVALID, "null tree or argmax");
+    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    st = check_capacity(c);
+    if (st != MSD_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (c->cfg.dtype == MSD_BF16) return verify_impl<bf16>(c, tree, argmax_dev, logits_dev, s);
+    return verify_impl<float>(c, tree, argmax_dev, logits_dev, s);
+}
+
+msd_status msd_accept_compact(msd_ctx *c, const msd_tree *tree, const int32_t *argmax_dev,
+                              int32_t *path_dev, int32_t *accept_len_dev, int32_t *bonus_dev,
+                              int32_t *index_map_dev, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!tree_ok(tree) || !argmax_dev) return fail(c, MSD_ERR_INVALID, "null tree or argmax");
+    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    st = check_capacity(c);
+    if (st != MSD_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (c->cfg.dtype == MSD_BF16)
+        return accept_impl<bf16>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev,
+                                 index_map_dev, s);
+    return accept_impl<float>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev,
+                              index_map_dev, s);
+}
+
+msd_status msd_linear(msd_ctx *c, const void *x, int32_t ldx, int32_t m, int32_t k, const void *w,
+                      int32_t o, float *y, int32_t ldy, int32_t accumulate, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    if (!x || !w || !y || m <= 0 || k <= 0 || o <= 0 || ldx < k || ldy < o)
+        return fail(c, MSD_ERR_INVALID, "bad msd_linear arguments");
+    if (c->cfg.dtype == MSD_BF16 && (ldx % 8 || k % 8))
+        return fail(c, MSD_ERR_INVALID, "bf16 rows must be 16-byte aligned");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const GemmW W = one(w, o);
+    const int epi = accumulate ? EPI_ADD : EPI_STORE;
+    if (c->cfg.dtype == MSD_BF16)
+        gemm<bf16>(c, static_cast<const bf16 *>(x), ldx, m, k, W, o, y, ldy, epi, s);
+    else
+        gemm<float>(c, static_cast<const float *>(x), ldx, m, k, W, o, y, ldy, epi, s);
+    return post_status(c, s);
+}
+
+msd_status msd_profile_enable(msd_ctx *c, int32_t on) {
+    if (!c) return MSD_ERR_INVALID;
+    if (c->gplan) gemm_profile_enable(c->gplan, on != 0);
+    return MSD_OK;
+}
+
+msd_status msd_profile_read(msd_ctx *c, msd_profile *out) {
+    if (!c || !out) return MSD_ERR_INVALID;
+    memset(out, 0, sizeof *out);
+    out->kernel_launches = launch_count();
+    if (c->gplan) {
+        const GemmProfile g = gemm_profile_read(c->gplan);
+        out->gemm_launches = g.launches;
+        out->gemm_ms = g.ms;
+        out->gemm_bytes = g.bytes;
+        out->gemm_weight_bytes = g.weight_bytes;
+    }
+    return MSD_OK;
+}
+
+msd_status msd_state(msd_ctx *c, msd_state_view *out) {
+    if (!c || !out) return MSD_ERR_INVALID;
+    out->target_kv = c->target_kv;
+    out->draft_kv = c->draft_kv;
+    out->seq_len = c->seq_len;
+    out->n_pending = c->n_pend;
+    out->root = c->root;
+    out->elem_bytes = (int64_t)c->esz;
+    return MSD_OK;
+}
+
+const char *msd_last_error(const msd_ctx *c) {
+    if (!c) return "null context";
+    return c->err.c_str();
+}
+
+}  // extern "C"

@@ -1,0 +1,92 @@
+"""Helpers for the GPU tests: move synthetic weights to the device, open an
+engine, and compare device outputs with the oracle."""
+import numpy as np
+import torch
+
+from paper_2505_14260_gb300 import msd, synth
+
+# Tolerances. bf16 against the float64 oracle: the stated bound for the
+# logits (max |d| <= 3e-2 and relative L2 <= 1e-2). fp32: float32 rounding of
+# a float64 computation over two layers.
+TOL = {"f32": dict(max_abs=2e-4, rel_l2=1e-5), "bf16": dict(max_abs=3e-2, rel_l2=1e-2)}
+KV_REL_L2 = {"f32": 1e-5, "bf16": 1e-2}
+
+
+def to_device(w: dict, device="cuda") -> dict:
+    out = {}
+    for k, v in w.items():
+        if k == "layers":
+            out[k] = [{n: t.to(device) for n, t in lw.items()} for lw in v]
+        elif k == "draft":
+            out[k] = {n: t.to(device) for n, t in v.items()}
+        else:
+            out[k] = v.to(device)
+    return out
+
+
+def open_engine(wl, weights_cpu=None, steps=None, batch=None):
+    w = synth.make_weights(wl) if weights_cpu is None else weights_cpu
+    wd = to_device(w)
+    cfg = msd.make_config(wl, wl.max_seq(steps), batch)
+    return msd.Engine(cfg, wd), w
+
+
+def rel_l2(a, b) -> float:
+    a = np.asarray(a, np.float64); b = np.asarray(b, np.float64)
+    return float(np.linalg.norm(a - b) / max(np.linalg.norm(b), 1e-30))
+
+
+def assert_close(gpu, ref, tol, what=""):
+    gpu = np.asarray(gpu, np.float64); ref = np.asarray(ref, np.float64)
+    d = float(np.max(np.abs(gpu - ref))) if gpu.size else 0.0
+    r = rel_l2(gpu, ref)
+    assert d <= tol["max_abs"] and r <= tol["rel_l2"], f"{what}: max|d|={d:.3e} relL2={r:.3e}"
+    return d, r
+
+
+def top2_margin(row) -> float:
+    s = np.sort(np.asarray(row, np.float64))
+    return float(s[-1] - s[-2])
+
+
+def record_buffers(wl, B=None):
+    B = wl.batch if B is None else B
+    D, k, V = wl.tree_depth, wl.topk, wl.vocab
+    return {"logits": torch.zeros(B, D, k, V, device="cuda"),
+            "topk_ids": torch.zeros(B, D, k, k, dtype=torch.int32, device="cuda"),
+            "topk_logp": torch.zeros(B, D, k, k, device="cuda")}
+
+
+def tree_numpy(tree: msd.Tree, b: int):
+    N = tree.N
+    sl = slice(b * N, (b + 1) * N)
+    toks = tree.tokens[sl].cpu().numpy().astype(np.int64)
+    par = tree.parent[sl].cpu().numpy().astype(np.int64)
+    dep = tree.depth[sl].cpu().numpy().astype(np.int64)
+    mask = tree.mask.view(torch.int64)[b * N * tree.W:(b + 1) * N * tree.W].cpu().numpy()
+    return toks, par, dep, mask.view(np.uint64).reshape(N, tree.W)
+
+
+def plant(tree: msd.Tree, b: int, tokens, parent):
+    """Writes a caller-planted tree for request b (depths and masks derived)."""
+    N = tree.N
+    n = len(tokens)
+    depth = np.zeros(n, np.int64)
+    for i in range(1, n):
+        depth[i] = depth[parent[i]] + 1
+    W = tree.W
+    mask = np.zeros((N, W), np.uint64)
+    for i in range(n):
+        j = i
+        while j >= 0:
+            mask[i, j // 64] |= np.uint64(1) << np.uint64(j % 64)
+            j = parent[j]
+    t = np.zeros(N, np.int32); t[:n] = tokens
+    p = np.full(N, -1, np.int32); p[:n] = parent
+    d = np.zeros(N, np.int32); d[:n] = depth
+    sl = slice(b * N, (b + 1) * N)
+    tree.tokens[sl] = torch.from_numpy(t).cuda()
+    tree.parent[sl] = torch.from_numpy(p).cuda()
+    tree.depth[sl] = torch.from_numpy(d).cuda()
+    tree.mask[b * N * W:(b + 1) * N * W] = torch.from_numpy(mask.reshape(-1).view(np.int64)).cuda()
+    tree.n_nodes[b] = n

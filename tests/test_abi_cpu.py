@@ -1,0 +1,70 @@
+"""The C-ABI library builds for sm_103a, loads, and exports every entry point
+declared in include/msd.h; argument validation that needs no GPU works."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def libmsd():
+    from paper_2505_14260_gb300 import build, msd
+    build.build()
+    return msd.lib()
+
+
+def declared_symbols():
+    text = open(os.path.join(ROOT, "include", "msd.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    return sorted(set(re.findall(r"\b(msd_[a-z_]+)\s*\(", text)))
+
+
+def test_header_declares_the_boundary():
+    names = declared_symbols()
+    for n in ["msd_create", "msd_prefill", "msd_draft_tree", "msd_verify", "msd_accept_compact"]:
+        assert n in names
+
+
+def test_library_exports_every_declared_symbol(libmsd):
+    for n in declared_symbols():
+        assert hasattr(libmsd, n), n
+
+
+def test_create_rejects_bad_configs_before_touching_the_gpu(libmsd):
+    from paper_2505_14260_gb300 import msd, synth
+    ctx = ctypes.c_void_p()
+    assert libmsd.msd_create(None, None, ctypes.byref(ctx)) == msd.MSD_ERR_INVALID
+    wl = synth.WORKLOADS["tiny"]
+    good = msd.make_config(wl, 256)
+    w = msd.msd_weights()
+    cases = [dict(head_dim=96), dict(n_heads=3), dict(topk=0), dict(topk=17),
+             dict(tree_nodes=300), dict(tree_depth=0), dict(max_batch=0), dict(dtype=7),
+             dict(tree_nodes=64, tree_depth=2, topk=2)]     # k + (D-1)k^2 = 6 < 63
+    for kw in cases:
+        cfg = msd.make_config(wl, 256)
+        for k, v in kw.items():
+            setattr(cfg, k, v)
+        assert libmsd.msd_create(ctypes.byref(cfg), ctypes.byref(w), ctypes.byref(ctx)) == \
+            msd.MSD_ERR_INVALID, kw
+    # a valid config with null weights is rejected too
+    assert libmsd.msd_create(ctypes.byref(good), ctypes.byref(w), ctypes.byref(ctx)) == \
+        msd.MSD_ERR_INVALID
+
+
+def test_null_context_calls_fail_cleanly(libmsd):
+    from paper_2505_14260_gb300 import msd
+    assert libmsd.msd_last_error(None) == b"null context"
+    assert libmsd.msd_destroy(None) == msd.MSD_OK
+    assert libmsd.msd_verify(None, None, None, None, None) == msd.MSD_ERR_INVALID
+    assert libmsd.msd_state(None, None) == msd.MSD_ERR_INVALID
+
+
+def test_binding_fails_loudly_without_the_library(tmp_path, monkeypatch):
+    from paper_2505_14260_gb300 import msd
+    monkeypatch.setattr(msd, "_LIB_PATH", str(tmp_path / "missing.so"))
+    monkeypatch.setattr(msd, "_lib", None)
+    with pytest.raises(RuntimeError, match="not built"):
+        msd.lib()

@@ -1,0 +1,273 @@
+"""GPU path vs the CPU oracle on the tiny workload (fp32 and bf16), every step.
+
+Integer work (draft trees, top-k ids, argmax, accepted path, accepted length,
+bonus, index map) is compared bit-exactly given the kernels' own float
+outputs; floating-point outputs (draft logits, verify logits, KV caches) are
+compared with the oracle's float64 values within the stated tolerances. The
+oracle follows the kernels' integer decisions so that both sides stay on the
+same tokens for all steps.
+"""
+import numpy as np
+import pytest
+import torch
+
+from oracle import msd_oracle as O
+from paper_2505_14260_gb300 import msd, synth
+from tests.gpu_support import (KV_REL_L2, TOL, assert_close, open_engine, plant,
+                               record_buffers, rel_l2, top2_margin, tree_numpy)
+from tests.oracle_support import oracle_model, prompt_numpy
+
+pytestmark = pytest.mark.gpu
+
+
+def _kv_compare(eng, st, wl, b, L, dtype, what):
+    s = eng.state()
+    nh, hd = wl.n_heads, wl.head_dim
+    for l in range(wl.n_layers):
+        for kv, ref in ((0, st.K[l]), (1, st.V[l])):
+            g = s["target_kv"][l, kv, b, :, :L, :].float().cpu().numpy()      # [nh, L, hd]
+            r = np.asarray(ref[:L]).reshape(L, nh, hd).transpose(1, 0, 2)
+            assert rel_l2(g, r) <= KV_REL_L2[dtype], f"{what} layer {l} kv {kv}: {rel_l2(g, r)}"
+    Ld = st.dK.shape[0]
+    for kv, ref in ((0, st.dK), (1, st.dV)):
+        g = s["draft_kv"][kv, b, :, :Ld, :].float().cpu().numpy()
+        r = np.asarray(ref).reshape(Ld, nh, hd).transpose(1, 0, 2)
+        assert rel_l2(g, r) <= KV_REL_L2[dtype], f"{what} draft kv {kv}: {rel_l2(g, r)}"
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_tiny_all_steps_match_oracle(dtype):
+    wl = synth.WORKLOADS["tiny"].with_(dtype=dtype)
+    tol = TOL[dtype]
+    eng, w = open_engine(wl)
+    m = oracle_model(wl, w)
+    prompts = synth.make_prompts(wl)
+    ids, lens, vis, offs = msd.upload_prompts(prompts)
+    eng.prefill(ids, lens, vis, offs)
+    ids_np, vis_np = prompt_numpy(prompts[0])
+    st = O.prefill(m, ids_np, vis_np)
+    torch.cuda.synchronize()
+    root = int(eng.root_out.cpu()[0])
+    # the root is the argmax of the last prompt position: equal unless a near tie
+    if root != st.root:
+        z = O.lm_logits(m, O.target_forward(
+            m, O.embed_prompt(m, ids_np, vis_np), np.arange(len(ids_np)),
+            [(np.zeros((0, wl.hidden)),) * 2] * wl.n_layers, np.zeros(len(ids_np), int), None,
+            O.causal_vis(len(ids_np)))[0][-1:])[0]
+        assert top2_margin(z) <= tol["max_abs"]
+        st.root = root; st.pend_next = np.array([root]); st.emitted = [root]
+    _kv_compare(eng, st, wl, 0, st.L, dtype, "prefill")
+
+    D, k, N, V = wl.tree_depth, wl.topk, wl.tree_nodes, wl.vocab
+    for step in range(wl.steps):
+        rec = record_buffers(wl)
+        eng.draft_tree(record=rec)
+        torch.cuda.synchronize()
+        R = {n: t.cpu().numpy() for n, t in rec.items()}
+
+        def forced(p, rows_logits):
+            n = rows_logits.shape[0]
+            return R["topk_ids"][0, p, :n].astype(np.int64), R["topk_logp"][0, p, :n].astype(np.float32)
+
+        orec = O.DraftRecord()
+        otree = O.draft_tree(m, st, record=orec, forced_logp=forced)
+        toks, par, dep, mask = tree_numpy(eng.tree, 0)
+        # integer parity of the tree, given the kernels' top-k decisions
+        np.testing.assert_array_equal(toks, otree.tokens, err_msg=f"step {step} tokens")
+        np.testing.assert_array_equal(par, otree.parent, err_msg=f"step {step} parent")
+        np.testing.assert_array_equal(dep, otree.depth, err_msg=f"step {step} depth")
+        np.testing.assert_array_equal(mask, otree.mask_words(), err_msg=f"step {step} mask")
+        for p in range(D):
+            rows = orec.logits[p].shape[0]
+            g = R["logits"][0, p, :rows]
+            assert_close(g, orec.logits[p], tol, f"step {step} draft pass {p} logits")
+            for r in range(rows):
+                # top-k of the kernels' own logits, and their log-softmax
+                np.testing.assert_array_equal(R["topk_ids"][0, p, r], O.topk_ids(g[r], k))
+                lp = O.log_softmax(g[r].astype(np.float64))[R["topk_ids"][0, p, r]]
+                np.testing.assert_allclose(R["topk_logp"][0, p, r], lp, atol=2e-5, rtol=1e-5)
+
+        logits = torch.zeros(N, V, device="cuda")
+        eng.verify(logits=logits)
+        torch.cuda.synchronize()
+        g_logits = logits.cpu().numpy()
+        g_arg = eng.argmax.cpu().numpy().astype(np.int64)
+        vr = O.verify(m, st, otree)
+        assert_close(g_logits, vr.logits, tol, f"step {step} verify logits")
+        for i in range(N):
+            assert g_arg[i] == O.argmax_lowest(g_logits[i])          # bit-exact given logits
+            if top2_margin(vr.logits[i]) > tol["max_abs"]:
+                assert g_arg[i] == vr.argmax[i], f"step {step} node {i} argmax"
+
+        eng.accept_compact()
+        torch.cuda.synchronize()
+        opath, oa, obonus = O.accept(otree, g_arg)
+        path = eng.path.cpu().numpy()
+        assert int(eng.accept_len.cpu()[0]) == oa and int(eng.bonus.cpu()[0]) == obonus
+        np.testing.assert_array_equal(path[:oa + 1], opath)
+        assert (path[oa + 1:] == -1).all()
+        imap = eng.index_map.cpu().numpy()
+        np.testing.assert_array_equal(imap[:oa + 1], st.L + np.arange(oa + 1))
+        O.compact(st, otree, vr, opath, obonus)
+        s = eng.state()
+        assert int(s["seq_len"].cpu()[0]) == st.L and int(s["root"].cpu()[0]) == st.root
+        assert int(s["n_pending"].cpu()[0]) == oa + 1
+        _kv_compare(eng, st, wl, 0, st.L, dtype, f"step {step}")
+    eng.close()
+
+
+def _gpu_greedy_ar(eng, n_tokens):
+    """Plain greedy decoding on the GPU path: single-node trees, one per token."""
+    out = [int(eng.state()["root"].cpu()[0])]
+    t = msd.Tree(1, eng.cfg.tree_nodes)
+    for _ in range(n_tokens - 1):
+        eng.draft_tree()            # keeps the draft cache caught up
+        plant(t, 0, [out[-1]], [-1])
+        eng.verify(tree=t)
+        eng.accept_compact(tree=t)
+        out.append(int(eng.bonus.cpu()[0]))
+    return out
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_lossless_planted_trees_match_greedy(dtype):
+    """Speculative decoding emits the greedy autoregressive tokens (the lossless
+    property), with planted trees forcing full and partial acceptance."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype=dtype)
+    D = wl.tree_depth
+    steps = 6
+    n_ar = 1 + steps * (D + 1) + D + 2
+    prompts = synth.make_prompts(wl)
+    ids, lens, vis, offs = msd.upload_prompts(prompts)
+    eng, w = open_engine(wl, steps=n_ar)
+    eng.prefill(ids, lens, vis, offs)
+    ar = _gpu_greedy_ar(eng, n_ar)
+    eng.close()
+    if dtype == "f32":      # the fp32 GPU path reproduces the oracle's greedy decode
+        m = oracle_model(wl, w)
+        ids_np, vis_np = prompt_numpy(prompts[0])
+        assert ar == O.greedy_ar(m, ids_np, vis_np, n_ar)
+
+    eng, _ = open_engine(wl, w, steps=n_ar)
+    eng.prefill(ids, lens, vis, offs)
+    rng = np.random.default_rng(0)
+    t = msd.Tree(1, wl.tree_nodes)
+    emitted = [int(eng.root_out.cpu()[0])]
+    for s in range(steps):
+        j = len(emitted) - 1
+        depth = D if s % 2 == 0 else int(rng.integers(0, D))
+        chain = [emitted[-1]] + ar[j + 1:j + 1 + depth]
+        parent = list(range(-1, depth))
+        toks = list(chain)
+        if depth < D:                         # a wrong child where the chain stops
+            parent.append(depth); toks.append((ar[j + 1 + depth] + 1) % wl.vocab)
+        while len(toks) < wl.tree_nodes:      # distractor leaves hanging off the root
+            cand = int(rng.integers(0, wl.vocab))
+            if cand != ar[j + 1] and cand not in toks[1:]:
+                parent.append(0); toks.append(cand)
+        eng.draft_tree()
+        plant(t, 0, toks, parent)
+        eng.verify(tree=t)
+        eng.accept_compact(tree=t)
+        a = int(eng.accept_len.cpu()[0])
+        assert a == depth, (s, a, depth)
+        path = eng.path.cpu().numpy()[:a + 1]
+        emitted += [toks[p] for p in path[1:]] + [int(eng.bonus.cpu()[0])]
+    assert emitted == ar[:len(emitted)]
+    eng.close()
+
+
+def test_causality_non_ancestor_rows_bit_identical():
+    """Changing one node's token leaves every row not descended from it
+    bit-identical (rows see only their ancestors), on the bf16 tensor-core path."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype="bf16")
+    eng, w = open_engine(wl)
+    ids, lens, vis, offs = msd.upload_prompts(synth.make_prompts(wl))
+    eng.prefill(ids, lens, vis, offs)
+    eng.draft_tree()
+    toks, par, dep, mask = tree_numpy(eng.tree, 0)
+    N, V = wl.tree_nodes, wl.vocab
+    l1 = torch.zeros(N, V, device="cuda")
+    eng.verify(logits=l1)
+    j = N - 1
+    eng.tree.tokens[j] = (int(toks[j]) + 7) % V
+    l2 = torch.zeros(N, V, device="cuda")
+    eng.verify(logits=l2)
+    torch.cuda.synchronize()
+    desc = [(int(mask[i, j // 64]) >> (j % 64)) & 1 for i in range(N)]
+    for i in range(N):
+        if desc[i]:
+            assert not torch.equal(l1[i], l2[i])
+        else:
+            assert torch.equal(l1[i], l2[i]), i
+    eng.close()
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_linear_matches_torch(dtype):
+    """The GEMM building block against a plain PyTorch fp32 product, over ragged
+    shapes that span several tiles, a split K and a ragged tail."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype=dtype)
+    eng, _ = open_engine(wl)
+    dt = torch.float32 if dtype == "f32" else torch.bfloat16
+    g = torch.Generator(device="cuda").manual_seed(5)
+    for (M, K, O) in [(1, 256, 1024), (7, 512, 256), (16, 688, 256), (60, 4096, 384),
+                      (129, 256, 200), (300, 1024, 640), (960, 512, 128)]:
+        x = torch.randn(M, K, device="cuda", generator=g).to(dt)
+        wt = (torch.randn(O, K, device="cuda", generator=g) * 0.02).to(dt)
+        y = torch.zeros(M, O, device="cuda")
+        eng.linear(x, wt, y)
+        ref = x.float() @ wt.float().T
+        torch.cuda.synchronize()
+        err = (y - ref).abs().max().item()
+        assert err <= 1e-4 * max(1.0, ref.abs().max().item()), (M, K, O, err)
+        y2 = y.clone()
+        eng.linear(x, wt, y2, accumulate=True)
+        torch.cuda.synchronize()
+        assert (y2 - 2 * ref).abs().max().item() <= 2e-4 * max(1.0, ref.abs().max().item())
+        y3 = torch.zeros(M, O, device="cuda")
+        eng.linear(x, wt, y3)
+        torch.cuda.synchronize()
+        assert torch.equal(y, y3)             # deterministic (split-K order is fixed)
+    eng.close()
+
+
+def test_bad_planted_tree_sets_device_status():
+    """A planted tree whose root token is not the current root is detected on the
+    device; the next call reports MSD_ERR_DEVICE."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype="f32")
+    eng, _ = open_engine(wl)
+    ids, lens, vis, offs = msd.upload_prompts(synth.make_prompts(wl))
+    eng.prefill(ids, lens, vis, offs)
+    t = msd.Tree(1, wl.tree_nodes)
+    root = int(eng.root_out.cpu()[0])
+    plant(t, 0, [(root + 1) % wl.vocab], [-1])
+    eng.verify(tree=t)
+    torch.cuda.synchronize()
+    with pytest.raises(msd.MsdError) as e:
+        eng.verify(tree=t)
+    assert e.value.status == msd.MSD_ERR_DEVICE
+    eng.close()
+
+
+def test_capacity_is_refused_on_the_host():
+    wl = synth.WORKLOADS["tiny"].with_(dtype="f32")
+    w = synth.make_weights(wl)
+    from tests.gpu_support import to_device
+    prompts = synth.make_prompts(wl)
+    L = prompts[0].length
+    cfg = msd.make_config(wl, L + wl.tree_depth + 1 + 2)       # room for about one step
+    eng = msd.Engine(cfg, to_device(w))
+    ids, lens, vis, offs = msd.upload_prompts(prompts)
+    eng.prefill(ids, lens, vis, offs)
+    with pytest.raises(msd.MsdError) as e:
+        for _ in range(4):
+            eng.step()
+    assert e.value.status == msd.MSD_ERR_CAPACITY
+    eng.close()
+    small = msd.make_config(wl, L)                              # prompt alone does not fit
+    eng2 = msd.Engine(small, to_device(w))
+    with pytest.raises(msd.MsdError) as e:
+        eng2.prefill(ids, lens, vis, offs)
+    assert e.value.status == msd.MSD_ERR_CAPACITY
+    eng2.close()
