@@ -184,6 +184,30 @@ msd_status msd_linear(msd_ctx *ctx, const void *x_dev, int32_t ldx, int32_t m, i
                       const void *w_dev, int32_t o, float *y_dev, int32_t ldy,
                       int32_t accumulate, void *stream);
 
+/* Allocation-free GEMM: the same y (=|+=) x w^T as msd_linear for bf16
+ * operands, for callers that cannot allocate device memory (a host program
+ * whose device memory is all owned by its own pool allocator, code running
+ * where an allocation would synchronise the device or is not permitted, a
+ * plug-in handed buffers but no allocator). It needs no context and allocates
+ * nothing: its split-K scratch is one static device array of 16 MiB of fp32
+ * partials plus 4096 int tile tickets, which every GPU that loads this library
+ * holds until the process exits. The paper has no counterpart; this is a
+ * service of the library, not a step of the method.
+ * Arguments are those of msd_linear (x [m][ldx], w [o][k] bf16 with ldx and k
+ * multiples of 8, y [m][ldy] fp32, all device memory on the current device).
+ * The first call made on a device looks up the array's device address on that
+ * device (cudaGetSymbolAddress) and sets the kernel's shared-memory limit;
+ * make that first call before any stream capture. Every call shares the array
+ * and it keeps the last call's contents; the tile tickets are cleared on
+ * `stream` before each launch that uses them. Calls that overlap on the GPU
+ * (other streams, other host threads) race on the array: serialise them.
+ * Errors: MSD_ERR_INVALID (null pointer, non-positive size, bad stride or
+ * alignment), MSD_ERR_CAPACITY (the shape's split-K partials would exceed the
+ * 16 MiB array or its 4096 tickets), MSD_ERR_CUDA (a runtime call failed). */
+msd_status msd_linear_noalloc(const void *x_dev, int32_t ldx, int32_t m, int32_t k,
+                              const void *w_dev, int32_t o, float *y_dev, int32_t ldy,
+                              int32_t accumulate, void *stream);
+
 /* Profiling counters (tracing subsystem). kernel_launches counts every kernel
  * the library has launched in this process. While profiling is enabled on a
  * context, each tensor-core GEMM launch (bf16 contexts) is bracketed by CUDA

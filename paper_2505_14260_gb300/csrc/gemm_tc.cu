@@ -25,10 +25,12 @@
 
 #include <cstdio>
 #include <cstring>
+#include <mutex>
 #include <unordered_map>
 #include <vector>
 
 #include "gemm_tc.h"
+#include "msd.h"
 
 namespace msd {
 
@@ -511,3 +513,140 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
 }
 
 }  // namespace msd
+
+// ---------------------------------------------------------------------------
+// Allocation-free GEMM entry point (msd_linear_noalloc in include/msd.h).
+//
+// Some callers cannot call cudaMalloc: a host program whose device memory is
+// entirely owned by its own pool allocator, code that runs where an allocation
+// would synchronise the device or is not permitted, or a plug-in that is handed
+// buffers but no allocator. For them the split-K scratch of the tensor-core
+// GEMM lives in one file-scope device array, loaded with the library and held
+// by every GPU that loads it until the process exits.
+//
+// Layout of the array: NOALLOC_COUNTERS int tile tickets, then the fp32
+// split-K partials (NOALLOC_PARTIAL_BYTES). In host code the array's name is
+// only a host-side stand-in; the device address comes from
+// cudaGetSymbolAddress, taken once per device (with that device current) on
+// the first call made on it. Every call shares the array and it keeps the last
+// call's contents: the tickets are cleared on the caller's stream before each
+// launch that uses them, and calls that overlap on the GPU race on the array.
+// ---------------------------------------------------------------------------
+namespace msd {
+namespace {
+constexpr int NOALLOC_COUNTERS = 4096;
+constexpr size_t NOALLOC_PARTIAL_BYTES = 16ull << 20;
+constexpr size_t NOALLOC_BYTES = NOALLOC_COUNTERS * sizeof(int) + NOALLOC_PARTIAL_BYTES;
+constexpr int NOALLOC_MAX_DEVICES = 64;
+}  // namespace
+
+static __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_BYTES];
+
+namespace {
+struct NoAllocDevice {
+    bool ready = false;
+    unsigned char *scratch = nullptr;   // device address of g_noalloc_scratch
+    int num_sms = 0;
+};
+std::mutex g_noalloc_mu;
+NoAllocDevice g_noalloc_dev[NOALLOC_MAX_DEVICES];
+GemmPlan g_noalloc_maps;                // host-side tensor-map cache only (no device memory)
+}  // namespace
+
+}  // namespace msd
+
+extern "C" msd_status msd_linear_noalloc(const void *x, int32_t ldx, int32_t m, int32_t k,
+                                         const void *w, int32_t o, float *y, int32_t ldy,
+                                         int32_t accumulate, void *stream) {
+    using namespace msd;
+    constexpr msd_status OK = MSD_OK, INVALID = MSD_ERR_INVALID, CAPACITY = MSD_ERR_CAPACITY,
+                         CUDA_ERR = MSD_ERR_CUDA;
+    if (!x || !w || !y || m <= 0 || k <= 0 || o <= 0 || ldx < k || ldy < o) return INVALID;
+    if (ldx % 8 || k % 8) return INVALID;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= NOALLOC_MAX_DEVICES) return CUDA_ERR;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    NoAllocDevice &d = g_noalloc_dev[dev];
+    if (!d.ready) {
+        void *ptr = nullptr;
+        if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return CUDA_ERR;
+        if (cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
+            return CUDA_ERR;
+        if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 200 * 1024 + 1024) != cudaSuccess)
+            return CUDA_ERR;
+        if (!g_noalloc_maps.encode) {
+            cudaDriverEntryPointQueryResult q;
+            void *fn = nullptr;
+            if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
+                                                 cudaEnableDefault, &q) != cudaSuccess ||
+                q != cudaDriverEntryPointSuccess || !fn)
+                return CUDA_ERR;
+            g_noalloc_maps.encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+        }
+        d.scratch = static_cast<unsigned char *>(ptr);
+        d.ready = true;
+    }
+    // The same plan as the context GEMM (tile shape, stages, split-K choice).
+    const int M = m, K = k, O = o;
+    const int tiles = (O + BM - 1) / BM;
+    const int nt = (M + 255) / 256;
+    int BN = (M + nt - 1) / nt;
+    BN = ((BN + 15) / 16) * 16;
+    const int kblocks = (K + BK - 1) / BK;
+    const uint32_t stage_bytes = A_BYTES + (uint32_t)BN * BK * 2;
+    const int ctas_per_sm = BN <= 128 ? 2 : 1;
+    int stages = (int)((ctas_per_sm == 2 ? 100u * 1024u : 200u * 1024u) / stage_bytes);
+    stages = stages < 2 ? 2 : (stages > MAX_STAGES ? MAX_STAGES : stages);
+    const size_t smem = 1024 + (size_t)stages * stage_bytes;
+    const long base = (long)tiles * nt;
+    const long slots = (long)d.num_sms * ctas_per_sm;
+    const size_t tile_bytes = (size_t)BN * BM * sizeof(float);
+    int best_s = 1;
+    double best = 1e30;
+    for (int sp = 1; sp <= 16 && sp <= kblocks; ++sp) {
+        const int kps = (kblocks + sp - 1) / sp;
+        const int se = (kblocks + kps - 1) / kps;
+        if (se > 1 && ((size_t)base * se * tile_bytes > WS_BYTES || base > N_COUNTERS)) continue;
+        const long waves = (base * se + slots - 1) / slots;
+        const double cost = (double)waves * kps + (se > 1 ? 2.0 : 0.0);
+        if (cost < best - 1e-9) { best = cost; best_s = se; }
+    }
+    const int kps = (kblocks + best_s - 1) / best_s;
+    const int splits = (kblocks + kps - 1) / kps;
+    // Sizes whose split-K partials or tickets exceed the static array are refused.
+    if (splits > 1 && ((size_t)base * splits * tile_bytes > NOALLOC_PARTIAL_BYTES ||
+                       base > NOALLOC_COUNTERS))
+        return CAPACITY;
+
+    TcParams tp;
+    memset(&tp, 0, sizeof tp);
+    tp.n_seg = 1;
+    tp.seg_tiles[0] = tiles;
+    tp.seg_rows[0] = O;
+    tp.seg_out[0] = 0;
+    tp.M = M;
+    tp.kblocks = kblocks;
+    tp.splits = splits;
+    tp.kb_per_split = kps;
+    tp.BN = BN;
+    tp.n_tiles_n = nt;
+    tp.stages = stages;
+    tp.tmem_cols = BN <= 32 ? 32 : (BN <= 64 ? 64 : (BN <= 128 ? 128 : 256));
+    tp.Y = y;
+    tp.ldy = ldy;
+    tp.epi = accumulate ? EPI_ADD : EPI_STORE;
+    tp.counters = reinterpret_cast<int *>(d.scratch);
+    tp.ws = reinterpret_cast<float *>(d.scratch + NOALLOC_COUNTERS * sizeof(int));
+    tp.status = nullptr;
+    const CUtensorMap *mw = get_map(&g_noalloc_maps, w, O, K, K, BM, nullptr);
+    const CUtensorMap *mx = get_map(&g_noalloc_maps, x, M, K, ldx, BN, nullptr);
+    if (!mw || !mx) return INVALID;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    if (splits > 1 && cudaMemsetAsync(tp.counters, 0, sizeof(int) * base, s) != cudaSuccess)
+        return CUDA_ERR;
+    gemm_tc_kernel<<<dim3(tiles, nt, splits), THREADS, smem, s>>>(*mw, *mw, *mw, *mx, tp);
+    note_launch();
+    return cudaGetLastError() == cudaSuccess ? OK : CUDA_ERR;
+}
+

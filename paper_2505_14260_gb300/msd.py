@@ -71,6 +71,8 @@ _SIGNATURES = {
                                      c_void_p, c_void_p, c_void_p]),
     "msd_linear": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32,
                              c_void_p, c_int32, c_int32, c_void_p]),
+    "msd_linear_noalloc": (c_int32, [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32,
+                                     c_void_p, c_int32, c_int32, c_void_p]),
     "msd_profile_enable": (c_int32, [c_void_p, c_int32]),
     "msd_profile_read": (c_int32, [c_void_p, POINTER(msd_profile)]),
     "msd_state": (c_int32, [c_void_p, POINTER(msd_state_view)]),
