@@ -52,6 +52,8 @@ def parse():
     ap.add_argument("--impl", default="msd", choices=["msd", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--gemm", default=None,
+                    help="M,K,O: time the tensor-core GEMM alone on that shape (kernel case)")
     return ap.parse_args()
 
 
@@ -217,6 +219,41 @@ def run_reference(args, rank, world):
     print(json.dumps(line), flush=True)
 
 
+def run_gemm_case(args):
+    """One GEMM shape through msd_linear: weights [O,K] bf16 larger than L2 for
+    the 7B shapes, timed per launch with CUDA events (a small kernel case for
+    ncu captures and tuning)."""
+    import torch
+    from paper_2505_14260_gb300 import msd, synth
+    M, K, O = (int(v) for v in args.gemm.split(","))
+    wl = synth.WORKLOADS["tiny"].with_(dtype="bf16")
+    w = {k: v.cuda() for k, v in synth.make_weights(wl).items() if hasattr(v, "cuda")}
+    w["layers"] = [{n: t.cuda() for n, t in lw.items()} for lw in synth.make_weights(wl)["layers"]]
+    w["draft"] = {n: t.cuda() for n, t in synth.make_weights(wl)["draft"].items()}
+    eng = msd.Engine(msd.make_config(wl, 256), w)
+    g = torch.Generator(device="cuda").manual_seed(3)
+    x = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
+    n_w = max(2, (512 << 20) // (O * K * 2) + 1)          # rotate weights: > L2 per pass
+    ws = [(torch.randn(O, K, device="cuda", generator=g) * 0.02).to(torch.bfloat16) for _ in range(n_w)]
+    y = torch.zeros(M, O, device="cuda")
+    for i in range(3):
+        eng.linear(x, ws[i % n_w], y)
+    torch.cuda.synchronize()
+    times = []
+    for i in range(20):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        e0.record(); eng.linear(x, ws[i % n_w], y); e1.record()
+        e1.synchronize()
+        times.append(e0.elapsed_time(e1))
+    hbm, kind = peaks()
+    ms = statistics.median(times)
+    byts = O * K * 2 + M * K * 2 + M * O * 4
+    print(json.dumps({"case": "gemm", "M": M, "K": K, "O": O, "ms_median": ms, "ms_min": min(times),
+                      "gbs": byts / (ms / 1e3) / 1e9, "frac": byts / (ms / 1e3) / 1e9 / hbm,
+                      "peak": hbm, "peak_kind": kind}), flush=True)
+    eng.close()
+
+
 def run_msd(args, rank, world, local_rank):
     import numpy as np
     import torch
@@ -247,10 +284,12 @@ def run_msd(args, rank, world, local_rank):
     stream = torch.cuda.current_stream()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
+    torch.cuda.nvtx.range_push("timed")
     e0.record(stream)
     for _ in range(K):
         eng.step()
     e1.record(stream)
+    torch.cuda.nvtx.range_pop()
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1)
     clk = clocks.stop()
@@ -353,6 +392,9 @@ def main():
     local_rank = int(os.environ.get("LOCAL_RANK", "0"))
     if args.impl == "reference":
         run_reference(args, rank, world)
+        return
+    if args.gemm:
+        run_gemm_case(args)
         return
     import torch
     import torch.distributed as dist
