@@ -1,0 +1,21 @@
+// Tree-masked attention on the tensor cores (bf16 path).
+#pragma once
+
+#include "kernels.h"
+
+namespace msd {
+
+struct AttnTcPlan;
+
+// Workspace for split-KV partials and the per-(row tile, head) tickets.
+bool attn_tc_plan_create(AttnTcPlan **out, size_t ws_bytes, int n_counters);
+void attn_tc_plan_destroy(AttnTcPlan *p);
+
+// a.R rows grouped by request in blocks of rows_per_req; every row's plen is
+// at most p_bound (used to size the split of the cache range). B is the
+// number of requests the cache buffers hold. Returns false if the shape is not
+// supported (the caller reports it).
+bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req,
+                         int p_bound, int *status, cudaStream_t s);
+
+}  // namespace msd

@@ -17,6 +17,7 @@
 #include "kernels.h"
 #include "kernels_tree.h"
 #include "gemm_tc.h"
+#include "attn_tc.h"
 
 using namespace msd;
 
@@ -52,6 +53,7 @@ struct msd_ctx {
     cudaEvent_t status_ev = nullptr;
     bool status_pending = false;
     GemmPlan *gplan = nullptr;
+    AttnTcPlan *aplan = nullptr;
     std::vector<void *> allocs;
     std::vector<long> L_bound;
     bool prefilled = false;
@@ -133,9 +135,35 @@ void gemm<bf16>(msd_ctx *c, const bf16 *X, int ldx, int M, int K, const GemmW &W
 
 // One pre-norm decoder layer over R rows (target or draft).
 template <typename T>
+void attention(msd_ctx *c, const AttnArgs<T> &a, int rows_per_req, int p_bound, cudaStream_t s);
+
+template <>
+void attention<float>(msd_ctx *c, const AttnArgs<float> &a, int, int, cudaStream_t s) {
+    launch_attention<float>(a, s);
+}
+
+template <>
+void attention<bf16>(msd_ctx *c, const AttnArgs<bf16> &a, int rows_per_req, int p_bound,
+                     cudaStream_t s) {
+    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, p_bound, c->status, s))
+        c->err = "tensor-core attention: unsupported shape or workspace too small";
+}
+
+// Largest L any request may have now (host-side upper bound).
+int max_L_bound(const msd_ctx *c) {
+    long m = 1;
+    for (long v : c->L_bound) m = std::max(m, v);
+    return (int)std::min<long>(m, c->S);
+}
+
+// One pre-norm decoder layer over R rows (target or draft). Rows come in
+// blocks of rows_per_req per request; every row attends to at most p_bound
+// cache positions.
+template <typename T>
 void run_layer(msd_ctx *c, const msd_layer &lw, int R, const RowDesc *rows, T *kdst, T *vdst,
                int dst_slots, const T *ck, const T *cv, int cslots, const T *tk, const T *tv,
-               int tslots, const uint64_t *mask, int mw, cudaStream_t s) {
+               int tslots, const uint64_t *mask, int mw, int rows_per_req, int p_bound,
+               cudaStream_t s) {
     const int H = c->H, F = c->F;
     const float eps = c->cfg.rms_eps;
     launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.attn_norm), R, H, eps,
@@ -160,7 +188,7 @@ void run_layer(msd_ctx *c, const msd_layer &lw, int R, const RowDesc *rows, T *k
     a.hd = c->hd;
     a.scale = 1.0f / sqrtf((float)c->hd);
     a.out = static_cast<T *>(c->attn);
-    launch_attention<T>(a, s);
+    attention<T>(c, a, rows_per_req, p_bound, s);
     GemmW wo = {{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1};
     gemm<T>(c, static_cast<const T *>(c->attn), H, R, H, wo, H, c->x, H, EPI_ADD, s);
     launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.mlp_norm), R, H, eps,
@@ -216,7 +244,7 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
             for (int l = 0; l < c->NL; ++l) {
                 T *K = tkv<T>(c, c->target_kv, l, 0, c->S), *Vv = tkv<T>(c, c->target_kv, l, 1, c->S);
                 run_layer<T>(c, c->layers[l], n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr,
-                             nullptr, 0, nullptr, 0, s);
+                             nullptr, 0, nullptr, 0, n, r0 + n, s);
             }
             launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), n, H, c->cfg.rms_eps,
                               static_cast<T *>(c->h_all) + (size_t)r0 * H, s);
@@ -240,7 +268,7 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
                                     c->src + r0, n, H, s);
             T *K = tkv<T>(c, c->draft_kv, 0, 0, c->S), *Vv = tkv<T>(c, c->draft_kv, 0, 1, c->S);
             run_layer<T>(c, c->w.draft, n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr, nullptr, 0,
-                         nullptr, 0, s);
+                         nullptr, 0, n, r0 + n, s);
             CU(cudaStreamSynchronize(s));
         }
         launch_prefill_finish<T>(c->argmax_tmp, h_last, b, L, D1, H, c->seq_len, c->n_pend, c->root,
@@ -304,8 +332,9 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
                             E, B, H, D1, V, static_cast<T *>(c->xfc), c->rows, c->status, s);
     gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, R1, 2 * H, one(c->w.draft_fc, H), H, c->x, H,
             EPI_STORE, s);
+    const int pb = max_L_bound(c);
     run_layer<T>(c, c->w.draft, R1, c->rows, dK, dV, S, dK, dV, S, nullptr, nullptr, 0, nullptr, 0,
-                 s);
+                 D1, pb, s);
     launch_root_gather<T>(c->x, c->n_pend, B, D1, H, c->hhat_root, static_cast<T *>(c->xr), s);
     gemm<T>(c, static_cast<const T *>(c->xr), H, B, H, one(c->w.lm_head, V), V, c->logits, V,
             EPI_STORE, s);
@@ -320,7 +349,7 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
         gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, Rk, 2 * H, one(c->w.draft_fc, H), H,
                 c->x, H, EPI_STORE, s);
         run_layer<T>(c, c->w.draft, Rk, c->rows, tK, tV, c->Td, dK, dV, S, tK, tV, c->Td,
-                     c->row_mask, c->Wd, s);
+                     c->row_mask, c->Wd, k, pb, s);
         launch_hhat_store<T>(c->x, c->rows, Rk, c->Td, H, c->hhat_slot, static_cast<T *>(c->xr), s);
         gemm<T>(c, static_cast<const T *>(c->xr), H, Rk, H, one(c->w.lm_head, V), V, c->logits, V,
                 EPI_STORE, s);
@@ -342,6 +371,7 @@ template <typename T>
 msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, float *logits_dev,
                        cudaStream_t s) {
     const int B = c->B, N = c->N, H = c->H, V = c->V, R = B * N;
+    const int pb = max_L_bound(c);
     TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
     launch_verify_setup(t, c->seq_len, c->root, B, N, V, c->rows, c->src, c->vmask, c->status, s);
     launch_embed_rows<T>(static_cast<const T *>(c->w.embed), nullptr, c->src, R, H, c->x, nullptr,
@@ -350,7 +380,7 @@ msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, fl
         T *K = tkv<T>(c, c->target_kv, l, 0, c->S), *Vv = tkv<T>(c, c->target_kv, l, 1, c->S);
         T *tK = tkv<T>(c, c->tree_kv, l, 0, N), *tV = tkv<T>(c, c->tree_kv, l, 1, N);
         run_layer<T>(c, c->layers[l], R, c->rows, tK, tV, N, K, Vv, c->S, tK, tV, N, c->vmask, c->W,
-                     s);
+                     N, pb, s);
     }
     launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), R, H, c->cfg.rms_eps,
                       static_cast<T *>(c->hT), s);
@@ -499,6 +529,7 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     if (ok) ok = cudaMallocHost(&c->status_host, sizeof(int)) == cudaSuccess;
     if (ok) ok = cudaEventCreateWithFlags(&c->status_ev, cudaEventDisableTiming) == cudaSuccess;
     if (ok && cfg->dtype == MSD_BF16) ok = gemm_plan_create(&c->gplan, c->Rmax, c->H, c->F, c->V);
+    if (ok && cfg->dtype == MSD_BF16) ok = attn_tc_plan_create(&c->aplan, 32ull << 20, 16384);
     if (!ok) {
         msd_destroy(c);
         cudaGetLastError();
@@ -530,6 +561,7 @@ msd_status msd_destroy(msd_ctx *c) {
     if (c->status_host) cudaFreeHost(c->status_host);
     if (c->status_ev) cudaEventDestroy(c->status_ev);
     if (c->gplan) gemm_plan_destroy(c->gplan);
+    if (c->aplan) attn_tc_plan_destroy(c->aplan);
     delete c;
     return MSD_OK;
 }
