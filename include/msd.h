@@ -178,8 +178,11 @@ msd_status msd_accept_compact(msd_ctx *ctx, const msd_tree *tree,
  * y[i][j] (= or, if accumulate != 0, +=) sum_t x[i][t] * w[j][t] for i < m,
  * j < o, t < k. x [m][ldx] and w [o][k] are in the context dtype (bf16 rows
  * 16-byte aligned: ldx and k multiples of 8), y [m][ldy] is fp32; all device.
- * bf16 runs on the tcgen05 tensor-core GEMM, fp32 on the CUDA-core GEMM.
- * Errors: MSD_ERR_INVALID on null pointers, non-positive sizes or bad strides. */
+ * bf16 runs on the tcgen05 tensor-core GEMM of the step: w is first re-laid
+ * into the context's packing scratch (grown on demand, so this call may
+ * allocate), then multiplied; fp32 runs on the CUDA-core GEMM.
+ * Errors: MSD_ERR_INVALID on null pointers, non-positive sizes or bad strides,
+ * MSD_ERR_OOM if the packing scratch cannot grow. */
 msd_status msd_linear(msd_ctx *ctx, const void *x_dev, int32_t ldx, int32_t m, int32_t k,
                       const void *w_dev, int32_t o, float *y_dev, int32_t ldy,
                       int32_t accumulate, void *stream);

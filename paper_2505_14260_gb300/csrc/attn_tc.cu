@@ -30,6 +30,7 @@ namespace {
 constexpr int ROWS = 64;          // query rows per CTA
 constexpr int KT = 64;            // keys per tile
 constexpr int STAGES = 3;
+constexpr int MAX_SPLITS = 32;    // cache splits + the tree split
 constexpr unsigned long long ATTN_TIMEOUT_NS = 2000000000ull;
 
 struct AttnTcParams {
@@ -123,6 +124,7 @@ __global__ void __launch_bounds__(128)
     attn_tc_kernel(const __grid_constant__ CUtensorMap mkc, const __grid_constant__ CUtensorMap mvc,
                    const __grid_constant__ CUtensorMap mkt, const __grid_constant__ CUtensorMap mvt,
                    const AttnTcParams p) {
+    allow_dependents();
     constexpr int NB = HD / 64;                   // 64-wide boxes per row
     constexpr int TILE_BYTES = KT * HD * 2;       // one K (or V) tile
     constexpr int NT_O = HD / 8;                  // O n-tiles per warp
@@ -364,21 +366,43 @@ __global__ void __launch_bounds__(128)
     __syncthreads();
     if (!s_last) return;
     __threadfence();
-    for (int idx = threadIdx.x; idx < (r_end - r0) * HD; idx += 128) {
-        const int rr = r0 + idx / HD, c = idx - (idx / HD) * HD;
+    // the KV stages are idle now: reuse them for the per-row split weights
+    float (*s_w)[MAX_SPLITS] =
+        reinterpret_cast<float (*)[MAX_SPLITS]>(smem_raw + (kv_s - su32(smem_raw)));
+    // weights of each split per row: exp2(m_s - M) / sum_s exp2(m_s - M) l_s
+    const int nrows = r_end - r0;
+    for (int rr = threadIdx.x; rr < nrows; rr += 128) {
         float M = -INFINITY;
         for (int sp = 0; sp < nsplit; ++sp)
-            M = fmaxf(M, __ldcg(p.ws_ml + (((size_t)sp * p.R + rr) * p.nh + h) * 2));
-        float num = 0.f, den = 0.f;
-        if (M != -INFINITY) {
-            for (int sp = 0; sp < nsplit; ++sp) {
-                const size_t b2 = ((size_t)sp * p.R + rr) * p.nh + h;
-                const float wgt = exp2f(__ldcg(p.ws_ml + b2 * 2) - M);
-                num += wgt * __ldcg(p.ws_o + b2 * HD + c);
-                den += wgt * __ldcg(p.ws_ml + b2 * 2 + 1);
-            }
+            M = fmaxf(M, __ldcg(p.ws_ml + (((size_t)sp * p.R + r0 + rr) * p.nh + h) * 2));
+        float den = 0.f;
+        for (int sp = 0; sp < nsplit; ++sp) {
+            const float2 ml = __ldcg(reinterpret_cast<const float2 *>(
+                p.ws_ml + (((size_t)sp * p.R + r0 + rr) * p.nh + h) * 2));
+            const float w = M == -INFINITY ? 0.f : exp2f(ml.x - M);
+            s_w[rr][sp] = w;
+            den += w * ml.y;
         }
-        p.out[(size_t)rr * H + h * HD + c] = __float2bfloat16_rn(den > 0.f ? num / den : 0.f);
+        const float inv = den > 0.f ? 1.f / den : 0.f;
+        for (int sp = 0; sp < nsplit; ++sp) s_w[rr][sp] *= inv;
+    }
+    __syncthreads();
+    // O = sum_s w_s O_s, float4 per thread, splits unrolled for independent loads
+    constexpr int C4 = HD / 4;
+    for (int e = threadIdx.x; e < nrows * C4; e += 128) {
+        const int rr = e / C4, c4 = e - rr * C4;
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll 4
+        for (int sp = 0; sp < nsplit; ++sp) {
+            const float4 v = __ldcg(reinterpret_cast<const float4 *>(
+                p.ws_o + (((size_t)sp * p.R + r0 + rr) * p.nh + h) * HD) + c4);
+            const float w = s_w[rr][sp];
+            acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+        }
+        uint2 packed;
+        packed.x = pack_bf16(acc.x, acc.y);
+        packed.y = pack_bf16(acc.z, acc.w);
+        *reinterpret_cast<uint2 *>(p.out + (size_t)(r0 + rr) * H + h * HD + c4 * 4) = packed;
     }
     if (threadIdx.x == 0) p.counters[ticket] = 0;
 }
@@ -472,7 +496,7 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     const int pb = std::max(1, std::min(p_bound, a.cache_slots));
     const int cache_tiles = (pb + KT - 1) / KT;
     int want = (int)((2L * p->num_sms + base - 1) / base) - has_tree;
-    want = std::max(1, std::min(want, cache_tiles));
+    want = std::max(1, std::min(std::min(want, cache_tiles), MAX_SPLITS - 1));
     int chunk_tiles = (cache_tiles + want - 1) / want;
     int nsplit = (cache_tiles + chunk_tiles - 1) / chunk_tiles;
     auto fits = [&](int ns) {

@@ -36,6 +36,13 @@ __device__ __forceinline__ void set_status(int *st, int code) {
     if (st) atomicCAS(st, 0, code);
 }
 
+// Lets a dependent kernel launched with programmatic stream serialization
+// start its prologue now; it still waits for this grid before reading any of
+// its outputs (griddepcontrol.wait).
+__device__ __forceinline__ void allow_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;");
+}
+
 template <typename T> __device__ __forceinline__ float to_f(T v);
 template <> __device__ __forceinline__ float to_f<float>(float v) { return v; }
 template <> __device__ __forceinline__ float to_f<bf16>(bf16 v) { return __bfloat162float(v); }

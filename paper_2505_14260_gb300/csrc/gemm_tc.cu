@@ -113,6 +113,18 @@ __device__ __forceinline__ void tma_load_2d(uint32_t dst, const CUtensorMap *map
         : "memory");
 }
 
+// Contiguous global -> shared copy completing on an mbarrier (16-byte aligned).
+__device__ __forceinline__ void bulk_load(uint32_t dst, const void *src, uint32_t bytes, uint32_t bar) {
+    asm volatile(
+        "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+            dst),
+        "l"(src), "r"(bytes), "r"(bar)
+        : "memory");
+}
+
+__device__ __forceinline__ void pdl_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void pdl_trigger() { asm volatile("griddepcontrol.launch_dependents;"); }
+
 // Shared-memory matrix descriptor: K-major operand, 128-byte swizzle, 8-row
 // core-matrix groups 1024 bytes apart, sm100 descriptor version 1.
 __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
@@ -319,6 +331,325 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
 }
 
+// ---------------------------------------------------------------------------
+// Persistent stream-K variant (the context GEMM).
+//
+// The work is the list of (tile, K-block) units, tile-major; CTA c of G takes
+// units [c*U/G, (c+1)*U/G), so every CTA streams about the same number of
+// weight bytes through one continuously running TMA -> MMA pipeline, across
+// tile boundaries. Roles (192 threads): warp 0 lane 0 issues TMA, warp 1
+// allocates TMEM and its lane 0 issues the MMAs, warps 2-5 drain the
+// accumulators. Two TMEM accumulators let the epilogue of one tile overlap the
+// MMAs of the next. A tile whose K range is cut between CTAs ("pieces") is
+// fixed up through the workspace: each piece is written to its CTA's slot (a
+// CTA has at most two cut tiles, its first and its last), and the CTA that
+// takes the tile's last ticket sums the pieces in CTA order (deterministic)
+// and applies the epilogue. No CTA ever waits on another.
+// ---------------------------------------------------------------------------
+constexpr int P_THREADS = 192;
+constexpr int P_MAX_STAGES = 12;
+constexpr int P_MAX_PIECES = 128;   // pieces of one cut tile (CTAs sharing it)
+
+struct PkParams {
+    int n_seg;
+    int seg_tiles[3];
+    int seg_rows[3];
+    int seg_out[3];
+    int M, kblocks, BN, n_tiles_n, stages, acc_stride, tmem_cols, grid;
+    long long units;
+    const bf16 *wpacked;    // pre-packed weights (tile-contiguous, pre-swizzled) or null
+    float *Y;
+    int ldy, epi;
+    float *ws;
+    int *counters;
+    int *status;
+};
+
+// CTA owning unit u under the balanced partition u0(c) = floor(c * U / G).
+__device__ __forceinline__ int owner_cta(long long u, long long U, int G) {
+    return (int)(((u + 1) * (long long)G - 1) / U);
+}
+
+__global__ void __launch_bounds__(P_THREADS, 1)
+    gemm_persist_kernel(const __grid_constant__ CUtensorMap mx, const PkParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t bars[2 * P_MAX_STAGES + 4];
+    __shared__ uint32_t tmem_base;
+    __shared__ volatile int abort_flag;
+    __shared__ int s_reduce;
+    __shared__ int s_slot[P_MAX_PIECES];
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int cta = blockIdx.x;
+    const long long U = p.units;
+    const long long u0 = (long long)cta * U / p.grid, u1 = (long long)(cta + 1) * U / p.grid;
+    const int KB = p.kblocks, stages = p.stages, BN = p.BN;
+    const uint32_t b_bytes = (uint32_t)BN * BK * 2;
+
+    const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+    const uint32_t a_base = sbase, b_base = sbase + stages * A_BYTES;
+    const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[P_MAX_STAGES]);
+    const uint32_t accf0 = smem_u32(&bars[2 * P_MAX_STAGES]);
+    const uint32_t acce0 = smem_u32(&bars[2 * P_MAX_STAGES + 2]);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < stages; ++s) {
+            mbar_init(full0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            mbar_init(accf0 + 8 * a, 1);
+            mbar_init(acce0 + 8 * a, 128);
+        }
+        abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(&tmem_base)),
+                     "r"(p.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tmem_base;
+
+    // (tile) -> weight segment map, weight rows, token rows
+    auto tile_geom = [&](int t, int &seg, int &row0, int &n0) {
+        const int wt = t / p.n_tiles_n, nt = t - wt * p.n_tiles_n;
+        int w = wt;
+        seg = 0;
+        while (seg < p.n_seg - 1 && w >= p.seg_tiles[seg]) {
+            w -= p.seg_tiles[seg];
+            ++seg;
+        }
+        row0 = w * BM;
+        n0 = nt * BN;
+    };
+
+    if (warp == 0) {
+        if (lane == 0) {
+            pdl_trigger();
+            asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
+            // Weights never depend on the previous kernel: the first stages'
+            // weight blocks are requested before waiting for it.
+            const long long n_pre = min((long long)stages, u1 - u0);
+            for (long long j = 0; j < n_pre; ++j) {
+                const int t = (int)((u0 + j) / KB), kb = (int)(u0 + j - (long long)t * KB);
+                const long long blk = (long long)(t / p.n_tiles_n) * KB + kb;
+                mbar_expect_tx(full0 + 8 * (int)j, A_BYTES + b_bytes);
+                bulk_load(a_base + (int)j * A_BYTES, p.wpacked + blk * (A_BYTES / 2), A_BYTES,
+                          full0 + 8 * (int)j);
+            }
+            pdl_wait();
+            long long i = 0;
+            for (long long u = u0; u < u1; ++u, ++i) {
+                const int t = (int)(u / KB), kb = (int)(u - (long long)t * KB);
+                int seg, row0, n0;
+                tile_geom(t, seg, row0, n0);
+                const int s = (int)(i % stages);
+                if (i >= n_pre) {
+                    const uint32_t ph = (uint32_t)(i / stages) & 1u;
+                    if (!mbar_wait(empty0 + 8 * s, ph ^ 1u, &abort_flag, p.status)) break;
+                    mbar_expect_tx(full0 + 8 * s, A_BYTES + b_bytes);
+                    const long long blk = (long long)(t / p.n_tiles_n) * KB + kb;
+                    bulk_load(a_base + s * A_BYTES, p.wpacked + blk * (A_BYTES / 2), A_BYTES,
+                              full0 + 8 * s);
+                }
+                tma_load_2d(b_base + s * b_bytes, &mx, kb * BK, n0, full0 + 8 * s);
+            }
+            if (abort_flag) {
+                volatile int never = 0;
+                const long long issued = i;
+                for (long long j = (issued > stages ? issued - stages : 0); j < issued; ++j)
+                    mbar_wait(full0 + 8 * (int)(j % stages), (uint32_t)(j / stages) & 1u, &never,
+                              p.status);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        pdl_wait();
+        if (lane == 0) {
+            const uint32_t idesc = instr_desc(BN);
+            long long i = 0;
+            int item = 0;
+            for (long long u = u0; u < u1 && !abort_flag; ++item) {
+                const int t = (int)(u / KB), kb_b = (int)(u - (long long)t * KB);
+                const int kb_e = (int)min((long long)KB, kb_b + (u1 - u));
+                const int a = item & 1;
+                if (!mbar_wait(acce0 + 8 * a, (uint32_t)((item >> 1) & 1) ^ 1u, &abort_flag,
+                               p.status))
+                    break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t acc = tmem + a * p.acc_stride;
+                for (int kb = kb_b; kb < kb_e; ++kb, ++i) {
+                    const int s = (int)(i % stages);
+                    const uint32_t ph = (uint32_t)(i / stages) & 1u;
+                    if (!mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status)) break;
+                    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                    const uint64_t ad = smem_desc(a_base + s * A_BYTES);
+                    const uint64_t bd = smem_desc(b_base + s * b_bytes);
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk)
+                        mma_bf16(acc, ad + 2 * kk, bd + 2 * kk, idesc, (kb != kb_b) || (kk != 0));
+                    mma_commit(empty0 + 8 * s);
+                }
+                mma_commit(accf0 + 8 * a);
+                u += kb_e - kb_b;
+            }
+        }
+        __syncwarp();
+    } else {
+        // epilogue warps: TMEM lane quarter (warp % 4)
+        pdl_wait();
+        const int q = warp & 3;
+        const int row = q * 32 + lane;
+        const int et = threadIdx.x - 64;     // 0..127
+        int item = 0;
+        for (long long u = u0; u < u1; ++item) {
+            const int t = (int)(u / KB), kb_b = (int)(u - (long long)t * KB);
+            const int kb_e = (int)min((long long)KB, kb_b + (u1 - u));
+            u += kb_e - kb_b;
+            const int a = item & 1;
+            const bool ok = mbar_wait(accf0 + 8 * a, (uint32_t)(item >> 1) & 1u, &abort_flag,
+                                      p.status) && !abort_flag;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            int seg, row0, n0;
+            tile_geom(t, seg, row0, n0);
+            const int o_local = row0 + row;
+            const bool row_ok = ok && o_local < p.seg_rows[seg];
+            const int o = p.seg_out[seg] + o_local;
+            const bool whole = kb_b == 0 && kb_e == KB;
+            const uint32_t taddr = tmem + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
+            const int slot = 2 * cta + (item == 0 ? 0 : 1);
+            float *part = p.ws + (size_t)slot * BN * BM;
+            for (int c0 = 0; c0 < BN; c0 += 16) {
+                uint32_t r[16];
+                tmem_ld16(taddr + c0, r);
+                if (whole) {
+                    if (row_ok) {
+#pragma unroll
+                        for (int j = 0; j < 16; ++j) {
+                            const int m = n0 + c0 + j;
+                            if (m < p.M) {
+                                float *y = p.Y + (size_t)m * p.ldy + o;
+                                const float v = __uint_as_float(r[j]);
+                                *y = p.epi == EPI_ADD ? *y + v : v;
+                            }
+                        }
+                    }
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 16; ++j)
+                        part[(size_t)(c0 + j) * BM + row] = __uint_as_float(r[j]);
+                }
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(acce0 + 8 * a) : "memory");
+            if (whole) continue;
+            // ticket for the cut tile; the last piece reduces all pieces in CTA order
+            __threadfence();
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            const int c_first = owner_cta((long long)t * KB, U, p.grid);
+            const int c_last = owner_cta((long long)(t + 1) * KB - 1, U, p.grid);
+            const int np = c_last - c_first + 1;
+            if (et == 0) {
+                const int prev = atomicAdd(&p.counters[t], 1);
+                s_reduce = prev == np - 1;
+            }
+            if (et < np && et < P_MAX_PIECES) {
+                const int cc = c_first + et;
+                const long long cu0 = (long long)cc * U / p.grid;
+                s_slot[et] = 2 * cc + (cu0 >= (long long)t * KB ? 0 : 1);
+            }
+            asm volatile("bar.sync 1, 128;" ::: "memory");
+            if (!s_reduce) continue;
+            if (np > P_MAX_PIECES) {
+                set_status(p.status, ST_RANGE);
+                continue;
+            }
+            __threadfence();
+            // flat float4 view of the [BN][128] pieces; 4 float4 per thread in flight per piece
+            const int n4 = BN * BM / 4;
+            const size_t piece4 = (size_t)BN * BM / 4;
+            const float4 *ws4 = reinterpret_cast<const float4 *>(p.ws);
+            for (int base4 = et; base4 < n4; base4 += 4 * 128) {
+                float4 acc[4];
+#pragma unroll
+                for (int g = 0; g < 4; ++g) acc[g] = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int i = 0; i < np; ++i) {
+                    const float4 *src = ws4 + (size_t)s_slot[i] * piece4;
+                    float4 v[4];
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        const int e4 = base4 + g * 128;
+                        v[g] = e4 < n4 ? __ldcg(src + e4) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    }
+#pragma unroll
+                    for (int g = 0; g < 4; ++g) {
+                        acc[g].x += v[g].x; acc[g].y += v[g].y;
+                        acc[g].z += v[g].z; acc[g].w += v[g].w;
+                    }
+                }
+#pragma unroll
+                for (int g = 0; g < 4; ++g) {
+                    const int e4 = base4 + g * 128;
+                    if (e4 >= n4) continue;
+                    const int col = (e4 * 4) / BM, r4 = (e4 * 4) - col * BM;
+                    const int m = n0 + col;
+                    if (m >= p.M || !ok) continue;
+                    const float vv[4] = {acc[g].x, acc[g].y, acc[g].z, acc[g].w};
+#pragma unroll
+                    for (int e = 0; e < 4; ++e) {
+                        const int ol = row0 + r4 + e;
+                        if (ol < p.seg_rows[seg]) {
+                            float *y = p.Y + (size_t)m * p.ldy + p.seg_out[seg] + ol;
+                            *y = p.epi == EPI_ADD ? *y + vv[e] : vv[e];
+                        }
+                    }
+                }
+            }
+            if (et == 0) p.counters[t] = 0;
+        }
+    }
+
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(p.tmem_cols)
+                     : "memory");
+    }
+}
+
+// One 16 KB packed block per CTA: rows row0..row0+127 of the block's segment,
+// columns kb*64 .. kb*64+63, written in the swizzled shared-memory order.
+__global__ void pack_kernel(GemmW W, int K, int KB, uint8_t *dst) {
+    const long long blk = blockIdx.x;
+    const int wt = (int)(blk / KB), kb = (int)(blk - (long long)wt * KB);
+    int seg = 0, w = wt;
+    while (seg < W.nseg - 1 && w >= (W.rows[seg] + BM - 1) / BM) {
+        w -= (W.rows[seg] + BM - 1) / BM;
+        ++seg;
+    }
+    const bf16 *src = static_cast<const bf16 *>(W.w[seg]);
+    const int rows = W.rows[seg], row0 = w * BM;
+    uint8_t *out = dst + blk * (long long)A_BYTES;
+    for (int q = threadIdx.x; q < BM * 8; q += blockDim.x) {
+        const int r = q >> 3, c = q & 7;
+        const int row = row0 + r, k = kb * BK + c * 8;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (row < rows && k + 8 <= K) v = *reinterpret_cast<const uint4 *>(src + (size_t)row * K + k);
+        *reinterpret_cast<uint4 *>(out + r * 128 + ((c ^ (r & 7)) << 4)) = v;
+    }
+}
+
+// Records a host-detected problem in the device status word, in stream order.
+__global__ void flag_kernel(int *status, int code) { set_status(status, code); }
+
 struct MapKey {
     const void *ptr;
     long rows, cols, ld, box_rows;
@@ -424,74 +755,85 @@ static const CUtensorMap *get_map(GemmPlan *p, const void *ptr, long rows, long 
     return &p->maps.emplace(key, m).first->second;
 }
 
+size_t gemm_pack_bytes(const GemmW &W, int K) {
+    long long tiles = 0;
+    for (int i = 0; i < W.nseg; ++i) tiles += (W.rows[i] + BM - 1) / BM;
+    return (size_t)tiles * ((K + BK - 1) / BK) * A_BYTES;
+}
+
+void gemm_pack(const GemmW &W, int K, void *dst, cudaStream_t s) {
+    const long long blocks = (long long)(gemm_pack_bytes(W, K) / A_BYTES);
+    if (blocks <= 0) return;
+    pack_kernel<<<(unsigned)blocks, 256, 0, s>>>(W, K, (K + BK - 1) / BK, static_cast<uint8_t *>(dst));
+    note_launch();
+}
+
 void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
                int ldy, int epi, int *status, cudaStream_t s) {
     if (M <= 0 || O <= 0) return;
-    TcParams tp;
-    memset(&tp, 0, sizeof tp);
-    tp.n_seg = W.nseg;
+    PkParams pk;
+    memset(&pk, 0, sizeof pk);
+    pk.n_seg = W.nseg;
     int tiles = 0, out_off = 0;
     for (int i = 0; i < W.nseg; ++i) {
-        tp.seg_rows[i] = W.rows[i];
-        tp.seg_tiles[i] = (W.rows[i] + BM - 1) / BM;
-        tp.seg_out[i] = out_off;
+        pk.seg_rows[i] = W.rows[i];
+        pk.seg_tiles[i] = (W.rows[i] + BM - 1) / BM;
+        pk.seg_out[i] = out_off;
         out_off += W.rows[i];
-        tiles += tp.seg_tiles[i];
+        tiles += pk.seg_tiles[i];
     }
     const int nt = (M + 255) / 256;
     int BN = (M + nt - 1) / nt;
     BN = ((BN + 15) / 16) * 16;
     const int kblocks = (K + BK - 1) / BK;
     const uint32_t stage_bytes = A_BYTES + (uint32_t)BN * BK * 2;
-    int ctas_per_sm = BN <= 128 ? 2 : 1;
-    int stages = (int)((ctas_per_sm == 2 ? 100u * 1024u : 200u * 1024u) / stage_bytes);
-    stages = stages < 2 ? 2 : (stages > MAX_STAGES ? MAX_STAGES : stages);
+    int stages = (int)((200u * 1024u) / stage_bytes);
+    stages = stages < 2 ? 2 : (stages > P_MAX_STAGES ? P_MAX_STAGES : stages);
     const size_t smem = 1024 + (size_t)stages * stage_bytes;
-
-    // split-K: fewest waves x k-blocks per CTA, plus a small reduction cost
-    const long base = (long)tiles * nt;
-    const long slots = (long)p->num_sms * ctas_per_sm;
-    const size_t tile_bytes = (size_t)BN * BM * sizeof(float);
-    int best_s = 1;
-    double best = 1e30;
-    for (int sp = 1; sp <= 16 && sp <= kblocks; ++sp) {
-        const int kps = (kblocks + sp - 1) / sp;
-        const int se = (kblocks + kps - 1) / kps;
-        if (se > 1 && ((size_t)base * se * tile_bytes > WS_BYTES || base > N_COUNTERS)) continue;
-        const long waves = (base * se + slots - 1) / slots;
-        const double cost = (double)waves * kps + (se > 1 ? 2.0 : 0.0);
-        if (cost < best - 1e-9) { best = cost; best_s = se; }
+    const long long tiles_total = (long long)tiles * nt;
+    const long long units = tiles_total * kblocks;
+    // one CTA per SM, at least 4 K-blocks each
+    long long G = units / 4;
+    if (G > p->num_sms) G = p->num_sms;
+    if (G < 1) G = 1;
+    const size_t ws_need = 2ull * G * BN * BM * sizeof(float);
+    if (ws_need > WS_BYTES || tiles_total > N_COUNTERS) {
+        flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
+        fprintf(stderr, "msd: GEMM shape M=%d K=%d O=%d exceeds the workspace\n", M, K, O);
+        return;
     }
-    const int kps = (kblocks + best_s - 1) / best_s;
-    tp.splits = (kblocks + kps - 1) / kps;
-    tp.kb_per_split = kps;
-    tp.M = M;
-    tp.kblocks = kblocks;
-    tp.BN = BN;
-    tp.n_tiles_n = nt;
-    tp.stages = stages;
-    tp.tmem_cols = BN <= 32 ? 32 : (BN <= 64 ? 64 : (BN <= 128 ? 128 : 256));
-    tp.Y = Y;
-    tp.ldy = ldy;
-    tp.epi = epi;
-    tp.ws = p->ws;
-    tp.counters = p->counters;
-    tp.status = status;
-
-    const CUtensorMap *mw[3] = {nullptr, nullptr, nullptr};
-    for (int i = 0; i < W.nseg; ++i) {
-        mw[i] = get_map(p, W.w[i], W.rows[i], K, K, BM, status);
-        if (!mw[i]) return;
+    int acc = 32;
+    while (acc < BN) acc <<= 1;
+    pk.M = M;
+    pk.kblocks = kblocks;
+    pk.BN = BN;
+    pk.n_tiles_n = nt;
+    pk.stages = stages;
+    pk.acc_stride = acc;
+    pk.tmem_cols = 2 * acc;
+    pk.grid = (int)G;
+    pk.units = units;
+    pk.Y = Y;
+    pk.ldy = ldy;
+    pk.epi = epi;
+    pk.ws = p->ws;
+    pk.counters = p->counters;
+    pk.status = status;
+    pk.wpacked = static_cast<const bf16 *>(W.packed);
+    if (!W.packed) {
+        flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
+        fprintf(stderr, "msd: GEMM weights were not packed\n");
+        return;
     }
-    for (int i = W.nseg; i < 3; ++i) mw[i] = mw[0];
     const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
     if (!mx) return;
     if (!p->smem_set) {
         cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              200 * 1024 + 1024);
+        cudaFuncSetAttribute(gemm_persist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             200 * 1024 + 1024);
         p->smem_set = true;
     }
-    dim3 grid(tiles, nt, tp.splits);
     const bool prof = p->profile;
     if (prof) {
         while (p->ev.size() < p->ev_used + 2) {
@@ -501,7 +843,21 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
         }
         cudaEventRecord(p->ev[p->ev_used], s);
     }
-    gemm_tc_kernel<<<grid, THREADS, smem, s>>>(*mw[0], *mw[1], *mw[2], *mx, tp);
+    // Programmatic dependent launch: the kernel may start while the previous
+    // kernel on the stream finishes; it waits (griddepcontrol.wait) before
+    // touching anything but weights.
+    cudaLaunchConfig_t lc;
+    memset(&lc, 0, sizeof lc);
+    lc.gridDim = dim3((unsigned)G);
+    lc.blockDim = dim3(P_THREADS);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = at;
+    lc.numAttrs = 1;
+    cudaLaunchKernelEx(&lc, gemm_persist_kernel, *mx, pk);
     note_launch();
     if (prof) {
         cudaEventRecord(p->ev[p->ev_used + 1], s);

@@ -16,6 +16,13 @@ void gemm_plan_destroy(GemmPlan *p);
 void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
                int ldy, int epi, int *status, cudaStream_t s);
 
+// Pre-packed weights: the segments' 128-row x 64-column blocks, tile-major then
+// K-block, each block stored exactly as the MMA reads it from shared memory
+// (K-major rows of 128 bytes, 128-byte swizzle), so one contiguous 16 KB copy
+// fills a pipeline stage. Rows past a segment's end and columns past K are 0.
+size_t gemm_pack_bytes(const GemmW &W, int K);
+void gemm_pack(const GemmW &W, int K, void *dst, cudaStream_t s);
+
 // Profiling: while enabled, every launch is bracketed by CUDA events on its
 // stream; gemm_profile_read synchronises on them and returns the launches,
 // their summed durations and their algorithmic bytes (weights + X + Y),

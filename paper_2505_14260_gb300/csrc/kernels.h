@@ -54,12 +54,22 @@ struct AttnArgs {
 template <typename T>
 void launch_attention(const AttnArgs<T> &a, cudaStream_t s);
 
-// out[r] = argmax_j logits[r][j] (ties: lower j)
-void launch_argmax(const float *logits, int R, int V, int *out, cudaStream_t s);
+// Scratch of the chunked top-k: per-chunk records and per-row tickets
+// (tickets must start at zero; the kernel leaves them at zero).
+struct TopkScratch {
+    float *ws;
+    int *counters;
+};
+size_t topk_scratch_floats(int max_rows, int V);
 
-// Top-k of each row (ties: lower id) and their log-softmax values.
-void launch_topk_logp(const float *logits, int R, int V, int k, int *ids,
-                      float *logp, cudaStream_t s);
+// out[r] = argmax_j logits[r][j] (ties: lower j)
+void launch_argmax(const float *logits, int R, int V, int *out, const TopkScratch &sc,
+                   cudaStream_t s);
+
+// Top-k of each row (ties: lower id) and their log-softmax values (logp
+// nullable). k <= 16.
+void launch_topk_logp(const float *logits, int R, int V, int k, int *ids, float *logp,
+                      const TopkScratch &sc, cudaStream_t s);
 
 template <typename T>
 void launch_convert(const float *x, T *y, long n, cudaStream_t s);
@@ -72,6 +82,7 @@ struct GemmW {
     const void *w[3];
     int rows[3];
     int nseg;
+    const void *packed;   // the same weights pre-packed by gemm_pack (bf16), or null
 };
 enum { EPI_STORE = 0, EPI_ADD = 1 };
 

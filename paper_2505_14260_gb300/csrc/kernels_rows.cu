@@ -2,6 +2,7 @@
 // SwiGLU, RoPE + K/V placement, argmax and top-k with log-softmax.
 #include "kernels.h"
 
+#include <algorithm>
 #include <atomic>
 
 namespace msd {
@@ -17,6 +18,7 @@ template <typename T>
 __global__ void embed_rows_kernel(const T *__restrict__ E, const T *__restrict__ vis,
                                   const int *__restrict__ src, int H, float *__restrict__ x,
                                   T *__restrict__ emb_out, int V, int *status) {
+    allow_dependents();
     const int r = blockIdx.x;
     int s = src[r];
     const T *row;
@@ -46,28 +48,66 @@ void launch_embed_rows(const T *E, const T *vis, const int *src, int R, int H, f
 // ---------------------------------------------------------------------------
 // RMSNorm: y = x / sqrt(mean(x^2) + eps) * g
 // ---------------------------------------------------------------------------
+template <typename T> struct Vec4;
+template <> struct Vec4<float> {
+    static __device__ __forceinline__ float4 load(const float *g) { return *reinterpret_cast<const float4 *>(g); }
+    static __device__ __forceinline__ void store(float *o, float4 v) { *reinterpret_cast<float4 *>(o) = v; }
+};
+template <> struct Vec4<bf16> {
+    static __device__ __forceinline__ float4 load(const bf16 *g) {
+        const uint2 u = *reinterpret_cast<const uint2 *>(g);
+        const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162 *>(&u.x);
+        const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&u.y);
+        return make_float4(__low2float(a), __high2float(a), __low2float(b), __high2float(b));
+    }
+    static __device__ __forceinline__ void store(bf16 *o, float4 v) {
+        __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+        uint2 u;
+        u.x = *reinterpret_cast<uint32_t *>(&a);
+        u.y = *reinterpret_cast<uint32_t *>(&b);
+        *reinterpret_cast<uint2 *>(o) = u;
+    }
+};
+
+// One CTA per row; the row stays in registers (H <= 8 * 4 * 256).
+constexpr int RMS_THREADS = 256;
+constexpr int RMS_VEC = 8;
+
 template <typename T>
-__global__ void rmsnorm_kernel(const float *__restrict__ x, const T *__restrict__ g, int H,
-                               float eps, T *__restrict__ out) {
+__global__ void __launch_bounds__(RMS_THREADS) rmsnorm_kernel(const float *__restrict__ x,
+                                                              const T *__restrict__ g, int H,
+                                                              float eps, T *__restrict__ out) {
+    allow_dependents();
     __shared__ float red[32];
-    const int r = blockIdx.x;
-    const float *xr = x + (size_t)r * H;
+    const int r = blockIdx.x, n4 = H >> 2;
+    const float4 *xr = reinterpret_cast<const float4 *>(x + (size_t)r * H);
+    float4 v[RMS_VEC];
     float ss = 0.f;
-    for (int j = threadIdx.x; j < H; j += blockDim.x) {
-        float v = xr[j];
-        ss += v * v;
+#pragma unroll
+    for (int i = 0; i < RMS_VEC; ++i) {
+        const int j = threadIdx.x + i * RMS_THREADS;
+        v[i] = j < n4 ? xr[j] : make_float4(0.f, 0.f, 0.f, 0.f);
+        ss += v[i].x * v[i].x + v[i].y * v[i].y + v[i].z * v[i].z + v[i].w * v[i].w;
     }
     ss = block_sum(ss, red);
     const float inv = rsqrtf(ss / (float)H + eps);
-    for (int j = threadIdx.x; j < H; j += blockDim.x)
-        out[(size_t)r * H + j] = from_f<T>(xr[j] * inv * to_f(g[j]));
+#pragma unroll
+    for (int i = 0; i < RMS_VEC; ++i) {
+        const int j = threadIdx.x + i * RMS_THREADS;
+        if (j < n4) {
+            const float4 gg = Vec4<T>::load(g + 4 * j);
+            Vec4<T>::store(out + (size_t)r * H + 4 * j,
+                           make_float4(v[i].x * inv * gg.x, v[i].y * inv * gg.y,
+                                       v[i].z * inv * gg.z, v[i].w * inv * gg.w));
+        }
+    }
 }
 
 template <typename T>
 void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
                     cudaStream_t s) {
     if (R <= 0) return;
-    rmsnorm_kernel<T><<<R, 256, 0, s>>>(x, g, H, eps, out); note_launch();
+    rmsnorm_kernel<T><<<R, RMS_THREADS, 0, s>>>(x, g, H, eps, out); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -75,6 +115,7 @@ void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
 // ---------------------------------------------------------------------------
 template <typename T>
 __global__ void swiglu_kernel(const float *__restrict__ gu, int F, T *__restrict__ act) {
+    allow_dependents();
     const int r = blockIdx.y;
     const float *row = gu + (size_t)r * 2 * F;
     for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < F; j += gridDim.x * blockDim.x) {
@@ -99,6 +140,7 @@ __global__ void rope_kv_kernel(const float *__restrict__ qkv, const RowDesc *__r
                                int nh, int hd, const float2 *__restrict__ tab, int max_pos,
                                T *__restrict__ q_out, T *__restrict__ kdst, T *__restrict__ vdst,
                                int slots, int *status) {
+    allow_dependents();
     const int r = blockIdx.x;
     const int H = nh * hd, half = hd >> 1;
     const RowDesc d = rows[r];
@@ -141,118 +183,152 @@ void launch_rope_kv(const float *qkv, const RowDesc *rows, int R, int nh, int hd
 }
 
 // ---------------------------------------------------------------------------
-// Argmax per row (ties: lower index)
+// Top-k per row with log-softmax values (argmax = top-1). The row is cut into
+// chunks, one CTA each: the CTA holds its chunk in shared memory, computes the
+// chunk max, the chunk sum of exp(z - max) and the chunk's top-k (k rounds of
+// a block-wide best-of with removal); the last CTA of the row (ticket) merges
+// the chunk results: lse = M + log(sum_c s_c exp(m_c - M)) and the top-k of the
+// chunk candidates. Order: larger value, then lower index.
 // ---------------------------------------------------------------------------
-__global__ void argmax_kernel(const float *__restrict__ logits, int V, int *__restrict__ out) {
-    __shared__ float sv[32];
-    __shared__ int si[32];
-    const int r = blockIdx.x;
-    const float *z = logits + (size_t)r * V;
-    float bv = -INFINITY;
-    int bi = 0x7fffffff;
-    for (int j = threadIdx.x; j < V; j += blockDim.x) {
-        float v = z[j];
-        if (better(v, j, bv, bi)) { bv = v; bi = j; }
-    }
+constexpr int TOPK_MAX = 16;
+constexpr int TK_THREADS = 256;
+constexpr int TK_REC = 2 + 2 * TOPK_MAX;     // floats per chunk record
+
+__device__ __forceinline__ void block_best(float &v, int &i, float *rv, int *ri) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
-        float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-        int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-        if (better(ov, oi, bv, bi)) { bv = ov; bi = oi; }
+        const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+        const int oi = __shfl_xor_sync(0xffffffffu, i, o);
+        if (better(ov, oi, v, i)) { v = ov; i = oi; }
     }
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    if (lane == 0) { sv[warp] = bv; si[warp] = bi; }
+    __syncthreads();
+    if (lane == 0) { rv[warp] = v; ri[warp] = i; }
     __syncthreads();
     if (warp == 0) {
         const int nw = blockDim.x >> 5;
-        bv = lane < nw ? sv[lane] : -INFINITY;
-        bi = lane < nw ? si[lane] : 0x7fffffff;
+        v = lane < nw ? rv[lane] : -INFINITY;
+        i = lane < nw ? ri[lane] : 0x7fffffff;
 #pragma unroll
         for (int o = 16; o > 0; o >>= 1) {
-            float ov = __shfl_xor_sync(0xffffffffu, bv, o);
-            int oi = __shfl_xor_sync(0xffffffffu, bi, o);
-            if (better(ov, oi, bv, bi)) { bv = ov; bi = oi; }
+            const float ov = __shfl_xor_sync(0xffffffffu, v, o);
+            const int oi = __shfl_xor_sync(0xffffffffu, i, o);
+            if (better(ov, oi, v, i)) { v = ov; i = oi; }
         }
-        if (lane == 0) out[r] = bi == 0x7fffffff ? 0 : bi;
+        if (lane == 0) { rv[0] = v; ri[0] = i; }
     }
+    __syncthreads();
+    v = rv[0];
+    i = ri[0];
 }
 
-void launch_argmax(const float *logits, int R, int V, int *out, cudaStream_t s) {
-    if (R <= 0) return;
-    argmax_kernel<<<R, 512, 0, s>>>(logits, V, out); note_launch();
-}
-
-// ---------------------------------------------------------------------------
-// Top-k + log-softmax per row. Each thread keeps a sorted local top-k of its
-// strided elements; k block-wide selection rounds merge them.
-// ---------------------------------------------------------------------------
-constexpr int TOPK_MAX = 16;
-constexpr int TOPK_THREADS = 256;
-
-__global__ void topk_logp_kernel(const float *__restrict__ logits, int V, int k,
-                                 int *__restrict__ ids, float *__restrict__ logp) {
-    __shared__ float red[32];
-    __shared__ float cand_v[TOPK_THREADS];
-    __shared__ int cand_i[TOPK_THREADS];
+__global__ void __launch_bounds__(TK_THREADS)
+    topk_rows_kernel(const float *__restrict__ logits, int V, int k, int *__restrict__ ids,
+                     float *__restrict__ logp, float *__restrict__ ws, int *__restrict__ counters) {
+    allow_dependents();
+    extern __shared__ float sv[];
+    __shared__ float rv[32];
+    __shared__ int ri[32];
     __shared__ float sel_v[TOPK_MAX];
     __shared__ int sel_i[TOPK_MAX];
-    const int r = blockIdx.x;
-    const float *z = logits + (size_t)r * V;
-
-    float lv[TOPK_MAX];
-    int li[TOPK_MAX];
-#pragma unroll
-    for (int t = 0; t < TOPK_MAX; ++t) { lv[t] = -INFINITY; li[t] = 0x7fffffff; }
+    __shared__ int s_last;
+    const int r = blockIdx.y, c = blockIdx.x, nc = gridDim.x;
+    const int CH = (V + nc - 1) / nc;
+    const int lo = c * CH, n = max(0, min(V, lo + CH) - lo);
+    const float *z = logits + (size_t)r * V + lo;
     float mx = -INFINITY;
-    for (int j = threadIdx.x; j < V; j += blockDim.x) {
+    for (int j = threadIdx.x; j < n; j += TK_THREADS) {
         const float v = z[j];
+        sv[j] = v;
         mx = fmaxf(mx, v);
-        if (better(v, j, lv[k - 1], li[k - 1])) {
-            // insert keeping lv sorted (best first); k is small
-            int p = k - 1;
-            while (p > 0 && better(v, j, lv[p - 1], li[p - 1])) {
-                lv[p] = lv[p - 1]; li[p] = li[p - 1];
-                --p;
-            }
-            lv[p] = v; li[p] = j;
-        }
     }
-    mx = block_max(mx, red);
+    mx = block_max(mx, rv);
     float se = 0.f;
-    for (int j = threadIdx.x; j < V; j += blockDim.x) se += __expf(z[j] - mx);
-    se = block_sum(se, red);
-    const float lse = mx + logf(se);
-
-    int head = 0;
-    for (int round = 0; round < k; ++round) {
-        cand_v[threadIdx.x] = head < k ? lv[head] : -INFINITY;
-        cand_i[threadIdx.x] = head < k ? li[head] : 0x7fffffff;
-        __syncthreads();
-        for (int stride = blockDim.x >> 1; stride > 0; stride >>= 1) {
-            if (threadIdx.x < stride) {
-                const float ov = cand_v[threadIdx.x + stride];
-                const int oi = cand_i[threadIdx.x + stride];
-                if (better(ov, oi, cand_v[threadIdx.x], cand_i[threadIdx.x])) {
-                    cand_v[threadIdx.x] = ov; cand_i[threadIdx.x] = oi;
-                }
-            }
-            __syncthreads();
-        }
-        const int win = cand_i[0];
-        if (threadIdx.x == 0) { sel_v[round] = cand_v[0]; sel_i[round] = win; }
-        if (head < k && li[head] == win) ++head;   // indices are unique per row
+    for (int j = threadIdx.x; j < n; j += TK_THREADS) se += __expf(sv[j] - mx);
+    se = block_sum(se, rv);
+    for (int t = 0; t < k; ++t) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff;
+        for (int j = threadIdx.x; j < n; j += TK_THREADS)
+            if (better(sv[j], lo + j, bv, bi)) { bv = sv[j]; bi = lo + j; }
+        block_best(bv, bi, rv, ri);
+        if (threadIdx.x == 0) { sel_v[t] = bv; sel_i[t] = bi; }
+        if (bi != 0x7fffffff && bi - lo >= 0 && bi - lo < n && ((bi - lo) % TK_THREADS) == threadIdx.x)
+            sv[bi - lo] = -INFINITY;
         __syncthreads();
     }
+    float *rec = ws + ((size_t)r * nc + c) * TK_REC;
+    if (threadIdx.x == 0) { rec[0] = mx; rec[1] = se; }
     if (threadIdx.x < k) {
-        ids[(size_t)r * k + threadIdx.x] = sel_i[threadIdx.x];
-        logp[(size_t)r * k + threadIdx.x] = sel_v[threadIdx.x] - lse;
+        rec[2 + threadIdx.x] = sel_v[threadIdx.x];
+        rec[2 + TOPK_MAX + threadIdx.x] = __int_as_float(sel_i[threadIdx.x]);
     }
+    __threadfence();
+    __syncthreads();
+    if (threadIdx.x == 0) s_last = atomicAdd(&counters[r], 1) == nc - 1;
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    // merge the chunk records of row r
+    const float *rrow = ws + (size_t)r * nc * TK_REC;
+    float M = -INFINITY;
+    for (int q = threadIdx.x; q < nc; q += TK_THREADS) M = fmaxf(M, __ldcg(rrow + q * TK_REC));
+    M = block_max(M, rv);
+    float S = 0.f;
+    for (int q = threadIdx.x; q < nc; q += TK_THREADS)
+        S += __ldcg(rrow + q * TK_REC + 1) * __expf(__ldcg(rrow + q * TK_REC) - M);
+    S = block_sum(S, rv);
+    const float lse = M + logf(S);
+    float *cv = sv;                                   // candidates: nc * k
+    int *ci = reinterpret_cast<int *>(sv + nc * k);
+    for (int q = threadIdx.x; q < nc * k; q += TK_THREADS) {
+        const int cc = q / k, t = q - cc * k;
+        cv[q] = __ldcg(rrow + cc * TK_REC + 2 + t);
+        ci[q] = __float_as_int(__ldcg(rrow + cc * TK_REC + 2 + TOPK_MAX + t));
+    }
+    __syncthreads();
+    for (int t = 0; t < k; ++t) {
+        float bv = -INFINITY;
+        int bi = 0x7fffffff, bq = -1;
+        for (int q = threadIdx.x; q < nc * k; q += TK_THREADS)
+            if (better(cv[q], ci[q], bv, bi)) { bv = cv[q]; bi = ci[q]; bq = q; }
+        float wv = bv;
+        int wi = bi;
+        block_best(wv, wi, rv, ri);
+        if (bq >= 0 && bi == wi) cv[bq] = -INFINITY;   // ids are unique within a row
+        if (threadIdx.x == 0) {
+            ids[(size_t)r * k + t] = wi == 0x7fffffff ? 0 : wi;
+            if (logp) logp[(size_t)r * k + t] = wv - lse;
+        }
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) counters[r] = 0;
+}
+
+static int topk_chunks(int V) {
+    int nc = 16;
+    while ((V + nc - 1) / nc > 4096) nc *= 2;
+    return nc;
+}
+
+size_t topk_scratch_floats(int max_rows, int V) {
+    return (size_t)max_rows * topk_chunks(V) * TK_REC;
 }
 
 void launch_topk_logp(const float *logits, int R, int V, int k, int *ids, float *logp,
-                      cudaStream_t s) {
+                      const TopkScratch &sc, cudaStream_t s) {
     if (R <= 0) return;
-    topk_logp_kernel<<<R, TOPK_THREADS, 0, s>>>(logits, V, k, ids, logp); note_launch();
+    const int nc = topk_chunks(V);
+    const int CH = (V + nc - 1) / nc;
+    const size_t smem = sizeof(float) * std::max<size_t>(CH, (size_t)2 * nc * k);
+    topk_rows_kernel<<<dim3(nc, R), TK_THREADS, smem, s>>>(logits, V, k, ids, logp, sc.ws,
+                                                          sc.counters);
+    note_launch();
+}
+
+void launch_argmax(const float *logits, int R, int V, int *out, const TopkScratch &sc,
+                   cudaStream_t s) {
+    launch_topk_logp(logits, R, V, 1, out, nullptr, sc, s);
 }
 
 // ---------------------------------------------------------------------------

@@ -16,6 +16,7 @@ __global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int 
                                      const T *__restrict__ pend_h, const int *__restrict__ pend_next,
                                      const T *__restrict__ E, int H, int D1, int V,
                                      T *__restrict__ xfc, RowDesc *__restrict__ rows, int *status) {
+    allow_dependents();
     const int r = blockIdx.x, b = r / D1, j = r - b * D1;
     const int L = seq_len[b], P = n_pend[b];
     const bool valid = j < P;
@@ -46,6 +47,7 @@ __global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int 
 template <typename T>
 __global__ void root_gather_kernel(const float *__restrict__ x, const int *__restrict__ n_pend, int D1,
                                    int H, float *__restrict__ hhat_root, T *__restrict__ xr) {
+    allow_dependents();
     const int b = blockIdx.x;
     const int r = b * D1 + max(n_pend[b] - 1, 0);
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
@@ -59,6 +61,7 @@ __global__ void root_gather_kernel(const float *__restrict__ x, const int *__res
 template <typename T>
 __global__ void hhat_store_kernel(const float *__restrict__ x, const RowDesc *__restrict__ rows,
                                   int Td, int H, float *__restrict__ hhat_slot, T *__restrict__ xb) {
+    allow_dependents();
     const int r = blockIdx.x;
     const RowDesc d = rows[r];
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
@@ -68,10 +71,11 @@ __global__ void hhat_store_kernel(const float *__restrict__ x, const RowDesc *__
     }
 }
 
-// Assemble the draft-pass row of frontier candidate c at row j, slot `slot`:
-// input Concat(h_hat of its parent, e of its token), position L-1+depth.
+// Assemble the draft-pass row j of request b for a frontier node with token
+// `tok` at `depth`: input Concat(h_hat of its parent, e of its token), draft
+// position L-1+depth, K/V slot `slot`, ancestor mask = parent's mask + own bit.
 template <typename T>
-__device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int c, int depth,
+__device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int tok, int depth,
                                   const float *parent_h, int slot, const uint64_t *parent_mask) {
     const int H = a.H, k = a.k, Wd = a.Wd;
     const int L = a.seq_len[b];
@@ -90,7 +94,6 @@ __device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int c, in
             a.row_mask[(size_t)r * Wd + w] = m;
         }
     }
-    int tok = a.cand_tok[(size_t)b * a.C + c];
     if (tok < 0 || tok >= a.V) tok = 0;
     T *dst = a.xfc + (size_t)r * 2 * H;
     const T *e = a.E + (size_t)tok * H;
@@ -100,75 +103,87 @@ __device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int c, in
     }
 }
 
-// Depth-1 candidates from the root slot's top-k; frontier = all of them, best
-// first; emit the rows of pass 2.
+// Depth-1 candidates from the root slot's top-k; the frontier of pass 2 is all
+// of them, best first. Grid (k, B): CTA j emits row j of pass 2; CTA 0 writes
+// the candidate arrays and the frontier (buffer 0).
 template <typename T>
 __global__ void tree_init_kernel(DraftArgs<T> a) {
-    const int b = blockIdx.x, k = a.k;
+    allow_dependents();
+    const int b = blockIdx.y, j = blockIdx.x, k = a.k;
     __shared__ float sc[TREE_MAXK];
+    __shared__ int front[TREE_MAXK];
     for (int t = threadIdx.x; t < k; t += blockDim.x) {
-        const size_t c = (size_t)b * a.C + t;
-        a.cand_tok[c] = a.ids[(size_t)b * k + t];
-        a.cand_par[c] = -1;
-        a.cand_depth[c] = 1;
         const float s = a.logp[(size_t)b * k + t];
-        a.cand_score[c] = s;
         sc[t] = s;
+        if (j == 0) {
+            const size_t c = (size_t)b * a.C + t;
+            a.cand_tok[c] = a.ids[(size_t)b * k + t];
+            a.cand_par[c] = -1;
+            a.cand_depth[c] = 1;
+            a.cand_score[c] = s;
+        }
     }
     __syncthreads();
     for (int t = threadIdx.x; t < k; t += blockDim.x) {
         int rank = 0;
         for (int u = 0; u < k; ++u) rank += better(sc[u], u, sc[t], t);
-        a.frontier[(size_t)b * k + rank] = t;
+        front[rank] = t;
     }
     __syncthreads();
+    if (j == 0)
+        for (int t = threadIdx.x; t < k; t += blockDim.x) a.frontier[(size_t)b * k + t] = front[t];
     if (a.D < 2) return;
-    for (int j = 0; j < k; ++j) {
-        const int c = a.frontier[(size_t)b * k + j];
-        emit_frontier_row(a, b, j, c, 1, a.hhat_root + (size_t)b * a.H, j, nullptr);
-    }
+    const int c = front[j];
+    emit_frontier_row(a, b, j, a.ids[(size_t)b * k + c], 1, a.hhat_root + (size_t)b * a.H, j,
+                      nullptr);
 }
 
-// After pass d (2..D): add the k*k children of the pass rows, then (d < D) pick
-// the k best of them as the next frontier and emit the rows of pass d+1.
+// After pass d (2..D): the k*k children of the pass rows, then (d < D) the k
+// best of them form the next frontier. Grid (k, B): every CTA ranks the
+// children itself (k*k values); CTA 0 writes the candidate arrays and the next
+// frontier (buffer (d+1)&1; this pass read buffer d&1); CTA j emits row j of
+// pass d+1.
 template <typename T>
 __global__ void tree_step_kernel(DraftArgs<T> a, int d) {
+    allow_dependents();
     extern __shared__ float smem[];
-    const int b = blockIdx.x, k = a.k, kk = k * k;
+    const int b = blockIdx.y, j = blockIdx.x, k = a.k, kk = k * k;
     const int base = k + (d - 2) * kk;
-    float *sc = smem;                                 // [kk]
-    int *newf = reinterpret_cast<int *>(smem + kk);   // [k]
+    float *sc = smem;                                  // [kk]
+    int *newf = reinterpret_cast<int *>(smem + kk);    // [k]
+    const int *fin = a.frontier + ((size_t)(d & 1) * a.B + b) * k;
+    int *fout = a.frontier + ((size_t)((d + 1) & 1) * a.B + b) * k;
     for (int e = threadIdx.x; e < kk; e += blockDim.x) {
-        const int j = e / k, t = e - j * k;
-        const int p = a.frontier[(size_t)b * k + j];
-        const size_t c = (size_t)b * a.C + base + e;
-        const size_t src = ((size_t)b * k + j) * k + t;
-        a.cand_tok[c] = a.ids[src];
-        a.cand_par[c] = p;
-        a.cand_depth[c] = d;
+        const int jr = e / k, t = e - jr * k;
+        const int p = fin[jr];
+        const size_t src = ((size_t)b * k + jr) * k + t;
         const float s = __fadd_rn(a.cand_score[(size_t)b * a.C + p], a.logp[src]);
-        a.cand_score[c] = s;
         sc[e] = s;
+        if (j == 0) {
+            const size_t c = (size_t)b * a.C + base + e;
+            a.cand_tok[c] = a.ids[src];
+            a.cand_par[c] = p;
+            a.cand_depth[c] = d;
+            a.cand_score[c] = s;
+        }
     }
     __syncthreads();
     if (d >= a.D) return;
     for (int e = threadIdx.x; e < kk; e += blockDim.x) {
         int rank = 0;
         for (int u = 0; u < kk; ++u) rank += better(sc[u], u, sc[e], e);
-        if (rank < k) newf[rank] = base + e;
+        if (rank < k) newf[rank] = e;
     }
     __syncthreads();
-    for (int j = threadIdx.x; j < k; j += blockDim.x) a.frontier[(size_t)b * k + j] = newf[j];
-    __syncthreads();
-    for (int j = 0; j < k; ++j) {
-        const int c = newf[j];
-        const int jp = (c - base) / k;                   // parent's row in pass d
-        const int sp = (d - 2) * k + jp;                 // parent's slot
-        const int slot = (d - 1) * k + j;
-        emit_frontier_row(a, b, j, c, d, a.hhat_slot + ((size_t)b * a.Td + sp) * a.H, slot,
-                          a.slot_mask + ((size_t)b * a.Td + sp) * a.Wd);
-        __syncthreads();
-    }
+    if (j == 0)
+        for (int t = threadIdx.x; t < k; t += blockDim.x) fout[t] = base + newf[t];
+    const int e = newf[j];
+    const int jp = e / k;                              // parent's row in pass d
+    const int sp = (d - 2) * k + jp;                   // parent's slot
+    const int slot = (d - 1) * k + j;
+    emit_frontier_row(a, b, j, a.ids[((size_t)b * k + jp) * k + (e - jp * k)], d,
+                      a.hhat_slot + ((size_t)b * a.Td + sp) * a.H, slot,
+                      a.slot_mask + ((size_t)b * a.Td + sp) * a.Wd);
 }
 
 // Final tree: the N-1 best candidates (score desc, creation asc), tree index
@@ -177,6 +192,7 @@ __global__ void tree_finalize_kernel(TreeOut t, const int *__restrict__ cand_tok
                                      const int *__restrict__ cand_par, const int *__restrict__ cand_depth,
                                      const float *__restrict__ cand_score, int *__restrict__ node_of,
                                      const int *__restrict__ root, int C, int N, int *status) {
+    allow_dependents();
     extern __shared__ float ssc[];   // [C]
     const int b = blockIdx.x, W = (N + 63) / 64;
     const size_t cb = (size_t)b * C;
@@ -228,6 +244,7 @@ __global__ void verify_setup_kernel(TreeIn t, const int *__restrict__ seq_len,
                                     const int *__restrict__ root, int B, int N, int V,
                                     RowDesc *__restrict__ rows, int *__restrict__ src,
                                     uint64_t *__restrict__ vmask, int *status) {
+    allow_dependents();
     const int r = blockIdx.x * blockDim.x + threadIdx.x;
     if (r >= B * N) return;
     const int b = r / N, i = r - b * N, W = (N + 63) / 64;
@@ -274,6 +291,7 @@ __global__ void accept_kernel(TreeIn t, const int *__restrict__ argmax, int N, i
                               int *__restrict__ acc_a, int *__restrict__ path_out,
                               int *__restrict__ accept_len_out, int *__restrict__ bonus_out,
                               int *__restrict__ index_map_out) {
+    allow_dependents();
     const int b = blockIdx.x, lane = threadIdx.x, D1 = D + 1;
     const size_t nb = (size_t)b * N;
     const int n = t.n_nodes ? t.n_nodes[b] : N;
@@ -319,6 +337,7 @@ __global__ void compact_kv_kernel(const uint4 *__restrict__ tree_kv, uint4 *__re
                                   const int *__restrict__ acc_path, const int *__restrict__ acc_L0,
                                   const int *__restrict__ acc_a, int B, int nh, int N, int S,
                                   int D1, int vec_per_row, int *status) {
+    allow_dependents();
     const int lkh = blockIdx.x, b = blockIdx.y;
     const int h = lkh % nh, lk = lkh / nh;           // lk = layer*2 + kv
     const int a = acc_a[b], L0 = acc_L0[b];
@@ -341,6 +360,7 @@ template <typename T>
 __global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ acc_path,
                               const int *__restrict__ acc_a, int N, int D1, int H,
                               T *__restrict__ pend_h) {
+    allow_dependents();
     const int b = blockIdx.x / D1, j = blockIdx.x - b * D1;
     if (j > acc_a[b]) return;
     const int node = acc_path[b * D1 + j];
@@ -356,6 +376,7 @@ __global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ 
 template <typename T>
 __global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict__ emb,
                                      const int *__restrict__ src, int H) {
+    allow_dependents();
     const int r = blockIdx.x;
     if (src[r] >= 0) return;
     for (int c = threadIdx.x; c < H; c += blockDim.x)
@@ -367,6 +388,7 @@ __global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict_
 template <typename T>
 __global__ void concat_next_kernel(const T *__restrict__ h, const T *__restrict__ emb, int H,
                                    T *__restrict__ xfc) {
+    allow_dependents();
     const int r = blockIdx.x;
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
         xfc[(size_t)r * 2 * H + c] = h[(size_t)r * H + c];
@@ -416,13 +438,15 @@ void launch_hhat_store(const float *x, const RowDesc *rows, int R, int Td, int H
 
 template <typename T>
 void launch_tree_init(const DraftArgs<T> &a, int B, cudaStream_t s) {
-    tree_init_kernel<T><<<B, 256, 0, s>>>(a); note_launch();
+    tree_init_kernel<T><<<dim3(a.k, B), 256, 0, s>>>(a);
+    note_launch();
 }
 
 template <typename T>
 void launch_tree_step(const DraftArgs<T> &a, int B, int d, cudaStream_t s) {
     const size_t sm = (size_t)a.k * a.k * sizeof(float) + (size_t)a.k * sizeof(int);
-    tree_step_kernel<T><<<B, 256, sm, s>>>(a, d); note_launch();
+    tree_step_kernel<T><<<dim3(a.k, B), 256, sm, s>>>(a, d);
+    note_launch();
 }
 
 void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand_par,

@@ -14,10 +14,10 @@ template <typename T>
 struct DraftArgs {
     const int *ids;             // top-k ids of the pass rows [rows][k]
     const float *logp;          // their log-probabilities
-    int k, D, C, H, V, Td, Wd;  // C = k + (D-1)k^2 candidates, Td = (D-1)k slots
+    int k, D, C, H, V, Td, Wd, B;  // C = k + (D-1)k^2 candidates, Td = (D-1)k slots
     int *cand_tok, *cand_par, *cand_depth;   // [B][C]
     float *cand_score;                       // [B][C]
-    int *frontier;                           // [B][k] candidate ids, best first
+    int *frontier;                           // [2][B][k] candidate ids, best first (by pass parity)
     const float *hhat_root;                  // [B][H]
     const float *hhat_slot;                  // [B][Td][H]
     const T *E;

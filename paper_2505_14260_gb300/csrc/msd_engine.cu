@@ -44,6 +44,7 @@ struct msd_ctx {
     uint64_t *slot_mask = nullptr, *row_mask = nullptr;
     int *topk_ids = nullptr;
     float *topk_logp = nullptr;
+    TopkScratch tks{nullptr, nullptr};
     void *hT = nullptr;
     int *acc_path = nullptr, *acc_L0 = nullptr, *acc_a = nullptr;
     float2 *rope_tab = nullptr;
@@ -54,6 +55,15 @@ struct msd_ctx {
     bool status_pending = false;
     GemmPlan *gplan = nullptr;
     AttnTcPlan *aplan = nullptr;
+    // pre-packed GEMM weights (bf16 contexts)
+    struct LayerPack {
+        const void *qkv = nullptr, *o = nullptr, *gu = nullptr, *down = nullptr;
+    };
+    std::vector<LayerPack> lpack;
+    LayerPack dpack;
+    const void *pk_lm = nullptr, *pk_fc = nullptr;
+    void *pk_scratch = nullptr;     // msd_linear: its weight, packed per call
+    size_t pk_scratch_bytes = 0;
     std::vector<void *> allocs;
     std::vector<long> L_bound;
     bool prefilled = false;
@@ -160,15 +170,15 @@ int max_L_bound(const msd_ctx *c) {
 // blocks of rows_per_req per request; every row attends to at most p_bound
 // cache positions.
 template <typename T>
-void run_layer(msd_ctx *c, const msd_layer &lw, int R, const RowDesc *rows, T *kdst, T *vdst,
-               int dst_slots, const T *ck, const T *cv, int cslots, const T *tk, const T *tv,
-               int tslots, const uint64_t *mask, int mw, int rows_per_req, int p_bound,
-               cudaStream_t s) {
+void run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int R,
+               const RowDesc *rows, T *kdst, T *vdst, int dst_slots, const T *ck, const T *cv,
+               int cslots, const T *tk, const T *tv, int tslots, const uint64_t *mask, int mw,
+               int rows_per_req, int p_bound, cudaStream_t s) {
     const int H = c->H, F = c->F;
     const float eps = c->cfg.rms_eps;
     launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.attn_norm), R, H, eps,
                       static_cast<T *>(c->xn), s);
-    GemmW wqkv = {{lw.wq, lw.wk, lw.wv}, {H, H, H}, 3};
+    GemmW wqkv = {{lw.wq, lw.wk, lw.wv}, {H, H, H}, 3, lp.qkv};
     gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wqkv, 3 * H, c->qkv, 3 * H, EPI_STORE, s);
     launch_rope_kv<T>(c->qkv, rows, R, c->nh, c->hd, c->rope_tab, c->S, static_cast<T *>(c->q),
                       kdst, vdst, dst_slots, c->status, s);
@@ -189,18 +199,20 @@ void run_layer(msd_ctx *c, const msd_layer &lw, int R, const RowDesc *rows, T *k
     a.scale = 1.0f / sqrtf((float)c->hd);
     a.out = static_cast<T *>(c->attn);
     attention<T>(c, a, rows_per_req, p_bound, s);
-    GemmW wo = {{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1};
+    GemmW wo = {{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1, lp.o};
     gemm<T>(c, static_cast<const T *>(c->attn), H, R, H, wo, H, c->x, H, EPI_ADD, s);
     launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.mlp_norm), R, H, eps,
                       static_cast<T *>(c->xn), s);
-    GemmW wgu = {{lw.w_gate, lw.w_up, nullptr}, {F, F, 0}, 2};
+    GemmW wgu = {{lw.w_gate, lw.w_up, nullptr}, {F, F, 0}, 2, lp.gu};
     gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wgu, 2 * F, c->gu, 2 * F, EPI_STORE, s);
     launch_swiglu<T>(c->gu, R, F, static_cast<T *>(c->act), s);
-    GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1};
+    GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, lp.down};
     gemm<T>(c, static_cast<const T *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD, s);
 }
 
-GemmW one(const void *w, int rows) { return GemmW{{w, nullptr, nullptr}, {rows, 0, 0}, 1}; }
+GemmW one(const void *w, int rows, const void *packed = nullptr) {
+    return GemmW{{w, nullptr, nullptr}, {rows, 0, 0}, 1, packed};
+}
 
 // ---------------------------------------------------------------------------
 // Prefill
@@ -243,7 +255,7 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
                                  static_cast<T *>(c->emb_all) + (size_t)r0 * H, V, c->status, s);
             for (int l = 0; l < c->NL; ++l) {
                 T *K = tkv<T>(c, c->target_kv, l, 0, c->S), *Vv = tkv<T>(c, c->target_kv, l, 1, c->S);
-                run_layer<T>(c, c->layers[l], n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr,
+                run_layer<T>(c, c->layers[l], c->lpack[l], n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr,
                              nullptr, 0, nullptr, 0, n, r0 + n, s);
             }
             launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), n, H, c->cfg.rms_eps,
@@ -251,8 +263,8 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
             CU(cudaStreamSynchronize(s));   // rd/src host vectors are reused
         }
         const T *h_last = static_cast<const T *>(c->h_all) + (size_t)(L - 1) * H;
-        gemm<T>(c, h_last, H, 1, H, one(c->w.lm_head, V), V, c->logits, V, EPI_STORE, s);
-        launch_argmax(c->logits, 1, V, c->argmax_tmp, s);
+        gemm<T>(c, h_last, H, 1, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V, EPI_STORE, s);
+        launch_argmax(c->logits, 1, V, c->argmax_tmp, c->tks, s);
         // draft cache over positions 0 .. L-2 with the decoupled input (Eq. 7)
         for (int r0 = 0; r0 < L - 1; r0 += c->chunk) {
             const int n = std::min(c->chunk, L - 1 - r0);
@@ -262,12 +274,12 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
             launch_concat_next<T>(static_cast<const T *>(c->h_all) + (size_t)r0 * H,
                                   static_cast<const T *>(c->emb_all) + (size_t)r0 * H, n, H,
                                   static_cast<T *>(c->xfc), s);
-            gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, n, 2 * H, one(c->w.draft_fc, H), H,
+            gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, n, 2 * H, one(c->w.draft_fc, H, c->pk_fc), H,
                     c->x, H, EPI_STORE, s);
             launch_select_visual<T>(c->x, static_cast<const T *>(c->emb_all) + (size_t)r0 * H,
                                     c->src + r0, n, H, s);
             T *K = tkv<T>(c, c->draft_kv, 0, 0, c->S), *Vv = tkv<T>(c, c->draft_kv, 0, 1, c->S);
-            run_layer<T>(c, c->w.draft, n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr, nullptr, 0,
+            run_layer<T>(c, c->w.draft, c->dpack, n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr, nullptr, 0,
                          nullptr, 0, n, r0 + n, s);
             CU(cudaStreamSynchronize(s));
         }
@@ -288,6 +300,7 @@ DraftArgs<T> draft_args(msd_ctx *c) {
     a.ids = c->topk_ids;
     a.logp = c->topk_logp;
     a.k = c->k; a.D = c->D; a.C = c->C; a.H = c->H; a.V = c->V; a.Td = c->Td; a.Wd = c->Wd;
+    a.B = c->B;
     a.cand_tok = c->cand_tok; a.cand_par = c->cand_par; a.cand_depth = c->cand_depth;
     a.cand_score = c->cand_score; a.frontier = c->frontier;
     a.hhat_root = c->hhat_root; a.hhat_slot = c->hhat_slot;
@@ -330,15 +343,15 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
     const int R1 = B * D1;
     launch_catchup_setup<T>(c->seq_len, c->n_pend, static_cast<const T *>(c->pend_h), c->pend_next,
                             E, B, H, D1, V, static_cast<T *>(c->xfc), c->rows, c->status, s);
-    gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, R1, 2 * H, one(c->w.draft_fc, H), H, c->x, H,
+    gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, R1, 2 * H, one(c->w.draft_fc, H, c->pk_fc), H, c->x, H,
             EPI_STORE, s);
     const int pb = max_L_bound(c);
-    run_layer<T>(c, c->w.draft, R1, c->rows, dK, dV, S, dK, dV, S, nullptr, nullptr, 0, nullptr, 0,
+    run_layer<T>(c, c->w.draft, c->dpack, R1, c->rows, dK, dV, S, dK, dV, S, nullptr, nullptr, 0, nullptr, 0,
                  D1, pb, s);
     launch_root_gather<T>(c->x, c->n_pend, B, D1, H, c->hhat_root, static_cast<T *>(c->xr), s);
-    gemm<T>(c, static_cast<const T *>(c->xr), H, B, H, one(c->w.lm_head, V), V, c->logits, V,
+    gemm<T>(c, static_cast<const T *>(c->xr), H, B, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V,
             EPI_STORE, s);
-    launch_topk_logp(c->logits, B, V, k, c->topk_ids, c->topk_logp, s);
+    launch_topk_logp(c->logits, B, V, k, c->topk_ids, c->topk_logp, c->tks, s);
     msd_status st = record_pass(c, rec, 0, 1, s);
     if (st != MSD_OK) return st;
     DraftArgs<T> a = draft_args<T>(c);
@@ -346,14 +359,14 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
     // passes 2..D: expand the frontier
     const int Rk = B * k;
     for (int d = 2; d <= c->D; ++d) {
-        gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, Rk, 2 * H, one(c->w.draft_fc, H), H,
+        gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, Rk, 2 * H, one(c->w.draft_fc, H, c->pk_fc), H,
                 c->x, H, EPI_STORE, s);
-        run_layer<T>(c, c->w.draft, Rk, c->rows, tK, tV, c->Td, dK, dV, S, tK, tV, c->Td,
+        run_layer<T>(c, c->w.draft, c->dpack, Rk, c->rows, tK, tV, c->Td, dK, dV, S, tK, tV, c->Td,
                      c->row_mask, c->Wd, k, pb, s);
         launch_hhat_store<T>(c->x, c->rows, Rk, c->Td, H, c->hhat_slot, static_cast<T *>(c->xr), s);
-        gemm<T>(c, static_cast<const T *>(c->xr), H, Rk, H, one(c->w.lm_head, V), V, c->logits, V,
+        gemm<T>(c, static_cast<const T *>(c->xr), H, Rk, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V,
                 EPI_STORE, s);
-        launch_topk_logp(c->logits, Rk, V, k, c->topk_ids, c->topk_logp, s);
+        launch_topk_logp(c->logits, Rk, V, k, c->topk_ids, c->topk_logp, c->tks, s);
         st = record_pass(c, rec, d - 1, k, s);
         if (st != MSD_OK) return st;
         launch_tree_step<T>(a, B, d, s);
@@ -379,15 +392,15 @@ msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, fl
     for (int l = 0; l < c->NL; ++l) {
         T *K = tkv<T>(c, c->target_kv, l, 0, c->S), *Vv = tkv<T>(c, c->target_kv, l, 1, c->S);
         T *tK = tkv<T>(c, c->tree_kv, l, 0, N), *tV = tkv<T>(c, c->tree_kv, l, 1, N);
-        run_layer<T>(c, c->layers[l], R, c->rows, tK, tV, N, K, Vv, c->S, tK, tV, N, c->vmask, c->W,
+        run_layer<T>(c, c->layers[l], c->lpack[l], R, c->rows, tK, tV, N, K, Vv, c->S, tK, tV, N, c->vmask, c->W,
                      N, pb, s);
     }
     launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), R, H, c->cfg.rms_eps,
                       static_cast<T *>(c->hT), s);
     float *lg = logits_dev ? logits_dev : c->logits;
-    gemm<T>(c, static_cast<const T *>(c->hT), H, R, H, one(c->w.lm_head, V), V, lg, V, EPI_STORE,
+    gemm<T>(c, static_cast<const T *>(c->hT), H, R, H, one(c->w.lm_head, V, c->pk_lm), V, lg, V, EPI_STORE,
             s);
-    launch_argmax(lg, R, V, argmax_dev, s);
+    launch_argmax(lg, R, V, argmax_dev, c->tks, s);
     return post_status(c, s);
 }
 
@@ -424,13 +437,40 @@ msd_status check_capacity(msd_ctx *c) {
     return MSD_OK;
 }
 
+// Packs every GEMM weight once (tile-contiguous, pre-swizzled) so that a
+// pipeline stage is one contiguous 16 KB read.
+bool pack_one(msd_ctx *c, const GemmW &W, int K, const void **out) {
+    void *dst = nullptr;
+    if (!dalloc(c, &dst, gemm_pack_bytes(W, K))) return false;
+    gemm_pack(W, K, dst, 0);
+    *out = dst;
+    return true;
+}
+
+bool pack_layer(msd_ctx *c, const msd_layer &lw, msd_ctx::LayerPack &lp) {
+    const int H = c->H, F = c->F;
+    return pack_one(c, GemmW{{lw.wq, lw.wk, lw.wv}, {H, H, H}, 3, nullptr}, H, &lp.qkv) &&
+           pack_one(c, GemmW{{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1, nullptr}, H, &lp.o) &&
+           pack_one(c, GemmW{{lw.w_gate, lw.w_up, nullptr}, {F, F, 0}, 2, nullptr}, H, &lp.gu) &&
+           pack_one(c, GemmW{{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, nullptr}, F, &lp.down);
+}
+
+bool pack_weights(msd_ctx *c) {
+    for (int l = 0; l < c->NL; ++l)
+        if (!pack_layer(c, c->layers[l], c->lpack[l])) return false;
+    if (!pack_layer(c, c->w.draft, c->dpack)) return false;
+    if (!pack_one(c, one(c->w.lm_head, c->V), c->H, &c->pk_lm)) return false;
+    if (!pack_one(c, one(c->w.draft_fc, c->H), 2 * c->H, &c->pk_fc)) return false;
+    return cudaDeviceSynchronize() == cudaSuccess;
+}
+
 msd_status validate_config(const msd_config *g) {
     if (!g) return MSD_ERR_INVALID;
     if (g->n_layers < 1 || g->hidden < 1 || g->n_heads < 1 || g->ffn < 1 || g->vocab < 2)
         return MSD_ERR_INVALID;
     if (g->head_dim != 64 && g->head_dim != 128) return MSD_ERR_INVALID;
     if (g->n_heads * g->head_dim != g->hidden) return MSD_ERR_INVALID;
-    if (g->hidden % 64 || g->ffn % 16) return MSD_ERR_INVALID;
+    if (g->hidden % 64 || g->ffn % 16 || g->hidden > 8192) return MSD_ERR_INVALID;
     if (g->dtype != MSD_F32 && g->dtype != MSD_BF16) return MSD_ERR_INVALID;
     if (g->max_batch < 1 || g->max_seq < 2) return MSD_ERR_INVALID;
     if (g->tree_nodes < 1 || g->tree_nodes > 256) return MSD_ERR_INVALID;
@@ -511,13 +551,15 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     ok &= dalloc(c, &c->cand_depth, sizeof(int) * c->B * c->C);
     ok &= dalloc(c, &c->cand_score, sizeof(float) * c->B * c->C);
     ok &= dalloc(c, &c->node_of, sizeof(int) * c->B * c->C);
-    ok &= dalloc(c, &c->frontier, sizeof(int) * c->B * c->k);
+    ok &= dalloc(c, &c->frontier, sizeof(int) * 2 * c->B * c->k);
     ok &= dalloc(c, &c->hhat_root, sizeof(float) * c->B * H);
     ok &= dalloc(c, &c->hhat_slot, sizeof(float) * c->B * c->Td * H);
     ok &= dalloc(c, &c->slot_mask, sizeof(uint64_t) * c->B * c->Td * c->Wd);
     ok &= dalloc(c, &c->row_mask, sizeof(uint64_t) * c->B * c->k * c->Wd);
     ok &= dalloc(c, &c->topk_ids, sizeof(int) * c->Rlog * c->k);
     ok &= dalloc(c, &c->topk_logp, sizeof(float) * c->Rlog * c->k);
+    ok &= dalloc(c, &c->tks.ws, sizeof(float) * topk_scratch_floats(c->Rlog, c->V));
+    ok &= dalloc(c, &c->tks.counters, sizeof(int) * c->Rlog);
     ok &= dalloc(c, &c->hT, (size_t)c->B * c->N * H * e);
     ok &= dalloc(c, &c->acc_path, sizeof(int) * c->B * c->D1);
     ok &= dalloc(c, &c->acc_L0, sizeof(int) * c->B);
@@ -530,6 +572,8 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     if (ok) ok = cudaEventCreateWithFlags(&c->status_ev, cudaEventDisableTiming) == cudaSuccess;
     if (ok && cfg->dtype == MSD_BF16) ok = gemm_plan_create(&c->gplan, c->Rmax, c->H, c->F, c->V);
     if (ok && cfg->dtype == MSD_BF16) ok = attn_tc_plan_create(&c->aplan, 32ull << 20, 16384);
+    c->lpack.assign(c->NL, msd_ctx::LayerPack());
+    if (ok && cfg->dtype == MSD_BF16) ok = pack_weights(c);
     if (!ok) {
         msd_destroy(c);
         cudaGetLastError();
@@ -562,6 +606,7 @@ msd_status msd_destroy(msd_ctx *c) {
     if (c->status_ev) cudaEventDestroy(c->status_ev);
     if (c->gplan) gemm_plan_destroy(c->gplan);
     if (c->aplan) attn_tc_plan_destroy(c->aplan);
+    if (c->pk_scratch) cudaFree(c->pk_scratch);
     delete c;
     return MSD_OK;
 }
@@ -651,11 +696,24 @@ msd_status msd_linear(msd_ctx *c, const void *x, int32_t ldx, int32_t m, int32_t
     if (c->cfg.dtype == MSD_BF16 && (ldx % 8 || k % 8))
         return fail(c, MSD_ERR_INVALID, "bf16 rows must be 16-byte aligned");
     cudaStream_t s = static_cast<cudaStream_t>(stream);
-    const GemmW W = one(w, o);
+    GemmW W = one(w, o);
     const int epi = accumulate ? EPI_ADD : EPI_STORE;
-    if (c->cfg.dtype == MSD_BF16)
+    if (c->cfg.dtype == MSD_BF16) {
+        // pack w into the context's scratch (grown on demand), then the GEMM
+        const size_t need = gemm_pack_bytes(W, k);
+        if (need > c->pk_scratch_bytes) {
+            CU(cudaStreamSynchronize(s));
+            if (c->pk_scratch) cudaFree(c->pk_scratch);
+            c->pk_scratch = nullptr;
+            c->pk_scratch_bytes = 0;
+            if (cudaMalloc(&c->pk_scratch, need) != cudaSuccess)
+                return fail(c, MSD_ERR_OOM, "msd_linear: packing scratch");
+            c->pk_scratch_bytes = need;
+        }
+        gemm_pack(W, k, c->pk_scratch, s);
+        W.packed = c->pk_scratch;
         gemm<bf16>(c, static_cast<const bf16 *>(x), ldx, m, k, W, o, y, ldy, epi, s);
-    else
+    } else
         gemm<float>(c, static_cast<const float *>(x), ldx, m, k, W, o, y, ldy, epi, s);
     return post_status(c, s);
 }
