@@ -434,37 +434,55 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             pdl_trigger();
             asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
             // Weights never depend on the previous kernel: the first stages'
-            // weight blocks are requested before waiting for it.
-            const long long n_pre = min((long long)stages, u1 - u0);
-            for (long long j = 0; j < n_pre; ++j) {
-                const int t = (int)((u0 + j) / KB), kb = (int)(u0 + j - (long long)t * KB);
-                const long long blk = (long long)(t / p.n_tiles_n) * KB + kb;
-                mbar_expect_tx(full0 + 8 * (int)j, A_BYTES + b_bytes);
-                bulk_load(a_base + (int)j * A_BYTES, p.wpacked + blk * (A_BYTES / 2), A_BYTES,
-                          full0 + 8 * (int)j);
+            // weight blocks are requested before waiting for it. All per-unit
+            // indices advance incrementally (no divisions on the issue path).
+            const int n = (int)(u1 - u0);
+            const int n_pre = min(stages, n);
+            const int t_first = (int)(u0 / KB), kb_first = (int)(u0 - (long long)t_first * KB);
+            const size_t blk_elems = A_BYTES / 2;
+            {
+                int t = t_first, kb = kb_first;
+                const bf16 *w = p.wpacked + ((size_t)(t / p.n_tiles_n) * KB + kb) * blk_elems;
+                for (int j = 0; j < n_pre; ++j) {
+                    mbar_expect_tx(full0 + 8 * j, A_BYTES + b_bytes);
+                    bulk_load(a_base + j * A_BYTES, w, A_BYTES, full0 + 8 * j);
+                    w += blk_elems;
+                    if (++kb == KB) {
+                        kb = 0;
+                        ++t;
+                        w = p.wpacked + (size_t)(t / p.n_tiles_n) * KB * blk_elems;
+                    }
+                }
             }
             pdl_wait();
-            long long i = 0;
-            for (long long u = u0; u < u1; ++u, ++i) {
-                const int t = (int)(u / KB), kb = (int)(u - (long long)t * KB);
-                int seg, row0, n0;
-                tile_geom(t, seg, row0, n0);
-                const int s = (int)(i % stages);
+            int t = t_first, kb = kb_first, s = 0;
+            uint32_t ph = 0;
+            int n0 = (t % p.n_tiles_n) * BN;
+            const bf16 *w = p.wpacked + ((size_t)(t / p.n_tiles_n) * KB + kb) * blk_elems;
+            int i = 0;
+            for (; i < n; ++i) {
                 if (i >= n_pre) {
-                    const uint32_t ph = (uint32_t)(i / stages) & 1u;
                     if (!mbar_wait(empty0 + 8 * s, ph ^ 1u, &abort_flag, p.status)) break;
                     mbar_expect_tx(full0 + 8 * s, A_BYTES + b_bytes);
-                    const long long blk = (long long)(t / p.n_tiles_n) * KB + kb;
-                    bulk_load(a_base + s * A_BYTES, p.wpacked + blk * (A_BYTES / 2), A_BYTES,
-                              full0 + 8 * s);
+                    bulk_load(a_base + s * A_BYTES, w, A_BYTES, full0 + 8 * s);
                 }
                 tma_load_2d(b_base + s * b_bytes, &mx, kb * BK, n0, full0 + 8 * s);
+                w += blk_elems;
+                if (++kb == KB) {
+                    kb = 0;
+                    ++t;
+                    n0 = (t % p.n_tiles_n) * BN;
+                    w = p.wpacked + (size_t)(t / p.n_tiles_n) * KB * blk_elems;
+                }
+                if (++s == stages) {
+                    s = 0;
+                    ph ^= 1u;
+                }
             }
             if (abort_flag) {
                 volatile int never = 0;
-                const long long issued = i;
-                for (long long j = (issued > stages ? issued - stages : 0); j < issued; ++j)
-                    mbar_wait(full0 + 8 * (int)(j % stages), (uint32_t)(j / stages) & 1u, &never,
+                for (int j = (i > stages ? i - stages : 0); j < i; ++j)
+                    mbar_wait(full0 + 8 * (j % stages), (uint32_t)(j / stages) & 1u, &never,
                               p.status);
             }
         }
@@ -473,31 +491,34 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         pdl_wait();
         if (lane == 0) {
             const uint32_t idesc = instr_desc(BN);
-            long long i = 0;
-            int item = 0;
-            for (long long u = u0; u < u1 && !abort_flag; ++item) {
-                const int t = (int)(u / KB), kb_b = (int)(u - (long long)t * KB);
-                const int kb_e = (int)min((long long)KB, kb_b + (u1 - u));
+            int remaining = (int)(u1 - u0);
+            int kb_b = (int)(u0 % KB), s = 0;
+            uint32_t ph = 0;
+            for (int item = 0; remaining > 0 && !abort_flag; ++item) {
+                const int cnt = min(KB - kb_b, remaining);
                 const int a = item & 1;
                 if (!mbar_wait(acce0 + 8 * a, (uint32_t)((item >> 1) & 1) ^ 1u, &abort_flag,
                                p.status))
                     break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t acc = tmem + a * p.acc_stride;
-                for (int kb = kb_b; kb < kb_e; ++kb, ++i) {
-                    const int s = (int)(i % stages);
-                    const uint32_t ph = (uint32_t)(i / stages) & 1u;
+                for (int j = 0; j < cnt; ++j) {
                     if (!mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status)) break;
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                     const uint64_t ad = smem_desc(a_base + s * A_BYTES);
                     const uint64_t bd = smem_desc(b_base + s * b_bytes);
 #pragma unroll
                     for (int kk = 0; kk < BK / 16; ++kk)
-                        mma_bf16(acc, ad + 2 * kk, bd + 2 * kk, idesc, (kb != kb_b) || (kk != 0));
+                        mma_bf16(acc, ad + 2 * kk, bd + 2 * kk, idesc, (j != 0) || (kk != 0));
                     mma_commit(empty0 + 8 * s);
+                    if (++s == stages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
                 }
                 mma_commit(accf0 + 8 * a);
-                u += kb_e - kb_b;
+                remaining -= cnt;
+                kb_b = 0;
             }
         }
         __syncwarp();
@@ -507,11 +528,11 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;
         const int et = threadIdx.x - 64;     // 0..127
-        int item = 0;
-        for (long long u = u0; u < u1; ++item) {
-            const int t = (int)(u / KB), kb_b = (int)(u - (long long)t * KB);
-            const int kb_e = (int)min((long long)KB, kb_b + (u1 - u));
-            u += kb_e - kb_b;
+        int remaining = (int)(u1 - u0);
+        int t = (int)(u0 / KB), kb_b = (int)(u0 - (long long)t * KB);
+        for (int item = 0; remaining > 0; ++item, ++t, kb_b = 0) {
+            const int kb_e = min(KB, kb_b + remaining);
+            remaining -= kb_e - kb_b;
             const int a = item & 1;
             const bool ok = mbar_wait(accf0 + 8 * a, (uint32_t)(item >> 1) & 1u, &abort_flag,
                                       p.status) && !abort_flag;
@@ -579,19 +600,26 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 float4 acc[4];
 #pragma unroll
                 for (int g = 0; g < 4; ++g) acc[g] = make_float4(0.f, 0.f, 0.f, 0.f);
-                for (int i = 0; i < np; ++i) {
-                    const float4 *src = ws4 + (size_t)s_slot[i] * piece4;
-                    float4 v[4];
+                for (int i0 = 0; i0 < np; i0 += 4) {
+                    float4 v[4][4];
 #pragma unroll
-                    for (int g = 0; g < 4; ++g) {
-                        const int e4 = base4 + g * 128;
-                        v[g] = e4 < n4 ? __ldcg(src + e4) : make_float4(0.f, 0.f, 0.f, 0.f);
+                    for (int pi = 0; pi < 4; ++pi) {
+                        const bool have = i0 + pi < np;
+                        const float4 *src = ws4 + (size_t)s_slot[have ? i0 + pi : 0] * piece4;
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) {
+                            const int e4 = base4 + g * 128;
+                            v[pi][g] = (have && e4 < n4) ? __ldcg(src + e4)
+                                                         : make_float4(0.f, 0.f, 0.f, 0.f);
+                        }
                     }
 #pragma unroll
-                    for (int g = 0; g < 4; ++g) {
-                        acc[g].x += v[g].x; acc[g].y += v[g].y;
-                        acc[g].z += v[g].z; acc[g].w += v[g].w;
-                    }
+                    for (int pi = 0; pi < 4; ++pi)
+#pragma unroll
+                        for (int g = 0; g < 4; ++g) {
+                            acc[g].x += v[pi][g].x; acc[g].y += v[pi][g].y;
+                            acc[g].z += v[pi][g].z; acc[g].w += v[pi][g].w;
+                        }
                 }
 #pragma unroll
                 for (int g = 0; g < 4; ++g) {
