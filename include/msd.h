@@ -173,6 +173,19 @@ msd_status msd_accept_compact(msd_ctx *ctx, const msd_tree *tree,
                               int32_t *accept_len_dev, int32_t *bonus_dev,
                               int32_t *index_map_dev, void *stream);
 
+/* One whole decode step: msd_draft_tree, msd_verify and msd_accept_compact in
+ * sequence (Sec. 3.2; Eq. 6 at T = 0), with the same arguments and outputs as
+ * those calls (the drafted tree is written to *tree and then verified). The
+ * context records the sequence once into a CUDA graph per set of output
+ * buffers and per bucket of cache lengths (512 positions) and replays it, so a
+ * step is one graph launch; the first step in a new bucket records a new graph
+ * (host work of a few milliseconds, and one host-device synchronisation to
+ * refresh the bound on L). While GEMM profiling is enabled the calls run
+ * without a graph. Errors: as for the three calls, and MSD_ERR_CUDA if the
+ * graph cannot be recorded. */
+msd_status msd_step(msd_ctx *ctx, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
+                    int32_t *accept_len_dev, int32_t *bonus_dev, void *stream);
+
 /* Building block used by every projection of the step (Sec. 3.1 decoder
  * layers, Eq. 4 f_down, Eq. 5 LM head), exposed for tests and kernel timing:
  * y[i][j] (= or, if accumulate != 0, +=) sum_t x[i][t] * w[j][t] for i < m,
@@ -212,7 +225,8 @@ msd_status msd_linear_noalloc(const void *x_dev, int32_t ldx, int32_t m, int32_t
                               int32_t accumulate, void *stream);
 
 /* Profiling counters (tracing subsystem). kernel_launches counts every kernel
- * the library has launched in this process. While profiling is enabled on a
+ * the library has run in this process (kernels executed by step graphs
+ * included, kernels merely recorded into graphs excluded). While profiling is enabled on a
  * context, each tensor-core GEMM launch (bf16 contexts) is bracketed by CUDA
  * events on its own stream; msd_profile_read synchronises on them and returns
  * the number of timed launches, their summed durations, and their algorithmic

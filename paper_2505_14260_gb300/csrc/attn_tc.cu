@@ -18,6 +18,7 @@
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
+#include <algorithm>
 #include <cstring>
 #include <unordered_map>
 
@@ -426,13 +427,19 @@ struct AttnTcPlan {
     size_t ws_o_floats = 0, ws_ml_floats = 0;
     int n_counters = 0;
     int num_sms = 148;
+    int chunk_tiles = 1;       // keys per cache split / 64: fixed per context
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     std::unordered_map<MapKey, CUtensorMap, MapKeyHash> maps;
     bool attr_set = false;
 };
 
-bool attn_tc_plan_create(AttnTcPlan **out, size_t ws_bytes, int n_counters) {
+bool attn_tc_plan_create(AttnTcPlan **out, size_t ws_bytes, int n_counters, int max_keys) {
     AttnTcPlan *p = new AttnTcPlan();
+    // The cache range is cut at fixed multiples of chunk_tiles * 64 keys, a
+    // function of the capacity only, so results never depend on how many
+    // (possibly empty) splits a launch covers.
+    const int tiles = (max_keys + KT - 1) / KT;
+    p->chunk_tiles = std::max(1, (tiles + MAX_SPLITS - 2) / (MAX_SPLITS - 1));
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev);
@@ -495,20 +502,15 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     const int has_tree = a.mask != nullptr;
     const int pb = std::max(1, std::min(p_bound, a.cache_slots));
     const int cache_tiles = (pb + KT - 1) / KT;
-    int want = (int)((2L * p->num_sms + base - 1) / base) - has_tree;
-    want = std::max(1, std::min(std::min(want, cache_tiles), MAX_SPLITS - 1));
-    int chunk_tiles = (cache_tiles + want - 1) / want;
-    int nsplit = (cache_tiles + chunk_tiles - 1) / chunk_tiles;
-    auto fits = [&](int ns) {
-        const int tot = ns + has_tree;
-        return tot == 1 || ((size_t)tot * a.R * a.nh * a.hd <= p->ws_o_floats &&
-                            (size_t)tot * a.R * a.nh * 2 <= p->ws_ml_floats && base <= p->n_counters);
-    };
-    while (nsplit > 1 && !fits(nsplit)) {
-        chunk_tiles *= 2;
-        nsplit = (cache_tiles + chunk_tiles - 1) / chunk_tiles;
-    }
-    if (!fits(nsplit)) return false;
+    // enough (row tile, head) CTAs already: one split over the whole range;
+    // otherwise fixed-size splits (the count only covers [0, p_bound))
+    const int chunk_tiles = base >= p->num_sms ? cache_tiles : p->chunk_tiles;
+    const int nsplit = (cache_tiles + chunk_tiles - 1) / chunk_tiles;
+    const int tot = nsplit + has_tree;
+    if (tot > MAX_SPLITS) return false;
+    if (tot > 1 && ((size_t)tot * a.R * a.nh * a.hd > p->ws_o_floats ||
+                    (size_t)tot * a.R * a.nh * 2 > p->ws_ml_floats || base > p->n_counters))
+        return false;
     const long kc_rows = (long)B * a.nh * a.cache_slots;
     const CUtensorMap *mkc = kv_map(p, a.cache_k, kc_rows, a.hd);
     const CUtensorMap *mvc = kv_map(p, a.cache_v, kc_rows, a.hd);

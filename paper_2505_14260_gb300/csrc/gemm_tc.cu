@@ -747,6 +747,8 @@ void gemm_profile_enable(GemmPlan *p, bool on) {
     p->prof_bytes = p->prof_wbytes = 0.0;
 }
 
+bool gemm_profile_on(const GemmPlan *p) { return p->profile; }
+
 GemmProfile gemm_profile_read(GemmPlan *p) {
     GemmProfile r{0, 0.0, p->prof_bytes, p->prof_wbytes};
     for (size_t i = 0; i + 1 < p->ev_used; i += 2) {

@@ -34,6 +34,7 @@ struct GemmProfile {
     double weight_bytes;
 };
 void gemm_profile_enable(GemmPlan *p, bool on);
+bool gemm_profile_on(const GemmPlan *p);
 GemmProfile gemm_profile_read(GemmPlan *p);
 
 }  // namespace msd

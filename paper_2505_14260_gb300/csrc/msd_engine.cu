@@ -9,6 +9,7 @@
 // read by the kernels from device state, so a step needs no host round trip.
 #include <cmath>
 #include <cstdio>
+#include <algorithm>
 #include <cstring>
 #include <string>
 #include <vector>
@@ -68,6 +69,21 @@ struct msd_ctx {
     std::vector<long> L_bound;
     bool prefilled = false;
     std::string err;
+    // whole-step CUDA graphs (msd_step), one per L bucket and buffer set
+    struct StepGraph {
+        cudaGraphExec_t exec = nullptr;
+        int bucket_hi = 0;
+        msd_tree tree{};
+        const void *argmax = nullptr, *path = nullptr, *alen = nullptr, *bonus = nullptr;
+        long kernels = 0;
+        long uses = 0;
+    };
+    std::vector<StepGraph> graphs;
+    cudaStream_t cap_stream = nullptr;
+    int pb_override = 0;        // attention p_bound while capturing a graph
+    bool capturing = false;
+    long captured_launches = 0; // launches recorded into graphs (not executed then)
+    long graph_kernels = 0;     // kernels executed by graph replays
 };
 
 namespace {
@@ -95,6 +111,16 @@ bool dalloc(msd_ctx *c, P **p, size_t bytes) {
     return true;
 }
 
+// A runtime error left pending by code outside this call (or by an earlier
+// teardown) is reported on stderr and cleared, so that a call's status reflects
+// only its own launches.
+bool report_stale_error(const char *where) {
+    const cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess)
+        fprintf(stderr, "msd: %s: found a pending CUDA error: %s\n", where, cudaGetErrorString(e));
+    return e != cudaSuccess;
+}
+
 // The device status word of earlier calls, observed without blocking.
 msd_status check_status(msd_ctx *c) {
     if (c->status_pending && cudaEventQuery(c->status_ev) == cudaSuccess) {
@@ -110,6 +136,7 @@ msd_status check_status(msd_ctx *c) {
 
 msd_status post_status(msd_ctx *c, cudaStream_t s) {
     CU(cudaGetLastError());
+    if (c->capturing) return MSD_OK;    // the step's entry point posts after the replay
     CU(cudaMemcpyAsync(c->status_host, c->status, sizeof(int), cudaMemcpyDeviceToHost, s));
     CU(cudaEventRecord(c->status_ev, s));
     c->status_pending = true;
@@ -159,8 +186,10 @@ void attention<bf16>(msd_ctx *c, const AttnArgs<bf16> &a, int rows_per_req, int 
         c->err = "tensor-core attention: unsupported shape or workspace too small";
 }
 
-// Largest L any request may have now (host-side upper bound).
+// Largest L any request may have now (host-side upper bound); while a step
+// graph is being captured, the upper end of its L bucket.
 int max_L_bound(const msd_ctx *c) {
+    if (c->pb_override > 0) return c->pb_override;
     long m = 1;
     for (long v : c->L_bound) m = std::max(m, v);
     return (int)std::min<long>(m, c->S);
@@ -414,7 +443,8 @@ msd_status accept_impl(msd_ctx *c, const msd_tree *tree, const int32_t *argmax, 
                       c->N, c->S, c->D1, (int)(c->hd * c->esz), c->status, s);
     launch_pend_h<T>(static_cast<const T *>(c->hT), c->acc_path, c->acc_a, c->B, c->N, c->D1, c->H,
                      static_cast<T *>(c->pend_h), s);
-    for (int b = 0; b < c->B; ++b) c->L_bound[b] += c->D1;
+    if (!c->capturing)
+        for (int b = 0; b < c->B; ++b) c->L_bound[b] += c->D1;
     return post_status(c, s);
 }
 
@@ -481,6 +511,22 @@ msd_status validate_config(const msd_config *g) {
     return MSD_OK;
 }
 
+template <typename T>
+msd_status step_eager(msd_ctx *c, const msd_tree *tree, int32_t *argmax, int32_t *path,
+                      int32_t *alen, int32_t *bonus, cudaStream_t s) {
+    msd_status st = draft_impl<T>(c, tree, nullptr, s);
+    if (st == MSD_OK) st = verify_impl<T>(c, tree, argmax, nullptr, s);
+    if (st == MSD_OK) st = accept_impl<T>(c, tree, argmax, path, alen, bonus, nullptr, s);
+    return st;
+}
+
+bool same_buffers(const msd_ctx::StepGraph &g, const msd_tree *t, const void *a,
+                         const void *p, const void *l, const void *b) {
+    return g.tree.tokens == t->tokens && g.tree.parent == t->parent && g.tree.depth == t->depth &&
+           g.tree.mask == t->mask && g.tree.n_nodes == t->n_nodes && g.argmax == a &&
+           g.path == p && g.alen == l && g.bonus == b;
+}
+
 }  // namespace
 
 // ---------------------------------------------------------------------------
@@ -491,6 +537,7 @@ extern "C" {
 msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out) {
     if (!out) return MSD_ERR_INVALID;
     *out = nullptr;
+    if (report_stale_error("msd_create")) return MSD_ERR_CUDA;
     if (validate_config(cfg) != MSD_OK || !w || !w->layers) return MSD_ERR_INVALID;
     const void *need[] = {w->embed, w->final_norm, w->lm_head, w->draft_fc, w->draft.attn_norm,
                           w->draft.wq, w->draft.wk, w->draft.wv, w->draft.wo, w->draft.mlp_norm,
@@ -571,7 +618,7 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     if (ok) ok = cudaMallocHost(&c->status_host, sizeof(int)) == cudaSuccess;
     if (ok) ok = cudaEventCreateWithFlags(&c->status_ev, cudaEventDisableTiming) == cudaSuccess;
     if (ok && cfg->dtype == MSD_BF16) ok = gemm_plan_create(&c->gplan, c->Rmax, c->H, c->F, c->V);
-    if (ok && cfg->dtype == MSD_BF16) ok = attn_tc_plan_create(&c->aplan, 32ull << 20, 16384);
+    if (ok && cfg->dtype == MSD_BF16) ok = attn_tc_plan_create(&c->aplan, 64ull << 20, 16384, c->S);
     c->lpack.assign(c->NL, msd_ctx::LayerPack());
     if (ok && cfg->dtype == MSD_BF16) ok = pack_weights(c);
     if (!ok) {
@@ -598,15 +645,32 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     return MSD_OK;
 }
 
+#define MSD_TEARDOWN(call)                                                               \
+    do {                                                                                 \
+        cudaError_t e_ = (call);                                                         \
+        if (e_ != cudaSuccess)                                                           \
+            fprintf(stderr, "msd_destroy: %s: %s\n", #call, cudaGetErrorString(e_));     \
+    } while (0)
+
 msd_status msd_destroy(msd_ctx *c) {
     if (!c) return MSD_OK;
-    cudaDeviceSynchronize();
-    for (void *p : c->allocs) cudaFree(p);
-    if (c->status_host) cudaFreeHost(c->status_host);
-    if (c->status_ev) cudaEventDestroy(c->status_ev);
+    report_stale_error("msd_destroy");
+    MSD_TEARDOWN(cudaDeviceSynchronize());
+    for (void *p : c->allocs) MSD_TEARDOWN(cudaFree(p));
+    if (c->status_host) MSD_TEARDOWN(cudaFreeHost(c->status_host));
+    if (c->status_ev) MSD_TEARDOWN(cudaEventDestroy(c->status_ev));
     if (c->gplan) gemm_plan_destroy(c->gplan);
     if (c->aplan) attn_tc_plan_destroy(c->aplan);
-    if (c->pk_scratch) cudaFree(c->pk_scratch);
+    if (c->pk_scratch) MSD_TEARDOWN(cudaFree(c->pk_scratch));
+    for (auto &g : c->graphs)
+        if (g.exec) MSD_TEARDOWN(cudaGraphExecDestroy(g.exec));
+    if (c->cap_stream) {
+        const cudaError_t e = cudaStreamDestroy(c->cap_stream);
+        if (e != cudaSuccess)
+            fprintf(stderr, "msd_destroy: ctx %p: cudaStreamDestroy(%p): %s\n", (void *)c,
+                    (void *)c->cap_stream, cudaGetErrorString(e));
+    }
+    report_stale_error("msd_destroy (end)");
     delete c;
     return MSD_OK;
 }
@@ -616,6 +680,8 @@ msd_status msd_prefill(msd_ctx *c, int32_t batch, const int32_t *seq_len_host,
                        const int64_t *vis_off_host, int32_t *root_out_dev, void *stream) {
     if (!c) return MSD_ERR_INVALID;
     c->err.clear();
+    if (report_stale_error("msd_prefill"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
     msd_status st = check_status(c);
     if (st != MSD_OK) return st;
     if (batch < 1 || batch > c->B || !seq_len_host || !ids_dev)
@@ -642,6 +708,8 @@ msd_status msd_draft_tree(msd_ctx *c, const msd_tree *out, const msd_draft_recor
                           void *stream) {
     if (!c) return MSD_ERR_INVALID;
     c->err.clear();
+    if (report_stale_error("msd_draft_tree"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
     msd_status st = check_status(c);
     if (st != MSD_OK) return st;
     if (!tree_ok(out)) return fail(c, MSD_ERR_INVALID, "null tree array");
@@ -657,6 +725,8 @@ msd_status msd_verify(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, flo
                       void *stream) {
     if (!c) return MSD_ERR_INVALID;
     c->err.clear();
+    if (report_stale_error("msd_verify"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
     msd_status st = check_status(c);
     if (st != MSD_OK) return st;
     if (!tree_ok(tree) || !argmax_dev) return fail(c, MSD_ERR_INVALID, "null tree or argmax");
@@ -673,6 +743,8 @@ msd_status msd_accept_compact(msd_ctx *c, const msd_tree *tree, const int32_t *a
                               int32_t *index_map_dev, void *stream) {
     if (!c) return MSD_ERR_INVALID;
     c->err.clear();
+    if (report_stale_error("msd_accept_compact"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
     msd_status st = check_status(c);
     if (st != MSD_OK) return st;
     if (!tree_ok(tree) || !argmax_dev) return fail(c, MSD_ERR_INVALID, "null tree or argmax");
@@ -687,10 +759,102 @@ msd_status msd_accept_compact(msd_ctx *c, const msd_tree *tree, const int32_t *a
                               index_map_dev, s);
 }
 
+msd_status msd_step(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
+                    int32_t *accept_len_dev, int32_t *bonus_dev, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    if (report_stale_error("msd_step"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!tree_ok(tree) || !argmax_dev) return fail(c, MSD_ERR_INVALID, "null tree or argmax");
+    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    st = check_capacity(c);
+    if (st != MSD_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const bool bf = c->cfg.dtype == MSD_BF16;
+    // While GEMM profiling is on, steps run eagerly (events bracket each GEMM).
+    if (bf && c->gplan && gemm_profile_on(c->gplan)) {
+        st = step_eager<bf16>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, s);
+        return st == MSD_OK ? post_status(c, s) : st;
+    }
+    int need = max_L_bound(c);
+    msd_ctx::StepGraph *g = nullptr;
+    bool rollover = false;
+    for (auto &x : c->graphs)
+        if (same_buffers(x, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev)) {
+            if (x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi)) g = &x;
+            else rollover = true;
+        }
+    if (!g) {
+        if (rollover) {   // refresh the bound of L from the device before a new bucket
+            std::vector<int> L(c->B);
+            CU(cudaStreamSynchronize(s));
+            CU(cudaMemcpy(L.data(), c->seq_len, sizeof(int) * c->B, cudaMemcpyDeviceToHost));
+            for (int b = 0; b < c->B; ++b) c->L_bound[b] = L[b];
+            need = max_L_bound(c);
+            for (auto &x : c->graphs)
+                if (same_buffers(x, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev) &&
+                    x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi))
+                    g = &x;
+        }
+    }
+    if (!g) {
+        msd_ctx::StepGraph ng;
+        ng.bucket_hi = std::min(c->S, ((need + c->D + 511) / 512) * 512);
+        ng.tree = *tree;
+        ng.argmax = argmax_dev; ng.path = path_dev; ng.alen = accept_len_dev; ng.bonus = bonus_dev;
+        if (!c->cap_stream)   // graphs are recorded on a stream of the context's own
+            CU(cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking));
+        const long l0 = launch_count();
+        c->pb_override = ng.bucket_hi;
+        c->capturing = true;
+        cudaGraph_t graph = nullptr;
+        cudaError_t ce = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
+        if (ce == cudaSuccess) {
+            st = bf ? step_eager<bf16>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev,
+                                       c->cap_stream)
+                    : step_eager<float>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev,
+                                        c->cap_stream);
+            ce = cudaStreamEndCapture(c->cap_stream, &graph);
+        }
+        c->capturing = false;
+        c->pb_override = 0;
+        ng.kernels = launch_count() - l0;
+        c->captured_launches += ng.kernels;
+        if (ce != cudaSuccess || st != MSD_OK || !graph) {
+            if (graph) cudaGraphDestroy(graph);
+            cudaGetLastError();
+            return st != MSD_OK ? st : fail(c, MSD_ERR_CUDA, std::string("step capture: ") +
+                                                                 cudaGetErrorString(ce));
+        }
+        ce = cudaGraphInstantiate(&ng.exec, graph, 0);
+        cudaGraphDestroy(graph);
+        if (ce != cudaSuccess)
+            return fail(c, MSD_ERR_CUDA, std::string("step graph: ") + cudaGetErrorString(ce));
+        if (c->graphs.size() >= 8) {     // keep the most used graphs
+            auto victim = std::min_element(c->graphs.begin(), c->graphs.end(),
+                                           [](const msd_ctx::StepGraph &a,
+                                              const msd_ctx::StepGraph &b) { return a.uses < b.uses; });
+            cudaGraphExecDestroy(victim->exec);
+            c->graphs.erase(victim);
+        }
+        c->graphs.push_back(ng);
+        g = &c->graphs.back();
+    }
+    CU(cudaGraphLaunch(g->exec, s));
+    g->uses += 1;
+    c->graph_kernels += g->kernels;
+    for (int b = 0; b < c->B; ++b) c->L_bound[b] += c->D1;
+    return post_status(c, s);
+}
+
 msd_status msd_linear(msd_ctx *c, const void *x, int32_t ldx, int32_t m, int32_t k, const void *w,
                       int32_t o, float *y, int32_t ldy, int32_t accumulate, void *stream) {
     if (!c) return MSD_ERR_INVALID;
     c->err.clear();
+    if (report_stale_error("msd_linear"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
     if (!x || !w || !y || m <= 0 || k <= 0 || o <= 0 || ldx < k || ldy < o)
         return fail(c, MSD_ERR_INVALID, "bad msd_linear arguments");
     if (c->cfg.dtype == MSD_BF16 && (ldx % 8 || k % 8))
@@ -703,7 +867,16 @@ msd_status msd_linear(msd_ctx *c, const void *x, int32_t ldx, int32_t m, int32_t
         const size_t need = gemm_pack_bytes(W, k);
         if (need > c->pk_scratch_bytes) {
             CU(cudaStreamSynchronize(s));
-            if (c->pk_scratch) cudaFree(c->pk_scratch);
+            if (c->pk_scratch) MSD_TEARDOWN(cudaFree(c->pk_scratch));
+    for (auto &g : c->graphs)
+        if (g.exec) MSD_TEARDOWN(cudaGraphExecDestroy(g.exec));
+    if (c->cap_stream) {
+        const cudaError_t e = cudaStreamDestroy(c->cap_stream);
+        if (e != cudaSuccess)
+            fprintf(stderr, "msd_destroy: ctx %p: cudaStreamDestroy(%p): %s\n", (void *)c,
+                    (void *)c->cap_stream, cudaGetErrorString(e));
+    }
+    report_stale_error("msd_destroy (end)");
             c->pk_scratch = nullptr;
             c->pk_scratch_bytes = 0;
             if (cudaMalloc(&c->pk_scratch, need) != cudaSuccess)
@@ -727,7 +900,7 @@ msd_status msd_profile_enable(msd_ctx *c, int32_t on) {
 msd_status msd_profile_read(msd_ctx *c, msd_profile *out) {
     if (!c || !out) return MSD_ERR_INVALID;
     memset(out, 0, sizeof *out);
-    out->kernel_launches = launch_count();
+    out->kernel_launches = launch_count() - c->captured_launches + c->graph_kernels;
     if (c->gplan) {
         const GemmProfile g = gemm_profile_read(c->gplan);
         out->gemm_launches = g.launches;

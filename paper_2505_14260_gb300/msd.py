@@ -69,6 +69,8 @@ _SIGNATURES = {
     "msd_verify": (c_int32, [c_void_p, POINTER(msd_tree), c_void_p, c_void_p, c_void_p]),
     "msd_accept_compact": (c_int32, [c_void_p, POINTER(msd_tree), c_void_p, c_void_p, c_void_p,
                                      c_void_p, c_void_p, c_void_p]),
+    "msd_step": (c_int32, [c_void_p, POINTER(msd_tree), c_void_p, c_void_p, c_void_p, c_void_p,
+                           c_void_p]),
     "msd_linear": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32,
                              c_void_p, c_int32, c_int32, c_void_p]),
     "msd_linear_noalloc": (c_int32, [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32,
@@ -226,7 +228,15 @@ class Engine:
         return self.path, self.accept_len, self.bonus
 
     def step(self, stream=None):
-        """draft -> verify -> accept/compact on the device, no host round trip."""
+        """draft -> verify -> accept/compact as one replayed CUDA graph (msd_step)."""
+        st = lib().msd_step(self.ctx, ctypes.byref(self.tree.c()), _ptr(self.argmax),
+                            _ptr(self.path), _ptr(self.accept_len), _ptr(self.bonus),
+                            _stream(stream))
+        self._check(st, "msd_step")
+        return self.path, self.accept_len, self.bonus
+
+    def step_calls(self, stream=None):
+        """The same step as three separate calls (no graph)."""
         self.draft_tree(stream=stream)
         self.verify(stream=stream)
         return self.accept_compact(stream=stream)

@@ -271,3 +271,32 @@ def test_capacity_is_refused_on_the_host():
         eng2.prefill(ids, lens, vis, offs)
     assert e.value.status == msd.MSD_ERR_CAPACITY
     eng2.close()
+
+
+def test_step_graph_matches_separate_calls():
+    """msd_step (replayed CUDA graphs, re-recorded when L crosses a 512-position
+    bucket) gives bit-identical steps to msd_draft_tree + msd_verify +
+    msd_accept_compact."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype="bf16", n_text=(440, 440), steps=24)
+    w = synth.make_weights(wl)
+    prompts = synth.make_prompts(wl)
+    ids, lens, vis, offs = msd.upload_prompts(prompts)
+    assert prompts[0].length > 500
+    ea, _ = open_engine(wl, w)
+    eb, _ = open_engine(wl, w)
+    ea.prefill(ids, lens, vis, offs)
+    eb.prefill(ids, lens, vis, offs)
+    for step in range(wl.steps):
+        pa = [t.clone() for t in ea.step()]
+        pb = [t.clone() for t in eb.step_calls()]
+        torch.cuda.synchronize()
+        for x, y in zip(pa, pb):
+            assert torch.equal(x, y), step
+        assert torch.equal(ea.tree.tokens, eb.tree.tokens)
+        assert torch.equal(ea.argmax, eb.argmax)
+    sa, sb = ea.state(), eb.state()
+    assert torch.equal(sa["seq_len"], sb["seq_len"]) and int(sa["seq_len"][0]) > 512
+    L = int(sa["seq_len"][0])
+    assert torch.equal(sa["target_kv"][..., :L, :], sb["target_kv"][..., :L, :])
+    assert torch.equal(sa["draft_kv"][..., :L - 8, :], sb["draft_kv"][..., :L - 8, :])
+    ea.close(); eb.close()
