@@ -31,7 +31,7 @@ namespace {
 constexpr int ROWS = 64;          // query rows per CTA
 constexpr int KT = 64;            // keys per tile
 constexpr int STAGES = 3;
-constexpr int MAX_SPLITS = 32;    // cache splits + the tree split
+constexpr int MAX_SPLITS = 16;    // cache splits + the tree split = cluster size (<= 16)
 constexpr unsigned long long ATTN_TIMEOUT_NS = 2000000000ull;
 
 struct AttnTcParams {
@@ -39,8 +39,6 @@ struct AttnTcParams {
     const RowDesc *rows;
     const uint64_t *mask;
     bf16 *out;
-    float *ws_o, *ws_ml;
-    int *counters;
     int *status;
     int R, rows_per_req, tiles_per_req, nh, cache_slots, tree_slots, mask_words;
     int nsplit_cache, has_tree, chunk;
@@ -115,6 +113,38 @@ __device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], 
         : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
 }
 
+__device__ __forceinline__ void cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+// Address of the same shared-memory location in CTA `rank` of the cluster.
+__device__ __forceinline__ uint32_t dsmem_addr(uint32_t local, int rank) {
+    uint32_t r;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
+    return r;
+}
+
+__device__ __forceinline__ float dsmem_ld_f32(uint32_t a) {
+    float v;
+    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ float4 dsmem_ld_f4(uint32_t a) {
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(a)
+                 : "memory");
+    return v;
+}
+
 __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
     __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
     return *reinterpret_cast<uint32_t *>(&v);
@@ -132,7 +162,6 @@ __global__ void __launch_bounds__(128)
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t bars[STAGES];
     __shared__ int s_pmax;
-    __shared__ int s_last;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int tile = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
@@ -348,64 +377,61 @@ __global__ void __launch_bounds__(128)
         return;
     }
 
-    // Partials: O (unnormalised) [split][R][nh][HD], (m, l) [split][R][nh][2].
-    const size_t so = (size_t)split * p.R;
+    // Several splits: this (row tile, head)'s CTAs form one thread-block
+    // cluster. Each leaves its partial (unnormalised O, running max m, running
+    // sum l) in its own shared memory; after a cluster barrier every CTA
+    // combines a slice of the rows, reading all partials through distributed
+    // shared memory in rank order (deterministic), and writes them out.
+    __syncthreads();                                   // KV stages are idle now
+    float *s_o = reinterpret_cast<float *>(smem_raw + (kv_s - su32(smem_raw)));   // [64][HD]
+    float *s_ml = s_o + ROWS * HD;                                               // [64][2]
+    {
+        const int la = warp * 16 + (lane >> 2), lb = la + 8;
 #pragma unroll
-    for (int j = 0; j < NT_O; ++j) {
-        const int c = 8 * j + col0;
-        if (va) *reinterpret_cast<float2 *>(p.ws_o + ((so + ra) * p.nh + h) * HD + c) = make_float2(o[j][0], o[j][1]);
-        if (vb) *reinterpret_cast<float2 *>(p.ws_o + ((so + rb) * p.nh + h) * HD + c) = make_float2(o[j][2], o[j][3]);
+        for (int j = 0; j < NT_O; ++j) {
+            const int c = 8 * j + col0;
+            *reinterpret_cast<float2 *>(s_o + la * HD + c) = make_float2(o[j][0], o[j][1]);
+            *reinterpret_cast<float2 *>(s_o + lb * HD + c) = make_float2(o[j][2], o[j][3]);
+        }
+        if ((lane & 3) == 0) {
+            *reinterpret_cast<float2 *>(s_ml + la * 2) = make_float2(m_a, l_a);
+            *reinterpret_cast<float2 *>(s_ml + lb * 2) = make_float2(m_b, l_b);
+        }
     }
-    if ((lane & 3) == 0) {
-        if (va) *reinterpret_cast<float2 *>(p.ws_ml + ((so + ra) * p.nh + h) * 2) = make_float2(m_a, l_a);
-        if (vb) *reinterpret_cast<float2 *>(p.ws_ml + ((so + rb) * p.nh + h) * 2) = make_float2(m_b, l_b);
-    }
-    __threadfence();
-    __syncthreads();
-    const int ticket = tile * p.nh + h;
-    if (threadIdx.x == 0) s_last = atomicAdd(&p.counters[ticket], 1) == nsplit - 1;
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-    // the KV stages are idle now: reuse them for the per-row split weights
-    float (*s_w)[MAX_SPLITS] =
-        reinterpret_cast<float (*)[MAX_SPLITS]>(smem_raw + (kv_s - su32(smem_raw)));
-    // weights of each split per row: exp2(m_s - M) / sum_s exp2(m_s - M) l_s
+    cluster_sync();
+    const uint32_t rank = cluster_rank();
     const int nrows = r_end - r0;
-    for (int rr = threadIdx.x; rr < nrows; rr += 128) {
+    const int per = (nrows + nsplit - 1) / nsplit;
+    const int row_lo = (int)rank * per, row_hi = min(nrows, row_lo + per);
+    const uint32_t o_local = su32(s_o), ml_local = su32(s_ml);
+    constexpr int C4 = HD / 4;
+    for (int rr = row_lo + warp; rr < row_hi; rr += 4) {
         float M = -INFINITY;
         for (int sp = 0; sp < nsplit; ++sp)
-            M = fmaxf(M, __ldcg(p.ws_ml + (((size_t)sp * p.R + r0 + rr) * p.nh + h) * 2));
+            M = fmaxf(M, dsmem_ld_f32(dsmem_addr(ml_local + rr * 8, sp)));
         float den = 0.f;
         for (int sp = 0; sp < nsplit; ++sp) {
-            const float2 ml = __ldcg(reinterpret_cast<const float2 *>(
-                p.ws_ml + (((size_t)sp * p.R + r0 + rr) * p.nh + h) * 2));
-            const float w = M == -INFINITY ? 0.f : exp2f(ml.x - M);
-            s_w[rr][sp] = w;
-            den += w * ml.y;
+            const uint32_t a2 = dsmem_addr(ml_local + rr * 8, sp);
+            const float w = M == -INFINITY ? 0.f : exp2f(dsmem_ld_f32(a2) - M);
+            den += w * dsmem_ld_f32(a2 + 4);
         }
         const float inv = den > 0.f ? 1.f / den : 0.f;
-        for (int sp = 0; sp < nsplit; ++sp) s_w[rr][sp] *= inv;
-    }
-    __syncthreads();
-    // O = sum_s w_s O_s, float4 per thread, splits unrolled for independent loads
-    constexpr int C4 = HD / 4;
-    for (int e = threadIdx.x; e < nrows * C4; e += 128) {
-        const int rr = e / C4, c4 = e - rr * C4;
-        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll 4
-        for (int sp = 0; sp < nsplit; ++sp) {
-            const float4 v = __ldcg(reinterpret_cast<const float4 *>(
-                p.ws_o + (((size_t)sp * p.R + r0 + rr) * p.nh + h) * HD) + c4);
-            const float w = s_w[rr][sp];
-            acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+        if (lane < C4) {
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int sp = 0; sp < nsplit; ++sp) {
+                const float msp = dsmem_ld_f32(dsmem_addr(ml_local + rr * 8, sp));
+                const float w = (M == -INFINITY ? 0.f : exp2f(msp - M)) * inv;
+                const float4 v = dsmem_ld_f4(dsmem_addr(o_local + (rr * HD + 4 * lane) * 4, sp));
+                acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
+            }
+            uint2 packed;
+            packed.x = pack_bf16(acc.x, acc.y);
+            packed.y = pack_bf16(acc.z, acc.w);
+            if (ok)
+                *reinterpret_cast<uint2 *>(p.out + (size_t)(r0 + rr) * H + h * HD + 4 * lane) = packed;
         }
-        uint2 packed;
-        packed.x = pack_bf16(acc.x, acc.y);
-        packed.y = pack_bf16(acc.z, acc.w);
-        *reinterpret_cast<uint2 *>(p.out + (size_t)(r0 + rr) * H + h * HD + c4 * 4) = packed;
     }
-    if (threadIdx.x == 0) p.counters[ticket] = 0;
+    cluster_sync();                                    // partials stay readable until all are done
 }
 
 struct MapKey {
@@ -422,10 +448,6 @@ struct MapKeyHash {
 }  // namespace
 
 struct AttnTcPlan {
-    float *ws_o = nullptr, *ws_ml = nullptr;
-    int *counters = nullptr;
-    size_t ws_o_floats = 0, ws_ml_floats = 0;
-    int n_counters = 0;
     int num_sms = 148;
     int chunk_tiles = 1;       // keys per cache split / 64: fixed per context
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
@@ -433,11 +455,12 @@ struct AttnTcPlan {
     bool attr_set = false;
 };
 
-bool attn_tc_plan_create(AttnTcPlan **out, size_t ws_bytes, int n_counters, int max_keys) {
+bool attn_tc_plan_create(AttnTcPlan **out, int max_keys) {
     AttnTcPlan *p = new AttnTcPlan();
     // The cache range is cut at fixed multiples of chunk_tiles * 64 keys, a
     // function of the capacity only, so results never depend on how many
-    // (possibly empty) splits a launch covers.
+    // (possibly empty) splits a launch covers; with the tree split a launch
+    // has at most MAX_SPLITS CTAs per cluster.
     const int tiles = (max_keys + KT - 1) / KT;
     p->chunk_tiles = std::max(1, (tiles + MAX_SPLITS - 2) / (MAX_SPLITS - 1));
     int dev = 0;
@@ -452,26 +475,11 @@ bool attn_tc_plan_create(AttnTcPlan **out, size_t ws_bytes, int n_counters, int 
         return false;
     }
     p->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-    p->ws_o_floats = ws_bytes / sizeof(float) * 64 / 65;
-    p->ws_ml_floats = ws_bytes / sizeof(float) - p->ws_o_floats;
-    p->n_counters = n_counters;
-    if (cudaMalloc(&p->ws_o, ws_bytes) != cudaSuccess ||
-        cudaMalloc(&p->counters, sizeof(int) * n_counters) != cudaSuccess) {
-        attn_tc_plan_destroy(p);
-        return false;
-    }
-    p->ws_ml = p->ws_o + p->ws_o_floats;
-    cudaMemset(p->counters, 0, sizeof(int) * n_counters);
     *out = p;
     return true;
 }
 
-void attn_tc_plan_destroy(AttnTcPlan *p) {
-    if (!p) return;
-    if (p->ws_o) cudaFree(p->ws_o);
-    if (p->counters) cudaFree(p->counters);
-    delete p;
-}
+void attn_tc_plan_destroy(AttnTcPlan *p) { delete p; }
 
 static const CUtensorMap *kv_map(AttnTcPlan *p, const void *ptr, long rows, int hd) {
     MapKey key{ptr, rows};
@@ -508,9 +516,6 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     const int nsplit = (cache_tiles + chunk_tiles - 1) / chunk_tiles;
     const int tot = nsplit + has_tree;
     if (tot > MAX_SPLITS) return false;
-    if (tot > 1 && ((size_t)tot * a.R * a.nh * a.hd > p->ws_o_floats ||
-                    (size_t)tot * a.R * a.nh * 2 > p->ws_ml_floats || base > p->n_counters))
-        return false;
     const long kc_rows = (long)B * a.nh * a.cache_slots;
     const CUtensorMap *mkc = kv_map(p, a.cache_k, kc_rows, a.hd);
     const CUtensorMap *mvc = kv_map(p, a.cache_v, kc_rows, a.hd);
@@ -527,9 +532,6 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.rows = a.rows;
     tp.mask = a.mask;
     tp.out = a.out;
-    tp.ws_o = p->ws_o;
-    tp.ws_ml = p->ws_ml;
-    tp.counters = p->counters;
     tp.status = status;
     tp.R = a.R;
     tp.rows_per_req = rows_per_req;
@@ -548,14 +550,29 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
                              1024 + ROWS * 128 * 2 + STAGES * 2 * KT * 128 * 2);
         cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              1024 + ROWS * 64 * 2 + STAGES * 2 * KT * 64 * 2);
+        cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
+        cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         p->attr_set = true;
     }
-    dim3 grid(row_tiles, a.nh, nsplit + has_tree);
-    if (a.hd == 128)
-        attn_tc_kernel<128><<<grid, 128, smem, s>>>(*mkc, *mvc, *mkt, *mvt, tp);
-    else
-        attn_tc_kernel<64><<<grid, 128, smem, s>>>(*mkc, *mvc, *mkt, *mvt, tp);
+    // the splits of one (row tile, head) run as one cluster (z = splits)
+    cudaLaunchConfig_t lc;
+    memset(&lc, 0, sizeof lc);
+    lc.gridDim = dim3(row_tiles, a.nh, tot);
+    lc.blockDim = dim3(128);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = 1;
+    at[0].val.clusterDim.y = 1;
+    at[0].val.clusterDim.z = tot;
+    lc.attrs = at;
+    lc.numAttrs = 1;
+    cudaError_t e = a.hd == 128
+                        ? cudaLaunchKernelEx(&lc, attn_tc_kernel<128>, *mkc, *mvc, *mkt, *mvt, tp)
+                        : cudaLaunchKernelEx(&lc, attn_tc_kernel<64>, *mkc, *mvc, *mkt, *mvt, tp);
     note_launch();
+    if (e != cudaSuccess) return false;
     return true;
 }
 

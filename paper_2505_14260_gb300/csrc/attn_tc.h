@@ -7,8 +7,8 @@ namespace msd {
 
 struct AttnTcPlan;
 
-// Workspace for split-KV partials and the per-(row tile, head) tickets.
-bool attn_tc_plan_create(AttnTcPlan **out, size_t ws_bytes, int n_counters, int max_keys);
+// Per-context plan (tensor-map cache, split size); max_keys = cache capacity.
+bool attn_tc_plan_create(AttnTcPlan **out, int max_keys);
 void attn_tc_plan_destroy(AttnTcPlan *p);
 
 // a.R rows grouped by request in blocks of rows_per_req; every row's plen is

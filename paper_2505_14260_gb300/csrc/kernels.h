@@ -74,6 +74,9 @@ void launch_topk_logp(const float *logits, int R, int V, int k, int *ids, float 
 template <typename T>
 void launch_convert(const float *x, T *y, long n, cudaStream_t s);
 
+// Sets the device status word (first code wins), in stream order.
+void launch_flag(int *status, int code, cudaStream_t s);
+
 // ---- GEMM ------------------------------------------------------------------
 
 // Y[m][o] (=|+=) sum_k X[m][k] * W[o][k], with W given as up to three row

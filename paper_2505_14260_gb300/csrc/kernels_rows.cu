@@ -346,6 +346,14 @@ void launch_convert(const float *x, T *y, long n, cudaStream_t s) {
     convert_kernel<T><<<(int)blocks, 256, 0, s>>>(x, y, n); note_launch();
 }
 
+__global__ void flag_status_kernel(int *status, int code) { set_status(status, code); }
+
+void launch_flag(int *status, int code, cudaStream_t s) {
+    cudaGetLastError();
+    flag_status_kernel<<<1, 1, 0, s>>>(status, code);
+    note_launch();
+}
+
 #define MSD_INST(T)                                                                          \
     template void launch_embed_rows<T>(const T *, const T *, const int *, int, int, float *,  \
                                        T *, int, int *, cudaStream_t);                       \

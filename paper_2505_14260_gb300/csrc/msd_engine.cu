@@ -182,8 +182,10 @@ void attention<float>(msd_ctx *c, const AttnArgs<float> &a, int, int, cudaStream
 template <>
 void attention<bf16>(msd_ctx *c, const AttnArgs<bf16> &a, int rows_per_req, int p_bound,
                      cudaStream_t s) {
-    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, p_bound, c->status, s))
-        c->err = "tensor-core attention: unsupported shape or workspace too small";
+    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, p_bound, c->status, s)) {
+        c->err = "tensor-core attention: unsupported shape or launch failure";
+        launch_flag(c->status, ST_RANGE, s);     // reported by the next call
+    }
 }
 
 // Largest L any request may have now (host-side upper bound); while a step
@@ -618,7 +620,7 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     if (ok) ok = cudaMallocHost(&c->status_host, sizeof(int)) == cudaSuccess;
     if (ok) ok = cudaEventCreateWithFlags(&c->status_ev, cudaEventDisableTiming) == cudaSuccess;
     if (ok && cfg->dtype == MSD_BF16) ok = gemm_plan_create(&c->gplan, c->Rmax, c->H, c->F, c->V);
-    if (ok && cfg->dtype == MSD_BF16) ok = attn_tc_plan_create(&c->aplan, 64ull << 20, 16384, c->S);
+    if (ok && cfg->dtype == MSD_BF16) ok = attn_tc_plan_create(&c->aplan, c->S);
     c->lpack.assign(c->NL, msd_ctx::LayerPack());
     if (ok && cfg->dtype == MSD_BF16) ok = pack_weights(c);
     if (!ok) {
