@@ -52,6 +52,8 @@ def parse():
     ap.add_argument("--impl", default="msd", choices=["msd", "reference"])
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--layers", type=int, default=None,
+                    help="cut the target to this many layers (small cases for profiling only)")
     ap.add_argument("--gemm", default=None,
                     help="M,K,O: time the tensor-core GEMM alone on that shape (kernel case)")
     return ap.parse_args()
@@ -266,6 +268,8 @@ def run_msd(args, rank, world, local_rank):
 
     torch.cuda.set_device(local_rank)
     wl = synth.WORKLOADS[args.workload]
+    if args.layers:
+        wl = wl.with_(n_layers=args.layers, name=f"{wl.name}-{args.layers}layers")
     B, N, D, V = wl.batch, wl.tree_nodes, wl.tree_depth, wl.vocab
     weights, prompts = make_inputs(wl, "cuda")
     K, W = args.steps, args.warmup

@@ -30,7 +30,7 @@ namespace {
 
 constexpr int ROWS = 64;          // query rows per CTA
 constexpr int KT = 64;            // keys per tile
-constexpr int STAGES = 3;
+constexpr int MAX_STAGES = 3;
 constexpr int MAX_SPLITS = 16;    // cache splits + the tree split = cluster size (<= 16)
 constexpr unsigned long long ATTN_TIMEOUT_NS = 2000000000ull;
 
@@ -41,7 +41,7 @@ struct AttnTcParams {
     bf16 *out;
     int *status;
     int R, rows_per_req, tiles_per_req, nh, cache_slots, tree_slots, mask_words;
-    int nsplit_cache, has_tree, chunk;
+    int nsplit_cache, has_tree, chunk, stages;
     float scale_log2;
 };
 
@@ -136,6 +136,12 @@ __device__ __forceinline__ float dsmem_ld_f32(uint32_t a) {
     return v;
 }
 
+__device__ __forceinline__ float2 dsmem_ld_f2(uint32_t a) {
+    float2 v;
+    asm volatile("ld.shared::cluster.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a) : "memory");
+    return v;
+}
+
 __device__ __forceinline__ float4 dsmem_ld_f4(uint32_t a) {
     float4 v;
     asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
@@ -160,7 +166,7 @@ __global__ void __launch_bounds__(128)
     constexpr int TILE_BYTES = KT * HD * 2;       // one K (or V) tile
     constexpr int NT_O = HD / 8;                  // O n-tiles per warp
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t bars[STAGES];
+    __shared__ __align__(8) uint64_t bars[MAX_STAGES];
     __shared__ int s_pmax;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -177,7 +183,7 @@ __global__ void __launch_bounds__(128)
     const uint32_t kv_s = base + ROWS * HD * 2;            // STAGES x (K tile, V tile)
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < STAGES; ++s)
+        for (int s = 0; s < p.stages; ++s)
             asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(&bars[s])), "r"(1));
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         s_pmax = 0;
@@ -221,8 +227,9 @@ __global__ void __launch_bounds__(128)
     const int ntiles = k_hi > k_lo ? (k_hi - k_lo + KT - 1) / KT : 0;
     const uint32_t stage_bytes = 2 * TILE_BYTES;
 
+    const int stages = p.stages;
     auto issue = [&](int i) {
-        const int s = i % STAGES;
+        const int s = i % stages;
         const uint32_t bar = su32(&bars[s]);
         const uint32_t kd = kv_s + s * stage_bytes, vd = kd + TILE_BYTES;
         asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar),
@@ -238,7 +245,7 @@ __global__ void __launch_bounds__(128)
     if (threadIdx.x == 0) {
         asm volatile("prefetch.tensormap [%0];" ::"l"(mk) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(mv) : "memory");
-        for (int i = 0; i < min(STAGES, ntiles); ++i) issue(i);
+        for (int i = 0; i < min(stages, ntiles); ++i) issue(i);
     }
 
     // Q fragments of the warp's 16 rows.
@@ -261,8 +268,8 @@ __global__ void __launch_bounds__(128)
     bool ok = true;
 
     for (int i = 0; i < ntiles; ++i) {
-        const int s = i % STAGES;
-        if (!bar_wait(su32(&bars[s]), (uint32_t)(i / STAGES) & 1u, p.status)) ok = false;
+        const int s = i % stages;
+        if (!bar_wait(su32(&bars[s]), (uint32_t)(i / stages) & 1u, p.status)) ok = false;
         const uint32_t ks = kv_s + s * stage_bytes, vs = ks + TILE_BYTES;
         const int key0 = k_lo + i * KT;
 
@@ -352,7 +359,7 @@ __global__ void __launch_bounds__(128)
             }
         }
         __syncthreads();                              // every warp is done with stage s
-        if (threadIdx.x == 0 && i + STAGES < ntiles) issue(i + STAGES);
+        if (threadIdx.x == 0 && i + stages < ntiles) issue(i + stages);
     }
 
     l_a += __shfl_xor_sync(0xffffffffu, l_a, 1);
@@ -406,24 +413,29 @@ __global__ void __launch_bounds__(128)
     const uint32_t o_local = su32(s_o), ml_local = su32(s_ml);
     constexpr int C4 = HD / 4;
     for (int rr = row_lo + warp; rr < row_hi; rr += 4) {
-        float M = -INFINITY;
-        for (int sp = 0; sp < nsplit; ++sp)
-            M = fmaxf(M, dsmem_ld_f32(dsmem_addr(ml_local + rr * 8, sp)));
-        float den = 0.f;
-        for (int sp = 0; sp < nsplit; ++sp) {
-            const uint32_t a2 = dsmem_addr(ml_local + rr * 8, sp);
-            const float w = M == -INFINITY ? 0.f : exp2f(dsmem_ld_f32(a2) - M);
-            den += w * dsmem_ld_f32(a2 + 4);
-        }
+        // lane sp fetches split sp's (m, l); warp shuffles give the max and the sum
+        float2 ml = make_float2(-INFINITY, 0.f);
+        if (lane < nsplit) ml = dsmem_ld_f2(dsmem_addr(ml_local + rr * 8, lane));
+        const float M = warp_max(ml.x);
+        const float w = (lane < nsplit && M != -INFINITY) ? exp2f(ml.x - M) : 0.f;
+        const float den = warp_sum(w * ml.y);
         const float inv = den > 0.f ? 1.f / den : 0.f;
+        const float wn = w * inv;
+        float wsp[MAX_SPLITS];
+#pragma unroll
+        for (int sp = 0; sp < MAX_SPLITS; ++sp) wsp[sp] = __shfl_sync(0xffffffffu, wn, sp);
         if (lane < C4) {
+            float4 v[MAX_SPLITS];
+#pragma unroll
+            for (int sp = 0; sp < MAX_SPLITS; ++sp)     // every load in flight at once
+                if (sp < nsplit) v[sp] = dsmem_ld_f4(dsmem_addr(o_local + (rr * HD + 4 * lane) * 4, sp));
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-            for (int sp = 0; sp < nsplit; ++sp) {
-                const float msp = dsmem_ld_f32(dsmem_addr(ml_local + rr * 8, sp));
-                const float w = (M == -INFINITY ? 0.f : exp2f(msp - M)) * inv;
-                const float4 v = dsmem_ld_f4(dsmem_addr(o_local + (rr * HD + 4 * lane) * 4, sp));
-                acc.x += w * v.x; acc.y += w * v.y; acc.z += w * v.z; acc.w += w * v.w;
-            }
+#pragma unroll
+            for (int sp = 0; sp < MAX_SPLITS; ++sp)
+                if (sp < nsplit) {
+                    acc.x += wsp[sp] * v[sp].x; acc.y += wsp[sp] * v[sp].y;
+                    acc.z += wsp[sp] * v[sp].z; acc.w += wsp[sp] * v[sp].w;
+                }
             uint2 packed;
             packed.x = pack_bf16(acc.x, acc.y);
             packed.y = pack_bf16(acc.z, acc.w);
@@ -462,7 +474,7 @@ bool attn_tc_plan_create(AttnTcPlan **out, int max_keys) {
     // (possibly empty) splits a launch covers; with the tree split a launch
     // has at most MAX_SPLITS CTAs per cluster.
     const int tiles = (max_keys + KT - 1) / KT;
-    p->chunk_tiles = std::max(1, (tiles + MAX_SPLITS - 2) / (MAX_SPLITS - 1));
+    p->chunk_tiles = std::max(2, (tiles + MAX_SPLITS - 2) / (MAX_SPLITS - 1));
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev);
@@ -543,13 +555,15 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.nsplit_cache = nsplit;
     tp.has_tree = has_tree;
     tp.chunk = chunk_tiles * KT;
+    // two stages when a split holds at most two tiles: 2 CTAs per SM fit
+    tp.stages = chunk_tiles <= 2 ? 2 : MAX_STAGES;
     tp.scale_log2 = a.scale * 1.4426950408889634f;
-    const size_t smem = 1024 + (size_t)ROWS * a.hd * 2 + (size_t)STAGES * 2 * KT * a.hd * 2;
+    const size_t smem = 1024 + (size_t)ROWS * a.hd * 2 + (size_t)tp.stages * 2 * KT * a.hd * 2;
     if (!p->attr_set) {
         cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             1024 + ROWS * 128 * 2 + STAGES * 2 * KT * 128 * 2);
+                             1024 + ROWS * 128 * 2 + MAX_STAGES * 2 * KT * 128 * 2);
         cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             1024 + ROWS * 64 * 2 + STAGES * 2 * KT * 64 * 2);
+                             1024 + ROWS * 64 * 2 + MAX_STAGES * 2 * KT * 64 * 2);
         cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         p->attr_set = true;
