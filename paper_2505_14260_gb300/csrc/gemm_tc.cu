@@ -165,6 +165,20 @@ __device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
     asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 }
 
+__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t *r) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
+        "%14,%15}, [%16];"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
+          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
+        : "r"(taddr));
+}
+
+__device__ __forceinline__ void tmem_wait_ld() {
+    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+}
+
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tc_kernel(const __grid_constant__ CUtensorMap mw0, const __grid_constant__ CUtensorMap mw1,
                    const __grid_constant__ CUtensorMap mw2, const __grid_constant__ CUtensorMap mx,
@@ -356,8 +370,9 @@ struct PkParams {
     int seg_rows[3];
     int seg_out[3];
     int M, kblocks, BN, n_tiles_n, stages, acc_stride, tmem_cols, grid;
-    long long units;
-    const bf16 *wpacked;    // pre-packed weights (tile-contiguous, pre-swizzled) or null
+    long long units;        // stream-K units: T_sk tiles x K-blocks
+    int T_sk, dp_rounds;    // stream-K tiles; whole-tile rounds of G tiles after them
+    const bf16 *wpacked;    // pre-packed weights (tile-contiguous, pre-swizzled)
     float *Y;
     int ldy, epi;
     float *ws;
@@ -370,6 +385,31 @@ __device__ __forceinline__ int owner_cta(long long u, long long U, int G) {
     return (int)(((u + 1) * (long long)G - 1) / U);
 }
 
+// The work items of one CTA, in order: its share of the stream-K tiles
+// [0, T_sk) (a contiguous range of (tile, K-block) units, cut at tile
+// boundaries), then its whole data-parallel tiles T_sk + cta + j*G.
+struct ItemIter {
+    long long u, u1;
+    int KB, T_sk, G, cta, dp_j, dp_rounds;
+    __device__ bool next(int &t, int &kb_b, int &kb_e) {
+        if (u < u1) {
+            t = (int)(u / KB);
+            kb_b = (int)(u - (long long)t * KB);
+            kb_e = (int)min((long long)KB, kb_b + (u1 - u));
+            u += kb_e - kb_b;
+            return true;
+        }
+        if (dp_j < dp_rounds) {
+            t = T_sk + cta + dp_j * G;
+            kb_b = 0;
+            kb_e = KB;
+            ++dp_j;
+            return true;
+        }
+        return false;
+    }
+};
+
 __global__ void __launch_bounds__(P_THREADS, 1)
     gemm_persist_kernel(const __grid_constant__ CUtensorMap mx, const PkParams p) {
     extern __shared__ uint8_t smem_raw[];
@@ -381,10 +421,11 @@ __global__ void __launch_bounds__(P_THREADS, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int cta = blockIdx.x;
-    const long long U = p.units;
+    const long long U = p.units;                      // stream-K units
     const long long u0 = (long long)cta * U / p.grid, u1 = (long long)(cta + 1) * U / p.grid;
     const int KB = p.kblocks, stages = p.stages, BN = p.BN;
     const uint32_t b_bytes = (uint32_t)BN * BK * 2;
+    const ItemIter items0{u0, u1, KB, p.T_sk, p.grid, cta, 0, p.dp_rounds};
 
     const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
     const uint32_t a_base = sbase, b_base = sbase + stages * A_BYTES;
@@ -416,7 +457,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_base;
 
-    // (tile) -> weight segment map, weight rows, token rows
+    // (tile) -> weight segment, weight rows, token rows
     auto tile_geom = [&](int t, int &seg, int &row0, int &n0) {
         const int wt = t / p.n_tiles_n, nt = t - wt * p.n_tiles_n;
         int w = wt;
@@ -428,55 +469,49 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         row0 = w * BM;
         n0 = nt * BN;
     };
+    const size_t blk_elems = A_BYTES / 2;
 
     if (warp == 0) {
         if (lane == 0) {
             pdl_trigger();
             asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
             // Weights never depend on the previous kernel: the first stages'
-            // weight blocks are requested before waiting for it. All per-unit
-            // indices advance incrementally (no divisions on the issue path).
-            const int n = (int)(u1 - u0);
-            const int n_pre = min(stages, n);
-            const int t_first = (int)(u0 / KB), kb_first = (int)(u0 - (long long)t_first * KB);
-            const size_t blk_elems = A_BYTES / 2;
+            // weight blocks are requested before waiting for it.
+            int n_pre = 0;
             {
-                int t = t_first, kb = kb_first;
-                const bf16 *w = p.wpacked + ((size_t)(t / p.n_tiles_n) * KB + kb) * blk_elems;
-                for (int j = 0; j < n_pre; ++j) {
-                    mbar_expect_tx(full0 + 8 * j, A_BYTES + b_bytes);
-                    bulk_load(a_base + j * A_BYTES, w, A_BYTES, full0 + 8 * j);
-                    w += blk_elems;
-                    if (++kb == KB) {
-                        kb = 0;
-                        ++t;
-                        w = p.wpacked + (size_t)(t / p.n_tiles_n) * KB * blk_elems;
+                ItemIter it = items0;
+                int t, kb_b, kb_e;
+                while (n_pre < stages && it.next(t, kb_b, kb_e)) {
+                    const bf16 *w = p.wpacked + ((size_t)(t / p.n_tiles_n) * KB + kb_b) * blk_elems;
+                    for (int kb = kb_b; kb < kb_e && n_pre < stages; ++kb, ++n_pre, w += blk_elems) {
+                        mbar_expect_tx(full0 + 8 * n_pre, A_BYTES + b_bytes);
+                        bulk_load(a_base + n_pre * A_BYTES, w, A_BYTES, full0 + 8 * n_pre);
                     }
                 }
             }
             pdl_wait();
-            int t = t_first, kb = kb_first, s = 0;
+            ItemIter it = items0;
+            int t, kb_b, kb_e, s = 0, i = 0;
             uint32_t ph = 0;
-            int n0 = (t % p.n_tiles_n) * BN;
-            const bf16 *w = p.wpacked + ((size_t)(t / p.n_tiles_n) * KB + kb) * blk_elems;
-            int i = 0;
-            for (; i < n; ++i) {
-                if (i >= n_pre) {
-                    if (!mbar_wait(empty0 + 8 * s, ph ^ 1u, &abort_flag, p.status)) break;
-                    mbar_expect_tx(full0 + 8 * s, A_BYTES + b_bytes);
-                    bulk_load(a_base + s * A_BYTES, w, A_BYTES, full0 + 8 * s);
-                }
-                tma_load_2d(b_base + s * b_bytes, &mx, kb * BK, n0, full0 + 8 * s);
-                w += blk_elems;
-                if (++kb == KB) {
-                    kb = 0;
-                    ++t;
-                    n0 = (t % p.n_tiles_n) * BN;
-                    w = p.wpacked + (size_t)(t / p.n_tiles_n) * KB * blk_elems;
-                }
-                if (++s == stages) {
-                    s = 0;
-                    ph ^= 1u;
+            bool stop = false;
+            while (!stop && it.next(t, kb_b, kb_e)) {
+                int seg, row0, n0;
+                tile_geom(t, seg, row0, n0);
+                const bf16 *w = p.wpacked + ((size_t)(t / p.n_tiles_n) * KB + kb_b) * blk_elems;
+                for (int kb = kb_b; kb < kb_e; ++kb, ++i, w += blk_elems) {
+                    if (i >= n_pre) {
+                        if (!mbar_wait(empty0 + 8 * s, ph ^ 1u, &abort_flag, p.status)) {
+                            stop = true;
+                            break;
+                        }
+                        mbar_expect_tx(full0 + 8 * s, A_BYTES + b_bytes);
+                        bulk_load(a_base + s * A_BYTES, w, A_BYTES, full0 + 8 * s);
+                    }
+                    tma_load_2d(b_base + s * b_bytes, &mx, kb * BK, n0, full0 + 8 * s);
+                    if (++s == stages) {
+                        s = 0;
+                        ph ^= 1u;
+                    }
                 }
             }
             if (abort_flag) {
@@ -491,18 +526,17 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         pdl_wait();
         if (lane == 0) {
             const uint32_t idesc = instr_desc(BN);
-            int remaining = (int)(u1 - u0);
-            int kb_b = (int)(u0 % KB), s = 0;
+            ItemIter it = items0;
+            int t, kb_b, kb_e, s = 0;
             uint32_t ph = 0;
-            for (int item = 0; remaining > 0 && !abort_flag; ++item) {
-                const int cnt = min(KB - kb_b, remaining);
+            for (int item = 0; !abort_flag && it.next(t, kb_b, kb_e); ++item) {
                 const int a = item & 1;
                 if (!mbar_wait(acce0 + 8 * a, (uint32_t)((item >> 1) & 1) ^ 1u, &abort_flag,
                                p.status))
                     break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint32_t acc = tmem + a * p.acc_stride;
-                for (int j = 0; j < cnt; ++j) {
+                for (int j = 0; j < kb_e - kb_b; ++j) {
                     if (!mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status)) break;
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                     const uint64_t ad = smem_desc(a_base + s * A_BYTES);
@@ -517,8 +551,6 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                     }
                 }
                 mma_commit(accf0 + 8 * a);
-                remaining -= cnt;
-                kb_b = 0;
             }
         }
         __syncwarp();
@@ -528,11 +560,9 @@ __global__ void __launch_bounds__(P_THREADS, 1)
         const int q = warp & 3;
         const int row = q * 32 + lane;
         const int et = threadIdx.x - 64;     // 0..127
-        int remaining = (int)(u1 - u0);
-        int t = (int)(u0 / KB), kb_b = (int)(u0 - (long long)t * KB);
-        for (int item = 0; remaining > 0; ++item, ++t, kb_b = 0) {
-            const int kb_e = min(KB, kb_b + remaining);
-            remaining -= kb_e - kb_b;
+        ItemIter it = items0;
+        int t, kb_b, kb_e;
+        for (int item = 0; it.next(t, kb_b, kb_e); ++item) {
             const int a = item & 1;
             const bool ok = mbar_wait(accf0 + 8 * a, (uint32_t)(item >> 1) & 1u, &abort_flag,
                                       p.status) && !abort_flag;
@@ -544,27 +574,38 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             const int o = p.seg_out[seg] + o_local;
             const bool whole = kb_b == 0 && kb_e == KB;
             const uint32_t taddr = tmem + a * p.acc_stride + ((uint32_t)(q * 32) << 16);
+            // a CTA cuts at most two stream-K tiles: its first item and its last
             const int slot = 2 * cta + (item == 0 ? 0 : 1);
             float *part = p.ws + (size_t)slot * BN * BM;
-            for (int c0 = 0; c0 < BN; c0 += 16) {
-                uint32_t r[16];
-                tmem_ld16(taddr + c0, r);
-                if (whole) {
-                    if (row_ok) {
+            const bool add = p.epi == EPI_ADD;
+            for (int g0 = 0; g0 < BN; g0 += 32) {
+                // up to 32 accumulator columns with one TMEM round trip
+                const int gw = min(32, BN - g0);
+                uint32_t r[32];
 #pragma unroll
-                        for (int j = 0; j < 16; ++j) {
-                            const int m = n0 + c0 + j;
-                            if (m < p.M) {
-                                float *y = p.Y + (size_t)m * p.ldy + o;
-                                const float v = __uint_as_float(r[j]);
-                                *y = p.epi == EPI_ADD ? *y + v : v;
-                            }
-                        }
+                for (int c = 0; c < 2; ++c)
+                    if (c * 16 < gw) tmem_ld16_nowait(taddr + g0 + c * 16, r + c * 16);
+                tmem_wait_ld();
+                if (!whole) {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j < gw) part[(size_t)(g0 + j) * BM + row] = __uint_as_float(r[j]);
+                } else if (row_ok) {
+                    float *yb = p.Y + (size_t)(n0 + g0) * p.ldy + o;
+                    const int mlim = p.M - (n0 + g0);
+                    if (add) {               // residual: every load in flight, then the stores
+                        float yin[32];
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            yin[j] = (j < gw && j < mlim) ? yb[(size_t)j * p.ldy] : 0.f;
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (j < gw && j < mlim) yb[(size_t)j * p.ldy] = yin[j] + __uint_as_float(r[j]);
+                    } else {
+#pragma unroll
+                        for (int j = 0; j < 32; ++j)
+                            if (j < gw && j < mlim) yb[(size_t)j * p.ldy] = __uint_as_float(r[j]);
                     }
-                } else {
-#pragma unroll
-                    for (int j = 0; j < 16; ++j)
-                        part[(size_t)(c0 + j) * BM + row] = __uint_as_float(r[j]);
                 }
             }
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -592,7 +633,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 continue;
             }
             __threadfence();
-            // flat float4 view of the [BN][128] pieces; 4 float4 per thread in flight per piece
+            // flat float4 view of the [BN][128] pieces; 16 float4 loads in flight per thread
             const int n4 = BN * BM / 4;
             const size_t piece4 = (size_t)BN * BM / 4;
             const float4 *ws4 = reinterpret_cast<const float4 *>(p.ws);
@@ -628,14 +669,22 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                     const int col = (e4 * 4) / BM, r4 = (e4 * 4) - col * BM;
                     const int m = n0 + col;
                     if (m >= p.M || !ok) continue;
-                    const float vv[4] = {acc[g].x, acc[g].y, acc[g].z, acc[g].w};
-#pragma unroll
-                    for (int e = 0; e < 4; ++e) {
-                        const int ol = row0 + r4 + e;
-                        if (ol < p.seg_rows[seg]) {
-                            float *y = p.Y + (size_t)m * p.ldy + p.seg_out[seg] + ol;
-                            *y = p.epi == EPI_ADD ? *y + vv[e] : vv[e];
+                    float *y = p.Y + (size_t)m * p.ldy + p.seg_out[seg] + row0 + r4;
+                    if (row0 + r4 + 4 <= p.seg_rows[seg]) {      // 4 rows, one 16-byte access
+                        float4 out = acc[g];
+                        if (p.epi == EPI_ADD) {
+                            const float4 yi = *reinterpret_cast<const float4 *>(y);
+                            out.x += yi.x; out.y += yi.y; out.z += yi.z; out.w += yi.w;
                         }
+                        *reinterpret_cast<float4 *>(y) = out;
+                    } else {
+                        const float vv[4] = {acc[g].x, acc[g].y, acc[g].z, acc[g].w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            if (row0 + r4 + e < p.seg_rows[seg]) {
+                                if (p.epi == EPI_ADD) y[e] = y[e] + vv[e];
+                                else y[e] = vv[e];
+                            }
                     }
                 }
             }
@@ -817,15 +866,20 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     BN = ((BN + 15) / 16) * 16;
     const int kblocks = (K + BK - 1) / BK;
     const uint32_t stage_bytes = A_BYTES + (uint32_t)BN * BK * 2;
+    // five stages measured best on the decode shapes (deeper rings were slower)
     int stages = (int)((200u * 1024u) / stage_bytes);
-    stages = stages < 2 ? 2 : (stages > P_MAX_STAGES ? P_MAX_STAGES : stages);
+    stages = stages < 2 ? 2 : (stages > 5 ? 5 : stages);
     const size_t smem = 1024 + (size_t)stages * stage_bytes;
     const long long tiles_total = (long long)tiles * nt;
-    const long long units = tiles_total * kblocks;
+    const long long all_units = tiles_total * kblocks;
     // one CTA per SM, at least 4 K-blocks each
-    long long G = units / 4;
+    long long G = all_units / 4;
     if (G > p->num_sms) G = p->num_sms;
     if (G < 1) G = 1;
+    // whole tiles in rounds of G, the remainder split stream-K across all CTAs
+    const int dp_rounds = (int)(tiles_total / G);
+    const int T_sk = (int)(tiles_total - (long long)dp_rounds * G);
+    const long long units = (long long)T_sk * kblocks;
     const size_t ws_need = 2ull * G * BN * BM * sizeof(float);
     if (ws_need > WS_BYTES || tiles_total > N_COUNTERS) {
         flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
@@ -843,6 +897,8 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     pk.tmem_cols = 2 * acc;
     pk.grid = (int)G;
     pk.units = units;
+    pk.T_sk = T_sk;
+    pk.dp_rounds = dp_rounds;
     pk.Y = Y;
     pk.ldy = ldy;
     pk.epi = epi;
