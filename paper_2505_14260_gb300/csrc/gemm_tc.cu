@@ -24,6 +24,7 @@
 #include <cudaTypedefs.h>
 
 #include <cstdio>
+#include <algorithm>
 #include <cstring>
 #include <mutex>
 #include <unordered_map>
@@ -670,7 +671,8 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                     const int m = n0 + col;
                     if (m >= p.M || !ok) continue;
                     float *y = p.Y + (size_t)m * p.ldy + p.seg_out[seg] + row0 + r4;
-                    if (row0 + r4 + 4 <= p.seg_rows[seg]) {      // 4 rows, one 16-byte access
+                    if (row0 + r4 + 4 <= p.seg_rows[seg] &&
+                        ((reinterpret_cast<uintptr_t>(y) & 15u) == 0)) {      // one 16-byte access
                         float4 out = acc[g];
                         if (p.epi == EPI_ADD) {
                             const float4 yi = *reinterpret_cast<const float4 *>(y);
@@ -690,6 +692,263 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             }
             if (et == 0) p.counters[t] = 0;
         }
+    }
+
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                     "r"(p.tmem_cols)
+                     : "memory");
+    }
+}
+
+// ---------------------------------------------------------------------------
+// Split-K with a cluster reduction (decode shapes, M <= 128 token rows).
+//
+// One CTA per (weight tile, token tile, K-split); the s K-splits of a tile are
+// one thread-block cluster. Each CTA streams its K range (pre-packed weight
+// blocks by cp.async.bulk before the previous kernel ends, token blocks by
+// TMA), accumulates in TMEM, and, with s > 1, leaves its fp32 partial in its
+// own shared memory; after a cluster barrier each CTA sums one slice of the
+// tile over all s partials through distributed shared memory, in rank order
+// (deterministic), and writes it. At most two CTAs share an SM, so every
+// launch of the decode step is a single wave.
+// ---------------------------------------------------------------------------
+constexpr int C_THREADS = 128;
+constexpr int C_STAGES = 4;
+
+struct CkParams {
+    int n_seg;
+    int seg_tiles[3];
+    int seg_rows[3];
+    int seg_out[3];
+    int M, kblocks, BN, n_tiles_n, splits, tmem_cols;
+    const bf16 *wpacked;
+    float *Y;
+    int ldy, epi;
+    int *status;
+};
+
+__device__ __forceinline__ void c_cluster_sync() {
+    asm volatile("barrier.cluster.arrive.release.aligned;\nbarrier.cluster.wait.acquire.aligned;" ::: "memory");
+}
+
+__device__ __forceinline__ uint32_t c_cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+
+__device__ __forceinline__ float4 c_dsmem_ld4(uint32_t local, uint32_t rank) {
+    uint32_t a;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(local), "r"(rank));
+    float4 v;
+    asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(a)
+                 : "memory");
+    return v;
+}
+
+__global__ void __launch_bounds__(C_THREADS)
+    gemm_cluster_kernel(const __grid_constant__ CUtensorMap mx, const CkParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    __shared__ __align__(8) uint64_t bars[2 * C_STAGES + 1];
+    __shared__ uint32_t tmem_base;
+    __shared__ volatile int abort_flag;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int wt = blockIdx.x, seg = 0;
+    while (seg < p.n_seg - 1 && wt >= p.seg_tiles[seg]) {
+        wt -= p.seg_tiles[seg];
+        ++seg;
+    }
+    const int row0 = wt * BM;
+    const int n0 = blockIdx.y * p.BN;
+    const int split = blockIdx.z, S = p.splits;
+    const int KB = p.kblocks;
+    const int kb0 = (int)((long long)split * KB / S), kb1 = (int)((long long)(split + 1) * KB / S);
+    const int nk = kb1 - kb0;
+    const int BN = p.BN;
+    const uint32_t b_bytes = (uint32_t)BN * BK * 2;
+    const size_t blk_elems = A_BYTES / 2;
+    const bf16 *wblk = p.wpacked + ((size_t)blockIdx.x * KB + kb0) * blk_elems;
+
+    const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
+    const uint32_t a_base = sbase, b_base = sbase + C_STAGES * A_BYTES;
+    const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[C_STAGES]);
+    const uint32_t done = smem_u32(&bars[2 * C_STAGES]);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < C_STAGES; ++s) {
+            mbar_init(full0 + 8 * s, 1);
+            mbar_init(empty0 + 8 * s, 1);
+        }
+        mbar_init(done, 1);
+        abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                         smem_u32(&tmem_base)),
+                     "r"(p.tmem_cols)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+    }
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tmem_base;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            pdl_trigger();
+            asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
+            // weights first (they never depend on the previous kernel), then wait
+            const int n_pre = min(C_STAGES, nk);
+            for (int j = 0; j < n_pre; ++j) {
+                mbar_expect_tx(full0 + 8 * j, A_BYTES + b_bytes);
+                bulk_load(a_base + j * A_BYTES, wblk + (size_t)j * blk_elems, A_BYTES, full0 + 8 * j);
+            }
+            pdl_wait();
+            int s = 0;
+            uint32_t ph = 0;
+            int i = 0;
+            for (; i < nk; ++i) {
+                if (i >= n_pre) {
+                    if (!mbar_wait(empty0 + 8 * s, ph ^ 1u, &abort_flag, p.status)) break;
+                    mbar_expect_tx(full0 + 8 * s, A_BYTES + b_bytes);
+                    bulk_load(a_base + s * A_BYTES, wblk + (size_t)i * blk_elems, A_BYTES, full0 + 8 * s);
+                }
+                tma_load_2d(b_base + s * b_bytes, &mx, (kb0 + i) * BK, n0, full0 + 8 * s);
+                if (++s == C_STAGES) {
+                    s = 0;
+                    ph ^= 1u;
+                }
+            }
+            if (abort_flag) {
+                volatile int never = 0;
+                for (int j = (i > C_STAGES ? i - C_STAGES : 0); j < i; ++j)
+                    mbar_wait(full0 + 8 * (j % C_STAGES), (uint32_t)(j / C_STAGES) & 1u, &never,
+                              p.status);
+            }
+        }
+        __syncwarp();
+    } else if (warp == 1) {
+        pdl_wait();
+        if (lane == 0) {
+            const uint32_t idesc = instr_desc(BN);
+            int s = 0;
+            uint32_t ph = 0;
+            for (int i = 0; i < nk; ++i) {
+                if (!mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status)) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint64_t ad = smem_desc(a_base + s * A_BYTES);
+                const uint64_t bd = smem_desc(b_base + s * b_bytes);
+#pragma unroll
+                for (int kk = 0; kk < BK / 16; ++kk)
+                    mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (i != 0) || (kk != 0));
+                mma_commit(empty0 + 8 * s);
+                if (++s == C_STAGES) {
+                    s = 0;
+                    ph ^= 1u;
+                }
+            }
+            mma_commit(done);
+        }
+        __syncwarp();
+    } else {
+        pdl_wait();
+    }
+
+    // ---- epilogue: all 4 warps, TMEM lane quarter = warp -------------------
+    const bool ok = mbar_wait(done, 0, &abort_flag, p.status) && !abort_flag;
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const int row = warp * 32 + lane;
+    const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
+    const bool add = p.epi == EPI_ADD;
+    const int rows_here = p.seg_rows[seg] - row0;           // valid weight rows in this tile
+    const int o_base = p.seg_out[seg] + row0;
+    if (S == 1) {
+        for (int g0 = 0; g0 < BN; g0 += 32) {
+            const int gw = min(32, BN - g0);
+            uint32_t r[32];
+#pragma unroll
+            for (int c = 0; c < 2; ++c)
+                if (c * 16 < gw) tmem_ld16_nowait(taddr + g0 + c * 16, r + c * 16);
+            tmem_wait_ld();
+            if (ok && row < rows_here) {
+                float *yb = p.Y + (size_t)(n0 + g0) * p.ldy + o_base + row;
+                const int mlim = p.M - (n0 + g0);
+                if (add) {
+                    float yin[32];
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        yin[j] = (j < gw && j < mlim) ? yb[(size_t)j * p.ldy] : 0.f;
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j < gw && j < mlim) yb[(size_t)j * p.ldy] = yin[j] + __uint_as_float(r[j]);
+                } else {
+#pragma unroll
+                    for (int j = 0; j < 32; ++j)
+                        if (j < gw && j < mlim) yb[(size_t)j * p.ldy] = __uint_as_float(r[j]);
+                }
+            }
+        }
+    } else {
+        // partial [BN][128] fp32 in this CTA's (now idle) stage memory
+        float *part = reinterpret_cast<float *>(smem_raw + (sbase - smem_u32(smem_raw)));
+        for (int g0 = 0; g0 < BN; g0 += 32) {
+            const int gw = min(32, BN - g0);
+            uint32_t r[32];
+#pragma unroll
+            for (int c = 0; c < 2; ++c)
+                if (c * 16 < gw) tmem_ld16_nowait(taddr + g0 + c * 16, r + c * 16);
+            tmem_wait_ld();
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+                if (j < gw) part[(g0 + j) * BM + row] = __uint_as_float(r[j]);
+        }
+        c_cluster_sync();
+        // this CTA's slice of the tile, as float4 (4 consecutive weight rows of one token)
+        const uint32_t rank = c_cluster_rank();
+        const int n4 = BN * BM / 4;
+        const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
+        const uint32_t part_s = smem_u32(part);
+        for (int e4 = lo + threadIdx.x; e4 < hi; e4 += C_THREADS) {
+            float4 v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (q < S) v[q] = c_dsmem_ld4(part_s + e4 * 16, q);
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (q < S) {
+                    acc.x += v[q].x; acc.y += v[q].y; acc.z += v[q].z; acc.w += v[q].w;
+                }
+            const int col = (e4 * 4) / BM, r4 = e4 * 4 - col * BM;
+            const int m = n0 + col;
+            if (!ok || m >= p.M) continue;
+            float *y = p.Y + (size_t)m * p.ldy + o_base + r4;
+            if (r4 + 4 <= rows_here && ((reinterpret_cast<uintptr_t>(y) & 15u) == 0)) {
+                if (add) {
+                    const float4 yi = *reinterpret_cast<const float4 *>(y);
+                    acc.x += yi.x; acc.y += yi.y; acc.z += yi.z; acc.w += yi.w;
+                }
+                *reinterpret_cast<float4 *>(y) = acc;
+            } else {
+                const float vv[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (r4 + e < rows_here) {
+                        if (add) y[e] = y[e] + vv[e];
+                        else y[e] = vv[e];
+                    }
+            }
+        }
+        c_cluster_sync();                 // partials stay readable until every slice is done
     }
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -752,6 +1011,7 @@ struct GemmPlan {
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     std::unordered_map<MapKey, CUtensorMap, MapKeyHash> maps;
     bool smem_set = false;
+    bool cluster_attr_set = false;
     bool profile = false;
     std::vector<cudaEvent_t> ev;
     size_t ev_used = 0;
@@ -847,6 +1107,82 @@ void gemm_pack(const GemmW &W, int K, void *dst, cudaStream_t s) {
     note_launch();
 }
 
+// Launch of the cluster split-K kernel: s K-splits per tile (a cluster), chosen
+// so that tiles * s fills two CTAs per SM once, s <= 8 and >= 2 K-blocks each.
+static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W,
+                         int tiles, int BN, int kblocks, float *Y, int ldy, int epi, int *status,
+                         cudaStream_t s, int O) {
+    CkParams ck;
+    memset(&ck, 0, sizeof ck);
+    ck.n_seg = W.nseg;
+    int out_off = 0;
+    for (int i = 0; i < W.nseg; ++i) {
+        ck.seg_rows[i] = W.rows[i];
+        ck.seg_tiles[i] = (W.rows[i] + BM - 1) / BM;
+        ck.seg_out[i] = out_off;
+        out_off += W.rows[i];
+    }
+    int S = (2 * p->num_sms) / tiles;
+    S = std::max(1, std::min(S, 8));
+    while (S > 1 && kblocks / S < 2) --S;
+    ck.M = M;
+    ck.kblocks = kblocks;
+    ck.BN = BN;
+    ck.n_tiles_n = 1;
+    ck.splits = S;
+    ck.tmem_cols = BN <= 32 ? 32 : (BN <= 64 ? 64 : 128);
+    ck.wpacked = static_cast<const bf16 *>(W.packed);
+    ck.Y = Y;
+    ck.ldy = ldy;
+    ck.epi = epi;
+    ck.status = status;
+    const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
+    if (!mx) return;
+    const size_t smem = 1024 + (size_t)C_STAGES * (A_BYTES + (size_t)BN * BK * 2);
+    if (!p->cluster_attr_set) {
+        cudaFuncSetAttribute(gemm_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)(1024 + C_STAGES * (A_BYTES + 128 * BK * 2)));
+        p->cluster_attr_set = true;
+    }
+    const bool prof = p->profile;
+    if (prof) {
+        while (p->ev.size() < p->ev_used + 2) {
+            cudaEvent_t e;
+            cudaEventCreate(&e);
+            p->ev.push_back(e);
+        }
+        cudaEventRecord(p->ev[p->ev_used], s);
+    }
+    cudaLaunchConfig_t lc;
+    memset(&lc, 0, sizeof lc);
+    lc.gridDim = dim3((unsigned)tiles, 1, (unsigned)S);
+    lc.blockDim = dim3(C_THREADS);
+    lc.dynamicSmemBytes = smem;
+    lc.stream = s;
+    cudaLaunchAttribute at[2];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    at[1].id = cudaLaunchAttributeClusterDimension;
+    at[1].val.clusterDim.x = 1;
+    at[1].val.clusterDim.y = 1;
+    at[1].val.clusterDim.z = (unsigned)S;
+    lc.attrs = at;
+    lc.numAttrs = 2;
+    if (cudaLaunchKernelEx(&lc, gemm_cluster_kernel, *mx, ck) != cudaSuccess) {
+        cudaGetLastError();
+        flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
+        fprintf(stderr, "msd: cluster GEMM launch failed (M=%d K=%d O=%d S=%d)\n", M, K, O, S);
+    }
+    note_launch();
+    if (prof) {
+        cudaEventRecord(p->ev[p->ev_used + 1], s);
+        p->ev_used += 2;
+        const double wb = (double)O * K * 2.0;
+        p->prof_wbytes += wb;
+        p->prof_bytes += wb + (double)M * K * 2.0 + (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
+    }
+}
+
 void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
                int ldy, int epi, int *status, cudaStream_t s) {
     if (M <= 0 || O <= 0) return;
@@ -865,6 +1201,10 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     int BN = (M + nt - 1) / nt;
     BN = ((BN + 15) / 16) * 16;
     const int kblocks = (K + BK - 1) / BK;
+    if (M <= 128 && W.packed) {
+        gemm_cluster(p, X, ldx, M, K, W, tiles, BN, kblocks, Y, ldy, epi, status, s, O);
+        return;
+    }
     const uint32_t stage_bytes = A_BYTES + (uint32_t)BN * BK * 2;
     // five stages measured best on the decode shapes (deeper rings were slower)
     int stages = (int)((200u * 1024u) / stage_bytes);
