@@ -729,6 +729,7 @@ struct CkParams {
     float *Y;
     int ldy, epi;
     int *status;
+    GemmFused fx;           // EPI_SWIGLU / EPI_ROPE_KV operands
 };
 
 __device__ __forceinline__ void c_cluster_sync() {
@@ -750,6 +751,100 @@ __device__ __forceinline__ float4 c_dsmem_ld4(uint32_t local, uint32_t rank) {
                  : "r"(a)
                  : "memory");
     return v;
+}
+
+__device__ __forceinline__ float4 c_smem_ld4(uint32_t local) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
+                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
+                 : "r"(local)
+                 : "memory");
+    return v;
+}
+
+__device__ __forceinline__ uint2 c_pack_bf16x4(float a, float b, float c, float d) {
+    const __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
+    return make_uint2(*reinterpret_cast<const uint32_t *>(&lo), *reinterpret_cast<const uint32_t *>(&hi));
+}
+
+// Paired epilogue over the tile's S partials ([BN][128] fp32 in each cluster
+// CTA's shared memory at part_s): element pairs (r, r + half) of one token,
+// with half = 64 for SwiGLU (gate row, up row) and hd/2 for RoPE (rotate-half
+// partners inside one head). This CTA takes its rank's share of the BN * 64
+// pairs, four consecutive rows at a time; the S partials are summed in rank
+// order, as in the plain reduction.
+__device__ __forceinline__ void c_epilogue_paired(const CkParams &p, uint32_t part_s, uint32_t rank,
+                                                  int S, bool ok, int seg, int wt, int row0, int n0,
+                                                  int rows_here) {
+    const GemmFused &f = p.fx;
+    const bool glu = p.epi == EPI_SWIGLU;
+    const int half = glu ? 64 : (f.hd >> 1), hd = 2 * half;
+    const int n4 = p.BN * 16;
+    const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
+    for (int e = lo + threadIdx.x; e < hi; e += C_THREADS) {
+        const int col = e >> 4, p4 = (e & 15) * 4;
+        const int r = (p4 / half) * hd + (p4 % half);
+        const uint32_t oa = part_s + (uint32_t)(col * BM + r) * 4u, ob = oa + (uint32_t)half * 4u;
+        float4 va[8], vb[8];
+        if (S == 1) {
+            va[0] = c_smem_ld4(oa);
+            vb[0] = c_smem_ld4(ob);
+        } else {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (q < S) {
+                    va[q] = c_dsmem_ld4(oa, q);
+                    vb[q] = c_dsmem_ld4(ob, q);
+                }
+        }
+        float a[4] = {0.f, 0.f, 0.f, 0.f}, b[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (q < S) {
+                a[0] += va[q].x; a[1] += va[q].y; a[2] += va[q].z; a[3] += va[q].w;
+                b[0] += vb[q].x; b[1] += vb[q].y; b[2] += vb[q].z; b[3] += vb[q].w;
+            }
+        const int m = n0 + col;
+        if (!ok || m >= p.M) continue;
+        if (glu) {
+            const int j = wt * 64 + p4;
+            if (j >= f.F) continue;                 // F % 4 == 0: whole groups
+            float o[4];
+#pragma unroll
+            for (int t = 0; t < 4; ++t) o[t] = a[t] / (1.f + __expf(-a[t])) * b[t];
+            *reinterpret_cast<uint2 *>(f.act + (size_t)m * f.F + j) = c_pack_bf16x4(o[0], o[1], o[2], o[3]);
+            continue;
+        }
+        if (r >= rows_here) continue;
+        const int o = row0 + r, h = o / hd, i = o - h * hd;
+        const RowDesc d = f.rows[m];
+        if (seg < 2) {
+            int pos = d.pos;
+            if (pos < 0 || pos >= f.max_pos) {
+                set_status(p.status, ST_RANGE);
+                pos = 0;
+            }
+            const float4 *cs = reinterpret_cast<const float4 *>(f.rope_tab + (size_t)pos * half + i);
+            const float4 c01 = cs[0], c23 = cs[1];
+            const float cx[4] = {c01.x, c01.z, c23.x, c23.z}, sy[4] = {c01.y, c01.w, c23.y, c23.w};
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+                const float x0 = a[t], x1 = b[t];
+                a[t] = x0 * cx[t] - x1 * sy[t];
+                b[t] = x1 * cx[t] + x0 * sy[t];
+            }
+        }
+        bf16 *dst;
+        if (seg == 0) {
+            dst = f.q_out + (size_t)m * (f.nh * hd) + o;
+        } else {
+            if (d.dst >= f.slots) set_status(p.status, ST_RANGE);
+            if (d.dst < 0 || d.dst >= f.slots) continue;
+            dst = (seg == 1 ? f.kdst : f.vdst) + ((size_t)(d.req * f.nh + h) * f.slots + d.dst) * hd + i;
+        }
+        *reinterpret_cast<uint2 *>(dst) = c_pack_bf16x4(a[0], a[1], a[2], a[3]);
+        *reinterpret_cast<uint2 *>(dst + half) = c_pack_bf16x4(b[0], b[1], b[2], b[3]);
+    }
 }
 
 __global__ void __launch_bounds__(C_THREADS)
@@ -865,13 +960,15 @@ __global__ void __launch_bounds__(C_THREADS)
 
     // ---- epilogue: all 4 warps, TMEM lane quarter = warp -------------------
     const bool ok = mbar_wait(done, 0, &abort_flag, p.status) && !abort_flag;
+    pdl_wait();                       // (every thread) before reading Y, rows or the table
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const int row = warp * 32 + lane;
     const uint32_t taddr = tmem + ((uint32_t)(warp * 32) << 16);
     const bool add = p.epi == EPI_ADD;
     const int rows_here = p.seg_rows[seg] - row0;           // valid weight rows in this tile
     const int o_base = p.seg_out[seg] + row0;
-    if (S == 1) {
+    const bool paired = p.epi >= EPI_SWIGLU;
+    if (S == 1 && !paired) {
         for (int g0 = 0; g0 < BN; g0 += 32) {
             const int gw = min(32, BN - g0);
             uint32_t r[32];
@@ -911,13 +1008,15 @@ __global__ void __launch_bounds__(C_THREADS)
             for (int j = 0; j < 32; ++j)
                 if (j < gw) part[(g0 + j) * BM + row] = __uint_as_float(r[j]);
         }
-        c_cluster_sync();
+        if (S > 1) c_cluster_sync();
+        else __syncthreads();
+        const uint32_t rank = S > 1 ? c_cluster_rank() : 0u;
+        const uint32_t part_s = smem_u32(part);
+        if (paired) c_epilogue_paired(p, part_s, rank, S, ok, seg, wt, row0, n0, rows_here);
         // this CTA's slice of the tile, as float4 (4 consecutive weight rows of one token)
-        const uint32_t rank = c_cluster_rank();
         const int n4 = BN * BM / 4;
         const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
-        const uint32_t part_s = smem_u32(part);
-        for (int e4 = lo + threadIdx.x; e4 < hi; e4 += C_THREADS) {
+        for (int e4 = lo + threadIdx.x; !paired && e4 < hi; e4 += C_THREADS) {
             float4 v[8];
 #pragma unroll
             for (int q = 0; q < 8; ++q)
@@ -948,7 +1047,7 @@ __global__ void __launch_bounds__(C_THREADS)
                     }
             }
         }
-        c_cluster_sync();                 // partials stay readable until every slice is done
+        if (S > 1) c_cluster_sync();      // partials stay readable until every slice is done
     }
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
@@ -979,6 +1078,22 @@ __global__ void pack_kernel(GemmW W, int K, int KB, uint8_t *dst) {
         const int row = row0 + r, k = kb * BK + c * 8;
         uint4 v = make_uint4(0, 0, 0, 0);
         if (row < rows && k + 8 <= K) v = *reinterpret_cast<const uint4 *>(src + (size_t)row * K + k);
+        *reinterpret_cast<uint4 *>(out + r * 128 + ((c ^ (r & 7)) << 4)) = v;
+    }
+}
+
+// Glu-packed gate/up: block (t, kb) takes gate rows 64t.. into its rows 0..63
+// and up rows 64t.. into rows 64..127 (rows past F are 0).
+__global__ void pack_glu_kernel(const bf16 *gate, const bf16 *up, int F, int K, int KB, uint8_t *dst) {
+    const long long blk = blockIdx.x;
+    const int t = (int)(blk / KB), kb = (int)(blk - (long long)t * KB);
+    uint8_t *out = dst + blk * (long long)A_BYTES;
+    for (int q = threadIdx.x; q < BM * 8; q += blockDim.x) {
+        const int r = q >> 3, c = q & 7;
+        const int frow = t * 64 + (r & 63), k = kb * BK + c * 8;
+        const bf16 *src = r < 64 ? gate : up;
+        uint4 v = make_uint4(0, 0, 0, 0);
+        if (frow < F && k + 8 <= K) v = *reinterpret_cast<const uint4 *>(src + (size_t)frow * K + k);
         *reinterpret_cast<uint4 *>(out + r * 128 + ((c ^ (r & 7)) << 4)) = v;
     }
 }
@@ -1107,13 +1222,27 @@ void gemm_pack(const GemmW &W, int K, void *dst, cudaStream_t s) {
     note_launch();
 }
 
+size_t gemm_pack_glu_bytes(int F, int K) {
+    return (size_t)((F + 63) / 64) * ((K + BK - 1) / BK) * A_BYTES;
+}
+
+void gemm_pack_glu(const void *gate, const void *up, int F, int K, void *dst, cudaStream_t s) {
+    const long long blocks = (long long)(gemm_pack_glu_bytes(F, K) / A_BYTES);
+    if (blocks <= 0) return;
+    pack_glu_kernel<<<(unsigned)blocks, 256, 0, s>>>(static_cast<const bf16 *>(gate),
+                                                      static_cast<const bf16 *>(up), F, K,
+                                                      (K + BK - 1) / BK, static_cast<uint8_t *>(dst));
+    note_launch();
+}
+
 // Launch of the cluster split-K kernel: s K-splits per tile (a cluster), chosen
 // so that tiles * s fills two CTAs per SM once, s <= 8 and >= 2 K-blocks each.
 static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W,
                          int tiles, int BN, int kblocks, float *Y, int ldy, int epi, int *status,
-                         cudaStream_t s, int O) {
+                         cudaStream_t s, int O, const GemmFused *fx = nullptr) {
     CkParams ck;
     memset(&ck, 0, sizeof ck);
+    if (fx) ck.fx = *fx;
     ck.n_seg = W.nseg;
     int out_off = 0;
     for (int i = 0; i < W.nseg; ++i) {
@@ -1179,8 +1308,27 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
         p->ev_used += 2;
         const double wb = (double)O * K * 2.0;
         p->prof_wbytes += wb;
-        p->prof_bytes += wb + (double)M * K * 2.0 + (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
+        double yb = (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
+        if (epi == EPI_SWIGLU) yb = (double)M * fx->F * 2.0;
+        if (epi == EPI_ROPE_KV) yb = (double)M * O * 2.0;
+        p->prof_bytes += wb + (double)M * K * 2.0 + yb;
     }
+}
+
+bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
+                     const GemmFused &fx, int *status, cudaStream_t s) {
+    if (M <= 0 || M > 128 || !W.packed || W.nseg < 1) return false;
+    if (fx.epi == EPI_SWIGLU && (W.nseg != 1 || W.rows[0] != glu_rows(fx.F) || fx.F % 4)) return false;
+    if (fx.epi == EPI_ROPE_KV &&
+        (W.nseg != 3 || (fx.hd != 64 && fx.hd != 128) || fx.nh * fx.hd != W.rows[0] ||
+         W.rows[1] != W.rows[0] || W.rows[2] != W.rows[0]))
+        return false;
+    if (fx.epi != EPI_SWIGLU && fx.epi != EPI_ROPE_KV) return false;
+    int tiles = 0;
+    for (int i = 0; i < W.nseg; ++i) tiles += (W.rows[i] + BM - 1) / BM;
+    const int BN = ((M + 15) / 16) * 16;
+    gemm_cluster(p, X, ldx, M, K, W, tiles, BN, (K + BK - 1) / BK, nullptr, 0, fx.epi, status, s, O, &fx);
+    return true;
 }
 
 void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,

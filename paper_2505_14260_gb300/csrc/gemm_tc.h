@@ -23,6 +23,38 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
 size_t gemm_pack_bytes(const GemmW &W, int K);
 void gemm_pack(const GemmW &W, int K, void *dst, cudaStream_t s);
 
+// Gate/up weights of a SwiGLU MLP packed interleaved: tile t holds gate rows
+// 64t .. 64t+63 in its rows 0..63 and the matching up rows in rows 64..127, so
+// one tile's epilogue has both operands of silu(g) * u. As a GemmW this is one
+// segment of glu_rows(F) rows; its product Y[m][128t + i] is gate row 64t + i
+// for i < 64 and up row 64t + i - 64 otherwise (rows past F are 0).
+inline int glu_rows(int F) { return 128 * ((F + 63) / 64); }
+size_t gemm_pack_glu_bytes(int F, int K);
+void gemm_pack_glu(const void *gate, const void *up, int F, int K, void *dst, cudaStream_t s);
+
+// Epilogues fused into the decode-shape GEMM (M <= 128, packed weights):
+//   EPI_SWIGLU   W glu-packed; act[m][j] = bf16(silu(g) * u), j < F
+//   EPI_ROPE_KV  W = wq;wk;wv (hd | 128); q rotated (RoPE, rotate-half pairs
+//                (i, i + hd/2), table (cos, sin) per position) into q_out
+//                [M][H]; k rotated and v into kdst/vdst [B][nh][slots][hd] at
+//                slot rows[m].dst of request rows[m].req (dst < 0: not
+//                written; dst >= slots or a position outside the table: status
+//                ST_RANGE).
+struct GemmFused {
+    int epi;
+    bf16 *act;
+    int F;
+    const RowDesc *rows;
+    const float2 *rope_tab;
+    int max_pos;
+    bf16 *q_out, *kdst, *vdst;
+    int slots, nh, hd;
+};
+// Runs the fused GEMM and returns true when the shape takes the decode path;
+// returns false (nothing launched) otherwise.
+bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
+                     const GemmFused &fx, int *status, cudaStream_t s);
+
 // Profiling: while enabled, every launch is bracketed by CUDA events on its
 // stream; gemm_profile_read synchronises on them and returns the launches,
 // their summed durations and their algorithmic bytes (weights + X + Y),

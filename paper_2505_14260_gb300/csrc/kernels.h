@@ -22,9 +22,11 @@ template <typename T>
 void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
                     cudaStream_t s);
 
-// act[r][j] = T(silu(gu[r][j]) * gu[r][F + j])
+// act[r][j] = T(silu(g) * u) with g = gu[r][j], u = gu[r][F + j], or, for
+// glu-packed gate/up products (glu = true, rows of 128 * ceil(F / 64)),
+// g = gu[r][128 (j / 64) + j % 64] and u 64 columns further.
 template <typename T>
-void launch_swiglu(const float *gu, int R, int F, T *act, cudaStream_t s);
+void launch_swiglu(const float *gu, int R, int F, bool glu, T *act, cudaStream_t s);
 
 // RoPE (rotate-half, table of (cos, sin) per position and pair) on q and k of
 // qkv [R][3H]; q -> q_out [R][H]; k, v -> kdst/vdst at slot rows[r].dst of
@@ -87,7 +89,7 @@ struct GemmW {
     int nseg;
     const void *packed;   // the same weights pre-packed by gemm_pack (bf16), or null
 };
-enum { EPI_STORE = 0, EPI_ADD = 1 };
+enum { EPI_STORE = 0, EPI_ADD = 1, EPI_SWIGLU = 2, EPI_ROPE_KV = 3 };
 
 template <typename T>
 void launch_gemm_simt(const T *X, int ldx, int M, int K, const GemmW &W, int O,

@@ -114,22 +114,24 @@ void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
 // SwiGLU: silu(gate) * up
 // ---------------------------------------------------------------------------
 template <typename T>
-__global__ void swiglu_kernel(const float *__restrict__ gu, int F, T *__restrict__ act) {
+__global__ void swiglu_kernel(const float *__restrict__ gu, int F, int glu, T *__restrict__ act) {
     allow_dependents();
     const int r = blockIdx.y;
-    const float *row = gu + (size_t)r * 2 * F;
+    const int ld = glu ? 128 * ((F + 63) / 64) : 2 * F;
+    const float *row = gu + (size_t)r * ld;
     for (int j = blockIdx.x * blockDim.x + threadIdx.x; j < F; j += gridDim.x * blockDim.x) {
-        float g = row[j], u = row[F + j];
-        float sg = g / (1.f + __expf(-g));
+        const int gi = glu ? ((j >> 6) << 7) + (j & 63) : j;
+        const float g = row[gi], u = row[gi + (glu ? 64 : F)];
+        const float sg = g / (1.f + __expf(-g));
         act[(size_t)r * F + j] = from_f<T>(sg * u);
     }
 }
 
 template <typename T>
-void launch_swiglu(const float *gu, int R, int F, T *act, cudaStream_t s) {
+void launch_swiglu(const float *gu, int R, int F, bool glu, T *act, cudaStream_t s) {
     if (R <= 0) return;
     dim3 grid((F + 255) / 256, R);
-    swiglu_kernel<T><<<grid, 256, 0, s>>>(gu, F, act); note_launch();
+    swiglu_kernel<T><<<grid, 256, 0, s>>>(gu, F, glu ? 1 : 0, act); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -359,7 +361,7 @@ void launch_flag(int *status, int code, cudaStream_t s) {
                                        T *, int, int *, cudaStream_t);                       \
     template void launch_rmsnorm<T>(const float *, const T *, int, int, float, T *,          \
                                     cudaStream_t);                                           \
-    template void launch_swiglu<T>(const float *, int, int, T *, cudaStream_t);              \
+    template void launch_swiglu<T>(const float *, int, int, bool, T *, cudaStream_t);              \
     template void launch_rope_kv<T>(const float *, const RowDesc *, int, int, int,           \
                                     const float2 *, int, T *, T *, T *, int, int *,          \
                                     cudaStream_t);                                           \

@@ -12,6 +12,7 @@
 #include <algorithm>
 #include <cstring>
 #include <string>
+#include <type_traits>
 #include <vector>
 
 #include "msd.h"
@@ -197,6 +198,61 @@ int max_L_bound(const msd_ctx *c) {
     return (int)std::min<long>(m, c->S);
 }
 
+// qkv = xn [wq;wk;wv]^T, then RoPE on q and k (Sec. 3.1 backbone), q to c->q
+// and k, v to kdst/vdst at each row's slot. Decode shapes run it as one GEMM
+// with the rotation and placement in its epilogue.
+template <typename T>
+void qkv_rope(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int R,
+              const RowDesc *rows, T *kdst, T *vdst, int dst_slots, cudaStream_t s) {
+    const int H = c->H;
+    GemmW wqkv = {{lw.wq, lw.wk, lw.wv}, {H, H, H}, 3, lp.qkv};
+    if constexpr (std::is_same<T, bf16>::value) {
+        GemmFused fx;
+        memset(&fx, 0, sizeof fx);
+        fx.epi = EPI_ROPE_KV;
+        fx.rows = rows;
+        fx.rope_tab = c->rope_tab;
+        fx.max_pos = c->S;
+        fx.q_out = static_cast<bf16 *>(c->q);
+        fx.kdst = kdst;
+        fx.vdst = vdst;
+        fx.slots = dst_slots;
+        fx.nh = c->nh;
+        fx.hd = c->hd;
+        if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), H, R, H, wqkv, 3 * H, fx,
+                            c->status, s))
+            return;
+    }
+    gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wqkv, 3 * H, c->qkv, 3 * H, EPI_STORE, s);
+    launch_rope_kv<T>(c->qkv, rows, R, c->nh, c->hd, c->rope_tab, c->S, static_cast<T *>(c->q),
+                      kdst, vdst, dst_slots, c->status, s);
+}
+
+// act = silu(xn wg^T) * (xn wu^T). bf16 contexts hold gate/up glu-packed; the
+// decode shapes apply the SwiGLU in the GEMM's epilogue.
+template <typename T>
+void gate_up_swiglu(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int R,
+                    cudaStream_t s) {
+    const int H = c->H, F = c->F;
+    if constexpr (std::is_same<T, bf16>::value) {
+        const int O = glu_rows(F);
+        GemmW wgu = {{nullptr, nullptr, nullptr}, {O, 0, 0}, 1, lp.gu};
+        GemmFused fx;
+        memset(&fx, 0, sizeof fx);
+        fx.epi = EPI_SWIGLU;
+        fx.act = static_cast<bf16 *>(c->act);
+        fx.F = F;
+        if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), H, R, H, wgu, O, fx, c->status, s))
+            return;
+        gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wgu, O, c->gu, O, EPI_STORE, s);
+        launch_swiglu<T>(c->gu, R, F, true, static_cast<T *>(c->act), s);
+    } else {
+        GemmW wgu = {{lw.w_gate, lw.w_up, nullptr}, {F, F, 0}, 2, nullptr};
+        gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wgu, 2 * F, c->gu, 2 * F, EPI_STORE, s);
+        launch_swiglu<T>(c->gu, R, F, false, static_cast<T *>(c->act), s);
+    }
+}
+
 // One pre-norm decoder layer over R rows (target or draft). Rows come in
 // blocks of rows_per_req per request; every row attends to at most p_bound
 // cache positions.
@@ -209,10 +265,7 @@ void run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, in
     const float eps = c->cfg.rms_eps;
     launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.attn_norm), R, H, eps,
                       static_cast<T *>(c->xn), s);
-    GemmW wqkv = {{lw.wq, lw.wk, lw.wv}, {H, H, H}, 3, lp.qkv};
-    gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wqkv, 3 * H, c->qkv, 3 * H, EPI_STORE, s);
-    launch_rope_kv<T>(c->qkv, rows, R, c->nh, c->hd, c->rope_tab, c->S, static_cast<T *>(c->q),
-                      kdst, vdst, dst_slots, c->status, s);
+    qkv_rope<T>(c, lw, lp, R, rows, kdst, vdst, dst_slots, s);
     AttnArgs<T> a;
     a.q = static_cast<const T *>(c->q);
     a.rows = rows;
@@ -234,9 +287,7 @@ void run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, in
     gemm<T>(c, static_cast<const T *>(c->attn), H, R, H, wo, H, c->x, H, EPI_ADD, s);
     launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.mlp_norm), R, H, eps,
                       static_cast<T *>(c->xn), s);
-    GemmW wgu = {{lw.w_gate, lw.w_up, nullptr}, {F, F, 0}, 2, lp.gu};
-    gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wgu, 2 * F, c->gu, 2 * F, EPI_STORE, s);
-    launch_swiglu<T>(c->gu, R, F, static_cast<T *>(c->act), s);
+    gate_up_swiglu<T>(c, lw, lp, R, s);
     GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, lp.down};
     gemm<T>(c, static_cast<const T *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD, s);
 }
@@ -479,11 +530,19 @@ bool pack_one(msd_ctx *c, const GemmW &W, int K, const void **out) {
     return true;
 }
 
+bool pack_glu(msd_ctx *c, const void *gate, const void *up, int F, int K, const void **out) {
+    void *dst = nullptr;
+    if (!dalloc(c, &dst, gemm_pack_glu_bytes(F, K))) return false;
+    gemm_pack_glu(gate, up, F, K, dst, 0);
+    *out = dst;
+    return true;
+}
+
 bool pack_layer(msd_ctx *c, const msd_layer &lw, msd_ctx::LayerPack &lp) {
     const int H = c->H, F = c->F;
     return pack_one(c, GemmW{{lw.wq, lw.wk, lw.wv}, {H, H, H}, 3, nullptr}, H, &lp.qkv) &&
            pack_one(c, GemmW{{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1, nullptr}, H, &lp.o) &&
-           pack_one(c, GemmW{{lw.w_gate, lw.w_up, nullptr}, {F, F, 0}, 2, nullptr}, H, &lp.gu) &&
+           pack_glu(c, lw.w_gate, lw.w_up, F, H, &lp.gu) &&
            pack_one(c, GemmW{{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, nullptr}, F, &lp.down);
 }
 
@@ -539,7 +598,6 @@ extern "C" {
 msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out) {
     if (!out) return MSD_ERR_INVALID;
     *out = nullptr;
-    if (report_stale_error("msd_create")) return MSD_ERR_CUDA;
     if (validate_config(cfg) != MSD_OK || !w || !w->layers) return MSD_ERR_INVALID;
     const void *need[] = {w->embed, w->final_norm, w->lm_head, w->draft_fc, w->draft.attn_norm,
                           w->draft.wq, w->draft.wk, w->draft.wv, w->draft.wo, w->draft.mlp_norm,
@@ -552,6 +610,8 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
         for (const void *p : lp)
             if (!p) return MSD_ERR_INVALID;
     }
+    // (arguments are checked first: that needs no GPU)
+    if (report_stale_error("msd_create")) return MSD_ERR_CUDA;
     msd_ctx *c = new msd_ctx();
     c->cfg = *cfg;
     c->w = *w;
@@ -586,7 +646,7 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     ok &= dalloc(c, &c->qkv, R * 3 * H * 4);
     ok &= dalloc(c, &c->q, R * H * e);
     ok &= dalloc(c, &c->attn, R * H * e);
-    ok &= dalloc(c, &c->gu, R * 2 * F * 4);
+    ok &= dalloc(c, &c->gu, R * std::max<size_t>(2 * F, glu_rows(c->F)) * 4);
     ok &= dalloc(c, &c->act, R * F * e);
     ok &= dalloc(c, &c->xfc, R * 2 * H * e);
     ok &= dalloc(c, &c->xr, R * H * e);

@@ -35,9 +35,15 @@ def _kv_compare(eng, st, wl, b, L, dtype, what):
         assert rel_l2(g, r) <= KV_REL_L2[dtype], f"{what} draft kv {kv}: {rel_l2(g, r)}"
 
 
-@pytest.mark.parametrize("dtype", ["f32", "bf16"])
-def test_tiny_all_steps_match_oracle(dtype):
+@pytest.mark.parametrize("dtype,long_prompt", [("f32", False), ("bf16", False), ("bf16", True)],
+                         ids=["f32", "bf16", "bf16-long-prompt"])
+def test_tiny_all_steps_match_oracle(dtype, long_prompt):
+    """The long prompt (364 positions) takes the prefill through the GEMM's
+    many-row path (separate RoPE and SwiGLU kernels); the short one and every
+    decode step through the fused-epilogue path."""
     wl = synth.WORKLOADS["tiny"].with_(dtype=dtype)
+    if long_prompt:
+        wl = wl.with_(n_text=(300, 300), steps=3)
     tol = TOL[dtype]
     eng, w = open_engine(wl)
     m = oracle_model(wl, w)
