@@ -9,6 +9,7 @@ namespace msd {
 template <typename T, int HD>
 __global__ void attn_simt_kernel(AttnArgs<T> a) {
     allow_dependents();
+    wait_prior();
     constexpr int EPL = HD / 32;    // elements per lane
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;
@@ -69,9 +70,9 @@ void launch_attention(const AttnArgs<T> &a, cudaStream_t s) {
     const int threads = 128;
     const int blocks = (int)((warps * 32 + threads - 1) / threads);
     if (a.hd == 128)
-        attn_simt_kernel<T, 128><<<blocks, threads, 0, s>>>(a);
+        launch_pdl(attn_simt_kernel<T, 128>, blocks, threads, 0, s, a);
     else
-        attn_simt_kernel<T, 64><<<blocks, threads, 0, s>>>(a);
+        launch_pdl(attn_simt_kernel<T, 64>, blocks, threads, 0, s, a);
     note_launch();
 }
 

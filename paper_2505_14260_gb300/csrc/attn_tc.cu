@@ -174,7 +174,6 @@ __global__ void __launch_bounds__(128)
     const int blk = tile / p.tiles_per_req;
     const int r0 = blk * p.rows_per_req + (tile - blk * p.tiles_per_req) * ROWS;
     const int r_end = min(r0 + ROWS, (blk + 1) * p.rows_per_req);
-    const int req = p.rows[r0].req;
     const bool is_tree = p.has_tree && split == p.nsplit_cache;
     const int H = p.nh * HD;
 
@@ -187,25 +186,18 @@ __global__ void __launch_bounds__(128)
             asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(&bars[s])), "r"(1));
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         s_pmax = 0;
+        asm volatile("prefetch.tensormap [%0];" ::"l"(&mkc) : "memory");
+        asm volatile("prefetch.tensormap [%0];" ::"l"(&mvc) : "memory");
     }
+    wait_prior();                  // q, the row descriptors and K/V come from earlier kernels
     __syncthreads();
+    const int req = p.rows[r0].req;
 
     // Rows of this thread: A = lane/4, B = lane/4 + 8 of the warp's 16.
     const int ra = r0 + warp * 16 + (lane >> 2), rb = ra + 8;
     const bool va = ra < r_end, vb = rb < r_end;
     const int plen_a = va ? p.rows[ra].plen : 0, plen_b = vb ? p.rows[rb].plen : 0;
     atomicMax(&s_pmax, max(plen_a, plen_b));
-
-    // Q tile -> shared (swizzled); rows past the request's rows are zero.
-    for (int i = threadIdx.x; i < ROWS * HD / 8; i += 128) {
-        const int row = i / (HD / 8), c = i - row * (HD / 8);
-        uint4 v = make_uint4(0, 0, 0, 0);
-        if (r0 + row < r_end)
-            v = *reinterpret_cast<const uint4 *>(p.q + (size_t)(r0 + row) * H + h * HD + c * 8);
-        asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(swz(q_s, row, c)), "r"(v.x),
-                     "r"(v.y), "r"(v.z), "r"(v.w)
-                     : "memory");
-    }
     __syncthreads();
 
     // Key range of this split.
@@ -242,11 +234,31 @@ __global__ void __launch_bounds__(128)
             tma2d(vd + b * 8192, mv, b * 64, y, bar);
         }
     };
-    if (threadIdx.x == 0) {
-        asm volatile("prefetch.tensormap [%0];" ::"l"(mk) : "memory");
-        asm volatile("prefetch.tensormap [%0];" ::"l"(mv) : "memory");
+    // K/V tiles in flight first, then the Q tile (all its loads issued before
+    // the first shared-memory store); rows past the request's rows are zero.
+    if (threadIdx.x == 0)
         for (int i = 0; i < min(stages, ntiles); ++i) issue(i);
+    {
+        constexpr int QV = ROWS * HD / 8 / 128;       // 16-byte pieces per thread
+        uint4 qv[QV];
+#pragma unroll
+        for (int j = 0; j < QV; ++j) {
+            const int i = threadIdx.x + j * 128;
+            const int row = i / (HD / 8), c = i - row * (HD / 8);
+            qv[j] = r0 + row < r_end
+                        ? __ldg(reinterpret_cast<const uint4 *>(p.q + (size_t)(r0 + row) * H + h * HD + c * 8))
+                        : make_uint4(0, 0, 0, 0);
+        }
+#pragma unroll
+        for (int j = 0; j < QV; ++j) {
+            const int i = threadIdx.x + j * 128;
+            const int row = i / (HD / 8), c = i - row * (HD / 8);
+            asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(swz(q_s, row, c)), "r"(qv[j].x),
+                         "r"(qv[j].y), "r"(qv[j].z), "r"(qv[j].w)
+                         : "memory");
+        }
     }
+    __syncthreads();
 
     // Q fragments of the warp's 16 rows.
     uint32_t qf[HD / 16][4];
@@ -575,13 +587,15 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     lc.blockDim = dim3(128);
     lc.dynamicSmemBytes = smem;
     lc.stream = s;
-    cudaLaunchAttribute at[1];
+    cudaLaunchAttribute at[2];
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = 1;
     at[0].val.clusterDim.y = 1;
     at[0].val.clusterDim.z = tot;
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = at;
-    lc.numAttrs = 1;
+    lc.numAttrs = 2;
     cudaError_t e = a.hd == 128
                         ? cudaLaunchKernelEx(&lc, attn_tc_kernel<128>, *mkc, *mvc, *mkt, *mvt, tp)
                         : cudaLaunchKernelEx(&lc, attn_tc_kernel<64>, *mkc, *mvc, *mkt, *mvt, tp);

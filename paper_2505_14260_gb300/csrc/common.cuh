@@ -4,6 +4,7 @@
 #include <cuda_runtime.h>
 #include <cuda_bf16.h>
 #include <cstdint>
+#include <utility>
 
 namespace msd {
 
@@ -41,6 +42,32 @@ __device__ __forceinline__ void set_status(int *st, int code) {
 // its outputs (griddepcontrol.wait).
 __device__ __forceinline__ void allow_dependents() {
     asm volatile("griddepcontrol.launch_dependents;");
+}
+
+// Waits until the grids this one depends on have completed and their writes
+// are visible. Every kernel launched by launch_pdl calls it before its first
+// global memory access, so that completion stays transitive along the stream.
+__device__ __forceinline__ void wait_prior() {
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Launches `kernel` with programmatic stream serialization: its CTAs may be
+// scheduled while the previous kernel on `s` finishes (its launch latency
+// overlaps that kernel's tail); the kernel orders itself with wait_prior().
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                              cudaStream_t s, Args &&...args) {
+    cudaLaunchConfig_t lc = {};
+    lc.gridDim = grid;
+    lc.blockDim = block;
+    lc.dynamicSmemBytes = smem;
+    lc.stream = s;
+    cudaLaunchAttribute at[1];
+    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[0].val.programmaticStreamSerializationAllowed = 1;
+    lc.attrs = at;
+    lc.numAttrs = 1;
+    return cudaLaunchKernelEx(&lc, kernel, std::forward<Args>(args)...);
 }
 
 template <typename T> __device__ __forceinline__ float to_f(T v);

@@ -19,6 +19,7 @@ template <typename T>
 __global__ void __launch_bounds__(256) gemm_simt_kernel(const T *__restrict__ X, int ldx, int M,
                                                         int K, GemmW W, int O, float *__restrict__ Y,
                                                         int ldy, int epi) {
+    wait_prior();
     __shared__ float Ws[SG_BK][SG_BO + 1];
     __shared__ float Xs[SG_BK][SG_BM + 1];
     const int o0 = blockIdx.x * SG_BO, m0 = blockIdx.y * SG_BM;
@@ -72,7 +73,7 @@ void launch_gemm_simt(const T *X, int ldx, int M, int K, const GemmW &W, int O, 
                       int ldy, int epi, cudaStream_t s) {
     if (M <= 0 || O <= 0) return;
     dim3 grid((O + SG_BO - 1) / SG_BO, (M + SG_BM - 1) / SG_BM);
-    gemm_simt_kernel<T><<<grid, 256, 0, s>>>(X, ldx, M, K, W, O, Y, ldy, epi); note_launch();
+    launch_pdl(gemm_simt_kernel<T>, grid, 256, 0, s, X, ldx, M, K, W, O, Y, ldy, epi); note_launch();
 }
 
 template void launch_gemm_simt<float>(const float *, int, int, int, const GemmW &, int, float *,

@@ -19,6 +19,7 @@ __global__ void embed_rows_kernel(const T *__restrict__ E, const T *__restrict__
                                   const int *__restrict__ src, int H, float *__restrict__ x,
                                   T *__restrict__ emb_out, int V, int *status) {
     allow_dependents();
+    wait_prior();
     const int r = blockIdx.x;
     int s = src[r];
     const T *row;
@@ -42,7 +43,7 @@ template <typename T>
 void launch_embed_rows(const T *E, const T *vis, const int *src, int R, int H, float *x,
                        T *emb_out, int V, int *status, cudaStream_t s) {
     if (R <= 0) return;
-    embed_rows_kernel<T><<<R, 256, 0, s>>>(E, vis, src, H, x, emb_out, V, status); note_launch();
+    launch_pdl(embed_rows_kernel<T>, R, 256, 0, s, E, vis, src, H, x, emb_out, V, status); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -78,6 +79,7 @@ __global__ void __launch_bounds__(RMS_THREADS) rmsnorm_kernel(const float *__res
                                                               const T *__restrict__ g, int H,
                                                               float eps, T *__restrict__ out) {
     allow_dependents();
+    wait_prior();
     __shared__ float red[32];
     const int r = blockIdx.x, n4 = H >> 2;
     const float4 *xr = reinterpret_cast<const float4 *>(x + (size_t)r * H);
@@ -107,7 +109,7 @@ template <typename T>
 void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
                     cudaStream_t s) {
     if (R <= 0) return;
-    rmsnorm_kernel<T><<<R, RMS_THREADS, 0, s>>>(x, g, H, eps, out); note_launch();
+    launch_pdl(rmsnorm_kernel<T>, R, RMS_THREADS, 0, s, x, g, H, eps, out); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -116,6 +118,7 @@ void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
 template <typename T>
 __global__ void swiglu_kernel(const float *__restrict__ gu, int F, int glu, T *__restrict__ act) {
     allow_dependents();
+    wait_prior();
     const int r = blockIdx.y;
     const int ld = glu ? 128 * ((F + 63) / 64) : 2 * F;
     const float *row = gu + (size_t)r * ld;
@@ -131,7 +134,7 @@ template <typename T>
 void launch_swiglu(const float *gu, int R, int F, bool glu, T *act, cudaStream_t s) {
     if (R <= 0) return;
     dim3 grid((F + 255) / 256, R);
-    swiglu_kernel<T><<<grid, 256, 0, s>>>(gu, F, glu ? 1 : 0, act); note_launch();
+    launch_pdl(swiglu_kernel<T>, grid, 256, 0, s, gu, F, glu ? 1 : 0, act); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -143,6 +146,7 @@ __global__ void rope_kv_kernel(const float *__restrict__ qkv, const RowDesc *__r
                                T *__restrict__ q_out, T *__restrict__ kdst, T *__restrict__ vdst,
                                int slots, int *status) {
     allow_dependents();
+    wait_prior();
     const int r = blockIdx.x;
     const int H = nh * hd, half = hd >> 1;
     const RowDesc d = rows[r];
@@ -180,7 +184,7 @@ void launch_rope_kv(const float *qkv, const RowDesc *rows, int R, int nh, int hd
                     const float2 *rope_tab, int max_pos, T *q_out, T *kdst, T *vdst,
                     int slots, int *status, cudaStream_t s) {
     if (R <= 0) return;
-    rope_kv_kernel<T><<<R, 256, 0, s>>>(qkv, rows, nh, hd, rope_tab, max_pos, q_out, kdst,
+    launch_pdl(rope_kv_kernel<T>, R, 256, 0, s, qkv, rows, nh, hd, rope_tab, max_pos, q_out, kdst,
                                         vdst, slots, status); note_launch();
 }
 
@@ -228,6 +232,7 @@ __global__ void __launch_bounds__(TK_THREADS)
     topk_rows_kernel(const float *__restrict__ logits, int V, int k, int *__restrict__ ids,
                      float *__restrict__ logp, float *__restrict__ ws, int *__restrict__ counters) {
     allow_dependents();
+    wait_prior();
     extern __shared__ float sv[];
     __shared__ float rv[32];
     __shared__ int ri[32];
@@ -323,7 +328,7 @@ void launch_topk_logp(const float *logits, int R, int V, int k, int *ids, float 
     const int nc = topk_chunks(V);
     const int CH = (V + nc - 1) / nc;
     const size_t smem = sizeof(float) * std::max<size_t>(CH, (size_t)2 * nc * k);
-    topk_rows_kernel<<<dim3(nc, R), TK_THREADS, smem, s>>>(logits, V, k, ids, logp, sc.ws,
+    launch_pdl(topk_rows_kernel, dim3(nc, R), TK_THREADS, smem, s, logits, V, k, ids, logp, sc.ws,
                                                           sc.counters);
     note_launch();
 }
@@ -336,6 +341,7 @@ void launch_argmax(const float *logits, int R, int V, int *out, const TopkScratc
 // ---------------------------------------------------------------------------
 template <typename T>
 __global__ void convert_kernel(const float *__restrict__ x, T *__restrict__ y, long n) {
+    wait_prior();
     for (long i = blockIdx.x * (long)blockDim.x + threadIdx.x; i < n; i += (long)gridDim.x * blockDim.x)
         y[i] = from_f<T>(x[i]);
 }
@@ -345,14 +351,14 @@ void launch_convert(const float *x, T *y, long n, cudaStream_t s) {
     if (n <= 0) return;
     long blocks = (n + 255) / 256;
     if (blocks > 4096) blocks = 4096;
-    convert_kernel<T><<<(int)blocks, 256, 0, s>>>(x, y, n); note_launch();
+    launch_pdl(convert_kernel<T>, (int)blocks, 256, 0, s, x, y, n); note_launch();
 }
 
-__global__ void flag_status_kernel(int *status, int code) { set_status(status, code); }
+__global__ void flag_status_kernel(int *status, int code) { wait_prior(); set_status(status, code); }
 
 void launch_flag(int *status, int code, cudaStream_t s) {
     cudaGetLastError();
-    flag_status_kernel<<<1, 1, 0, s>>>(status, code);
+    launch_pdl(flag_status_kernel, 1, 1, 0, s, status, code);
     note_launch();
 }
 

@@ -17,6 +17,7 @@ __global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int 
                                      const T *__restrict__ E, int H, int D1, int V,
                                      T *__restrict__ xfc, RowDesc *__restrict__ rows, int *status) {
     allow_dependents();
+    wait_prior();
     const int r = blockIdx.x, b = r / D1, j = r - b * D1;
     const int L = seq_len[b], P = n_pend[b];
     const bool valid = j < P;
@@ -48,6 +49,7 @@ template <typename T>
 __global__ void root_gather_kernel(const float *__restrict__ x, const int *__restrict__ n_pend, int D1,
                                    int H, float *__restrict__ hhat_root, T *__restrict__ xr) {
     allow_dependents();
+    wait_prior();
     const int b = blockIdx.x;
     const int r = b * D1 + max(n_pend[b] - 1, 0);
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
@@ -62,6 +64,7 @@ template <typename T>
 __global__ void hhat_store_kernel(const float *__restrict__ x, const RowDesc *__restrict__ rows,
                                   int Td, int H, float *__restrict__ hhat_slot, T *__restrict__ xb) {
     allow_dependents();
+    wait_prior();
     const int r = blockIdx.x;
     const RowDesc d = rows[r];
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
@@ -109,6 +112,7 @@ __device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int tok, 
 template <typename T>
 __global__ void tree_init_kernel(DraftArgs<T> a) {
     allow_dependents();
+    wait_prior();
     const int b = blockIdx.y, j = blockIdx.x, k = a.k;
     __shared__ float sc[TREE_MAXK];
     __shared__ int front[TREE_MAXK];
@@ -146,6 +150,7 @@ __global__ void tree_init_kernel(DraftArgs<T> a) {
 template <typename T>
 __global__ void tree_step_kernel(DraftArgs<T> a, int d) {
     allow_dependents();
+    wait_prior();
     extern __shared__ float smem[];
     const int b = blockIdx.y, j = blockIdx.x, k = a.k, kk = k * k;
     const int base = k + (d - 2) * kk;
@@ -193,6 +198,7 @@ __global__ void tree_finalize_kernel(TreeOut t, const int *__restrict__ cand_tok
                                      const float *__restrict__ cand_score, int *__restrict__ node_of,
                                      const int *__restrict__ root, int C, int N, int *status) {
     allow_dependents();
+    wait_prior();
     extern __shared__ float ssc[];   // [C]
     const int b = blockIdx.x, W = (N + 63) / 64;
     const size_t cb = (size_t)b * C;
@@ -245,6 +251,7 @@ __global__ void verify_setup_kernel(TreeIn t, const int *__restrict__ seq_len,
                                     RowDesc *__restrict__ rows, int *__restrict__ src,
                                     uint64_t *__restrict__ vmask, int *status) {
     allow_dependents();
+    wait_prior();
     const int r = blockIdx.x * blockDim.x + threadIdx.x;
     if (r >= B * N) return;
     const int b = r / N, i = r - b * N, W = (N + 63) / 64;
@@ -292,6 +299,7 @@ __global__ void accept_kernel(TreeIn t, const int *__restrict__ argmax, int N, i
                               int *__restrict__ accept_len_out, int *__restrict__ bonus_out,
                               int *__restrict__ index_map_out) {
     allow_dependents();
+    wait_prior();
     const int b = blockIdx.x, lane = threadIdx.x, D1 = D + 1;
     const size_t nb = (size_t)b * N;
     const int n = t.n_nodes ? t.n_nodes[b] : N;
@@ -338,6 +346,7 @@ __global__ void compact_kv_kernel(const uint4 *__restrict__ tree_kv, uint4 *__re
                                   const int *__restrict__ acc_a, int B, int nh, int N, int S,
                                   int D1, int vec_per_row, int *status) {
     allow_dependents();
+    wait_prior();
     const int lkh = blockIdx.x, b = blockIdx.y;
     const int h = lkh % nh, lk = lkh / nh;           // lk = layer*2 + kv
     const int a = acc_a[b], L0 = acc_L0[b];
@@ -361,6 +370,7 @@ __global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ 
                               const int *__restrict__ acc_a, int N, int D1, int H,
                               T *__restrict__ pend_h) {
     allow_dependents();
+    wait_prior();
     const int b = blockIdx.x / D1, j = blockIdx.x - b * D1;
     if (j > acc_a[b]) return;
     const int node = acc_path[b * D1 + j];
@@ -377,6 +387,7 @@ template <typename T>
 __global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict__ emb,
                                      const int *__restrict__ src, int H) {
     allow_dependents();
+    wait_prior();
     const int r = blockIdx.x;
     if (src[r] >= 0) return;
     for (int c = threadIdx.x; c < H; c += blockDim.x)
@@ -389,6 +400,7 @@ template <typename T>
 __global__ void concat_next_kernel(const T *__restrict__ h, const T *__restrict__ emb, int H,
                                    T *__restrict__ xfc) {
     allow_dependents();
+    wait_prior();
     const int r = blockIdx.x;
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
         xfc[(size_t)r * 2 * H + c] = h[(size_t)r * H + c];
@@ -402,6 +414,7 @@ __global__ void prefill_finish_kernel(const int *__restrict__ argmax1, const T *
                                       int *__restrict__ n_pend, int *__restrict__ root,
                                       int *__restrict__ pend_next, T *__restrict__ pend_h,
                                       int *__restrict__ root_out) {
+    wait_prior();
     const int x = argmax1[0];
     if (threadIdx.x == 0) {
         seq_len[b] = L;
@@ -420,39 +433,39 @@ template <typename T>
 void launch_catchup_setup(const int *seq_len, const int *n_pend, const T *pend_h,
                           const int *pend_next, const T *E, int B, int H, int D1, int V, T *xfc,
                           RowDesc *rows, int *status, cudaStream_t s) {
-    catchup_setup_kernel<T><<<B * D1, 256, 0, s>>>(seq_len, n_pend, pend_h, pend_next, E, H, D1,
+    launch_pdl(catchup_setup_kernel<T>, B * D1, 256, 0, s, seq_len, n_pend, pend_h, pend_next, E, H, D1,
                                                    V, xfc, rows, status); note_launch();
 }
 
 template <typename T>
 void launch_root_gather(const float *x, const int *n_pend, int B, int D1, int H, float *hhat_root,
                         T *xr, cudaStream_t s) {
-    root_gather_kernel<T><<<B, 256, 0, s>>>(x, n_pend, D1, H, hhat_root, xr); note_launch();
+    launch_pdl(root_gather_kernel<T>, B, 256, 0, s, x, n_pend, D1, H, hhat_root, xr); note_launch();
 }
 
 template <typename T>
 void launch_hhat_store(const float *x, const RowDesc *rows, int R, int Td, int H,
                        float *hhat_slot, T *xb, cudaStream_t s) {
-    hhat_store_kernel<T><<<R, 256, 0, s>>>(x, rows, Td, H, hhat_slot, xb); note_launch();
+    launch_pdl(hhat_store_kernel<T>, R, 256, 0, s, x, rows, Td, H, hhat_slot, xb); note_launch();
 }
 
 template <typename T>
 void launch_tree_init(const DraftArgs<T> &a, int B, cudaStream_t s) {
-    tree_init_kernel<T><<<dim3(a.k, B), 256, 0, s>>>(a);
+    launch_pdl(tree_init_kernel<T>, dim3(a.k, B), 256, 0, s, a);
     note_launch();
 }
 
 template <typename T>
 void launch_tree_step(const DraftArgs<T> &a, int B, int d, cudaStream_t s) {
     const size_t sm = (size_t)a.k * a.k * sizeof(float) + (size_t)a.k * sizeof(int);
-    tree_step_kernel<T><<<dim3(a.k, B), 256, sm, s>>>(a, d);
+    launch_pdl(tree_step_kernel<T>, dim3(a.k, B), 256, sm, s, a, d);
     note_launch();
 }
 
 void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand_par,
                           const int *cand_depth, const float *cand_score, int *node_of,
                           const int *root, int B, int C, int N, int *status, cudaStream_t s) {
-    tree_finalize_kernel<<<B, 512, (size_t)C * sizeof(float), s>>>(
+    launch_pdl(tree_finalize_kernel, B, 512, (size_t)C * sizeof(float), s, 
         t, cand_tok, cand_par, cand_depth, cand_score, node_of, root, C, N, status); note_launch();
 }
 
@@ -460,7 +473,7 @@ void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, i
                          int V, RowDesc *rows, int *src, uint64_t *vmask, int *status,
                          cudaStream_t s) {
     const int R = B * N;
-    verify_setup_kernel<<<(R + 127) / 128, 128, 0, s>>>(t, seq_len, root, B, N, V, rows, src,
+    launch_pdl(verify_setup_kernel, (R + 127) / 128, 128, 0, s, t, seq_len, root, B, N, V, rows, src,
                                                           vmask, status); note_launch();
 }
 
@@ -468,7 +481,7 @@ void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int 
                    int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
                    int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,
                    cudaStream_t s) {
-    accept_kernel<<<B, 32, 0, s>>>(t, argmax, N, D, seq_len, n_pend, root, pend_next, acc_path,
+    launch_pdl(accept_kernel, B, 32, 0, s, t, argmax, N, D, seq_len, n_pend, root, pend_next, acc_path,
                                    acc_L0, acc_a, path_out, accept_len_out, bonus_out,
                                    index_map_out); note_launch();
 }
@@ -477,7 +490,7 @@ void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, co
                        const int *acc_a, int n_layers, int B, int nh, int N, int S, int D1,
                        int row_bytes, int *status, cudaStream_t s) {
     dim3 grid(n_layers * 2 * nh, B);
-    compact_kv_kernel<<<grid, 128, 0, s>>>(static_cast<const uint4 *>(tree_kv),
+    launch_pdl(compact_kv_kernel, grid, 128, 0, s, static_cast<const uint4 *>(tree_kv),
                                            static_cast<uint4 *>(cache), acc_path, acc_L0, acc_a,
                                            B, nh, N, S, D1, row_bytes / 16, status); note_launch();
 }
@@ -485,26 +498,26 @@ void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, co
 template <typename T>
 void launch_pend_h(const T *hT, const int *acc_path, const int *acc_a, int B, int N, int D1,
                    int H, T *pend_h, cudaStream_t s) {
-    pend_h_kernel<T><<<B * D1, 256, 0, s>>>(hT, acc_path, acc_a, N, D1, H, pend_h); note_launch();
+    launch_pdl(pend_h_kernel<T>, B * D1, 256, 0, s, hT, acc_path, acc_a, N, D1, H, pend_h); note_launch();
 }
 
 template <typename T>
 void launch_select_visual(float *x, const T *emb, const int *src, int R, int H, cudaStream_t s) {
     if (R <= 0) return;
-    select_visual_kernel<T><<<R, 256, 0, s>>>(x, emb, src, H); note_launch();
+    launch_pdl(select_visual_kernel<T>, R, 256, 0, s, x, emb, src, H); note_launch();
 }
 
 template <typename T>
 void launch_concat_next(const T *h, const T *emb, int R, int H, T *xfc, cudaStream_t s) {
     if (R <= 0) return;
-    concat_next_kernel<T><<<R, 256, 0, s>>>(h, emb, H, xfc); note_launch();
+    launch_pdl(concat_next_kernel<T>, R, 256, 0, s, h, emb, H, xfc); note_launch();
 }
 
 template <typename T>
 void launch_prefill_finish(const int *argmax1, const T *h_last, int b, int L, int D1, int H,
                            int *seq_len, int *n_pend, int *root, int *pend_next, T *pend_h,
                            int *root_out, cudaStream_t s) {
-    prefill_finish_kernel<T><<<1, 256, 0, s>>>(argmax1, h_last, b, L, D1, H, seq_len, n_pend,
+    launch_pdl(prefill_finish_kernel<T>, 1, 256, 0, s, argmax1, h_last, b, L, D1, H, seq_len, n_pend,
                                                root, pend_next, pend_h, root_out); note_launch();
 }
 
