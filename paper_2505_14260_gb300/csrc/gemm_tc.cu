@@ -767,201 +767,84 @@ __device__ __forceinline__ uint2 c_pack_bf16x4(float a, float b, float c, float 
     return make_uint2(*reinterpret_cast<const uint32_t *>(&lo), *reinterpret_cast<const uint32_t *>(&hi));
 }
 
-__device__ __forceinline__ void c_cluster_arrive() {
-    asm volatile("barrier.cluster.arrive.release;" ::: "memory");
-}
-
-__device__ __forceinline__ void c_cluster_wait() {
-    asm volatile("barrier.cluster.wait.acquire;" ::: "memory");
-}
-
-// float4 of rank q's partial at local offset `addr` (S == 1: this CTA's own).
-template <int S>
-__device__ __forceinline__ float4 c_part_ld4(uint32_t addr, int q) {
-    if constexpr (S == 1) return c_smem_ld4(addr);
-    else return c_dsmem_ld4(addr, (uint32_t)q);
-}
-
-// Plain split-K reduction (S > 1) of this CTA's slice of the tile: float4s of
-// 4 consecutive weight rows of one token, the S partials summed in rank order
-// (deterministic). Every remote load of a chunk is issued before the first is
-// used, and the thread arrives on the cluster barrier right after its last
-// remote read, so that the stores overlap the other CTAs' reads.
-template <int S>
-__device__ __forceinline__ void c_reduce_plain(const CkParams &p, uint32_t part_s, uint32_t rank,
-                                               bool ok, int o_base, int rows_here, int n0) {
-    constexpr int IT = 16 / S;
-    const bool add = p.epi == EPI_ADD;
-    const int n4 = p.BN * BM / 4;
-    const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
-    bool arrived = false;
-    for (int base = lo + threadIdx.x; base < hi; base += IT * C_THREADS) {
-        float4 v[IT][S];
-        float4 yi[IT];
-        float *yp[IT];
-        bool vec[IT], live[IT];
-#pragma unroll
-        for (int it = 0; it < IT; ++it) {
-            const int e4 = base + it * C_THREADS;
-            const int col = (e4 * 4) / BM, r4 = e4 * 4 - col * BM;
-            const int m = n0 + col;
-            live[it] = e4 < hi && ok && m < p.M;
-            yp[it] = p.Y + (size_t)m * p.ldy + o_base + r4;
-            vec[it] = r4 + 4 <= rows_here && ((reinterpret_cast<uintptr_t>(yp[it]) & 15u) == 0);
-            if (e4 < hi) {
-#pragma unroll
-                for (int q = 0; q < S; ++q) v[it][q] = c_part_ld4<S>(part_s + e4 * 16, q);
-            }
-            yi[it] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (add && live[it] && vec[it]) yi[it] = *reinterpret_cast<const float4 *>(yp[it]);
-        }
-        float4 acc[IT];
-#pragma unroll
-        for (int it = 0; it < IT; ++it) {
-            acc[it] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (base + it * C_THREADS < hi) {
-#pragma unroll
-                for (int q = 0; q < S; ++q) {
-                    acc[it].x += v[it][q].x; acc[it].y += v[it][q].y;
-                    acc[it].z += v[it][q].z; acc[it].w += v[it][q].w;
-                }
-            }
-        }
-        if (base + IT * C_THREADS >= hi) {
-            c_cluster_arrive();
-            arrived = true;
-        }
-#pragma unroll
-        for (int it = 0; it < IT; ++it) {
-            if (!live[it]) continue;
-            float *y = yp[it];
-            const int r4 = (base + it * C_THREADS) * 4 % BM;
-            if (vec[it]) {
-                float4 o = acc[it];
-                if (add) { o.x += yi[it].x; o.y += yi[it].y; o.z += yi[it].z; o.w += yi[it].w; }
-                *reinterpret_cast<float4 *>(y) = o;
-            } else {
-                const float vv[4] = {acc[it].x, acc[it].y, acc[it].z, acc[it].w};
-#pragma unroll
-                for (int e = 0; e < 4; ++e)
-                    if (r4 + e < rows_here) {
-                        if (add) y[e] = y[e] + vv[e];
-                        else y[e] = vv[e];
-                    }
-            }
-        }
-    }
-    if (!arrived) c_cluster_arrive();
-}
-
 // Paired epilogue over the tile's S partials ([BN][128] fp32 in each cluster
 // CTA's shared memory at part_s): element pairs (r, r + half) of one token,
 // with half = 64 for SwiGLU (gate row, up row) and hd/2 for RoPE (rotate-half
 // partners inside one head). This CTA takes its rank's share of the BN * 64
 // pairs, four consecutive rows at a time; the S partials are summed in rank
-// order, as in the plain reduction. With S > 1 the thread arrives on the
-// cluster barrier after its last remote read.
-template <int S>
+// order, as in the plain reduction.
 __device__ __forceinline__ void c_epilogue_paired(const CkParams &p, uint32_t part_s, uint32_t rank,
-                                                  bool ok, int seg, int wt, int row0, int n0,
+                                                  int S, bool ok, int seg, int wt, int row0, int n0,
                                                   int rows_here) {
-    constexpr int IT = S >= 8 ? 1 : 8 / S;
     const GemmFused &f = p.fx;
     const bool glu = p.epi == EPI_SWIGLU;
     const int half = glu ? 64 : (f.hd >> 1), hd = 2 * half;
     const int n4 = p.BN * 16;
     const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
-    bool arrived = false;
-    for (int base = lo + threadIdx.x; base < hi; base += IT * C_THREADS) {
-        float4 va[IT][S], vb[IT][S];
+    for (int e = lo + threadIdx.x; e < hi; e += C_THREADS) {
+        const int col = e >> 4, p4 = (e & 15) * 4;
+        const int r = (p4 / half) * hd + (p4 % half);
+        const uint32_t oa = part_s + (uint32_t)(col * BM + r) * 4u, ob = oa + (uint32_t)half * 4u;
+        float4 va[8], vb[8];
+        if (S == 1) {
+            va[0] = c_smem_ld4(oa);
+            vb[0] = c_smem_ld4(ob);
+        } else {
 #pragma unroll
-        for (int it = 0; it < IT; ++it) {
-            const int e = base + it * C_THREADS;
-            if (e >= hi) continue;
-            const int col = e >> 4, p4 = (e & 15) * 4;
-            const int r = (p4 / half) * hd + (p4 % half);
-            const uint32_t oa = part_s + (uint32_t)(col * BM + r) * 4u, ob = oa + (uint32_t)half * 4u;
-#pragma unroll
-            for (int q = 0; q < S; ++q) {
-                va[it][q] = c_part_ld4<S>(oa, q);
-                vb[it][q] = c_part_ld4<S>(ob, q);
-            }
-        }
-        float a[IT][4], b[IT][4];
-#pragma unroll
-        for (int it = 0; it < IT; ++it) {
-#pragma unroll
-            for (int t = 0; t < 4; ++t) a[it][t] = b[it][t] = 0.f;
-            if (base + it * C_THREADS >= hi) continue;
-#pragma unroll
-            for (int q = 0; q < S; ++q) {
-                a[it][0] += va[it][q].x; a[it][1] += va[it][q].y; a[it][2] += va[it][q].z; a[it][3] += va[it][q].w;
-                b[it][0] += vb[it][q].x; b[it][1] += vb[it][q].y; b[it][2] += vb[it][q].z; b[it][3] += vb[it][q].w;
-            }
-        }
-        if (S > 1 && base + IT * C_THREADS >= hi) {
-            c_cluster_arrive();
-            arrived = true;
-        }
-#pragma unroll
-        for (int it = 0; it < IT; ++it) {
-            const int e = base + it * C_THREADS;
-            if (e >= hi) continue;
-            const int col = e >> 4, p4 = (e & 15) * 4;
-            const int r = (p4 / half) * hd + (p4 % half);
-            const int m = n0 + col;
-            if (!ok || m >= p.M) continue;
-            if (glu) {
-                const int j = wt * 64 + p4;
-                if (j >= f.F) continue;                 // F % 4 == 0: whole groups
-                float o[4];
-#pragma unroll
-                for (int t = 0; t < 4; ++t) o[t] = a[it][t] / (1.f + __expf(-a[it][t])) * b[it][t];
-                *reinterpret_cast<uint2 *>(f.act + (size_t)m * f.F + j) = c_pack_bf16x4(o[0], o[1], o[2], o[3]);
-                continue;
-            }
-            if (r >= rows_here) continue;
-            const int o = row0 + r, h = o / hd, i = o - h * hd;
-            const RowDesc d = f.rows[m];
-            float x0[4], x1[4];
-#pragma unroll
-            for (int t = 0; t < 4; ++t) { x0[t] = a[it][t]; x1[t] = b[it][t]; }
-            if (seg < 2) {
-                int pos = d.pos;
-                if (pos < 0 || pos >= f.max_pos) {
-                    set_status(p.status, ST_RANGE);
-                    pos = 0;
+            for (int q = 0; q < 8; ++q)
+                if (q < S) {
+                    va[q] = c_dsmem_ld4(oa, q);
+                    vb[q] = c_dsmem_ld4(ob, q);
                 }
-                const float4 *cs = reinterpret_cast<const float4 *>(f.rope_tab + (size_t)pos * half + i);
-                const float4 c01 = cs[0], c23 = cs[1];
-                const float cx[4] = {c01.x, c01.z, c23.x, c23.z}, sy[4] = {c01.y, c01.w, c23.y, c23.w};
-#pragma unroll
-                for (int t = 0; t < 4; ++t) {
-                    x0[t] = a[it][t] * cx[t] - b[it][t] * sy[t];
-                    x1[t] = b[it][t] * cx[t] + a[it][t] * sy[t];
-                }
-            }
-            bf16 *dst;
-            if (seg == 0) {
-                dst = f.q_out + (size_t)m * (f.nh * hd) + o;
-            } else {
-                if (d.dst >= f.slots) set_status(p.status, ST_RANGE);
-                if (d.dst < 0 || d.dst >= f.slots) continue;
-                dst = (seg == 1 ? f.kdst : f.vdst) + ((size_t)(d.req * f.nh + h) * f.slots + d.dst) * hd + i;
-            }
-            *reinterpret_cast<uint2 *>(dst) = c_pack_bf16x4(x0[0], x0[1], x0[2], x0[3]);
-            *reinterpret_cast<uint2 *>(dst + half) = c_pack_bf16x4(x1[0], x1[1], x1[2], x1[3]);
         }
+        float a[4] = {0.f, 0.f, 0.f, 0.f}, b[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (q < S) {
+                a[0] += va[q].x; a[1] += va[q].y; a[2] += va[q].z; a[3] += va[q].w;
+                b[0] += vb[q].x; b[1] += vb[q].y; b[2] += vb[q].z; b[3] += vb[q].w;
+            }
+        const int m = n0 + col;
+        if (!ok || m >= p.M) continue;
+        if (glu) {
+            const int j = wt * 64 + p4;
+            if (j >= f.F) continue;                 // F % 4 == 0: whole groups
+            float o[4];
+#pragma unroll
+            for (int t = 0; t < 4; ++t) o[t] = a[t] / (1.f + __expf(-a[t])) * b[t];
+            *reinterpret_cast<uint2 *>(f.act + (size_t)m * f.F + j) = c_pack_bf16x4(o[0], o[1], o[2], o[3]);
+            continue;
+        }
+        if (r >= rows_here) continue;
+        const int o = row0 + r, h = o / hd, i = o - h * hd;
+        const RowDesc d = f.rows[m];
+        if (seg < 2) {
+            int pos = d.pos;
+            if (pos < 0 || pos >= f.max_pos) {
+                set_status(p.status, ST_RANGE);
+                pos = 0;
+            }
+            const float4 *cs = reinterpret_cast<const float4 *>(f.rope_tab + (size_t)pos * half + i);
+            const float4 c01 = cs[0], c23 = cs[1];
+            const float cx[4] = {c01.x, c01.z, c23.x, c23.z}, sy[4] = {c01.y, c01.w, c23.y, c23.w};
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+                const float x0 = a[t], x1 = b[t];
+                a[t] = x0 * cx[t] - x1 * sy[t];
+                b[t] = x1 * cx[t] + x0 * sy[t];
+            }
+        }
+        bf16 *dst;
+        if (seg == 0) {
+            dst = f.q_out + (size_t)m * (f.nh * hd) + o;
+        } else {
+            if (d.dst >= f.slots) set_status(p.status, ST_RANGE);
+            if (d.dst < 0 || d.dst >= f.slots) continue;
+            dst = (seg == 1 ? f.kdst : f.vdst) + ((size_t)(d.req * f.nh + h) * f.slots + d.dst) * hd + i;
+        }
+        *reinterpret_cast<uint2 *>(dst) = c_pack_bf16x4(a[0], a[1], a[2], a[3]);
+        *reinterpret_cast<uint2 *>(dst + half) = c_pack_bf16x4(b[0], b[1], b[2], b[3]);
     }
-    if (S > 1 && !arrived) c_cluster_arrive();
-}
-
-template <int S>
-__device__ __forceinline__ void c_epilogue_split(const CkParams &p, uint32_t part_s, uint32_t rank, bool paired,
-                                                 bool ok, int seg, int wt, int row0, int n0, int o_base,
-                                                 int rows_here) {
-    if (paired) c_epilogue_paired<S>(p, part_s, rank, ok, seg, wt, row0, n0, rows_here);
-    else if constexpr (S > 1) c_reduce_plain<S>(p, part_s, rank, ok, o_base, rows_here, n0);
 }
 
 __global__ void __launch_bounds__(C_THREADS)
@@ -1129,17 +1012,42 @@ __global__ void __launch_bounds__(C_THREADS)
         else __syncthreads();
         const uint32_t rank = S > 1 ? c_cluster_rank() : 0u;
         const uint32_t part_s = smem_u32(part);
-        switch (S) {
-            case 1: c_epilogue_split<1>(p, part_s, rank, paired, ok, seg, wt, row0, n0, o_base, rows_here); break;
-            case 2: c_epilogue_split<2>(p, part_s, rank, paired, ok, seg, wt, row0, n0, o_base, rows_here); break;
-            case 3: c_epilogue_split<3>(p, part_s, rank, paired, ok, seg, wt, row0, n0, o_base, rows_here); break;
-            case 4: c_epilogue_split<4>(p, part_s, rank, paired, ok, seg, wt, row0, n0, o_base, rows_here); break;
-            case 5: c_epilogue_split<5>(p, part_s, rank, paired, ok, seg, wt, row0, n0, o_base, rows_here); break;
-            case 6: c_epilogue_split<6>(p, part_s, rank, paired, ok, seg, wt, row0, n0, o_base, rows_here); break;
-            case 7: c_epilogue_split<7>(p, part_s, rank, paired, ok, seg, wt, row0, n0, o_base, rows_here); break;
-            default: c_epilogue_split<8>(p, part_s, rank, paired, ok, seg, wt, row0, n0, o_base, rows_here); break;
+        if (paired) c_epilogue_paired(p, part_s, rank, S, ok, seg, wt, row0, n0, rows_here);
+        // this CTA's slice of the tile, as float4 (4 consecutive weight rows of one token)
+        const int n4 = BN * BM / 4;
+        const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
+        for (int e4 = lo + threadIdx.x; !paired && e4 < hi; e4 += C_THREADS) {
+            float4 v[8];
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (q < S) v[q] = c_dsmem_ld4(part_s + e4 * 16, q);
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (q < S) {
+                    acc.x += v[q].x; acc.y += v[q].y; acc.z += v[q].z; acc.w += v[q].w;
+                }
+            const int col = (e4 * 4) / BM, r4 = e4 * 4 - col * BM;
+            const int m = n0 + col;
+            if (!ok || m >= p.M) continue;
+            float *y = p.Y + (size_t)m * p.ldy + o_base + r4;
+            if (r4 + 4 <= rows_here && ((reinterpret_cast<uintptr_t>(y) & 15u) == 0)) {
+                if (add) {
+                    const float4 yi = *reinterpret_cast<const float4 *>(y);
+                    acc.x += yi.x; acc.y += yi.y; acc.z += yi.z; acc.w += yi.w;
+                }
+                *reinterpret_cast<float4 *>(y) = acc;
+            } else {
+                const float vv[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (r4 + e < rows_here) {
+                        if (add) y[e] = y[e] + vv[e];
+                        else y[e] = vv[e];
+                    }
+            }
         }
-        if (S > 1) c_cluster_wait();      // partials stay readable until every CTA has read them
+        if (S > 1) c_cluster_sync();      // partials stay readable until every slice is done
     }
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
