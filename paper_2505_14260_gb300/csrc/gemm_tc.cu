@@ -730,6 +730,7 @@ struct CkParams {
     int ldy, epi;
     int *status;
     GemmFused fx;           // EPI_SWIGLU / EPI_ROPE_KV operands
+    GemmNorm nout, nin;     // folded RMSNorm: producer / consumer side (ss null: off)
 };
 
 __device__ __forceinline__ void c_cluster_sync() {
@@ -775,7 +776,7 @@ __device__ __forceinline__ uint2 c_pack_bf16x4(float a, float b, float c, float 
 // order, as in the plain reduction.
 __device__ __forceinline__ void c_epilogue_paired(const CkParams &p, uint32_t part_s, uint32_t rank,
                                                   int S, bool ok, int seg, int wt, int row0, int n0,
-                                                  int rows_here) {
+                                                  int rows_here, const float *rinv) {
     const GemmFused &f = p.fx;
     const bool glu = p.epi == EPI_SWIGLU;
     const int half = glu ? 64 : (f.hd >> 1), hd = 2 * half;
@@ -806,6 +807,14 @@ __device__ __forceinline__ void c_epilogue_paired(const CkParams &p, uint32_t pa
             }
         const int m = n0 + col;
         if (!ok || m >= p.M) continue;
+        if (rinv) {                                   // folded RMSNorm: the row's 1/rms
+            const float sc = rinv[col];
+#pragma unroll
+            for (int t = 0; t < 4; ++t) {
+                a[t] *= sc;
+                b[t] *= sc;
+            }
+        }
         if (glu) {
             const int j = wt * 64 + p4;
             if (j >= f.F) continue;                 // F % 4 == 0: whole groups
@@ -847,12 +856,76 @@ __device__ __forceinline__ void c_epilogue_paired(const CkParams &p, uint32_t pa
     }
 }
 
+// Producer side of a folded RMSNorm: this CTA's share of the tile's token
+// columns, one warp per column (lane = 4 consecutive weight rows): the S
+// partials summed in rank order, the residual added, then Y (fp32), xg =
+// bf16(y * g) and the column's sum of squares over the tile's rows (a warp
+// reduction in a fixed order) into ss[m][tile].
+__device__ __forceinline__ void c_reduce_norm(const CkParams &p, uint32_t part_s, uint32_t rank, int S,
+                                              bool ok, int tile, int o_base, int rows_here, int n0) {
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const bool add = p.epi == EPI_ADD;
+    const int c_lo = (int)((long long)rank * p.BN / S), c_hi = (int)((long long)(rank + 1) * p.BN / S);
+    const int r4 = lane * 4;
+    for (int c = c_lo + warp; c < c_hi; c += C_THREADS / 32) {
+        const uint32_t addr = part_s + (uint32_t)(c * BM + r4) * 4u;
+        float4 v[8];
+        if (S == 1) {
+            v[0] = c_smem_ld4(addr);
+        } else {
+#pragma unroll
+            for (int q = 0; q < 8; ++q)
+                if (q < S) v[q] = c_dsmem_ld4(addr, q);
+        }
+        float a[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll
+        for (int q = 0; q < 8; ++q)
+            if (q < S) {
+                a[0] += v[q].x; a[1] += v[q].y; a[2] += v[q].z; a[3] += v[q].w;
+            }
+        const int m = n0 + c;
+        const bool live = ok && m < p.M;                  // warp-uniform
+        float ss = 0.f;
+        if (live) {
+            float *y = p.Y + (size_t)m * p.ldy + o_base + r4;
+            bf16 *xg = p.nout.xg + (size_t)m * p.ldy + o_base + r4;
+            const bf16 *g = p.nout.g + o_base + r4;
+            if (r4 + 4 <= rows_here) {
+                if (add) {
+                    const float4 yi = *reinterpret_cast<const float4 *>(y);
+                    a[0] += yi.x; a[1] += yi.y; a[2] += yi.z; a[3] += yi.w;
+                }
+                *reinterpret_cast<float4 *>(y) = make_float4(a[0], a[1], a[2], a[3]);
+                const uint2 gw = *reinterpret_cast<const uint2 *>(g);
+                const __nv_bfloat162 g01 = *reinterpret_cast<const __nv_bfloat162 *>(&gw.x);
+                const __nv_bfloat162 g23 = *reinterpret_cast<const __nv_bfloat162 *>(&gw.y);
+                *reinterpret_cast<uint2 *>(xg) =
+                    c_pack_bf16x4(a[0] * __low2float(g01), a[1] * __high2float(g01),
+                                  a[2] * __low2float(g23), a[3] * __high2float(g23));
+                ss = a[0] * a[0] + a[1] * a[1] + a[2] * a[2] + a[3] * a[3];
+            } else {
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (r4 + e < rows_here) {
+                        const float ye = add ? y[e] + a[e] : a[e];
+                        y[e] = ye;
+                        xg[e] = __float2bfloat16_rn(ye * __bfloat162float(g[e]));
+                        ss += ye * ye;
+                    }
+            }
+        }
+        ss = warp_sum(ss);
+        if (live && lane == 0) p.nout.ss[(size_t)m * p.nout.ld + tile] = ss;
+    }
+}
+
 __global__ void __launch_bounds__(C_THREADS)
     gemm_cluster_kernel(const __grid_constant__ CUtensorMap mx, const CkParams p) {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t bars[2 * C_STAGES + 1];
     __shared__ uint32_t tmem_base;
     __shared__ volatile int abort_flag;
+    __shared__ float s_rinv[128];     // folded RMSNorm (consumer): 1/rms of each token column
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int wt = blockIdx.x, seg = 0;
@@ -956,6 +1029,15 @@ __global__ void __launch_bounds__(C_THREADS)
         __syncwarp();
     } else {
         pdl_wait();
+        // idle during the main loop: the row scales of a folded RMSNorm
+        if (p.nin.ss)
+            for (int t = threadIdx.x - 64; t < p.BN; t += C_THREADS - 64) {
+                const int m = n0 + t;
+                float sum = 0.f;
+                if (m < p.M)
+                    for (int j = 0; j < p.nin.parts; ++j) sum += p.nin.ss[(size_t)m * p.nin.ld + j];
+                s_rinv[t] = rsqrtf(sum / (float)p.nin.H + p.nin.eps);
+            }
     }
 
     // ---- epilogue: all 4 warps, TMEM lane quarter = warp -------------------
@@ -968,7 +1050,8 @@ __global__ void __launch_bounds__(C_THREADS)
     const int rows_here = p.seg_rows[seg] - row0;           // valid weight rows in this tile
     const int o_base = p.seg_out[seg] + row0;
     const bool paired = p.epi >= EPI_SWIGLU;
-    if (S == 1 && !paired) {
+    const bool norm_out = p.nout.ss != nullptr;
+    if (S == 1 && !paired && !norm_out) {
         for (int g0 = 0; g0 < BN; g0 += 32) {
             const int gw = min(32, BN - g0);
             uint32_t r[32];
@@ -1012,11 +1095,13 @@ __global__ void __launch_bounds__(C_THREADS)
         else __syncthreads();
         const uint32_t rank = S > 1 ? c_cluster_rank() : 0u;
         const uint32_t part_s = smem_u32(part);
-        if (paired) c_epilogue_paired(p, part_s, rank, S, ok, seg, wt, row0, n0, rows_here);
+        if (paired) c_epilogue_paired(p, part_s, rank, S, ok, seg, wt, row0, n0, rows_here,
+                                      p.nin.ss ? s_rinv : nullptr);
+        else if (norm_out) c_reduce_norm(p, part_s, rank, S, ok, wt, o_base, rows_here, n0);
         // this CTA's slice of the tile, as float4 (4 consecutive weight rows of one token)
         const int n4 = BN * BM / 4;
         const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
-        for (int e4 = lo + threadIdx.x; !paired && e4 < hi; e4 += C_THREADS) {
+        for (int e4 = lo + threadIdx.x; !paired && !norm_out && e4 < hi; e4 += C_THREADS) {
             float4 v[8];
 #pragma unroll
             for (int q = 0; q < 8; ++q)
@@ -1239,10 +1324,13 @@ void gemm_pack_glu(const void *gate, const void *up, int F, int K, void *dst, cu
 // so that tiles * s fills two CTAs per SM once, s <= 8 and >= 2 K-blocks each.
 static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W,
                          int tiles, int BN, int kblocks, float *Y, int ldy, int epi, int *status,
-                         cudaStream_t s, int O, const GemmFused *fx = nullptr) {
+                         cudaStream_t s, int O, const GemmFused *fx = nullptr,
+                         const GemmNorm *nout = nullptr, const GemmNorm *nin = nullptr) {
     CkParams ck;
     memset(&ck, 0, sizeof ck);
     if (fx) ck.fx = *fx;
+    if (nout) ck.nout = *nout;
+    if (nin) ck.nin = *nin;
     ck.n_seg = W.nseg;
     int out_off = 0;
     for (int i = 0; i < W.nseg; ++i) {
@@ -1316,7 +1404,7 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
 }
 
 bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
-                     const GemmFused &fx, int *status, cudaStream_t s) {
+                     const GemmFused &fx, int *status, cudaStream_t s, const GemmNorm *norm_in) {
     if (M <= 0 || M > 128 || !W.packed || W.nseg < 1) return false;
     if (fx.epi == EPI_SWIGLU && (W.nseg != 1 || W.rows[0] != glu_rows(fx.F) || fx.F % 4)) return false;
     if (fx.epi == EPI_ROPE_KV &&
@@ -1327,13 +1415,19 @@ bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const Ge
     int tiles = 0;
     for (int i = 0; i < W.nseg; ++i) tiles += (W.rows[i] + BM - 1) / BM;
     const int BN = ((M + 15) / 16) * 16;
-    gemm_cluster(p, X, ldx, M, K, W, tiles, BN, (K + BK - 1) / BK, nullptr, 0, fx.epi, status, s, O, &fx);
+    if (norm_in && (!norm_in->ss || norm_in->parts <= 0 || norm_in->parts > norm_in->ld || BN > 128))
+        return false;
+    gemm_cluster(p, X, ldx, M, K, W, tiles, BN, (K + BK - 1) / BK, nullptr, 0, fx.epi, status, s, O, &fx,
+                 nullptr, norm_in);
     return true;
 }
 
-void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
-               int ldy, int epi, int *status, cudaStream_t s) {
-    if (M <= 0 || O <= 0) return;
+bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
+               int ldy, int epi, int *status, cudaStream_t s, const GemmNorm *norm_out) {
+    if (M <= 0 || O <= 0) return true;
+    if (norm_out && (M > 128 || !W.packed || W.nseg != 1 || !norm_out->ss || !norm_out->xg || !norm_out->g ||
+                     (O + BM - 1) / BM > norm_out->ld || O % 4 || ldy % 4))
+        return false;
     PkParams pk;
     memset(&pk, 0, sizeof pk);
     pk.n_seg = W.nseg;
@@ -1350,8 +1444,8 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     BN = ((BN + 15) / 16) * 16;
     const int kblocks = (K + BK - 1) / BK;
     if (M <= 128 && W.packed) {
-        gemm_cluster(p, X, ldx, M, K, W, tiles, BN, kblocks, Y, ldy, epi, status, s, O);
-        return;
+        gemm_cluster(p, X, ldx, M, K, W, tiles, BN, kblocks, Y, ldy, epi, status, s, O, nullptr, norm_out);
+        return true;
     }
     const uint32_t stage_bytes = A_BYTES + (uint32_t)BN * BK * 2;
     // five stages measured best on the decode shapes (deeper rings were slower)
@@ -1372,7 +1466,7 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     if (ws_need > WS_BYTES || tiles_total > N_COUNTERS) {
         flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
         fprintf(stderr, "msd: GEMM shape M=%d K=%d O=%d exceeds the workspace\n", M, K, O);
-        return;
+        return true;
     }
     int acc = 32;
     while (acc < BN) acc <<= 1;
@@ -1397,10 +1491,10 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     if (!W.packed) {
         flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
         fprintf(stderr, "msd: GEMM weights were not packed\n");
-        return;
+        return true;
     }
     const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
-    if (!mx) return;
+    if (!mx) return true;
     if (!p->smem_set) {
         cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              200 * 1024 + 1024);
@@ -1440,6 +1534,7 @@ void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
         p->prof_wbytes += wb;
         p->prof_bytes += wb + (double)M * K * 2.0 + (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
     }
+    return true;
 }
 
 }  // namespace msd

@@ -6,6 +6,7 @@
 namespace msd {
 
 struct GemmPlan;
+struct GemmNorm;
 
 // Host-side plan: split-K workspace, tile counters, tensor-map cache.
 bool gemm_plan_create(GemmPlan **out, int max_rows, int hidden, int ffn, int vocab);
@@ -13,8 +14,11 @@ void gemm_plan_destroy(GemmPlan *p);
 
 // Y[m][o] (=|+=) sum_k X[m][k] W[o][k]; X, W bf16 (K contiguous, rows 16-byte
 // aligned), Y fp32. Weight tiles fill the MMA's M = 128 side, tokens its N side.
-void gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
-               int ldy, int epi, int *status, cudaStream_t s);
+// norm_out (nullable, decode shapes M <= 128 with packed W only): the
+// producer side of a folded RMSNorm (GemmNorm below); returns false (nothing
+// launched) when it is given for a shape off the decode path.
+bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
+               int ldy, int epi, int *status, cudaStream_t s, const GemmNorm *norm_out = nullptr);
 
 // Pre-packed weights: the segments' 128-row x 64-column blocks, tile-major then
 // K-block, each block stored exactly as the MMA reads it from shared memory
@@ -50,10 +54,27 @@ struct GemmFused {
     bf16 *q_out, *kdst, *vdst;
     int slots, nh, hd;
 };
+// RMSNorm folded into a pair of decode GEMMs (the norm's per-row scale
+// commutes with the projection that follows it):
+//   producer (an H-output GEMM, EPI_STORE / EPI_ADD): besides Y = x, writes
+//     xg[m][o] = bf16(x[m][o] * g[o]) and ss[m][tile] = sum over the tile's 128
+//     rows of x[m][o]^2 (fixed order), ld = row stride of ss;
+//   consumer (EPI_ROPE_KV / EPI_SWIGLU on X = xg): scales its accumulator row m
+//     by 1 / sqrt(sum_{j < parts} ss[m][j] / H + eps) (summed in j order) before
+//     the rotation or the SwiGLU.
+struct GemmNorm {
+    float *ss;
+    int ld;
+    bf16 *xg;
+    const bf16 *g;
+    int parts, H;
+    float eps;
+};
+
 // Runs the fused GEMM and returns true when the shape takes the decode path;
 // returns false (nothing launched) otherwise.
 bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
-                     const GemmFused &fx, int *status, cudaStream_t s);
+                     const GemmFused &fx, int *status, cudaStream_t s, const GemmNorm *norm_in = nullptr);
 
 // Profiling: while enabled, every launch is bracketed by CUDA events on its
 // stream; gemm_profile_read synchronises on them and returns the launches,

@@ -35,6 +35,8 @@ struct msd_ctx {
     int *seq_len = nullptr, *n_pend = nullptr, *root = nullptr, *pend_next = nullptr;
     void *pend_h = nullptr;
     float *x = nullptr, *qkv = nullptr, *gu = nullptr, *logits = nullptr;
+    float *ss_part = nullptr;   // folded RMSNorm: per-tile sums of squares [Rmax][ss_ld]
+    int ss_ld = 0;
     void *xn = nullptr, *q = nullptr, *attn = nullptr, *act = nullptr, *xfc = nullptr, *xr = nullptr;
     int *argmax_tmp = nullptr;
     RowDesc *rows = nullptr;
@@ -203,7 +205,8 @@ int max_L_bound(const msd_ctx *c) {
 // with the rotation and placement in its epilogue.
 template <typename T>
 void qkv_rope(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int R,
-              const RowDesc *rows, T *kdst, T *vdst, int dst_slots, cudaStream_t s) {
+              const RowDesc *rows, T *kdst, T *vdst, int dst_slots, cudaStream_t s,
+              const GemmNorm *norm_in = nullptr) {
     const int H = c->H;
     GemmW wqkv = {{lw.wq, lw.wk, lw.wv}, {H, H, H}, 3, lp.qkv};
     if constexpr (std::is_same<T, bf16>::value) {
@@ -220,7 +223,7 @@ void qkv_rope(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int
         fx.nh = c->nh;
         fx.hd = c->hd;
         if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), H, R, H, wqkv, 3 * H, fx,
-                            c->status, s))
+                            c->status, s, norm_in))
             return;
     }
     gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wqkv, 3 * H, c->qkv, 3 * H, EPI_STORE, s);
@@ -232,7 +235,7 @@ void qkv_rope(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int
 // decode shapes apply the SwiGLU in the GEMM's epilogue.
 template <typename T>
 void gate_up_swiglu(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int R,
-                    cudaStream_t s) {
+                    cudaStream_t s, const GemmNorm *norm_in = nullptr) {
     const int H = c->H, F = c->F;
     if constexpr (std::is_same<T, bf16>::value) {
         const int O = glu_rows(F);
@@ -242,7 +245,8 @@ void gate_up_swiglu(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &l
         fx.epi = EPI_SWIGLU;
         fx.act = static_cast<bf16 *>(c->act);
         fx.F = F;
-        if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), H, R, H, wgu, O, fx, c->status, s))
+        if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), H, R, H, wgu, O, fx, c->status, s,
+                            norm_in))
             return;
         gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wgu, O, c->gu, O, EPI_STORE, s);
         launch_swiglu<T>(c->gu, R, F, true, static_cast<T *>(c->act), s);
@@ -253,19 +257,42 @@ void gate_up_swiglu(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &l
     }
 }
 
+// Folded RMSNorm (bf16 decode shapes with packed weights): the GEMM that
+// writes the residual stream also writes bf16(x * g) into c->xn and per-tile
+// sums of squares into c->ss_part; the next projection scales its rows by
+// 1/rms in its epilogue. Elsewhere the RMSNorm kernel runs.
+bool folds(const msd_ctx *c, int R, const void *packed) {
+    return c->esz == 2 && R <= 128 && packed != nullptr;
+}
+
+GemmNorm norm_out(msd_ctx *c, const void *g) {
+    return GemmNorm{c->ss_part, c->ss_ld, static_cast<bf16 *>(c->xn), static_cast<const bf16 *>(g),
+                    0, c->H, c->cfg.rms_eps};
+}
+
+GemmNorm norm_in(msd_ctx *c) {
+    return GemmNorm{c->ss_part, c->ss_ld, nullptr, nullptr, c->ss_ld, c->H, c->cfg.rms_eps};
+}
+
 // One pre-norm decoder layer over R rows (target or draft). Rows come in
 // blocks of rows_per_req per request; every row attends to at most p_bound
-// cache positions.
+// cache positions. in_folded: the layer's input norm was folded into the GEMM
+// that produced x; out_norm_g (nullable): the next layer's input-norm gain,
+// to fold into this layer's last GEMM. Returns whether it did.
 template <typename T>
-void run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int R,
+bool run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int R,
                const RowDesc *rows, T *kdst, T *vdst, int dst_slots, const T *ck, const T *cv,
                int cslots, const T *tk, const T *tv, int tslots, const uint64_t *mask, int mw,
-               int rows_per_req, int p_bound, cudaStream_t s) {
+               int rows_per_req, int p_bound, cudaStream_t s, bool in_folded = false,
+               const void *out_norm_g = nullptr) {
     const int H = c->H, F = c->F;
     const float eps = c->cfg.rms_eps;
-    launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.attn_norm), R, H, eps,
-                      static_cast<T *>(c->xn), s);
-    qkv_rope<T>(c, lw, lp, R, rows, kdst, vdst, dst_slots, s);
+    const bool fold = folds(c, R, lp.o) && lp.qkv && lp.gu && lp.down;
+    const GemmNorm nin = norm_in(c);
+    if (!(fold && in_folded))
+        launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.attn_norm), R, H, eps,
+                          static_cast<T *>(c->xn), s);
+    qkv_rope<T>(c, lw, lp, R, rows, kdst, vdst, dst_slots, s, fold && in_folded ? &nin : nullptr);
     AttnArgs<T> a;
     a.q = static_cast<const T *>(c->q);
     a.rows = rows;
@@ -284,16 +311,50 @@ void run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, in
     a.out = static_cast<T *>(c->attn);
     attention<T>(c, a, rows_per_req, p_bound, s);
     GemmW wo = {{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1, lp.o};
+    GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, lp.down};
+    if constexpr (std::is_same<T, bf16>::value) {
+        if (fold) {
+            const GemmNorm no = norm_out(c, lw.mlp_norm);
+            gemm_bf16(c->gplan, static_cast<const bf16 *>(c->attn), H, R, H, wo, H, c->x, H, EPI_ADD,
+                      c->status, s, &no);
+            gate_up_swiglu<T>(c, lw, lp, R, s, &nin);
+            if (out_norm_g) {
+                const GemmNorm nd = norm_out(c, out_norm_g);
+                gemm_bf16(c->gplan, static_cast<const bf16 *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD,
+                          c->status, s, &nd);
+                return true;
+            }
+            gemm<T>(c, static_cast<const T *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD, s);
+            return false;
+        }
+    }
     gemm<T>(c, static_cast<const T *>(c->attn), H, R, H, wo, H, c->x, H, EPI_ADD, s);
     launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.mlp_norm), R, H, eps,
                       static_cast<T *>(c->xn), s);
     gate_up_swiglu<T>(c, lw, lp, R, s);
-    GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, lp.down};
     gemm<T>(c, static_cast<const T *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD, s);
+    return false;
 }
 
 GemmW one(const void *w, int rows, const void *packed = nullptr) {
     return GemmW{{w, nullptr, nullptr}, {rows, 0, 0}, 1, packed};
+}
+
+// x = f_down(xfc) for R draft rows; with a folded norm also the draft layer's
+// input norm. Returns whether it folded.
+template <typename T>
+bool draft_fc(msd_ctx *c, int R, cudaStream_t s) {
+    const int H = c->H;
+    const GemmW W = one(c->w.draft_fc, H, c->pk_fc);
+    if constexpr (std::is_same<T, bf16>::value) {
+        if (folds(c, R, c->pk_fc) && c->dpack.o) {
+            const GemmNorm no = norm_out(c, c->w.draft.attn_norm);
+            return gemm_bf16(c->gplan, static_cast<const bf16 *>(c->xfc), 2 * H, R, 2 * H, W, H, c->x, H,
+                             EPI_STORE, c->status, s, &no);
+        }
+    }
+    gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, R, 2 * H, W, H, c->x, H, EPI_STORE, s);
+    return false;
 }
 
 // ---------------------------------------------------------------------------
@@ -425,11 +486,10 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
     const int R1 = B * D1;
     launch_catchup_setup<T>(c->seq_len, c->n_pend, static_cast<const T *>(c->pend_h), c->pend_next,
                             E, B, H, D1, V, static_cast<T *>(c->xfc), c->rows, c->status, s);
-    gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, R1, 2 * H, one(c->w.draft_fc, H, c->pk_fc), H, c->x, H,
-            EPI_STORE, s);
+    bool folded = draft_fc<T>(c, R1, s);
     const int pb = max_L_bound(c);
     run_layer<T>(c, c->w.draft, c->dpack, R1, c->rows, dK, dV, S, dK, dV, S, nullptr, nullptr, 0, nullptr, 0,
-                 D1, pb, s);
+                 D1, pb, s, folded);
     launch_root_gather<T>(c->x, c->n_pend, B, D1, H, c->hhat_root, static_cast<T *>(c->xr), s);
     gemm<T>(c, static_cast<const T *>(c->xr), H, B, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V,
             EPI_STORE, s);
@@ -441,10 +501,9 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
     // passes 2..D: expand the frontier
     const int Rk = B * k;
     for (int d = 2; d <= c->D; ++d) {
-        gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, Rk, 2 * H, one(c->w.draft_fc, H, c->pk_fc), H,
-                c->x, H, EPI_STORE, s);
+        folded = draft_fc<T>(c, Rk, s);
         run_layer<T>(c, c->w.draft, c->dpack, Rk, c->rows, tK, tV, c->Td, dK, dV, S, tK, tV, c->Td,
-                     c->row_mask, c->Wd, k, pb, s);
+                     c->row_mask, c->Wd, k, pb, s, folded);
         launch_hhat_store<T>(c->x, c->rows, Rk, c->Td, H, c->hhat_slot, static_cast<T *>(c->xr), s);
         gemm<T>(c, static_cast<const T *>(c->xr), H, Rk, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V,
                 EPI_STORE, s);
@@ -471,11 +530,13 @@ msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, fl
     launch_verify_setup(t, c->seq_len, c->root, B, N, V, c->rows, c->src, c->vmask, c->status, s);
     launch_embed_rows<T>(static_cast<const T *>(c->w.embed), nullptr, c->src, R, H, c->x, nullptr,
                          V, c->status, s);
+    bool folded = false;
     for (int l = 0; l < c->NL; ++l) {
         T *K = tkv<T>(c, c->target_kv, l, 0, c->S), *Vv = tkv<T>(c, c->target_kv, l, 1, c->S);
         T *tK = tkv<T>(c, c->tree_kv, l, 0, N), *tV = tkv<T>(c, c->tree_kv, l, 1, N);
-        run_layer<T>(c, c->layers[l], c->lpack[l], R, c->rows, tK, tV, N, K, Vv, c->S, tK, tV, N, c->vmask, c->W,
-                     N, pb, s);
+        const void *next_g = l + 1 < c->NL ? c->layers[l + 1].attn_norm : nullptr;
+        folded = run_layer<T>(c, c->layers[l], c->lpack[l], R, c->rows, tK, tV, N, K, Vv, c->S, tK, tV, N,
+                              c->vmask, c->W, N, pb, s, folded, next_g);
     }
     launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), R, H, c->cfg.rms_eps,
                       static_cast<T *>(c->hT), s);
@@ -646,6 +707,8 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     ok &= dalloc(c, &c->qkv, R * 3 * H * 4);
     ok &= dalloc(c, &c->q, R * H * e);
     ok &= dalloc(c, &c->attn, R * H * e);
+    c->ss_ld = (H + 127) / 128;
+    ok &= dalloc(c, &c->ss_part, R * (size_t)c->ss_ld * 4);
     ok &= dalloc(c, &c->gu, R * std::max<size_t>(2 * F, glu_rows(c->F)) * 4);
     ok &= dalloc(c, &c->act, R * F * e);
     ok &= dalloc(c, &c->xfc, R * 2 * H * e);
