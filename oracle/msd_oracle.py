@@ -150,26 +150,35 @@ def attend(q, cache_k, cache_v, prefix_len, tree_k, tree_v, tree_vis,
            n_heads, head_dim):
     """Softmax attention of each query row over the keys it may see.
 
-    Row r sees cache rows [0, prefix_len[r]) followed by the tree rows j with
-    tree_vis[r, j] true (in index order). Keys and values are [rows, H].
+    Row r sees cache rows [0, prefix_len[r]) and the tree rows j with
+    tree_vis[r, j] true. Keys and values are [rows, H]. Written as masked
+    attention: the scores of a block of rows against every key, the keys a row
+    may not see set to -inf (weight exactly 0 after the softmax), then the
+    weighted sum of the values.
     """
     R = q.shape[0]
-    out = np.zeros((R, n_heads * head_dim), F64)
+    H = n_heads * head_dim
+    keys = [np.asarray(cache_k, F64).reshape(-1, H)]
+    vals = [np.asarray(cache_v, F64).reshape(-1, H)]
+    C = keys[0].shape[0]
+    has_tree = tree_k is not None and tree_k.shape[0] > 0
+    if has_tree:
+        keys.append(np.asarray(tree_k, F64).reshape(-1, H))
+        vals.append(np.asarray(tree_v, F64).reshape(-1, H))
+    K = np.concatenate(keys, axis=0).reshape(-1, n_heads, head_dim).transpose(1, 0, 2)   # [h, T, d]
+    V = np.concatenate(vals, axis=0).reshape(-1, n_heads, head_dim).transpose(1, 0, 2)
     scale = 1.0 / np.sqrt(head_dim)
-    for r in range(R):
-        P = int(prefix_len[r])
-        ks = [np.asarray(cache_k[:P], F64)]
-        vs = [np.asarray(cache_v[:P], F64)]
-        if tree_k is not None and tree_k.shape[0] > 0:
-            sel = np.flatnonzero(tree_vis[r])
-            ks.append(np.asarray(tree_k[sel], F64))
-            vs.append(np.asarray(tree_v[sel], F64))
-        K = np.concatenate(ks, axis=0).reshape(-1, n_heads, head_dim)
-        V = np.concatenate(vs, axis=0).reshape(-1, n_heads, head_dim)
-        qh = q[r].reshape(n_heads, head_dim)
-        s = np.einsum("hd,thd->ht", qh, K) * scale
+    out = np.zeros((R, H), F64)
+    for r0 in range(0, R, 128):
+        r1 = min(R, r0 + 128)
+        qh = np.asarray(q[r0:r1], F64).reshape(-1, n_heads, head_dim).transpose(1, 0, 2)  # [h, n, d]
+        s = np.matmul(qh, K.transpose(0, 2, 1)) * scale                                  # [h, n, T]
+        vis = np.arange(C)[None, :] < np.asarray(prefix_len[r0:r1])[:, None]              # [n, C]
+        if has_tree:
+            vis = np.concatenate([vis, np.asarray(tree_vis[r0:r1], bool)], axis=1)
+        s = np.where(vis[None], s, -np.inf)
         p = softmax(s)
-        out[r] = np.einsum("ht,thd->hd", p, V).reshape(-1)
+        out[r0:r1] = np.matmul(p, V).transpose(1, 0, 2).reshape(r1 - r0, H)
     return out
 
 
