@@ -13,113 +13,24 @@ import torch
 
 from oracle import msd_oracle as O
 from paper_2505_14260_gb300 import msd, synth
-from tests.gpu_support import (KV_REL_L2, TOL, assert_close, open_engine, plant,
-                               record_buffers, rel_l2, top2_margin, tree_numpy)
+from tests.gpu_support import TOL, open_engine, plant, tree_numpy
 from tests.oracle_support import oracle_model, prompt_numpy
+from tests.parity_support import run_parity
 
 pytestmark = pytest.mark.gpu
-
-
-def _kv_compare(eng, st, wl, b, L, dtype, what):
-    s = eng.state()
-    nh, hd = wl.n_heads, wl.head_dim
-    for l in range(wl.n_layers):
-        for kv, ref in ((0, st.K[l]), (1, st.V[l])):
-            g = s["target_kv"][l, kv, b, :, :L, :].float().cpu().numpy()      # [nh, L, hd]
-            r = np.asarray(ref[:L]).reshape(L, nh, hd).transpose(1, 0, 2)
-            assert rel_l2(g, r) <= KV_REL_L2[dtype], f"{what} layer {l} kv {kv}: {rel_l2(g, r)}"
-    Ld = st.dK.shape[0]
-    for kv, ref in ((0, st.dK), (1, st.dV)):
-        g = s["draft_kv"][kv, b, :, :Ld, :].float().cpu().numpy()
-        r = np.asarray(ref).reshape(Ld, nh, hd).transpose(1, 0, 2)
-        assert rel_l2(g, r) <= KV_REL_L2[dtype], f"{what} draft kv {kv}: {rel_l2(g, r)}"
 
 
 @pytest.mark.parametrize("dtype,long_prompt", [("f32", False), ("bf16", False), ("bf16", True)],
                          ids=["f32", "bf16", "bf16-long-prompt"])
 def test_tiny_all_steps_match_oracle(dtype, long_prompt):
-    """The long prompt (364 positions) takes the prefill through the GEMM's
-    many-row path (separate RoPE and SwiGLU kernels); the short one and every
-    decode step through the fused-epilogue path."""
+    """Every step of the tiny workload against the oracle. The long prompt
+    (364 positions) takes the prefill through the GEMM's many-row path
+    (separate RoPE, SwiGLU and RMSNorm kernels); the short one and every decode
+    step through the fused-epilogue path."""
     wl = synth.WORKLOADS["tiny"].with_(dtype=dtype)
     if long_prompt:
         wl = wl.with_(n_text=(300, 300), steps=3)
-    tol = TOL[dtype]
-    eng, w = open_engine(wl)
-    m = oracle_model(wl, w)
-    prompts = synth.make_prompts(wl)
-    ids, lens, vis, offs = msd.upload_prompts(prompts)
-    eng.prefill(ids, lens, vis, offs)
-    ids_np, vis_np = prompt_numpy(prompts[0])
-    st = O.prefill(m, ids_np, vis_np)
-    torch.cuda.synchronize()
-    root = int(eng.root_out.cpu()[0])
-    # the root is the argmax of the last prompt position: equal unless a near tie
-    if root != st.root:
-        z = O.lm_logits(m, O.target_forward(
-            m, O.embed_prompt(m, ids_np, vis_np), np.arange(len(ids_np)),
-            [(np.zeros((0, wl.hidden)),) * 2] * wl.n_layers, np.zeros(len(ids_np), int), None,
-            O.causal_vis(len(ids_np)))[0][-1:])[0]
-        assert top2_margin(z) <= tol["max_abs"]
-        st.root = root; st.pend_next = np.array([root]); st.emitted = [root]
-    _kv_compare(eng, st, wl, 0, st.L, dtype, "prefill")
-
-    D, k, N, V = wl.tree_depth, wl.topk, wl.tree_nodes, wl.vocab
-    for step in range(wl.steps):
-        rec = record_buffers(wl)
-        eng.draft_tree(record=rec)
-        torch.cuda.synchronize()
-        R = {n: t.cpu().numpy() for n, t in rec.items()}
-
-        def forced(p, rows_logits):
-            n = rows_logits.shape[0]
-            return R["topk_ids"][0, p, :n].astype(np.int64), R["topk_logp"][0, p, :n].astype(np.float32)
-
-        orec = O.DraftRecord()
-        otree = O.draft_tree(m, st, record=orec, forced_logp=forced)
-        toks, par, dep, mask = tree_numpy(eng.tree, 0)
-        # integer parity of the tree, given the kernels' top-k decisions
-        np.testing.assert_array_equal(toks, otree.tokens, err_msg=f"step {step} tokens")
-        np.testing.assert_array_equal(par, otree.parent, err_msg=f"step {step} parent")
-        np.testing.assert_array_equal(dep, otree.depth, err_msg=f"step {step} depth")
-        np.testing.assert_array_equal(mask, otree.mask_words(), err_msg=f"step {step} mask")
-        for p in range(D):
-            rows = orec.logits[p].shape[0]
-            g = R["logits"][0, p, :rows]
-            assert_close(g, orec.logits[p], tol, f"step {step} draft pass {p} logits")
-            for r in range(rows):
-                # top-k of the kernels' own logits, and their log-softmax
-                np.testing.assert_array_equal(R["topk_ids"][0, p, r], O.topk_ids(g[r], k))
-                lp = O.log_softmax(g[r].astype(np.float64))[R["topk_ids"][0, p, r]]
-                np.testing.assert_allclose(R["topk_logp"][0, p, r], lp, atol=2e-5, rtol=1e-5)
-
-        logits = torch.zeros(N, V, device="cuda")
-        eng.verify(logits=logits)
-        torch.cuda.synchronize()
-        g_logits = logits.cpu().numpy()
-        g_arg = eng.argmax.cpu().numpy().astype(np.int64)
-        vr = O.verify(m, st, otree)
-        assert_close(g_logits, vr.logits, tol, f"step {step} verify logits")
-        for i in range(N):
-            assert g_arg[i] == O.argmax_lowest(g_logits[i])          # bit-exact given logits
-            if top2_margin(vr.logits[i]) > tol["max_abs"]:
-                assert g_arg[i] == vr.argmax[i], f"step {step} node {i} argmax"
-
-        eng.accept_compact()
-        torch.cuda.synchronize()
-        opath, oa, obonus = O.accept(otree, g_arg)
-        path = eng.path.cpu().numpy()
-        assert int(eng.accept_len.cpu()[0]) == oa and int(eng.bonus.cpu()[0]) == obonus
-        np.testing.assert_array_equal(path[:oa + 1], opath)
-        assert (path[oa + 1:] == -1).all()
-        imap = eng.index_map.cpu().numpy()
-        np.testing.assert_array_equal(imap[:oa + 1], st.L + np.arange(oa + 1))
-        O.compact(st, otree, vr, opath, obonus)
-        s = eng.state()
-        assert int(s["seq_len"].cpu()[0]) == st.L and int(s["root"].cpu()[0]) == st.root
-        assert int(s["n_pending"].cpu()[0]) == oa + 1
-        _kv_compare(eng, st, wl, 0, st.L, dtype, f"step {step}")
-    eng.close()
+    run_parity(wl, wl.steps)
 
 
 def _gpu_greedy_ar(eng, n_tokens):
