@@ -15,9 +15,13 @@ value        steps/s, device-timed with CUDA events over K back-to-back steps
 e2e          steps/s through the public API with host buffers: prompt copied
              from pinned host memory, prefill, then every step reads its
              emitted tokens back to pinned host memory and synchronises
-roofline     the tensor-core GEMM (the dominant kernel): algorithmic bytes per
-             launch / CUDA-event duration of each launch in the timed region,
-             against the measured HBM copy bandwidth
+roofline     the decode GEMM (gemm_cluster_kernel, 80% of the step's kernel time):
+             algorithmic bytes per launch / CUDA-event duration of each launch,
+             events around every GEMM launch over K_prof steps run right after
+             the timed region (separate launches, not the graph), against the
+             measured HBM copy bandwidth; traffic = DRAM bytes per launch from
+             an ncu capture (profiles/gemm_cluster_llava7b.md), reported while
+             the GEMM source is the one it was captured on
 cpu_baseline the CPU oracle on a bounded sample of the same step (target cut to
              2 of its layers, layer time scaled to the full depth)
 --impl reference times the same oracle sample as the reference arm.
@@ -57,6 +61,27 @@ def parse():
     ap.add_argument("--gemm", default=None,
                     help="M,K,O: time the tensor-core GEMM alone on that shape (kernel case)")
     return ap.parse_args()
+
+
+# DRAM traffic of the decode GEMM: ncu dram__bytes_read.sum + dram__bytes_write.sum
+# over the 45 GEMM launches of one 2-layer 7B-width step, divided by the same
+# launches' algorithmic bytes (0.996: no re-reads); per launch of the full
+# workload it is this ratio times its algorithmic bytes per launch. Valid for
+# the GEMM source with this SHA-1 only.
+GEMM_TRAFFIC = {"source_sha1": "ed83c37b788f99cda45fb046abfb5416c040f754", "ratio": 0.9959}
+
+
+def gemm_traffic(bytes_per_launch):
+    import hashlib
+    src = os.path.join(ROOT, "paper_2505_14260_gb300", "csrc", "gemm_tc.cu")
+    try:
+        with open(src, "rb") as f:
+            sha = hashlib.sha1(f.read()).hexdigest()
+    except OSError:
+        return None
+    if sha != GEMM_TRAFFIC["source_sha1"] or not bytes_per_launch:
+        return None
+    return GEMM_TRAFFIC["ratio"] * bytes_per_launch
 
 
 def peaks():
@@ -387,8 +412,11 @@ def run_msd(args, rank, world, local_rank):
             "tokens_per_s": world * tokens / (ms / 1e3),
             "tau": tokens / (K * B),
             "roofline": {"bound": "hbm", "achieved": gemm_gbs, "peak": hbm, "unit": "GB/s",
-                         "frac": (gemm_gbs / hbm) if gemm_gbs else None, "traffic": None,
-                         "kernel": "gemm_tc_kernel (tcgen05 bf16 GEMM, all projections)",
+                         "frac": (gemm_gbs / hbm) if gemm_gbs else None,
+                         "traffic": gemm_traffic(prof["gemm_bytes"] / max(prof["gemm_launches"], 1)),
+                         "kernel": "gemm_cluster_kernel (tcgen05 bf16 decode GEMM: 128-row weight tiles x "
+                                   "token rows, split-K over a thread-block cluster, fused epilogues; "
+                                   "all projections of the step)",
                          "launches": prof["gemm_launches"], "peak_kind": peak_kind,
                          "measured": f"CUDA events around each GEMM launch over {K_prof} steps "
                                      "right after the timed region (separate launches while profiling)",
