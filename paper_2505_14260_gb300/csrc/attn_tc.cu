@@ -32,6 +32,7 @@ constexpr int ROWS = 64;          // query rows per CTA
 constexpr int KT = 64;            // keys per tile
 constexpr int MAX_STAGES = 3;
 constexpr int MAX_SPLITS = 16;    // cache splits + the tree split = cluster size (<= 16)
+constexpr int CACHE_SPLITS = 8;   // cache splits of a decode launch (capacity-derived chunk)
 constexpr unsigned long long ATTN_TIMEOUT_NS = 2000000000ull;
 
 struct AttnTcParams {
@@ -486,7 +487,10 @@ bool attn_tc_plan_create(AttnTcPlan **out, int max_keys) {
     // (possibly empty) splits a launch covers; with the tree split a launch
     // has at most MAX_SPLITS CTAs per cluster.
     const int tiles = (max_keys + KT - 1) / KT;
-    p->chunk_tiles = std::max(2, (tiles + MAX_SPLITS - 2) / (MAX_SPLITS - 1));
+    // At most CACHE_SPLITS cache splits (+ the tree split): one cluster of <= 9
+    // two-stage CTAs per (row tile, head), two CTAs per SM, so a decode launch
+    // is one wave at any prefix length.
+    p->chunk_tiles = std::max(2, (tiles + CACHE_SPLITS - 1) / CACHE_SPLITS);
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev);
@@ -567,8 +571,9 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.nsplit_cache = nsplit;
     tp.has_tree = has_tree;
     tp.chunk = chunk_tiles * KT;
-    // two stages when a split holds at most two tiles: 2 CTAs per SM fit
-    tp.stages = chunk_tiles <= 2 ? 2 : MAX_STAGES;
+    // two stages keep two CTAs on an SM; three only where a split holds more
+    // than two tiles and the CTAs fit on the SMs at one per SM
+    tp.stages = (chunk_tiles <= 2 || (long)row_tiles * a.nh * (nsplit + has_tree) > p->num_sms) ? 2 : MAX_STAGES;
     tp.scale_log2 = a.scale * 1.4426950408889634f;
     const size_t smem = 1024 + (size_t)ROWS * a.hd * 2 + (size_t)tp.stages * 2 * KT * a.hd * 2;
     if (!p->attr_set) {
