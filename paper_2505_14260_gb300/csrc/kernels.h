@@ -72,6 +72,9 @@ void launch_argmax(const float *logits, int R, int V, int *out, const TopkScratc
 // nullable). k <= 16.
 void launch_topk_logp(const float *logits, int R, int V, int k, int *ids, float *logp,
                       const TopkScratch &sc, cudaStream_t s);
+// Whether the top-k kernel takes vocabulary V with k <= 16 (ceil(V / 4096) * k
+// candidates <= 256 in its row merge).
+bool topk_supported(int V, int k);
 
 template <typename T>
 void launch_convert(const float *x, T *y, long n, cudaStream_t s);

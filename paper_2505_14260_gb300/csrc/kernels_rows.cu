@@ -198,125 +198,150 @@ void launch_rope_kv(const float *qkv, const RowDesc *rows, int R, int nh, int hd
 // ---------------------------------------------------------------------------
 constexpr int TOPK_MAX = 16;
 constexpr int TK_THREADS = 256;
-constexpr int TK_REC = 2 + 2 * TOPK_MAX;     // floats per chunk record
+constexpr int TK_EPT = 16;                         // logits per thread
+constexpr int TK_CHUNK = TK_THREADS * TK_EPT;      // logits per CTA
+constexpr int TK_REC = 2 + 2 * TOPK_MAX;           // floats per chunk record
+constexpr int TK_NONE = 0x7fffffff;                // index of an empty slot
+constexpr int TK_MERGE_SLOTS = 8;                  // row merge: nc * k <= 32 * 8 candidates
 
-__device__ __forceinline__ void block_best(float &v, int &i, float *rv, int *ri) {
+// (max, sum of exp(x - max)) pairs combined exactly
+__device__ __forceinline__ void lse_combine(float &m, float &s, float om, float os) {
+    const float nm = fmaxf(m, om);
+    if (nm == -INFINITY) return;
+    s = s * __expf(m - nm) + os * __expf(om - nm);
+    m = nm;
+}
+
+__device__ __forceinline__ void warp_lse(float &m, float &s) {
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const float om = __shfl_xor_sync(0xffffffffu, m, o), os = __shfl_xor_sync(0xffffffffu, s, o);
+        lse_combine(m, s, om, os);
+    }
+}
+
+// Best (value, index) of a warp; every lane gets it.
+__device__ __forceinline__ void warp_best(float &v, int &i) {
 #pragma unroll
     for (int o = 16; o > 0; o >>= 1) {
         const float ov = __shfl_xor_sync(0xffffffffu, v, o);
         const int oi = __shfl_xor_sync(0xffffffffu, i, o);
         if (better(ov, oi, v, i)) { v = ov; i = oi; }
     }
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
-    __syncthreads();
-    if (lane == 0) { rv[warp] = v; ri[warp] = i; }
-    __syncthreads();
-    if (warp == 0) {
-        const int nw = blockDim.x >> 5;
-        v = lane < nw ? rv[lane] : -INFINITY;
-        i = lane < nw ? ri[lane] : 0x7fffffff;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) {
-            const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-            const int oi = __shfl_xor_sync(0xffffffffu, i, o);
-            if (better(ov, oi, v, i)) { v = ov; i = oi; }
-        }
-        if (lane == 0) { rv[0] = v; ri[0] = i; }
-    }
-    __syncthreads();
-    v = rv[0];
-    i = ri[0];
 }
 
+// Top-k of the NS (value, index) slots held by each lane of a warp, in k
+// rounds of warp arg-max: the winner's slot is retired by index (indices are
+// unique), so no slot is ever indexed dynamically. Lane 0 gets the result.
+template <int NS>
+__device__ __forceinline__ void warp_topk(float (&v)[NS], int (&ix)[NS], int k, float *out_v, int *out_i) {
+    for (int t = 0; t < k; ++t) {
+        float bv = -INFINITY;
+        int bi = TK_NONE;
+#pragma unroll
+        for (int e = 0; e < NS; ++e)
+            if (better(v[e], ix[e], bv, bi)) { bv = v[e]; bi = ix[e]; }
+        warp_best(bv, bi);
+#pragma unroll
+        for (int e = 0; e < NS; ++e)
+            if (ix[e] == bi) { v[e] = -INFINITY; ix[e] = TK_NONE; }
+        if ((threadIdx.x & 31) == 0) { out_v[t] = bv; out_i[t] = bi; }
+    }
+}
+
+// Per row: chunks of TK_CHUNK logits, one CTA each. Each warp takes the top-k
+// of its 512 logits and their (max, sum exp); one warp merges the CTA's warps,
+// and the row's last CTA (ticket) merges the chunks; log-probabilities are
+// logit - logsumexp.
 __global__ void __launch_bounds__(TK_THREADS)
     topk_rows_kernel(const float *__restrict__ logits, int V, int k, int *__restrict__ ids,
                      float *__restrict__ logp, float *__restrict__ ws, int *__restrict__ counters) {
     allow_dependents();
     wait_prior();
-    extern __shared__ float sv[];
-    __shared__ float rv[32];
-    __shared__ int ri[32];
-    __shared__ float sel_v[TOPK_MAX];
-    __shared__ int sel_i[TOPK_MAX];
+    constexpr int NW = TK_THREADS / 32;
+    __shared__ float s_v[NW * TOPK_MAX];
+    __shared__ int s_i[NW * TOPK_MAX];
+    __shared__ float s_m[NW], s_s[NW];
     __shared__ int s_last;
     const int r = blockIdx.y, c = blockIdx.x, nc = gridDim.x;
-    const int CH = (V + nc - 1) / nc;
-    const int lo = c * CH, n = max(0, min(V, lo + CH) - lo);
-    const float *z = logits + (size_t)r * V + lo;
-    float mx = -INFINITY;
-    for (int j = threadIdx.x; j < n; j += TK_THREADS) {
-        const float v = z[j];
-        sv[j] = v;
-        mx = fmaxf(mx, v);
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
+    const int lo = c * TK_CHUNK + warp * (32 * TK_EPT);       // this warp's 512 logits
+    const float *z = logits + (size_t)r * V;
+    float x[TK_EPT];
+    int xi[TK_EPT];
+#pragma unroll
+    for (int e = 0; e < TK_EPT; ++e) {
+        const int j = lo + lane + e * 32;
+        x[e] = j < V ? z[j] : -INFINITY;
+        xi[e] = j < V ? j : TK_NONE;
     }
-    mx = block_max(mx, rv);
-    float se = 0.f;
-    for (int j = threadIdx.x; j < n; j += TK_THREADS) se += __expf(sv[j] - mx);
-    se = block_sum(se, rv);
-    for (int t = 0; t < k; ++t) {
-        float bv = -INFINITY;
-        int bi = 0x7fffffff;
-        for (int j = threadIdx.x; j < n; j += TK_THREADS)
-            if (better(sv[j], lo + j, bv, bi)) { bv = sv[j]; bi = lo + j; }
-        block_best(bv, bi, rv, ri);
-        if (threadIdx.x == 0) { sel_v[t] = bv; sel_i[t] = bi; }
-        if (bi != 0x7fffffff && bi - lo >= 0 && bi - lo < n && ((bi - lo) % TK_THREADS) == threadIdx.x)
-            sv[bi - lo] = -INFINITY;
-        __syncthreads();
-    }
+    float m = -INFINITY, sum = 0.f;
+#pragma unroll
+    for (int e = 0; e < TK_EPT; ++e) m = fmaxf(m, x[e]);
+#pragma unroll
+    for (int e = 0; e < TK_EPT; ++e)
+        if (xi[e] != TK_NONE) sum += __expf(x[e] - m);
+    warp_lse(m, sum);
+    warp_topk<TK_EPT>(x, xi, k, s_v + warp * TOPK_MAX, s_i + warp * TOPK_MAX);
+    if (lane == 0) { s_m[warp] = m; s_s[warp] = sum; }
+    __syncthreads();
     float *rec = ws + ((size_t)r * nc + c) * TK_REC;
-    if (threadIdx.x == 0) { rec[0] = mx; rec[1] = se; }
-    if (threadIdx.x < k) {
-        rec[2 + threadIdx.x] = sel_v[threadIdx.x];
-        rec[2 + TOPK_MAX + threadIdx.x] = __int_as_float(sel_i[threadIdx.x]);
+    if (warp == 0) {
+        // the NW warps' k candidates, NW * TOPK_MAX / 32 slots per lane
+        constexpr int NS = NW * TOPK_MAX / 32;
+        float cv[NS];
+        int ci[NS];
+#pragma unroll
+        for (int e = 0; e < NS; ++e) {
+            const int q = lane + e * 32, w = q / TOPK_MAX, t = q - w * TOPK_MAX;
+            cv[e] = t < k ? s_v[q] : -INFINITY;
+            ci[e] = t < k ? s_i[q] : TK_NONE;
+        }
+        m = lane < NW ? s_m[lane] : -INFINITY;
+        sum = lane < NW ? s_s[lane] : 0.f;
+        warp_lse(m, sum);
+        if (lane == 0) { rec[0] = m; rec[1] = sum; }
+        __syncwarp();                      // the candidates are in registers: reuse s_v / s_i
+        warp_topk<NS>(cv, ci, k, s_v, s_i);
+        __syncwarp();
+        if (lane < k) {
+            rec[2 + lane] = s_v[lane];
+            rec[2 + TOPK_MAX + lane] = __int_as_float(s_i[lane]);
+        }
     }
     __threadfence();
     __syncthreads();
     if (threadIdx.x == 0) s_last = atomicAdd(&counters[r], 1) == nc - 1;
     __syncthreads();
-    if (!s_last) return;
+    if (!s_last || warp != 0) return;
     __threadfence();
-    // merge the chunk records of row r
+    // merge the row's chunk records: nc * k candidates, TK_MERGE_SLOTS per lane
     const float *rrow = ws + (size_t)r * nc * TK_REC;
-    float M = -INFINITY;
-    for (int q = threadIdx.x; q < nc; q += TK_THREADS) M = fmaxf(M, __ldcg(rrow + q * TK_REC));
-    M = block_max(M, rv);
-    float S = 0.f;
-    for (int q = threadIdx.x; q < nc; q += TK_THREADS)
-        S += __ldcg(rrow + q * TK_REC + 1) * __expf(__ldcg(rrow + q * TK_REC) - M);
-    S = block_sum(S, rv);
-    const float lse = M + logf(S);
-    float *cv = sv;                                   // candidates: nc * k
-    int *ci = reinterpret_cast<int *>(sv + nc * k);
-    for (int q = threadIdx.x; q < nc * k; q += TK_THREADS) {
-        const int cc = q / k, t = q - cc * k;
-        cv[q] = __ldcg(rrow + cc * TK_REC + 2 + t);
-        ci[q] = __float_as_int(__ldcg(rrow + cc * TK_REC + 2 + TOPK_MAX + t));
+    float cv[TK_MERGE_SLOTS];
+    int ci[TK_MERGE_SLOTS];
+#pragma unroll
+    for (int e = 0; e < TK_MERGE_SLOTS; ++e) {
+        const int q = lane + e * 32, cc = q / k, t = q - cc * k;
+        const bool have = cc < nc;
+        cv[e] = have ? __ldcg(rrow + cc * TK_REC + 2 + t) : -INFINITY;
+        ci[e] = have ? __float_as_int(__ldcg(rrow + cc * TK_REC + 2 + TOPK_MAX + t)) : TK_NONE;
     }
-    __syncthreads();
-    for (int t = 0; t < k; ++t) {
-        float bv = -INFINITY;
-        int bi = 0x7fffffff, bq = -1;
-        for (int q = threadIdx.x; q < nc * k; q += TK_THREADS)
-            if (better(cv[q], ci[q], bv, bi)) { bv = cv[q]; bi = ci[q]; bq = q; }
-        float wv = bv;
-        int wi = bi;
-        block_best(wv, wi, rv, ri);
-        if (bq >= 0 && bi == wi) cv[bq] = -INFINITY;   // ids are unique within a row
-        if (threadIdx.x == 0) {
-            ids[(size_t)r * k + t] = wi == 0x7fffffff ? 0 : wi;
-            if (logp) logp[(size_t)r * k + t] = wv - lse;
-        }
-        __syncthreads();
+    m = -INFINITY;
+    sum = 0.f;
+    for (int q = lane; q < nc; q += 32)
+        lse_combine(m, sum, __ldcg(rrow + q * TK_REC), __ldcg(rrow + q * TK_REC + 1));
+    warp_lse(m, sum);
+    const float lse = m + logf(sum);
+    warp_topk<TK_MERGE_SLOTS>(cv, ci, k, s_v, s_i);
+    __syncwarp();
+    if (lane < k) {
+        ids[(size_t)r * k + lane] = s_i[lane] == TK_NONE ? 0 : s_i[lane];
+        if (logp) logp[(size_t)r * k + lane] = s_v[lane] - lse;
     }
-    if (threadIdx.x == 0) counters[r] = 0;
+    if (lane == 0) counters[r] = 0;
 }
 
-static int topk_chunks(int V) {
-    int nc = 16;
-    while ((V + nc - 1) / nc > 4096) nc *= 2;
-    return nc;
-}
+static int topk_chunks(int V) { return (V + TK_CHUNK - 1) / TK_CHUNK; }
 
 size_t topk_scratch_floats(int max_rows, int V) {
     return (size_t)max_rows * topk_chunks(V) * TK_REC;
@@ -324,13 +349,16 @@ size_t topk_scratch_floats(int max_rows, int V) {
 
 void launch_topk_logp(const float *logits, int R, int V, int k, int *ids, float *logp,
                       const TopkScratch &sc, cudaStream_t s) {
-    if (R <= 0) return;
+    if (R <= 0 || k < 1 || k > TOPK_MAX) return;
     const int nc = topk_chunks(V);
-    const int CH = (V + nc - 1) / nc;
-    const size_t smem = sizeof(float) * std::max<size_t>(CH, (size_t)2 * nc * k);
-    launch_pdl(topk_rows_kernel, dim3(nc, R), TK_THREADS, smem, s, logits, V, k, ids, logp, sc.ws,
-                                                          sc.counters);
+    if (nc * k > 32 * TK_MERGE_SLOTS) return;            // refused at msd_create
+    launch_pdl(topk_rows_kernel, dim3(nc, R), TK_THREADS, 0, s, logits, V, k, ids, logp, sc.ws,
+               sc.counters);
     note_launch();
+}
+
+bool topk_supported(int V, int k) {
+    return k >= 1 && k <= TOPK_MAX && topk_chunks(V) * k <= 32 * TK_MERGE_SLOTS;
 }
 
 void launch_argmax(const float *logits, int R, int V, int *out, const TopkScratch &sc,

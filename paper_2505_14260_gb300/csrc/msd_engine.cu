@@ -628,6 +628,7 @@ msd_status validate_config(const msd_config *g) {
     if (g->tree_nodes < 1 || g->tree_nodes > 256) return MSD_ERR_INVALID;
     if (g->tree_depth < 1 || g->tree_depth > TREE_MAXD) return MSD_ERR_INVALID;
     if (g->topk < 1 || g->topk > TREE_MAXK || g->topk > g->vocab) return MSD_ERR_INVALID;
+    if (!topk_supported(g->vocab, g->topk)) return MSD_ERR_INVALID;
     const long cand = g->topk + (long)(g->tree_depth - 1) * g->topk * g->topk;
     if (cand < g->tree_nodes - 1) return MSD_ERR_INVALID;
     return MSD_OK;
