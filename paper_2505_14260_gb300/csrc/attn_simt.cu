@@ -8,8 +8,8 @@ namespace msd {
 
 template <typename T, int HD>
 __global__ void attn_simt_kernel(AttnArgs<T> a) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     constexpr int EPL = HD / 32;    // elements per lane
     const int warp = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
     const int lane = threadIdx.x & 31;

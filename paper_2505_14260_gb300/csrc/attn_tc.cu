@@ -1,12 +1,15 @@
 // Tree-masked attention on the tensor cores for the bf16 path.
 //
-// A CTA (4 warps) takes 64 query rows of one request and one head; each warp
-// owns 16 rows. Keys come in tiles of 64, staged by TMA (two 64x64 boxes per
-// tile for head_dim 128, 128-byte swizzle) into a ring of shared-memory stages
-// completed on mbarriers. Per tile: S = Q K^T with mma.sync m16n8k16 (bf16,
-// fp32 accumulate), masking, an online softmax in base 2 (row max and sum
-// across the 4 lanes of a quad with shuffles), and O += P V (P re-packed from
-// the S accumulators as the A operand, V read with ldmatrix.trans).
+// A CTA (8 warps) takes 64 query rows of one request and one head: warps g and
+// g + 4 own rows 16g .. 16g + 15, and split every key tile between them (keys
+// 0-31 and 32-63), each with its own online-softmax state; the two halves merge
+// once, after the CTA's last tile. Keys come in tiles of 64, staged by TMA (two
+// 64x64 boxes per tile for head_dim 128, 128-byte swizzle) into a ring of
+// shared-memory stages completed on mbarriers. Per tile and warp: S = Q K^T
+// over its 32 keys with mma.sync m16n8k16 (bf16, fp32 accumulate), masking, an
+// online softmax in base 2 (row max and sum across the 4 lanes of a quad with
+// shuffles), and O += P V (P re-packed from the S accumulators as the A
+// operand, V read with ldmatrix.trans).
 //
 // Visible keys of a row (Sec. 3.2: a candidate is conditioned on its prefix
 // only): cache positions [0, plen) of its request, and tree slots whose bit is
@@ -30,6 +33,10 @@ namespace {
 
 constexpr int ROWS = 64;          // query rows per CTA
 constexpr int KT = 64;            // keys per tile
+constexpr int THREADS = 256;      // 8 warps: 4 row groups x 2 key halves
+// row stride (floats) of the fp32 partials in shared memory: padded so that the
+// 8 rows a warp writes at once fall in different banks
+template <int HD> constexpr int PART_LD = HD + 8;
 constexpr int MAX_STAGES = 3;
 constexpr int MAX_SPLITS = 16;    // cache splits + the tree split = cluster size (<= 16)
 constexpr int CACHE_SPLITS = 8;   // cache splits of a decode launch (capacity-derived chunk)
@@ -43,6 +50,7 @@ struct AttnTcParams {
     int *status;
     int R, rows_per_req, tiles_per_req, nh, cache_slots, tree_slots, mask_words;
     int nsplit_cache, has_tree, chunk, stages;
+    int cache_early;          // cache K/V may be requested before the wait (not written by the previous kernel)
     float scale_log2;
 };
 
@@ -158,11 +166,10 @@ __device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
 }
 
 template <int HD>
-__global__ void __launch_bounds__(128)
+__global__ void __launch_bounds__(THREADS, 2)
     attn_tc_kernel(const __grid_constant__ CUtensorMap mkc, const __grid_constant__ CUtensorMap mvc,
                    const __grid_constant__ CUtensorMap mkt, const __grid_constant__ CUtensorMap mvt,
                    const AttnTcParams p) {
-    allow_dependents();
     constexpr int NB = HD / 64;                   // 64-wide boxes per row
     constexpr int TILE_BYTES = KT * HD * 2;       // one K (or V) tile
     constexpr int NT_O = HD / 8;                  // O n-tiles per warp
@@ -171,6 +178,7 @@ __global__ void __launch_bounds__(128)
     __shared__ int s_pmax;
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int grp = warp & 3, half = warp >> 2;     // row group, key half of each tile
     const int tile = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
     const int blk = tile / p.tiles_per_req;
     const int r0 = blk * p.rows_per_req + (tile - blk * p.tiles_per_req) * ROWS;
@@ -190,12 +198,14 @@ __global__ void __launch_bounds__(128)
         asm volatile("prefetch.tensormap [%0];" ::"l"(&mkc) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(&mvc) : "memory");
     }
-    wait_prior();                  // q, the row descriptors and K/V come from earlier kernels
     __syncthreads();
+    // Before the wait: the row descriptors (written by set-up kernels at least
+    // two launches back) and, unless the previous kernel wrote into it, the
+    // cache K/V. The previous kernel's q and tree K/V are read after the wait.
     const int req = p.rows[r0].req;
 
     // Rows of this thread: A = lane/4, B = lane/4 + 8 of the warp's 16.
-    const int ra = r0 + warp * 16 + (lane >> 2), rb = ra + 8;
+    const int ra = r0 + grp * 16 + (lane >> 2), rb = ra + 8;
     const bool va = ra < r_end, vb = rb < r_end;
     const int plen_a = va ? p.rows[ra].plen : 0, plen_b = vb ? p.rows[rb].plen : 0;
     atomicMax(&s_pmax, max(plen_a, plen_b));
@@ -237,14 +247,19 @@ __global__ void __launch_bounds__(128)
     };
     // K/V tiles in flight first, then the Q tile (all its loads issued before
     // the first shared-memory store); rows past the request's rows are zero.
-    if (threadIdx.x == 0)
+    const bool early = !is_tree && p.cache_early;
+    if (threadIdx.x == 0 && early)
+        for (int i = 0; i < min(stages, ntiles); ++i) issue(i);
+    wait_prior();
+    allow_dependents();
+    if (threadIdx.x == 0 && !early)
         for (int i = 0; i < min(stages, ntiles); ++i) issue(i);
     {
-        constexpr int QV = ROWS * HD / 8 / 128;       // 16-byte pieces per thread
+        constexpr int QV = ROWS * HD / 8 / THREADS;   // 16-byte pieces per thread
         uint4 qv[QV];
 #pragma unroll
         for (int j = 0; j < QV; ++j) {
-            const int i = threadIdx.x + j * 128;
+            const int i = threadIdx.x + j * THREADS;
             const int row = i / (HD / 8), c = i - row * (HD / 8);
             qv[j] = r0 + row < r_end
                         ? __ldg(reinterpret_cast<const uint4 *>(p.q + (size_t)(r0 + row) * H + h * HD + c * 8))
@@ -252,7 +267,7 @@ __global__ void __launch_bounds__(128)
         }
 #pragma unroll
         for (int j = 0; j < QV; ++j) {
-            const int i = threadIdx.x + j * 128;
+            const int i = threadIdx.x + j * THREADS;
             const int row = i / (HD / 8), c = i - row * (HD / 8);
             asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(swz(q_s, row, c)), "r"(qv[j].x),
                          "r"(qv[j].y), "r"(qv[j].z), "r"(qv[j].w)
@@ -261,14 +276,9 @@ __global__ void __launch_bounds__(128)
     }
     __syncthreads();
 
-    // Q fragments of the warp's 16 rows.
-    uint32_t qf[HD / 16][4];
-#pragma unroll
-    for (int kk = 0; kk < HD / 16; ++kk) {
-        const int m = lane >> 3;
-        const int row = warp * 16 + (m & 1) * 8 + (lane & 7);
-        ldsm4(swz(q_s, row, 2 * kk + (m >> 1)), qf[kk][0], qf[kk][1], qf[kk][2], qf[kk][3]);
-    }
+    // Q fragments of the warp's 16 rows are re-read from shared memory per tile
+    // (ldmatrix), which keeps two 8-warp CTAs' registers on an SM.
+    const int q_row = grp * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
 
     // Tree-mask words of the two rows (tree split only).
     const uint64_t *mask_a = (is_tree && va) ? p.mask + (size_t)ra * p.mask_words : nullptr;
@@ -286,19 +296,23 @@ __global__ void __launch_bounds__(128)
         const uint32_t ks = kv_s + s * stage_bytes, vs = ks + TILE_BYTES;
         const int key0 = k_lo + i * KT;
 
-        float sc[8][4];
+        // this warp's 32 keys of the tile: kh .. kh + 31
+        const int kh = half * 32;
+        float sc[4][4];
 #pragma unroll
-        for (int j = 0; j < 8; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
+        for (int j = 0; j < 4; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
 #pragma unroll
         for (int kk = 0; kk < HD / 16; ++kk) {
+            uint32_t qf[4];
+            ldsm4(swz(q_s, q_row, 2 * kk + (lane >> 4)), qf[0], qf[1], qf[2], qf[3]);
 #pragma unroll
-            for (int np = 0; np < 4; ++np) {
+            for (int np = 0; np < 2; ++np) {
                 const int m = lane >> 3;
-                const int key = np * 16 + (m >> 1) * 8 + (lane & 7);
+                const int key = kh + np * 16 + (m >> 1) * 8 + (lane & 7);
                 uint32_t b0, b1, b2, b3;
                 ldsm4(swz(ks, key, 2 * kk + (m & 1)), b0, b1, b2, b3);
-                mma16816(sc[2 * np], qf[kk], b0, b1);
-                mma16816(sc[2 * np + 1], qf[kk], b2, b3);
+                mma16816(sc[2 * np], qf, b0, b1);
+                mma16816(sc[2 * np + 1], qf, b2, b3);
             }
         }
         // mask + scale (base-2 logits)
@@ -310,10 +324,10 @@ __global__ void __launch_bounds__(128)
         }
         float mx_a = -INFINITY, mx_b = -INFINITY;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < 4; ++j) {
 #pragma unroll
             for (int e = 0; e < 4; ++e) {
-                const int kl = 8 * j + 2 * (lane & 3) + (e & 1);
+                const int kl = kh + 8 * j + 2 * (lane & 3) + (e & 1);
                 const int key = key0 + kl;
                 bool vis;
                 if (is_tree) {
@@ -338,7 +352,7 @@ __global__ void __launch_bounds__(128)
         m_b = mn_b;
         float rs_a = 0.f, rs_b = 0.f;
 #pragma unroll
-        for (int j = 0; j < 8; ++j) {
+        for (int j = 0; j < 4; ++j) {
             sc[j][0] = exp2f(sc[j][0] - use_a);
             sc[j][1] = exp2f(sc[j][1] - use_a);
             sc[j][2] = exp2f(sc[j][2] - use_b);
@@ -353,9 +367,9 @@ __global__ void __launch_bounds__(128)
             o[j][0] *= cf_a; o[j][1] *= cf_a;
             o[j][2] *= cf_b; o[j][3] *= cf_b;
         }
-        // O += P V
+        // O += P V over the warp's 32 keys
 #pragma unroll
-        for (int kk = 0; kk < 4; ++kk) {
+        for (int kk = 0; kk < 2; ++kk) {
             uint32_t pa[4];
             pa[0] = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
             pa[1] = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
@@ -364,7 +378,7 @@ __global__ void __launch_bounds__(128)
 #pragma unroll
             for (int dp = 0; dp < HD / 16; ++dp) {
                 const int m = lane >> 3;
-                const int key = kk * 16 + (m & 1) * 8 + (lane & 7);
+                const int key = kh + kk * 16 + (m & 1) * 8 + (lane & 7);
                 uint32_t b0, b1, b2, b3;
                 ldsm4t(swz(vs, key, 2 * dp + (m >> 1)), b0, b1, b2, b3);
                 mma16816(o[2 * dp], pa, b0, b1);
@@ -380,9 +394,55 @@ __global__ void __launch_bounds__(128)
     l_b += __shfl_xor_sync(0xffffffffu, l_b, 1);
     l_b += __shfl_xor_sync(0xffffffffu, l_b, 2);
 
-    const int nsplit = p.nsplit_cache + p.has_tree;
+    // Merge the two key halves of each row group: the upper warps leave (O, m,
+    // l) in shared memory (the K/V stages are idle now), the lower warps fold
+    // them into theirs; the result is left in the same place for the cluster
+    // combine below.
     const int col0 = 2 * (lane & 3);
+    __syncthreads();
+    constexpr int LD = PART_LD<HD>;
+    float *s_o = reinterpret_cast<float *>(smem_raw + (kv_s - su32(smem_raw)));   // [64][LD]
+    float *s_ml = s_o + ROWS * LD;                                               // [64][2]
+    const int la = grp * 16 + (lane >> 2), lb = la + 8;
+    if (half == 1) {
+#pragma unroll
+        for (int j = 0; j < NT_O; ++j) {
+            const int c = 8 * j + col0;
+            *reinterpret_cast<float2 *>(s_o + la * LD + c) = make_float2(o[j][0], o[j][1]);
+            *reinterpret_cast<float2 *>(s_o + lb * LD + c) = make_float2(o[j][2], o[j][3]);
+        }
+        if ((lane & 3) == 0) {
+            *reinterpret_cast<float2 *>(s_ml + la * 2) = make_float2(m_a, l_a);
+            *reinterpret_cast<float2 *>(s_ml + lb * 2) = make_float2(m_b, l_b);
+        }
+    }
+    __syncthreads();
+    if (half == 0) {
+        const float2 ua = *reinterpret_cast<const float2 *>(s_ml + la * 2);
+        const float2 ub = *reinterpret_cast<const float2 *>(s_ml + lb * 2);
+        const float Ma = fmaxf(m_a, ua.x), Mb = fmaxf(m_b, ub.x);
+        const float ba = Ma == -INFINITY ? 0.f : Ma, bb = Mb == -INFINITY ? 0.f : Mb;
+        const float c0a = exp2f(m_a - ba), c1a = exp2f(ua.x - ba);
+        const float c0b = exp2f(m_b - bb), c1b = exp2f(ub.x - bb);
+#pragma unroll
+        for (int j = 0; j < NT_O; ++j) {
+            const int c = 8 * j + col0;
+            const float2 xa = *reinterpret_cast<const float2 *>(s_o + la * LD + c);
+            const float2 xb = *reinterpret_cast<const float2 *>(s_o + lb * LD + c);
+            o[j][0] = o[j][0] * c0a + xa.x * c1a;
+            o[j][1] = o[j][1] * c0a + xa.y * c1a;
+            o[j][2] = o[j][2] * c0b + xb.x * c1b;
+            o[j][3] = o[j][3] * c0b + xb.y * c1b;
+        }
+        l_a = l_a * c0a + ua.y * c1a;
+        l_b = l_b * c0b + ub.y * c1b;
+        m_a = Ma;
+        m_b = Mb;
+    }
+
+    const int nsplit = p.nsplit_cache + p.has_tree;
     if (nsplit == 1) {
+        if (half == 1) return;
         const float ia = l_a > 0.f ? 1.f / l_a : 0.f, ib = l_b > 0.f ? 1.f / l_b : 0.f;
 #pragma unroll
         for (int j = 0; j < NT_O; ++j) {
@@ -402,16 +462,13 @@ __global__ void __launch_bounds__(128)
     // sum l) in its own shared memory; after a cluster barrier every CTA
     // combines a slice of the rows, reading all partials through distributed
     // shared memory in rank order (deterministic), and writes them out.
-    __syncthreads();                                   // KV stages are idle now
-    float *s_o = reinterpret_cast<float *>(smem_raw + (kv_s - su32(smem_raw)));   // [64][HD]
-    float *s_ml = s_o + ROWS * HD;                                               // [64][2]
-    {
-        const int la = warp * 16 + (lane >> 2), lb = la + 8;
+    __syncwarp();                      // the quad's reads of s_ml above are done
+    if (half == 0) {
 #pragma unroll
         for (int j = 0; j < NT_O; ++j) {
             const int c = 8 * j + col0;
-            *reinterpret_cast<float2 *>(s_o + la * HD + c) = make_float2(o[j][0], o[j][1]);
-            *reinterpret_cast<float2 *>(s_o + lb * HD + c) = make_float2(o[j][2], o[j][3]);
+            *reinterpret_cast<float2 *>(s_o + la * LD + c) = make_float2(o[j][0], o[j][1]);
+            *reinterpret_cast<float2 *>(s_o + lb * LD + c) = make_float2(o[j][2], o[j][3]);
         }
         if ((lane & 3) == 0) {
             *reinterpret_cast<float2 *>(s_ml + la * 2) = make_float2(m_a, l_a);
@@ -425,7 +482,7 @@ __global__ void __launch_bounds__(128)
     const int row_lo = (int)rank * per, row_hi = min(nrows, row_lo + per);
     const uint32_t o_local = su32(s_o), ml_local = su32(s_ml);
     constexpr int C4 = HD / 4;
-    for (int rr = row_lo + warp; rr < row_hi; rr += 4) {
+    for (int rr = row_lo + warp; rr < row_hi; rr += THREADS / 32) {
         // lane sp fetches split sp's (m, l); warp shuffles give the max and the sum
         float2 ml = make_float2(-INFINITY, 0.f);
         if (lane < nsplit) ml = dsmem_ld_f2(dsmem_addr(ml_local + rr * 8, lane));
@@ -441,7 +498,7 @@ __global__ void __launch_bounds__(128)
             float4 v[MAX_SPLITS];
 #pragma unroll
             for (int sp = 0; sp < MAX_SPLITS; ++sp)     // every load in flight at once
-                if (sp < nsplit) v[sp] = dsmem_ld_f4(dsmem_addr(o_local + (rr * HD + 4 * lane) * 4, sp));
+                if (sp < nsplit) v[sp] = dsmem_ld_f4(dsmem_addr(o_local + (rr * LD + 4 * lane) * 4, sp));
             float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
             for (int sp = 0; sp < MAX_SPLITS; ++sp)
@@ -574,6 +631,7 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     // two stages keep two CTAs on an SM; three only where a split holds more
     // than two tiles and the CTAs fit on the SMs at one per SM
     tp.stages = (chunk_tiles <= 2 || (long)row_tiles * a.nh * (nsplit + has_tree) > p->num_sms) ? 2 : MAX_STAGES;
+    tp.cache_early = a.cache_fresh ? 0 : 1;
     tp.scale_log2 = a.scale * 1.4426950408889634f;
     const size_t smem = 1024 + (size_t)ROWS * a.hd * 2 + (size_t)tp.stages * 2 * KT * a.hd * 2;
     if (!p->attr_set) {
@@ -589,7 +647,7 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     cudaLaunchConfig_t lc;
     memset(&lc, 0, sizeof lc);
     lc.gridDim = dim3(row_tiles, a.nh, tot);
-    lc.blockDim = dim3(128);
+    lc.blockDim = dim3(THREADS);
     lc.dynamicSmemBytes = smem;
     lc.stream = s;
     cudaLaunchAttribute at[2];

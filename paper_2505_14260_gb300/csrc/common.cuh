@@ -39,14 +39,19 @@ __device__ __forceinline__ void set_status(int *st, int code) {
 
 // Lets a dependent kernel launched with programmatic stream serialization
 // start its prologue now; it still waits for this grid before reading any of
-// its outputs (griddepcontrol.wait).
+// its outputs (griddepcontrol.wait). Every kernel calls it only after its own
+// wait_prior(): a kernel that has started therefore implies that the kernel
+// two launches back has completed, so a prologue may read, before its own
+// wait, data last written two or more launches earlier (weights, caches
+// written by earlier steps, row descriptors of earlier set-up kernels).
 __device__ __forceinline__ void allow_dependents() {
     asm volatile("griddepcontrol.launch_dependents;");
 }
 
 // Waits until the grids this one depends on have completed and their writes
-// are visible. Every kernel launched by launch_pdl calls it before its first
-// global memory access, so that completion stays transitive along the stream.
+// are visible. Every kernel launched by launch_pdl calls it before it reads
+// anything the previous kernel may have written, so that completion stays
+// transitive along the stream.
 __device__ __forceinline__ void wait_prior() {
     asm volatile("griddepcontrol.wait;" ::: "memory");
 }

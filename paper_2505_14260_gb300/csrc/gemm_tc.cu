@@ -474,7 +474,6 @@ __global__ void __launch_bounds__(P_THREADS, 1)
 
     if (warp == 0) {
         if (lane == 0) {
-            pdl_trigger();
             asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
             // Weights never depend on the previous kernel: the first stages'
             // weight blocks are requested before waiting for it.
@@ -491,6 +490,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 }
             }
             pdl_wait();
+            pdl_trigger();
             ItemIter it = items0;
             int t, kb_b, kb_e, s = 0, i = 0;
             uint32_t ph = 0;
@@ -972,7 +972,6 @@ __global__ void __launch_bounds__(C_THREADS)
 
     if (warp == 0) {
         if (lane == 0) {
-            pdl_trigger();
             asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
             // weights first (they never depend on the previous kernel), then wait
             const int n_pre = min(C_STAGES, nk);
@@ -981,6 +980,7 @@ __global__ void __launch_bounds__(C_THREADS)
                 bulk_load(a_base + j * A_BYTES, wblk + (size_t)j * blk_elems, A_BYTES, full0 + 8 * j);
             }
             pdl_wait();
+            pdl_trigger();
             int s = 0;
             uint32_t ph = 0;
             int i = 0;

@@ -52,6 +52,7 @@ struct AttnArgs {
     int nh, hd;
     float scale;
     T *out;                     // [R][nh*hd]
+    bool cache_fresh;           // the kernel launched just before may have written cache_k/v
 };
 template <typename T>
 void launch_attention(const AttnArgs<T> &a, cudaStream_t s);

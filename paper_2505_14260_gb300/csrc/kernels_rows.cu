@@ -18,8 +18,8 @@ template <typename T>
 __global__ void embed_rows_kernel(const T *__restrict__ E, const T *__restrict__ vis,
                                   const int *__restrict__ src, int H, float *__restrict__ x,
                                   T *__restrict__ emb_out, int V, int *status) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int r = blockIdx.x;
     int s = src[r];
     const T *row;
@@ -78,8 +78,8 @@ template <typename T>
 __global__ void __launch_bounds__(RMS_THREADS) rmsnorm_kernel(const float *__restrict__ x,
                                                               const T *__restrict__ g, int H,
                                                               float eps, T *__restrict__ out) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     __shared__ float red[32];
     const int r = blockIdx.x, n4 = H >> 2;
     const float4 *xr = reinterpret_cast<const float4 *>(x + (size_t)r * H);
@@ -117,8 +117,8 @@ void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
 // ---------------------------------------------------------------------------
 template <typename T>
 __global__ void swiglu_kernel(const float *__restrict__ gu, int F, int glu, T *__restrict__ act) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int r = blockIdx.y;
     const int ld = glu ? 128 * ((F + 63) / 64) : 2 * F;
     const float *row = gu + (size_t)r * ld;
@@ -145,8 +145,8 @@ __global__ void rope_kv_kernel(const float *__restrict__ qkv, const RowDesc *__r
                                int nh, int hd, const float2 *__restrict__ tab, int max_pos,
                                T *__restrict__ q_out, T *__restrict__ kdst, T *__restrict__ vdst,
                                int slots, int *status) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int r = blockIdx.x;
     const int H = nh * hd, half = hd >> 1;
     const RowDesc d = rows[r];
@@ -256,8 +256,8 @@ __device__ __forceinline__ void warp_topk(float (&v)[NS], int (&ix)[NS], int k, 
 __global__ void __launch_bounds__(TK_THREADS)
     topk_rows_kernel(const float *__restrict__ logits, int V, int k, int *__restrict__ ids,
                      float *__restrict__ logp, float *__restrict__ ws, int *__restrict__ counters) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     constexpr int NW = TK_THREADS / 32;
     __shared__ float s_v[NW * TOPK_MAX];
     __shared__ int s_i[NW * TOPK_MAX];

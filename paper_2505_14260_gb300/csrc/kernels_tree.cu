@@ -16,8 +16,8 @@ __global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int 
                                      const T *__restrict__ pend_h, const int *__restrict__ pend_next,
                                      const T *__restrict__ E, int H, int D1, int V,
                                      T *__restrict__ xfc, RowDesc *__restrict__ rows, int *status) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int r = blockIdx.x, b = r / D1, j = r - b * D1;
     const int L = seq_len[b], P = n_pend[b];
     const bool valid = j < P;
@@ -48,8 +48,8 @@ __global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int 
 template <typename T>
 __global__ void root_gather_kernel(const float *__restrict__ x, const int *__restrict__ n_pend, int D1,
                                    int H, float *__restrict__ hhat_root, T *__restrict__ xr) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int b = blockIdx.x;
     const int r = b * D1 + max(n_pend[b] - 1, 0);
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
@@ -63,8 +63,8 @@ __global__ void root_gather_kernel(const float *__restrict__ x, const int *__res
 template <typename T>
 __global__ void hhat_store_kernel(const float *__restrict__ x, const RowDesc *__restrict__ rows,
                                   int Td, int H, float *__restrict__ hhat_slot, T *__restrict__ xb) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int r = blockIdx.x;
     const RowDesc d = rows[r];
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
@@ -111,8 +111,8 @@ __device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int tok, 
 // the candidate arrays and the frontier (buffer 0).
 template <typename T>
 __global__ void tree_init_kernel(DraftArgs<T> a) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int b = blockIdx.y, j = blockIdx.x, k = a.k;
     __shared__ float sc[TREE_MAXK];
     __shared__ int front[TREE_MAXK];
@@ -149,8 +149,8 @@ __global__ void tree_init_kernel(DraftArgs<T> a) {
 // pass d+1.
 template <typename T>
 __global__ void tree_step_kernel(DraftArgs<T> a, int d) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     extern __shared__ float smem[];
     const int b = blockIdx.y, j = blockIdx.x, k = a.k, kk = k * k;
     const int base = k + (d - 2) * kk;
@@ -197,8 +197,8 @@ __global__ void tree_finalize_kernel(TreeOut t, const int *__restrict__ cand_tok
                                      const int *__restrict__ cand_par, const int *__restrict__ cand_depth,
                                      const float *__restrict__ cand_score, int *__restrict__ node_of,
                                      const int *__restrict__ root, int C, int N, int *status) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     extern __shared__ float ssc[];   // [C]
     const int b = blockIdx.x, W = (N + 63) / 64;
     const size_t cb = (size_t)b * C;
@@ -250,8 +250,8 @@ __global__ void verify_setup_kernel(TreeIn t, const int *__restrict__ seq_len,
                                     const int *__restrict__ root, int B, int N, int V,
                                     RowDesc *__restrict__ rows, int *__restrict__ src,
                                     uint64_t *__restrict__ vmask, int *status) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int r = blockIdx.x * blockDim.x + threadIdx.x;
     if (r >= B * N) return;
     const int b = r / N, i = r - b * N, W = (N + 63) / 64;
@@ -298,8 +298,8 @@ __global__ void accept_kernel(TreeIn t, const int *__restrict__ argmax, int N, i
                               int *__restrict__ acc_a, int *__restrict__ path_out,
                               int *__restrict__ accept_len_out, int *__restrict__ bonus_out,
                               int *__restrict__ index_map_out) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int b = blockIdx.x, lane = threadIdx.x, D1 = D + 1;
     const size_t nb = (size_t)b * N;
     const int n = t.n_nodes ? t.n_nodes[b] : N;
@@ -345,8 +345,8 @@ __global__ void compact_kv_kernel(const uint4 *__restrict__ tree_kv, uint4 *__re
                                   const int *__restrict__ acc_path, const int *__restrict__ acc_L0,
                                   const int *__restrict__ acc_a, int B, int nh, int N, int S,
                                   int D1, int vec_per_row, int *status) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int lkh = blockIdx.x, b = blockIdx.y;
     const int h = lkh % nh, lk = lkh / nh;           // lk = layer*2 + kv
     const int a = acc_a[b], L0 = acc_L0[b];
@@ -369,8 +369,8 @@ template <typename T>
 __global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ acc_path,
                               const int *__restrict__ acc_a, int N, int D1, int H,
                               T *__restrict__ pend_h) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int b = blockIdx.x / D1, j = blockIdx.x - b * D1;
     if (j > acc_a[b]) return;
     const int node = acc_path[b * D1 + j];
@@ -386,8 +386,8 @@ __global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ 
 template <typename T>
 __global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict__ emb,
                                      const int *__restrict__ src, int H) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int r = blockIdx.x;
     if (src[r] >= 0) return;
     for (int c = threadIdx.x; c < H; c += blockDim.x)
@@ -399,8 +399,8 @@ __global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict_
 template <typename T>
 __global__ void concat_next_kernel(const T *__restrict__ h, const T *__restrict__ emb, int H,
                                    T *__restrict__ xfc) {
-    allow_dependents();
     wait_prior();
+    allow_dependents();
     const int r = blockIdx.x;
     for (int c = threadIdx.x; c < H; c += blockDim.x) {
         xfc[(size_t)r * 2 * H + c] = h[(size_t)r * H + c];

@@ -309,6 +309,7 @@ bool run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, in
     a.hd = c->hd;
     a.scale = 1.0f / sqrtf((float)c->hd);
     a.out = static_cast<T *>(c->attn);
+    a.cache_fresh = kdst == ck;         // this layer's own K/V go into the cache it reads
     attention<T>(c, a, rows_per_req, p_bound, s);
     GemmW wo = {{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1, lp.o};
     GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, lp.down};
