@@ -126,6 +126,98 @@ __device__ __forceinline__ float block_max(float v, float *red) {
 
 // Total order used for every top-k / argmax decision: larger value first,
 // then lower index.
+template <typename T> struct Vec4;
+template <> struct Vec4<float> {
+    static __device__ __forceinline__ float4 load(const float *g) { return *reinterpret_cast<const float4 *>(g); }
+    static __device__ __forceinline__ void store(float *o, float4 v) { *reinterpret_cast<float4 *>(o) = v; }
+};
+template <> struct Vec4<bf16> {
+    static __device__ __forceinline__ float4 load(const bf16 *g) {
+        const uint2 u = *reinterpret_cast<const uint2 *>(g);
+        const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162 *>(&u.x);
+        const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&u.y);
+        return make_float4(__low2float(a), __high2float(a), __low2float(b), __high2float(b));
+    }
+    static __device__ __forceinline__ void store(bf16 *o, float4 v) {
+        __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+        uint2 u;
+        u.x = *reinterpret_cast<uint32_t *>(&a);
+        u.y = *reinterpret_cast<uint32_t *>(&b);
+        *reinterpret_cast<uint2 *>(o) = u;
+    }
+};
+
+// Row copies of the small per-row kernels, n a multiple of 4 and rows 4-element
+// aligned: every thread of the CTA requests up to 4 groups of 4 elements (16-
+// or 8-byte accesses) before it stores any, so one pass costs about one memory
+// round trip instead of one per element.
+template <typename TD, typename TS>
+__device__ __forceinline__ void copy_row(TD *__restrict__ dst, const TS *__restrict__ src, int n) {
+    const int n4 = n >> 2;
+    for (int g0 = threadIdx.x; g0 < n4; g0 += 4 * blockDim.x) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) v[u] = Vec4<TS>::load(src + 4 * g);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) Vec4<TD>::store(dst + 4 * g, v[u]);
+        }
+    }
+}
+
+// One source row to two destinations (d2 nullable).
+template <typename TD1, typename TD2, typename TS>
+__device__ __forceinline__ void copy_row_2dst(TD1 *__restrict__ d1, TD2 *__restrict__ d2,
+                                              const TS *__restrict__ src, int n) {
+    const int n4 = n >> 2;
+    for (int g0 = threadIdx.x; g0 < n4; g0 += 4 * blockDim.x) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) v[u] = Vec4<TS>::load(src + 4 * g);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) {
+                Vec4<TD1>::store(d1 + 4 * g, v[u]);
+                if (d2) Vec4<TD2>::store(d2 + 4 * g, v[u]);
+            }
+        }
+    }
+}
+
+// Two independent row copies in one pass (s1 null: d1 gets zeros).
+template <typename TD1, typename TS1, typename TD2, typename TS2>
+__device__ __forceinline__ void copy_rows2(TD1 *__restrict__ d1, const TS1 *__restrict__ s1,
+                                           TD2 *__restrict__ d2, const TS2 *__restrict__ s2, int n) {
+    const int n4 = n >> 2;
+    for (int g0 = threadIdx.x; g0 < n4; g0 += 2 * blockDim.x) {
+        float4 a[2], b[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) {
+                a[u] = s1 ? Vec4<TS1>::load(s1 + 4 * g) : make_float4(0.f, 0.f, 0.f, 0.f);
+                b[u] = Vec4<TS2>::load(s2 + 4 * g);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) {
+                Vec4<TD1>::store(d1 + 4 * g, a[u]);
+                Vec4<TD2>::store(d2 + 4 * g, b[u]);
+            }
+        }
+    }
+}
+
 __device__ __forceinline__ bool better(float va, int ia, float vb, int ib) {
     return va > vb || (va == vb && ia < ib);
 }

@@ -32,11 +32,7 @@ __global__ void embed_rows_kernel(const T *__restrict__ E, const T *__restrict__
     } else {
         row = vis + (size_t)(-1 - s) * H;
     }
-    for (int j = threadIdx.x; j < H; j += blockDim.x) {
-        T v = row[j];
-        x[(size_t)r * H + j] = to_f(v);
-        if (emb_out) emb_out[(size_t)r * H + j] = v;
-    }
+    copy_row_2dst(x + (size_t)r * H, emb_out ? emb_out + (size_t)r * H : nullptr, row, H);
 }
 
 template <typename T>
@@ -49,27 +45,6 @@ void launch_embed_rows(const T *E, const T *vis, const int *src, int R, int H, f
 // ---------------------------------------------------------------------------
 // RMSNorm: y = x / sqrt(mean(x^2) + eps) * g
 // ---------------------------------------------------------------------------
-template <typename T> struct Vec4;
-template <> struct Vec4<float> {
-    static __device__ __forceinline__ float4 load(const float *g) { return *reinterpret_cast<const float4 *>(g); }
-    static __device__ __forceinline__ void store(float *o, float4 v) { *reinterpret_cast<float4 *>(o) = v; }
-};
-template <> struct Vec4<bf16> {
-    static __device__ __forceinline__ float4 load(const bf16 *g) {
-        const uint2 u = *reinterpret_cast<const uint2 *>(g);
-        const __nv_bfloat162 a = *reinterpret_cast<const __nv_bfloat162 *>(&u.x);
-        const __nv_bfloat162 b = *reinterpret_cast<const __nv_bfloat162 *>(&u.y);
-        return make_float4(__low2float(a), __high2float(a), __low2float(b), __high2float(b));
-    }
-    static __device__ __forceinline__ void store(bf16 *o, float4 v) {
-        __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
-        uint2 u;
-        u.x = *reinterpret_cast<uint32_t *>(&a);
-        u.y = *reinterpret_cast<uint32_t *>(&b);
-        *reinterpret_cast<uint2 *>(o) = u;
-    }
-};
-
 // One CTA per row; the row stays in registers (H <= 8 * 4 * 256).
 constexpr int RMS_THREADS = 256;
 constexpr int RMS_VEC = 8;
@@ -220,32 +195,46 @@ __device__ __forceinline__ void warp_lse(float &m, float &s) {
     }
 }
 
-// Best (value, index) of a warp; every lane gets it.
-__device__ __forceinline__ void warp_best(float &v, int &i) {
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) {
-        const float ov = __shfl_xor_sync(0xffffffffu, v, o);
-        const int oi = __shfl_xor_sync(0xffffffffu, i, o);
-        if (better(ov, oi, v, i)) { v = ov; i = oi; }
-    }
+// Order-preserving 32-bit key of a logit: larger value, larger key; -0 as +0
+// and NaN lowest, as in better().
+__device__ __forceinline__ unsigned tk_key(float v) {
+    if (v != v) return 0u;
+    const unsigned u = __float_as_uint(v == 0.f ? 0.f : v);
+    return u ^ ((u >> 31) ? 0xffffffffu : 0x80000000u);
+}
+__device__ __forceinline__ float tk_value(unsigned key) {
+    return __uint_as_float(key ^ ((key >> 31) ? 0x80000000u : 0xffffffffu));
 }
 
 // Top-k of the NS (value, index) slots held by each lane of a warp, in k
-// rounds of warp arg-max: the winner's slot is retired by index (indices are
-// unique), so no slot is ever indexed dynamically. Lane 0 gets the result.
+// rounds: every lane keeps its best remaining slot (its head); a round takes
+// the warp's best head with two single-instruction warp reductions (largest
+// key, then lowest index among the lanes holding it), and only the winning
+// lane retires that slot (by index: indices are unique, so no slot is indexed
+// dynamically) and rescans for its next head. Lane 0 gets the result.
 template <int NS>
 __device__ __forceinline__ void warp_topk(float (&v)[NS], int (&ix)[NS], int k, float *out_v, int *out_i) {
+    float hv = -INFINITY;
+    int hi = TK_NONE;
+#pragma unroll
+    for (int e = 0; e < NS; ++e)
+        if (better(v[e], ix[e], hv, hi)) { hv = v[e]; hi = ix[e]; }
     for (int t = 0; t < k; ++t) {
-        float bv = -INFINITY;
-        int bi = TK_NONE;
+        const unsigned hk = tk_key(hv);
+        const unsigned mk = __reduce_max_sync(0xffffffffu, hk);
+        const unsigned mi = __reduce_min_sync(0xffffffffu, hk == mk ? (unsigned)hi : 0xffffffffu);
+        if ((threadIdx.x & 31) == 0) { out_v[t] = tk_value(mk); out_i[t] = (int)mi; }
+        if (hk == mk && (unsigned)hi == mi) {
 #pragma unroll
-        for (int e = 0; e < NS; ++e)
-            if (better(v[e], ix[e], bv, bi)) { bv = v[e]; bi = ix[e]; }
-        warp_best(bv, bi);
+            for (int e = 0; e < NS; ++e)
+                if (ix[e] == hi) { v[e] = -INFINITY; ix[e] = TK_NONE; }
+            hv = -INFINITY;
+            hi = TK_NONE;
 #pragma unroll
-        for (int e = 0; e < NS; ++e)
-            if (ix[e] == bi) { v[e] = -INFINITY; ix[e] = TK_NONE; }
-        if ((threadIdx.x & 31) == 0) { out_v[t] = bv; out_i[t] = bi; }
+            for (int e = 0; e < NS; ++e)
+                if (better(v[e], ix[e], hv, hi)) { hv = v[e]; hi = ix[e]; }
+        }
+        __syncwarp();
     }
 }
 

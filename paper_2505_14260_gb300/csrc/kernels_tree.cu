@@ -36,12 +36,7 @@ __global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int 
         tok = 0;
     }
     T *dst = xfc + (size_t)r * 2 * H;
-    const T *hsrc = pend_h + (size_t)(b * D1 + j) * H;
-    const T *esrc = E + (size_t)tok * H;
-    for (int c = threadIdx.x; c < H; c += blockDim.x) {
-        dst[c] = valid ? hsrc[c] : from_f<T>(0.f);
-        dst[H + c] = esrc[c];
-    }
+    copy_rows2(dst, valid ? pend_h + (size_t)(b * D1 + j) * H : nullptr, dst + H, E + (size_t)tok * H, H);
 }
 
 // h_hat of the root slot = draft output of the last pending row.
@@ -52,11 +47,7 @@ __global__ void root_gather_kernel(const float *__restrict__ x, const int *__res
     allow_dependents();
     const int b = blockIdx.x;
     const int r = b * D1 + max(n_pend[b] - 1, 0);
-    for (int c = threadIdx.x; c < H; c += blockDim.x) {
-        const float v = x[(size_t)r * H + c];
-        hhat_root[(size_t)b * H + c] = v;
-        xr[(size_t)b * H + c] = from_f<T>(v);
-    }
+    copy_row_2dst(hhat_root + (size_t)b * H, xr + (size_t)b * H, x + (size_t)r * H, H);
 }
 
 // Store h_hat of a tree pass's rows by slot, and a T copy for the LM head.
@@ -67,11 +58,7 @@ __global__ void hhat_store_kernel(const float *__restrict__ x, const RowDesc *__
     allow_dependents();
     const int r = blockIdx.x;
     const RowDesc d = rows[r];
-    for (int c = threadIdx.x; c < H; c += blockDim.x) {
-        const float v = x[(size_t)r * H + c];
-        hhat_slot[((size_t)d.req * Td + d.dst) * H + c] = v;
-        xb[(size_t)r * H + c] = from_f<T>(v);
-    }
+    copy_row_2dst(hhat_slot + ((size_t)d.req * Td + d.dst) * H, xb + (size_t)r * H, x + (size_t)r * H, H);
 }
 
 // Assemble the draft-pass row j of request b for a frontier node with token
@@ -99,11 +86,7 @@ __device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int tok, 
     }
     if (tok < 0 || tok >= a.V) tok = 0;
     T *dst = a.xfc + (size_t)r * 2 * H;
-    const T *e = a.E + (size_t)tok * H;
-    for (int q = threadIdx.x; q < H; q += blockDim.x) {
-        dst[q] = from_f<T>(parent_h[q]);
-        dst[H + q] = e[q];
-    }
+    copy_rows2(dst, parent_h, dst + H, a.E + (size_t)tok * H, H);
 }
 
 // Depth-1 candidates from the root slot's top-k; the frontier of pass 2 is all
@@ -192,46 +175,61 @@ __global__ void tree_step_kernel(DraftArgs<T> a, int d) {
 }
 
 // Final tree: the N-1 best candidates (score desc, creation asc), tree index
-// 1 + rank; parents, depths and ancestor masks; the root is node 0.
+// 1 + rank; parents, depths and ancestor masks; the root is node 0. Scores,
+// parents and tree indices of all candidates sit in shared memory, so the
+// ancestor walks read no global memory.
+constexpr int FIN_MAXW = 4;      // mask words of a node (tree_nodes <= 256)
+
 __global__ void tree_finalize_kernel(TreeOut t, const int *__restrict__ cand_tok,
                                      const int *__restrict__ cand_par, const int *__restrict__ cand_depth,
                                      const float *__restrict__ cand_score, int *__restrict__ node_of,
                                      const int *__restrict__ root, int C, int N, int *status) {
     wait_prior();
     allow_dependents();
-    extern __shared__ float ssc[];   // [C]
+    extern __shared__ float ssc[];   // [C] scores, then [C] parents, [C] tree indices
+    int *spar = reinterpret_cast<int *>(ssc + C), *snode = spar + C;
     const int b = blockIdx.x, W = (N + 63) / 64;
     const size_t cb = (size_t)b * C;
-    for (int c = threadIdx.x; c < C; c += blockDim.x) ssc[c] = cand_score[cb + c];
+    for (int c = threadIdx.x; c < C; c += blockDim.x) {
+        ssc[c] = cand_score[cb + c];
+        spar[c] = cand_par[cb + c];
+    }
     __syncthreads();
     for (int c = threadIdx.x; c < C; c += blockDim.x) {
         int rank = 0;
         const float s = ssc[c];
         for (int u = 0; u < C; ++u) rank += better(ssc[u], u, s, c);
-        node_of[cb + c] = rank < N - 1 ? 1 + rank : -1;
+        const int node = rank < N - 1 ? 1 + rank : -1;
+        snode[c] = node;
+        node_of[cb + c] = node;
     }
     __syncthreads();
     const size_t nb = (size_t)b * N;
     for (int c = threadIdx.x; c < C; c += blockDim.x) {
-        const int i = node_of[cb + c];
+        const int i = snode[c];
         if (i < 0) continue;
         t.tokens[nb + i] = cand_tok[cb + c];
         t.depth[nb + i] = cand_depth[cb + c];
-        const int p = cand_par[cb + c];
-        int pi = p < 0 ? 0 : node_of[cb + p];
+        const int p = spar[c];
+        int pi = p < 0 ? 0 : snode[p];
         if (pi < 0 || pi >= i) { set_status(status, ST_BAD_TREE); pi = 0; }
         t.parent[nb + i] = pi;
-        for (int w = 0; w < W; ++w) t.mask[(nb + i) * W + w] = 0ull;
         // ancestors-or-self: walk the candidate chain, then the root
+        uint64_t mw[FIN_MAXW] = {0ull, 0ull, 0ull, 0ull};
         int cur = c, node = i;
         while (true) {
-            t.mask[(nb + i) * W + node / 64] |= 1ull << (node % 64);
+#pragma unroll
+            for (int w = 0; w < FIN_MAXW; ++w)
+                if (w == (node >> 6)) mw[w] |= 1ull << (node & 63);
             if (cur < 0) break;
-            const int pc = cand_par[cb + cur];
-            node = pc < 0 ? 0 : node_of[cb + pc];
+            const int pc = spar[cur];
+            node = pc < 0 ? 0 : snode[pc];
             if (node < 0) break;
             cur = pc;
         }
+#pragma unroll
+        for (int w = 0; w < FIN_MAXW; ++w)
+            if (w < W) t.mask[(nb + i) * W + w] = mw[w];
     }
     if (threadIdx.x == 0) {
         t.tokens[nb] = root[b];
@@ -375,8 +373,7 @@ __global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ 
     if (j > acc_a[b]) return;
     const int node = acc_path[b * D1 + j];
     const T *s = hT + ((size_t)b * N + node) * H;
-    T *d = pend_h + ((size_t)b * D1 + j) * H;
-    for (int c = threadIdx.x; c < H; c += blockDim.x) d[c] = s[c];
+    copy_row(pend_h + ((size_t)b * D1 + j) * H, s, H);
 }
 
 // ---------------------------------------------------------------------------
@@ -390,8 +387,7 @@ __global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict_
     allow_dependents();
     const int r = blockIdx.x;
     if (src[r] >= 0) return;
-    for (int c = threadIdx.x; c < H; c += blockDim.x)
-        x[(size_t)r * H + c] = to_f(emb[(size_t)r * H + c]);
+    copy_row(x + (size_t)r * H, emb + (size_t)r * H, H);
 }
 
 // Concat(h_i, e_{i+1}) rows for the draft prefill (text positions; visual rows
@@ -402,10 +398,7 @@ __global__ void concat_next_kernel(const T *__restrict__ h, const T *__restrict_
     wait_prior();
     allow_dependents();
     const int r = blockIdx.x;
-    for (int c = threadIdx.x; c < H; c += blockDim.x) {
-        xfc[(size_t)r * 2 * H + c] = h[(size_t)r * H + c];
-        xfc[(size_t)r * 2 * H + H + c] = emb[(size_t)(r + 1) * H + c];
-    }
+    copy_rows2(xfc + (size_t)r * 2 * H, h + (size_t)r * H, xfc + (size_t)r * 2 * H + H, emb + (size_t)(r + 1) * H, H);
 }
 
 template <typename T>
@@ -423,7 +416,7 @@ __global__ void prefill_finish_kernel(const int *__restrict__ argmax1, const T *
         pend_next[b * D1] = x;
         if (root_out) root_out[b] = x;
     }
-    for (int c = threadIdx.x; c < H; c += blockDim.x) pend_h[(size_t)b * D1 * H + c] = h_last[c];
+    copy_row(pend_h + (size_t)b * D1 * H, h_last, H);
 }
 
 // ---------------------------------------------------------------------------
@@ -465,8 +458,15 @@ void launch_tree_step(const DraftArgs<T> &a, int B, int d, cudaStream_t s) {
 void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand_par,
                           const int *cand_depth, const float *cand_score, int *node_of,
                           const int *root, int B, int C, int N, int *status, cudaStream_t s) {
-    launch_pdl(tree_finalize_kernel, B, 512, (size_t)C * sizeof(float), s, 
-        t, cand_tok, cand_par, cand_depth, cand_score, node_of, root, C, N, status); note_launch();
+    const size_t smem = (size_t)C * 3 * sizeof(float);
+    static bool attr = false;       // candidate arrays beyond 48 KB (deep, wide trees)
+    if (!attr) {
+        cudaFuncSetAttribute(tree_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
+        attr = true;
+    }
+    launch_pdl(tree_finalize_kernel, B, 512, smem, s, t, cand_tok, cand_par, cand_depth, cand_score, node_of,
+               root, C, N, status);
+    note_launch();
 }
 
 void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, int B, int N,
