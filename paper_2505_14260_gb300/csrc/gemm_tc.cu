@@ -749,17 +749,17 @@ __device__ __forceinline__ float4 c_dsmem_ld4(uint32_t local, uint32_t rank) {
     float4 v;
     asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
                  : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(a)
-                 : "memory");
+                 : "r"(a));
     return v;
 }
 
+// (no memory clobber: the partials are read only after a barrier, which is
+// itself a compiler barrier, and the loads may overlap one another)
 __device__ __forceinline__ float4 c_smem_ld4(uint32_t local) {
     float4 v;
     asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
                  : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(local)
-                 : "memory");
+                 : "r"(local));
     return v;
 }
 
@@ -768,154 +768,237 @@ __device__ __forceinline__ uint2 c_pack_bf16x4(float a, float b, float c, float 
     return make_uint2(*reinterpret_cast<const uint32_t *>(&lo), *reinterpret_cast<const uint32_t *>(&hi));
 }
 
-// Paired epilogue over the tile's S partials ([BN][128] fp32 in each cluster
-// CTA's shared memory at part_s): element pairs (r, r + half) of one token,
-// with half = 64 for SwiGLU (gate row, up row) and hd/2 for RoPE (rotate-half
-// partners inside one head). This CTA takes its rank's share of the BN * 64
-// pairs, four consecutive rows at a time; the S partials are summed in rank
-// order, as in the plain reduction.
-__device__ __forceinline__ void c_epilogue_paired(const CkParams &p, uint32_t part_s, uint32_t rank,
-                                                  int S, bool ok, int seg, int wt, int row0, int n0,
-                                                  int rows_here, const float *rinv) {
-    const GemmFused &f = p.fx;
-    const bool glu = p.epi == EPI_SWIGLU;
-    const int half = glu ? 64 : (f.hd >> 1), hd = 2 * half;
-    const int n4 = p.BN * 16;
-    const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
-    for (int e = lo + threadIdx.x; e < hi; e += C_THREADS) {
-        const int col = e >> 4, p4 = (e & 15) * 4;
-        const int r = (p4 / half) * hd + (p4 % half);
-        const uint32_t oa = part_s + (uint32_t)(col * BM + r) * 4u, ob = oa + (uint32_t)half * 4u;
-        float4 va[8], vb[8];
-        if (S == 1) {
-            va[0] = c_smem_ld4(oa);
-            vb[0] = c_smem_ld4(ob);
-        } else {
+// Generic address of the same shared-memory location in cluster CTA `rank`
+// (plain loads through it read distributed shared memory; a pure function, so
+// the compiler may schedule the loads freely).
+__device__ __forceinline__ const float4 *c_map_rank(const float4 *p, uint32_t rank) {
+    uint64_t r;
+    asm("mapa.u64 %0, %1, %2;" : "=l"(r) : "l"(reinterpret_cast<uint64_t>(p)), "r"(rank));
+    return reinterpret_cast<const float4 *>(r);
+}
+
+// Sums, in rank order, of the S partials' float4 at K offsets (in float4) of
+// the partial buffer `part` (each cluster CTA's partial sits at the same
+// offset; S == 1: local). All loads are issued before the first sum.
+template <int K>
+__device__ __forceinline__ void c_part_sums(const float4 *part, const int (&idx)[K], const bool (&use)[K], int S,
+                                            float4 (&out)[K]) {
+    float4 v[K][8];
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
-                if (q < S) {
-                    va[q] = c_dsmem_ld4(oa, q);
-                    vb[q] = c_dsmem_ld4(ob, q);
-                }
-        }
-        float a[4] = {0.f, 0.f, 0.f, 0.f}, b[4] = {0.f, 0.f, 0.f, 0.f};
+    for (int q = 0; q < 8; ++q) {
+        if (q >= S) break;
+        const float4 *src = S == 1 ? part : c_map_rank(part, (uint32_t)q);
+#pragma unroll
+        for (int k = 0; k < K; ++k)
+            if (use[k]) v[k][q] = src[idx[k]];
+    }
+#pragma unroll
+    for (int k = 0; k < K; ++k) {
+        float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
         for (int q = 0; q < 8; ++q)
-            if (q < S) {
-                a[0] += va[q].x; a[1] += va[q].y; a[2] += va[q].z; a[3] += va[q].w;
-                b[0] += vb[q].x; b[1] += vb[q].y; b[2] += vb[q].z; b[3] += vb[q].w;
+            if (q < S && use[k]) {
+                a.x += v[k][q].x; a.y += v[k][q].y; a.z += v[k][q].z; a.w += v[k][q].w;
             }
-        const int m = n0 + col;
-        if (!ok || m >= p.M) continue;
-        if (rinv) {                                   // folded RMSNorm: the row's 1/rms
-            const float sc = rinv[col];
+        out[k] = a;
+    }
+}
+
+// The fused epilogues read the tile's S partials ([BN][128] fp32 in each
+// cluster CTA's shared memory at part_s) and take this CTA's rank share of the
+// BN * 16 groups of four rows of one token; the partials are summed in rank
+// order, as in the plain reduction. Each thread handles two groups per pass,
+// with every load of both issued before either is used, so that a pass costs
+// about one round trip to distributed shared memory and one to global memory.
+
+// SwiGLU (glu-packed tile: rows 0-63 gate, 64-127 up):
+// act[m][64 t + i] = bf16(silu(g) * u), scaled first by the folded-norm 1/rms.
+__device__ __forceinline__ void c_epi_swiglu(const CkParams &p, const float4 *part, uint32_t rank, int S,
+                                             bool ok, int wt, int n0, const float *rinv) {
+    bf16 *const act = p.fx.act;
+    const int F = p.fx.F, M = p.M, n4 = p.BN * 16;
+    const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
+    for (int e0 = lo + threadIdx.x; e0 < hi; e0 += 2 * C_THREADS) {
+        int ad[4];
+        bool use[4];
+        int col[2], p4[2];
 #pragma unroll
-            for (int t = 0; t < 4; ++t) {
-                a[t] *= sc;
-                b[t] *= sc;
-            }
+        for (int u = 0; u < 2; ++u) {
+            const int e = e0 + u * C_THREADS;
+            col[u] = e >> 4;
+            p4[u] = (e & 15) << 2;
+            ad[2 * u] = (col[u] * BM + p4[u]) >> 2;
+            ad[2 * u + 1] = ad[2 * u] + 16;
+            use[2 * u] = use[2 * u + 1] = e < hi;
         }
-        if (glu) {
-            const int j = wt * 64 + p4;
-            if (j >= f.F) continue;                 // F % 4 == 0: whole groups
-            float o[4];
+        float4 v[4];
+        c_part_sums<4>(part, ad, use, S, v);
 #pragma unroll
-            for (int t = 0; t < 4; ++t) o[t] = a[t] / (1.f + __expf(-a[t])) * b[t];
-            *reinterpret_cast<uint2 *>(f.act + (size_t)m * f.F + j) = c_pack_bf16x4(o[0], o[1], o[2], o[3]);
-            continue;
-        }
-        if (r >= rows_here) continue;
-        const int o = row0 + r, h = o / hd, i = o - h * hd;
-        const RowDesc d = f.rows[m];
-        if (seg < 2) {
-            int pos = d.pos;
-            if (pos < 0 || pos >= f.max_pos) {
-                set_status(p.status, ST_RANGE);
-                pos = 0;
+        for (int u = 0; u < 2; ++u) {
+            float4 a = v[2 * u], b = v[2 * u + 1];
+            const int m = n0 + col[u], j = wt * 64 + p4[u];
+            if (!use[2 * u] || !ok || m >= M || j >= F) continue;     // F % 4 == 0: whole groups
+            if (rinv) {
+                const float sc = rinv[col[u]];
+                a.x *= sc; a.y *= sc; a.z *= sc; a.w *= sc;
+                b.x *= sc; b.y *= sc; b.z *= sc; b.w *= sc;
             }
-            const float4 *cs = reinterpret_cast<const float4 *>(f.rope_tab + (size_t)pos * half + i);
-            const float4 c01 = cs[0], c23 = cs[1];
-            const float cx[4] = {c01.x, c01.z, c23.x, c23.z}, sy[4] = {c01.y, c01.w, c23.y, c23.w};
+            const float o0 = __fdividef(a.x, 1.f + __expf(-a.x)) * b.x;
+            const float o1 = __fdividef(a.y, 1.f + __expf(-a.y)) * b.y;
+            const float o2 = __fdividef(a.z, 1.f + __expf(-a.z)) * b.z;
+            const float o3 = __fdividef(a.w, 1.f + __expf(-a.w)) * b.w;
+            *reinterpret_cast<uint2 *>(act + (size_t)m * F + j) = c_pack_bf16x4(o0, o1, o2, o3);
+        }
+    }
+}
+
+// RoPE + K/V placement (tile of wq;wk;wv rows, hd | 128): rotate-half pairs
+// (i, i + hd/2) of one head; q rotated into q_out [M][H], k rotated and v into
+// kdst / vdst [B][nh][slots][hd] at the row's slot. Row descriptors come from
+// shared memory (loaded while the MMAs ran).
+__device__ __forceinline__ void c_epi_rope(const CkParams &p, const float4 *part, uint32_t rank, int S,
+                                           bool ok, int seg, int row0, int n0, int rows_here,
+                                           const float *rinv, const RowDesc *srow) {
+    const GemmFused &f = p.fx;
+    const int hd = f.hd, lh = hd == 128 ? 6 : 5, half = 1 << lh, lhd = lh + 1;
+    const float2 *const rope_tab = f.rope_tab;
+    const int max_pos = f.max_pos, slots = f.slots, nh = f.nh, M = p.M;
+    bf16 *const qo = f.q_out, *const kvd = seg == 1 ? f.kdst : f.vdst;
+    const int n4 = p.BN * 16;
+    const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
+    for (int e0 = lo + threadIdx.x; e0 < hi; e0 += 2 * C_THREADS) {
+        int ad[4];
+        bool use[4];
+        int col[2], r[2];
+        bool live[2];
+        RowDesc d[2];
+        float4 c01[2], c23[2];
 #pragma unroll
-            for (int t = 0; t < 4; ++t) {
-                const float x0 = a[t], x1 = b[t];
-                a[t] = x0 * cx[t] - x1 * sy[t];
-                b[t] = x1 * cx[t] + x0 * sy[t];
+        for (int u = 0; u < 2; ++u) {
+            const int e = e0 + u * C_THREADS;
+            col[u] = e >> 4;
+            const int p4 = (e & 15) << 2;
+            r[u] = ((p4 >> lh) << lhd) | (p4 & (half - 1));
+            ad[2 * u] = (col[u] * BM + r[u]) >> 2;
+            ad[2 * u + 1] = ad[2 * u] + (half >> 2);
+            use[2 * u] = use[2 * u + 1] = e < hi;
+            live[u] = e < hi && ok && n0 + col[u] < M && r[u] < rows_here;
+            d[u] = live[u] ? srow[col[u]] : RowDesc{0, 0, 0, -1};
+            if (live[u] && seg < 2) {                 // the rotation's table entries, in flight early
+                int pos = d[u].pos;
+                if (pos < 0 || pos >= max_pos) {
+                    set_status(p.status, ST_RANGE);
+                    pos = 0;
+                }
+                const int i = (row0 + r[u]) & (hd - 1);
+                const float4 *cs = reinterpret_cast<const float4 *>(rope_tab + (size_t)pos * half + i);
+                c01[u] = cs[0];
+                c23[u] = cs[1];
             }
         }
-        bf16 *dst;
-        if (seg == 0) {
-            dst = f.q_out + (size_t)m * (f.nh * hd) + o;
-        } else {
-            if (d.dst >= f.slots) set_status(p.status, ST_RANGE);
-            if (d.dst < 0 || d.dst >= f.slots) continue;
-            dst = (seg == 1 ? f.kdst : f.vdst) + ((size_t)(d.req * f.nh + h) * f.slots + d.dst) * hd + i;
+        float4 v[4];
+        c_part_sums<4>(part, ad, use, S, v);
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            if (!live[u]) continue;
+            float4 a = v[2 * u], b = v[2 * u + 1];
+            if (rinv) {
+                const float sc = rinv[col[u]];
+                a.x *= sc; a.y *= sc; a.z *= sc; a.w *= sc;
+                b.x *= sc; b.y *= sc; b.z *= sc; b.w *= sc;
+            }
+            const int m = n0 + col[u], o = row0 + r[u], h = o >> lhd, i = o & (hd - 1);
+            if (seg < 2) {
+                const float x0 = a.x, x1 = a.y, x2 = a.z, x3 = a.w;
+                a.x = x0 * c01[u].x - b.x * c01[u].y; b.x = b.x * c01[u].x + x0 * c01[u].y;
+                a.y = x1 * c01[u].z - b.y * c01[u].w; b.y = b.y * c01[u].z + x1 * c01[u].w;
+                a.z = x2 * c23[u].x - b.z * c23[u].y; b.z = b.z * c23[u].x + x2 * c23[u].y;
+                a.w = x3 * c23[u].z - b.w * c23[u].w; b.w = b.w * c23[u].z + x3 * c23[u].w;
+            }
+            bf16 *dst;
+            if (seg == 0) {
+                dst = qo + (size_t)m * (nh * hd) + o;
+            } else {
+                if (d[u].dst >= slots) set_status(p.status, ST_RANGE);
+                if (d[u].dst < 0 || d[u].dst >= slots) continue;
+                dst = kvd + ((size_t)(d[u].req * nh + h) * slots + d[u].dst) * hd + i;
+            }
+            *reinterpret_cast<uint2 *>(dst) = c_pack_bf16x4(a.x, a.y, a.z, a.w);
+            *reinterpret_cast<uint2 *>(dst + half) = c_pack_bf16x4(b.x, b.y, b.z, b.w);
         }
-        *reinterpret_cast<uint2 *>(dst) = c_pack_bf16x4(a[0], a[1], a[2], a[3]);
-        *reinterpret_cast<uint2 *>(dst + half) = c_pack_bf16x4(b[0], b[1], b[2], b[3]);
     }
 }
 
 // Producer side of a folded RMSNorm: this CTA's share of the tile's token
-// columns, one warp per column (lane = 4 consecutive weight rows): the S
-// partials summed in rank order, the residual added, then Y (fp32), xg =
-// bf16(y * g) and the column's sum of squares over the tile's rows (a warp
-// reduction in a fixed order) into ss[m][tile].
-__device__ __forceinline__ void c_reduce_norm(const CkParams &p, uint32_t part_s, uint32_t rank, int S,
+// columns, one warp per column (lane = 4 consecutive weight rows), two columns
+// of a warp per pass: the S partials summed in rank order, the residual added,
+// then Y (fp32), xg = bf16(y * g) and the column's sum of squares over the
+// tile's rows (a warp reduction in a fixed order) into ss[m][tile].
+__device__ __forceinline__ void c_reduce_norm(const CkParams &p, const float4 *part, uint32_t rank, int S,
                                               bool ok, int tile, int o_base, int rows_here, int n0) {
+    constexpr int NW = C_THREADS / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const bool add = p.epi == EPI_ADD;
     const int c_lo = (int)((long long)rank * p.BN / S), c_hi = (int)((long long)(rank + 1) * p.BN / S);
     const int r4 = lane * 4;
-    for (int c = c_lo + warp; c < c_hi; c += C_THREADS / 32) {
-        const uint32_t addr = part_s + (uint32_t)(c * BM + r4) * 4u;
-        float4 v[8];
-        if (S == 1) {
-            v[0] = c_smem_ld4(addr);
-        } else {
+    const bool full = r4 + 4 <= rows_here;
+    float g4[4] = {0.f, 0.f, 0.f, 0.f};
+    if (full) {
+        const uint2 gw = *reinterpret_cast<const uint2 *>(p.nout.g + o_base + r4);
+        const __nv_bfloat162 g01 = *reinterpret_cast<const __nv_bfloat162 *>(&gw.x);
+        const __nv_bfloat162 g23 = *reinterpret_cast<const __nv_bfloat162 *>(&gw.y);
+        g4[0] = __low2float(g01); g4[1] = __high2float(g01);
+        g4[2] = __low2float(g23); g4[3] = __high2float(g23);
+    }
+    float *const Y = p.Y;
+    bf16 *const XG = p.nout.xg;
+    const int ldy = p.ldy, M = p.M;
+    for (int c0 = c_lo + warp; c0 < c_hi; c0 += 2 * NW) {
+        int ad[2];
+        bool use[2], live[2];
+        float4 yi[2];
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
-                if (q < S) v[q] = c_dsmem_ld4(addr, q);
+        for (int u = 0; u < 2; ++u) {
+            const int c = c0 + u * NW;
+            ad[u] = (c * BM + r4) >> 2;
+            use[u] = c < c_hi;
+            live[u] = use[u] && ok && n0 + c < M;        // warp-uniform
+            yi[u] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (live[u] && full && add)
+                yi[u] = *reinterpret_cast<const float4 *>(Y + (size_t)(n0 + c) * ldy + o_base + r4);
         }
-        float a[4] = {0.f, 0.f, 0.f, 0.f};
+        float4 v[2];
+        c_part_sums<2>(part, ad, use, S, v);
 #pragma unroll
-        for (int q = 0; q < 8; ++q)
-            if (q < S) {
-                a[0] += v[q].x; a[1] += v[q].y; a[2] += v[q].z; a[3] += v[q].w;
-            }
-        const int m = n0 + c;
-        const bool live = ok && m < p.M;                  // warp-uniform
-        float ss = 0.f;
-        if (live) {
-            float *y = p.Y + (size_t)m * p.ldy + o_base + r4;
-            bf16 *xg = p.nout.xg + (size_t)m * p.ldy + o_base + r4;
-            const bf16 *g = p.nout.g + o_base + r4;
-            if (r4 + 4 <= rows_here) {
-                if (add) {
-                    const float4 yi = *reinterpret_cast<const float4 *>(y);
-                    a[0] += yi.x; a[1] += yi.y; a[2] += yi.z; a[3] += yi.w;
+        for (int u = 0; u < 2; ++u) {
+            if (!use[u]) continue;
+            const int m = n0 + c0 + u * NW;
+            float a[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
+            float ss = 0.f;
+            if (live[u]) {
+                float *y = Y + (size_t)m * ldy + o_base + r4;
+                bf16 *xg = XG + (size_t)m * ldy + o_base + r4;
+                if (full) {
+                    a[0] += yi[u].x; a[1] += yi[u].y; a[2] += yi[u].z; a[3] += yi[u].w;
+                    *reinterpret_cast<float4 *>(y) = make_float4(a[0], a[1], a[2], a[3]);
+                    *reinterpret_cast<uint2 *>(xg) =
+                        c_pack_bf16x4(a[0] * g4[0], a[1] * g4[1], a[2] * g4[2], a[3] * g4[3]);
+                    ss = a[0] * a[0] + a[1] * a[1] + a[2] * a[2] + a[3] * a[3];
+                } else {
+                    const bf16 *g = p.nout.g + o_base + r4;
+#pragma unroll
+                    for (int e = 0; e < 4; ++e)
+                        if (r4 + e < rows_here) {
+                            const float ye = add ? y[e] + a[e] : a[e];
+                            y[e] = ye;
+                            xg[e] = __float2bfloat16_rn(ye * __bfloat162float(g[e]));
+                            ss += ye * ye;
+                        }
                 }
-                *reinterpret_cast<float4 *>(y) = make_float4(a[0], a[1], a[2], a[3]);
-                const uint2 gw = *reinterpret_cast<const uint2 *>(g);
-                const __nv_bfloat162 g01 = *reinterpret_cast<const __nv_bfloat162 *>(&gw.x);
-                const __nv_bfloat162 g23 = *reinterpret_cast<const __nv_bfloat162 *>(&gw.y);
-                *reinterpret_cast<uint2 *>(xg) =
-                    c_pack_bf16x4(a[0] * __low2float(g01), a[1] * __high2float(g01),
-                                  a[2] * __low2float(g23), a[3] * __high2float(g23));
-                ss = a[0] * a[0] + a[1] * a[1] + a[2] * a[2] + a[3] * a[3];
-            } else {
-#pragma unroll
-                for (int e = 0; e < 4; ++e)
-                    if (r4 + e < rows_here) {
-                        const float ye = add ? y[e] + a[e] : a[e];
-                        y[e] = ye;
-                        xg[e] = __float2bfloat16_rn(ye * __bfloat162float(g[e]));
-                        ss += ye * ye;
-                    }
             }
+            ss = warp_sum(ss);
+            if (live[u] && lane == 0) p.nout.ss[(size_t)m * p.nout.ld + tile] = ss;
         }
-        ss = warp_sum(ss);
-        if (live && lane == 0) p.nout.ss[(size_t)m * p.nout.ld + tile] = ss;
     }
 }
 
@@ -926,6 +1009,7 @@ __global__ void __launch_bounds__(C_THREADS)
     __shared__ uint32_t tmem_base;
     __shared__ volatile int abort_flag;
     __shared__ float s_rinv[128];     // folded RMSNorm (consumer): 1/rms of each token column
+    __shared__ RowDesc s_rows[128];   // EPI_ROPE_KV: the token columns' row descriptors
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int wt = blockIdx.x, seg = 0;
@@ -1038,6 +1122,11 @@ __global__ void __launch_bounds__(C_THREADS)
                     for (int j = 0; j < p.nin.parts; ++j) sum += p.nin.ss[(size_t)m * p.nin.ld + j];
                 s_rinv[t] = rsqrtf(sum / (float)p.nin.H + p.nin.eps);
             }
+        if (p.epi == EPI_ROPE_KV)
+            for (int t = threadIdx.x - 64; t < p.BN; t += C_THREADS - 64) {
+                const int m = n0 + t;
+                s_rows[t] = m < p.M ? p.fx.rows[m] : RowDesc{0, 0, 0, -1};
+            }
     }
 
     // ---- epilogue: all 4 warps, TMEM lane quarter = warp -------------------
@@ -1095,12 +1184,16 @@ __global__ void __launch_bounds__(C_THREADS)
         else __syncthreads();
         const uint32_t rank = S > 1 ? c_cluster_rank() : 0u;
         const uint32_t part_s = smem_u32(part);
-        if (paired) c_epilogue_paired(p, part_s, rank, S, ok, seg, wt, row0, n0, rows_here,
-                                      p.nin.ss ? s_rinv : nullptr);
-        else if (norm_out) c_reduce_norm(p, part_s, rank, S, ok, wt, o_base, rows_here, n0);
+        const float4 *part4 = reinterpret_cast<const float4 *>(part);
+        if (p.epi == EPI_SWIGLU)
+            c_epi_swiglu(p, part4, rank, S, ok, wt, n0, p.nin.ss ? s_rinv : nullptr);
+        else if (paired)
+            c_epi_rope(p, part4, rank, S, ok, seg, row0, n0, rows_here, p.nin.ss ? s_rinv : nullptr, s_rows);
+        else if (norm_out) c_reduce_norm(p, part4, rank, S, ok, wt, o_base, rows_here, n0);
         // this CTA's slice of the tile, as float4 (4 consecutive weight rows of one token)
         const int n4 = BN * BM / 4;
         const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
+#pragma unroll 2
         for (int e4 = lo + threadIdx.x; !paired && !norm_out && e4 < hi; e4 += C_THREADS) {
             float4 v[8];
 #pragma unroll

@@ -213,7 +213,8 @@ __device__ __forceinline__ float tk_value(unsigned key) {
 // lane retires that slot (by index: indices are unique, so no slot is indexed
 // dynamically) and rescans for its next head. Lane 0 gets the result.
 template <int NS>
-__device__ __forceinline__ void warp_topk(float (&v)[NS], int (&ix)[NS], int k, float *out_v, int *out_i) {
+__device__ __forceinline__ void warp_topk_rounds(float (&v)[NS], int (&ix)[NS], int k, float *out_v,
+                                                 int *out_i) {
     float hv = -INFINITY;
     int hi = TK_NONE;
 #pragma unroll
@@ -238,6 +239,74 @@ __device__ __forceinline__ void warp_topk(float (&v)[NS], int (&ix)[NS], int k, 
     }
 }
 
+// Top-k of a warp's NS slots per lane by threshold and rank. The k-th best of
+// the 32 lane heads (ranked by counting) is a threshold that at least k slots
+// reach; the slots that reach it (NaN and empty slots never do) are compacted
+// into the warp's 32-entry scratch and each ranked by counting how many beat
+// it, so no step is repeated k times. More than 32 such slots (heavy ties)
+// falls back to warp_topk_rounds. The result is the same ordered list as
+// warp_topk_rounds: larger value first, then lower index; (-inf, TK_NONE)
+// fills the places beyond the valid slots. Written by the lanes that own a
+// place; the caller synchronises the warp before reading it.
+template <int NS>
+__device__ __forceinline__ void warp_topk(float (&v)[NS], int (&ix)[NS], int k, float *out_v, int *out_i,
+                                          float *scr_v, int *scr_i) {
+    const int lane = threadIdx.x & 31;
+    float hv = -INFINITY;
+    int hi = TK_NONE;
+#pragma unroll
+    for (int e = 0; e < NS; ++e)
+        if (better(v[e], ix[e], hv, hi)) { hv = v[e]; hi = ix[e]; }
+    // rank of this lane's head among the 32 heads
+    int hr = 0;
+#pragma unroll 8
+    for (int j = 0; j < 32; ++j) {
+        const float ov = __shfl_sync(0xffffffffu, hv, j);
+        const int oi = __shfl_sync(0xffffffffu, hi, j);
+        hr += better(ov, oi, hv, hi);
+    }
+    // threshold = the k-th best head (or no threshold if fewer than k lanes hold a slot)
+    const unsigned at_k = __ballot_sync(0xffffffffu, hr == k - 1 && hi != TK_NONE);
+    const int src = at_k ? __ffs(at_k) - 1 : 0;
+    const float tv = __shfl_sync(0xffffffffu, hv, src);
+    const int ti = at_k ? __shfl_sync(0xffffffffu, hi, src) : TK_NONE;
+    int cnt = 0;
+#pragma unroll
+    for (int e = 0; e < NS; ++e)
+        cnt += ix[e] != TK_NONE && v[e] == v[e] && (ti == TK_NONE || !better(tv, ti, v[e], ix[e]));
+    int off = cnt;                                   // inclusive prefix over lanes
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, off, o);
+        if (lane >= o) off += y;
+    }
+    const int total = __shfl_sync(0xffffffffu, off, 31);
+    if (total > 32) {
+        warp_topk_rounds<NS>(v, ix, k, out_v, out_i);
+        return;
+    }
+    off -= cnt;
+#pragma unroll
+    for (int e = 0; e < NS; ++e)
+        if (ix[e] != TK_NONE && v[e] == v[e] && (ti == TK_NONE || !better(tv, ti, v[e], ix[e]))) {
+            scr_v[off] = v[e];
+            scr_i[off] = ix[e];
+            ++off;
+        }
+    __syncwarp();
+    if (lane < total) {
+        const float cv = scr_v[lane];
+        const int ci = scr_i[lane];
+        int r = 0;
+        for (int j = 0; j < total; ++j) r += better(scr_v[j], scr_i[j], cv, ci);
+        if (r < k) { out_v[r] = cv; out_i[r] = ci; }
+    } else if (lane < k) {
+        out_v[lane] = -INFINITY;
+        out_i[lane] = TK_NONE;
+    }
+    __syncwarp();
+}
+
 // Per row: chunks of TK_CHUNK logits, one CTA each. Each warp takes the top-k
 // of its 512 logits and their (max, sum exp); one warp merges the CTA's warps,
 // and the row's last CTA (ticket) merges the chunks; log-probabilities are
@@ -251,6 +320,8 @@ __global__ void __launch_bounds__(TK_THREADS)
     __shared__ float s_v[NW * TOPK_MAX];
     __shared__ int s_i[NW * TOPK_MAX];
     __shared__ float s_m[NW], s_s[NW];
+    __shared__ float s_cv[NW * 32];         // per-warp compaction scratch of warp_topk
+    __shared__ int s_ci[NW * 32];
     __shared__ int s_last;
     const int r = blockIdx.y, c = blockIdx.x, nc = gridDim.x;
     const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
@@ -271,7 +342,7 @@ __global__ void __launch_bounds__(TK_THREADS)
     for (int e = 0; e < TK_EPT; ++e)
         if (xi[e] != TK_NONE) sum += __expf(x[e] - m);
     warp_lse(m, sum);
-    warp_topk<TK_EPT>(x, xi, k, s_v + warp * TOPK_MAX, s_i + warp * TOPK_MAX);
+    warp_topk<TK_EPT>(x, xi, k, s_v + warp * TOPK_MAX, s_i + warp * TOPK_MAX, s_cv + warp * 32, s_ci + warp * 32);
     if (lane == 0) { s_m[warp] = m; s_s[warp] = sum; }
     __syncthreads();
     float *rec = ws + ((size_t)r * nc + c) * TK_REC;
@@ -291,7 +362,7 @@ __global__ void __launch_bounds__(TK_THREADS)
         warp_lse(m, sum);
         if (lane == 0) { rec[0] = m; rec[1] = sum; }
         __syncwarp();                      // the candidates are in registers: reuse s_v / s_i
-        warp_topk<NS>(cv, ci, k, s_v, s_i);
+        warp_topk<NS>(cv, ci, k, s_v, s_i, s_cv, s_ci);
         __syncwarp();
         if (lane < k) {
             rec[2 + lane] = s_v[lane];
@@ -321,7 +392,7 @@ __global__ void __launch_bounds__(TK_THREADS)
         lse_combine(m, sum, __ldcg(rrow + q * TK_REC), __ldcg(rrow + q * TK_REC + 1));
     warp_lse(m, sum);
     const float lse = m + logf(sum);
-    warp_topk<TK_MERGE_SLOTS>(cv, ci, k, s_v, s_i);
+    warp_topk<TK_MERGE_SLOTS>(cv, ci, k, s_v, s_i, s_cv, s_ci);
     __syncwarp();
     if (lane < k) {
         ids[(size_t)r * k + lane] = s_i[lane] == TK_NONE ? 0 : s_i[lane];
