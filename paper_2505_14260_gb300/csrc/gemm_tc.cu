@@ -743,6 +743,12 @@ __device__ __forceinline__ uint32_t c_cluster_rank() {
     return r;
 }
 
+__device__ __forceinline__ uint32_t c_mapa(uint32_t local, uint32_t rank) {
+    uint32_t a;
+    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(local), "r"(rank));
+    return a;
+}
+
 __device__ __forceinline__ float4 c_dsmem_ld4(uint32_t local, uint32_t rank) {
     uint32_t a;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(local), "r"(rank));
@@ -768,36 +774,39 @@ __device__ __forceinline__ uint2 c_pack_bf16x4(float a, float b, float c, float 
     return make_uint2(*reinterpret_cast<const uint32_t *>(&lo), *reinterpret_cast<const uint32_t *>(&hi));
 }
 
-// Generic address of the same shared-memory location in cluster CTA `rank`
-// (plain loads through it read distributed shared memory; a pure function, so
-// the compiler may schedule the loads freely).
-__device__ __forceinline__ const float4 *c_map_rank(const float4 *p, uint32_t rank) {
-    uint64_t r;
-    asm("mapa.u64 %0, %1, %2;" : "=l"(r) : "l"(reinterpret_cast<uint64_t>(p)), "r"(rank));
-    return reinterpret_cast<const float4 *>(r);
-}
+// Where a CTA finds the S partials of the token columns it owns, [c_lo,
+// c_hi) = [rank * BN / S, (rank + 1) * BN / S): its own partial ([BN][128]
+// fp32, all columns) and, for S > 1, the other ranks' slices of its columns,
+// pushed into its receive buffer by bulk copies (slot q < rank ? q : q - 1,
+// `span` columns each).
+struct PartSrc {
+    const float *own, *recv;
+    int rank, S, c_lo, c_hi, span;
+    __device__ __forceinline__ const float4 *at(int q, int col, int row) const {
+        const float *b = q == rank ? own + col * BM : recv + ((q < rank ? q : q - 1) * span + (col - c_lo)) * BM;
+        return reinterpret_cast<const float4 *>(b + row);
+    }
+};
 
-// Sums, in rank order, of the S partials' float4 at K offsets (in float4) of
-// the partial buffer `part` (each cluster CTA's partial sits at the same
-// offset; S == 1: local). All loads are issued before the first sum.
+// Sums, in rank order, of the S partials' float4 at K (column, row) places
+// (all in this CTA's shared memory); every load is issued before the first sum.
 template <int K>
-__device__ __forceinline__ void c_part_sums(const float4 *part, const int (&idx)[K], const bool (&use)[K], int S,
-                                            float4 (&out)[K]) {
+__device__ __forceinline__ void c_part_sums(const PartSrc &ps, const int (&col)[K], const int (&row)[K],
+                                            const bool (&use)[K], float4 (&out)[K]) {
     float4 v[K][8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
-        if (q >= S) break;
-        const float4 *src = S == 1 ? part : c_map_rank(part, (uint32_t)q);
+        if (q >= ps.S) break;
 #pragma unroll
         for (int k = 0; k < K; ++k)
-            if (use[k]) v[k][q] = src[idx[k]];
+            if (use[k]) v[k][q] = *ps.at(q, col[k], row[k]);
     }
 #pragma unroll
     for (int k = 0; k < K; ++k) {
         float4 a = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
         for (int q = 0; q < 8; ++q)
-            if (q < S && use[k]) {
+            if (q < ps.S && use[k]) {
                 a.x += v[k][q].x; a.y += v[k][q].y; a.z += v[k][q].z; a.w += v[k][q].w;
             }
         out[k] = a;
@@ -813,33 +822,31 @@ __device__ __forceinline__ void c_part_sums(const float4 *part, const int (&idx)
 
 // SwiGLU (glu-packed tile: rows 0-63 gate, 64-127 up):
 // act[m][64 t + i] = bf16(silu(g) * u), scaled first by the folded-norm 1/rms.
-__device__ __forceinline__ void c_epi_swiglu(const CkParams &p, const float4 *part, uint32_t rank, int S,
-                                             bool ok, int wt, int n0, const float *rinv) {
+__device__ __forceinline__ void c_epi_swiglu(const CkParams &p, const PartSrc &ps, bool ok, int wt, int n0,
+                                             const float *rinv) {
     bf16 *const act = p.fx.act;
-    const int F = p.fx.F, M = p.M, n4 = p.BN * 16;
-    const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
-    for (int e0 = lo + threadIdx.x; e0 < hi; e0 += 2 * C_THREADS) {
-        int ad[4];
+    const int F = p.fx.F, M = p.M;
+    const int n = (ps.c_hi - ps.c_lo) * 16;         // groups of this CTA's columns
+    for (int e0 = threadIdx.x; e0 < n; e0 += 2 * C_THREADS) {
+        int col[4], row[4];
         bool use[4];
-        int col[2], p4[2];
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
             const int e = e0 + u * C_THREADS;
-            col[u] = e >> 4;
-            p4[u] = (e & 15) << 2;
-            ad[2 * u] = (col[u] * BM + p4[u]) >> 2;
-            ad[2 * u + 1] = ad[2 * u] + 16;
-            use[2 * u] = use[2 * u + 1] = e < hi;
+            col[2 * u] = col[2 * u + 1] = ps.c_lo + (e >> 4);
+            row[2 * u] = (e & 15) << 2;
+            row[2 * u + 1] = row[2 * u] + 64;
+            use[2 * u] = use[2 * u + 1] = e < n;
         }
         float4 v[4];
-        c_part_sums<4>(part, ad, use, S, v);
+        c_part_sums<4>(ps, col, row, use, v);
 #pragma unroll
         for (int u = 0; u < 2; ++u) {
             float4 a = v[2 * u], b = v[2 * u + 1];
-            const int m = n0 + col[u], j = wt * 64 + p4[u];
+            const int c = col[2 * u], m = n0 + c, j = wt * 64 + row[2 * u];
             if (!use[2 * u] || !ok || m >= M || j >= F) continue;     // F % 4 == 0: whole groups
             if (rinv) {
-                const float sc = rinv[col[u]];
+                const float sc = rinv[c];
                 a.x *= sc; a.y *= sc; a.z *= sc; a.w *= sc;
                 b.x *= sc; b.y *= sc; b.z *= sc; b.w *= sc;
             }
@@ -852,94 +859,138 @@ __device__ __forceinline__ void c_epi_swiglu(const CkParams &p, const float4 *pa
     }
 }
 
+// Global operands of the first EPI_PRE groups (RoPE) or columns (norm) of a
+// thread are requested before the split-K exchange, so that their round trip
+// overlaps it; later ones (large column shares only) are loaded in the loop.
+constexpr int EPI_PRE = 4;
+
+struct RopePre {
+    RowDesc d[EPI_PRE];
+    float4 c01[EPI_PRE], c23[EPI_PRE];
+};
+
 // RoPE + K/V placement (tile of wq;wk;wv rows, hd | 128): rotate-half pairs
 // (i, i + hd/2) of one head; q rotated into q_out [M][H], k rotated and v into
 // kdst / vdst [B][nh][slots][hd] at the row's slot. Row descriptors come from
 // shared memory (loaded while the MMAs ran).
-__device__ __forceinline__ void c_epi_rope(const CkParams &p, const float4 *part, uint32_t rank, int S,
-                                           bool ok, int seg, int row0, int n0, int rows_here,
-                                           const float *rinv, const RowDesc *srow) {
-    const GemmFused &f = p.fx;
-    const int hd = f.hd, lh = hd == 128 ? 6 : 5, half = 1 << lh, lhd = lh + 1;
-    const float2 *const rope_tab = f.rope_tab;
-    const int max_pos = f.max_pos, slots = f.slots, nh = f.nh, M = p.M;
-    bf16 *const qo = f.q_out, *const kvd = seg == 1 ? f.kdst : f.vdst;
-    const int n4 = p.BN * 16;
-    const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
-    for (int e0 = lo + threadIdx.x; e0 < hi; e0 += 2 * C_THREADS) {
-        int ad[4];
-        bool use[4];
-        int col[2], r[2];
-        bool live[2];
-        RowDesc d[2];
-        float4 c01[2], c23[2];
+struct RopeGeom {
+    int hd, lh, half, lhd, n;
+    __device__ __forceinline__ RopeGeom(int hd_, const PartSrc &ps)
+        : hd(hd_), lh(hd_ == 128 ? 6 : 5), half(1 << lh), lhd(lh + 1), n((ps.c_hi - ps.c_lo) * 16) {}
+    // group e of this CTA's columns: token column and first row of the pair
+    __device__ __forceinline__ void at(const PartSrc &ps, int e, int &c, int &r) const {
+        c = ps.c_lo + (e >> 4);
+        const int p4 = (e & 15) << 2;
+        r = ((p4 >> lh) << lhd) | (p4 & (half - 1));
+    }
+};
+
+// the rotation-table entries (cos, sin of 4 consecutive frequencies) of one group
+__device__ __forceinline__ void c_rope_tab(const CkParams &p, const RopeGeom &g, int pos, int row0, int r,
+                                           float4 &c01, float4 &c23) {
+    if (pos < 0 || pos >= p.fx.max_pos) {
+        set_status(p.status, ST_RANGE);
+        pos = 0;
+    }
+    const int i = (row0 + r) & (g.hd - 1);
+    const float4 *cs = reinterpret_cast<const float4 *>(p.fx.rope_tab + (size_t)pos * g.half + i);
+    c01 = cs[0];
+    c23 = cs[1];
+}
+
+__device__ __forceinline__ void c_rope_pre(const CkParams &p, const PartSrc &ps, bool ok, int seg, int row0,
+                                           int n0, int rows_here, const RowDesc *srow, RopePre &pre) {
+    const RopeGeom g(p.fx.hd, ps);
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int e = e0 + u * C_THREADS;
-            col[u] = e >> 4;
-            const int p4 = (e & 15) << 2;
-            r[u] = ((p4 >> lh) << lhd) | (p4 & (half - 1));
-            ad[2 * u] = (col[u] * BM + r[u]) >> 2;
-            ad[2 * u + 1] = ad[2 * u] + (half >> 2);
-            use[2 * u] = use[2 * u + 1] = e < hi;
-            live[u] = e < hi && ok && n0 + col[u] < M && r[u] < rows_here;
-            d[u] = live[u] ? srow[col[u]] : RowDesc{0, 0, 0, -1};
-            if (live[u] && seg < 2) {                 // the rotation's table entries, in flight early
-                int pos = d[u].pos;
-                if (pos < 0 || pos >= max_pos) {
-                    set_status(p.status, ST_RANGE);
-                    pos = 0;
-                }
-                const int i = (row0 + r[u]) & (hd - 1);
-                const float4 *cs = reinterpret_cast<const float4 *>(rope_tab + (size_t)pos * half + i);
-                c01[u] = cs[0];
-                c23[u] = cs[1];
-            }
-        }
-        float4 v[4];
-        c_part_sums<4>(part, ad, use, S, v);
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            if (!live[u]) continue;
-            float4 a = v[2 * u], b = v[2 * u + 1];
-            if (rinv) {
-                const float sc = rinv[col[u]];
-                a.x *= sc; a.y *= sc; a.z *= sc; a.w *= sc;
-                b.x *= sc; b.y *= sc; b.z *= sc; b.w *= sc;
-            }
-            const int m = n0 + col[u], o = row0 + r[u], h = o >> lhd, i = o & (hd - 1);
-            if (seg < 2) {
-                const float x0 = a.x, x1 = a.y, x2 = a.z, x3 = a.w;
-                a.x = x0 * c01[u].x - b.x * c01[u].y; b.x = b.x * c01[u].x + x0 * c01[u].y;
-                a.y = x1 * c01[u].z - b.y * c01[u].w; b.y = b.y * c01[u].z + x1 * c01[u].w;
-                a.z = x2 * c23[u].x - b.z * c23[u].y; b.z = b.z * c23[u].x + x2 * c23[u].y;
-                a.w = x3 * c23[u].z - b.w * c23[u].w; b.w = b.w * c23[u].z + x3 * c23[u].w;
-            }
-            bf16 *dst;
-            if (seg == 0) {
-                dst = qo + (size_t)m * (nh * hd) + o;
-            } else {
-                if (d[u].dst >= slots) set_status(p.status, ST_RANGE);
-                if (d[u].dst < 0 || d[u].dst >= slots) continue;
-                dst = kvd + ((size_t)(d[u].req * nh + h) * slots + d[u].dst) * hd + i;
-            }
-            *reinterpret_cast<uint2 *>(dst) = c_pack_bf16x4(a.x, a.y, a.z, a.w);
-            *reinterpret_cast<uint2 *>(dst + half) = c_pack_bf16x4(b.x, b.y, b.z, b.w);
-        }
+    for (int k = 0; k < EPI_PRE; ++k) {
+        const int e = threadIdx.x + k * C_THREADS;
+        if (e >= g.n) break;
+        int c, r;
+        g.at(ps, e, c, r);
+        pre.d[k] = srow[c];
+        if (ok && seg < 2 && n0 + c < p.M && r < rows_here)
+            c_rope_tab(p, g, pre.d[k].pos, row0, r, pre.c01[k], pre.c23[k]);
     }
 }
 
-// Producer side of a folded RMSNorm: this CTA's share of the tile's token
-// columns, one warp per column (lane = 4 consecutive weight rows), two columns
-// of a warp per pass: the S partials summed in rank order, the residual added,
-// then Y (fp32), xg = bf16(y * g) and the column's sum of squares over the
-// tile's rows (a warp reduction in a fixed order) into ss[m][tile].
-__device__ __forceinline__ void c_reduce_norm(const CkParams &p, const float4 *part, uint32_t rank, int S,
-                                              bool ok, int tile, int o_base, int rows_here, int n0) {
+__device__ __forceinline__ void c_epi_rope(const CkParams &p, const PartSrc &ps, bool ok, int seg, int row0,
+                                           int n0, int rows_here, const float *rinv, const RowDesc *srow,
+                                           const RopePre &pre) {
+    const RopeGeom g(p.fx.hd, ps);
+    const int slots = p.fx.slots, nh = p.fx.nh, M = p.M, hd = g.hd, half = g.half;
+    bf16 *const qo = p.fx.q_out, *const kvd = seg == 1 ? p.fx.kdst : p.fx.vdst;
+    for (int k = 0;; ++k) {
+        const int e = threadIdx.x + k * C_THREADS;
+        if (e >= g.n) break;
+        int c, r;
+        g.at(ps, e, c, r);
+        const int m = n0 + c;
+        if (!ok || m >= M || r >= rows_here) continue;
+        RowDesc d;
+        float4 c01, c23;
+        if (k < EPI_PRE) {
+#pragma unroll
+            for (int j = 0; j < EPI_PRE; ++j)       // static indices only
+                if (j == k) { d = pre.d[j]; c01 = pre.c01[j]; c23 = pre.c23[j]; }
+        } else {
+            d = srow[c];
+            if (seg < 2) c_rope_tab(p, g, d.pos, row0, r, c01, c23);
+        }
+        const int col[2] = {c, c}, row[2] = {r, r + half};
+        const bool use[2] = {true, true};
+        float4 v[2];
+        c_part_sums<2>(ps, col, row, use, v);
+        float4 a = v[0], b = v[1];
+        if (rinv) {
+            const float sc = rinv[c];
+            a.x *= sc; a.y *= sc; a.z *= sc; a.w *= sc;
+            b.x *= sc; b.y *= sc; b.z *= sc; b.w *= sc;
+        }
+        const int o = row0 + r, h = o >> g.lhd, i = o & (hd - 1);
+        if (seg < 2) {
+            const float x0 = a.x, x1 = a.y, x2 = a.z, x3 = a.w;
+            a.x = x0 * c01.x - b.x * c01.y; b.x = b.x * c01.x + x0 * c01.y;
+            a.y = x1 * c01.z - b.y * c01.w; b.y = b.y * c01.z + x1 * c01.w;
+            a.z = x2 * c23.x - b.z * c23.y; b.z = b.z * c23.x + x2 * c23.y;
+            a.w = x3 * c23.z - b.w * c23.w; b.w = b.w * c23.z + x3 * c23.w;
+        }
+        bf16 *dst;
+        if (seg == 0) {
+            dst = qo + (size_t)m * (nh * hd) + o;
+        } else {
+            if (d.dst >= slots) set_status(p.status, ST_RANGE);
+            if (d.dst < 0 || d.dst >= slots) continue;
+            dst = kvd + ((size_t)(d.req * nh + h) * slots + d.dst) * hd + i;
+        }
+        *reinterpret_cast<uint2 *>(dst) = c_pack_bf16x4(a.x, a.y, a.z, a.w);
+        *reinterpret_cast<uint2 *>(dst + half) = c_pack_bf16x4(b.x, b.y, b.z, b.w);
+    }
+}
+
+// Residual rows of the first EPI_PRE columns of a warp (folded-norm producer
+// with accumulation), requested before the exchange.
+__device__ __forceinline__ void c_norm_pre(const CkParams &p, const PartSrc &ps, bool ok, int o_base,
+                                           int rows_here, int n0, float4 (&yv)[EPI_PRE]) {
+    const int warp = threadIdx.x >> 5, r4 = (threadIdx.x & 31) * 4;
+    if (p.epi != EPI_ADD || r4 + 4 > rows_here) return;
+#pragma unroll
+    for (int k = 0; k < EPI_PRE; ++k) {
+        const int c = ps.c_lo + warp + k * (C_THREADS / 32);
+        if (ok && c < ps.c_hi && n0 + c < p.M)
+            yv[k] = *reinterpret_cast<const float4 *>(p.Y + (size_t)(n0 + c) * p.ldy + o_base + r4);
+    }
+}
+
+// Producer side of a folded RMSNorm: this CTA's token columns, one warp per
+// column (lane = 4 consecutive weight rows): the S partials summed in rank
+// order, the residual added, then Y (fp32), xg = bf16(y * g) and the column's
+// sum of squares over the tile's rows (a warp reduction in a fixed order) into
+// ss[m][tile].
+__device__ __forceinline__ void c_reduce_norm(const CkParams &p, const PartSrc &ps, bool ok, int tile, int o_base,
+                                              int rows_here, int n0, const float4 (&yv)[EPI_PRE]) {
     constexpr int NW = C_THREADS / 32;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const bool add = p.epi == EPI_ADD;
-    const int c_lo = (int)((long long)rank * p.BN / S), c_hi = (int)((long long)(rank + 1) * p.BN / S);
     const int r4 = lane * 4;
     const bool full = r4 + 4 <= rows_here;
     float g4[4] = {0.f, 0.f, 0.f, 0.f};
@@ -953,59 +1004,57 @@ __device__ __forceinline__ void c_reduce_norm(const CkParams &p, const float4 *p
     float *const Y = p.Y;
     bf16 *const XG = p.nout.xg;
     const int ldy = p.ldy, M = p.M;
-    for (int c0 = c_lo + warp; c0 < c_hi; c0 += 2 * NW) {
-        int ad[2];
-        bool use[2], live[2];
-        float4 yi[2];
+    for (int k = 0;; ++k) {
+        const int c = ps.c_lo + warp + k * NW;
+        if (c >= ps.c_hi) break;                         // warp-uniform
+        const int col[1] = {c}, row[1] = {r4};
+        const bool use[1] = {true};
+        float4 v[1];
+        c_part_sums<1>(ps, col, row, use, v);
+        float a[4] = {v[0].x, v[0].y, v[0].z, v[0].w};
+        const int m = n0 + c;
+        const bool live = ok && m < M;                   // warp-uniform
+        float ss = 0.f;
+        if (live) {
+            float *y = Y + (size_t)m * ldy + o_base + r4;
+            bf16 *xg = XG + (size_t)m * ldy + o_base + r4;
+            if (full) {
+                if (add) {
+                    float4 yi;
+                    if (k < EPI_PRE) {
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            const int c = c0 + u * NW;
-            ad[u] = (c * BM + r4) >> 2;
-            use[u] = c < c_hi;
-            live[u] = use[u] && ok && n0 + c < M;        // warp-uniform
-            yi[u] = make_float4(0.f, 0.f, 0.f, 0.f);
-            if (live[u] && full && add)
-                yi[u] = *reinterpret_cast<const float4 *>(Y + (size_t)(n0 + c) * ldy + o_base + r4);
-        }
-        float4 v[2];
-        c_part_sums<2>(part, ad, use, S, v);
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            if (!use[u]) continue;
-            const int m = n0 + c0 + u * NW;
-            float a[4] = {v[u].x, v[u].y, v[u].z, v[u].w};
-            float ss = 0.f;
-            if (live[u]) {
-                float *y = Y + (size_t)m * ldy + o_base + r4;
-                bf16 *xg = XG + (size_t)m * ldy + o_base + r4;
-                if (full) {
-                    a[0] += yi[u].x; a[1] += yi[u].y; a[2] += yi[u].z; a[3] += yi[u].w;
-                    *reinterpret_cast<float4 *>(y) = make_float4(a[0], a[1], a[2], a[3]);
-                    *reinterpret_cast<uint2 *>(xg) =
-                        c_pack_bf16x4(a[0] * g4[0], a[1] * g4[1], a[2] * g4[2], a[3] * g4[3]);
-                    ss = a[0] * a[0] + a[1] * a[1] + a[2] * a[2] + a[3] * a[3];
-                } else {
-                    const bf16 *g = p.nout.g + o_base + r4;
-#pragma unroll
-                    for (int e = 0; e < 4; ++e)
-                        if (r4 + e < rows_here) {
-                            const float ye = add ? y[e] + a[e] : a[e];
-                            y[e] = ye;
-                            xg[e] = __float2bfloat16_rn(ye * __bfloat162float(g[e]));
-                            ss += ye * ye;
-                        }
+                        for (int j = 0; j < EPI_PRE; ++j)
+                            if (j == k) yi = yv[j];
+                    } else {
+                        yi = *reinterpret_cast<const float4 *>(y);
+                    }
+                    a[0] += yi.x; a[1] += yi.y; a[2] += yi.z; a[3] += yi.w;
                 }
+                *reinterpret_cast<float4 *>(y) = make_float4(a[0], a[1], a[2], a[3]);
+                *reinterpret_cast<uint2 *>(xg) =
+                    c_pack_bf16x4(a[0] * g4[0], a[1] * g4[1], a[2] * g4[2], a[3] * g4[3]);
+                ss = a[0] * a[0] + a[1] * a[1] + a[2] * a[2] + a[3] * a[3];
+            } else {
+                const bf16 *g = p.nout.g + o_base + r4;
+#pragma unroll
+                for (int e = 0; e < 4; ++e)
+                    if (r4 + e < rows_here) {
+                        const float ye = add ? y[e] + a[e] : a[e];
+                        y[e] = ye;
+                        xg[e] = __float2bfloat16_rn(ye * __bfloat162float(g[e]));
+                        ss += ye * ye;
+                    }
             }
-            ss = warp_sum(ss);
-            if (live[u] && lane == 0) p.nout.ss[(size_t)m * p.nout.ld + tile] = ss;
         }
+        ss = warp_sum(ss);
+        if (live && lane == 0) p.nout.ss[(size_t)m * p.nout.ld + tile] = ss;
     }
 }
 
 __global__ void __launch_bounds__(C_THREADS)
     gemm_cluster_kernel(const __grid_constant__ CUtensorMap mx, const CkParams p) {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t bars[2 * C_STAGES + 1];
+    __shared__ __align__(8) uint64_t bars[2 * C_STAGES + 2];
     __shared__ uint32_t tmem_base;
     __shared__ volatile int abort_flag;
     __shared__ float s_rinv[128];     // folded RMSNorm (consumer): 1/rms of each token column
@@ -1032,6 +1081,7 @@ __global__ void __launch_bounds__(C_THREADS)
     const uint32_t a_base = sbase, b_base = sbase + C_STAGES * A_BYTES;
     const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[C_STAGES]);
     const uint32_t done = smem_u32(&bars[2 * C_STAGES]);
+    const uint32_t recv_bar = smem_u32(&bars[2 * C_STAGES + 1]);   // the other ranks' slices have landed
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < C_STAGES; ++s) {
@@ -1039,6 +1089,7 @@ __global__ void __launch_bounds__(C_THREADS)
             mbar_init(empty0 + 8 * s, 1);
         }
         mbar_init(done, 1);
+        mbar_init(recv_bar, 1);
         abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -1180,52 +1231,98 @@ __global__ void __launch_bounds__(C_THREADS)
             for (int j = 0; j < 32; ++j)
                 if (j < gw) part[(g0 + j) * BM + row] = __uint_as_float(r[j]);
         }
-        if (S > 1) c_cluster_sync();
-        else __syncthreads();
+        // Split-K reduction, push style: after a cluster barrier (every rank's
+        // MMAs are done, so every rank's stage memory is free), each rank sends
+        // every other rank the slice of its partial that holds that rank's
+        // columns, by bulk copies into the receiver's buffer that complete on the
+        // receiver's mbarrier; each rank then reduces its own columns from its
+        // own shared memory, in rank order.
         const uint32_t rank = S > 1 ? c_cluster_rank() : 0u;
-        const uint32_t part_s = smem_u32(part);
-        const float4 *part4 = reinterpret_cast<const float4 *>(part);
+        const int span = (BN + S - 1) / S;
+        PartSrc ps;
+        ps.own = part;
+        ps.recv = part + BN * BM;
+        ps.rank = (int)rank;
+        ps.S = S;
+        ps.c_lo = (int)rank * BN / S;
+        ps.c_hi = ((int)rank + 1) * BN / S;
+        ps.span = span;
+        bool okr = ok;
+        __syncthreads();                 // the staged row descriptors, for every warp
+        RopePre rpre;
+        float4 yv[EPI_PRE];
+        if (paired && p.epi == EPI_ROPE_KV) c_rope_pre(p, ps, ok, seg, row0, n0, rows_here, s_rows, rpre);
+        if (norm_out) c_norm_pre(p, ps, ok, o_base, rows_here, n0, yv);
+        if (S > 1) {
+            asm volatile("fence.proxy.async.shared::cta;" ::: "memory");    // part, for the bulk copies
+            c_cluster_sync();
+            if (threadIdx.x == 0) {
+                mbar_expect_tx(recv_bar, (uint32_t)((S - 1) * (ps.c_hi - ps.c_lo) * BM * 4));
+                for (int t = 0; t < S; ++t) {
+                    const int t_lo = t * BN / S, t_hi = (t + 1) * BN / S;
+                    if (t == (int)rank || t_hi == t_lo) continue;
+                    const int slot = (int)rank < t ? (int)rank : (int)rank - 1;
+                    const uint32_t src = smem_u32(part + t_lo * BM);
+                    const uint32_t dst = c_mapa(smem_u32(ps.recv + slot * span * BM), (uint32_t)t);
+                    asm volatile(
+                        "cp.async.bulk.shared::cluster.shared::cta.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+                            dst),
+                        "r"(src), "r"((uint32_t)((t_hi - t_lo) * BM * 4)), "r"(c_mapa(recv_bar, (uint32_t)t))
+                        : "memory");
+                }
+                asm volatile("cp.async.bulk.commit_group;" ::: "memory");
+            }
+            okr = mbar_wait(recv_bar, 0, &abort_flag, p.status) && ok;
+        } else {
+            __syncthreads();
+        }
         if (p.epi == EPI_SWIGLU)
-            c_epi_swiglu(p, part4, rank, S, ok, wt, n0, p.nin.ss ? s_rinv : nullptr);
+            c_epi_swiglu(p, ps, okr, wt, n0, p.nin.ss ? s_rinv : nullptr);
         else if (paired)
-            c_epi_rope(p, part4, rank, S, ok, seg, row0, n0, rows_here, p.nin.ss ? s_rinv : nullptr, s_rows);
-        else if (norm_out) c_reduce_norm(p, part4, rank, S, ok, wt, o_base, rows_here, n0);
-        // this CTA's slice of the tile, as float4 (4 consecutive weight rows of one token)
-        const int n4 = BN * BM / 4;
-        const int lo = (int)((long long)rank * n4 / S), hi = (int)((long long)(rank + 1) * n4 / S);
-#pragma unroll 2
-        for (int e4 = lo + threadIdx.x; !paired && !norm_out && e4 < hi; e4 += C_THREADS) {
-            float4 v[8];
+            c_epi_rope(p, ps, okr, seg, row0, n0, rows_here, p.nin.ss ? s_rinv : nullptr, s_rows, rpre);
+        else if (norm_out)
+            c_reduce_norm(p, ps, okr, wt, o_base, rows_here, n0, yv);
+        else {
+            // plain reduction of this CTA's columns, float4 = 4 consecutive weight rows of one token
+            const int n = (ps.c_hi - ps.c_lo) * (BM / 4);
+            for (int e0 = threadIdx.x; e0 < n; e0 += 2 * C_THREADS) {
+                int col[2], row[2];
+                bool use[2];
 #pragma unroll
-            for (int q = 0; q < 8; ++q)
-                if (q < S) v[q] = c_dsmem_ld4(part_s + e4 * 16, q);
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-#pragma unroll
-            for (int q = 0; q < 8; ++q)
-                if (q < S) {
-                    acc.x += v[q].x; acc.y += v[q].y; acc.z += v[q].z; acc.w += v[q].w;
+                for (int u = 0; u < 2; ++u) {
+                    const int e = e0 + u * C_THREADS;
+                    col[u] = ps.c_lo + e / (BM / 4);
+                    row[u] = (e % (BM / 4)) * 4;
+                    use[u] = e < n;
                 }
-            const int col = (e4 * 4) / BM, r4 = e4 * 4 - col * BM;
-            const int m = n0 + col;
-            if (!ok || m >= p.M) continue;
-            float *y = p.Y + (size_t)m * p.ldy + o_base + r4;
-            if (r4 + 4 <= rows_here && ((reinterpret_cast<uintptr_t>(y) & 15u) == 0)) {
-                if (add) {
-                    const float4 yi = *reinterpret_cast<const float4 *>(y);
-                    acc.x += yi.x; acc.y += yi.y; acc.z += yi.z; acc.w += yi.w;
-                }
-                *reinterpret_cast<float4 *>(y) = acc;
-            } else {
-                const float vv[4] = {acc.x, acc.y, acc.z, acc.w};
+                float4 v[2];
+                c_part_sums<2>(ps, col, row, use, v);
 #pragma unroll
-                for (int e = 0; e < 4; ++e)
-                    if (r4 + e < rows_here) {
-                        if (add) y[e] = y[e] + vv[e];
-                        else y[e] = vv[e];
+                for (int u = 0; u < 2; ++u) {
+                    const int m = n0 + col[u], r4 = row[u];
+                    if (!use[u] || !okr || m >= p.M) continue;
+                    float4 acc = v[u];
+                    float *y = p.Y + (size_t)m * p.ldy + o_base + r4;
+                    if (r4 + 4 <= rows_here && ((reinterpret_cast<uintptr_t>(y) & 15u) == 0)) {
+                        if (add) {
+                            const float4 yi = *reinterpret_cast<const float4 *>(y);
+                            acc.x += yi.x; acc.y += yi.y; acc.z += yi.z; acc.w += yi.w;
+                        }
+                        *reinterpret_cast<float4 *>(y) = acc;
+                    } else {
+                        const float vv[4] = {acc.x, acc.y, acc.z, acc.w};
+#pragma unroll
+                        for (int e = 0; e < 4; ++e)
+                            if (r4 + e < rows_here) {
+                                if (add) y[e] = y[e] + vv[e];
+                                else y[e] = vv[e];
+                            }
                     }
+                }
             }
         }
-        if (S > 1) c_cluster_sync();      // partials stay readable until every slice is done
+        // this CTA's outgoing copies have read its partial before it exits
+        if (S > 1 && threadIdx.x == 0) asm volatile("cp.async.bulk.wait_group.read 0;" ::: "memory");
     }
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
