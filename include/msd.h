@@ -186,6 +186,22 @@ msd_status msd_accept_compact(msd_ctx *ctx, const msd_tree *tree,
 msd_status msd_step(msd_ctx *ctx, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
                     int32_t *accept_len_dev, int32_t *bonus_dev, void *stream);
 
+/* Plain greedy autoregressive decoding, the baseline against which the paper
+ * measures its speedup ratio (Sec. 4.1, Eq. 9: T_p, the target's time per
+ * generated token): one target forward over each request's current root token
+ * at position L, its K/V appended to the cache at L, L <- L + 1, and the argmax
+ * (ties: lower id) becomes the new root and is written to token_dev[b] (B int32,
+ * device). The same kernels as msd_verify and msd_accept_compact run it (a
+ * tree of the root alone), recorded once into a CUDA graph per token_dev and
+ * bucket of cache lengths and replayed, as msd_step. A context created with
+ * tree_nodes = 1 runs it on B token rows; with more tree nodes the other rows
+ * are computed and ignored. The draft is not run, so after this call the draft
+ * cache no longer follows the target's: msd_draft_tree and msd_step return
+ * MSD_ERR_INVALID until the next msd_prefill. Errors: MSD_ERR_INVALID (null
+ * token_dev, no prefill), MSD_ERR_CAPACITY, MSD_ERR_DEVICE, MSD_ERR_CUDA, as
+ * for msd_step. */
+msd_status msd_ar_step(msd_ctx *ctx, int32_t *token_dev, void *stream);
+
 /* Building block used by every projection of the step (Sec. 3.1 decoder
  * layers, Eq. 4 f_down, Eq. 5 LM head), exposed for tests and kernel timing:
  * y[i][j] (= or, if accumulate != 0, +=) sum_t x[i][t] * w[j][t] for i < m,

@@ -38,8 +38,8 @@ constexpr int THREADS = 256;      // 8 warps: 4 row groups x 2 key halves
 // 8 rows a warp writes at once fall in different banks
 template <int HD> constexpr int PART_LD = HD + 8;
 constexpr int MAX_STAGES = 3;
-constexpr int MAX_SPLITS = 16;    // cache splits + the tree split = cluster size (<= 16)
 constexpr int CACHE_SPLITS = 8;   // cache splits of a decode launch (capacity-derived chunk)
+constexpr int MAX_SPLITS = CACHE_SPLITS + 1;   // + the tree split = cluster size
 constexpr unsigned long long ATTN_TIMEOUT_NS = 2000000000ull;
 
 struct AttnTcParams {
@@ -145,9 +145,11 @@ __device__ __forceinline__ float dsmem_ld_f32(uint32_t a) {
     return v;
 }
 
+// (no memory clobber: the partials are read only between two cluster
+// barriers, themselves compiler barriers, so the loads may overlap)
 __device__ __forceinline__ float2 dsmem_ld_f2(uint32_t a) {
     float2 v;
-    asm volatile("ld.shared::cluster.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a) : "memory");
+    asm volatile("ld.shared::cluster.v2.f32 {%0,%1}, [%2];" : "=f"(v.x), "=f"(v.y) : "r"(a));
     return v;
 }
 
@@ -155,8 +157,7 @@ __device__ __forceinline__ float4 dsmem_ld_f4(uint32_t a) {
     float4 v;
     asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
                  : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(a)
-                 : "memory");
+                 : "r"(a));
     return v;
 }
 
@@ -481,36 +482,51 @@ __global__ void __launch_bounds__(THREADS, 2)
     const int per = (nrows + nsplit - 1) / nsplit;
     const int row_lo = (int)rank * per, row_hi = min(nrows, row_lo + per);
     const uint32_t o_local = su32(s_o), ml_local = su32(s_ml);
-    constexpr int C4 = HD / 4;
-    for (int rr = row_lo + warp; rr < row_hi; rr += THREADS / 32) {
-        // lane sp fetches split sp's (m, l); warp shuffles give the max and the sum
-        float2 ml = make_float2(-INFINITY, 0.f);
-        if (lane < nsplit) ml = dsmem_ld_f2(dsmem_addr(ml_local + rr * 8, lane));
-        const float M = warp_max(ml.x);
-        const float w = (lane < nsplit && M != -INFINITY) ? exp2f(ml.x - M) : 0.f;
-        const float den = warp_sum(w * ml.y);
-        const float inv = den > 0.f ? 1.f / den : 0.f;
-        const float wn = w * inv;
-        float wsp[MAX_SPLITS];
+    constexpr int C4 = HD / 4, NWARP = THREADS / 32;
+    // a warp combines two of the CTA's rows per pass, every partial load of
+    // both (max and sum of each split, then its O) issued before any is used
+    for (int rr0 = row_lo + warp; rr0 < row_hi; rr0 += 2 * NWARP) {
+        const int rr[2] = {rr0, rr0 + NWARP};
+        const bool has[2] = {true, rr0 + NWARP < row_hi};
+        float2 ml[2];
+        float4 v[2][MAX_SPLITS];
 #pragma unroll
-        for (int sp = 0; sp < MAX_SPLITS; ++sp) wsp[sp] = __shfl_sync(0xffffffffu, wn, sp);
-        if (lane < C4) {
-            float4 v[MAX_SPLITS];
+        for (int u = 0; u < 2; ++u) {
+            ml[u] = make_float2(-INFINITY, 0.f);
+            if (has[u] && lane < nsplit) ml[u] = dsmem_ld_f2(dsmem_addr(ml_local + rr[u] * 8, lane));
+        }
 #pragma unroll
-            for (int sp = 0; sp < MAX_SPLITS; ++sp)     // every load in flight at once
-                if (sp < nsplit) v[sp] = dsmem_ld_f4(dsmem_addr(o_local + (rr * LD + 4 * lane) * 4, sp));
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int u = 0; u < 2; ++u)
 #pragma unroll
             for (int sp = 0; sp < MAX_SPLITS; ++sp)
-                if (sp < nsplit) {
-                    acc.x += wsp[sp] * v[sp].x; acc.y += wsp[sp] * v[sp].y;
-                    acc.z += wsp[sp] * v[sp].z; acc.w += wsp[sp] * v[sp].w;
-                }
-            uint2 packed;
-            packed.x = pack_bf16(acc.x, acc.y);
-            packed.y = pack_bf16(acc.z, acc.w);
-            if (ok)
-                *reinterpret_cast<uint2 *>(p.out + (size_t)(r0 + rr) * H + h * HD + 4 * lane) = packed;
+                if (has[u] && lane < C4 && sp < nsplit)
+                    v[u][sp] = dsmem_ld_f4(dsmem_addr(o_local + (rr[u] * LD + 4 * lane) * 4, sp));
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            if (!has[u]) continue;                         // warp-uniform
+            // lane sp holds split sp's (m, l); warp shuffles give the max and the sum
+            const float M = warp_max(ml[u].x);
+            const float w = (lane < nsplit && M != -INFINITY) ? exp2f(ml[u].x - M) : 0.f;
+            const float den = warp_sum(w * ml[u].y);
+            const float inv = den > 0.f ? 1.f / den : 0.f;
+            const float wn = w * inv;
+            float wsp[MAX_SPLITS];
+#pragma unroll
+            for (int sp = 0; sp < MAX_SPLITS; ++sp) wsp[sp] = __shfl_sync(0xffffffffu, wn, sp);
+            if (lane < C4) {
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                for (int sp = 0; sp < MAX_SPLITS; ++sp)
+                    if (sp < nsplit) {
+                        acc.x += wsp[sp] * v[u][sp].x; acc.y += wsp[sp] * v[u][sp].y;
+                        acc.z += wsp[sp] * v[u][sp].z; acc.w += wsp[sp] * v[u][sp].w;
+                    }
+                uint2 packed;
+                packed.x = pack_bf16(acc.x, acc.y);
+                packed.y = pack_bf16(acc.z, acc.w);
+                if (ok)
+                    *reinterpret_cast<uint2 *>(p.out + (size_t)(r0 + rr[u]) * H + h * HD + 4 * lane) = packed;
+            }
         }
     }
     cluster_sync();                                    // partials stay readable until all are done

@@ -286,6 +286,23 @@ __global__ void verify_setup_kernel(TreeIn t, const int *__restrict__ seq_len,
 }
 
 // ---------------------------------------------------------------------------
+// Root-only tree of plain greedy decoding: one thread per request.
+// ---------------------------------------------------------------------------
+__global__ void root_tree_kernel(const int *__restrict__ root, int B, int N, int W, int *__restrict__ tokens,
+                                 int *__restrict__ parent, int *__restrict__ depth, uint64_t *__restrict__ mask,
+                                 int *__restrict__ n_nodes) {
+    wait_prior();
+    allow_dependents();
+    const int b = blockIdx.x * blockDim.x + threadIdx.x;
+    if (b >= B) return;
+    tokens[(size_t)b * N] = root[b];
+    parent[(size_t)b * N] = -1;
+    depth[(size_t)b * N] = 0;
+    for (int w = 0; w < W; ++w) mask[(size_t)b * N * W + w] = w == 0 ? 1ull : 0ull;
+    n_nodes[b] = 1;
+}
+
+// ---------------------------------------------------------------------------
 // Greedy acceptance (Eq. 6 at T = 0): one warp per request walks from the root
 // to the child whose token is the target argmax of the current node.
 // ---------------------------------------------------------------------------
@@ -475,6 +492,12 @@ void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, i
     const int R = B * N;
     launch_pdl(verify_setup_kernel, (R + 127) / 128, 128, 0, s, t, seq_len, root, B, N, V, rows, src,
                                                           vmask, status); note_launch();
+}
+
+void launch_root_tree(const int *root, int B, int N, int W, int *tokens, int *parent, int *depth,
+                      uint64_t *mask, int *n_nodes, cudaStream_t s) {
+    launch_pdl(root_tree_kernel, (B + 127) / 128, 128, 0, s, root, B, N, W, tokens, parent, depth, mask, n_nodes);
+    note_launch();
 }
 
 void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int *seq_len,

@@ -60,6 +60,11 @@ void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand
 void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, int B, int N,
                          int V, RowDesc *rows, int *src, uint64_t *vmask, int *status,
                          cudaStream_t s);
+// A tree of each request's root alone (plain greedy decoding): node 0 = root,
+// parent -1, depth 0, mask = itself, n_nodes = 1; nodes 1.. are not part of it.
+void launch_root_tree(const int *root, int B, int N, int W, int *tokens, int *parent, int *depth,
+                      uint64_t *mask, int *n_nodes, cudaStream_t s);
+
 void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int *seq_len,
                    int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
                    int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,

@@ -51,6 +51,10 @@ struct msd_ctx {
     TopkScratch tks{nullptr, nullptr};
     void *hT = nullptr;
     int *acc_path = nullptr, *acc_L0 = nullptr, *acc_a = nullptr;
+    // plain greedy decoding (msd_ar_step): a root-only tree and its argmax
+    msd_tree ar_tree{};
+    int *ar_argmax = nullptr;
+    bool draft_stale = false;   // msd_ar_step ran: the draft cache no longer follows the target's
     float2 *rope_tab = nullptr;
     void *h_all = nullptr, *emb_all = nullptr;
     int *status = nullptr;
@@ -75,6 +79,7 @@ struct msd_ctx {
     // whole-step CUDA graphs (msd_step), one per L bucket and buffer set
     struct StepGraph {
         cudaGraphExec_t exec = nullptr;
+        int kind = 0;               // 0: draft-verify-accept step, 1: plain greedy step
         int bucket_hi = 0;
         msd_tree tree{};
         const void *argmax = nullptr, *path = nullptr, *alen = nullptr, *bonus = nullptr;
@@ -432,6 +437,7 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
         c->L_bound[b] = L;
     }
     c->prefilled = true;
+    c->draft_stale = false;
     return post_status(c, s);
 }
 
@@ -550,7 +556,7 @@ msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, fl
 
 template <typename T>
 msd_status accept_impl(msd_ctx *c, const msd_tree *tree, const int32_t *argmax, int32_t *path,
-                       int32_t *alen, int32_t *bonus, int32_t *imap, cudaStream_t s) {
+                       int32_t *alen, int32_t *bonus, int32_t *imap, cudaStream_t s, int grow = -1) {
     TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
     launch_accept(t, argmax, c->B, c->N, c->D, c->seq_len, c->n_pend, c->root, c->pend_next,
                   c->acc_path, c->acc_L0, c->acc_a, path, alen, bonus, imap, s);
@@ -559,8 +565,22 @@ msd_status accept_impl(msd_ctx *c, const msd_tree *tree, const int32_t *argmax, 
     launch_pend_h<T>(static_cast<const T *>(c->hT), c->acc_path, c->acc_a, c->B, c->N, c->D1, c->H,
                      static_cast<T *>(c->pend_h), s);
     if (!c->capturing)
-        for (int b = 0; b < c->B; ++b) c->L_bound[b] += c->D1;
+        for (int b = 0; b < c->B; ++b) c->L_bound[b] += grow < 0 ? c->D1 : grow;
     return post_status(c, s);
+}
+
+// Plain greedy autoregressive decoding, the baseline of the speedup ratio
+// (Sec. 4.1, Eq. 9's T_p): a tree of the root alone, verified and accepted —
+// one target forward over each request's root token at position L, its K/V
+// appended at L, the argmax the next root.
+template <typename T>
+msd_status ar_impl(msd_ctx *c, int32_t *token_out, cudaStream_t s) {
+    launch_root_tree(c->root, c->B, c->N, c->W, c->ar_tree.tokens, c->ar_tree.parent, c->ar_tree.depth,
+                     c->ar_tree.mask, c->ar_tree.n_nodes, s);
+    msd_status st = verify_impl<T>(c, &c->ar_tree, c->ar_argmax, nullptr, s);
+    if (st == MSD_OK)
+        st = accept_impl<T>(c, &c->ar_tree, c->ar_argmax, nullptr, nullptr, token_out, nullptr, s, 1);
+    return st;
 }
 
 // A step writes at most positions L .. L+D (tree K/V land at L+depth only in
@@ -644,9 +664,9 @@ msd_status step_eager(msd_ctx *c, const msd_tree *tree, int32_t *argmax, int32_t
     return st;
 }
 
-bool same_buffers(const msd_ctx::StepGraph &g, const msd_tree *t, const void *a,
+bool same_buffers(const msd_ctx::StepGraph &g, int kind, const msd_tree *t, const void *a,
                          const void *p, const void *l, const void *b) {
-    return g.tree.tokens == t->tokens && g.tree.parent == t->parent && g.tree.depth == t->depth &&
+    return g.kind == kind && g.tree.tokens == t->tokens && g.tree.parent == t->parent && g.tree.depth == t->depth &&
            g.tree.mask == t->mask && g.tree.n_nodes == t->n_nodes && g.argmax == a &&
            g.path == p && g.alen == l && g.bonus == b;
 }
@@ -738,6 +758,12 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     ok &= dalloc(c, &c->acc_path, sizeof(int) * c->B * c->D1);
     ok &= dalloc(c, &c->acc_L0, sizeof(int) * c->B);
     ok &= dalloc(c, &c->acc_a, sizeof(int) * c->B);
+    ok &= dalloc(c, &c->ar_tree.tokens, sizeof(int) * c->B * c->N);
+    ok &= dalloc(c, &c->ar_tree.parent, sizeof(int) * c->B * c->N);
+    ok &= dalloc(c, &c->ar_tree.depth, sizeof(int) * c->B * c->N);
+    ok &= dalloc(c, &c->ar_tree.mask, sizeof(uint64_t) * c->B * c->N * c->W);
+    ok &= dalloc(c, &c->ar_tree.n_nodes, sizeof(int) * c->B);
+    ok &= dalloc(c, &c->ar_argmax, sizeof(int) * c->B * c->N);
     ok &= dalloc(c, &c->rope_tab, sizeof(float2) * (size_t)c->S * (c->hd / 2));
     ok &= dalloc(c, &c->h_all, (size_t)c->S * H * e);
     ok &= dalloc(c, &c->emb_all, (size_t)c->S * H * e);
@@ -841,6 +867,8 @@ msd_status msd_draft_tree(msd_ctx *c, const msd_tree *out, const msd_draft_recor
     if (st != MSD_OK) return st;
     if (!tree_ok(out)) return fail(c, MSD_ERR_INVALID, "null tree array");
     if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    if (c->draft_stale)
+        return fail(c, MSD_ERR_INVALID, "msd_ar_step ran since the last msd_prefill: the draft cache is stale");
     st = check_capacity(c);
     if (st != MSD_OK) return st;
     cudaStream_t s = static_cast<cudaStream_t>(stream);
@@ -886,30 +914,33 @@ msd_status msd_accept_compact(msd_ctx *c, const msd_tree *tree, const int32_t *a
                               index_map_dev, s);
 }
 
-msd_status msd_step(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
-                    int32_t *accept_len_dev, int32_t *bonus_dev, void *stream) {
-    if (!c) return MSD_ERR_INVALID;
-    c->err.clear();
-    if (report_stale_error("msd_step"))
-        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
-    msd_status st = check_status(c);
-    if (st != MSD_OK) return st;
-    if (!tree_ok(tree) || !argmax_dev) return fail(c, MSD_ERR_INVALID, "null tree or argmax");
-    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
-    st = check_capacity(c);
-    if (st != MSD_OK) return st;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
+namespace {
+
+// One step (kind 0: draft, verify, accept; kind 1: plain greedy) recorded once
+// into a CUDA graph per set of buffers and per bucket of cache lengths, then
+// replayed.
+msd_status step_kind_eager(msd_ctx *c, int kind, const msd_tree *tree, int32_t *argmax_dev,
+                           int32_t *path_dev, int32_t *accept_len_dev, int32_t *bonus_dev, cudaStream_t s) {
     const bool bf = c->cfg.dtype == MSD_BF16;
+    if (kind == 1) return bf ? ar_impl<bf16>(c, bonus_dev, s) : ar_impl<float>(c, bonus_dev, s);
+    return bf ? step_eager<bf16>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, s)
+              : step_eager<float>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, s);
+}
+
+msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
+                          int32_t *accept_len_dev, int32_t *bonus_dev, cudaStream_t s) {
+    msd_status st;
+    const int grow = kind == 1 ? 1 : c->D1;      // upper bound of L's growth per step
     // While GEMM profiling is on, steps run eagerly (events bracket each GEMM).
-    if (bf && c->gplan && gemm_profile_on(c->gplan)) {
-        st = step_eager<bf16>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, s);
+    if (c->cfg.dtype == MSD_BF16 && c->gplan && gemm_profile_on(c->gplan)) {
+        st = step_kind_eager(c, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, s);
         return st == MSD_OK ? post_status(c, s) : st;
     }
     int need = max_L_bound(c);
     msd_ctx::StepGraph *g = nullptr;
     bool rollover = false;
     for (auto &x : c->graphs)
-        if (same_buffers(x, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev)) {
+        if (same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev)) {
             if (x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi)) g = &x;
             else rollover = true;
         }
@@ -921,13 +952,14 @@ msd_status msd_step(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, int32
             for (int b = 0; b < c->B; ++b) c->L_bound[b] = L[b];
             need = max_L_bound(c);
             for (auto &x : c->graphs)
-                if (same_buffers(x, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev) &&
+                if (same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev) &&
                     x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi))
                     g = &x;
         }
     }
     if (!g) {
         msd_ctx::StepGraph ng;
+        ng.kind = kind;
         ng.bucket_hi = std::min(c->S, ((need + c->D + 511) / 512) * 512);
         ng.tree = *tree;
         ng.argmax = argmax_dev; ng.path = path_dev; ng.alen = accept_len_dev; ng.bonus = bonus_dev;
@@ -939,11 +971,10 @@ msd_status msd_step(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, int32
         cudaGraph_t graph = nullptr;
         cudaError_t ce = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
         if (ce == cudaSuccess) {
-            st = bf ? step_eager<bf16>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev,
-                                       c->cap_stream)
-                    : step_eager<float>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev,
-                                        c->cap_stream);
+            st = step_kind_eager(c, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, c->cap_stream);
             ce = cudaStreamEndCapture(c->cap_stream, &graph);
+        } else {
+            st = MSD_OK;
         }
         c->capturing = false;
         c->pb_override = 0;
@@ -972,8 +1003,44 @@ msd_status msd_step(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, int32
     CU(cudaGraphLaunch(g->exec, s));
     g->uses += 1;
     c->graph_kernels += g->kernels;
-    for (int b = 0; b < c->B; ++b) c->L_bound[b] += c->D1;
+    for (int b = 0; b < c->B; ++b) c->L_bound[b] += grow;
     return post_status(c, s);
+}
+
+}  // namespace
+
+msd_status msd_step(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
+                    int32_t *accept_len_dev, int32_t *bonus_dev, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    if (report_stale_error("msd_step"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!tree_ok(tree) || !argmax_dev) return fail(c, MSD_ERR_INVALID, "null tree or argmax");
+    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    if (c->draft_stale)
+        return fail(c, MSD_ERR_INVALID, "msd_ar_step ran since the last msd_prefill: the draft cache is stale");
+    st = check_capacity(c);
+    if (st != MSD_OK) return st;
+    return run_step_graph(c, 0, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev,
+                          static_cast<cudaStream_t>(stream));
+}
+
+msd_status msd_ar_step(msd_ctx *c, int32_t *token_dev, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    if (report_stale_error("msd_ar_step"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!token_dev) return fail(c, MSD_ERR_INVALID, "null token output");
+    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    st = check_capacity(c);
+    if (st != MSD_OK) return st;
+    c->draft_stale = true;
+    return run_step_graph(c, 1, &c->ar_tree, c->ar_argmax, nullptr, nullptr, token_dev,
+                          static_cast<cudaStream_t>(stream));
 }
 
 msd_status msd_linear(msd_ctx *c, const void *x, int32_t ldx, int32_t m, int32_t k, const void *w,

@@ -71,6 +71,7 @@ _SIGNATURES = {
                                      c_void_p, c_void_p, c_void_p]),
     "msd_step": (c_int32, [c_void_p, POINTER(msd_tree), c_void_p, c_void_p, c_void_p, c_void_p,
                            c_void_p]),
+    "msd_ar_step": (c_int32, [c_void_p, c_void_p, c_void_p]),
     "msd_linear": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32,
                              c_void_p, c_int32, c_int32, c_void_p]),
     "msd_linear_noalloc": (c_int32, [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32,
@@ -240,6 +241,16 @@ class Engine:
         self.draft_tree(stream=stream)
         self.verify(stream=stream)
         return self.accept_compact(stream=stream)
+
+    def ar_step(self, out: torch.Tensor | None = None, stream=None):
+        """One plain greedy decode step (msd_ar_step): the next token of every request."""
+        if out is None:
+            if getattr(self, "_ar_out", None) is None:
+                self._ar_out = torch.zeros(self.cfg.max_batch, dtype=torch.int32, device="cuda")
+            out = self._ar_out
+        st = lib().msd_ar_step(self.ctx, _ptr(out), _stream(stream))
+        self._check(st, "msd_ar_step")
+        return out
 
     def linear(self, x: torch.Tensor, w: torch.Tensor, y: torch.Tensor, accumulate=False,
                stream=None):
