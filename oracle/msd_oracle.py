@@ -43,6 +43,17 @@ Readings where the paper is silent (each also listed in the design notes):
   R5 draft positions: the draft row that carries h_i sits at position i; a
      depth-d tree node sits at draft position L-1+d and target position L+d.
   R6 a prefix must end with a text token.
+  R7 temperature T > 0 (speculative sampling): the target distribution at a
+     node is p = softmax(logits / T). The tree's candidates are the draft's
+     top-k choices, not samples of q, so the distribution that proposed a
+     candidate -- given the siblings already rejected -- is a point mass at it:
+     Eq. 6's min(1, p/q) accepts it with probability p(x), and the adjusted
+     distribution norm(max(0, p - q)) is p with x removed and renormalised.
+     Children are tried in tree order (best draft score first); the token that
+     ends the walk is drawn from the adjusted p (all children rejected) or from
+     p itself (a leaf). Draws are inverse-CDF in token-id order. The uniforms
+     are inputs: u[d][j] for the j-th child tried at depth d, u[d][k] for the
+     token drawn at depth d.
 """
 from __future__ import annotations
 
@@ -577,6 +588,56 @@ def accept(tree: Tree, argmax) -> tuple:
         cur = nxt[0]
         path.append(cur)
     return np.array(path, np.int64), len(path) - 1, int(argmax[cur])
+
+
+def sample_index(p: np.ndarray, u: float, removed=()) -> int:
+    """Inverse-CDF draw from p restricted to the tokens not in `removed`:
+    the smallest token id t whose cumulative mass (token-id order, removed
+    tokens skipped) exceeds u times the remaining mass (R7)."""
+    q = np.asarray(p, F64).copy()
+    for x in removed:
+        q[x] = 0.0
+    target = float(u) * q.sum()
+    c = np.cumsum(q)
+    hit = np.flatnonzero(c > target)
+    if hit.size:
+        return int(hit[0])
+    return int(np.flatnonzero(q > 0)[-1])           # rounding at the very top
+
+
+def accept_sample(tree: Tree, logits, temperature: float, u, k: int) -> tuple:
+    """Speculative sampling over the tree at temperature T > 0 (Sec. 3.2,
+    Eq. 6 and the adjusted distribution after it; reading R7).
+
+    From the root: p = softmax(logits[node] / T); each child x in tree order is
+    accepted with probability p_adj(x) (a draw u < p_adj(x)); a rejection
+    removes x from p_adj. An accepted child becomes the node and the walk goes
+    on; when a node's children are all rejected, or it has none, the next
+    token is drawn from p_adj and the walk ends. Returns (path, a, bonus).
+    """
+    path = [0]
+    cur = 0
+    d = 0
+    while True:
+        z = np.asarray(logits[cur], F64) / float(temperature)
+        p = softmax(z)
+        children = [c for c in range(tree.n) if tree.parent[c] == cur]
+        removed = []
+        nxt = None
+        for j, c in enumerate(children):
+            x = int(tree.tokens[c])
+            rest = 1.0 - sum(p[r] for r in removed)
+            px = 0.0 if x in removed else p[x]
+            if u[d][j] * rest < px:
+                nxt = c
+                break
+            if x not in removed:
+                removed.append(x)
+        if nxt is None:
+            return np.array(path, np.int64), len(path) - 1, sample_index(p, u[d][k], removed)
+        path.append(nxt)
+        cur = nxt
+        d += 1
 
 
 def compact(st: RequestState, tree: Tree, vr: VerifyResult, path, bonus):
