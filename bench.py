@@ -58,6 +58,8 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-ar", action="store_true",
                     help="skip the plain greedy decoding baseline (speedup ratio)")
+    ap.add_argument("--no-sampling", action="store_true",
+                    help="skip the temperature-1 speculative sampling step timing")
     ap.add_argument("--layers", type=int, default=None,
                     help="cut the target to this many layers (small cases for profiling only)")
     ap.add_argument("--gemm", default=None,
@@ -441,6 +443,38 @@ def run_msd(args, rank, world, local_rank):
                 "note": "projection: the paper's average acceptance length of trained MSD drafts, "
                         "not measured here"}
 
+    # ---- speculative sampling at T = 1 (Eq. 6 over the tree): msd_step_sample,
+    # a replayed graph of draft, verify and the sampling walk + compaction; the
+    # uniforms are inputs, copied device to device into the step's buffer
+    sampling = None
+    if not args.no_sampling:
+        K_s, T_s = min(K, 32), 1.0
+        shape = (B, D + 1, wl.topk + 1)
+        g_u = torch.Generator(device="cuda").manual_seed(1234)
+        u_all = torch.rand((K_s + 3,) + shape, device="cuda", generator=g_u)
+        u_buf = torch.empty(shape, device="cuda")
+        for i in range(3):
+            u_buf.copy_(u_all[i])
+            eng.step_sample(T_s, u_buf)
+        torch.cuda.synchronize()
+        Ls0 = eng.state()["seq_len"].cpu().numpy().astype(np.int64)
+        e0.record(stream)
+        for i in range(K_s):
+            u_buf.copy_(u_all[3 + i], non_blocking=True)
+            eng.step_sample(T_s, u_buf)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        ms_s = e0.elapsed_time(e1)
+        Ls1 = eng.state()["seq_len"].cpu().numpy().astype(np.int64)
+        tok_s = int((Ls1 - Ls0).sum())
+        sampling = {"temperature": T_s, "steps": K_s, "ms_per_step": ms_s / K_s,
+                    "steps_per_s": world * K_s / (ms_s / 1e3), "tokens_per_s": world * tok_s / (ms_s / 1e3),
+                    "tau": tok_s / (K_s * B),
+                    "note": "msd_step_sample: draft tree, verify, speculative sampling over the tree "
+                            "(Eq. 6, top-k candidates as point-mass proposals) and compaction, one replayed "
+                            "graph per step after 3 warm-up steps; uniforms copied into its buffer before "
+                            "each step (inside the timed region)"}
+
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
         try:
@@ -483,6 +517,7 @@ def run_msd(args, rank, world, local_rank):
             "cpu_baseline": cpu,
             "e2e": e2e,
             "speedup": speedup,
+            "sampling": sampling,
             "gpu_launches": int(launches1 - launches0),
             "clocks": clk,
         }

@@ -1,7 +1,7 @@
 /*
  * msd.h - C ABI of the GB300 (sm_103a) hot path of Multimodal Speculative
- * Decoding (MSD, arXiv 2505.14260): one greedy draft -> verify -> accept ->
- * compact decode step of a LLaVA-style decoder.
+ * Decoding (MSD, arXiv 2505.14260): one draft -> verify -> accept -> compact
+ * decode step of a LLaVA-style decoder, greedy (T = 0) or sampling (T > 0).
  *
  * Conventions shared by every call
  * --------------------------------
@@ -173,6 +173,38 @@ msd_status msd_accept_compact(msd_ctx *ctx, const msd_tree *tree,
                               int32_t *accept_len_dev, int32_t *bonus_dev,
                               int32_t *index_map_dev, void *stream);
 
+/* Accept and compact at temperature T > 0: speculative sampling over the tree
+ * (Sec. 3.2, Eq. 6 and the adjusted distribution norm(max(0, p - q)) after it).
+ * The target distribution at node i is p = softmax(logits[b][i] / T). The
+ * tree's candidates are the draft's top-k choices, not draws from q, so the
+ * proposal of a child -- given its siblings already rejected -- is a point mass
+ * at its token x: Eq. 6 accepts it with probability p_adj(x), and the adjusted
+ * distribution is p_adj with x removed and renormalised (p_adj = p at first).
+ * From the root, the children of the current node are tried in tree order
+ * (index order: best draft score first) with u_dev[(b*(D+1) + d)*(k+1) + j]
+ * for the j-th child tried at depth d (d = drafts accepted so far); an accepted
+ * child becomes the current node. When all of a node's children are rejected,
+ * or it has none, the next token (the bonus) is drawn from p_adj by inverse CDF
+ * in token-id order: the smallest token whose cumulative mass exceeds
+ * u_dev[(b*(D+1) + d)*(k+1) + k] times the remaining mass.
+ * logits_dev: the fp32 [B][N][V] logits of the preceding msd_verify -- the
+ * same pointer that call was given, or NULL if it was given NULL (the context
+ * keeps them then). u_dev: [B][D+1][k+1] fp32 uniforms in [0, 1), device,
+ * caller-owned (the random numbers are inputs, so a step is reproducible).
+ * temperature: finite, > 0. A node with more than k children in a
+ * caller-planted tree has only its first k tried and sets the device status.
+ * Decisions are taken on the fp32 logits with fp32 exponentials and
+ * error-free (fp32 pair / fp64) sums: they agree with an exact evaluation
+ * except where a uniform lies within about 1e-6 (relative) of a boundary.
+ * Outputs, compaction and state update as msd_accept_compact (path, accepted
+ * length a, bonus = the drawn token, index map). Errors: MSD_ERR_INVALID (null
+ * tree or u_dev, bad temperature, no prefill), MSD_ERR_CAPACITY,
+ * MSD_ERR_DEVICE, MSD_ERR_CUDA. */
+msd_status msd_accept_sample(msd_ctx *ctx, const msd_tree *tree, const float *logits_dev,
+                             float temperature, const float *u_dev, int32_t *path_dev,
+                             int32_t *accept_len_dev, int32_t *bonus_dev, int32_t *index_map_dev,
+                             void *stream);
+
 /* One whole decode step: msd_draft_tree, msd_verify and msd_accept_compact in
  * sequence (Sec. 3.2; Eq. 6 at T = 0), with the same arguments and outputs as
  * those calls (the drafted tree is written to *tree and then verified). The
@@ -185,6 +217,17 @@ msd_status msd_accept_compact(msd_ctx *ctx, const msd_tree *tree,
  * graph cannot be recorded. */
 msd_status msd_step(msd_ctx *ctx, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
                     int32_t *accept_len_dev, int32_t *bonus_dev, void *stream);
+
+/* One whole decode step at temperature T > 0: msd_draft_tree, msd_verify (its
+ * logits kept in the context) and msd_accept_sample, recorded and replayed as a
+ * CUDA graph exactly as msd_step (one graph per set of buffers, u_dev pointer,
+ * temperature and bucket of cache lengths). The caller refills u_dev
+ * ([B][D+1][k+1] uniforms in [0, 1)) before each step; the graph reads it when
+ * it runs. Errors: as msd_step, and MSD_ERR_INVALID for a null u_dev or a
+ * temperature that is not finite and > 0. */
+msd_status msd_step_sample(msd_ctx *ctx, const msd_tree *tree, float temperature,
+                           const float *u_dev, int32_t *argmax_dev, int32_t *path_dev,
+                           int32_t *accept_len_dev, int32_t *bonus_dev, void *stream);
 
 /* Plain greedy autoregressive decoding, the baseline against which the paper
  * measures its speedup ratio (Sec. 4.1, Eq. 9: T_p, the target's time per

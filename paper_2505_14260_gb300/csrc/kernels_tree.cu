@@ -306,6 +306,39 @@ __global__ void root_tree_kernel(const int *__restrict__ root, int B, int N, int
 // Greedy acceptance (Eq. 6 at T = 0): one warp per request walks from the root
 // to the child whose token is the target argmax of the current node.
 // ---------------------------------------------------------------------------
+// Outcome of an acceptance walk of request b: path (root 0, then the a accepted
+// nodes, -1 beyond) and the index map; the pending draft rows (each accepted
+// position paired with the token after it: the next accepted draft token, or
+// the bonus); the state update L <- L + a + 1, root <- bonus. `path` is in
+// shared memory, visible to every thread of the block.
+__device__ __forceinline__ void write_acceptance(const TreeIn &t, const int *path, int a, int bonus,
+                                                 int b, int N, int D1, int *__restrict__ seq_len,
+                                                 int *__restrict__ n_pend, int *__restrict__ root,
+                                                 int *__restrict__ pend_next, int *__restrict__ acc_path,
+                                                 int *__restrict__ acc_L0, int *__restrict__ acc_a,
+                                                 int *__restrict__ path_out, int *__restrict__ accept_len_out,
+                                                 int *__restrict__ bonus_out, int *__restrict__ index_map_out) {
+    const size_t nb = (size_t)b * N;
+    const int L0 = seq_len[b];
+    for (int j = threadIdx.x; j < D1; j += blockDim.x) {
+        const int pj = j <= a ? path[j] : -1;
+        acc_path[b * D1 + j] = pj;
+        if (path_out) path_out[b * D1 + j] = pj;
+        if (index_map_out) index_map_out[b * D1 + j] = j <= a ? L0 + j : -1;
+        if (j <= a) pend_next[b * D1 + j] = j < a ? t.tokens[nb + path[j + 1]] : bonus;
+    }
+    __syncthreads();   // every thread has read seq_len[b] before it changes
+    if (threadIdx.x == 0) {
+        acc_L0[b] = L0;
+        acc_a[b] = a;
+        if (accept_len_out) accept_len_out[b] = a;
+        if (bonus_out) bonus_out[b] = bonus;
+        n_pend[b] = a + 1;
+        seq_len[b] = L0 + a + 1;
+        root[b] = bonus;
+    }
+}
+
 __global__ void accept_kernel(TreeIn t, const int *__restrict__ argmax, int N, int D,
                               int *__restrict__ seq_len, int *__restrict__ n_pend,
                               int *__restrict__ root, int *__restrict__ pend_next,
@@ -315,7 +348,7 @@ __global__ void accept_kernel(TreeIn t, const int *__restrict__ argmax, int N, i
                               int *__restrict__ index_map_out) {
     wait_prior();
     allow_dependents();
-    const int b = blockIdx.x, lane = threadIdx.x, D1 = D + 1;
+    const int b = blockIdx.x, lane = threadIdx.x;
     const size_t nb = (size_t)b * N;
     const int n = t.n_nodes ? t.n_nodes[b] : N;
     __shared__ int path[TREE_MAXD + 1];
@@ -334,24 +367,217 @@ __global__ void accept_kernel(TreeIn t, const int *__restrict__ argmax, int N, i
         if (lane == 0) path[a] = cur;
     }
     __syncwarp();
-    const int bonus = argmax[nb + cur];
-    const int L0 = seq_len[b];
-    for (int j = lane; j < D1; j += 32) {
-        const int pj = j <= a ? path[j] : -1;
-        acc_path[b * D1 + j] = pj;
-        if (path_out) path_out[b * D1 + j] = pj;
-        if (index_map_out) index_map_out[b * D1 + j] = j <= a ? L0 + j : -1;
-        if (j <= a) pend_next[b * D1 + j] = j < a ? t.tokens[nb + path[j + 1]] : bonus;
+    write_acceptance(t, path, a, argmax[nb + cur], b, N, D + 1, seq_len, n_pend, root, pend_next,
+                     acc_path, acc_L0, acc_a, path_out, accept_len_out, bonus_out, index_map_out);
+}
+
+// ---------------------------------------------------------------------------
+// Speculative sampling over the tree at temperature T > 0 (Sec. 3.2, Eq. 6 and
+// the adjusted distribution after it). The tree's candidates are the draft's
+// top-k choices, so the proposal of a child -- given the siblings already
+// rejected -- is a point mass at its token x: Eq. 6's min(1, p/q) accepts it
+// with probability p_adj(x), and the adjusted distribution norm(max(0, p - q))
+// is p_adj with x removed and renormalised. At a node, p = softmax(z / T) of
+// its verify logits; the children are tried in tree order (best draft score
+// first) with uniforms u[b][d][j] (d = accepted so far, j = child ordinal); an
+// accepted child becomes the node. When every child is rejected, or the node
+// is a leaf, the next token is drawn from p_adj by inverse CDF in token-id
+// order with u[b][d][k] (the smallest token whose cumulative mass exceeds u
+// times the remaining mass).
+//
+// One CTA per request. Each thread owns a contiguous run of the vocabulary; a
+// node's row is reduced twice (max, then the sum of exp((z - max) / T)), every
+// exponential in fp32 and every sum as an fp32 TwoSum pair (Knuth's error-free
+// addition) combined across threads in fp64, so the decisions carry only the
+// exponentials' rounding (about 1e-6 relative).
+// ---------------------------------------------------------------------------
+constexpr int SAMPLE_THREADS = 1024;
+
+// hi + lo += x with the rounding error of the addition kept in lo.
+__device__ __forceinline__ void two_sum_add(float &hi, float &lo, float x) {
+    const float s = hi + x;
+    const float bp = s - hi;
+    lo += (hi - (s - bp)) + (x - bp);
+    hi = s;
+}
+
+__device__ __forceinline__ double block_sum_f64(double v, double *red) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    __syncthreads();
+    if (lane == 0) red[warp] = v;
+    __syncthreads();
+    if (warp == 0) {
+        double w = lane < nw ? red[lane] : 0.0;
+#pragma unroll
+        for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
+        if (lane == 0) red[32] = w;
     }
-    if (lane == 0) {
-        acc_L0[b] = L0;
-        acc_a[b] = a;
-        if (accept_len_out) accept_len_out[b] = a;
-        if (bonus_out) bonus_out[b] = bonus;
-        n_pend[b] = a + 1;
-        seq_len[b] = L0 + a + 1;
-        root[b] = bonus;
+    __syncthreads();
+    return red[32];
+}
+
+// Exclusive prefix sum over the block in thread order; *total = the sum of all.
+__device__ __forceinline__ double block_exscan_f64(double v, double *red, double *total) {
+    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
+    double inc = v;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const double y = __shfl_up_sync(0xffffffffu, inc, o);
+        if (lane >= o) inc += y;
     }
+    double excl = __shfl_up_sync(0xffffffffu, inc, 1);
+    if (lane == 0) excl = 0.0;
+    __syncthreads();
+    if (lane == 31) red[warp] = inc;
+    __syncthreads();
+    if (warp == 0) {
+        double w = lane < nw ? red[lane] : 0.0;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const double y = __shfl_up_sync(0xffffffffu, w, o);
+            if (lane >= o) w += y;
+        }
+        red[lane] = w;            // inclusive prefix of the warp totals
+    }
+    __syncthreads();
+    *total = red[nw - 1];
+    return (warp > 0 ? red[warp - 1] : 0.0) + excl;
+}
+
+__global__ void __launch_bounds__(SAMPLE_THREADS)
+accept_sample_kernel(TreeIn t, const float *__restrict__ logits, int N, int D, int k, int V,
+                     float inv_temp, const float *__restrict__ u, int *__restrict__ seq_len,
+                     int *__restrict__ n_pend, int *__restrict__ root, int *__restrict__ pend_next,
+                     int *__restrict__ acc_path, int *__restrict__ acc_L0, int *__restrict__ acc_a,
+                     int *__restrict__ path_out, int *__restrict__ accept_len_out,
+                     int *__restrict__ bonus_out, int *__restrict__ index_map_out, int *status) {
+    wait_prior();
+    allow_dependents();
+    const int b = blockIdx.x, tid = threadIdx.x, D1 = D + 1;
+    const size_t nb = (size_t)b * N;
+    const int n = t.n_nodes ? min(max(t.n_nodes[b], 1), N) : N;
+    const float *ub = u + (size_t)b * D1 * (k + 1);
+    __shared__ int path[TREE_MAXD + 1];
+    __shared__ int kids[TREE_MAXK], removed[TREE_MAXK];
+    __shared__ int sh_next, sh_nrem, sh_pick, sh_last;
+    __shared__ float redf[32];
+    __shared__ double red[33];
+    __shared__ double bound[SAMPLE_THREADS + 1];
+    const int per = (V + blockDim.x - 1) / blockDim.x;
+    const int lo = min(tid * per, V), hi = min(lo + per, V);
+    if (tid == 0) path[0] = 0;
+    int cur = 0, a = 0;
+    const float *row;
+    float M;
+    for (;;) {
+        row = logits + (nb + cur) * V;
+        float m = -INFINITY;
+        for (int i = lo; i < hi; ++i) m = fmaxf(m, row[i]);
+        M = block_max(m, redf);
+        float sh = 0.f, sl = 0.f;
+        for (int i = lo; i < hi; ++i) two_sum_add(sh, sl, expf((row[i] - M) * inv_temp));
+        const double S = block_sum_f64((double)sh + (double)sl, red);
+        if (tid < 32) {
+            // children of the node, in tree order (at most k are tried)
+            int cnt = 0;
+            for (int c0 = 1; c0 < n; c0 += 32) {
+                const int c = c0 + tid;
+                const bool is = c < n && t.parent[nb + c] == cur;
+                const unsigned bal = __ballot_sync(0xffffffffu, is);
+                const int slot = cnt + __popc(bal & ((1u << tid) - 1u));
+                if (is && slot < k) kids[slot] = c;
+                cnt += __popc(bal);
+            }
+            __syncwarp();
+            if (tid == 0) {
+                if (cnt > k) set_status(status, ST_BAD_TREE);
+                const int nk = a < D ? min(cnt, k) : 0;
+                int next = -1, nrem = 0;
+                double gone = 0.0;        // mass of the tokens already rejected at this node
+                for (int j = 0; j < nk; ++j) {
+                    const int x = t.tokens[nb + kids[j]];
+                    if (x < 0 || x >= V) {
+                        set_status(status, ST_BAD_TOKEN);
+                        continue;
+                    }
+                    bool dup = false;
+                    for (int r = 0; r < nrem; ++r) dup |= removed[r] == x;
+                    const double px = dup ? 0.0 : (double)expf((row[x] - M) * inv_temp) / S;
+                    if ((double)ub[a * (k + 1) + j] * (1.0 - gone) < px) {
+                        next = kids[j];
+                        break;
+                    }
+                    if (!dup) {
+                        removed[nrem++] = x;
+                        gone += px;
+                    }
+                }
+                sh_next = next;
+                sh_nrem = nrem;
+                sh_pick = -1;
+                sh_last = -1;
+            }
+        }
+        __syncthreads();
+        const int next = sh_next;
+        if (next < 0) break;
+        cur = next;
+        ++a;
+        if (tid == 0) path[a] = cur;
+    }
+    // the next token: inverse CDF of p_adj at the last node, in token-id order
+    const int nrem = sh_nrem;
+    float ph = 0.f, pl = 0.f;
+    int last = -1;
+    for (int i = lo; i < hi; ++i) {
+        bool rm = false;
+        for (int r = 0; r < nrem; ++r) rm |= removed[r] == i;
+        if (rm) continue;
+        const float e = expf((row[i] - M) * inv_temp);
+        two_sum_add(ph, pl, e);
+        if (e > 0.f) last = i;
+    }
+    double total;
+    const double excl = block_exscan_f64((double)ph + (double)pl, red, &total);
+    bound[tid] = excl;
+    if (tid == 0) bound[blockDim.x] = total;
+    if (last >= 0) atomicMax(&sh_last, last);
+    __syncthreads();
+    const double target = (double)ub[a * (k + 1) + k] * total;
+    if (bound[tid] <= target && target < bound[tid + 1]) {
+        double c = excl;
+        int pick = -1, lastp = -1;
+        for (int i = lo; i < hi; ++i) {
+            bool rm = false;
+            for (int r = 0; r < nrem; ++r) rm |= removed[r] == i;
+            if (rm) continue;
+            const float e = expf((row[i] - M) * inv_temp);
+            if (e > 0.f) lastp = i;
+            c += (double)e;
+            if (c > target) {
+                pick = i;
+                break;
+            }
+        }
+        sh_pick = pick >= 0 ? pick : lastp;   // the bounds partition [0, total): one thread
+    }
+    __syncthreads();
+    if (tid == 0) {
+        int bo = sh_pick >= 0 ? sh_pick : sh_last;
+        if (bo < 0) {
+            // no mass left (only with u >= 1 or every positive token removed): the argmax
+            bo = 0;
+            for (int i = 0; i < V; ++i)
+                if (row[i] == M) { bo = i; break; }
+        }
+        sh_next = bo;
+    }
+    __syncthreads();
+    const int bonus = sh_next;
+    write_acceptance(t, path, a, bonus, b, N, D1, seq_len, n_pend, root, pend_next, acc_path, acc_L0,
+                     acc_a, path_out, accept_len_out, bonus_out, index_map_out);
 }
 
 // K/V of accepted node path[j] -> cache position L0 + j, all layers and heads.
@@ -507,6 +733,16 @@ void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int 
     launch_pdl(accept_kernel, B, 32, 0, s, t, argmax, N, D, seq_len, n_pend, root, pend_next, acc_path,
                                    acc_L0, acc_a, path_out, accept_len_out, bonus_out,
                                    index_map_out); note_launch();
+}
+
+void launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, int D, int k, int V,
+                          float inv_temp, const float *u, int *seq_len, int *n_pend, int *root,
+                          int *pend_next, int *acc_path, int *acc_L0, int *acc_a, int *path_out,
+                          int *accept_len_out, int *bonus_out, int *index_map_out, int *status,
+                          cudaStream_t s) {
+    launch_pdl(accept_sample_kernel, B, SAMPLE_THREADS, 0, s, t, logits, N, D, k, V, inv_temp, u, seq_len,
+               n_pend, root, pend_next, acc_path, acc_L0, acc_a, path_out, accept_len_out, bonus_out,
+               index_map_out, status); note_launch();
 }
 
 void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, const int *acc_L0,

@@ -5,6 +5,8 @@
 //                      model (Sec. 3.2, Eq. 4-5) with the decoupled input (Eq. 7)
 //   msd_verify         one tree-masked target forward (Sec. 3.2, verification)
 //   msd_accept_compact greedy acceptance (Eq. 6 at T = 0) + KV compaction
+//   msd_accept_sample  speculative sampling over the tree (Eq. 6, T > 0) + KV
+//                      compaction
 // Every size a kernel needs at run time (L, accepted length, pending rows) is
 // read by the kernels from device state, so a step needs no host round trip.
 #include <cmath>
@@ -79,10 +81,13 @@ struct msd_ctx {
     // whole-step CUDA graphs (msd_step), one per L bucket and buffer set
     struct StepGraph {
         cudaGraphExec_t exec = nullptr;
-        int kind = 0;               // 0: draft-verify-accept step, 1: plain greedy step
+        int kind = 0;               // 0: draft-verify-accept step, 1: plain greedy step,
+                                    // 2: draft-verify-sample step
         int bucket_hi = 0;
         msd_tree tree{};
         const void *argmax = nullptr, *path = nullptr, *alen = nullptr, *bonus = nullptr;
+        const void *u = nullptr;    // kind 2: the uniforms' buffer and the temperature
+        float temp = 0.f;
         long kernels = 0;
         long uses = 0;
     };
@@ -554,12 +559,11 @@ msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, fl
     return post_status(c, s);
 }
 
+// Compaction after an acceptance kernel has written acc_path / acc_L0 / acc_a:
+// the accepted nodes' K/V move into the cache, their features become the
+// draft's pending rows.
 template <typename T>
-msd_status accept_impl(msd_ctx *c, const msd_tree *tree, const int32_t *argmax, int32_t *path,
-                       int32_t *alen, int32_t *bonus, int32_t *imap, cudaStream_t s, int grow = -1) {
-    TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
-    launch_accept(t, argmax, c->B, c->N, c->D, c->seq_len, c->n_pend, c->root, c->pend_next,
-                  c->acc_path, c->acc_L0, c->acc_a, path, alen, bonus, imap, s);
+msd_status compact_impl(msd_ctx *c, cudaStream_t s, int grow) {
     launch_compact_kv(c->tree_kv, c->target_kv, c->acc_path, c->acc_L0, c->acc_a, c->NL, c->B, c->nh,
                       c->N, c->S, c->D1, (int)(c->hd * c->esz), c->status, s);
     launch_pend_h<T>(static_cast<const T *>(c->hT), c->acc_path, c->acc_a, c->B, c->N, c->D1, c->H,
@@ -567,6 +571,28 @@ msd_status accept_impl(msd_ctx *c, const msd_tree *tree, const int32_t *argmax, 
     if (!c->capturing)
         for (int b = 0; b < c->B; ++b) c->L_bound[b] += grow < 0 ? c->D1 : grow;
     return post_status(c, s);
+}
+
+template <typename T>
+msd_status accept_impl(msd_ctx *c, const msd_tree *tree, const int32_t *argmax, int32_t *path,
+                       int32_t *alen, int32_t *bonus, int32_t *imap, cudaStream_t s, int grow = -1) {
+    TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
+    launch_accept(t, argmax, c->B, c->N, c->D, c->seq_len, c->n_pend, c->root, c->pend_next,
+                  c->acc_path, c->acc_L0, c->acc_a, path, alen, bonus, imap, s);
+    return compact_impl<T>(c, s, grow);
+}
+
+// Speculative sampling at temperature T > 0 (Eq. 6 over the tree), then the
+// same compaction. `logits` are the verify pass's [B][N][V].
+template <typename T>
+msd_status accept_sample_impl(msd_ctx *c, const msd_tree *tree, const float *logits, float temp,
+                              const float *u, int32_t *path, int32_t *alen, int32_t *bonus,
+                              int32_t *imap, cudaStream_t s) {
+    TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
+    launch_accept_sample(t, logits, c->B, c->N, c->D, c->k, c->V, (float)(1.0 / (double)temp), u,
+                         c->seq_len, c->n_pend, c->root, c->pend_next, c->acc_path, c->acc_L0, c->acc_a,
+                         path, alen, bonus, imap, c->status, s);
+    return compact_impl<T>(c, s, -1);
 }
 
 // Plain greedy autoregressive decoding, the baseline of the speedup ratio
@@ -664,11 +690,29 @@ msd_status step_eager(msd_ctx *c, const msd_tree *tree, int32_t *argmax, int32_t
     return st;
 }
 
+// The sampling step: the verify logits stay in the context's buffer.
+template <typename T>
+msd_status step_sample_eager(msd_ctx *c, const msd_tree *tree, int32_t *argmax, float temp,
+                             const float *u, int32_t *path, int32_t *alen, int32_t *bonus,
+                             cudaStream_t s) {
+    msd_status st = draft_impl<T>(c, tree, nullptr, s);
+    if (st == MSD_OK) st = verify_impl<T>(c, tree, argmax, nullptr, s);
+    if (st == MSD_OK) st = accept_sample_impl<T>(c, tree, c->logits, temp, u, path, alen, bonus, nullptr, s);
+    return st;
+}
+
+// Sampling parameters of a kind-2 step.
+struct SampleArgs {
+    const float *u;
+    float temp;
+};
+
 bool same_buffers(const msd_ctx::StepGraph &g, int kind, const msd_tree *t, const void *a,
-                         const void *p, const void *l, const void *b) {
+                         const void *p, const void *l, const void *b, const SampleArgs *sa) {
     return g.kind == kind && g.tree.tokens == t->tokens && g.tree.parent == t->parent && g.tree.depth == t->depth &&
            g.tree.mask == t->mask && g.tree.n_nodes == t->n_nodes && g.argmax == a &&
-           g.path == p && g.alen == l && g.bonus == b;
+           g.path == p && g.alen == l && g.bonus == b &&
+           (!sa || (g.u == sa->u && g.temp == sa->temp));
 }
 
 }  // namespace
@@ -920,27 +964,34 @@ namespace {
 // into a CUDA graph per set of buffers and per bucket of cache lengths, then
 // replayed.
 msd_status step_kind_eager(msd_ctx *c, int kind, const msd_tree *tree, int32_t *argmax_dev,
-                           int32_t *path_dev, int32_t *accept_len_dev, int32_t *bonus_dev, cudaStream_t s) {
+                           int32_t *path_dev, int32_t *accept_len_dev, int32_t *bonus_dev,
+                           const SampleArgs *sa, cudaStream_t s) {
     const bool bf = c->cfg.dtype == MSD_BF16;
     if (kind == 1) return bf ? ar_impl<bf16>(c, bonus_dev, s) : ar_impl<float>(c, bonus_dev, s);
+    if (kind == 2)
+        return bf ? step_sample_eager<bf16>(c, tree, argmax_dev, sa->temp, sa->u, path_dev, accept_len_dev,
+                                            bonus_dev, s)
+                  : step_sample_eager<float>(c, tree, argmax_dev, sa->temp, sa->u, path_dev, accept_len_dev,
+                                             bonus_dev, s);
     return bf ? step_eager<bf16>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, s)
               : step_eager<float>(c, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, s);
 }
 
 msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
-                          int32_t *accept_len_dev, int32_t *bonus_dev, cudaStream_t s) {
+                          int32_t *accept_len_dev, int32_t *bonus_dev, const SampleArgs *sa,
+                          cudaStream_t s) {
     msd_status st;
     const int grow = kind == 1 ? 1 : c->D1;      // upper bound of L's growth per step
     // While GEMM profiling is on, steps run eagerly (events bracket each GEMM).
     if (c->cfg.dtype == MSD_BF16 && c->gplan && gemm_profile_on(c->gplan)) {
-        st = step_kind_eager(c, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, s);
+        st = step_kind_eager(c, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa, s);
         return st == MSD_OK ? post_status(c, s) : st;
     }
     int need = max_L_bound(c);
     msd_ctx::StepGraph *g = nullptr;
     bool rollover = false;
     for (auto &x : c->graphs)
-        if (same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev)) {
+        if (same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa)) {
             if (x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi)) g = &x;
             else rollover = true;
         }
@@ -952,7 +1003,7 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
             for (int b = 0; b < c->B; ++b) c->L_bound[b] = L[b];
             need = max_L_bound(c);
             for (auto &x : c->graphs)
-                if (same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev) &&
+                if (same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa) &&
                     x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi))
                     g = &x;
         }
@@ -963,6 +1014,7 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
         ng.bucket_hi = std::min(c->S, ((need + c->D + 511) / 512) * 512);
         ng.tree = *tree;
         ng.argmax = argmax_dev; ng.path = path_dev; ng.alen = accept_len_dev; ng.bonus = bonus_dev;
+        if (sa) { ng.u = sa->u; ng.temp = sa->temp; }
         if (!c->cap_stream)   // graphs are recorded on a stream of the context's own
             CU(cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking));
         const long l0 = launch_count();
@@ -971,7 +1023,8 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
         cudaGraph_t graph = nullptr;
         cudaError_t ce = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
         if (ce == cudaSuccess) {
-            st = step_kind_eager(c, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, c->cap_stream);
+            st = step_kind_eager(c, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa,
+                                 c->cap_stream);
             ce = cudaStreamEndCapture(c->cap_stream, &graph);
         } else {
             st = MSD_OK;
@@ -1023,7 +1076,7 @@ msd_status msd_step(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, int32
         return fail(c, MSD_ERR_INVALID, "msd_ar_step ran since the last msd_prefill: the draft cache is stale");
     st = check_capacity(c);
     if (st != MSD_OK) return st;
-    return run_step_graph(c, 0, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev,
+    return run_step_graph(c, 0, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, nullptr,
                           static_cast<cudaStream_t>(stream));
 }
 
@@ -1039,7 +1092,58 @@ msd_status msd_ar_step(msd_ctx *c, int32_t *token_dev, void *stream) {
     st = check_capacity(c);
     if (st != MSD_OK) return st;
     c->draft_stale = true;
-    return run_step_graph(c, 1, &c->ar_tree, c->ar_argmax, nullptr, nullptr, token_dev,
+    return run_step_graph(c, 1, &c->ar_tree, c->ar_argmax, nullptr, nullptr, token_dev, nullptr,
+                          static_cast<cudaStream_t>(stream));
+}
+
+// The kernel scales logits by the fp32 1/T: T must be finite, > 0, and have a
+// finite fp32 reciprocal.
+static bool temperature_ok(float t) {
+    return std::isfinite(t) && t > 0.f && std::isfinite((float)(1.0 / (double)t));
+}
+
+msd_status msd_accept_sample(msd_ctx *c, const msd_tree *tree, const float *logits_dev, float temperature,
+                             const float *u_dev, int32_t *path_dev, int32_t *accept_len_dev,
+                             int32_t *bonus_dev, int32_t *index_map_dev, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    if (report_stale_error("msd_accept_sample"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!tree_ok(tree) || !u_dev) return fail(c, MSD_ERR_INVALID, "null tree or uniforms");
+    if (!temperature_ok(temperature)) return fail(c, MSD_ERR_INVALID, "temperature must be finite and > 0");
+    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    st = check_capacity(c);
+    if (st != MSD_OK) return st;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const float *lg = logits_dev ? logits_dev : c->logits;
+    if (c->cfg.dtype == MSD_BF16)
+        return accept_sample_impl<bf16>(c, tree, lg, temperature, u_dev, path_dev, accept_len_dev, bonus_dev,
+                                        index_map_dev, s);
+    return accept_sample_impl<float>(c, tree, lg, temperature, u_dev, path_dev, accept_len_dev, bonus_dev,
+                                     index_map_dev, s);
+}
+
+msd_status msd_step_sample(msd_ctx *c, const msd_tree *tree, float temperature, const float *u_dev,
+                           int32_t *argmax_dev, int32_t *path_dev, int32_t *accept_len_dev,
+                           int32_t *bonus_dev, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    if (report_stale_error("msd_step_sample"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!tree_ok(tree) || !argmax_dev || !u_dev)
+        return fail(c, MSD_ERR_INVALID, "null tree, argmax or uniforms");
+    if (!temperature_ok(temperature)) return fail(c, MSD_ERR_INVALID, "temperature must be finite and > 0");
+    if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
+    if (c->draft_stale)
+        return fail(c, MSD_ERR_INVALID, "msd_ar_step ran since the last msd_prefill: the draft cache is stale");
+    st = check_capacity(c);
+    if (st != MSD_OK) return st;
+    const SampleArgs sa{u_dev, temperature};
+    return run_step_graph(c, 2, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, &sa,
                           static_cast<cudaStream_t>(stream));
 }
 

@@ -69,8 +69,12 @@ _SIGNATURES = {
     "msd_verify": (c_int32, [c_void_p, POINTER(msd_tree), c_void_p, c_void_p, c_void_p]),
     "msd_accept_compact": (c_int32, [c_void_p, POINTER(msd_tree), c_void_p, c_void_p, c_void_p,
                                      c_void_p, c_void_p, c_void_p]),
+    "msd_accept_sample": (c_int32, [c_void_p, POINTER(msd_tree), c_void_p, c_float, c_void_p,
+                                    c_void_p, c_void_p, c_void_p, c_void_p, c_void_p]),
     "msd_step": (c_int32, [c_void_p, POINTER(msd_tree), c_void_p, c_void_p, c_void_p, c_void_p,
                            c_void_p]),
+    "msd_step_sample": (c_int32, [c_void_p, POINTER(msd_tree), c_float, c_void_p, c_void_p, c_void_p,
+                                  c_void_p, c_void_p, c_void_p]),
     "msd_ar_step": (c_int32, [c_void_p, c_void_p, c_void_p]),
     "msd_linear": (c_int32, [c_void_p, c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32,
                              c_void_p, c_int32, c_int32, c_void_p]),
@@ -226,6 +230,27 @@ class Engine:
                                       _ptr(self.path), _ptr(self.accept_len), _ptr(self.bonus),
                                       _ptr(self.index_map), _stream(stream))
         self._check(st, "msd_accept_compact")
+        return self.path, self.accept_len, self.bonus
+
+    def accept_sample(self, temperature: float, u: torch.Tensor, logits: torch.Tensor | None = None,
+                      tree: Tree | None = None, stream=None):
+        """Speculative sampling at temperature T > 0 + compaction (msd_accept_sample).
+        u: fp32 [B, D+1, k+1] uniforms on the device; logits: the tensor given to
+        verify(), or None if verify() kept them in the context."""
+        t = self.tree if tree is None else tree
+        st = lib().msd_accept_sample(self.ctx, ctypes.byref(t.c()), _ptr(logits), float(temperature),
+                                     _ptr(u), _ptr(self.path), _ptr(self.accept_len), _ptr(self.bonus),
+                                     _ptr(self.index_map), _stream(stream))
+        self._check(st, "msd_accept_sample")
+        return self.path, self.accept_len, self.bonus
+
+    def step_sample(self, temperature: float, u: torch.Tensor, stream=None):
+        """draft -> verify -> sample/compact at temperature T as one replayed
+        CUDA graph (msd_step_sample); u is read when the step runs."""
+        st = lib().msd_step_sample(self.ctx, ctypes.byref(self.tree.c()), float(temperature), _ptr(u),
+                                   _ptr(self.argmax), _ptr(self.path), _ptr(self.accept_len),
+                                   _ptr(self.bonus), _stream(stream))
+        self._check(st, "msd_step_sample")
         return self.path, self.accept_len, self.bonus
 
     def step(self, stream=None):
