@@ -54,6 +54,13 @@ Readings where the paper is silent (each also listed in the design notes):
      p itself (a leaf). Draws are inverse-CDF in token-id order. The uniforms
      are inputs: u[d][j] for the j-th child tried at depth d, u[d][k] for the
      token drawn at depth d.
+  R8 draft input of a visual prefix position (Sec. 5.3, ablation of the input
+     strategy; the paper compares three): "embedding" -- MSD, Eq. 7, the raw
+     visual embedding e_{x_i}; "concat" -- the Baseline of Sec. 3.3, the same
+     f_down(Concat(h_{x_i}, e_{x_{i+1}})) as a text position; "feature" -- the
+     target's feature h_{x_i} of that position (R2), with no concatenation.
+     Text positions always take the concatenation. Only prefix positions can
+     be visual: the decode step's positions are generated text.
 """
 from __future__ import annotations
 
@@ -81,6 +88,10 @@ class OracleConfig:
     topk: int
     rms_eps: float = 1e-6
     rope_base: float = 10000.0
+    draft_input: str = "embedding"      # R8: "embedding" (MSD), "concat", "feature"
+
+
+DRAFT_INPUTS = ("embedding", "concat", "feature")
 
 
 class OracleModel:
@@ -279,15 +290,22 @@ def decoupled_draft_inputs(model: OracleModel, ids, emb, h) -> np.ndarray:
 
     Text position i: f_down(Concat(h_{x_i}, e_{x_{i+1}})), where e_{x_{i+1}} is
     whatever embedding the next position carries (text or visual).
-    Visual position i: the raw embedding e_{x_i}.
+    Visual position i, by the model's draft-input strategy (R8): the raw
+    embedding e_{x_i} (MSD, Eq. 7), the same concatenation as a text position
+    (Baseline, Sec. 3.3), or the target feature h_{x_i} (Visual Feature).
     """
+    mode = model.cfg.draft_input
+    if mode not in DRAFT_INPUTS:
+        raise ValueError(f"unknown draft input strategy {mode!r}")
     L = len(ids)
     rows = []
     for i in range(L - 1):
-        if ids[i] >= 0:
+        if ids[i] >= 0 or mode == "concat":
             rows.append(draft_fc(model, h[i:i + 1], emb[i + 1:i + 2])[0])
-        else:
+        elif mode == "embedding":
             rows.append(np.asarray(emb[i], F64))
+        else:
+            rows.append(np.asarray(h[i], F64))
     return np.stack(rows) if rows else np.zeros((0, model.cfg.hidden))
 
 

@@ -283,6 +283,71 @@ def test_decoupled_inputs_follow_eq7(tiny_setup):
     assert [i for i in range(len(f)) if np.any(f3[i] != f[i])] == [3]
 
 
+def _variant(m, mode):
+    import dataclasses
+    return O.OracleModel(dataclasses.replace(m.cfg, draft_input=mode), m.w)
+
+
+@pytest.mark.parametrize("mode,moved_by_pos3,moved_by_pos7", [
+    ("embedding", [3], [6, 7]),      # MSD: a visual row is its own embedding
+    ("concat", [2], [6]),            # Baseline: a row carries the NEXT position's embedding
+    ("feature", [], [6]),            # Visual Feature: a visual row is h, no embedding at all
+])
+def test_draft_input_strategies_dependency_structure(tiny_setup, mode, moved_by_pos3, moved_by_pos7):
+    """The three visual-input strategies of the paper's ablation (Sec. 5.3),
+    told apart by which draft rows a visual embedding reaches (h held fixed):
+    ids 4 8 V V V 12 13 V 20 with visual rows at positions 2, 3, 4 and 7."""
+    wl, w, m, _, _ = tiny_setup
+    mv = _variant(m, mode)
+    H = wl.hidden
+    rng = np.random.default_rng(8)
+    ids = np.array([4, 8, -1, -1, -1, 12, 13, -1, 20])
+    vis = rng.normal(size=(4, H)) * 0.5
+    h = rng.normal(size=(len(ids), H))
+    f = O.decoupled_draft_inputs(mv, ids, O.embed_prompt(mv, ids, vis), h)
+    for row, expect in ((1, moved_by_pos3), (3, moved_by_pos7)):
+        v2 = vis.copy(); v2[row] += 1.0
+        f2 = O.decoupled_draft_inputs(mv, ids, O.embed_prompt(mv, ids, v2), h)
+        assert [i for i in range(len(f)) if np.any(f2[i] != f[i])] == expect, (mode, row)
+
+
+def test_draft_input_strategies_rows(tiny_setup):
+    """Visual Feature rows are the features bit-exactly; Baseline rows are the
+    split-matrix form W[:, :H] h_i + W[:, H:] e_{i+1} at every position; text
+    rows are the same under all three strategies."""
+    wl, w, m, _, _ = tiny_setup
+    H = wl.hidden
+    rng = np.random.default_rng(9)
+    ids = np.array([3, -1, -1, 7, -1, 9])
+    vis = rng.normal(size=(3, H)) * 0.5
+    emb = O.embed_prompt(m, ids, vis)
+    h = rng.normal(size=(len(ids), H))
+    Wfc = np.asarray(m.w["draft_fc"], np.float64)
+    fe = O.decoupled_draft_inputs(_variant(m, "embedding"), ids, emb, h)
+    fc = O.decoupled_draft_inputs(_variant(m, "concat"), ids, emb, h)
+    ff = O.decoupled_draft_inputs(_variant(m, "feature"), ids, emb, h)
+    for i in range(len(ids) - 1):
+        np.testing.assert_allclose(fc[i], Wfc[:, :H] @ h[i] + Wfc[:, H:] @ emb[i + 1], rtol=1e-10, atol=1e-12)
+        if ids[i] < 0:
+            np.testing.assert_array_equal(ff[i], h[i])
+            np.testing.assert_array_equal(fe[i], emb[i])
+        else:
+            np.testing.assert_array_equal(fe[i], fc[i])
+            np.testing.assert_array_equal(ff[i], fc[i])
+    with pytest.raises(ValueError):
+        O.decoupled_draft_inputs(_variant(m, "bogus"), ids, emb, h)
+
+
+def test_draft_input_strategies_agree_without_visual_tokens(tiny_setup):
+    """On a text-only prompt the three strategies build the same draft cache."""
+    wl, w, m, _, _ = tiny_setup
+    ids = np.arange(5, 25)
+    sts = [O.prefill(_variant(m, mode), ids, np.zeros((0, wl.hidden))) for mode in O.DRAFT_INPUTS]
+    for st in sts[1:]:
+        np.testing.assert_array_equal(st.dK, sts[0].dK)
+        np.testing.assert_array_equal(st.dV, sts[0].dV)
+
+
 def test_draft_node_equals_causal_draft_chain(tiny_setup):
     """A depth-d draft row equals the draft layer run causally over the committed
     draft cache and the chain of its ancestors' inputs at consecutive positions."""
