@@ -58,6 +58,11 @@ def parse():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-ar", action="store_true",
                     help="skip the plain greedy decoding baseline (speedup ratio)")
+    ap.add_argument("--draft-input", default="embedding", choices=["embedding", "concat", "feature"],
+                    help="draft input of visual prefix positions: MSD's embedding (default), the "
+                         "Baseline concatenation, or the target feature (the paper's ablation)")
+    ap.add_argument("--no-chain", action="store_true",
+                    help="skip the chain-draft timing (T_q, T_v(gamma), n-alpha and Eq. 9)")
     ap.add_argument("--no-sampling", action="store_true",
                     help="skip the temperature-1 speculative sampling step timing")
     ap.add_argument("--layers", type=int, default=None,
@@ -99,7 +104,8 @@ PAPER_TAU = {"llava7b": 4.45, "long7b": 4.45, "batch16": 4.45, "llava13b": 4.18}
 
 def speedup_ratio(n_out, t_p, t_step, tau, t_prof):
     """Eq. 9: (N T_p + T_profiling) / (N (step time / tokens per step) + T_profiling)."""
-    return (n_out * t_p + t_prof) / (n_out * t_step / tau + t_prof)
+    from paper_2505_14260_gb300 import metrics
+    return metrics.speedup_ratio(n_out, t_p, t_prof, t_step, tau)
 
 
 def peaks():
@@ -192,7 +198,7 @@ class OracleSample:
         cfg = O.OracleConfig(n_layers=layers, hidden=wl.hidden, n_heads=wl.n_heads,
                              head_dim=wl.head_dim, ffn=wl.ffn, vocab=wl.vocab,
                              tree_nodes=wl.tree_nodes, tree_depth=wl.tree_depth, topk=wl.topk,
-                             rms_eps=wl.rms_eps, rope_base=wl.rope_base)
+                             rms_eps=wl.rms_eps, rope_base=wl.rope_base, draft_input=wl.draft_input)
         f = synth.to_numpy_f32
         w = {k: f(v) for k, v in weights.items() if hasattr(v, "dtype") and k != "layers"}
         w["layers"] = [{n: f(t) for n, t in lw.items()} for lw in weights["layers"][:layers]]
@@ -310,7 +316,7 @@ def run_msd(args, rank, world, local_rank):
     from paper_2505_14260_gb300 import msd, synth
 
     torch.cuda.set_device(local_rank)
-    wl = synth.WORKLOADS[args.workload]
+    wl = synth.WORKLOADS[args.workload].with_(draft_input=args.draft_input)
     if args.layers:
         wl = wl.with_(n_layers=args.layers, name=f"{wl.name}-{args.layers}layers")
     B, N, D, V = wl.batch, wl.tree_nodes, wl.tree_depth, wl.vocab
@@ -458,11 +464,13 @@ def run_msd(args, rank, world, local_rank):
             eng.step_sample(T_s, u_buf)
         torch.cuda.synchronize()
         Ls0 = eng.state()["seq_len"].cpu().numpy().astype(np.int64)
+        torch.cuda.nvtx.range_push("timed_sample")
         e0.record(stream)
         for i in range(K_s):
             u_buf.copy_(u_all[3 + i], non_blocking=True)
             eng.step_sample(T_s, u_buf)
         e1.record(stream)
+        torch.cuda.nvtx.range_pop()
         torch.cuda.synchronize()
         ms_s = e0.elapsed_time(e1)
         Ls1 = eng.state()["seq_len"].cpu().numpy().astype(np.int64)
@@ -474,6 +482,52 @@ def run_msd(args, rank, world, local_rank):
                             "(Eq. 6, top-k candidates as point-mass proposals) and compaction, one replayed "
                             "graph per step after 3 warm-up steps; uniforms copied into its buffer before "
                             "each step (inside the timed region)"}
+
+    # ---- chain drafts (top-1 per depth, N = D + 1): the drafting mode of the
+    # paper's n-alpha, and Eq. 9 in its own terms: gamma T_q + T_v(gamma) per
+    # cycle, omega(gamma, alpha) tokens per cycle
+    chain = None
+    if not args.no_chain:
+        from paper_2505_14260_gb300 import metrics
+        wl_c = wl.with_(topk=1, tree_nodes=D + 1)
+        K_c = min(K, 32)
+        ce = msd.Engine(msd.make_config(wl_c, wl.max_prompt + (2 * K_c + 8) * (D + 1) + 16), weights)
+        ce.prefill(ids, lens, vis, offs)
+        for _ in range(3):
+            ce.step()
+        torch.cuda.synchronize()
+        e0.record(stream)
+        for _ in range(K_c):
+            ce.step()
+        e1.record(stream)
+        torch.cuda.synchronize()
+        t_cycle = e0.elapsed_time(e1) / K_c
+        ev = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+        ph = [0.0, 0.0, 0.0]
+        alens = []
+        for _ in range(K_c):                # the same step as separate calls, per phase
+            ev[0].record(stream)
+            ce.draft_tree()
+            ev[1].record(stream)
+            ce.verify()
+            ev[2].record(stream)
+            ce.accept_compact()
+            ev[3].record(stream)
+            torch.cuda.synchronize()
+            for i in range(3):
+                ph[i] += ev[i].elapsed_time(ev[i + 1]) / K_c
+            alens += [int(x) for x in ce.accept_len.cpu().tolist()]
+        ce.close()
+        alpha = metrics.acceptance_rate(alens, D)
+        chain = {"gamma": D, "ms_per_cycle": t_cycle, "t_q_ms": ph[0] / D, "t_v_ms": ph[1],
+                 "accept_compact_ms": ph[2], "n_alpha": metrics.n_alpha(alens, D), "alpha": alpha,
+                 "tau": metrics.tau(alens),
+                 "note": f"N={D + 1}, k=1 context on the same weights; cycle = replayed msd_step over {K_c} "
+                         "steps after 3 warm-up; T_q = msd_draft_tree time / gamma and T_v(gamma) = "
+                         f"msd_verify time from {K_c} steps run as separate calls (CUDA events)"}
+        if speedup is not None and alpha is not None:
+            chain["sr_eq9"] = metrics.speedup_ratio(PAPER_OUTPUT_LEN, speedup["ar_ms_per_token"],
+                                                    speedup["prefill_ms"], t_cycle, metrics.omega(D, alpha))
 
     cpu = None
     if rank == 0 and not args.no_cpu_baseline:
@@ -498,6 +552,7 @@ def run_msd(args, rank, world, local_rank):
                        "vocab": V, "prompt": f"{wl.n_sys} text + {wl.n_vis} visual + rest text, "
                                              f"{int(L0.mean())} tokens at the timed start",
                        "tree": f"N={N} D={D} k={wl.topk}", "parallelism": f"replicas x{world}",
+                       "draft_input": wl.draft_input,
                        "l2": "inputs larger than L2 (weights streamed every step)"},
             "tokens_per_s": world * tokens / (ms / 1e3),
             "tau": tokens / (K * B),
@@ -518,6 +573,7 @@ def run_msd(args, rank, world, local_rank):
             "e2e": e2e,
             "speedup": speedup,
             "sampling": sampling,
+            "chain": chain,
             "gpu_launches": int(launches1 - launches0),
             "clocks": clk,
         }

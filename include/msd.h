@@ -50,6 +50,16 @@ typedef enum {
 
 enum { MSD_F32 = 0, MSD_BF16 = 1 };
 
+/* Draft input of a VISUAL prefix position (the three strategies of the paper's
+ * ablation of the input strategy, Sec. 5.3; text positions always take
+ * f_down(Concat(h_i, e_{i+1}))). Decode-step positions are generated text, so
+ * the strategy only changes the draft cache built by msd_prefill. */
+enum {
+    MSD_DRAFT_EMBEDDING = 0,  /* MSD (Sec. 4.1, Eq. 7): the raw visual embedding e_i */
+    MSD_DRAFT_CONCAT = 1,     /* Baseline (Sec. 3.3): f_down(Concat(h_i, e_{i+1})) as text */
+    MSD_DRAFT_FEATURE = 2     /* Visual Feature: the target's feature h_i, no concatenation */
+};
+
 /* Model and capacity. The target is a pre-norm LLaMA-style decoder (the LLM of
  * LLaVA-1.5, Sec. 3.1); the draft model is one decoder layer of the same shape
  * plus the fc projection f_down of Eq. 4 (Sec. 3.2). */
@@ -62,6 +72,7 @@ typedef struct {
     int32_t tree_nodes;     /* N, including the root; 1 <= N <= 256 */
     int32_t tree_depth;     /* D >= 1: draft passes per step */
     int32_t topk;           /* k >= 1; k + (D-1)k^2 >= N-1 */
+    int32_t draft_input;    /* MSD_DRAFT_*; 0 (zero-initialised) = MSD's Eq. 7 */
 } msd_config;
 
 /* One decoder layer: RMSNorm gains [H]; wq, wk, wv, wo [H,H];
@@ -131,8 +142,9 @@ msd_status msd_destroy(msd_ctx *ctx);
  * vis_dev ([rows][H], model dtype) in order starting at row vis_off_host[b].
  * Runs the target over the prompt (filling its KV cache), writes the root token
  * x_L = argmax of the last position's logits to root_out_dev[b], and builds the
- * draft cache over positions 0..L-2 with f = e at visual positions and
- * f = f_down(Concat(h, e_next)) at text positions (Eq. 7).
+ * draft cache over positions 0..L-2 with f = f_down(Concat(h, e_next)) at text
+ * positions and, at visual positions, f = e (Eq. 7; or the strategy chosen by
+ * msd_config.draft_input).
  * Errors: MSD_ERR_INVALID (batch out of range, empty prompt, prompt not ending
  * in a text token), MSD_ERR_CAPACITY (L + 1 + N > max_seq). Resets all state. */
 msd_status msd_prefill(msd_ctx *ctx, int32_t batch, const int32_t *seq_len_host,
@@ -191,11 +203,13 @@ msd_status msd_accept_compact(msd_ctx *ctx, const msd_tree *tree,
  * same pointer that call was given, or NULL if it was given NULL (the context
  * keeps them then). u_dev: [B][D+1][k+1] fp32 uniforms in [0, 1), device,
  * caller-owned (the random numbers are inputs, so a step is reproducible).
- * temperature: finite, > 0. A node with more than k children in a
+ * temperature: finite, > 0. vocab <= 393216. A node with more than k children in a
  * caller-planted tree has only its first k tried and sets the device status.
  * Decisions are taken on the fp32 logits with fp32 exponentials and
  * error-free (fp32 pair / fp64) sums: they agree with an exact evaluation
  * except where a uniform lies within about 1e-6 (relative) of a boundary.
+ * Launches two kernels (per-row statistics of all N rows, then the walk and
+ * the draw, one CTA per request) and uses context scratch for the statistics.
  * Outputs, compaction and state update as msd_accept_compact (path, accepted
  * length a, bonus = the drawn token, index map). Errors: MSD_ERR_INVALID (null
  * tree or u_dev, bad temperature, no prefill), MSD_ERR_CAPACITY,

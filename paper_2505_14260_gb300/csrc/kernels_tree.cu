@@ -385,13 +385,25 @@ __global__ void accept_kernel(TreeIn t, const int *__restrict__ argmax, int N, i
 // order with u[b][d][k] (the smallest token whose cumulative mass exceeds u
 // times the remaining mass).
 //
-// One CTA per request. Each thread owns a contiguous run of the vocabulary; a
-// node's row is reduced twice (max, then the sum of exp((z - max) / T)), every
-// exponential in fp32 and every sum as an fp32 TwoSum pair (Knuth's error-free
-// addition) combined across threads in fp64, so the decisions carry only the
-// exponentials' rounding (about 1e-6 relative).
+// Two kernels. sample_stats_kernel: per verify row, M = max z and
+// S = sum exp((z - M) / T) (one CTA per row, coalesced). accept_sample_kernel
+// (one CTA per request): one warp walks the tree with those statistics, then
+// the block draws the token. Every exponential is exp2 of (z - M) * log2(e)/T
+// in fp32 (ex2.approx, relative error below 2^-22); every sum is an fp32
+// TwoSum pair (Knuth's error-free addition) per thread, pairs combined
+// error-free across threads, so the decisions carry only the exponentials'
+// rounding (about 1e-6 relative).
 // ---------------------------------------------------------------------------
 constexpr int SAMPLE_THREADS = 1024;
+constexpr int STATS_THREADS = 1024;
+constexpr int STATS_VEC = 8;         // float4 per thread held in registers (rows up to 32768)
+constexpr int DRAW_ROUNDS = 16;      // rounds of 32 tokens a warp loads at once in the draw
+
+__device__ __forceinline__ float exp2_fast(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
 
 // hi + lo += x with the rounding error of the addition kept in lo.
 __device__ __forceinline__ void two_sum_add(float &hi, float &lo, float x) {
@@ -401,111 +413,153 @@ __device__ __forceinline__ void two_sum_add(float &hi, float &lo, float x) {
     hi = s;
 }
 
-__device__ __forceinline__ double block_sum_f64(double v, double *red) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-#pragma unroll
-    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    __syncthreads();
-    if (lane == 0) red[warp] = v;
-    __syncthreads();
-    if (warp == 0) {
-        double w = lane < nw ? red[lane] : 0.0;
-#pragma unroll
-        for (int o = 16; o > 0; o >>= 1) w += __shfl_xor_sync(0xffffffffu, w, o);
-        if (lane == 0) red[32] = w;
-    }
-    __syncthreads();
-    return red[32];
+// (hi, lo) += (h2, l2); the same result on every lane of a butterfly.
+__device__ __forceinline__ void pair_add(float &hi, float &lo, float h2, float l2) {
+    const float s = hi + h2;
+    const float bp = s - hi;
+    const float e = (hi - (s - bp)) + (h2 - bp);
+    lo = (lo + l2) + e;
+    hi = s;
 }
 
-// Exclusive prefix sum over the block in thread order; *total = the sum of all.
-__device__ __forceinline__ double block_exscan_f64(double v, double *red, double *total) {
-    const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, nw = blockDim.x >> 5;
-    double inc = v;
+__device__ __forceinline__ void warp_pair_sum(float &hi, float &lo) {
 #pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const double y = __shfl_up_sync(0xffffffffu, inc, o);
-        if (lane >= o) inc += y;
+    for (int o = 16; o > 0; o >>= 1) {
+        const float h2 = __shfl_xor_sync(0xffffffffu, hi, o), l2 = __shfl_xor_sync(0xffffffffu, lo, o);
+        pair_add(hi, lo, h2, l2);
     }
-    double excl = __shfl_up_sync(0xffffffffu, inc, 1);
-    if (lane == 0) excl = 0.0;
-    __syncthreads();
-    if (lane == 31) red[warp] = inc;
+}
+
+// Per verify row: M = max z, S = sum exp2((z - M) * scale) with scale =
+// log2(e) / T. One CTA per row; a 16-byte-aligned row of at most 32768 logits
+// is loaded once into registers (every load in flight at once), longer or
+// unaligned rows are streamed twice.
+__global__ void __launch_bounds__(STATS_THREADS)
+sample_stats_kernel(const float *__restrict__ logits, int V, float scale, float *__restrict__ row_max,
+                    double *__restrict__ row_sum) {
+    wait_prior();
+    allow_dependents();
+    __shared__ float redf[32], rh[32], rl[32];
+    const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+    const float *z = logits + (size_t)blockIdx.x * V;
+    float hi = 0.f, lo = 0.f, M;
+    if ((V & 3) == 0 && V <= 4 * STATS_VEC * STATS_THREADS &&
+        (reinterpret_cast<uintptr_t>(z) & 15) == 0 && blockDim.x == STATS_THREADS) {
+        const float4 *z4 = reinterpret_cast<const float4 *>(z);
+        const int V4 = V >> 2;
+        float4 v[STATS_VEC];
+#pragma unroll
+        for (int j = 0; j < STATS_VEC; ++j) {
+            const int i = tid + j * STATS_THREADS;
+            v[j] = i < V4 ? z4[i] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+        }
+        float m = -INFINITY;
+#pragma unroll
+        for (int j = 0; j < STATS_VEC; ++j) m = fmaxf(fmaxf(m, fmaxf(v[j].x, v[j].y)), fmaxf(v[j].z, v[j].w));
+        M = block_max(m, redf);
+#pragma unroll
+        for (int j = 0; j < STATS_VEC; ++j) {
+            if (tid + j * STATS_THREADS < V4) {
+                two_sum_add(hi, lo, exp2_fast((v[j].x - M) * scale));
+                two_sum_add(hi, lo, exp2_fast((v[j].y - M) * scale));
+                two_sum_add(hi, lo, exp2_fast((v[j].z - M) * scale));
+                two_sum_add(hi, lo, exp2_fast((v[j].w - M) * scale));
+            }
+        }
+    } else {
+        float m = -INFINITY;
+#pragma unroll 8
+        for (int i = tid; i < V; i += blockDim.x) m = fmaxf(m, z[i]);
+        M = block_max(m, redf);
+#pragma unroll 8
+        for (int i = tid; i < V; i += blockDim.x) two_sum_add(hi, lo, exp2_fast((z[i] - M) * scale));
+    }
+    warp_pair_sum(hi, lo);
+    if (lane == 0) { rh[warp] = hi; rl[warp] = lo; }
     __syncthreads();
     if (warp == 0) {
-        double w = lane < nw ? red[lane] : 0.0;
-#pragma unroll
-        for (int o = 1; o < 32; o <<= 1) {
-            const double y = __shfl_up_sync(0xffffffffu, w, o);
-            if (lane >= o) w += y;
+        hi = lane < nw ? rh[lane] : 0.f;
+        lo = lane < nw ? rl[lane] : 0.f;
+        warp_pair_sum(hi, lo);
+        if (lane == 0) {
+            row_max[blockIdx.x] = M;
+            row_sum[blockIdx.x] = (double)hi + (double)lo;
         }
-        red[lane] = w;            // inclusive prefix of the warp totals
     }
-    __syncthreads();
-    *total = red[nw - 1];
-    return (warp > 0 ? red[warp - 1] : 0.0) + excl;
+}
+
+__device__ __forceinline__ bool is_removed(const unsigned *bits, int i) {
+    return (bits[i >> 5] >> (i & 31)) & 1u;
 }
 
 __global__ void __launch_bounds__(SAMPLE_THREADS)
-accept_sample_kernel(TreeIn t, const float *__restrict__ logits, int N, int D, int k, int V,
-                     float inv_temp, const float *__restrict__ u, int *__restrict__ seq_len,
-                     int *__restrict__ n_pend, int *__restrict__ root, int *__restrict__ pend_next,
-                     int *__restrict__ acc_path, int *__restrict__ acc_L0, int *__restrict__ acc_a,
-                     int *__restrict__ path_out, int *__restrict__ accept_len_out,
-                     int *__restrict__ bonus_out, int *__restrict__ index_map_out, int *status) {
+accept_sample_kernel(TreeIn t, const float *__restrict__ logits, const float *__restrict__ row_max,
+                     const double *__restrict__ row_sum, int N, int D, int k, int V, float scale,
+                     const float *__restrict__ u, int *__restrict__ seq_len, int *__restrict__ n_pend,
+                     int *__restrict__ root, int *__restrict__ pend_next, int *__restrict__ acc_path,
+                     int *__restrict__ acc_L0, int *__restrict__ acc_a, int *__restrict__ path_out,
+                     int *__restrict__ accept_len_out, int *__restrict__ bonus_out,
+                     int *__restrict__ index_map_out, int *status) {
     wait_prior();
     allow_dependents();
-    const int b = blockIdx.x, tid = threadIdx.x, D1 = D + 1;
+    extern __shared__ unsigned removed_bits[];          // [(V + 31) / 32]
+    const int b = blockIdx.x, tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+    const int nw = blockDim.x >> 5, D1 = D + 1, words = (V + 31) >> 5;
     const size_t nb = (size_t)b * N;
     const int n = t.n_nodes ? min(max(t.n_nodes[b], 1), N) : N;
     const float *ub = u + (size_t)b * D1 * (k + 1);
     __shared__ int path[TREE_MAXD + 1];
-    __shared__ int kids[TREE_MAXK], removed[TREE_MAXK];
-    __shared__ int sh_next, sh_nrem, sh_pick, sh_last;
-    __shared__ float redf[32];
-    __shared__ double red[33];
-    __shared__ double bound[SAMPLE_THREADS + 1];
-    const int per = (V + blockDim.x - 1) / blockDim.x;
-    const int lo = min(tid * per, V), hi = min(lo + per, V);
-    if (tid == 0) path[0] = 0;
-    int cur = 0, a = 0;
-    const float *row;
-    float M;
-    for (;;) {
-        row = logits + (nb + cur) * V;
-        float m = -INFINITY;
-        for (int i = lo; i < hi; ++i) m = fmaxf(m, row[i]);
-        M = block_max(m, redf);
-        float sh = 0.f, sl = 0.f;
-        for (int i = lo; i < hi; ++i) two_sum_add(sh, sl, expf((row[i] - M) * inv_temp));
-        const double S = block_sum_f64((double)sh + (double)sl, red);
-        if (tid < 32) {
-            // children of the node, in tree order (at most k are tried)
+    __shared__ int kids[TREE_MAXK], removed[TREE_MAXK], kid_tok[TREE_MAXK];
+    __shared__ double kid_p[TREE_MAXK];
+    __shared__ float kid_u[TREE_MAXK];
+    __shared__ int sh_cur, sh_a, sh_nrem, sh_warp, sh_pick;
+    __shared__ double wsum[32], sh_base, sh_target;
+    __shared__ int wlast[32];
+    for (int i = tid; i < words; i += blockDim.x) removed_bits[i] = 0u;
+
+    // the walk (warp 0): Eq. 6 with point-mass proposals at every node. The
+    // lanes fetch the children's tokens, probabilities and uniforms at once;
+    // lane 0 then takes the decisions in tree order.
+    if (warp == 0) {
+        int cur = 0, a = 0, nrem = 0;
+        if (lane == 0) path[0] = 0;
+        for (;;) {
+            const float M = row_max[nb + cur];
+            const double S = row_sum[nb + cur];
             int cnt = 0;
             for (int c0 = 1; c0 < n; c0 += 32) {
-                const int c = c0 + tid;
+                const int c = c0 + lane;
                 const bool is = c < n && t.parent[nb + c] == cur;
                 const unsigned bal = __ballot_sync(0xffffffffu, is);
-                const int slot = cnt + __popc(bal & ((1u << tid) - 1u));
+                const int slot = cnt + __popc(bal & ((1u << lane) - 1u));
                 if (is && slot < k) kids[slot] = c;
                 cnt += __popc(bal);
             }
             __syncwarp();
-            if (tid == 0) {
+            const int nk = a < D ? min(cnt, k) : 0;
+            if (lane < nk) {
+                const int x = t.tokens[nb + kids[lane]];
+                const bool ok = x >= 0 && x < V;
+                kid_tok[lane] = ok ? x : -1;
+                kid_p[lane] = ok ? (double)exp2_fast((logits[(nb + cur) * V + x] - M) * scale) / S : 0.0;
+                kid_u[lane] = ub[a * (k + 1) + lane];
+            }
+            __syncwarp();
+            int next = -1;
+            nrem = 0;
+            if (lane == 0) {
                 if (cnt > k) set_status(status, ST_BAD_TREE);
-                const int nk = a < D ? min(cnt, k) : 0;
-                int next = -1, nrem = 0;
                 double gone = 0.0;        // mass of the tokens already rejected at this node
                 for (int j = 0; j < nk; ++j) {
-                    const int x = t.tokens[nb + kids[j]];
-                    if (x < 0 || x >= V) {
+                    const int x = kid_tok[j];
+                    if (x < 0) {
                         set_status(status, ST_BAD_TOKEN);
                         continue;
                     }
                     bool dup = false;
                     for (int r = 0; r < nrem; ++r) dup |= removed[r] == x;
-                    const double px = dup ? 0.0 : (double)expf((row[x] - M) * inv_temp) / S;
-                    if ((double)ub[a * (k + 1) + j] * (1.0 - gone) < px) {
+                    const double px = dup ? 0.0 : kid_p[j];
+                    if ((double)kid_u[j] * (1.0 - gone) < px) {
                         next = kids[j];
                         break;
                     }
@@ -514,69 +568,129 @@ accept_sample_kernel(TreeIn t, const float *__restrict__ logits, int N, int D, i
                         gone += px;
                     }
                 }
-                sh_next = next;
-                sh_nrem = nrem;
-                sh_pick = -1;
-                sh_last = -1;
             }
+            next = __shfl_sync(0xffffffffu, next, 0);
+            nrem = __shfl_sync(0xffffffffu, nrem, 0);
+            if (next < 0) break;
+            cur = next;
+            ++a;
+            if (lane == 0) path[a] = cur;
+            __syncwarp();
         }
-        __syncthreads();
-        const int next = sh_next;
-        if (next < 0) break;
-        cur = next;
-        ++a;
-        if (tid == 0) path[a] = cur;
+        if (lane == 0) {
+            sh_cur = cur;
+            sh_a = a;
+            sh_nrem = nrem;
+            sh_warp = -1;
+            sh_pick = -1;
+        }
     }
-    // the next token: inverse CDF of p_adj at the last node, in token-id order
-    const int nrem = sh_nrem;
-    float ph = 0.f, pl = 0.f;
+    __syncthreads();
+    const int cur = sh_cur, a = sh_a, nrem = sh_nrem;
+    if (tid < nrem) atomicOr(&removed_bits[removed[tid] >> 5], 1u << (removed[tid] & 31));
+    __syncthreads();
+
+    // the draw: inverse CDF of p_adj at the last node in token-id order. Warp w
+    // owns tokens [w*seg, (w+1)*seg) in rounds of 32 consecutive tokens (lane l
+    // takes token 32j + l of round j: coalesced), DRAW_ROUNDS rounds loaded at once.
+    const float *z = logits + (nb + cur) * V;
+    const float M = row_max[nb + cur];
+    const int seg = 32 * ((V + 32 * nw - 1) / (32 * nw));
+    const int t0 = warp * seg, t1 = min(t0 + seg, V);
+    float hi = 0.f, lo = 0.f;
     int last = -1;
-    for (int i = lo; i < hi; ++i) {
-        bool rm = false;
-        for (int r = 0; r < nrem; ++r) rm |= removed[r] == i;
-        if (rm) continue;
-        const float e = expf((row[i] - M) * inv_temp);
-        two_sum_add(ph, pl, e);
-        if (e > 0.f) last = i;
+    for (int c0 = t0; c0 < t1; c0 += 32 * DRAW_ROUNDS) {
+        float v[DRAW_ROUNDS];
+#pragma unroll
+        for (int j = 0; j < DRAW_ROUNDS; ++j) {
+            const int i = c0 + 32 * j + lane;
+            v[j] = i < t1 ? z[i] : 0.f;
+        }
+#pragma unroll
+        for (int j = 0; j < DRAW_ROUNDS; ++j) {
+            const int i = c0 + 32 * j + lane;
+            const float e = (i < t1 && !is_removed(removed_bits, i)) ? exp2_fast((v[j] - M) * scale) : 0.f;
+            two_sum_add(hi, lo, e);
+            if (e > 0.f) last = i;
+        }
     }
-    double total;
-    const double excl = block_exscan_f64((double)ph + (double)pl, red, &total);
-    bound[tid] = excl;
-    if (tid == 0) bound[blockDim.x] = total;
-    if (last >= 0) atomicMax(&sh_last, last);
+    warp_pair_sum(hi, lo);
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) last = max(last, __shfl_xor_sync(0xffffffffu, last, o));
+    if (lane == 0) {
+        wsum[warp] = (double)hi + (double)lo;
+        wlast[warp] = last;
+    }
     __syncthreads();
-    const double target = (double)ub[a * (k + 1) + k] * total;
-    if (bound[tid] <= target && target < bound[tid + 1]) {
-        double c = excl;
-        int pick = -1, lastp = -1;
-        for (int i = lo; i < hi; ++i) {
-            bool rm = false;
-            for (int r = 0; r < nrem; ++r) rm |= removed[r] == i;
-            if (rm) continue;
-            const float e = expf((row[i] - M) * inv_temp);
-            if (e > 0.f) lastp = i;
-            c += (double)e;
-            if (c > target) {
-                pick = i;
-                break;
+    if (warp == 0) {
+        // exclusive scan of the warp segments' masses; the segment holding the target
+        const double v = lane < nw ? wsum[lane] : 0.0;
+        double inc = v;
+#pragma unroll
+        for (int o = 1; o < 32; o <<= 1) {
+            const double y = __shfl_up_sync(0xffffffffu, inc, o);
+            if (lane >= o) inc += y;
+        }
+        const double total = __shfl_sync(0xffffffffu, inc, 31);
+        const double target = (double)ub[a * (k + 1) + k] * total;
+        double excl = __shfl_up_sync(0xffffffffu, inc, 1);   // the intervals tile [0, total)
+        if (lane == 0) excl = 0.0;
+        const bool here = lane < nw && v > 0.0 && excl <= target && target < inc;
+        const unsigned bal = __ballot_sync(0xffffffffu, here);
+        if (lane == 0) {
+            sh_target = target;
+            if (bal) {
+                sh_warp = __ffs(bal) - 1;
+            } else {
+                // no segment (u >= 1 or no mass left): the last token with mass
+                int lp = -1;
+                for (int w = 0; w < nw; ++w) lp = max(lp, wlast[w]);
+                sh_pick = lp;
             }
         }
-        sh_pick = pick >= 0 ? pick : lastp;   // the bounds partition [0, total): one thread
+        if (bal && lane == __ffs(bal) - 1) sh_base = excl;
     }
     __syncthreads();
-    if (tid == 0) {
-        int bo = sh_pick >= 0 ? sh_pick : sh_last;
-        if (bo < 0) {
-            // no mass left (only with u >= 1 or every positive token removed): the argmax
-            bo = 0;
-            for (int i = 0; i < V; ++i)
-                if (row[i] == M) { bo = i; break; }
+    if (warp == sh_warp) {
+        // walk the segment round by round: fp32 inclusive scan of each round on
+        // top of the fp64 mass of the rounds before it
+        const double target = sh_target;
+        double cum = sh_base;
+        int pick = -1;
+        for (int c0 = t0; c0 < t1 && pick < 0; c0 += 32 * DRAW_ROUNDS) {
+            float v[DRAW_ROUNDS];
+#pragma unroll
+            for (int j = 0; j < DRAW_ROUNDS; ++j) {
+                const int i = c0 + 32 * j + lane;
+                v[j] = i < t1 ? z[i] : 0.f;
+            }
+#pragma unroll
+            for (int j = 0; j < DRAW_ROUNDS; ++j) {
+                const int i = c0 + 32 * j + lane;
+                const float e = (i < t1 && !is_removed(removed_bits, i)) ? exp2_fast((v[j] - M) * scale) : 0.f;
+                float inc = e;
+#pragma unroll
+                for (int o = 1; o < 32; o <<= 1) {
+                    const float y = __shfl_up_sync(0xffffffffu, inc, o);
+                    if (lane >= o) inc += y;
+                }
+                const unsigned hit = __ballot_sync(0xffffffffu, pick < 0 && e > 0.f && cum + (double)inc > target);
+                if (hit && pick < 0) pick = c0 + 32 * j + __ffs(hit) - 1;
+                cum += (double)__shfl_sync(0xffffffffu, inc, 31);
+            }
         }
-        sh_next = bo;
+        if (lane == 0) sh_pick = pick >= 0 ? pick : wlast[warp];
     }
     __syncthreads();
-    const int bonus = sh_next;
-    write_acceptance(t, path, a, bonus, b, N, D1, seq_len, n_pend, root, pend_next, acc_path, acc_L0,
+    if (tid == 0 && sh_pick < 0) {
+        // nothing drawable at all: the node's argmax
+        int am = 0;
+        for (int i = 0; i < V; ++i)
+            if (z[i] == M) { am = i; break; }
+        sh_pick = am;
+    }
+    __syncthreads();
+    write_acceptance(t, path, a, sh_pick, b, N, D1, seq_len, n_pend, root, pend_next, acc_path, acc_L0,
                      acc_a, path_out, accept_len_out, bonus_out, index_map_out);
 }
 
@@ -736,13 +850,18 @@ void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int 
 }
 
 void launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, int D, int k, int V,
-                          float inv_temp, const float *u, int *seq_len, int *n_pend, int *root,
-                          int *pend_next, int *acc_path, int *acc_L0, int *acc_a, int *path_out,
-                          int *accept_len_out, int *bonus_out, int *index_map_out, int *status,
-                          cudaStream_t s) {
-    launch_pdl(accept_sample_kernel, B, SAMPLE_THREADS, 0, s, t, logits, N, D, k, V, inv_temp, u, seq_len,
-               n_pend, root, pend_next, acc_path, acc_L0, acc_a, path_out, accept_len_out, bonus_out,
-               index_map_out, status); note_launch();
+                          float inv_temp, const float *u, float *row_max, double *row_sum, int *seq_len,
+                          int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
+                          int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,
+                          int *status, cudaStream_t s) {
+    const float scale = (float)(1.4426950408889634 * (double)inv_temp);     // log2(e) / T
+    launch_pdl(sample_stats_kernel, B * N, STATS_THREADS, 0, s, logits, V, scale, row_max, row_sum);
+    note_launch();
+    const size_t smem = sizeof(unsigned) * (size_t)((V + 31) / 32);
+    launch_pdl(accept_sample_kernel, B, SAMPLE_THREADS, smem, s, t, logits, (const float *)row_max,
+               (const double *)row_sum, N, D, k, V, scale, u, seq_len, n_pend, root, pend_next, acc_path,
+               acc_L0, acc_a, path_out, accept_len_out, bonus_out, index_map_out, status);
+    note_launch();
 }
 
 void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, const int *acc_L0,

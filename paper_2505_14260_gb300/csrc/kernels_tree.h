@@ -71,13 +71,14 @@ void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int 
                    cudaStream_t s);
 // Speculative sampling over the tree at temperature T > 0 (Eq. 6 with the
 // draft's top-k candidates as point-mass proposals): logits [B][N][V] fp32 of
-// the verify pass, inv_temp = 1/T, u [B][D+1][k+1] uniforms in [0, 1). Same
-// outputs and state update as launch_accept.
+// the verify pass, inv_temp = 1/T, u [B][D+1][k+1] uniforms in [0, 1);
+// row_max [B*N] and row_sum [B*N] are scratch for the per-row statistics.
+// Same outputs and state update as launch_accept. Two launches.
 void launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, int D, int k, int V,
-                          float inv_temp, const float *u, int *seq_len, int *n_pend, int *root,
-                          int *pend_next, int *acc_path, int *acc_L0, int *acc_a, int *path_out,
-                          int *accept_len_out, int *bonus_out, int *index_map_out, int *status,
-                          cudaStream_t s);
+                          float inv_temp, const float *u, float *row_max, double *row_sum, int *seq_len,
+                          int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
+                          int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,
+                          int *status, cudaStream_t s);
 void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, const int *acc_L0,
                        const int *acc_a, int n_layers, int B, int nh, int N, int S, int D1,
                        int row_bytes, int *status, cudaStream_t s);

@@ -53,6 +53,8 @@ struct msd_ctx {
     TopkScratch tks{nullptr, nullptr};
     void *hT = nullptr;
     int *acc_path = nullptr, *acc_L0 = nullptr, *acc_a = nullptr;
+    float *samp_max = nullptr;      // sampling (T > 0): per verify row max logit and
+    double *samp_sum = nullptr;     // sum of exp((z - max) / T)
     // plain greedy decoding (msd_ar_step): a root-only tree and its argmax
     msd_tree ar_tree{};
     int *ar_argmax = nullptr;
@@ -419,7 +421,9 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
         const T *h_last = static_cast<const T *>(c->h_all) + (size_t)(L - 1) * H;
         gemm<T>(c, h_last, H, 1, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V, EPI_STORE, s);
         launch_argmax(c->logits, 1, V, c->argmax_tmp, c->tks, s);
-        // draft cache over positions 0 .. L-2 with the decoupled input (Eq. 7)
+        // draft cache over positions 0 .. L-2 with the decoupled input (Eq. 7): text
+        // rows f_down(Concat(h, e_next)); visual rows e (MSD), the same
+        // concatenation (Baseline) or h (Visual Feature), Sec. 5.3
         for (int r0 = 0; r0 < L - 1; r0 += c->chunk) {
             const int n = std::min(c->chunk, L - 1 - r0);
             rd.resize(n);
@@ -430,8 +434,11 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
                                   static_cast<T *>(c->xfc), s);
             gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, n, 2 * H, one(c->w.draft_fc, H, c->pk_fc), H,
                     c->x, H, EPI_STORE, s);
-            launch_select_visual<T>(c->x, static_cast<const T *>(c->emb_all) + (size_t)r0 * H,
-                                    c->src + r0, n, H, s);
+            if (c->cfg.draft_input != MSD_DRAFT_CONCAT) {
+                const void *vis_rows = c->cfg.draft_input == MSD_DRAFT_FEATURE ? c->h_all : c->emb_all;
+                launch_select_visual<T>(c->x, static_cast<const T *>(vis_rows) + (size_t)r0 * H,
+                                        c->src + r0, n, H, s);
+            }
             T *K = tkv<T>(c, c->draft_kv, 0, 0, c->S), *Vv = tkv<T>(c, c->draft_kv, 0, 1, c->S);
             run_layer<T>(c, c->w.draft, c->dpack, n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr, nullptr, 0,
                          nullptr, 0, n, r0 + n, s);
@@ -590,8 +597,8 @@ msd_status accept_sample_impl(msd_ctx *c, const msd_tree *tree, const float *log
                               int32_t *imap, cudaStream_t s) {
     TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
     launch_accept_sample(t, logits, c->B, c->N, c->D, c->k, c->V, (float)(1.0 / (double)temp), u,
-                         c->seq_len, c->n_pend, c->root, c->pend_next, c->acc_path, c->acc_L0, c->acc_a,
-                         path, alen, bonus, imap, c->status, s);
+                         c->samp_max, c->samp_sum, c->seq_len, c->n_pend, c->root, c->pend_next, c->acc_path,
+                         c->acc_L0, c->acc_a, path, alen, bonus, imap, c->status, s);
     return compact_impl<T>(c, s, -1);
 }
 
@@ -676,6 +683,9 @@ msd_status validate_config(const msd_config *g) {
     if (g->tree_depth < 1 || g->tree_depth > TREE_MAXD) return MSD_ERR_INVALID;
     if (g->topk < 1 || g->topk > TREE_MAXK || g->topk > g->vocab) return MSD_ERR_INVALID;
     if (!topk_supported(g->vocab, g->topk)) return MSD_ERR_INVALID;
+    if (g->draft_input != MSD_DRAFT_EMBEDDING && g->draft_input != MSD_DRAFT_CONCAT &&
+        g->draft_input != MSD_DRAFT_FEATURE)
+        return MSD_ERR_INVALID;
     const long cand = g->topk + (long)(g->tree_depth - 1) * g->topk * g->topk;
     if (cand < g->tree_nodes - 1) return MSD_ERR_INVALID;
     return MSD_OK;
@@ -802,6 +812,8 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     ok &= dalloc(c, &c->acc_path, sizeof(int) * c->B * c->D1);
     ok &= dalloc(c, &c->acc_L0, sizeof(int) * c->B);
     ok &= dalloc(c, &c->acc_a, sizeof(int) * c->B);
+    ok &= dalloc(c, &c->samp_max, sizeof(float) * c->B * c->N);
+    ok &= dalloc(c, &c->samp_sum, sizeof(double) * c->B * c->N);
     ok &= dalloc(c, &c->ar_tree.tokens, sizeof(int) * c->B * c->N);
     ok &= dalloc(c, &c->ar_tree.parent, sizeof(int) * c->B * c->N);
     ok &= dalloc(c, &c->ar_tree.depth, sizeof(int) * c->B * c->N);
@@ -1098,6 +1110,10 @@ msd_status msd_ar_step(msd_ctx *c, int32_t *token_dev, void *stream) {
 
 // The kernel scales logits by the fp32 1/T: T must be finite, > 0, and have a
 // finite fp32 reciprocal.
+// The sampling kernel keeps a bitmap of the rejected tokens in shared memory
+// (one bit per token, within the default 48 KB of dynamic shared memory).
+constexpr int MSD_SAMPLE_MAX_VOCAB = 48 * 1024 * 8;
+
 static bool temperature_ok(float t) {
     return std::isfinite(t) && t > 0.f && std::isfinite((float)(1.0 / (double)t));
 }
@@ -1113,6 +1129,7 @@ msd_status msd_accept_sample(msd_ctx *c, const msd_tree *tree, const float *logi
     if (st != MSD_OK) return st;
     if (!tree_ok(tree) || !u_dev) return fail(c, MSD_ERR_INVALID, "null tree or uniforms");
     if (!temperature_ok(temperature)) return fail(c, MSD_ERR_INVALID, "temperature must be finite and > 0");
+    if (c->V > MSD_SAMPLE_MAX_VOCAB) return fail(c, MSD_ERR_INVALID, "vocabulary too large for sampling");
     if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
     st = check_capacity(c);
     if (st != MSD_OK) return st;
@@ -1137,6 +1154,7 @@ msd_status msd_step_sample(msd_ctx *c, const msd_tree *tree, float temperature, 
     if (!tree_ok(tree) || !argmax_dev || !u_dev)
         return fail(c, MSD_ERR_INVALID, "null tree, argmax or uniforms");
     if (!temperature_ok(temperature)) return fail(c, MSD_ERR_INVALID, "temperature must be finite and > 0");
+    if (c->V > MSD_SAMPLE_MAX_VOCAB) return fail(c, MSD_ERR_INVALID, "vocabulary too large for sampling");
     if (!c->prefilled) return fail(c, MSD_ERR_INVALID, "msd_prefill has not run");
     if (c->draft_stale)
         return fail(c, MSD_ERR_INVALID, "msd_ar_step ran since the last msd_prefill: the draft cache is stale");

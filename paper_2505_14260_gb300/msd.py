@@ -17,6 +17,7 @@ _LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libmsd.so"
 
 MSD_OK, MSD_ERR_INVALID, MSD_ERR_CAPACITY, MSD_ERR_OOM, MSD_ERR_CUDA, MSD_ERR_DEVICE = 0, -1, -2, -3, -4, -5
 MSD_F32, MSD_BF16 = 0, 1
+DRAFT_INPUTS = {"embedding": 0, "concat": 1, "feature": 2}     # MSD_DRAFT_*
 STATUS_NAMES = {0: "MSD_OK", -1: "MSD_ERR_INVALID", -2: "MSD_ERR_CAPACITY", -3: "MSD_ERR_OOM",
                 -4: "MSD_ERR_CUDA", -5: "MSD_ERR_DEVICE"}
 
@@ -26,7 +27,7 @@ class msd_config(ctypes.Structure):
                 ("head_dim", c_int32), ("ffn", c_int32), ("vocab", c_int32),
                 ("rms_eps", c_float), ("rope_base", c_float), ("dtype", c_int32),
                 ("max_batch", c_int32), ("max_seq", c_int32), ("tree_nodes", c_int32),
-                ("tree_depth", c_int32), ("topk", c_int32)]
+                ("tree_depth", c_int32), ("topk", c_int32), ("draft_input", c_int32)]
 
 
 LAYER_FIELDS = ("attn_norm", "wq", "wk", "wv", "wo", "mlp_norm", "w_gate", "w_up", "w_down")
@@ -316,7 +317,8 @@ def make_config(wl, max_seq: int, batch: int | None = None) -> msd_config:
                       rope_base=wl.rope_base,
                       dtype=MSD_BF16 if wl.dtype == "bf16" else MSD_F32,
                       max_batch=wl.batch if batch is None else batch, max_seq=max_seq,
-                      tree_nodes=wl.tree_nodes, tree_depth=wl.tree_depth, topk=wl.topk)
+                      tree_nodes=wl.tree_nodes, tree_depth=wl.tree_depth, topk=wl.topk,
+                      draft_input=DRAFT_INPUTS[wl.draft_input])
 
 
 def upload_prompts(prompts, device="cuda"):

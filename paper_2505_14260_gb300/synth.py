@@ -56,6 +56,7 @@ class Workload:
     dtype: str               # "f32" or "bf16"
     rms_eps: float = 1e-6
     rope_base: float = 10000.0
+    draft_input: str = "embedding"   # visual draft input: "embedding" (MSD), "concat", "feature"
 
     def with_(self, **kw) -> "Workload":
         return dataclasses.replace(self, **kw)

@@ -9,7 +9,8 @@ def oracle_config(wl: synth.Workload) -> OracleConfig:
     return OracleConfig(n_layers=wl.n_layers, hidden=wl.hidden, n_heads=wl.n_heads,
                         head_dim=wl.head_dim, ffn=wl.ffn, vocab=wl.vocab,
                         tree_nodes=wl.tree_nodes, tree_depth=wl.tree_depth,
-                        topk=wl.topk, rms_eps=wl.rms_eps, rope_base=wl.rope_base)
+                        topk=wl.topk, rms_eps=wl.rms_eps, rope_base=wl.rope_base,
+                        draft_input=wl.draft_input)
 
 
 def oracle_model(wl: synth.Workload, weights_torch: dict) -> OracleModel:

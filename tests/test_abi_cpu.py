@@ -42,7 +42,8 @@ def test_create_rejects_bad_configs_before_touching_the_gpu(libmsd):
     w = msd.msd_weights()
     cases = [dict(head_dim=96), dict(n_heads=3), dict(topk=0), dict(topk=17),
              dict(tree_nodes=300), dict(tree_depth=0), dict(max_batch=0), dict(dtype=7),
-             dict(tree_nodes=64, tree_depth=2, topk=2)]     # k + (D-1)k^2 = 6 < 63
+             dict(tree_nodes=64, tree_depth=2, topk=2),     # k + (D-1)k^2 = 6 < 63
+             dict(draft_input=3), dict(draft_input=-1)]
     for kw in cases:
         cfg = msd.make_config(wl, 256)
         for k, v in kw.items():

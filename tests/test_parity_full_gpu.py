@@ -34,6 +34,14 @@ def test_full_width_two_layers_match_oracle(name, requests):
     run_parity(wl, 2, requests, TOL_FULL, KV_REL_L2_FULL)
 
 
+def test_llava7b_chain_drafts_two_layers_match_oracle():
+    """Chain drafts at the 7B width (top-1 at every depth, N = D + 1 = 7), the
+    drafting mode of the paper's n-alpha measurement and of the bench's chain
+    timing, cut to 2 layers."""
+    wl = synth.WORKLOADS["llava7b"].with_(n_layers=2, topk=1, tree_nodes=7)
+    run_parity(wl, 2, None, TOL_FULL, KV_REL_L2_FULL)
+
+
 def test_llava7b_full_depth_lossless_chain():
     wl = synth.WORKLOADS["llava7b"]
     D, N, V = wl.tree_depth, wl.tree_nodes, wl.vocab

@@ -33,6 +33,24 @@ def test_tiny_all_steps_match_oracle(dtype, long_prompt):
     run_parity(wl, wl.steps)
 
 
+@pytest.mark.parametrize("dtype,mode", [("f32", "concat"), ("f32", "feature"), ("bf16", "concat"),
+                                        ("bf16", "feature")])
+def test_draft_input_strategies_match_oracle(dtype, mode):
+    """The paper's other visual draft-input strategies (Baseline concatenation,
+    Visual Feature; Sec. 5.3) through msd_prefill's draft cache and two steps,
+    against the oracle with the same strategy."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype=dtype, draft_input=mode, steps=2)
+    run_parity(wl, wl.steps)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_chain_drafts_match_oracle(dtype):
+    """Chain drafts (top-1 at every depth, N = D + 1), the drafting mode of the
+    paper's n-alpha measurement (Sec. 5.1), against the oracle."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype=dtype, topk=1, tree_nodes=5, steps=3)
+    run_parity(wl, wl.steps)
+
+
 def _gpu_greedy_ar(eng, n_tokens):
     """Plain greedy decoding on the GPU path: single-node trees, one per token."""
     out = [int(eng.state()["root"].cpu()[0])]
