@@ -379,7 +379,15 @@ struct PkParams {
     float *ws;
     int *counters;
     int *status;
+    bf16 *act;              // EPI_SWIGLU (glu-packed gate/up): act [M][F] bf16
+    int F;
+    uint32_t stg_off;       // EPI_SWIGLU: byte offset of the 16 KB staging tile
 };
+
+// silu(g) * u, the SwiGLU product of the fused epilogues.
+__device__ __forceinline__ float swiglu_fused(float g, float u) {
+    return __fdividef(g, 1.f + __expf(-g)) * u;
+}
 
 // CTA owning unit u under the balanced partition u0(c) = floor(c * U / G).
 __device__ __forceinline__ int owner_cta(long long u, long long U, int G) {
@@ -579,6 +587,8 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             const int slot = 2 * cta + (item == 0 ? 0 : 1);
             float *part = p.ws + (size_t)slot * BN * BM;
             const bool add = p.epi == EPI_ADD;
+            const bool glu = p.epi == EPI_SWIGLU;
+            float *stg = reinterpret_cast<float *>(smem_raw + p.stg_off);   // [32 columns][128 rows]
             for (int g0 = 0; g0 < BN; g0 += 32) {
                 // up to 32 accumulator columns with one TMEM round trip
                 const int gw = min(32, BN - g0);
@@ -587,7 +597,26 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 for (int c = 0; c < 2; ++c)
                     if (c * 16 < gw) tmem_ld16_nowait(taddr + g0 + c * 16, r + c * 16);
                 tmem_wait_ld();
-                if (!whole) {
+                if (whole && glu) {
+                    // gate row i and up row 64 + i of the tile sit in different
+                    // warps: exchange through shared memory, then thread (i, h)
+                    // writes act[m][64 t + i] for the columns of half h
+                    asm volatile("bar.sync 1, 128;" ::: "memory");
+#pragma unroll
+                    for (int j = 0; j < 32; ++j) stg[j * BM + row] = __uint_as_float(r[j]);
+                    asm volatile("bar.sync 1, 128;" ::: "memory");
+                    const int i = et & 63, h = et >> 6;
+                    const int jo = (row0 >> 1) + i;
+                    if (ok && jo < p.F) {
+#pragma unroll 4
+                        for (int c = 16 * h; c < 16 * h + 16; ++c) {
+                            const int m = n0 + g0 + c;
+                            if (c < gw && m < p.M)
+                                p.act[(size_t)m * p.F + jo] =
+                                    __float2bfloat16_rn(swiglu_fused(stg[c * BM + i], stg[c * BM + 64 + i]));
+                        }
+                    }
+                } else if (!whole) {
 #pragma unroll
                     for (int j = 0; j < 32; ++j)
                         if (j < gw) part[(size_t)(g0 + j) * BM + row] = __uint_as_float(r[j]);
@@ -666,6 +695,29 @@ __global__ void __launch_bounds__(P_THREADS, 1)
 #pragma unroll
                 for (int g = 0; g < 4; ++g) {
                     const int e4 = base4 + g * 128;
+                    if (p.epi == EPI_SWIGLU) {
+                        // lane l < 16 holds gate rows 4l..4l+3 of a column, lane
+                        // l + 16 the matching up rows (e4 % 32 is the lane; the
+                        // branch conditions below are uniform over the warp)
+                        float4 up;
+                        up.x = __shfl_xor_sync(0xffffffffu, acc[g].x, 16);
+                        up.y = __shfl_xor_sync(0xffffffffu, acc[g].y, 16);
+                        up.z = __shfl_xor_sync(0xffffffffu, acc[g].z, 16);
+                        up.w = __shfl_xor_sync(0xffffffffu, acc[g].w, 16);
+                        if (e4 >= n4) continue;
+                        const int col = (e4 * 4) / BM, r4 = (e4 * 4) - col * BM;
+                        const int m = n0 + col;
+                        const int jo = (row0 >> 1) + r4;
+                        if (m >= p.M || !ok || r4 >= 64 || jo >= p.F) continue;
+                        bf16 *dst = p.act + (size_t)m * p.F + jo;
+                        __nv_bfloat162 lo2 = __floats2bfloat162_rn(swiglu_fused(acc[g].x, up.x),
+                                                                   swiglu_fused(acc[g].y, up.y));
+                        __nv_bfloat162 hi2 = __floats2bfloat162_rn(swiglu_fused(acc[g].z, up.z),
+                                                                   swiglu_fused(acc[g].w, up.w));
+                        reinterpret_cast<__nv_bfloat162 *>(dst)[0] = lo2;   // F % 4 == 0: 8-byte aligned
+                        reinterpret_cast<__nv_bfloat162 *>(dst)[1] = hi2;
+                        continue;
+                    }
                     if (e4 >= n4) continue;
                     const int col = (e4 * 4) / BM, r4 = (e4 * 4) - col * BM;
                     const int m = n0 + col;
@@ -1593,10 +1645,23 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
     }
 }
 
+// The persistent stream-K GEMM (many token rows). fx: EPI_SWIGLU writes
+// act = silu(g) * u from glu-packed gate/up weights instead of Y.
+static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
+                         float *Y, int ldy, int epi, const GemmFused *fx, int *status, cudaStream_t s);
+
 bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
                      const GemmFused &fx, int *status, cudaStream_t s, const GemmNorm *norm_in) {
-    if (M <= 0 || M > 128 || !W.packed || W.nseg < 1) return false;
+    if (M <= 0 || !W.packed || W.nseg < 1) return false;
     if (fx.epi == EPI_SWIGLU && (W.nseg != 1 || W.rows[0] != glu_rows(fx.F) || fx.F % 4)) return false;
+    if (M > 128) {
+        // many token rows: the persistent GEMM with SwiGLU fused into its
+        // epilogue (RoPE/KV stays a separate kernel there: fused, its
+        // per-column gathers outlasted the main loop, measured slower)
+        if (fx.epi != EPI_SWIGLU || norm_in || !fx.act) return false;
+        gemm_persist(p, X, ldx, M, K, W, O, nullptr, 0, EPI_SWIGLU, &fx, status, s);
+        return true;
+    }
     if (fx.epi == EPI_ROPE_KV &&
         (W.nseg != 3 || (fx.hd != 64 && fx.hd != 128) || fx.nh * fx.hd != W.rows[0] ||
          W.rows[1] != W.rows[0] || W.rows[2] != W.rows[0]))
@@ -1618,6 +1683,20 @@ bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     if (norm_out && (M > 128 || !W.packed || W.nseg != 1 || !norm_out->ss || !norm_out->xg || !norm_out->g ||
                      (O + BM - 1) / BM > norm_out->ld || O % 4 || ldy % 4))
         return false;
+    if (M <= 128 && W.packed) {
+        int tiles = 0;
+        for (int i = 0; i < W.nseg; ++i) tiles += (W.rows[i] + BM - 1) / BM;
+        gemm_cluster(p, X, ldx, M, K, W, tiles, ((M + 15) / 16) * 16, (K + BK - 1) / BK, Y, ldy, epi, status,
+                     s, O, nullptr, norm_out);
+        return true;
+    }
+    gemm_persist(p, X, ldx, M, K, W, O, Y, ldy, epi, nullptr, status, s);
+    return true;
+}
+
+static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
+                         float *Y, int ldy, int epi, const GemmFused *fx, int *status, cudaStream_t s) {
+    const bool glu = fx && fx->epi == EPI_SWIGLU;
     PkParams pk;
     memset(&pk, 0, sizeof pk);
     pk.n_seg = W.nseg;
@@ -1633,15 +1712,13 @@ bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     int BN = (M + nt - 1) / nt;
     BN = ((BN + 15) / 16) * 16;
     const int kblocks = (K + BK - 1) / BK;
-    if (M <= 128 && W.packed) {
-        gemm_cluster(p, X, ldx, M, K, W, tiles, BN, kblocks, Y, ldy, epi, status, s, O, nullptr, norm_out);
-        return true;
-    }
     const uint32_t stage_bytes = A_BYTES + (uint32_t)BN * BK * 2;
-    // five stages measured best on the decode shapes (deeper rings were slower)
-    int stages = (int)((200u * 1024u) / stage_bytes);
+    // five stages measured best on the decode shapes (deeper rings were slower);
+    // the fused SwiGLU epilogue takes 16 KB of staging from the ring's budget
+    const uint32_t stg_bytes = glu ? 32u * BM * 4u : 0u;
+    int stages = (int)((200u * 1024u - stg_bytes) / stage_bytes);
     stages = stages < 2 ? 2 : (stages > 5 ? 5 : stages);
-    const size_t smem = 1024 + (size_t)stages * stage_bytes;
+    const size_t smem = 1024 + (size_t)stages * stage_bytes + stg_bytes;
     const long long tiles_total = (long long)tiles * nt;
     const long long all_units = tiles_total * kblocks;
     // one CTA per SM, at least 4 K-blocks each
@@ -1656,7 +1733,7 @@ bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     if (ws_need > WS_BYTES || tiles_total > N_COUNTERS) {
         flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
         fprintf(stderr, "msd: GEMM shape M=%d K=%d O=%d exceeds the workspace\n", M, K, O);
-        return true;
+        return;
     }
     int acc = 32;
     while (acc < BN) acc <<= 1;
@@ -1678,13 +1755,19 @@ bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     pk.counters = p->counters;
     pk.status = status;
     pk.wpacked = static_cast<const bf16 *>(W.packed);
+    if (glu) {
+        pk.epi = EPI_SWIGLU;
+        pk.act = fx->act;
+        pk.F = fx->F;
+        pk.stg_off = (uint32_t)(1024 + (size_t)stages * stage_bytes);
+    }
     if (!W.packed) {
         flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
         fprintf(stderr, "msd: GEMM weights were not packed\n");
-        return true;
+        return;
     }
     const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
-    if (!mx) return true;
+    if (!mx) return;
     if (!p->smem_set) {
         cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              200 * 1024 + 1024);
@@ -1722,9 +1805,9 @@ bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
         p->ev_used += 2;
         const double wb = (double)O * K * 2.0;
         p->prof_wbytes += wb;
-        p->prof_bytes += wb + (double)M * K * 2.0 + (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
+        p->prof_bytes += wb + (double)M * K * 2.0 +
+                         (glu ? (double)M * fx->F * 2.0 : (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1));
     }
-    return true;
 }
 
 }  // namespace msd
