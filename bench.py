@@ -235,6 +235,27 @@ class OracleSample:
                 f"target-layer time scaled x{wl.n_layers / self.layers:g}")
 
 
+# ----------------------------------------------------------------------------
+# Replicas (--gpus N under torchrun): the step does not shard, so each rank runs
+# its own copy of the workload; the only collectives are the barriers around
+# the timed region and the maximum of the ranks' times.
+# ----------------------------------------------------------------------------
+def max_over_ranks(ms: float, world: int, device) -> float:
+    """The slowest rank's time (ms); every rank gets the same value."""
+    import torch
+    import torch.distributed as dist
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def aggregate_rate(units_per_rank: float, world: int, ms_max: float) -> float:
+    """Whole-job throughput: the units all ranks processed over the slowest
+    rank's time (weak scaling: each rank processes the same units)."""
+    return world * units_per_rank / (ms_max / 1e3)
+
+
 def make_inputs(wl, device):
     import torch
     from paper_2505_14260_gb300 import synth
@@ -362,12 +383,10 @@ def run_msd(args, rank, world, local_rank):
     torch.cuda.synchronize()
     prof = eng.profile_read()
     eng.profile_enable(False)
-    t = torch.tensor([ms], dtype=torch.float64, device="cuda")
     if world > 1:
         dist.barrier()
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    ms_max = float(t.item())
-    steps_s = world * K / (ms_max / 1e3)
+    ms_max = max_over_ranks(ms, world, "cuda")
+    steps_s = aggregate_rate(K, world, ms_max)
 
     hbm, peak_kind = peaks()
     gemm_gbs = prof["gemm_bytes"] / (prof["gemm_ms"] / 1e3) / 1e9 if prof["gemm_ms"] > 0 else None
@@ -400,12 +419,10 @@ def run_msd(args, rank, world, local_rank):
         e1.record(stream)
         torch.cuda.synchronize()
         ms_e2e = e0.elapsed_time(e1)
-        t2 = torch.tensor([ms_e2e], dtype=torch.float64, device="cuda")
-        if world > 1:
-            dist.all_reduce(t2, op=dist.ReduceOp.MAX)
+        ms_e2e = max_over_ranks(ms_e2e, world, "cuda")
         h2d = ids_h.numel() * 4 + (vis_h.numel() * vis_h.element_size() if vis_h is not None else 0)
         d2h = (out_tok.numel() + out_path.numel() + out_a.numel() + out_b.numel()) * 4
-        e2e = {"value": world * K / (float(t2.item()) / 1e3), "unit": "steps/s",
+        e2e = {"value": aggregate_rate(K, world, ms_e2e), "unit": "steps/s",
                "h2d_bytes_per_step": h2d / K, "d2h_bytes_per_step": d2h,
                "note": "prompt H2D + prefill amortised over the steps; tokens read back every step"}
 
