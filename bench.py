@@ -466,6 +466,44 @@ def run_msd(args, rank, world, local_rank):
                 "note": "projection: the paper's average acceptance length of trained MSD drafts, "
                         "not measured here"}
 
+    # ---- per-step distribution and per-phase times, after the timed region on
+    # a fresh prefill (the timed number above is untouched): K_prof replayed
+    # steps each bracketed by events, then K_prof steps as separate calls
+    eng.prefill(ids, lens, vis, offs)
+    for _ in range(3):
+        eng.step()
+    torch.cuda.synchronize()
+    pairs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+             for _ in range(K_prof)]
+    for a, b in pairs:
+        a.record(stream)
+        eng.step()
+        b.record(stream)
+    torch.cuda.synchronize()
+    per_step = sorted(a.elapsed_time(b) for a, b in pairs)
+
+    def pct(q):
+        return per_step[min(len(per_step) - 1, int(q * (len(per_step) - 1) + 0.5))]
+
+    evp = [torch.cuda.Event(enable_timing=True) for _ in range(4)]
+    phase = [0.0, 0.0, 0.0]
+    for _ in range(K_prof):
+        evp[0].record(stream)
+        eng.draft_tree()
+        evp[1].record(stream)
+        eng.verify()
+        evp[2].record(stream)
+        eng.accept_compact()
+        evp[3].record(stream)
+        torch.cuda.synchronize()
+        for i in range(3):
+            phase[i] += evp[i].elapsed_time(evp[i + 1]) / K_prof
+    distribution = {"p10_ms": pct(0.1), "p50_ms": pct(0.5), "p90_ms": pct(0.9), "steps": K_prof,
+                    "phases_ms": {"draft_tree": phase[0], "verify": phase[1], "accept_compact": phase[2]},
+                    "note": "after a fresh prefill: per-step CUDA events around replayed msd_step "
+                            f"({K_prof} steps after 3 warm-up); phases from {K_prof} steps run as separate "
+                            "calls (msd_draft_tree, msd_verify, msd_accept_compact)"}
+
     # ---- speculative sampling at T = 1 (Eq. 6 over the tree): msd_step_sample,
     # a replayed graph of draft, verify and the sampling walk + compaction; the
     # uniforms are inputs, copied device to device into the step's buffer
@@ -589,6 +627,7 @@ def run_msd(args, rank, world, local_rank):
             "cpu_baseline": cpu,
             "e2e": e2e,
             "speedup": speedup,
+            "distribution": distribution,
             "sampling": sampling,
             "chain": chain,
             "gpu_launches": int(launches1 - launches0),
