@@ -504,6 +504,29 @@ def run_msd(args, rank, world, local_rank):
                             f"({K_prof} steps after 3 warm-up); phases from {K_prof} steps run as separate "
                             "calls (msd_draft_tree, msd_verify, msd_accept_compact)"}
 
+    # ---- compaction worst case: a planted chain of the target's own argmax
+    # tokens (grown by verifying it one node at a time), accepted in full (a = D)
+    worst = None
+    if B == 1:
+        chain_tree = msd.Tree(B, N)
+        toks, par = [int(eng.state()["root"].cpu()[0])], [-1]
+        eng.draft_tree()                  # keeps the draft cache caught up
+        for d in range(D):
+            chain_tree.plant(0, toks, par)
+            eng.verify(tree=chain_tree)
+            toks.append(int(eng.argmax[d].cpu()))
+            par.append(d)
+        chain_tree.plant(0, toks, par)
+        eng.verify(tree=chain_tree)
+        torch.cuda.synchronize()
+        e0.record(stream)
+        eng.accept_compact(tree=chain_tree)
+        e1.record(stream)
+        torch.cuda.synchronize()
+        worst = {"accept_len": int(eng.accept_len.cpu()[0]), "accept_compact_ms": e0.elapsed_time(e1),
+                 "note": "msd_accept_compact on a planted chain of the target's argmax tokens "
+                         "(D + 1 positions compacted in every layer), one call timed with CUDA events"}
+
     # ---- speculative sampling at T = 1 (Eq. 6 over the tree): msd_step_sample,
     # a replayed graph of draft, verify and the sampling walk + compaction; the
     # uniforms are inputs, copied device to device into the step's buffer
@@ -628,6 +651,7 @@ def run_msd(args, rank, world, local_rank):
             "e2e": e2e,
             "speedup": speedup,
             "distribution": distribution,
+            "compaction_worst_case": worst,
             "sampling": sampling,
             "chain": chain,
             "gpu_launches": int(launches1 - launches0),

@@ -151,6 +151,35 @@ class Tree:
         return msd_tree(_ptr(self.tokens), _ptr(self.parent), _ptr(self.depth), _ptr(self.mask),
                         _ptr(self.n_nodes))
 
+    def plant(self, b: int, tokens, parent):
+        """Writes a caller-planted tree for request b: node i has token tokens[i]
+        and parent parent[i] (-1 for the root, else < i); depths and ancestor
+        masks are derived (host-side layout work, then one copy per array)."""
+        n = len(tokens)
+        if n < 1 or n > self.N or len(parent) != n or parent[0] != -1:
+            raise ValueError("a tree needs 1..N nodes with node 0 as its root")
+        depth = [0] * n
+        for i in range(1, n):
+            if not 0 <= parent[i] < i:
+                raise ValueError("parent[i] must precede node i")
+            depth[i] = depth[parent[i]] + 1
+        mask = [[0] * self.W for _ in range(self.N)]
+        for i in range(n):
+            j = i
+            while j >= 0:
+                mask[i][j // 64] |= 1 << (j % 64)
+                j = parent[j]
+        pad = self.N - n
+        sl = slice(b * self.N, (b + 1) * self.N)
+        dev = self.tokens.device
+        self.tokens[sl] = torch.tensor(list(tokens) + [0] * pad, dtype=torch.int32, device=dev)
+        self.parent[sl] = torch.tensor(list(parent) + [-1] * pad, dtype=torch.int32, device=dev)
+        self.depth[sl] = torch.tensor(depth + [0] * pad, dtype=torch.int32, device=dev)
+        words = [w - (1 << 64) if w >= 1 << 63 else w for row in mask for w in row]
+        self.mask[b * self.N * self.W:(b + 1) * self.N * self.W] = torch.tensor(words, dtype=torch.int64,
+                                                                                device=dev)
+        self.n_nodes[b] = n
+
 
 class Engine:
     """One context of the C ABI plus the caller-owned buffers of a step."""

@@ -92,24 +92,4 @@ def tree_numpy(tree: msd.Tree, b: int):
 
 def plant(tree: msd.Tree, b: int, tokens, parent):
     """Writes a caller-planted tree for request b (depths and masks derived)."""
-    N = tree.N
-    n = len(tokens)
-    depth = np.zeros(n, np.int64)
-    for i in range(1, n):
-        depth[i] = depth[parent[i]] + 1
-    W = tree.W
-    mask = np.zeros((N, W), np.uint64)
-    for i in range(n):
-        j = i
-        while j >= 0:
-            mask[i, j // 64] |= np.uint64(1) << np.uint64(j % 64)
-            j = parent[j]
-    t = np.zeros(N, np.int32); t[:n] = tokens
-    p = np.full(N, -1, np.int32); p[:n] = parent
-    d = np.zeros(N, np.int32); d[:n] = depth
-    sl = slice(b * N, (b + 1) * N)
-    tree.tokens[sl] = torch.from_numpy(t).cuda()
-    tree.parent[sl] = torch.from_numpy(p).cuda()
-    tree.depth[sl] = torch.from_numpy(d).cuda()
-    tree.mask[b * N * W:(b + 1) * N * W] = torch.from_numpy(mask.reshape(-1).view(np.int64)).cuda()
-    tree.n_nodes[b] = n
+    tree.plant(b, [int(x) for x in tokens], [int(x) for x in parent])
