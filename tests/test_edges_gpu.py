@@ -1,0 +1,71 @@
+"""Edge cases of the decode step on the GPU path, against the oracle: the
+degenerate depth-1 tree (no tree-expansion pass), the largest tree the
+configuration admits (N = 256 nodes in four mask words, k = 16, 1296
+candidates), speculative sampling over that tree (16 children per node), and
+the prompts msd_prefill must refuse before any launch."""
+import pytest
+import torch
+
+from paper_2505_14260_gb300 import msd, synth
+from tests.gpu_support import open_engine
+from tests.parity_support import run_parity
+from tests.test_sample_gpu import run_sampling
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_depth_one_tree_matches_oracle(dtype):
+    """D = 1: the root slot's top-k are the whole tree (N = 1 + k)."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype=dtype, tree_depth=1, tree_nodes=5, steps=3)
+    run_parity(wl, wl.steps)
+
+
+@pytest.mark.parametrize("dtype", ["f32", "bf16"])
+def test_largest_tree_matches_oracle(dtype):
+    """N = 256 (four 64-bit mask words per node, four query-row tiles and four
+    tree key tiles per request in attention, a many-row verify GEMM), k = 16,
+    D = 6: k + (D-1) k^2 = 1296 candidates ranked for 255 slots."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype=dtype, tree_nodes=256, tree_depth=6, topk=16, steps=2)
+    run_parity(wl, wl.steps)
+
+
+def test_sampling_over_the_largest_tree_matches_oracle():
+    wl = synth.WORKLOADS["tiny"].with_(dtype="bf16", tree_nodes=256, tree_depth=6, topk=16, steps=2)
+    near, _ = run_sampling(wl, 1.0, wl.steps, seed=5)
+    assert near <= 1
+
+
+def test_prefill_refuses_invalid_prompts():
+    """Refused on the host with MSD_ERR_INVALID (MSD_ERR_CAPACITY for a prompt
+    that leaves no room for a step), before anything is launched."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype="f32")
+    eng, _ = open_engine(wl)
+    prompts = synth.make_prompts(wl)
+    ids, lens, vis, offs = msd.upload_prompts(prompts)
+    L = lens[0]
+
+    def expect(status, ids_, lens_, vis_=vis, offs_=offs):
+        with pytest.raises(msd.MsdError) as e:
+            eng.prefill(ids_, lens_, vis_, offs_)
+        assert e.value.status == status
+
+    expect(msd.MSD_ERR_INVALID, ids, [0])                                 # empty prompt
+    expect(msd.MSD_ERR_INVALID, ids, [L + 1])                             # longer than its row
+    vis_end = ids.clone()
+    vis_end[0, L - 1] = -1
+    expect(msd.MSD_ERR_INVALID, vis_end, lens)                            # ends in a visual slot
+    bad = ids.clone()
+    bad[0, 3] = wl.vocab
+    expect(msd.MSD_ERR_INVALID, bad, lens)                                # token id out of range
+    bad[0, 3] = -2
+    expect(msd.MSD_ERR_INVALID, bad, lens)
+    expect(msd.MSD_ERR_INVALID, ids, lens, None, offs)                    # visual slots, no rows
+    eng.close()
+    small, _ = open_engine(wl.with_(n_text=(4, 4)), steps=0)
+    expect_small = small.cfg.max_seq
+    long_ids = torch.zeros(1, expect_small, dtype=torch.int32, device="cuda")
+    with pytest.raises(msd.MsdError) as e:
+        small.prefill(long_ids, [expect_small], None, [0])
+    assert e.value.status == msd.MSD_ERR_CAPACITY                        # no room for a step
+    small.close()
