@@ -256,6 +256,32 @@ def aggregate_rate(units_per_rank: float, world: int, ms_max: float) -> float:
     return world * units_per_rank / (ms_max / 1e3)
 
 
+def oracle_one_thread(workload: str, steps: int = 3):
+    """The oracle's step on one host thread (BLAS pinned to one thread in a
+    child process, so the parent's thread pools are untouched): steps/s."""
+    code = (
+        "import sys, time, json, statistics\n"
+        f"sys.path.insert(0, {ROOT!r})\n"
+        "import bench\n"
+        "from paper_2505_14260_gb300 import synth\n"
+        f"wl = synth.WORKLOADS[{workload!r}]\n"
+        "w = synth.make_weights(wl)\n"
+        "w = {k: v for k, v in w.items() if k != 'layers'} | {'layers': w['layers'][:2]}\n"
+        "s = bench.OracleSample(wl, w, synth.make_prompts(wl))\n"
+        f"est = [s.step_seconds()[0] for _ in range({steps})]\n"
+        "print(json.dumps({'value': 1.0 / statistics.mean(est)}))\n")
+    env = dict(os.environ, OMP_NUM_THREADS="1", OPENBLAS_NUM_THREADS="1", MKL_NUM_THREADS="1",
+               CUDA_VISIBLE_DEVICES="")
+    try:
+        r = subprocess.run([sys.executable, "-c", code], env=env, capture_output=True, text=True,
+                           timeout=300)
+        v = json.loads(r.stdout.strip().splitlines()[-1])["value"]
+        return {"value": v, "unit": "steps/s", "cores": 1, "kind": "oracle",
+                "sample": f"the same oracle step, BLAS and OpenMP pinned to one thread, mean of {steps} steps"}
+    except Exception as ex:
+        return {"value": None, "unit": "steps/s", "cores": 1, "kind": "oracle", "sample": f"failed: {ex!r}"}
+
+
 def make_inputs(wl, device):
     import torch
     from paper_2505_14260_gb300 import synth
@@ -619,6 +645,10 @@ def run_msd(args, rank, world, local_rank):
         except Exception as ex:           # the bench line must still print
             cpu = {"value": None, "unit": "steps/s", "cores": None, "kind": "oracle",
                    "sample": f"failed: {ex!r}"}
+        if cpu.get("value") and wl.name == "tiny":
+            cpu["one_thread"] = oracle_one_thread(wl.name)
+
+
 
     if rank == 0:
         line = {
