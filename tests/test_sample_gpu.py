@@ -247,3 +247,35 @@ def test_sample_argument_errors():
         eng.verify(tree=t)
     assert e.value.status == msd.MSD_ERR_DEVICE
     eng.close()
+
+
+def test_many_walks_match_oracle():
+    """96 walks (32 ragged requests x 3 steps at T = 0.2, 1 and 3) against the
+    oracle's accept_sample on the kernels' logits with the same uniforms: the
+    walk and the drawn token only (the caches are checked by the tests above)."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype="bf16", batch=32, n_text=(8, 60), steps=3)
+    B, N, D, k, V = wl.batch, wl.tree_nodes, wl.tree_depth, wl.topk, wl.vocab
+    eng, _ = open_engine(wl, steps=wl.steps)
+    ids, lens, vis, offs = msd.upload_prompts(synth.make_prompts(wl))
+    eng.prefill(ids, lens, vis, offs)
+    logits = torch.zeros(B * N, V, device="cuda")
+    gen = torch.Generator().manual_seed(21)
+    near = walks = 0
+    for step, T in enumerate((0.2, 1.0, 3.0)):
+        eng.draft_tree()
+        eng.verify(logits=logits)
+        u = torch.rand(B, D + 1, k + 1, generator=gen)
+        eng.accept_sample(T, u.cuda(), logits=logits)
+        torch.cuda.synchronize()
+        g_all = logits.cpu().numpy().astype(np.float64)
+        path_all, alen, bonus = eng.path.cpu().numpy(), eng.accept_len.cpu().numpy(), eng.bonus.cpu().numpy()
+        for b in range(B):
+            toks, par, dep, _ = tree_numpy(eng.tree, b)
+            otree = O.Tree(tokens=toks, parent=par, depth=dep)
+            a = int(alen[b])
+            gpu = ([int(x) for x in path_all[b * (D + 1):b * (D + 1) + a + 1]], a, int(bonus[b]))
+            near += check_walk(gpu, otree, g_all[b * N:(b + 1) * N], T, u[b].numpy().astype(np.float64), k,
+                               f"T={T} request {b} step {step}")
+            walks += 1
+    eng.close()
+    assert walks == 96 and near <= 2
