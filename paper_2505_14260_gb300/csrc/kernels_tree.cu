@@ -398,6 +398,8 @@ constexpr int SAMPLE_THREADS = 1024;
 constexpr int STATS_THREADS = 1024;
 constexpr int STATS_VEC = 8;         // float4 per thread held in registers (rows up to 32768)
 constexpr int DRAW_ROUNDS = 16;      // rounds of 32 tokens a warp loads at once in the draw
+constexpr int SAMPLE_MAXN = 256;     // tree nodes (the configuration's limit)
+constexpr int SAMPLE_MAXU = (TREE_MAXD + 1) * (TREE_MAXK + 1);   // uniforms of one request
 
 __device__ __forceinline__ float exp2_fast(float x) {
     float y;
@@ -511,11 +513,24 @@ accept_sample_kernel(TreeIn t, const float *__restrict__ logits, const float *__
     __shared__ int path[TREE_MAXD + 1];
     __shared__ int kids[TREE_MAXK], removed[TREE_MAXK], kid_tok[TREE_MAXK];
     __shared__ double kid_p[TREE_MAXK];
-    __shared__ float kid_u[TREE_MAXK];
     __shared__ int sh_cur, sh_a, sh_nrem, sh_warp, sh_pick;
     __shared__ double wsum[32], sh_base, sh_target;
     __shared__ int wlast[32];
+    // the request's tree, row statistics and uniforms, loaded once: the walk
+    // then waits on one global round trip per node (its children's logits)
+    __shared__ int s_par[SAMPLE_MAXN], s_tok[SAMPLE_MAXN];
+    __shared__ float s_rmax[SAMPLE_MAXN];
+    __shared__ double s_rsum[SAMPLE_MAXN];
+    __shared__ float s_u[SAMPLE_MAXU];
     for (int i = tid; i < words; i += blockDim.x) removed_bits[i] = 0u;
+    for (int i = tid; i < n; i += blockDim.x) {
+        s_par[i] = t.parent[nb + i];
+        s_tok[i] = t.tokens[nb + i];
+        s_rmax[i] = row_max[nb + i];
+        s_rsum[i] = row_sum[nb + i];
+    }
+    for (int i = tid; i < D1 * (k + 1); i += blockDim.x) s_u[i] = ub[i];
+    __syncthreads();
 
     // the walk (warp 0): Eq. 6 with point-mass proposals at every node. The
     // lanes fetch the children's tokens, probabilities and uniforms at once;
@@ -524,12 +539,12 @@ accept_sample_kernel(TreeIn t, const float *__restrict__ logits, const float *__
         int cur = 0, a = 0, nrem = 0;
         if (lane == 0) path[0] = 0;
         for (;;) {
-            const float M = row_max[nb + cur];
-            const double S = row_sum[nb + cur];
+            const float M = s_rmax[cur];
+            const double S = s_rsum[cur];
             int cnt = 0;
             for (int c0 = 1; c0 < n; c0 += 32) {
                 const int c = c0 + lane;
-                const bool is = c < n && t.parent[nb + c] == cur;
+                const bool is = c < n && s_par[c] == cur;
                 const unsigned bal = __ballot_sync(0xffffffffu, is);
                 const int slot = cnt + __popc(bal & ((1u << lane) - 1u));
                 if (is && slot < k) kids[slot] = c;
@@ -538,11 +553,10 @@ accept_sample_kernel(TreeIn t, const float *__restrict__ logits, const float *__
             __syncwarp();
             const int nk = a < D ? min(cnt, k) : 0;
             if (lane < nk) {
-                const int x = t.tokens[nb + kids[lane]];
+                const int x = s_tok[kids[lane]];
                 const bool ok = x >= 0 && x < V;
                 kid_tok[lane] = ok ? x : -1;
                 kid_p[lane] = ok ? (double)exp2_fast((logits[(nb + cur) * V + x] - M) * scale) / S : 0.0;
-                kid_u[lane] = ub[a * (k + 1) + lane];
             }
             __syncwarp();
             int next = -1;
@@ -559,7 +573,7 @@ accept_sample_kernel(TreeIn t, const float *__restrict__ logits, const float *__
                     bool dup = false;
                     for (int r = 0; r < nrem; ++r) dup |= removed[r] == x;
                     const double px = dup ? 0.0 : kid_p[j];
-                    if ((double)kid_u[j] * (1.0 - gone) < px) {
+                    if ((double)s_u[a * (k + 1) + j] * (1.0 - gone) < px) {
                         next = kids[j];
                         break;
                     }
@@ -594,7 +608,7 @@ accept_sample_kernel(TreeIn t, const float *__restrict__ logits, const float *__
     // owns tokens [w*seg, (w+1)*seg) in rounds of 32 consecutive tokens (lane l
     // takes token 32j + l of round j: coalesced), DRAW_ROUNDS rounds loaded at once.
     const float *z = logits + (nb + cur) * V;
-    const float M = row_max[nb + cur];
+    const float M = s_rmax[cur];
     const int seg = 32 * ((V + 32 * nw - 1) / (32 * nw));
     const int t0 = warp * seg, t1 = min(t0 + seg, V);
     float hi = 0.f, lo = 0.f;
@@ -632,7 +646,7 @@ accept_sample_kernel(TreeIn t, const float *__restrict__ logits, const float *__
             if (lane >= o) inc += y;
         }
         const double total = __shfl_sync(0xffffffffu, inc, 31);
-        const double target = (double)ub[a * (k + 1) + k] * total;
+        const double target = (double)s_u[a * (k + 1) + k] * total;
         double excl = __shfl_up_sync(0xffffffffu, inc, 1);   // the intervals tile [0, total)
         if (lane == 0) excl = 0.0;
         const bool here = lane < nw && v > 0.0 && excl <= target && target < inc;
