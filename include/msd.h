@@ -237,8 +237,9 @@ msd_status msd_step(msd_ctx *ctx, const msd_tree *tree, int32_t *argmax_dev, int
  * CUDA graph exactly as msd_step (one graph per set of buffers, u_dev pointer,
  * temperature and bucket of cache lengths). The caller refills u_dev
  * ([B][D+1][k+1] uniforms in [0, 1)) before each step; the graph reads it when
- * it runs. Errors: as msd_step, and MSD_ERR_INVALID for a null u_dev or a
- * temperature that is not finite and > 0. */
+ * it runs. Errors: as msd_step, and MSD_ERR_INVALID for a null u_dev, a
+ * temperature that is not finite and > 0, or vocab > 393216 (as
+ * msd_accept_sample). */
 msd_status msd_step_sample(msd_ctx *ctx, const msd_tree *tree, float temperature,
                            const float *u_dev, int32_t *argmax_dev, int32_t *path_dev,
                            int32_t *accept_len_dev, int32_t *bonus_dev, void *stream);
