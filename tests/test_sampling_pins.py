@@ -140,3 +140,21 @@ def test_zero_temperature_limit_is_greedy_acceptance(drafted):
         path, a, bonus = O.accept_sample(tree, vr.logits, 1e-4, rng.random((wl.tree_depth + 1, wl.topk + 1)),
                                          wl.topk)
         assert list(path) == list(path_g) and a == a_g and bonus == bonus_g
+
+
+def test_duplicate_sibling_tokens_add_no_mass():
+    """A caller-planted tree may repeat a token among siblings: once rejected,
+    the token has no mass left in the adjusted distribution, so its duplicate
+    is never accepted and the draw excludes it (the emitted distribution is
+    that of the tree without the duplicate)."""
+    tree = _tree([9, 3, 3, 2], [-1, 0, 0, 0])
+    rows = np.repeat(ROWS[:1], 4, axis=0)      # every node's row: the root's p (only the root is visited)
+    u = np.full((2, 4), 0.999)
+    u[0, 0] = 0.41                       # 3 rejected (0.41 >= 0.4)
+    u[0, 1] = 0.0                        # the duplicate 3: p_adj(3) = 0, rejected even at u = 0
+    u[0, 2] = 0.99                       # 2 rejected: 0.99 * 0.6 >= 0.3
+    u[0, 3] = 0.5                        # draw from (0.1, 0.2) renormalised: 0.5 * 0.3 = 0.15 -> 1
+    path, a, bonus = O.accept_sample(tree, rows, 1.0, u, 3)
+    assert list(path) == [0] and a == 0 and bonus == 1
+    ref = O.accept_sample(_tree([9, 3, 2], [-1, 0, 0]), rows, 1.0, u[:, [0, 2, 2, 3]], 3)
+    assert ref[1] == 0 and ref[2] == bonus
