@@ -538,11 +538,11 @@ def run_msd(args, rank, world, local_rank):
         toks, par = [int(eng.state()["root"].cpu()[0])], [-1]
         eng.draft_tree()                  # keeps the draft cache caught up
         for d in range(D):
-            chain_tree.plant(0, toks, par)
+            eng.plant(chain_tree, 0, toks, par)
             eng.verify(tree=chain_tree)
             toks.append(int(eng.argmax[d].cpu()))
             par.append(d)
-        chain_tree.plant(0, toks, par)
+        eng.plant(chain_tree, 0, toks, par)
         eng.verify(tree=chain_tree)
         torch.cuda.synchronize()
         e0.record(stream)

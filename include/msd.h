@@ -173,6 +173,18 @@ msd_status msd_draft_tree(msd_ctx *ctx, const msd_tree *out,
 msd_status msd_verify(msd_ctx *ctx, const msd_tree *tree, int32_t *argmax_dev,
                       float *logits_dev, void *stream);
 
+/* Completes a caller-planted tree (the draft-tree structure of Sec. 3.2: a
+ * candidate is conditioned on its ancestors): for request b = `request` (or
+ * every request b < max_batch if request is -1), from parent[b*N+i] of its n_nodes[b] nodes (all N if n_nodes is NULL) it
+ * writes depth[b*N+i] (the number of ancestors) and the ancestor-or-self mask
+ * words of the layout above; nodes at or past n_nodes[b] get depth 0 and an
+ * empty mask. tokens are not read. A node whose parent does not precede it
+ * (parent[b*N+i] outside [0, i) for i > 0, or a root with a parent) sets the
+ * device status word (reported by the next call as MSD_ERR_DEVICE) and is
+ * treated as a child of the root. Errors: MSD_ERR_INVALID (null arrays, request
+ * outside [-1, max_batch)). */
+msd_status msd_tree_complete(msd_ctx *ctx, const msd_tree *tree, int32_t request, void *stream);
+
 /* Accept and compact (Eq. 6 at temperature 0, and the rule that rejected
  * drafts are discarded): from the root, follow the child whose token equals the
  * target argmax at the current node; path_dev[b*(D+1)+j] (j <= a, rest -1),
@@ -279,24 +291,42 @@ msd_status msd_linear(msd_ctx *ctx, const void *x_dev, int32_t ldx, int32_t m, i
  * whose device memory is all owned by its own pool allocator, code running
  * where an allocation would synchronise the device or is not permitted, a
  * plug-in handed buffers but no allocator). It needs no context and allocates
- * nothing: its split-K scratch is one static device array of 16 MiB of fp32
- * partials plus 4096 int tile tickets, which every GPU that loads this library
- * holds until the process exits. The paper has no counterpart; this is a
- * service of the library, not a step of the method.
+ * nothing: its scratch is one static device array (a 256-byte status word,
+ * 4096 int tile tickets and 16 MiB of fp32 split-K partials) which every GPU
+ * that loads this library holds until the process exits. The paper has no
+ * counterpart; this is a service of the library, not a step of the method.
  * Arguments are those of msd_linear (x [m][ldx], w [o][k] bf16 with ldx and k
  * multiples of 8, y [m][ldy] fp32, all device memory on the current device).
- * The first call made on a device looks up the array's device address on that
- * device (cudaGetSymbolAddress) and sets the kernel's shared-memory limit;
- * make that first call before any stream capture. Every call shares the array
- * and it keeps the last call's contents; the tile tickets are cleared on
- * `stream` before each launch that uses them. Calls that overlap on the GPU
- * (other streams, other host threads) race on the array: serialise them.
+ * The split-K choice is limited to what the array holds: a shape whose best
+ * split would need more partials or tickets runs with fewer splits (none at
+ * worst), so no shape is refused for its scratch. The first call made on a
+ * device looks up the array's device address on that device
+ * (cudaGetSymbolAddress) and sets the kernel's shared-memory limit; make that
+ * first call before any stream capture. Every call shares the array and it
+ * keeps the last call's contents; the tile tickets are cleared on `stream`
+ * before each launch that uses them. Calls that overlap on the GPU (other
+ * streams, other host threads) race on the array: serialise them.
+ * Device-side errors: a bounded wait of the kernel that runs out (2 s) sets the
+ * array's status word. Each call first reads that word back on `stream` (so it
+ * returns only after the work queued before it on `stream` has finished); if it
+ * is set, the call clears it, launches nothing and returns MSD_ERR_DEVICE: the
+ * failed call's y is not to be trusted.
  * Errors: MSD_ERR_INVALID (null pointer, non-positive size, bad stride or
- * alignment), MSD_ERR_CAPACITY (the shape's split-K partials would exceed the
- * 16 MiB array or its 4096 tickets), MSD_ERR_CUDA (a runtime call failed). */
+ * alignment), MSD_ERR_CAPACITY (m > 65535 * 256, the token-tile grid limit),
+ * MSD_ERR_DEVICE (see above), MSD_ERR_CUDA (a runtime call failed). */
 msd_status msd_linear_noalloc(const void *x_dev, int32_t ldx, int32_t m, int32_t k,
                               const void *w_dev, int32_t o, float *y_dev, int32_t ldy,
                               int32_t accumulate, void *stream);
+
+/* Test hook of the failure detection (no counterpart in the paper): launches
+ * one CTA that waits, through the library's bounded mbarrier wait, on a
+ * barrier that nothing ever arrives at; after limit_ns (1e3 .. 2e9) it gives up
+ * and records a timeout in the device status word of ctx -- or, for ctx NULL,
+ * in the status word of msd_linear_noalloc on the current device. No copy or
+ * MMA is in flight during the wait, so nothing else is disturbed; the next call
+ * on that context (or the next msd_linear_noalloc) reports MSD_ERR_DEVICE.
+ * Errors: MSD_ERR_INVALID (limit out of range), MSD_ERR_CUDA. */
+msd_status msd_test_wait_timeout(msd_ctx *ctx, int64_t limit_ns, void *stream);
 
 /* Profiling counters (tracing subsystem). kernel_launches counts every kernel
  * the library has run in this process (kernels executed by step graphs

@@ -1,5 +1,5 @@
-// Tree-masked attention on CUDA cores (the fp32 path and the bf16 draft
-// passes). One warp per (row, head); online softmax over the visible keys:
+// Tree-masked attention on CUDA cores (the fp32 path; bf16 contexts run
+// attn_tc.cu for every pass). One warp per (row, head); online softmax over the visible keys:
 // the cache prefix [0, plen) of the row's request, then the tree slots whose
 // bit is set in the row's mask (Sec. 3.2: a candidate sees its prefix only).
 #include "kernels.h"

@@ -85,14 +85,17 @@ __device__ __forceinline__ bool mbar_try(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-// Bounded wait for the phase with the given parity to complete.
-__device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag, int *status) {
+// Bounded wait for the phase with the given parity to complete: gives up when
+// another thread of the CTA has set *abort_flag, or after limit_ns, when it
+// sets *abort_flag and records ST_TIMEOUT in the status word.
+__device__ bool mbar_wait(uint32_t bar, uint32_t parity, volatile int *abort_flag, int *status,
+                          unsigned long long limit_ns = TIMEOUT_NS) {
     if (mbar_try(bar, parity)) return true;
     const unsigned long long t0 = gtimer();
     while (true) {
         if (mbar_try(bar, parity)) return true;
         if (*abort_flag) return false;
-        if (gtimer() - t0 > TIMEOUT_NS) {
+        if (gtimer() - t0 > limit_ns) {
             *abort_flag = 1;
             set_status(status, ST_TIMEOUT);
             return false;
@@ -271,6 +274,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                 mma_commit(empty0 + 8 * s);
             }
             mma_commit(done);   // arrives once every MMA issued above has completed
+            // after an abort the epilogue may skip its wait: the tensor memory is
+            // freed only once every MMA issued here has completed
+            volatile int never = 0;
+            mbar_wait(done, 0, &never, p.status);
         }
         __syncwarp();
     }
@@ -422,7 +429,7 @@ struct ItemIter {
 __global__ void __launch_bounds__(P_THREADS, 1)
     gemm_persist_kernel(const __grid_constant__ CUtensorMap mx, const PkParams p) {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t bars[2 * P_MAX_STAGES + 4];
+    __shared__ __align__(8) uint64_t bars[2 * P_MAX_STAGES + 5];
     __shared__ uint32_t tmem_base;
     __shared__ volatile int abort_flag;
     __shared__ int s_reduce;
@@ -441,6 +448,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[P_MAX_STAGES]);
     const uint32_t accf0 = smem_u32(&bars[2 * P_MAX_STAGES]);
     const uint32_t acce0 = smem_u32(&bars[2 * P_MAX_STAGES + 2]);
+    const uint32_t drain = smem_u32(&bars[2 * P_MAX_STAGES + 4]);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < stages; ++s) {
@@ -451,6 +459,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
             mbar_init(accf0 + 8 * a, 1);
             mbar_init(acce0 + 8 * a, 128);
         }
+        mbar_init(drain, 1);
         abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
@@ -561,6 +570,10 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 }
                 mma_commit(accf0 + 8 * a);
             }
+            // every MMA issued above completes before the CTA frees its TMEM
+            mma_commit(drain);
+            volatile int never = 0;
+            mbar_wait(drain, 0, &never, p.status);
         }
         __syncwarp();
     } else {
@@ -1212,6 +1225,8 @@ __global__ void __launch_bounds__(C_THREADS)
                 }
             }
             mma_commit(done);
+            volatile int never = 0;     // (as gemm_tc_kernel: no MMA outlives the CTA's TMEM)
+            mbar_wait(done, 0, &never, p.status);
         }
         __syncwarp();
     } else {
@@ -1822,20 +1837,26 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
 // GEMM lives in one file-scope device array, loaded with the library and held
 // by every GPU that loads it until the process exits.
 //
-// Layout of the array: NOALLOC_COUNTERS int tile tickets, then the fp32
-// split-K partials (NOALLOC_PARTIAL_BYTES). In host code the array's name is
-// only a host-side stand-in; the device address comes from
-// cudaGetSymbolAddress, taken once per device (with that device current) on
-// the first call made on it. Every call shares the array and it keeps the last
-// call's contents: the tickets are cleared on the caller's stream before each
-// launch that uses them, and calls that overlap on the GPU race on the array.
+// Layout of the array: a status word (padded to 256 bytes), NOALLOC_COUNTERS
+// int tile tickets, then the fp32 split-K partials (NOALLOC_PARTIAL_BYTES). In
+// host code the array's name is only a host-side stand-in; the device address
+// comes from cudaGetSymbolAddress, taken once per device (with that device
+// current) on the first call made on it. Every call shares the array and it
+// keeps the last call's contents: the tickets are cleared on the caller's
+// stream before each launch that uses them, and calls that overlap on the GPU
+// race on the array. The split-K choice is limited to what the array holds, so
+// a shape that would split further on the context GEMM runs with fewer splits
+// (none at worst) instead of being refused.
 // ---------------------------------------------------------------------------
 namespace msd {
 namespace {
+constexpr size_t NOALLOC_STATUS_BYTES = 256;
 constexpr int NOALLOC_COUNTERS = 4096;
 constexpr size_t NOALLOC_PARTIAL_BYTES = 16ull << 20;
-constexpr size_t NOALLOC_BYTES = NOALLOC_COUNTERS * sizeof(int) + NOALLOC_PARTIAL_BYTES;
+constexpr size_t NOALLOC_BYTES = NOALLOC_STATUS_BYTES + NOALLOC_COUNTERS * sizeof(int) + NOALLOC_PARTIAL_BYTES;
 constexpr int NOALLOC_MAX_DEVICES = 64;
+constexpr size_t NOALLOC_MAX_MAPS = 256;   // cached weight tensor maps per process
+constexpr long NOALLOC_MAX_ROWS = 65535L * 256;   // token-tile grid dimension limit
 }  // namespace
 
 static __device__ __align__(256) unsigned char g_noalloc_scratch[NOALLOC_BYTES];
@@ -1845,11 +1866,81 @@ struct NoAllocDevice {
     bool ready = false;
     unsigned char *scratch = nullptr;   // device address of g_noalloc_scratch
     int num_sms = 0;
+    int status_host = 0;                // last value read back from the status word
 };
 std::mutex g_noalloc_mu;
 NoAllocDevice g_noalloc_dev[NOALLOC_MAX_DEVICES];
 GemmPlan g_noalloc_maps;                // host-side tensor-map cache only (no device memory)
+
+// One-time set-up of the current device (caller holds g_noalloc_mu).
+bool noalloc_setup(int dev) {
+    NoAllocDevice &d = g_noalloc_dev[dev];
+    if (d.ready) return true;
+    void *ptr = nullptr;
+    if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return false;
+    if (cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess) return false;
+    if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 200 * 1024 + 1024) !=
+        cudaSuccess)
+        return false;
+    if (!g_noalloc_maps.encode) {
+        cudaDriverEntryPointQueryResult q;
+        void *fn = nullptr;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+                cudaSuccess ||
+            q != cudaDriverEntryPointSuccess || !fn)
+            return false;
+        g_noalloc_maps.encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
+    }
+    d.scratch = static_cast<unsigned char *>(ptr);
+    d.ready = true;
+    return true;
+}
+
+// Tensor map of an activation operand: encoded on every call (a host-only
+// computation), so the cache holds weight maps alone.
+bool encode_x_map(const void *x, long rows, long cols, long ld, long box_rows, CUtensorMap *m) {
+    memset(m, 0, sizeof *m);
+    cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)ld * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)box_rows};
+    cuuint32_t estr[2] = {1, 1};
+    return g_noalloc_maps.encode(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(x), dims, strides, box,
+                                 estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+                                 CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) ==
+           CUDA_SUCCESS;
+}
 }  // namespace
+
+// Device address of the no-alloc status word on the current device (set-up
+// included); null if the set-up failed.
+int *noalloc_status_word() {
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= NOALLOC_MAX_DEVICES) return nullptr;
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!noalloc_setup(dev)) return nullptr;
+    return reinterpret_cast<int *>(g_noalloc_dev[dev].scratch);
+}
+
+// Test hook of the bounded waits: one CTA waits on an mbarrier that nothing
+// arrives at, through the same bounded wait as the GEMM kernels, gives up
+// after limit_ns and records ST_TIMEOUT in *status. No copy or MMA is in
+// flight while it waits.
+__global__ void wait_probe_kernel(int *status, unsigned long long limit_ns) {
+    __shared__ __align__(8) uint64_t bar;
+    __shared__ volatile int abort_flag;
+    if (threadIdx.x == 0) {
+        mbar_init(smem_u32(&bar), 1);
+        abort_flag = 0;
+        asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+        mbar_wait(smem_u32(&bar), 0, &abort_flag, status, limit_ns);
+    }
+}
+
+bool launch_wait_probe(int *status, long long limit_ns, cudaStream_t s) {
+    wait_probe_kernel<<<1, 32, 0, s>>>(status, (unsigned long long)limit_ns);
+    note_launch();
+    return cudaGetLastError() == cudaSuccess;
+}
 
 }  // namespace msd
 
@@ -1858,34 +1949,31 @@ extern "C" msd_status msd_linear_noalloc(const void *x, int32_t ldx, int32_t m, 
                                          int32_t accumulate, void *stream) {
     using namespace msd;
     constexpr msd_status OK = MSD_OK, INVALID = MSD_ERR_INVALID, CAPACITY = MSD_ERR_CAPACITY,
-                         CUDA_ERR = MSD_ERR_CUDA;
+                         CUDA_ERR = MSD_ERR_CUDA, DEVICE = MSD_ERR_DEVICE;
     if (!x || !w || !y || m <= 0 || k <= 0 || o <= 0 || ldx < k || ldy < o) return INVALID;
     if (ldx % 8 || k % 8) return INVALID;
+    if ((long)m > NOALLOC_MAX_ROWS) return CAPACITY;
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= NOALLOC_MAX_DEVICES) return CUDA_ERR;
     std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    if (!noalloc_setup(dev)) return CUDA_ERR;
     NoAllocDevice &d = g_noalloc_dev[dev];
-    if (!d.ready) {
-        void *ptr = nullptr;
-        if (cudaGetSymbolAddress(&ptr, g_noalloc_scratch) != cudaSuccess || !ptr) return CUDA_ERR;
-        if (cudaDeviceGetAttribute(&d.num_sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess)
-            return CUDA_ERR;
-        if (cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 200 * 1024 + 1024) != cudaSuccess)
-            return CUDA_ERR;
-        if (!g_noalloc_maps.encode) {
-            cudaDriverEntryPointQueryResult q;
-            void *fn = nullptr;
-            if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000,
-                                                 cudaEnableDefault, &q) != cudaSuccess ||
-                q != cudaDriverEntryPointSuccess || !fn)
-                return CUDA_ERR;
-            g_noalloc_maps.encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
-        }
-        d.scratch = static_cast<unsigned char *>(ptr);
-        d.ready = true;
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int *status = reinterpret_cast<int *>(d.scratch);
+    // The status word left by earlier launches on this device (a bounded wait
+    // that ran out): read back into pageable host memory, so the copy returns
+    // once the work queued before it on `stream` has finished; a set word is
+    // cleared and reported once.
+    if (cudaMemcpyAsync(&d.status_host, status, sizeof(int), cudaMemcpyDeviceToHost, s) != cudaSuccess)
+        return CUDA_ERR;
+    if (cudaStreamSynchronize(s) != cudaSuccess) return CUDA_ERR;
+    if (d.status_host != 0) {
+        d.status_host = 0;
+        if (cudaMemsetAsync(status, 0, sizeof(int), s) != cudaSuccess) return CUDA_ERR;
+        return DEVICE;
     }
-    // The same plan as the context GEMM (tile shape, stages, split-K choice).
+    // The same tile shape and stages as the context GEMM; the split-K choice is
+    // limited to what the array holds.
     const int M = m, K = k, O = o;
     const int tiles = (O + BM - 1) / BM;
     const int nt = (M + 255) / 256;
@@ -1905,17 +1993,14 @@ extern "C" msd_status msd_linear_noalloc(const void *x, int32_t ldx, int32_t m, 
     for (int sp = 1; sp <= 16 && sp <= kblocks; ++sp) {
         const int kps = (kblocks + sp - 1) / sp;
         const int se = (kblocks + kps - 1) / kps;
-        if (se > 1 && ((size_t)base * se * tile_bytes > WS_BYTES || base > N_COUNTERS)) continue;
+        if (se > 1 && ((size_t)base * se * tile_bytes > NOALLOC_PARTIAL_BYTES || base > NOALLOC_COUNTERS))
+            continue;
         const long waves = (base * se + slots - 1) / slots;
         const double cost = (double)waves * kps + (se > 1 ? 2.0 : 0.0);
         if (cost < best - 1e-9) { best = cost; best_s = se; }
     }
     const int kps = (kblocks + best_s - 1) / best_s;
     const int splits = (kblocks + kps - 1) / kps;
-    // Sizes whose split-K partials or tickets exceed the static array are refused.
-    if (splits > 1 && ((size_t)base * splits * tile_bytes > NOALLOC_PARTIAL_BYTES ||
-                       base > NOALLOC_COUNTERS))
-        return CAPACITY;
 
     TcParams tp;
     memset(&tp, 0, sizeof tp);
@@ -1934,17 +2019,16 @@ extern "C" msd_status msd_linear_noalloc(const void *x, int32_t ldx, int32_t m, 
     tp.Y = y;
     tp.ldy = ldy;
     tp.epi = accumulate ? EPI_ADD : EPI_STORE;
-    tp.counters = reinterpret_cast<int *>(d.scratch);
-    tp.ws = reinterpret_cast<float *>(d.scratch + NOALLOC_COUNTERS * sizeof(int));
-    tp.status = nullptr;
+    tp.counters = reinterpret_cast<int *>(d.scratch + NOALLOC_STATUS_BYTES);
+    tp.ws = reinterpret_cast<float *>(d.scratch + NOALLOC_STATUS_BYTES + NOALLOC_COUNTERS * sizeof(int));
+    tp.status = status;
+    if (g_noalloc_maps.maps.size() >= NOALLOC_MAX_MAPS) g_noalloc_maps.maps.clear();
     const CUtensorMap *mw = get_map(&g_noalloc_maps, w, O, K, K, BM, nullptr);
-    const CUtensorMap *mx = get_map(&g_noalloc_maps, x, M, K, ldx, BN, nullptr);
-    if (!mw || !mx) return INVALID;
-    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    CUtensorMap mx;
+    if (!mw || !encode_x_map(x, M, K, ldx, BN, &mx)) return INVALID;
     if (splits > 1 && cudaMemsetAsync(tp.counters, 0, sizeof(int) * base, s) != cudaSuccess)
         return CUDA_ERR;
-    gemm_tc_kernel<<<dim3(tiles, nt, splits), THREADS, smem, s>>>(*mw, *mw, *mw, *mx, tp);
+    gemm_tc_kernel<<<dim3(tiles, nt, splits), THREADS, smem, s>>>(*mw, *mw, *mw, mx, tp);
     note_launch();
     return cudaGetLastError() == cudaSuccess ? OK : CUDA_ERR;
 }
-

@@ -86,6 +86,15 @@ struct GemmProfile {
     double bytes;
     double weight_bytes;
 };
+// Device address of msd_linear_noalloc's status word on the current device
+// (first use sets the device up); null if that failed.
+int *noalloc_status_word();
+
+// Test hook of the bounded mbarrier waits: one CTA waits on a barrier that
+// nothing arrives at, gives up after limit_ns and records ST_TIMEOUT in
+// *status. Returns false if the launch failed.
+bool launch_wait_probe(int *status, long long limit_ns, cudaStream_t s);
+
 void gemm_profile_enable(GemmPlan *p, bool on);
 bool gemm_profile_on(const GemmPlan *p);
 GemmProfile gemm_profile_read(GemmPlan *p);

@@ -303,6 +303,47 @@ __global__ void root_tree_kernel(const int *__restrict__ root, int B, int N, int
 }
 
 // ---------------------------------------------------------------------------
+// Depths and ancestor masks of a caller-planted tree (Sec. 3.2: a candidate is
+// conditioned on its prefix, i.e. on its ancestors): one CTA per request, the
+// parent array staged in shared memory, one thread per node walking its
+// parent links to the root (at most N steps). A node whose parent does not
+// precede it (or a root with a parent) sets ST_BAD_TREE and is treated as a
+// child of the root, so every walk ends.
+// ---------------------------------------------------------------------------
+__global__ void tree_complete_kernel(const int *__restrict__ parent, int *__restrict__ depth,
+                                     uint64_t *__restrict__ mask, const int *__restrict__ n_nodes, int N,
+                                     int W, int b0, int *status) {
+    wait_prior();
+    allow_dependents();
+    __shared__ int s_par[256];
+    const int b = b0 + blockIdx.x;
+    const int n = n_nodes ? min(max(n_nodes[b], 0), N) : N;
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+        int p = i < n ? parent[(size_t)b * N + i] : -1;
+        if (i < n && (i == 0 ? p != -1 : (p < 0 || p >= i))) {
+            set_status(status, ST_BAD_TREE);
+            p = i == 0 ? -1 : 0;
+        }
+        s_par[i] = p;
+    }
+    __syncthreads();
+    for (int i = threadIdx.x; i < N; i += blockDim.x) {
+        uint64_t *m = mask + ((size_t)b * N + i) * W;
+        for (int w = 0; w < W; ++w) m[w] = 0ull;
+        if (i >= n) {
+            depth[(size_t)b * N + i] = 0;
+            continue;
+        }
+        int d = 0;
+        for (int j = i; j >= 0; j = s_par[j]) {      // parents strictly decrease: <= N steps
+            m[j >> 6] |= 1ull << (j & 63);
+            if (j != i) ++d;
+        }
+        depth[(size_t)b * N + i] = d;
+    }
+}
+
+// ---------------------------------------------------------------------------
 // Greedy acceptance (Eq. 6 at T = 0): one warp per request walks from the root
 // to the child whose token is the target argmax of the current node.
 // ---------------------------------------------------------------------------
@@ -830,11 +871,8 @@ void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand
                           const int *cand_depth, const float *cand_score, int *node_of,
                           const int *root, int B, int C, int N, int *status, cudaStream_t s) {
     const size_t smem = (size_t)C * 3 * sizeof(float);
-    static bool attr = false;       // candidate arrays beyond 48 KB (deep, wide trees)
-    if (!attr) {
-        cudaFuncSetAttribute(tree_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-        attr = true;
-    }
+    // candidate arrays beyond 48 KB (deep, wide trees); the attribute is per device
+    cudaFuncSetAttribute(tree_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
     launch_pdl(tree_finalize_kernel, B, 512, smem, s, t, cand_tok, cand_par, cand_depth, cand_score, node_of,
                root, C, N, status);
     note_launch();
@@ -846,6 +884,12 @@ void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, i
     const int R = B * N;
     launch_pdl(verify_setup_kernel, (R + 127) / 128, 128, 0, s, t, seq_len, root, B, N, V, rows, src,
                                                           vmask, status); note_launch();
+}
+
+void launch_tree_complete(const int *parent, int *depth, uint64_t *mask, const int *n_nodes, int b0, int nb,
+                          int N, int *status, cudaStream_t s) {
+    launch_pdl(tree_complete_kernel, nb, 256, 0, s, parent, depth, mask, n_nodes, N, (N + 63) / 64, b0, status);
+    note_launch();
 }
 
 void launch_root_tree(const int *root, int B, int N, int W, int *tokens, int *parent, int *depth,
@@ -863,19 +907,30 @@ void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int 
                                    index_map_out); note_launch();
 }
 
-void launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, int D, int k, int V,
+bool launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, int D, int k, int V,
                           float inv_temp, const float *u, float *row_max, double *row_sum, int *seq_len,
                           int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
                           int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,
                           int *status, cudaStream_t s) {
+    if (V > SAMPLE_MAX_VOCAB) return false;
+    // the rejected-token bitmap (dynamic) sits beside about 10 KB of static
+    // shared memory: raise the dynamic limit to the bitmap of the largest
+    // vocabulary taken (the attribute is per device: set on every call)
+    if (cudaFuncSetAttribute(accept_sample_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)(sizeof(unsigned) * (SAMPLE_MAX_VOCAB / 32))) != cudaSuccess)
+        return false;
     const float scale = (float)(1.4426950408889634 * (double)inv_temp);     // log2(e) / T
-    launch_pdl(sample_stats_kernel, B * N, STATS_THREADS, 0, s, logits, V, scale, row_max, row_sum);
+    if (launch_pdl(sample_stats_kernel, B * N, STATS_THREADS, 0, s, logits, V, scale, row_max, row_sum) !=
+        cudaSuccess)
+        return false;
     note_launch();
     const size_t smem = sizeof(unsigned) * (size_t)((V + 31) / 32);
-    launch_pdl(accept_sample_kernel, B, SAMPLE_THREADS, smem, s, t, logits, (const float *)row_max,
-               (const double *)row_sum, N, D, k, V, scale, u, seq_len, n_pend, root, pend_next, acc_path,
-               acc_L0, acc_a, path_out, accept_len_out, bonus_out, index_map_out, status);
+    if (launch_pdl(accept_sample_kernel, B, SAMPLE_THREADS, smem, s, t, logits, (const float *)row_max,
+                   (const double *)row_sum, N, D, k, V, scale, u, seq_len, n_pend, root, pend_next, acc_path,
+                   acc_L0, acc_a, path_out, accept_len_out, bonus_out, index_map_out, status) != cudaSuccess)
+        return false;
     note_launch();
+    return true;
 }
 
 void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, const int *acc_L0,

@@ -60,6 +60,12 @@ void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand
 void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, int B, int N,
                          int V, RowDesc *rows, int *src, uint64_t *vmask, int *status,
                          cudaStream_t s);
+// Depths and ancestor-or-self masks of caller-planted trees from their parent
+// arrays, for requests b0 .. b0+nb-1 (n_nodes[b] nodes of request b; nodes
+// past it get depth 0 and an empty mask). A parent that does not precede its
+// node sets ST_BAD_TREE.
+void launch_tree_complete(const int *parent, int *depth, uint64_t *mask, const int *n_nodes, int b0, int nb,
+                          int N, int *status, cudaStream_t s);
 // A tree of each request's root alone (plain greedy decoding): node 0 = root,
 // parent -1, depth 0, mask = itself, n_nodes = 1; nodes 1.. are not part of it.
 void launch_root_tree(const int *root, int B, int N, int W, int *tokens, int *parent, int *depth,
@@ -73,8 +79,11 @@ void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int 
 // draft's top-k candidates as point-mass proposals): logits [B][N][V] fp32 of
 // the verify pass, inv_temp = 1/T, u [B][D+1][k+1] uniforms in [0, 1);
 // row_max [B*N] and row_sum [B*N] are scratch for the per-row statistics.
-// Same outputs and state update as launch_accept. Two launches.
-void launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, int D, int k, int V,
+// Same outputs and state update as launch_accept. Two launches. Returns
+// false (and launches nothing more) if V > SAMPLE_MAX_VOCAB or a launch
+// failed, so that the caller does not compact on stale acceptance outputs.
+constexpr int SAMPLE_MAX_VOCAB = 48 * 1024 * 8;   // one bit per token in 48 KB of shared memory
+bool launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, int D, int k, int V,
                           float inv_temp, const float *u, float *row_max, double *row_sum, int *seq_len,
                           int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
                           int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,

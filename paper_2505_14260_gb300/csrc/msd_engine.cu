@@ -596,9 +596,12 @@ msd_status accept_sample_impl(msd_ctx *c, const msd_tree *tree, const float *log
                               const float *u, int32_t *path, int32_t *alen, int32_t *bonus,
                               int32_t *imap, cudaStream_t s) {
     TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
-    launch_accept_sample(t, logits, c->B, c->N, c->D, c->k, c->V, (float)(1.0 / (double)temp), u,
-                         c->samp_max, c->samp_sum, c->seq_len, c->n_pend, c->root, c->pend_next, c->acc_path,
-                         c->acc_L0, c->acc_a, path, alen, bonus, imap, c->status, s);
+    if (!launch_accept_sample(t, logits, c->B, c->N, c->D, c->k, c->V, (float)(1.0 / (double)temp), u,
+                              c->samp_max, c->samp_sum, c->seq_len, c->n_pend, c->root, c->pend_next,
+                              c->acc_path, c->acc_L0, c->acc_a, path, alen, bonus, imap, c->status, s)) {
+        const cudaError_t e = cudaGetLastError();
+        return fail(c, MSD_ERR_CUDA, std::string("sampling kernels did not launch: ") + cudaGetErrorString(e));
+    }
     return compact_impl<T>(c, s, -1);
 }
 
@@ -1112,7 +1115,7 @@ msd_status msd_ar_step(msd_ctx *c, int32_t *token_dev, void *stream) {
 // finite fp32 reciprocal.
 // The sampling kernel keeps a bitmap of the rejected tokens in shared memory
 // (one bit per token, within the default 48 KB of dynamic shared memory).
-constexpr int MSD_SAMPLE_MAX_VOCAB = 48 * 1024 * 8;
+constexpr int MSD_SAMPLE_MAX_VOCAB = SAMPLE_MAX_VOCAB;
 
 static bool temperature_ok(float t) {
     return std::isfinite(t) && t > 0.f && std::isfinite((float)(1.0 / (double)t));
@@ -1183,16 +1186,7 @@ msd_status msd_linear(msd_ctx *c, const void *x, int32_t ldx, int32_t m, int32_t
         const size_t need = gemm_pack_bytes(W, k);
         if (need > c->pk_scratch_bytes) {
             CU(cudaStreamSynchronize(s));
-            if (c->pk_scratch) MSD_TEARDOWN(cudaFree(c->pk_scratch));
-    for (auto &g : c->graphs)
-        if (g.exec) MSD_TEARDOWN(cudaGraphExecDestroy(g.exec));
-    if (c->cap_stream) {
-        const cudaError_t e = cudaStreamDestroy(c->cap_stream);
-        if (e != cudaSuccess)
-            fprintf(stderr, "msd_destroy: ctx %p: cudaStreamDestroy(%p): %s\n", (void *)c,
-                    (void *)c->cap_stream, cudaGetErrorString(e));
-    }
-    report_stale_error("msd_destroy (end)");
+            if (c->pk_scratch) CU(cudaFree(c->pk_scratch));
             c->pk_scratch = nullptr;
             c->pk_scratch_bytes = 0;
             if (cudaMalloc(&c->pk_scratch, need) != cudaSuccess)
@@ -1225,6 +1219,32 @@ msd_status msd_profile_read(msd_ctx *c, msd_profile *out) {
         out->gemm_weight_bytes = g.weight_bytes;
     }
     return MSD_OK;
+}
+
+msd_status msd_tree_complete(msd_ctx *c, const msd_tree *tree, int32_t request, void *stream) {
+    if (!c) return MSD_ERR_INVALID;
+    c->err.clear();
+    if (report_stale_error("msd_tree_complete"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
+    msd_status st = check_status(c);
+    if (st != MSD_OK) return st;
+    if (!tree_ok(tree)) return fail(c, MSD_ERR_INVALID, "null tree array");
+    if (request < -1 || request >= c->B) return fail(c, MSD_ERR_INVALID, "request out of range");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    const int b0 = request < 0 ? 0 : request, nb = request < 0 ? c->B : 1;
+    launch_tree_complete(tree->parent, tree->depth, tree->mask, tree->n_nodes, b0, nb, c->N, c->status, s);
+    return post_status(c, s);
+}
+
+msd_status msd_test_wait_timeout(msd_ctx *c, int64_t limit_ns, void *stream) {
+    if (limit_ns < 1000 || limit_ns > 2000000000LL) return fail(c, MSD_ERR_INVALID, "limit out of range");
+    if (report_stale_error("msd_test_wait_timeout"))
+        return fail(c, MSD_ERR_CUDA, "a CUDA error was pending before the call");
+    cudaStream_t s = static_cast<cudaStream_t>(stream);
+    int *status = c ? c->status : noalloc_status_word();
+    if (!status) return MSD_ERR_CUDA;
+    if (!launch_wait_probe(status, (long long)limit_ns, s)) return fail(c, MSD_ERR_CUDA, "probe launch failed");
+    return c ? post_status(c, s) : MSD_OK;
 }
 
 msd_status msd_state(msd_ctx *c, msd_state_view *out) {

@@ -81,6 +81,8 @@ _SIGNATURES = {
                              c_void_p, c_int32, c_int32, c_void_p]),
     "msd_linear_noalloc": (c_int32, [c_void_p, c_int32, c_int32, c_int32, c_void_p, c_int32,
                                      c_void_p, c_int32, c_int32, c_void_p]),
+    "msd_tree_complete": (c_int32, [c_void_p, POINTER(msd_tree), c_int32, c_void_p]),
+    "msd_test_wait_timeout": (c_int32, [c_void_p, c_int64, c_void_p]),
     "msd_profile_enable": (c_int32, [c_void_p, c_int32]),
     "msd_profile_read": (c_int32, [c_void_p, POINTER(msd_profile)]),
     "msd_state": (c_int32, [c_void_p, POINTER(msd_state_view)]),
@@ -151,33 +153,18 @@ class Tree:
         return msd_tree(_ptr(self.tokens), _ptr(self.parent), _ptr(self.depth), _ptr(self.mask),
                         _ptr(self.n_nodes))
 
-    def plant(self, b: int, tokens, parent):
-        """Writes a caller-planted tree for request b: node i has token tokens[i]
-        and parent parent[i] (-1 for the root, else < i); depths and ancestor
-        masks are derived (host-side layout work, then one copy per array)."""
+    def set_nodes(self, b: int, tokens, parent):
+        """Writes the tokens and parent links of request b (n <= N nodes, node 0
+        the root; the rest padded). Depths and ancestor masks are derived by the
+        library: Engine.plant (msd_tree_complete)."""
         n = len(tokens)
-        if n < 1 or n > self.N or len(parent) != n or parent[0] != -1:
-            raise ValueError("a tree needs 1..N nodes with node 0 as its root")
-        depth = [0] * n
-        for i in range(1, n):
-            if not 0 <= parent[i] < i:
-                raise ValueError("parent[i] must precede node i")
-            depth[i] = depth[parent[i]] + 1
-        mask = [[0] * self.W for _ in range(self.N)]
-        for i in range(n):
-            j = i
-            while j >= 0:
-                mask[i][j // 64] |= 1 << (j % 64)
-                j = parent[j]
+        if n < 1 or n > self.N or len(parent) != n:
+            raise ValueError("a tree needs 1..N nodes and one parent entry per node")
         pad = self.N - n
         sl = slice(b * self.N, (b + 1) * self.N)
         dev = self.tokens.device
         self.tokens[sl] = torch.tensor(list(tokens) + [0] * pad, dtype=torch.int32, device=dev)
         self.parent[sl] = torch.tensor(list(parent) + [-1] * pad, dtype=torch.int32, device=dev)
-        self.depth[sl] = torch.tensor(depth + [0] * pad, dtype=torch.int32, device=dev)
-        words = [w - (1 << 64) if w >= 1 << 63 else w for row in mask for w in row]
-        self.mask[b * self.N * self.W:(b + 1) * self.N * self.W] = torch.tensor(words, dtype=torch.int64,
-                                                                                device=dev)
         self.n_nodes[b] = n
 
 
@@ -314,6 +301,21 @@ class Engine:
                               w.shape[0], _ptr(y), y.stride(0), int(accumulate), _stream(stream))
         self._check(st, "msd_linear")
         return y
+
+    def plant(self, tree: Tree, b: int, tokens, parent, stream=None):
+        """A caller-planted tree for request b: tokens and parent links are
+        copied, depths and ancestor masks derived on the device
+        (msd_tree_complete; a parent that does not precede its node is reported
+        by the next call as MSD_ERR_DEVICE)."""
+        tree.set_nodes(b, tokens, parent)
+        st = lib().msd_tree_complete(self.ctx, ctypes.byref(tree.c()), int(b), _stream(stream))
+        self._check(st, "msd_tree_complete")
+        return tree
+
+    def test_wait_timeout(self, limit_ns: int, stream=None):
+        """Test hook: a bounded wait that runs out and sets the status word."""
+        st = lib().msd_test_wait_timeout(self.ctx, int(limit_ns), _stream(stream))
+        self._check(st, "msd_test_wait_timeout")
 
     def profile_enable(self, on: bool = True):
         self._check(lib().msd_profile_enable(self.ctx, int(on)), "msd_profile_enable")

@@ -90,6 +90,7 @@ def tree_numpy(tree: msd.Tree, b: int):
     return toks, par, dep, mask.view(np.uint64).reshape(N, tree.W)
 
 
-def plant(tree: msd.Tree, b: int, tokens, parent):
-    """Writes a caller-planted tree for request b (depths and masks derived)."""
-    tree.plant(b, [int(x) for x in tokens], [int(x) for x in parent])
+def plant(eng: msd.Engine, tree: msd.Tree, b: int, tokens, parent):
+    """A caller-planted tree for request b (depths and masks derived by the
+    library, msd_tree_complete)."""
+    eng.plant(tree, b, [int(x) for x in tokens], [int(x) for x in parent])

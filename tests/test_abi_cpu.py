@@ -71,30 +71,22 @@ def test_binding_fails_loudly_without_the_library(tmp_path, monkeypatch):
         msd.lib()
 
 
-def test_tree_plant_builds_depths_and_ancestor_masks():
-    """Tree.plant (caller-planted trees) derives depths and the ancestor-or-self
-    bitmasks of include/msd.h from the parent array: checked against a walk up
-    the parents, across a 64-node word boundary, on CPU tensors."""
-    import numpy as np
+def test_tree_set_nodes_copies_tokens_and_parents_only():
+    """The binding only copies a planted tree's tokens and parent links (and its
+    node count); depths and masks are derived by the library
+    (msd_tree_complete, tested on the GPU)."""
     from paper_2505_14260_gb300 import msd
     N = 70
     t = msd.Tree(2, N, device="cpu")
     n = 66
-    parent = [-1] + [(i - 1) // 2 if i % 5 else i - 1 for i in range(1, n)]
-    t.plant(1, list(range(100, 100 + n)), parent)
-    W = t.W
-    got = t.mask[N * W:2 * N * W].numpy().view(np.uint64).reshape(N, W)
-    for i in range(N):
-        anc, j = set(), (i if i < n else -1)
-        while j >= 0:
-            anc.add(j)
-            j = parent[j]
-        bits = {w * 64 + k for w in range(W) for k in range(64) if (int(got[i, w]) >> k) & 1}
-        assert bits == anc, i
-    depth = t.depth[N:2 * N].tolist()
-    for i in range(1, n):
-        assert depth[i] == depth[parent[i]] + 1
-    assert t.tokens[N:2 * N].tolist()[:n] == list(range(100, 100 + n)) and int(t.n_nodes[1]) == n
+    parent = [-1] + [(i - 1) // 2 for i in range(1, n)]
+    t.set_nodes(1, list(range(100, 100 + n)), parent)
+    assert t.tokens[N:2 * N].tolist() == list(range(100, 100 + n)) + [0] * (N - n)
+    assert t.parent[N:2 * N].tolist() == parent + [-1] * (N - n)
+    assert int(t.n_nodes[1]) == n and int(t.n_nodes[0]) == N
     assert t.parent[:N].tolist() == [-1] * N              # request 0 untouched
+    assert not t.depth.any() and not t.mask.any()         # left to the library
     with pytest.raises(ValueError):
-        t.plant(0, [1, 2], [-1, 1])                         # a parent must precede its child
+        t.set_nodes(0, [1, 2], [-1])                      # one parent entry per node
+    with pytest.raises(ValueError):
+        t.set_nodes(0, list(range(N + 1)), [-1] * (N + 1))

@@ -25,7 +25,7 @@ def _planted_greedy(eng, n):
     out = [int(eng.state()["root"].cpu()[0])]
     t = msd.Tree(1, eng.cfg.tree_nodes)
     for _ in range(n - 1):
-        plant(t, 0, [out[-1]], [-1])
+        plant(eng, t, 0, [out[-1]], [-1])
         eng.verify(tree=t)
         eng.accept_compact(tree=t)
         out.append(int(eng.bonus.cpu()[0]))

@@ -6,6 +6,9 @@ the prompts msd_prefill must refuse before any launch."""
 import pytest
 import torch
 
+import numpy as np
+
+from oracle import msd_oracle as O
 from paper_2505_14260_gb300 import msd, synth
 from tests.gpu_support import open_engine
 from tests.parity_support import run_parity
@@ -69,3 +72,55 @@ def test_prefill_refuses_invalid_prompts():
         small.prefill(long_ids, [expect_small], None, [0])
     assert e.value.status == msd.MSD_ERR_CAPACITY                        # no room for a step
     small.close()
+
+
+def _depth(par, i):
+    d, j = 0, par[i]
+    while j >= 0:
+        d, j = d + 1, par[j]
+    return d
+
+
+def test_tree_complete_derives_depths_and_ancestor_masks():
+    """msd_tree_complete (the binding's Engine.plant) derives the depths and the
+    ancestor-or-self bitmasks of caller-planted trees on the device: compared
+    with the oracle's Tree (a walk of the parent links) for two requests, one
+    across a 64-node word boundary, the other a chain; a parent that does not
+    precede its node is reported by the next call."""
+    wl = synth.WORKLOADS["tiny"].with_(batch=2, tree_nodes=70, tree_depth=6, topk=16, steps=1)
+    eng, _ = open_engine(wl)
+    t = msd.Tree(2, 70)
+    trees = {0: [-1] + [(i - 1) // 2 if i % 5 else i - 1 for i in range(1, 66)],
+             1: list(range(-1, 69))}
+    for b, par in trees.items():
+        eng.plant(t, b, [3] * len(par), par)
+    torch.cuda.synchronize()
+    W = t.W
+    mask = t.mask.cpu().numpy().view(np.uint64).reshape(2, 70, W)
+    depth = t.depth.cpu().numpy().reshape(2, 70)
+    for b, par in trees.items():
+        n = len(par)
+        ref = O.Tree(tokens=np.zeros(n, np.int64), parent=np.array(par), depth=np.zeros(n, np.int64))
+        np.testing.assert_array_equal(mask[b, :n], ref.mask_words())
+        assert not mask[b, n:].any()
+        np.testing.assert_array_equal(depth[b, :n], [_depth(par, i) for i in range(n)])
+    eng.plant(t, 0, [3, 4, 5], [-1, 2, 0])          # node 1's parent follows it
+    torch.cuda.synchronize()
+    with pytest.raises(msd.MsdError) as e:
+        eng.plant(t, 0, [3], [-1])
+    assert e.value.status == msd.MSD_ERR_DEVICE
+    eng.close()
+
+
+def test_bounded_wait_that_runs_out_is_reported():
+    """Failure detection without a fault: the library's bounded mbarrier wait,
+    given a 1 ms limit on a barrier that nothing arrives at, gives up and sets
+    the context's status word; the next call reports MSD_ERR_DEVICE."""
+    wl = synth.WORKLOADS["tiny"].with_(dtype="bf16", steps=1)
+    eng, _ = open_engine(wl)
+    eng.test_wait_timeout(1_000_000)
+    torch.cuda.synchronize()
+    with pytest.raises(msd.MsdError) as e:
+        eng.draft_tree()
+    assert e.value.status == msd.MSD_ERR_DEVICE
+    eng.close()

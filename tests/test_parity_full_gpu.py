@@ -62,7 +62,7 @@ def test_llava7b_full_depth_lossless_chain():
     ar_logits = []
     for _ in range(n_ar - 1):
         eng.draft_tree()
-        plant(t, 0, [ar[-1]], [-1])
+        plant(eng, t, 0, [ar[-1]], [-1])
         eng.verify(tree=t, logits=logits)
         eng.accept_compact(tree=t)
         ar_logits.append(logits[0].cpu().numpy().copy())
@@ -78,7 +78,7 @@ def test_llava7b_full_depth_lossless_chain():
         j = len(emitted) - 1
         chain = [emitted[-1]] + ar[j + 1:j + 1 + D]
         eng.draft_tree()
-        plant(t, 0, chain, list(range(-1, D)))
+        plant(eng, t, 0, chain, list(range(-1, D)))
         eng.verify(tree=t, logits=logits)
         eng.accept_compact(tree=t)
         g = logits[:D + 1].cpu().numpy()

@@ -57,7 +57,7 @@ def _gpu_greedy_ar(eng, n_tokens):
     t = msd.Tree(1, eng.cfg.tree_nodes)
     for _ in range(n_tokens - 1):
         eng.draft_tree()            # keeps the draft cache caught up
-        plant(t, 0, [out[-1]], [-1])
+        plant(eng, t, 0, [out[-1]], [-1])
         eng.verify(tree=t)
         eng.accept_compact(tree=t)
         out.append(int(eng.bonus.cpu()[0]))
@@ -101,7 +101,7 @@ def test_lossless_planted_trees_match_greedy(dtype):
             if cand != ar[j + 1] and cand not in toks[1:]:
                 parent.append(0); toks.append(cand)
         eng.draft_tree()
-        plant(t, 0, toks, parent)
+        plant(eng, t, 0, toks, parent)
         eng.verify(tree=t)
         eng.accept_compact(tree=t)
         a = int(eng.accept_len.cpu()[0])
@@ -176,7 +176,7 @@ def test_bad_planted_tree_sets_device_status():
     eng.prefill(ids, lens, vis, offs)
     t = msd.Tree(1, wl.tree_nodes)
     root = int(eng.root_out.cpu()[0])
-    plant(t, 0, [(root + 1) % wl.vocab], [-1])
+    plant(eng, t, 0, [(root + 1) % wl.vocab], [-1])
     eng.verify(tree=t)
     torch.cuda.synchronize()
     with pytest.raises(msd.MsdError) as e:

@@ -56,10 +56,10 @@ def spine_tree(eng, logits, wl, b, width):
     roots = eng.state()["root"].cpu().numpy()
     t = msd.Tree(wl.batch, N)
     for r in range(wl.batch):
-        plant(t, r, [int(roots[r])], [-1])
+        plant(eng, t, r, [int(roots[r])], [-1])
     toks, par, head = [int(roots[b])], [-1], 0
     for _ in range(D):
-        plant(t, b, toks, par)
+        plant(eng, t, b, toks, par)
         eng.verify(tree=t, logits=logits)
         row = logits[b * N + head].cpu().numpy()
         top = O.topk_ids(row, width)
@@ -67,7 +67,7 @@ def spine_tree(eng, logits, wl, b, width):
         toks += [int(x) for x in top]
         par += [head] * width
         head = first
-    plant(t, b, toks, par)
+    plant(eng, t, b, toks, par)
     return t
 
 
@@ -239,7 +239,7 @@ def test_sample_argument_errors():
     eng.draft_tree()
     root = int(eng.state()["root"].cpu()[0])
     t = msd.Tree(1, N)
-    plant(t, 0, [root] + list(range(k + 1)), [-1] + [0] * (k + 1))     # k + 1 children
+    plant(eng, t, 0, [root] + list(range(k + 1)), [-1] + [0] * (k + 1))     # k + 1 children
     eng.verify(tree=t)
     eng.accept_sample(1.0, u, tree=t)
     torch.cuda.synchronize()

@@ -6,12 +6,14 @@ allocation would synchronise the device or is not permitted, or a plug-in that
 is handed buffers but no allocator. Its split-K scratch is a static device
 array inside the library instead of context memory.
 
-The test calls it through the C ABI twice in a row (the array keeps the last
+The tests call it through the C ABI twice in a row (the array keeps the last
 call's contents, so the second call must not be disturbed by the first) and
-compares each result with the context entry point msd_linear on the same
-inputs, within the GEMM tolerance used by the other GPU tests. It also checks
-that a shape whose scratch would not fit the array is refused. It runs last in
-the suite and also passes on its own in a fresh process.
+compare each result with the context entry point msd_linear on the same inputs
+and with the fp32 product x.float() @ w.float().T, within the GEMM tolerance
+used by the other GPU tests. A shape whose best split would not fit the array
+runs with fewer splits and still matches; a bounded wait that runs out is
+reported by the next call. The file runs last in the suite and also passes on
+its own in a fresh process.
 """
 import ctypes
 
@@ -31,6 +33,12 @@ def _noalloc(x, w, y, accumulate=False):
                                         int(accumulate), ctypes.c_void_p(stream))
 
 
+def _close(y, ref, tol=1e-4):
+    scale = max(1.0, ref.abs().max().item())
+    err = (y - ref).abs().max().item()
+    return err <= tol * scale, err
+
+
 def test_noalloc_linear_matches_context_linear_on_two_calls():
     build.build()
     wl = synth.WORKLOADS["tiny"].with_(dtype="bf16")
@@ -46,21 +54,48 @@ def test_noalloc_linear_matches_context_linear_on_two_calls():
             y = torch.full((M, O), float("nan"), device="cuda")
             assert _noalloc(x, w, y) == msd.MSD_OK
             torch.cuda.synchronize()
-            scale = max(1.0, y_ref.abs().max().item())
-            err = (y - y_ref).abs().max().item()
-            assert err <= 1e-4 * scale, (M, K, O, call, err)
+            ok, err = _close(y, y_ref)
+            assert ok, (M, K, O, call, err)
+            ok, err = _close(y, x.float() @ w.float().T)
+            assert ok, (M, K, O, call, "vs fp32 product", err)
         y2 = y.clone()
         assert _noalloc(xs[-1], w, y2, accumulate=True) == msd.MSD_OK
         torch.cuda.synchronize()
-        assert (y2 - 2 * y_ref).abs().max().item() <= 2e-4 * scale
+        assert _close(y2, 2 * y_ref, 2e-4)[0]
     eng.close()
 
 
-def test_noalloc_linear_refuses_shapes_beyond_its_scratch():
+def test_noalloc_linear_splits_within_its_scratch():
+    """A product whose best split-K would need more partials than the 16 MiB
+    array runs with fewer splits instead of being refused, and matches the fp32
+    product; bad strides are still refused."""
     build.build()
-    M, K, O = 256, 8192, 2048       # 9-way split-K partials of 18 MiB > the 16 MiB array
-    x = torch.zeros(M, K, device="cuda", dtype=torch.bfloat16)
-    w = torch.zeros(O, K, device="cuda", dtype=torch.bfloat16)
-    y = torch.zeros(M, O, device="cuda")
-    assert _noalloc(x, w, y) == msd.MSD_ERR_CAPACITY
+    g = torch.Generator(device="cuda").manual_seed(12)
+    M, K, O = 256, 8192, 2048
+    x = torch.randn(M, K, device="cuda", generator=g).to(torch.bfloat16)
+    w = (torch.randn(O, K, device="cuda", generator=g) * 0.02).to(torch.bfloat16)
+    for _ in range(2):
+        y = torch.full((M, O), float("nan"), device="cuda")
+        assert _noalloc(x, w, y) == msd.MSD_OK
+        torch.cuda.synchronize()
+        ok, err = _close(y, x.float() @ w.float().T)
+        assert ok, err
     assert _noalloc(x[:, :12], w[:, :12], y) == msd.MSD_ERR_INVALID   # k not a multiple of 8
+
+
+def test_noalloc_linear_reports_a_bounded_wait_that_ran_out():
+    """The status word in the static array: a bounded wait given a 1 ms limit on
+    a barrier that nothing arrives at records a timeout there; the next call
+    reports MSD_ERR_DEVICE (launching nothing) and clears it, and the call after
+    that computes normally."""
+    build.build()
+    g = torch.Generator(device="cuda").manual_seed(13)
+    x = torch.randn(16, 512, device="cuda", generator=g).to(torch.bfloat16)
+    w = (torch.randn(256, 512, device="cuda", generator=g) * 0.02).to(torch.bfloat16)
+    y = torch.zeros(16, 256, device="cuda")
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    assert msd.lib().msd_test_wait_timeout(None, 1_000_000, stream) == msd.MSD_OK
+    assert _noalloc(x, w, y) == msd.MSD_ERR_DEVICE
+    assert _noalloc(x, w, y) == msd.MSD_OK
+    torch.cuda.synchronize()
+    assert _close(y, x.float() @ w.float().T)[0]
