@@ -121,11 +121,17 @@ typedef struct {
  *   draft_kv   [2][B][n_heads][max_seq][head_dim]
  *   seq_len    int32 [B]  L of each request
  *   n_pending  int32 [B]  draft rows still to be caught up (draft cache = L - n_pending)
- *   root       int32 [B]  current root token x_L                                  */
+ *   root       int32 [B]  current root token x_L
+ * bf16 contexts keep every cache entry (and every activation that enters a
+ * tensor-core product) as a pair of bf16 values hi + lo with hi = bf16(v) and
+ * lo = bf16(v - hi), which carries v to about 2^-17 relative: the lo value of
+ * the element at p sits lo_offset elements after it (lo_offset = 0 for fp32
+ * contexts, whose caches hold the fp32 values).                               */
 typedef struct {
     void *target_kv, *draft_kv;
     int32_t *seq_len, *n_pending, *root;
     int64_t elem_bytes;
+    int64_t lo_offset;
 } msd_state_view;
 
 /* Creates a context on the current device: validates the configuration,

@@ -1,23 +1,38 @@
-// Tree-masked attention on the tensor cores for the bf16 path.
+// Tree-masked attention on the 5th-generation tensor cores (bf16 contexts).
 //
-// A CTA (8 warps) takes 64 query rows of one request and one head: warps g and
-// g + 4 own rows 16g .. 16g + 15, and split every key tile between them (keys
-// 0-31 and 32-63), each with its own online-softmax state; the two halves merge
-// once, after the CTA's last tile. Keys come in tiles of 64, staged by TMA (two
-// 64x64 boxes per tile for head_dim 128, 128-byte swizzle) into a ring of
-// shared-memory stages completed on mbarriers. Per tile and warp: S = Q K^T
-// over its 32 keys with mma.sync m16n8k16 (bf16, fp32 accumulate), masking, an
-// online softmax in base 2 (row max and sum across the 4 lanes of a quad with
-// shuffles), and O += P V (P re-packed from the S accumulators as the A
-// operand, V read with ldmatrix.trans).
+// Every operand is a split bf16 pair (hi + lo, common.cuh), so both products
+// run as three tcgen05.mma each into one fp32 accumulator in tensor memory:
+//   S = Q K^T  as  Qh Kh + Ql Kh + Qh Kl
+//   O += P V   as  Ph Vh + Pl Vh + Ph Vl
+// (the dropped lo*lo terms are 2^-18 of the product), which keeps the
+// attention as precise as an fp32 evaluation.
+//
+// A CTA takes 64 query rows of one request and one head (the MMA's M = 64)
+// and one range of keys (a split). Roles (320 threads):
+//   warp 0 lane 0   TMA: K and V tiles of 64 keys (hi and lo planes, 128-byte
+//                   swizzle) into a three-stage shared-memory ring
+//   warp 1          allocates tensor memory; lane 0 issues the MMAs
+//   warps 2-9       two per TMEM lane quarter (an M = 64 accumulator keeps
+//                   rows 16q .. 16q+15 in lanes 0-15 of quarter q), each
+//                   taking half of a tile's keys and of O's columns: load the
+//                   query rows into TMEM, then per key tile read S, mask it
+//                   (prefix length, tree bitmask), run the online softmax in
+//                   base 2 and write P (hi, lo) back over S as the A operand
+//                   of the P V product
+// Q and P are A operands read from tensor memory (P of a tile's keys 32h ..
+// 32h+31 written over those keys' S columns, hi pairs then lo pairs, by the
+// warps that read them), so shared memory holds only the K/V ring; S is
+// double-buffered so the Q K^T of tile j+1 overlaps the softmax of tile j. O stays in TMEM; a row's running maximum is moved (and O
+// and the row sum rescaled) only when a tile's maximum exceeds it by more than
+// 2^8, so P <= 256.
 //
 // Visible keys of a row (Sec. 3.2: a candidate is conditioned on its prefix
 // only): cache positions [0, plen) of its request, and tree slots whose bit is
-// set in its mask. The cache range is split across CTAs (z < nsplit_cache);
-// the tree part is one more split. With more than one split, every CTA writes
-// unnormalised partials (O, running max, running sum) to a workspace and the
-// last CTA of a (row tile, head) combines them in split order (deterministic),
-// then resets its ticket. All mbarrier waits are bounded.
+// set in its mask. The cache range is cut into splits (a function of the
+// capacity only, so results never depend on L) plus one tree split; the splits
+// of a (row tile, head) form a thread-block cluster and combine their
+// partials (O, max, sum) through distributed shared memory in split order:
+// deterministic. Every mbarrier wait is bounded.
 #include <cuda.h>
 #include <cudaTypedefs.h>
 
@@ -31,25 +46,36 @@ namespace msd {
 
 namespace {
 
-constexpr int ROWS = 64;          // query rows per CTA
-constexpr int KT = 64;            // keys per tile
-constexpr int THREADS = 256;      // 8 warps: 4 row groups x 2 key halves
-// row stride (floats) of the fp32 partials in shared memory: padded so that the
-// 8 rows a warp writes at once fall in different banks
-template <int HD> constexpr int PART_LD = HD + 8;
-constexpr int MAX_STAGES = 3;
-constexpr int CACHE_SPLITS = 8;   // cache splits of a decode launch (capacity-derived chunk)
-constexpr int MAX_SPLITS = CACHE_SPLITS + 1;   // + the tree split = cluster size
+constexpr int ROWS = 64;          // query rows per CTA (MMA M)
+constexpr int KT = 64;            // keys per tile (N of Q K^T, K of P V)
+constexpr int THREADS = 320;      // warp 0 TMA, warp 1 MMA, warps 2-9 softmax
+constexpr int STAGES = 3;
+constexpr int MAX_SPLITS = 9;     // cache splits + the tree split = cluster size
 constexpr unsigned long long ATTN_TIMEOUT_NS = 2000000000ull;
+constexpr float RESCALE_LOG2 = 8.f;
+
+template <int HD>
+struct Lay {
+    static constexpr int NB = HD / 64;                    // 64-column boxes of a row
+    static constexpr uint32_t BOX = KT * 128;             // [64 rows][64 bf16] = 8 KB
+    static constexpr uint32_t TILE = NB * BOX;            // one plane of a K or V tile
+    static constexpr uint32_t STAGE = 4 * TILE;           // K hi, K lo, V hi, V lo
+    // tensor-memory columns: Q hi, Q lo (bf16 pairs), two S/P buffers, O
+    static constexpr uint32_t T_QH = 0, T_QL = HD / 2, T_S = HD, T_O = HD + 2 * KT;
+    static constexpr uint32_t T_COLS = T_O + HD <= 256 ? 256 : 512;
+    static constexpr int LD = HD + 4;                     // fp32 partial row stride (floats)
+};
 
 struct AttnTcParams {
     const bf16 *q;
     const RowDesc *rows;
     const uint64_t *mask;
     bf16 *out;
+    long lo;                  // lo planes of q and out (elements); K/V: lo_rows rows on
+    int lo_rows;
     int *status;
     int R, rows_per_req, tiles_per_req, nh, cache_slots, tree_slots, mask_words;
-    int nsplit_cache, has_tree, chunk, stages;
+    int nsplit_cache, has_tree, chunk;
     int cache_early;          // cache K/V may be requested before the wait (not written by the previous kernel)
     float scale_log2;
 };
@@ -73,16 +99,30 @@ __device__ __forceinline__ bool bar_try(uint32_t bar, uint32_t parity) {
     return ok != 0;
 }
 
-__device__ bool bar_wait(uint32_t bar, uint32_t parity, int *status) {
+// Bounded wait: gives up when *abort is set by another thread, or after the
+// limit (then sets *abort and records ST_TIMEOUT).
+__device__ bool bar_wait(uint32_t bar, uint32_t parity, volatile int *abort, int *status) {
     if (bar_try(bar, parity)) return true;
     const unsigned long long t0 = gtime();
     while (!bar_try(bar, parity)) {
+        if (*abort) return false;
         if (gtime() - t0 > ATTN_TIMEOUT_NS) {
+            *abort = 1;
             set_status(status, ST_TIMEOUT);
             return false;
         }
     }
     return true;
+}
+
+__device__ __forceinline__ void bar_init(uint32_t bar, uint32_t count) {
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
+}
+__device__ __forceinline__ void bar_arrive(uint32_t bar) {
+    asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(bar) : "memory");
+}
+__device__ __forceinline__ void bar_expect_tx(uint32_t bar, uint32_t bytes) {
+    asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
 }
 
 __device__ __forceinline__ void tma2d(uint32_t dst, const CUtensorMap *m, int x, int y, uint32_t bar) {
@@ -93,33 +133,89 @@ __device__ __forceinline__ void tma2d(uint32_t dst, const CUtensorMap *m, int x,
         : "memory");
 }
 
-// Byte address of 16-byte chunk `c` of row `row` in a [64][HD] bf16 tile
-// stored as HD/64 boxes of [64 rows][128 B] with the 128-byte swizzle.
-__device__ __forceinline__ uint32_t swz(uint32_t base, int row, int c) {
-    return base + (c >> 3) * 8192 + row * 128 + (((c & 7) ^ (row & 7)) << 4);
+// Shared-memory matrix descriptor (sm100 version 1, 128-byte swizzle): start
+// address, leading byte offset (MN-major: the stride between 64-element
+// atoms along M/N) and stride byte offset (the stride between 8-row groups).
+__device__ __forceinline__ uint64_t sdesc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+    return (uint64_t)((saddr & 0x3FFFFu) >> 4) | ((uint64_t)((lbo >> 4) & 0x3FFFu) << 16) |
+           ((uint64_t)((sbo >> 4) & 0x3FFFu) << 32) | ((uint64_t)1 << 46) | ((uint64_t)2 << 61);
 }
 
-__device__ __forceinline__ void ldsm4(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
-                                      uint32_t &r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
+// Instruction descriptor, kind::f16: fp32 accumulate, bf16 A and B, A
+// K-major, B K-major (b_mn = 0) or MN-major (1).
+__device__ __forceinline__ uint32_t idesc(int M, int N, int b_mn) {
+    return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)b_mn << 16) | ((uint32_t)(N >> 3) << 17) |
+           ((uint32_t)(M >> 4) << 24);
 }
 
-__device__ __forceinline__ void ldsm4t(uint32_t addr, uint32_t &r0, uint32_t &r1, uint32_t &r2,
-                                       uint32_t &r3) {
-    asm volatile("ldmatrix.sync.aligned.m8n8.x4.trans.shared.b16 {%0,%1,%2,%3}, [%4];"
-                 : "=r"(r0), "=r"(r1), "=r"(r2), "=r"(r3)
-                 : "r"(addr));
-}
-
-__device__ __forceinline__ void mma16816(float (&d)[4], const uint32_t (&a)[4], uint32_t b0,
-                                         uint32_t b1) {
+// D (+)= A B^T with A read from tensor memory and B from shared memory.
+__device__ __forceinline__ void mma_ts(uint32_t d, uint32_t a, uint64_t b, uint32_t id, uint32_t acc) {
     asm volatile(
-        "mma.sync.aligned.m16n8k16.row.col.f32.bf16.bf16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, "
-        "{%8,%9}, {%0,%1,%2,%3};"
-        : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
-        : "r"(a[0]), "r"(a[1]), "r"(a[2]), "r"(a[3]), "r"(b0), "r"(b1));
+        "{\n.reg .pred p;\nsetp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}" ::"r"(d),
+        "r"(a), "l"(b), "r"(id), "r"(acc));
+}
+
+__device__ __forceinline__ void mma_commit(uint32_t bar) {
+    asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
+                 : "memory");
+}
+
+// 32 columns of this warp's lanes, waited for in the same asm statement: the
+// compiler sees the registers defined only once the data has landed.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *r) {
+    asm volatile(
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+          "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+          "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+          "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
+}
+
+
+// Stores of 32 / 16 columns, waited for in the same asm statement, so the
+// source registers are not reused before the tensor memory has taken them.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t *r) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};\n"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15]), "r"(r[16]),
+        "r"(r[17]), "r"(r[18]), "r"(r[19]), "r"(r[20]), "r"(r[21]), "r"(r[22]), "r"(r[23]), "r"(r[24]),
+        "r"(r[25]), "r"(r[26]), "r"(r[27]), "r"(r[28]), "r"(r[29]), "r"(r[30]), "r"(r[31])
+        : "memory");
+}
+
+__device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *r) {
+    asm volatile(
+        "tcgen05.st.sync.aligned.32x32b.x16.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,%16};\n"
+        "tcgen05.wait::st.sync.aligned;" ::"r"(taddr),
+        "r"(r[0]), "r"(r[1]), "r"(r[2]), "r"(r[3]), "r"(r[4]), "r"(r[5]), "r"(r[6]), "r"(r[7]), "r"(r[8]),
+        "r"(r[9]), "r"(r[10]), "r"(r[11]), "r"(r[12]), "r"(r[13]), "r"(r[14]), "r"(r[15])
+        : "memory");
+}
+
+// Barrier of the 256 softmax threads (named barrier 1; the TMA and MMA warps
+// never join it). The warp reconverges first: the barrier's aligned form needs
+// every lane of a warp to reach it together.
+__device__ __forceinline__ void softmax_sync() {
+    __syncwarp();
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    asm volatile("barrier.sync.aligned 1, 256;" ::: "memory");
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+
+// 2^x (the SFU approximation; 2^-inf = 0)
+__device__ __forceinline__ float ex2_fast(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
 }
 
 __device__ __forceinline__ void cluster_sync() {
@@ -132,17 +228,10 @@ __device__ __forceinline__ uint32_t cluster_rank() {
     return r;
 }
 
-// Address of the same shared-memory location in CTA `rank` of the cluster.
 __device__ __forceinline__ uint32_t dsmem_addr(uint32_t local, int rank) {
     uint32_t r;
     asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(r) : "r"(local), "r"(rank));
     return r;
-}
-
-__device__ __forceinline__ float dsmem_ld_f32(uint32_t a) {
-    float v;
-    asm volatile("ld.shared::cluster.f32 %0, [%1];" : "=f"(v) : "r"(a) : "memory");
-    return v;
 }
 
 // (no memory clobber: the partials are read only between two cluster
@@ -161,25 +250,28 @@ __device__ __forceinline__ float4 dsmem_ld_f4(uint32_t a) {
     return v;
 }
 
-__device__ __forceinline__ uint32_t pack_bf16(float lo, float hi) {
-    __nv_bfloat162 v = __floats2bfloat162_rn(lo, hi);
-    return *reinterpret_cast<uint32_t *>(&v);
+// hi and lo bf16 pairs of two fp32 values (element 2c in the low half).
+__device__ __forceinline__ void split_pair(float a, float b, uint32_t &hi, uint32_t &lo) {
+    const __nv_bfloat162 h = __floats2bfloat162_rn(a, b);
+    const __nv_bfloat162 l = __floats2bfloat162_rn(a - __low2float(h), b - __high2float(h));
+    hi = *reinterpret_cast<const uint32_t *>(&h);
+    lo = *reinterpret_cast<const uint32_t *>(&l);
 }
 
 template <int HD>
-__global__ void __launch_bounds__(THREADS, 2)
+__global__ void __launch_bounds__(THREADS, 1)
     attn_tc_kernel(const __grid_constant__ CUtensorMap mkc, const __grid_constant__ CUtensorMap mvc,
                    const __grid_constant__ CUtensorMap mkt, const __grid_constant__ CUtensorMap mvt,
                    const AttnTcParams p) {
-    constexpr int NB = HD / 64;                   // 64-wide boxes per row
-    constexpr int TILE_BYTES = KT * HD * 2;       // one K (or V) tile
-    constexpr int NT_O = HD / 8;                  // O n-tiles per warp
+    using L = Lay<HD>;
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t bars[MAX_STAGES];
+    __shared__ __align__(8) uint64_t bars[2 * STAGES + 8];
+    __shared__ uint32_t tmem_base;
     __shared__ int s_pmax;
+    __shared__ volatile int abort_flag;
+    __shared__ float s_xmax[6 * ROWS];     // tile maxima [tile parity][half][row], then row sums [half][row]
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int grp = warp & 3, half = warp >> 2;     // row group, key half of each tile
     const int tile = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
     const int blk = tile / p.tiles_per_req;
     const int r0 = blk * p.rows_per_req + (tile - blk * p.tiles_per_req) * ROWS;
@@ -188,29 +280,54 @@ __global__ void __launch_bounds__(THREADS, 2)
     const int H = p.nh * HD;
 
     const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
-    const uint32_t q_s = base;                             // [64][HD]
-    const uint32_t kv_s = base + ROWS * HD * 2;            // STAGES x (K tile, V tile)
+    const uint32_t full0 = su32(&bars[0]), empty0 = su32(&bars[STAGES]);
+    const uint32_t s_full0 = su32(&bars[2 * STAGES]), p_full0 = su32(&bars[2 * STAGES + 2]);
+    const uint32_t o_ready = su32(&bars[2 * STAGES + 4]), q_ready = su32(&bars[2 * STAGES + 5]);
+    const uint32_t drain = su32(&bars[2 * STAGES + 6]);
+
+    // softmax threads: warps 2-9 read TMEM lane quarter q = warp & 3, whose
+    // lanes 0-15 hold rows 16q .. 16q+15 of the M = 64 accumulators
+    const bool smx = warp >= 2;
+    const int quarter = warp & 3;
+    const int row_local = 16 * quarter + lane;
+    const int row = r0 + row_local;
+    const bool valid = smx && lane < 16 && row < r_end;
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < p.stages; ++s)
-            asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(&bars[s])), "r"(1));
+        for (int s = 0; s < STAGES; ++s) {
+            bar_init(full0 + 8 * s, 1);
+            bar_init(empty0 + 8 * s, 1);
+        }
+        for (int b = 0; b < 2; ++b) {
+            bar_init(s_full0 + 8 * b, 1);
+            bar_init(p_full0 + 8 * b, 256);
+        }
+        bar_init(o_ready, 1);
+        bar_init(q_ready, 256);
+        bar_init(drain, 1);
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
         s_pmax = 0;
+        abort_flag = 0;
         asm volatile("prefetch.tensormap [%0];" ::"l"(&mkc) : "memory");
         asm volatile("prefetch.tensormap [%0];" ::"l"(&mvc) : "memory");
+    }
+    if (warp == 1) {
+        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(su32(&tmem_base)),
+                     "r"(L::T_COLS)
+                     : "memory");
+        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
     }
     __syncthreads();
     // Before the wait: the row descriptors (written by set-up kernels at least
     // two launches back) and, unless the previous kernel wrote into it, the
     // cache K/V. The previous kernel's q and tree K/V are read after the wait.
     const int req = p.rows[r0].req;
-
-    // Rows of this thread: A = lane/4, B = lane/4 + 8 of the warp's 16.
-    const int ra = r0 + grp * 16 + (lane >> 2), rb = ra + 8;
-    const bool va = ra < r_end, vb = rb < r_end;
-    const int plen_a = va ? p.rows[ra].plen : 0, plen_b = vb ? p.rows[rb].plen : 0;
-    atomicMax(&s_pmax, max(plen_a, plen_b));
+    const int plen = valid ? p.rows[row].plen : 0;
+    if (valid) atomicMax(&s_pmax, plen);
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
+    asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+    const uint32_t tmem = tmem_base;
 
     // Key range of this split.
     int k_lo, k_hi, row_base;
@@ -229,285 +346,284 @@ __global__ void __launch_bounds__(THREADS, 2)
         mv = &mvc;
     }
     const int ntiles = k_hi > k_lo ? (k_hi - k_lo + KT - 1) / KT : 0;
-    const uint32_t stage_bytes = 2 * TILE_BYTES;
 
-    const int stages = p.stages;
     auto issue = [&](int i) {
-        const int s = i % stages;
-        const uint32_t bar = su32(&bars[s]);
-        const uint32_t kd = kv_s + s * stage_bytes, vd = kd + TILE_BYTES;
-        asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar),
-                     "r"(stage_bytes)
-                     : "memory");
+        const int s = i % STAGES;
+        const uint32_t bar = full0 + 8 * s;
+        const uint32_t kd = base + s * L::STAGE;
+        bar_expect_tx(bar, L::STAGE);
         const int y = row_base + k_lo + i * KT;
 #pragma unroll
-        for (int b = 0; b < NB; ++b) {
-            tma2d(kd + b * 8192, mk, b * 64, y, bar);
-            tma2d(vd + b * 8192, mv, b * 64, y, bar);
+        for (int b = 0; b < L::NB; ++b) {
+            tma2d(kd + b * L::BOX, mk, b * 64, y, bar);
+            tma2d(kd + L::TILE + b * L::BOX, mk, b * 64, y + p.lo_rows, bar);
+            tma2d(kd + 2 * L::TILE + b * L::BOX, mv, b * 64, y, bar);
+            tma2d(kd + 3 * L::TILE + b * L::BOX, mv, b * 64, y + p.lo_rows, bar);
         }
     };
-    // K/V tiles in flight first, then the Q tile (all its loads issued before
-    // the first shared-memory store); rows past the request's rows are zero.
     const bool early = !is_tree && p.cache_early;
+    const int n_pre = min(STAGES, ntiles);
     if (threadIdx.x == 0 && early)
-        for (int i = 0; i < min(stages, ntiles); ++i) issue(i);
+        for (int i = 0; i < n_pre; ++i) issue(i);
     wait_prior();
     allow_dependents();
-    if (threadIdx.x == 0 && !early)
-        for (int i = 0; i < min(stages, ntiles); ++i) issue(i);
-    {
-        constexpr int QV = ROWS * HD / 8 / THREADS;   // 16-byte pieces per thread
-        uint4 qv[QV];
-#pragma unroll
-        for (int j = 0; j < QV; ++j) {
-            const int i = threadIdx.x + j * THREADS;
-            const int row = i / (HD / 8), c = i - row * (HD / 8);
-            qv[j] = r0 + row < r_end
-                        ? __ldg(reinterpret_cast<const uint4 *>(p.q + (size_t)(r0 + row) * H + h * HD + c * 8))
-                        : make_uint4(0, 0, 0, 0);
-        }
-#pragma unroll
-        for (int j = 0; j < QV; ++j) {
-            const int i = threadIdx.x + j * THREADS;
-            const int row = i / (HD / 8), c = i - row * (HD / 8);
-            asm volatile("st.shared.v4.b32 [%0], {%1,%2,%3,%4};" ::"r"(swz(q_s, row, c)), "r"(qv[j].x),
-                         "r"(qv[j].y), "r"(qv[j].z), "r"(qv[j].w)
-                         : "memory");
-        }
-    }
-    __syncthreads();
 
-    // Q fragments of the warp's 16 rows are re-read from shared memory per tile
-    // (ldmatrix), which keeps two 8-warp CTAs' registers on an SM.
-    const int q_row = grp * 16 + ((lane >> 3) & 1) * 8 + (lane & 7);
+    // TMEM addresses of this warp's lane quarter
+    const uint32_t tq = tmem + ((uint32_t)(32 * quarter) << 16);
 
-    // Tree-mask words of the two rows (tree split only).
-    const uint64_t *mask_a = (is_tree && va) ? p.mask + (size_t)ra * p.mask_words : nullptr;
-    const uint64_t *mask_b = (is_tree && vb) ? p.mask + (size_t)rb * p.mask_words : nullptr;
-
-    float o[NT_O][4];
-#pragma unroll
-    for (int j = 0; j < NT_O; ++j) o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
-    float m_a = -INFINITY, m_b = -INFINITY, l_a = 0.f, l_b = 0.f;
-    bool ok = true;
-
-    for (int i = 0; i < ntiles; ++i) {
-        const int s = i % stages;
-        if (!bar_wait(su32(&bars[s]), (uint32_t)(i / stages) & 1u, p.status)) ok = false;
-        const uint32_t ks = kv_s + s * stage_bytes, vs = ks + TILE_BYTES;
-        const int key0 = k_lo + i * KT;
-
-        // this warp's 32 keys of the tile: kh .. kh + 31
-        const int kh = half * 32;
-        float sc[4][4];
-#pragma unroll
-        for (int j = 0; j < 4; ++j) sc[j][0] = sc[j][1] = sc[j][2] = sc[j][3] = 0.f;
-#pragma unroll
-        for (int kk = 0; kk < HD / 16; ++kk) {
-            uint32_t qf[4];
-            ldsm4(swz(q_s, q_row, 2 * kk + (lane >> 4)), qf[0], qf[1], qf[2], qf[3]);
-#pragma unroll
-            for (int np = 0; np < 2; ++np) {
-                const int m = lane >> 3;
-                const int key = kh + np * 16 + (m >> 1) * 8 + (lane & 7);
-                uint32_t b0, b1, b2, b3;
-                ldsm4(swz(ks, key, 2 * kk + (m & 1)), b0, b1, b2, b3);
-                mma16816(sc[2 * np], qf, b0, b1);
-                mma16816(sc[2 * np + 1], qf, b2, b3);
+    if (warp == 0) {
+        // ---- producer ------------------------------------------------------
+        if (lane == 0) {
+            if (!early)
+                for (int i = 0; i < n_pre; ++i) issue(i);
+            int i = n_pre;
+            for (; i < ntiles; ++i) {
+                const int s = i % STAGES;
+                if (!bar_wait(empty0 + 8 * s, (uint32_t)(i / STAGES - 1) & 1u, &abort_flag, p.status)) break;
+                issue(i);
+            }
+            if (abort_flag) {       // the copies still in flight land before the CTA exits
+                volatile int never = 0;
+                for (int j = (i > STAGES ? i - STAGES : 0); j < i; ++j)
+                    bar_wait(full0 + 8 * (j % STAGES), (uint32_t)(j / STAGES) & 1u, &never, p.status);
             }
         }
-        // mask + scale (base-2 logits)
-        uint64_t wa = 0, wb = 0;
-        if (is_tree) {
-            const int w = key0 >> 6;
-            if (mask_a && w < p.mask_words) wa = mask_a[w];
-            if (mask_b && w < p.mask_words) wb = mask_b[w];
-        }
-        float mx_a = -INFINITY, mx_b = -INFINITY;
+        __syncwarp();
+    } else if (warp == 1) {
+        // ---- MMA issue -----------------------------------------------------
+        if (lane == 0 && ntiles > 0) {
+            const uint32_t id_qk = idesc(ROWS, KT, 0), id_pv = idesc(ROWS, HD, 1);
+            auto qk = [&](int t) -> bool {
+                const int s = t % STAGES;
+                if (!bar_wait(full0 + 8 * s, (uint32_t)(t / STAGES) & 1u, &abort_flag, p.status)) return false;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t kd = base + s * L::STAGE;
+                const uint32_t sd = tmem + L::T_S + (t & 1) * KT;
 #pragma unroll
-        for (int j = 0; j < 4; ++j) {
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-                const int kl = kh + 8 * j + 2 * (lane & 3) + (e & 1);
-                const int key = key0 + kl;
-                bool vis;
-                if (is_tree) {
-                    const uint64_t wd = e < 2 ? wa : wb;
-                    vis = key < k_hi && ((wd >> (key & 63)) & 1ull);
-                } else {
-                    vis = key < k_hi && key < (e < 2 ? plen_a : plen_b);
+                for (int kk = 0; kk < HD / 16; ++kk) {
+                    const uint32_t ko = (kk >> 2) * L::BOX + (kk & 3) * 32;
+                    const uint64_t kh = sdesc(kd + ko, 16, 1024), kl = sdesc(kd + L::TILE + ko, 16, 1024);
+                    mma_ts(sd, tmem + L::T_QH + kk * 8, kh, id_qk, kk > 0);
+                    mma_ts(sd, tmem + L::T_QL + kk * 8, kh, id_qk, 1u);
+                    mma_ts(sd, tmem + L::T_QH + kk * 8, kl, id_qk, 1u);
                 }
-                const float v = vis ? sc[j][e] * p.scale_log2 : -INFINITY;
-                sc[j][e] = v;
-                if (e < 2) mx_a = fmaxf(mx_a, v); else mx_b = fmaxf(mx_b, v);
+                mma_commit(s_full0 + 8 * (t & 1));
+                return true;
+            };
+            bool ok = bar_wait(q_ready, 0, &abort_flag, p.status);
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            if (ok) ok = qk(0);
+            if (ok && ntiles > 1) ok = qk(1);
+            for (int j = 0; ok && j < ntiles; ++j) {
+                if (!bar_wait(p_full0 + 8 * (j & 1), (uint32_t)(j >> 1) & 1u, &abort_flag, p.status)) break;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const uint32_t vd = base + (j % STAGES) * L::STAGE + 2 * L::TILE;
+                // P of keys 32h .. 32h+31 sits in S columns 32h .. 32h+31: hi pairs
+                // in the first 16, lo pairs in the next 16
+                const uint32_t pd = tmem + L::T_S + (j & 1) * KT;
+#pragma unroll
+                for (int kk = 0; kk < KT / 16; ++kk) {
+                    const uint32_t ph = pd + (kk >> 1) * 32 + (kk & 1) * 8, pl = ph + 16;
+                    const uint64_t vh = sdesc(vd + kk * 2048, L::BOX, 1024);
+                    const uint64_t vl = sdesc(vd + L::TILE + kk * 2048, L::BOX, 1024);
+                    mma_ts(tmem + L::T_O, ph, vh, id_pv, (j > 0) || (kk > 0));
+                    mma_ts(tmem + L::T_O, pl, vh, id_pv, 1u);
+                    mma_ts(tmem + L::T_O, ph, vl, id_pv, 1u);
+                }
+                mma_commit(empty0 + 8 * (j % STAGES));
+                mma_commit(o_ready);
+                if (j + 2 < ntiles) ok = qk(j + 2);
             }
+            // no MMA outlives the CTA's tensor memory
+            mma_commit(drain);
+            volatile int never = 0;
+            bar_wait(drain, 0, &never, p.status);
         }
-        mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 1));
-        mx_a = fmaxf(mx_a, __shfl_xor_sync(0xffffffffu, mx_a, 2));
-        mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 1));
-        mx_b = fmaxf(mx_b, __shfl_xor_sync(0xffffffffu, mx_b, 2));
-        const float mn_a = fmaxf(m_a, mx_a), mn_b = fmaxf(m_b, mx_b);
-        const float use_a = mn_a == -INFINITY ? 0.f : mn_a, use_b = mn_b == -INFINITY ? 0.f : mn_b;
-        const float cf_a = exp2f(m_a - use_a), cf_b = exp2f(m_b - use_b);
-        m_a = mn_a;
-        m_b = mn_b;
-        float rs_a = 0.f, rs_b = 0.f;
-#pragma unroll
-        for (int j = 0; j < 4; ++j) {
-            sc[j][0] = exp2f(sc[j][0] - use_a);
-            sc[j][1] = exp2f(sc[j][1] - use_a);
-            sc[j][2] = exp2f(sc[j][2] - use_b);
-            sc[j][3] = exp2f(sc[j][3] - use_b);
-            rs_a += sc[j][0] + sc[j][1];
-            rs_b += sc[j][2] + sc[j][3];
-        }
-        l_a = l_a * cf_a + rs_a;
-        l_b = l_b * cf_b + rs_b;
-#pragma unroll
-        for (int j = 0; j < NT_O; ++j) {
-            o[j][0] *= cf_a; o[j][1] *= cf_a;
-            o[j][2] *= cf_b; o[j][3] *= cf_b;
-        }
-        // O += P V over the warp's 32 keys
-#pragma unroll
-        for (int kk = 0; kk < 2; ++kk) {
-            uint32_t pa[4];
-            pa[0] = pack_bf16(sc[2 * kk][0], sc[2 * kk][1]);
-            pa[1] = pack_bf16(sc[2 * kk][2], sc[2 * kk][3]);
-            pa[2] = pack_bf16(sc[2 * kk + 1][0], sc[2 * kk + 1][1]);
-            pa[3] = pack_bf16(sc[2 * kk + 1][2], sc[2 * kk + 1][3]);
-#pragma unroll
-            for (int dp = 0; dp < HD / 16; ++dp) {
-                const int m = lane >> 3;
-                const int key = kh + kk * 16 + (m & 1) * 8 + (lane & 7);
-                uint32_t b0, b1, b2, b3;
-                ldsm4t(swz(vs, key, 2 * dp + (m >> 1)), b0, b1, b2, b3);
-                mma16816(o[2 * dp], pa, b0, b1);
-                mma16816(o[2 * dp + 1], pa, b2, b3);
-            }
-        }
-        __syncthreads();                              // every warp is done with stage s
-        if (threadIdx.x == 0 && i + stages < ntiles) issue(i + stages);
+        __syncwarp();
     }
 
-    l_a += __shfl_xor_sync(0xffffffffu, l_a, 1);
-    l_a += __shfl_xor_sync(0xffffffffu, l_a, 2);
-    l_b += __shfl_xor_sync(0xffffffffu, l_b, 1);
-    l_b += __shfl_xor_sync(0xffffffffu, l_b, 2);
-
-    // Merge the two key halves of each row group: the upper warps leave (O, m,
-    // l) in shared memory (the K/V stages are idle now), the lower warps fold
-    // them into theirs; the result is left in the same place for the cluster
-    // combine below.
-    const int col0 = 2 * (lane & 3);
-    __syncthreads();
-    constexpr int LD = PART_LD<HD>;
-    float *s_o = reinterpret_cast<float *>(smem_raw + (kv_s - su32(smem_raw)));   // [64][LD]
-    float *s_ml = s_o + ROWS * LD;                                               // [64][2]
-    const int la = grp * 16 + (lane >> 2), lb = la + 8;
-    if (half == 1) {
+    // ---- softmax warps ----------------------------------------------------
+    // Two warps share each TMEM lane quarter and take half of every tile's keys
+    // (half 0: keys 0-31, half 1: keys 32-63) and half of O's columns; the two
+    // halves of a row exchange their tile maxima through shared memory, so both
+    // keep the same reference maximum. A failed (timed-out) wait makes a warp
+    // skip the work of the remaining tiles but not the CTA barriers, so the
+    // warps stay in step.
+    auto wwait = [&](uint32_t bar, uint32_t parity) {
+        const bool r = bar_wait(bar, parity, &abort_flag, p.status);
+        return __all_sync(0xffffffffu, r);
+    };
+    const int hf = (warp - 2) >> 2;                   // column half of a softmax warp
+    constexpr int OH = HD / 2;                        // O columns per half
+    uint32_t o_acc[OH];                               // this half of the row's O (fp32 bits)
+    float m_used = -INFINITY, l_sum = 0.f;
+    bool dead = false;
+    if (smx) {
+        // query row (hi, lo) into tensor memory, the A operand of Q K^T: this
+        // half's HD/4 bf16 pairs of each plane
+        {
+            const uint4 *qh = reinterpret_cast<const uint4 *>(p.q + (size_t)row * H + h * HD);
+            const uint4 *ql = reinterpret_cast<const uint4 *>(p.q + p.lo + (size_t)row * H + h * HD);
+            uint32_t rh[HD / 4], rl[HD / 4];
 #pragma unroll
-        for (int j = 0; j < NT_O; ++j) {
-            const int c = 8 * j + col0;
-            *reinterpret_cast<float2 *>(s_o + la * LD + c) = make_float2(o[j][0], o[j][1]);
-            *reinterpret_cast<float2 *>(s_o + lb * LD + c) = make_float2(o[j][2], o[j][3]);
-        }
-        if ((lane & 3) == 0) {
-            *reinterpret_cast<float2 *>(s_ml + la * 2) = make_float2(m_a, l_a);
-            *reinterpret_cast<float2 *>(s_ml + lb * 2) = make_float2(m_b, l_b);
-        }
-    }
-    __syncthreads();
-    if (half == 0) {
-        const float2 ua = *reinterpret_cast<const float2 *>(s_ml + la * 2);
-        const float2 ub = *reinterpret_cast<const float2 *>(s_ml + lb * 2);
-        const float Ma = fmaxf(m_a, ua.x), Mb = fmaxf(m_b, ub.x);
-        const float ba = Ma == -INFINITY ? 0.f : Ma, bb = Mb == -INFINITY ? 0.f : Mb;
-        const float c0a = exp2f(m_a - ba), c1a = exp2f(ua.x - ba);
-        const float c0b = exp2f(m_b - bb), c1b = exp2f(ub.x - bb);
+            for (int u = 0; u < HD / 16; ++u) {
+                const int g = hf * (HD / 16) + u;            // uint4 index in the row
+                const uint4 a4 = valid ? qh[g] : make_uint4(0, 0, 0, 0);
+                const uint4 b4 = valid && p.lo ? ql[g] : make_uint4(0, 0, 0, 0);
+                rh[4 * u] = a4.x; rh[4 * u + 1] = a4.y; rh[4 * u + 2] = a4.z; rh[4 * u + 3] = a4.w;
+                rl[4 * u] = b4.x; rl[4 * u + 1] = b4.y; rl[4 * u + 2] = b4.z; rl[4 * u + 3] = b4.w;
+            }
 #pragma unroll
-        for (int j = 0; j < NT_O; ++j) {
-            const int c = 8 * j + col0;
-            const float2 xa = *reinterpret_cast<const float2 *>(s_o + la * LD + c);
-            const float2 xb = *reinterpret_cast<const float2 *>(s_o + lb * LD + c);
-            o[j][0] = o[j][0] * c0a + xa.x * c1a;
-            o[j][1] = o[j][1] * c0a + xa.y * c1a;
-            o[j][2] = o[j][2] * c0b + xb.x * c1b;
-            o[j][3] = o[j][3] * c0b + xb.y * c1b;
+            for (int c0 = 0; c0 < HD / 4; c0 += 16) {
+                tmem_st16(tq + L::T_QH + hf * (HD / 4) + c0, rh + c0);
+                tmem_st16(tq + L::T_QL + hf * (HD / 4) + c0, rl + c0);
+            }
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            bar_arrive(q_ready);
         }
-        l_a = l_a * c0a + ua.y * c1a;
-        l_b = l_b * c0b + ub.y * c1b;
-        m_a = Ma;
-        m_b = Mb;
+        const uint64_t *mrow = (is_tree && valid) ? p.mask + (size_t)row * p.mask_words : nullptr;
+        const int klim = valid ? (is_tree ? k_hi : min(k_hi, plen)) : 0;     // keys visible by position
+        for (int j = 0; j < ntiles; ++j) {
+            if (!dead && !wwait(s_full0 + 8 * (j & 1), (uint32_t)(j >> 1) & 1u)) dead = true;
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            const uint32_t sd = tq + L::T_S + (j & 1) * KT;
+            uint32_t sr[32];
+            tmem_ld32(sd + 32 * hf, sr);
+            const int key0 = k_lo + j * KT + 32 * hf;
+            const int lim = klim - key0;                  // columns c < lim are inside the range
+            uint32_t bits = 0xffffffffu;
+            if (mrow) {
+                const int w = (k_lo + j * KT) >> 6;
+                bits = w < p.mask_words ? (uint32_t)(mrow[w] >> (32 * hf)) : 0u;
+            }
+            float v[32];
+            float mx = -INFINITY;
+#pragma unroll
+            for (int c = 0; c < 32; ++c) {
+                const bool vis = c < lim && ((bits >> c) & 1u);
+                v[c] = vis ? __uint_as_float(sr[c]) * p.scale_log2 : -INFINITY;
+                mx = fmaxf(mx, v[c]);
+            }
+            // the row's tile maximum over both halves
+            float *xm = s_xmax + ((j & 1) * 2 + hf) * ROWS;
+            if (lane < 16) xm[row_local] = mx;
+            softmax_sync();
+            if (lane < 16) mx = fmaxf(mx, s_xmax[((j & 1) * 2 + (hf ^ 1)) * ROWS + row_local]);
+            // move the reference maximum only when the tile's exceeds it by > 2^8
+            // (and O already holds visible keys: otherwise O is exactly 0). The
+            // rescale waits for P V of tile j-1 on o_ready: the completed Q K^T of
+            // tile j implies P V of tile j-2, so the barrier is at most one phase
+            // behind and its parity names the phase.
+            const bool need = m_used != -INFINITY && mx > m_used + RESCALE_LOG2;
+            if (__any_sync(0xffffffffu, need)) {
+                if (!dead && !wwait(o_ready, (uint32_t)(j - 1) & 1u)) dead = true;
+                asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+                const float f = need ? ex2_fast(m_used - mx) : 1.f;
+#pragma unroll
+                for (int c0 = 0; c0 < OH; c0 += 32) {
+                    uint32_t r[32];
+                    tmem_ld32(tq + L::T_O + hf * OH + c0, r);
+#pragma unroll
+                    for (int i = 0; i < 32; ++i) r[i] = __float_as_uint(__uint_as_float(r[i]) * f);
+                    tmem_st32(tq + L::T_O + hf * OH + c0, r);
+                }
+                l_sum *= f;
+                if (need) m_used = mx;
+            }
+            if (m_used == -INFINITY) m_used = mx;
+            const float use = m_used == -INFINITY ? 0.f : m_used;
+            float rs = 0.f;
+            uint32_t ph[16], pl[16];
+#pragma unroll
+            for (int c = 0; c < 32; c += 2) {
+                const float e0 = ex2_fast(v[c] - use), e1 = ex2_fast(v[c + 1] - use);
+                rs += e0 + e1;
+                split_pair(e0, e1, ph[c / 2], pl[c / 2]);
+            }
+            l_sum += rs;
+            tmem_st16(sd + 32 * hf, ph);                  // over this half's own S columns:
+            tmem_st16(sd + 32 * hf + 16, pl);             // hi pairs, then lo pairs
+            asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+            bar_arrive(p_full0 + 8 * (j & 1));
+        }
+        // every MMA of the split has completed (the drain barrier completes once,
+        // after the last P V; o_ready's parity could not tell its last phase from
+        // the one two phases back)
+        if (!dead && ntiles > 0 && !wwait(drain, 0u)) dead = true;
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        if (ntiles > 0) {
+#pragma unroll
+            for (int c0 = 0; c0 < OH; c0 += 32) tmem_ld32(tq + L::T_O + hf * OH + c0, o_acc + c0);
+        } else {
+#pragma unroll
+            for (int c = 0; c < OH; ++c) o_acc[c] = 0u;
+        }
+        // the row's sum over both halves
+        if (lane < 16) s_xmax[(4 + hf) * ROWS + row_local] = l_sum;
+        softmax_sync();
+        if (lane < 16) l_sum += s_xmax[(4 + (hf ^ 1)) * ROWS + row_local];
     }
+    const bool ok = !dead && !abort_flag;
 
     const int nsplit = p.nsplit_cache + p.has_tree;
     if (nsplit == 1) {
-        if (half == 1) return;
-        const float ia = l_a > 0.f ? 1.f / l_a : 0.f, ib = l_b > 0.f ? 1.f / l_b : 0.f;
+        if (valid && ok) {
+            const float inv = l_sum > 0.f ? 1.f / l_sum : 0.f;
+            bf16 *dst = p.out + (size_t)row * H + h * HD + hf * OH;
 #pragma unroll
-        for (int j = 0; j < NT_O; ++j) {
-            const int col = h * HD + 8 * j + col0;
-            if (va && ok)
-                *reinterpret_cast<uint32_t *>(p.out + (size_t)ra * H + col) =
-                    pack_bf16(o[j][0] * ia, o[j][1] * ia);
-            if (vb && ok)
-                *reinterpret_cast<uint32_t *>(p.out + (size_t)rb * H + col) =
-                    pack_bf16(o[j][2] * ib, o[j][3] * ib);
+            for (int c = 0; c < OH; c += 4)
+                Split<bf16>::store4(dst + c, p.lo,
+                                    make_float4(__uint_as_float(o_acc[c]) * inv, __uint_as_float(o_acc[c + 1]) * inv,
+                                                __uint_as_float(o_acc[c + 2]) * inv,
+                                                __uint_as_float(o_acc[c + 3]) * inv));
         }
-        return;
-    }
-
-    // Several splits: this (row tile, head)'s CTAs form one thread-block
-    // cluster. Each leaves its partial (unnormalised O, running max m, running
-    // sum l) in its own shared memory; after a cluster barrier every CTA
-    // combines a slice of the rows, reading all partials through distributed
-    // shared memory in rank order (deterministic), and writes them out.
-    __syncwarp();                      // the quad's reads of s_ml above are done
-    if (half == 0) {
+    } else {
+        // Several splits: this (row tile, head)'s CTAs form one cluster. Each
+        // leaves its partial (unnormalised O, reference max m, sum l) in its own
+        // shared memory (the K/V ring is idle now); after a cluster barrier every
+        // CTA combines a slice of the rows, reading all partials through
+        // distributed shared memory in rank order, and writes them out.
+        float *s_o = reinterpret_cast<float *>(smem_raw + (base - su32(smem_raw)));   // [64][LD]
+        float *s_ml = s_o + ROWS * L::LD;                                             // [64][2]
+        __syncthreads();                  // every TMA into the ring has landed and been used
+        if (smx && lane < 16) {
+            const bool live = valid && ok;
 #pragma unroll
-        for (int j = 0; j < NT_O; ++j) {
-            const int c = 8 * j + col0;
-            *reinterpret_cast<float2 *>(s_o + la * LD + c) = make_float2(o[j][0], o[j][1]);
-            *reinterpret_cast<float2 *>(s_o + lb * LD + c) = make_float2(o[j][2], o[j][3]);
+            for (int c = 0; c < OH; c += 4)
+                *reinterpret_cast<float4 *>(s_o + row_local * L::LD + hf * OH + c) =
+                    live ? make_float4(__uint_as_float(o_acc[c]), __uint_as_float(o_acc[c + 1]),
+                                       __uint_as_float(o_acc[c + 2]), __uint_as_float(o_acc[c + 3]))
+                         : make_float4(0.f, 0.f, 0.f, 0.f);
+            if (hf == 0)
+                *reinterpret_cast<float2 *>(s_ml + row_local * 2) =
+                    live ? make_float2(m_used, l_sum) : make_float2(-INFINITY, 0.f);
         }
-        if ((lane & 3) == 0) {
-            *reinterpret_cast<float2 *>(s_ml + la * 2) = make_float2(m_a, l_a);
-            *reinterpret_cast<float2 *>(s_ml + lb * 2) = make_float2(m_b, l_b);
-        }
-    }
-    cluster_sync();
-    const uint32_t rank = cluster_rank();
-    const int nrows = r_end - r0;
-    const int per = (nrows + nsplit - 1) / nsplit;
-    const int row_lo = (int)rank * per, row_hi = min(nrows, row_lo + per);
-    const uint32_t o_local = su32(s_o), ml_local = su32(s_ml);
-    constexpr int C4 = HD / 4, NWARP = THREADS / 32;
-    // a warp combines two of the CTA's rows per pass, every partial load of
-    // both (max and sum of each split, then its O) issued before any is used
-    for (int rr0 = row_lo + warp; rr0 < row_hi; rr0 += 2 * NWARP) {
-        const int rr[2] = {rr0, rr0 + NWARP};
-        const bool has[2] = {true, rr0 + NWARP < row_hi};
-        float2 ml[2];
-        float4 v[2][MAX_SPLITS];
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            ml[u] = make_float2(-INFINITY, 0.f);
-            if (has[u] && lane < nsplit) ml[u] = dsmem_ld_f2(dsmem_addr(ml_local + rr[u] * 8, lane));
-        }
-#pragma unroll
-        for (int u = 0; u < 2; ++u)
+        cluster_sync();
+        const uint32_t rank = cluster_rank();
+        const int nrows = r_end - r0;
+        const int per = (nrows + nsplit - 1) / nsplit;
+        const int row_lo = (int)rank * per, row_hi = min(nrows, row_lo + per);
+        const uint32_t o_local = su32(s_o), ml_local = su32(s_ml);
+        constexpr int C4 = HD / 4, NWARP = THREADS / 32;
+        for (int rr = row_lo + warp; rr < row_hi; rr += NWARP) {
+            float2 ml = make_float2(-INFINITY, 0.f);
+            if (lane < nsplit) ml = dsmem_ld_f2(dsmem_addr(ml_local + rr * 8, lane));
+            float4 v[MAX_SPLITS];
 #pragma unroll
             for (int sp = 0; sp < MAX_SPLITS; ++sp)
-                if (has[u] && lane < C4 && sp < nsplit)
-                    v[u][sp] = dsmem_ld_f4(dsmem_addr(o_local + (rr[u] * LD + 4 * lane) * 4, sp));
-#pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            if (!has[u]) continue;                         // warp-uniform
+                if (lane < C4 && sp < nsplit) v[sp] = dsmem_ld_f4(dsmem_addr(o_local + (rr * L::LD + 4 * lane) * 4, sp));
             // lane sp holds split sp's (m, l); warp shuffles give the max and the sum
-            const float M = warp_max(ml[u].x);
-            const float w = (lane < nsplit && M != -INFINITY) ? exp2f(ml[u].x - M) : 0.f;
-            const float den = warp_sum(w * ml[u].y);
+            const float M = warp_max(ml.x);
+            const float w = (lane < nsplit && M != -INFINITY) ? exp2f(ml.x - M) : 0.f;
+            // the normaliser summed in split order (empty splits add exact zeros),
+            // so a launch's result never depends on how many empty splits it has
+            const float wl = w * ml.y;
+            float den = 0.f;
+#pragma unroll
+            for (int sp = 0; sp < MAX_SPLITS; ++sp) {
+                const float t = __shfl_sync(0xffffffffu, wl, sp);
+                if (sp < nsplit) den += t;
+            }
             const float inv = den > 0.f ? 1.f / den : 0.f;
             const float wn = w * inv;
             float wsp[MAX_SPLITS];
@@ -518,18 +634,23 @@ __global__ void __launch_bounds__(THREADS, 2)
 #pragma unroll
                 for (int sp = 0; sp < MAX_SPLITS; ++sp)
                     if (sp < nsplit) {
-                        acc.x += wsp[sp] * v[u][sp].x; acc.y += wsp[sp] * v[u][sp].y;
-                        acc.z += wsp[sp] * v[u][sp].z; acc.w += wsp[sp] * v[u][sp].w;
+                        acc.x += wsp[sp] * v[sp].x; acc.y += wsp[sp] * v[sp].y;
+                        acc.z += wsp[sp] * v[sp].z; acc.w += wsp[sp] * v[sp].w;
                     }
-                uint2 packed;
-                packed.x = pack_bf16(acc.x, acc.y);
-                packed.y = pack_bf16(acc.z, acc.w);
-                if (ok)
-                    *reinterpret_cast<uint2 *>(p.out + (size_t)(r0 + rr[u]) * H + h * HD + 4 * lane) = packed;
+                if (!abort_flag)
+                    Split<bf16>::store4(p.out + (size_t)(r0 + rr) * H + h * HD + 4 * lane, p.lo, acc);
             }
         }
+        cluster_sync();                    // partials stay readable until all are done
     }
-    cluster_sync();                                    // partials stay readable until all are done
+
+    asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+    __syncthreads();
+    if (warp == 1) {
+        asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+        asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(L::T_COLS)
+                     : "memory");
+    }
 }
 
 struct MapKey {
@@ -553,24 +674,23 @@ struct AttnTcPlan {
     bool attr_set = false;
 };
 
-bool attn_tc_plan_create(AttnTcPlan **out, int max_keys) {
+bool attn_tc_plan_create(AttnTcPlan **out, int max_keys, int decode_ctas) {
     AttnTcPlan *p = new AttnTcPlan();
-    // The cache range is cut at fixed multiples of chunk_tiles * 64 keys, a
-    // function of the capacity only, so results never depend on how many
-    // (possibly empty) splits a launch covers; with the tree split a launch
-    // has at most MAX_SPLITS CTAs per cluster.
-    const int tiles = (max_keys + KT - 1) / KT;
-    // At most CACHE_SPLITS cache splits (+ the tree split): one cluster of <= 9
-    // two-stage CTAs per (row tile, head), two CTAs per SM, so a decode launch
-    // is one wave at any prefix length.
-    p->chunk_tiles = std::max(2, (tiles + CACHE_SPLITS - 1) / CACHE_SPLITS);
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev);
+    // The cache range is cut at fixed multiples of chunk_tiles * 64 keys, a
+    // function of the capacity only, so results never depend on how many
+    // (possibly empty) splits a launch covers. A CTA fills an SM (one per SM):
+    // a decode launch of decode_ctas (row tile, head) pairs takes as many cache
+    // splits as keep it, with the tree split, within one wave.
+    const int tiles = (max_keys + KT - 1) / KT;
+    const int splits = std::max(1, std::min(MAX_SPLITS - 1, p->num_sms / std::max(1, decode_ctas) - 1));
+    p->chunk_tiles = std::max(2, (tiles + splits - 1) / splits);
     cudaDriverEntryPointQueryResult q;
     void *fn = nullptr;
-    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault,
-                                         &q) != cudaSuccess ||
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
+            cudaSuccess ||
         q != cudaDriverEntryPointSuccess || !fn) {
         delete p;
         return false;
@@ -582,6 +702,7 @@ bool attn_tc_plan_create(AttnTcPlan **out, int max_keys) {
 
 void attn_tc_plan_destroy(AttnTcPlan *p) { delete p; }
 
+// Tensor map over `rows` rows of hd bf16 (boxes of 64 rows x 64 columns).
 static const CUtensorMap *kv_map(AttnTcPlan *p, const void *ptr, long rows, int hd) {
     MapKey key{ptr, rows};
     auto it = p->maps.find(key);
@@ -592,18 +713,18 @@ static const CUtensorMap *kv_map(AttnTcPlan *p, const void *ptr, long rows, int 
     cuuint64_t strides[1] = {(cuuint64_t)hd * 2};
     cuuint32_t box[2] = {64, (cuuint32_t)KT};
     cuuint32_t estr[2] = {1, 1};
-    if (p->encode(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box,
-                  estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
-                  CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+    if (p->encode(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(ptr), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS)
         return nullptr;
     return &p->maps.emplace(key, m).first->second;
 }
 
-bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req,
-                         int p_bound, int *status, cudaStream_t s) {
+bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, int p_bound,
+                         int *status, cudaStream_t s) {
     if (a.R <= 0) return true;
     if (a.hd != 64 && a.hd != 128) return false;
+    if (a.lo % a.hd) return false;
     const int tiles_per_req = (rows_per_req + ROWS - 1) / ROWS;
     const int n_blocks = a.R / rows_per_req;
     const int row_tiles = n_blocks * tiles_per_req;
@@ -613,16 +734,17 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     const int cache_tiles = (pb + KT - 1) / KT;
     // enough (row tile, head) CTAs already: one split over the whole range;
     // otherwise fixed-size splits (the count only covers [0, p_bound))
-    const int chunk_tiles = base >= p->num_sms ? cache_tiles : p->chunk_tiles;
+    const int chunk_tiles = base * (1 + has_tree) >= p->num_sms ? cache_tiles : p->chunk_tiles;
     const int nsplit = (cache_tiles + chunk_tiles - 1) / chunk_tiles;
     const int tot = nsplit + has_tree;
     if (tot > MAX_SPLITS) return false;
-    const long kc_rows = (long)B * a.nh * a.cache_slots;
+    const long lo_rows = a.lo / a.hd;
+    const long kc_rows = (long)B * a.nh * a.cache_slots + lo_rows;
     const CUtensorMap *mkc = kv_map(p, a.cache_k, kc_rows, a.hd);
     const CUtensorMap *mvc = kv_map(p, a.cache_v, kc_rows, a.hd);
     const CUtensorMap *mkt = mkc, *mvt = mvc;
     if (has_tree) {
-        const long kt_rows = (long)B * a.nh * a.tree_slots;
+        const long kt_rows = (long)B * a.nh * a.tree_slots + lo_rows;
         mkt = kv_map(p, a.tree_k, kt_rows, a.hd);
         mvt = kv_map(p, a.tree_v, kt_rows, a.hd);
     }
@@ -633,6 +755,8 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.rows = a.rows;
     tp.mask = a.mask;
     tp.out = a.out;
+    tp.lo = a.lo;
+    tp.lo_rows = (int)lo_rows;
     tp.status = status;
     tp.R = a.R;
     tp.rows_per_req = rows_per_req;
@@ -644,17 +768,14 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.nsplit_cache = nsplit;
     tp.has_tree = has_tree;
     tp.chunk = chunk_tiles * KT;
-    // two stages keep two CTAs on an SM; three only where a split holds more
-    // than two tiles and the CTAs fit on the SMs at one per SM
-    tp.stages = (chunk_tiles <= 2 || (long)row_tiles * a.nh * (nsplit + has_tree) > p->num_sms) ? 2 : MAX_STAGES;
     tp.cache_early = a.cache_fresh ? 0 : 1;
     tp.scale_log2 = a.scale * 1.4426950408889634f;
-    const size_t smem = 1024 + (size_t)ROWS * a.hd * 2 + (size_t)tp.stages * 2 * KT * a.hd * 2;
+    const size_t smem = 1024 + (a.hd == 128 ? (size_t)STAGES * Lay<128>::STAGE : (size_t)STAGES * Lay<64>::STAGE);
     if (!p->attr_set) {
         cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             1024 + ROWS * 128 * 2 + MAX_STAGES * 2 * KT * 128 * 2);
+                             (int)(1024 + STAGES * Lay<128>::STAGE));
         cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             1024 + ROWS * 64 * 2 + MAX_STAGES * 2 * KT * 64 * 2);
+                             (int)(1024 + STAGES * Lay<64>::STAGE));
         cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         cudaFuncSetAttribute(attn_tc_kernel<64>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1);
         p->attr_set = true;
@@ -675,9 +796,8 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     at[1].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = at;
     lc.numAttrs = 2;
-    cudaError_t e = a.hd == 128
-                        ? cudaLaunchKernelEx(&lc, attn_tc_kernel<128>, *mkc, *mvc, *mkt, *mvt, tp)
-                        : cudaLaunchKernelEx(&lc, attn_tc_kernel<64>, *mkc, *mvc, *mkt, *mvt, tp);
+    cudaError_t e = a.hd == 128 ? cudaLaunchKernelEx(&lc, attn_tc_kernel<128>, *mkc, *mvc, *mkt, *mvt, tp)
+                                : cudaLaunchKernelEx(&lc, attn_tc_kernel<64>, *mkc, *mvc, *mkt, *mvt, tp);
     note_launch();
     if (e != cudaSuccess) return false;
     return true;

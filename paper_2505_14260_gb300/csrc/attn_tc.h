@@ -1,4 +1,5 @@
-// Tree-masked attention on the tensor cores (bf16 path).
+// Tree-masked attention on the 5th-generation tensor cores (bf16 path): split
+// bf16 operands (hi + lo planes, `lo` elements apart, a multiple of hd).
 #pragma once
 
 #include "kernels.h"
@@ -7,8 +8,9 @@ namespace msd {
 
 struct AttnTcPlan;
 
-// Per-context plan (tensor-map cache, split size); max_keys = cache capacity.
-bool attn_tc_plan_create(AttnTcPlan **out, int max_keys);
+// Per-context plan (tensor-map cache, split size); max_keys = cache capacity,
+// decode_ctas = the (row tile of 64, head) pairs of a decode launch.
+bool attn_tc_plan_create(AttnTcPlan **out, int max_keys, int decode_ctas);
 void attn_tc_plan_destroy(AttnTcPlan *p);
 
 // a.R rows grouped by request in blocks of rows_per_req; every row's plen is

@@ -147,6 +147,58 @@ template <> struct Vec4<bf16> {
     }
 };
 
+// Split-bf16 operands. Every bf16 activation that feeds a tensor-core product
+// (and every K/V cache entry) is kept as a pair hi = bf16(v), lo = bf16(v - hi):
+// hi + lo carries v to about 2^-17 relative, so a product of an exact bf16
+// weight with the pair (two MMAs into one fp32 accumulator) is as precise as an
+// fp32 product. The lo value sits `lo` elements after its hi value (one offset
+// for all of a context's bf16 buffers: they are carved from one arena whose
+// upper half holds the lo planes); lo = 0 means no lo plane (fp32 contexts,
+// caller-owned operands). For T = float the pair is the value itself.
+template <typename T> struct Split;
+template <> struct Split<float> {
+    static __device__ __forceinline__ void store(float *o, long, float v) { *o = v; }
+    static __device__ __forceinline__ float load(const float *g, long) { return *g; }
+    static __device__ __forceinline__ void store4(float *o, long, float4 v) {
+        *reinterpret_cast<float4 *>(o) = v;
+    }
+    static __device__ __forceinline__ float4 load4(const float *g, long) {
+        return *reinterpret_cast<const float4 *>(g);
+    }
+};
+template <> struct Split<bf16> {
+    static __device__ __forceinline__ void store(bf16 *o, long lo, float v) {
+        const bf16 h = __float2bfloat16_rn(v);
+        *o = h;
+        if (lo) o[lo] = __float2bfloat16_rn(v - __bfloat162float(h));
+    }
+    static __device__ __forceinline__ float load(const bf16 *g, long lo) {
+        return lo ? __bfloat162float(g[0]) + __bfloat162float(g[lo]) : __bfloat162float(g[0]);
+    }
+    static __device__ __forceinline__ void store4(bf16 *o, long lo, float4 v) {
+        const __nv_bfloat162 a = __floats2bfloat162_rn(v.x, v.y), b = __floats2bfloat162_rn(v.z, v.w);
+        uint2 u;
+        u.x = *reinterpret_cast<const uint32_t *>(&a);
+        u.y = *reinterpret_cast<const uint32_t *>(&b);
+        *reinterpret_cast<uint2 *>(o) = u;
+        if (lo) {
+            const __nv_bfloat162 c = __floats2bfloat162_rn(v.x - __low2float(a), v.y - __high2float(a));
+            const __nv_bfloat162 d = __floats2bfloat162_rn(v.z - __low2float(b), v.w - __high2float(b));
+            u.x = *reinterpret_cast<const uint32_t *>(&c);
+            u.y = *reinterpret_cast<const uint32_t *>(&d);
+            *reinterpret_cast<uint2 *>(o + lo) = u;
+        }
+    }
+    static __device__ __forceinline__ float4 load4(const bf16 *g, long lo) {
+        float4 h = Vec4<bf16>::load(g);
+        if (lo) {
+            const float4 l = Vec4<bf16>::load(g + lo);
+            h.x += l.x; h.y += l.y; h.z += l.z; h.w += l.w;
+        }
+        return h;
+    }
+};
+
 // Row copies of the small per-row kernels, n a multiple of 4 and rows 4-element
 // aligned: every thread of the CTA requests up to 4 groups of 4 elements (16-
 // or 8-byte accesses) before it stores any, so one pass costs about one memory
@@ -213,6 +265,80 @@ __device__ __forceinline__ void copy_rows2(TD1 *__restrict__ d1, const TS1 *__re
             if (g < n4) {
                 Vec4<TD1>::store(d1 + 4 * g, a[u]);
                 Vec4<TD2>::store(d2 + 4 * g, b[u]);
+            }
+        }
+    }
+}
+
+// Row copy between split buffers (source lo plane at slo, destination at dlo;
+// 0 = none): the pair's sum is re-split, so an exact bf16 source gets lo = 0.
+template <typename TD, typename TS>
+__device__ __forceinline__ void copy_row_split(TD *__restrict__ dst, long dlo, const TS *__restrict__ src,
+                                               long slo, int n) {
+    const int n4 = n >> 2;
+    for (int g0 = threadIdx.x; g0 < n4; g0 += 4 * blockDim.x) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) v[u] = Split<TS>::load4(src + 4 * g, slo);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) Split<TD>::store4(dst + 4 * g, dlo, v[u]);
+        }
+    }
+}
+
+// One fp32 source row to an fp32 row (d1, nullable) and a split row (d2, lo
+// plane at dlo).
+template <typename TD2>
+__device__ __forceinline__ void copy_row_2dst_split(float *__restrict__ d1, TD2 *__restrict__ d2, long dlo,
+                                                    const float *__restrict__ src, int n) {
+    const int n4 = n >> 2;
+    for (int g0 = threadIdx.x; g0 < n4; g0 += 4 * blockDim.x) {
+        float4 v[4];
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) v[u] = *reinterpret_cast<const float4 *>(src + 4 * g);
+        }
+#pragma unroll
+        for (int u = 0; u < 4; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) {
+                if (d1) *reinterpret_cast<float4 *>(d1 + 4 * g) = v[u];
+                Split<TD2>::store4(d2 + 4 * g, dlo, v[u]);
+            }
+        }
+    }
+}
+
+// Two row copies in one pass into split rows (lo planes at dlo): d1 <- s1 (a
+// split source with lo plane at s1lo, or fp32; null: zeros), d2 <- s2 (read
+// as its hi values alone: exact bf16 embeddings).
+template <typename TD, typename TS1, typename TS2>
+__device__ __forceinline__ void copy_rows2_split(TD *__restrict__ d1, const TS1 *__restrict__ s1, long s1lo,
+                                                 TD *__restrict__ d2, const TS2 *__restrict__ s2, int n,
+                                                 long dlo) {
+    const int n4 = n >> 2;
+    for (int g0 = threadIdx.x; g0 < n4; g0 += 2 * blockDim.x) {
+        float4 a[2], b[2];
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) {
+                a[u] = s1 ? Split<TS1>::load4(s1 + 4 * g, s1lo) : make_float4(0.f, 0.f, 0.f, 0.f);
+                b[u] = Vec4<TS2>::load(s2 + 4 * g);
+            }
+        }
+#pragma unroll
+        for (int u = 0; u < 2; ++u) {
+            const int g = g0 + u * blockDim.x;
+            if (g < n4) {
+                Split<TD>::store4(d1 + 4 * g, dlo, a[u]);
+                Split<TD>::store4(d2 + 4 * g, dlo, b[u]);
             }
         }
     }

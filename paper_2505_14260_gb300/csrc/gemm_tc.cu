@@ -158,29 +158,39 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
         : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t (&r)[16]) {
+// TMEM loads of this warp's 32 lanes, 16 or 32 columns, each waited for in
+// the same asm statement: the compiler sees the registers defined only once
+// the data has landed, so no use can be scheduled ahead of the wait.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, uint32_t *r) {
     asm volatile(
         "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-        "%14,%15}, [%16];"
+        "%14,%15}, [%16];\n"
+        "tcgen05.wait::ld.sync.aligned;"
         : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
           "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
           "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+        : "r"(taddr)
+        : "memory");
 }
 
-__device__ __forceinline__ void tmem_ld16_nowait(uint32_t taddr, uint32_t *r) {
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t *r) {
     asm volatile(
-        "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,"
-        "%14,%15}, [%16];"
-        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
-          "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]),
-          "=r"(r[13]), "=r"(r[14]), "=r"(r[15])
-        : "r"(taddr));
+        "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,%15,"
+        "%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];\n"
+        "tcgen05.wait::ld.sync.aligned;"
+        : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]), "=r"(r[7]),
+          "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]), "=r"(r[14]),
+          "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]), "=r"(r[21]),
+          "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]), "=r"(r[28]),
+          "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+        : "r"(taddr)
+        : "memory");
 }
 
-__device__ __forceinline__ void tmem_wait_ld() {
-    asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+// gw (16 or 32: tiles are multiples of 16 columns) columns into r[0 .. gw)
+__device__ __forceinline__ void tmem_ld_cols(uint32_t taddr, uint32_t *r, int gw) {
+    if (gw > 16) tmem_ld32(taddr, r);
+    else tmem_ld16(taddr, r);
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
@@ -386,9 +396,11 @@ struct PkParams {
     float *ws;
     int *counters;
     int *status;
-    bf16 *act;              // EPI_SWIGLU (glu-packed gate/up): act [M][F] bf16
+    bf16 *act;              // EPI_SWIGLU (glu-packed gate/up): act [M][F] split bf16
     int F;
     uint32_t stg_off;       // EPI_SWIGLU: byte offset of the 16 KB staging tile
+    int has_lo;             // X is a split pair: its lo plane comes through the second map
+    long lo;                // lo-plane offset of act (elements)
 };
 
 // silu(g) * u, the SwiGLU product of the fused epilogues.
@@ -427,7 +439,8 @@ struct ItemIter {
 };
 
 __global__ void __launch_bounds__(P_THREADS, 1)
-    gemm_persist_kernel(const __grid_constant__ CUtensorMap mx, const PkParams p) {
+    gemm_persist_kernel(const __grid_constant__ CUtensorMap mx, const __grid_constant__ CUtensorMap mxl,
+                        const PkParams p) {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t bars[2 * P_MAX_STAGES + 5];
     __shared__ uint32_t tmem_base;
@@ -440,7 +453,9 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     const long long U = p.units;                      // stream-K units
     const long long u0 = (long long)cta * U / p.grid, u1 = (long long)(cta + 1) * U / p.grid;
     const int KB = p.kblocks, stages = p.stages, BN = p.BN;
-    const uint32_t b_bytes = (uint32_t)BN * BK * 2;
+    const bool has_lo = p.has_lo != 0;
+    const uint32_t b_bytes = (uint32_t)BN * BK * 2;           // one plane of a token stage
+    const uint32_t bs_bytes = has_lo ? 2 * b_bytes : b_bytes;  // hi, then lo
     const ItemIter items0{u0, u1, KB, p.T_sk, p.grid, cta, 0, p.dp_rounds};
 
     const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
@@ -492,6 +507,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     if (warp == 0) {
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
+            if (has_lo) asm volatile("prefetch.tensormap [%0];" ::"l"(&mxl) : "memory");
             // Weights never depend on the previous kernel: the first stages'
             // weight blocks are requested before waiting for it.
             int n_pre = 0;
@@ -501,7 +517,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 while (n_pre < stages && it.next(t, kb_b, kb_e)) {
                     const bf16 *w = p.wpacked + ((size_t)(t / p.n_tiles_n) * KB + kb_b) * blk_elems;
                     for (int kb = kb_b; kb < kb_e && n_pre < stages; ++kb, ++n_pre, w += blk_elems) {
-                        mbar_expect_tx(full0 + 8 * n_pre, A_BYTES + b_bytes);
+                        mbar_expect_tx(full0 + 8 * n_pre, A_BYTES + bs_bytes);
                         bulk_load(a_base + n_pre * A_BYTES, w, A_BYTES, full0 + 8 * n_pre);
                     }
                 }
@@ -522,10 +538,11 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                             stop = true;
                             break;
                         }
-                        mbar_expect_tx(full0 + 8 * s, A_BYTES + b_bytes);
+                        mbar_expect_tx(full0 + 8 * s, A_BYTES + bs_bytes);
                         bulk_load(a_base + s * A_BYTES, w, A_BYTES, full0 + 8 * s);
                     }
-                    tma_load_2d(b_base + s * b_bytes, &mx, kb * BK, n0, full0 + 8 * s);
+                    tma_load_2d(b_base + s * bs_bytes, &mx, kb * BK, n0, full0 + 8 * s);
+                    if (has_lo) tma_load_2d(b_base + s * bs_bytes + b_bytes, &mxl, kb * BK, n0, full0 + 8 * s);
                     if (++s == stages) {
                         s = 0;
                         ph ^= 1u;
@@ -558,10 +575,13 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                     if (!mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status)) break;
                     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                     const uint64_t ad = smem_desc(a_base + s * A_BYTES);
-                    const uint64_t bd = smem_desc(b_base + s * b_bytes);
+                    const uint64_t bd = smem_desc(b_base + s * bs_bytes);
+                    const uint64_t bl = smem_desc(b_base + s * bs_bytes + b_bytes);
 #pragma unroll
-                    for (int kk = 0; kk < BK / 16; ++kk)
+                    for (int kk = 0; kk < BK / 16; ++kk) {
                         mma_bf16(acc, ad + 2 * kk, bd + 2 * kk, idesc, (j != 0) || (kk != 0));
+                        if (has_lo) mma_bf16(acc, ad + 2 * kk, bl + 2 * kk, idesc, 1u);
+                    }
                     mma_commit(empty0 + 8 * s);
                     if (++s == stages) {
                         s = 0;
@@ -606,10 +626,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 // up to 32 accumulator columns with one TMEM round trip
                 const int gw = min(32, BN - g0);
                 uint32_t r[32];
-#pragma unroll
-                for (int c = 0; c < 2; ++c)
-                    if (c * 16 < gw) tmem_ld16_nowait(taddr + g0 + c * 16, r + c * 16);
-                tmem_wait_ld();
+                tmem_ld_cols(taddr + g0, r, gw);
                 if (whole && glu) {
                     // gate row i and up row 64 + i of the tile sit in different
                     // warps: exchange through shared memory, then thread (i, h)
@@ -625,8 +642,8 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                         for (int c = 16 * h; c < 16 * h + 16; ++c) {
                             const int m = n0 + g0 + c;
                             if (c < gw && m < p.M)
-                                p.act[(size_t)m * p.F + jo] =
-                                    __float2bfloat16_rn(swiglu_fused(stg[c * BM + i], stg[c * BM + 64 + i]));
+                                Split<bf16>::store(p.act + (size_t)m * p.F + jo, p.lo,
+                                                   swiglu_fused(stg[c * BM + i], stg[c * BM + 64 + i]));
                         }
                     }
                 } else if (!whole) {
@@ -722,13 +739,10 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                         const int m = n0 + col;
                         const int jo = (row0 >> 1) + r4;
                         if (m >= p.M || !ok || r4 >= 64 || jo >= p.F) continue;
-                        bf16 *dst = p.act + (size_t)m * p.F + jo;
-                        __nv_bfloat162 lo2 = __floats2bfloat162_rn(swiglu_fused(acc[g].x, up.x),
-                                                                   swiglu_fused(acc[g].y, up.y));
-                        __nv_bfloat162 hi2 = __floats2bfloat162_rn(swiglu_fused(acc[g].z, up.z),
-                                                                   swiglu_fused(acc[g].w, up.w));
-                        reinterpret_cast<__nv_bfloat162 *>(dst)[0] = lo2;   // F % 4 == 0: 8-byte aligned
-                        reinterpret_cast<__nv_bfloat162 *>(dst)[1] = hi2;
+                        bf16 *dst = p.act + (size_t)m * p.F + jo;     // F % 4 == 0: 8-byte aligned
+                        Split<bf16>::store4(dst, p.lo,
+                                            make_float4(swiglu_fused(acc[g].x, up.x), swiglu_fused(acc[g].y, up.y),
+                                                        swiglu_fused(acc[g].z, up.z), swiglu_fused(acc[g].w, up.w)));
                         continue;
                     }
                     if (e4 >= n4) continue;
@@ -790,6 +804,8 @@ struct CkParams {
     int seg_rows[3];
     int seg_out[3];
     int M, kblocks, BN, n_tiles_n, splits, tmem_cols;
+    int stages;             // ring depth (<= C_STAGES)
+    int has_lo;             // X is a split pair: its lo plane comes through the second map
     const bf16 *wpacked;
     float *Y;
     int ldy, epi;
@@ -834,10 +850,6 @@ __device__ __forceinline__ float4 c_smem_ld4(uint32_t local) {
     return v;
 }
 
-__device__ __forceinline__ uint2 c_pack_bf16x4(float a, float b, float c, float d) {
-    const __nv_bfloat162 lo = __floats2bfloat162_rn(a, b), hi = __floats2bfloat162_rn(c, d);
-    return make_uint2(*reinterpret_cast<const uint32_t *>(&lo), *reinterpret_cast<const uint32_t *>(&hi));
-}
 
 // Where a CTA finds the S partials of the token columns it owns, [c_lo,
 // c_hi) = [rank * BN / S, (rank + 1) * BN / S): its own partial ([BN][128]
@@ -919,7 +931,7 @@ __device__ __forceinline__ void c_epi_swiglu(const CkParams &p, const PartSrc &p
             const float o1 = __fdividef(a.y, 1.f + __expf(-a.y)) * b.y;
             const float o2 = __fdividef(a.z, 1.f + __expf(-a.z)) * b.z;
             const float o3 = __fdividef(a.w, 1.f + __expf(-a.w)) * b.w;
-            *reinterpret_cast<uint2 *>(act + (size_t)m * F + j) = c_pack_bf16x4(o0, o1, o2, o3);
+            Split<bf16>::store4(act + (size_t)m * F + j, p.fx.lo, make_float4(o0, o1, o2, o3));
         }
     }
 }
@@ -1027,8 +1039,8 @@ __device__ __forceinline__ void c_epi_rope(const CkParams &p, const PartSrc &ps,
             if (d.dst < 0 || d.dst >= slots) continue;
             dst = kvd + ((size_t)(d.req * nh + h) * slots + d.dst) * hd + i;
         }
-        *reinterpret_cast<uint2 *>(dst) = c_pack_bf16x4(a.x, a.y, a.z, a.w);
-        *reinterpret_cast<uint2 *>(dst + half) = c_pack_bf16x4(b.x, b.y, b.z, b.w);
+        Split<bf16>::store4(dst, p.fx.lo, a);
+        Split<bf16>::store4(dst + half, p.fx.lo, b);
     }
 }
 
@@ -1096,8 +1108,8 @@ __device__ __forceinline__ void c_reduce_norm(const CkParams &p, const PartSrc &
                     a[0] += yi.x; a[1] += yi.y; a[2] += yi.z; a[3] += yi.w;
                 }
                 *reinterpret_cast<float4 *>(y) = make_float4(a[0], a[1], a[2], a[3]);
-                *reinterpret_cast<uint2 *>(xg) =
-                    c_pack_bf16x4(a[0] * g4[0], a[1] * g4[1], a[2] * g4[2], a[3] * g4[3]);
+                Split<bf16>::store4(xg, p.nout.lo,
+                                    make_float4(a[0] * g4[0], a[1] * g4[1], a[2] * g4[2], a[3] * g4[3]));
                 ss = a[0] * a[0] + a[1] * a[1] + a[2] * a[2] + a[3] * a[3];
             } else {
                 const bf16 *g = p.nout.g + o_base + r4;
@@ -1106,7 +1118,7 @@ __device__ __forceinline__ void c_reduce_norm(const CkParams &p, const PartSrc &
                     if (r4 + e < rows_here) {
                         const float ye = add ? y[e] + a[e] : a[e];
                         y[e] = ye;
-                        xg[e] = __float2bfloat16_rn(ye * __bfloat162float(g[e]));
+                        Split<bf16>::store(xg + e, p.nout.lo, ye * __bfloat162float(g[e]));
                         ss += ye * ye;
                     }
             }
@@ -1117,7 +1129,8 @@ __device__ __forceinline__ void c_reduce_norm(const CkParams &p, const PartSrc &
 }
 
 __global__ void __launch_bounds__(C_THREADS)
-    gemm_cluster_kernel(const __grid_constant__ CUtensorMap mx, const CkParams p) {
+    gemm_cluster_kernel(const __grid_constant__ CUtensorMap mx, const __grid_constant__ CUtensorMap mxl,
+                        const CkParams p) {
     extern __shared__ uint8_t smem_raw[];
     __shared__ __align__(8) uint64_t bars[2 * C_STAGES + 2];
     __shared__ uint32_t tmem_base;
@@ -1138,18 +1151,21 @@ __global__ void __launch_bounds__(C_THREADS)
     const int kb0 = (int)((long long)split * KB / S), kb1 = (int)((long long)(split + 1) * KB / S);
     const int nk = kb1 - kb0;
     const int BN = p.BN;
-    const uint32_t b_bytes = (uint32_t)BN * BK * 2;
+    const int stages = p.stages;
+    const bool has_lo = p.has_lo != 0;
+    const uint32_t b_bytes = (uint32_t)BN * BK * 2;          // one plane of a token stage
+    const uint32_t bs_bytes = has_lo ? 2 * b_bytes : b_bytes; // hi, then lo
     const size_t blk_elems = A_BYTES / 2;
     const bf16 *wblk = p.wpacked + ((size_t)blockIdx.x * KB + kb0) * blk_elems;
 
     const uint32_t sbase = (smem_u32(smem_raw) + 1023u) & ~1023u;
-    const uint32_t a_base = sbase, b_base = sbase + C_STAGES * A_BYTES;
+    const uint32_t a_base = sbase, b_base = sbase + stages * A_BYTES;
     const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[C_STAGES]);
     const uint32_t done = smem_u32(&bars[2 * C_STAGES]);
     const uint32_t recv_bar = smem_u32(&bars[2 * C_STAGES + 1]);   // the other ranks' slices have landed
 
     if (threadIdx.x == 0) {
-        for (int s = 0; s < C_STAGES; ++s) {
+        for (int s = 0; s < stages; ++s) {
             mbar_init(full0 + 8 * s, 1);
             mbar_init(empty0 + 8 * s, 1);
         }
@@ -1173,10 +1189,11 @@ __global__ void __launch_bounds__(C_THREADS)
     if (warp == 0) {
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
+            if (has_lo) asm volatile("prefetch.tensormap [%0];" ::"l"(&mxl) : "memory");
             // weights first (they never depend on the previous kernel), then wait
-            const int n_pre = min(C_STAGES, nk);
+            const int n_pre = min(stages, nk);
             for (int j = 0; j < n_pre; ++j) {
-                mbar_expect_tx(full0 + 8 * j, A_BYTES + b_bytes);
+                mbar_expect_tx(full0 + 8 * j, A_BYTES + bs_bytes);
                 bulk_load(a_base + j * A_BYTES, wblk + (size_t)j * blk_elems, A_BYTES, full0 + 8 * j);
             }
             pdl_wait();
@@ -1187,20 +1204,20 @@ __global__ void __launch_bounds__(C_THREADS)
             for (; i < nk; ++i) {
                 if (i >= n_pre) {
                     if (!mbar_wait(empty0 + 8 * s, ph ^ 1u, &abort_flag, p.status)) break;
-                    mbar_expect_tx(full0 + 8 * s, A_BYTES + b_bytes);
+                    mbar_expect_tx(full0 + 8 * s, A_BYTES + bs_bytes);
                     bulk_load(a_base + s * A_BYTES, wblk + (size_t)i * blk_elems, A_BYTES, full0 + 8 * s);
                 }
-                tma_load_2d(b_base + s * b_bytes, &mx, (kb0 + i) * BK, n0, full0 + 8 * s);
-                if (++s == C_STAGES) {
+                tma_load_2d(b_base + s * bs_bytes, &mx, (kb0 + i) * BK, n0, full0 + 8 * s);
+                if (has_lo) tma_load_2d(b_base + s * bs_bytes + b_bytes, &mxl, (kb0 + i) * BK, n0, full0 + 8 * s);
+                if (++s == stages) {
                     s = 0;
                     ph ^= 1u;
                 }
             }
             if (abort_flag) {
                 volatile int never = 0;
-                for (int j = (i > C_STAGES ? i - C_STAGES : 0); j < i; ++j)
-                    mbar_wait(full0 + 8 * (j % C_STAGES), (uint32_t)(j / C_STAGES) & 1u, &never,
-                              p.status);
+                for (int j = (i > stages ? i - stages : 0); j < i; ++j)
+                    mbar_wait(full0 + 8 * (j % stages), (uint32_t)(j / stages) & 1u, &never, p.status);
             }
         }
         __syncwarp();
@@ -1214,12 +1231,15 @@ __global__ void __launch_bounds__(C_THREADS)
                 if (!mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status)) break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint64_t ad = smem_desc(a_base + s * A_BYTES);
-                const uint64_t bd = smem_desc(b_base + s * b_bytes);
+                const uint64_t bd = smem_desc(b_base + s * bs_bytes);
+                const uint64_t bl = smem_desc(b_base + s * bs_bytes + b_bytes);
 #pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk)
+                for (int kk = 0; kk < BK / 16; ++kk) {
                     mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (i != 0) || (kk != 0));
+                    if (has_lo) mma_bf16(tmem, ad + 2 * kk, bl + 2 * kk, idesc, 1u);
+                }
                 mma_commit(empty0 + 8 * s);
-                if (++s == C_STAGES) {
+                if (++s == stages) {
                     s = 0;
                     ph ^= 1u;
                 }
@@ -1262,10 +1282,7 @@ __global__ void __launch_bounds__(C_THREADS)
         for (int g0 = 0; g0 < BN; g0 += 32) {
             const int gw = min(32, BN - g0);
             uint32_t r[32];
-#pragma unroll
-            for (int c = 0; c < 2; ++c)
-                if (c * 16 < gw) tmem_ld16_nowait(taddr + g0 + c * 16, r + c * 16);
-            tmem_wait_ld();
+            tmem_ld_cols(taddr + g0, r, gw);
             if (ok && row < rows_here) {
                 float *yb = p.Y + (size_t)(n0 + g0) * p.ldy + o_base + row;
                 const int mlim = p.M - (n0 + g0);
@@ -1290,10 +1307,7 @@ __global__ void __launch_bounds__(C_THREADS)
         for (int g0 = 0; g0 < BN; g0 += 32) {
             const int gw = min(32, BN - g0);
             uint32_t r[32];
-#pragma unroll
-            for (int c = 0; c < 2; ++c)
-                if (c * 16 < gw) tmem_ld16_nowait(taddr + g0 + c * 16, r + c * 16);
-            tmem_wait_ld();
+            tmem_ld_cols(taddr + g0, r, gw);
 #pragma unroll
             for (int j = 0; j < 32; ++j)
                 if (j < gw) part[(g0 + j) * BM + row] = __uint_as_float(r[j]);
@@ -1578,8 +1592,12 @@ void gemm_pack_glu(const void *gate, const void *up, int F, int K, void *dst, cu
 }
 
 // Launch of the cluster split-K kernel: s K-splits per tile (a cluster), chosen
-// so that tiles * s fills two CTAs per SM once, s <= 8 and >= 2 K-blocks each.
-static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W,
+// so that tiles * s fills the CTAs the SMs hold at once, s <= 8 and >= 2
+// K-blocks each. Two CTAs share an SM when three stages fit in half of its
+// shared memory (token tiles of up to 64 split rows), otherwise one with up to
+// four stages; the split count keeps every split's partial slices within the
+// stage memory they reuse.
+static void gemm_cluster(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, int M, int K, const GemmW &W,
                          int tiles, int BN, int kblocks, float *Y, int ldy, int epi, int *status,
                          cudaStream_t s, int O, const GemmFused *fx = nullptr,
                          const GemmNorm *nout = nullptr, const GemmNorm *nin = nullptr) {
@@ -1596,14 +1614,24 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
         ck.seg_out[i] = out_off;
         out_off += W.rows[i];
     }
-    int S = (2 * p->num_sms) / tiles;
+    const int nb = X_lo ? 2 : 1;
+    const size_t stage = A_BYTES + (size_t)nb * BN * BK * 2;
+    constexpr size_t HALF_SM = 104u * 1024u, FULL_SM = 200u * 1024u;
+    const int per_sm = 3 * stage <= HALF_SM ? 2 : 1;
+    int stages = (int)((per_sm == 2 ? HALF_SM : FULL_SM) / stage);
+    stages = std::max(2, std::min(stages, C_STAGES));
+    int S = (per_sm * p->num_sms) / tiles;
     S = std::max(1, std::min(S, 8));
     while (S > 1 && kblocks / S < 2) --S;
+    // own partial [BN][128] fp32 plus the other ranks' slices of this rank's columns
+    while (S > 1 && (size_t)BN * BM * 4 + (size_t)(S - 1) * ((BN + S - 1) / S) * BM * 4 > stages * stage) --S;
     ck.M = M;
     ck.kblocks = kblocks;
     ck.BN = BN;
     ck.n_tiles_n = 1;
     ck.splits = S;
+    ck.stages = stages;
+    ck.has_lo = X_lo ? 1 : 0;
     ck.tmem_cols = BN <= 32 ? 32 : (BN <= 64 ? 64 : 128);
     ck.wpacked = static_cast<const bf16 *>(W.packed);
     ck.Y = Y;
@@ -1611,11 +1639,12 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
     ck.epi = epi;
     ck.status = status;
     const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
-    if (!mx) return;
-    const size_t smem = 1024 + (size_t)C_STAGES * (A_BYTES + (size_t)BN * BK * 2);
+    const CUtensorMap *mxl = X_lo ? get_map(p, X_lo, M, K, ldx, BN, status) : mx;
+    if (!mx || !mxl) return;
+    const size_t smem = 1024 + (size_t)stages * stage;
     if (!p->cluster_attr_set) {
         cudaFuncSetAttribute(gemm_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             (int)(1024 + C_STAGES * (A_BYTES + 128 * BK * 2)));
+                             (int)(1024 + FULL_SM));
         p->cluster_attr_set = true;
     }
     const bool prof = p->profile;
@@ -1642,7 +1671,7 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
     at[1].val.clusterDim.z = (unsigned)S;
     lc.attrs = at;
     lc.numAttrs = 2;
-    if (cudaLaunchKernelEx(&lc, gemm_cluster_kernel, *mx, ck) != cudaSuccess) {
+    if (cudaLaunchKernelEx(&lc, gemm_cluster_kernel, *mx, *mxl, ck) != cudaSuccess) {
         cudaGetLastError();
         flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
         fprintf(stderr, "msd: cluster GEMM launch failed (M=%d K=%d O=%d S=%d)\n", M, K, O, S);
@@ -1654,19 +1683,19 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
         const double wb = (double)O * K * 2.0;
         p->prof_wbytes += wb;
         double yb = (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
-        if (epi == EPI_SWIGLU) yb = (double)M * fx->F * 2.0;
-        if (epi == EPI_ROPE_KV) yb = (double)M * O * 2.0;
-        p->prof_bytes += wb + (double)M * K * 2.0 + yb;
+        if (epi == EPI_SWIGLU) yb = (double)M * fx->F * 2.0 * nb;
+        if (epi == EPI_ROPE_KV) yb = (double)M * O * 2.0 * nb;
+        p->prof_bytes += wb + (double)M * K * 2.0 * nb + yb;
     }
 }
 
 // The persistent stream-K GEMM (many token rows). fx: EPI_SWIGLU writes
 // act = silu(g) * u from glu-packed gate/up weights instead of Y.
-static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
-                         float *Y, int ldy, int epi, const GemmFused *fx, int *status, cudaStream_t s);
+static void gemm_persist(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, int M, int K, const GemmW &W,
+                         int O, float *Y, int ldy, int epi, const GemmFused *fx, int *status, cudaStream_t s);
 
-bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
-                     const GemmFused &fx, int *status, cudaStream_t s, const GemmNorm *norm_in) {
+bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, int M, int K, const GemmW &W,
+                     int O, const GemmFused &fx, int *status, cudaStream_t s, const GemmNorm *norm_in) {
     if (M <= 0 || !W.packed || W.nseg < 1) return false;
     if (fx.epi == EPI_SWIGLU && (W.nseg != 1 || W.rows[0] != glu_rows(fx.F) || fx.F % 4)) return false;
     if (M > 128) {
@@ -1674,7 +1703,7 @@ bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const Ge
         // epilogue (RoPE/KV stays a separate kernel there: fused, its
         // per-column gathers outlasted the main loop, measured slower)
         if (fx.epi != EPI_SWIGLU || norm_in || !fx.act) return false;
-        gemm_persist(p, X, ldx, M, K, W, O, nullptr, 0, EPI_SWIGLU, &fx, status, s);
+        gemm_persist(p, X, X_lo, ldx, M, K, W, O, nullptr, 0, EPI_SWIGLU, &fx, status, s);
         return true;
     }
     if (fx.epi == EPI_ROPE_KV &&
@@ -1687,13 +1716,13 @@ bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const Ge
     const int BN = ((M + 15) / 16) * 16;
     if (norm_in && (!norm_in->ss || norm_in->parts <= 0 || norm_in->parts > norm_in->ld || BN > 128))
         return false;
-    gemm_cluster(p, X, ldx, M, K, W, tiles, BN, (K + BK - 1) / BK, nullptr, 0, fx.epi, status, s, O, &fx,
+    gemm_cluster(p, X, X_lo, ldx, M, K, W, tiles, BN, (K + BK - 1) / BK, nullptr, 0, fx.epi, status, s, O, &fx,
                  nullptr, norm_in);
     return true;
 }
 
-bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
-               int ldy, int epi, int *status, cudaStream_t s, const GemmNorm *norm_out) {
+bool gemm_bf16(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, int M, int K, const GemmW &W, int O,
+               float *Y, int ldy, int epi, int *status, cudaStream_t s, const GemmNorm *norm_out) {
     if (M <= 0 || O <= 0) return true;
     if (norm_out && (M > 128 || !W.packed || W.nseg != 1 || !norm_out->ss || !norm_out->xg || !norm_out->g ||
                      (O + BM - 1) / BM > norm_out->ld || O % 4 || ldy % 4))
@@ -1701,16 +1730,16 @@ bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W
     if (M <= 128 && W.packed) {
         int tiles = 0;
         for (int i = 0; i < W.nseg; ++i) tiles += (W.rows[i] + BM - 1) / BM;
-        gemm_cluster(p, X, ldx, M, K, W, tiles, ((M + 15) / 16) * 16, (K + BK - 1) / BK, Y, ldy, epi, status,
-                     s, O, nullptr, norm_out);
+        gemm_cluster(p, X, X_lo, ldx, M, K, W, tiles, ((M + 15) / 16) * 16, (K + BK - 1) / BK, Y, ldy, epi,
+                     status, s, O, nullptr, norm_out);
         return true;
     }
-    gemm_persist(p, X, ldx, M, K, W, O, Y, ldy, epi, nullptr, status, s);
+    gemm_persist(p, X, X_lo, ldx, M, K, W, O, Y, ldy, epi, nullptr, status, s);
     return true;
 }
 
-static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
-                         float *Y, int ldy, int epi, const GemmFused *fx, int *status, cudaStream_t s) {
+static void gemm_persist(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, int M, int K, const GemmW &W,
+                         int O, float *Y, int ldy, int epi, const GemmFused *fx, int *status, cudaStream_t s) {
     const bool glu = fx && fx->epi == EPI_SWIGLU;
     PkParams pk;
     memset(&pk, 0, sizeof pk);
@@ -1723,15 +1752,21 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
         out_off += W.rows[i];
         tiles += pk.seg_tiles[i];
     }
-    const int nt = (M + 255) / 256;
-    int BN = (M + nt - 1) / nt;
-    BN = ((BN + 15) / 16) * 16;
-    const int kblocks = (K + BK - 1) / BK;
-    const uint32_t stage_bytes = A_BYTES + (uint32_t)BN * BK * 2;
-    // five stages measured best on the decode shapes (deeper rings were slower);
+    const int nb = X_lo ? 2 : 1;
     // the fused SwiGLU epilogue takes 16 KB of staging from the ring's budget
     const uint32_t stg_bytes = glu ? 32u * BM * 4u : 0u;
-    int stages = (int)((200u * 1024u - stg_bytes) / stage_bytes);
+    constexpr uint32_t BUDGET = 208u * 1024u;
+    // token tiles: the widest (fewest tiles, most weight reuse) that keeps three
+    // stages in shared memory; five stages measured best on decode shapes
+    int nt = (M + 255) / 256, BN = 0;
+    for (;; ++nt) {
+        BN = ((M + nt - 1) / nt + 15) / 16 * 16;
+        const uint32_t st = A_BYTES + (uint32_t)nb * BN * BK * 2;
+        if (3u * st + stg_bytes <= BUDGET || BN <= 16) break;
+    }
+    const int kblocks = (K + BK - 1) / BK;
+    const uint32_t stage_bytes = A_BYTES + (uint32_t)nb * BN * BK * 2;
+    int stages = (int)((BUDGET - stg_bytes) / stage_bytes);
     stages = stages < 2 ? 2 : (stages > 5 ? 5 : stages);
     const size_t smem = 1024 + (size_t)stages * stage_bytes + stg_bytes;
     const long long tiles_total = (long long)tiles * nt;
@@ -1770,10 +1805,12 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
     pk.counters = p->counters;
     pk.status = status;
     pk.wpacked = static_cast<const bf16 *>(W.packed);
+    pk.has_lo = X_lo ? 1 : 0;
     if (glu) {
         pk.epi = EPI_SWIGLU;
         pk.act = fx->act;
         pk.F = fx->F;
+        pk.lo = fx->lo;
         pk.stg_off = (uint32_t)(1024 + (size_t)stages * stage_bytes);
     }
     if (!W.packed) {
@@ -1782,12 +1819,11 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
         return;
     }
     const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
-    if (!mx) return;
+    const CUtensorMap *mxl = X_lo ? get_map(p, X_lo, M, K, ldx, BN, status) : mx;
+    if (!mx || !mxl) return;
     if (!p->smem_set) {
-        cudaFuncSetAttribute(gemm_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             200 * 1024 + 1024);
         cudaFuncSetAttribute(gemm_persist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                             200 * 1024 + 1024);
+                             (int)(BUDGET + 1024));
         p->smem_set = true;
     }
     const bool prof = p->profile;
@@ -1813,15 +1849,15 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, int ldx, int M, int K, cons
     at[0].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = at;
     lc.numAttrs = 1;
-    cudaLaunchKernelEx(&lc, gemm_persist_kernel, *mx, pk);
+    cudaLaunchKernelEx(&lc, gemm_persist_kernel, *mx, *mxl, pk);
     note_launch();
     if (prof) {
         cudaEventRecord(p->ev[p->ev_used + 1], s);
         p->ev_used += 2;
         const double wb = (double)O * K * 2.0;
         p->prof_wbytes += wb;
-        p->prof_bytes += wb + (double)M * K * 2.0 +
-                         (glu ? (double)M * fx->F * 2.0 : (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1));
+        p->prof_bytes += wb + (double)M * K * 2.0 * nb +
+                         (glu ? (double)M * fx->F * 2.0 * nb : (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1));
     }
 }
 

@@ -14,11 +14,13 @@ void gemm_plan_destroy(GemmPlan *p);
 
 // Y[m][o] (=|+=) sum_k X[m][k] W[o][k]; X, W bf16 (K contiguous, rows 16-byte
 // aligned), Y fp32. Weight tiles fill the MMA's M = 128 side, tokens its N side.
+// X_lo (nullable): the lo plane of a split-bf16 X (same layout): the product
+// is then W (X + X_lo), two MMAs per K step into one fp32 accumulator.
 // norm_out (nullable, decode shapes M <= 128 with packed W only): the
 // producer side of a folded RMSNorm (GemmNorm below); returns false (nothing
 // launched) when it is given for a shape off the decode path.
-bool gemm_bf16(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
-               int ldy, int epi, int *status, cudaStream_t s, const GemmNorm *norm_out = nullptr);
+bool gemm_bf16(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, int M, int K, const GemmW &W, int O,
+               float *Y, int ldy, int epi, int *status, cudaStream_t s, const GemmNorm *norm_out = nullptr);
 
 // Pre-packed weights: the segments' 128-row x 64-column blocks, tile-major then
 // K-block, each block stored exactly as the MMA reads it from shared memory
@@ -44,6 +46,8 @@ void gemm_pack_glu(const void *gate, const void *up, int F, int K, void *dst, cu
 //                slot rows[m].dst of request rows[m].req (dst < 0: not
 //                written; dst >= slots or a position outside the table: status
 //                ST_RANGE).
+// Outputs are split bf16 pairs, lo planes `lo` elements after act, q_out,
+// kdst and vdst (lo = 0: hi values only).
 struct GemmFused {
     int epi;
     bf16 *act;
@@ -53,12 +57,14 @@ struct GemmFused {
     int max_pos;
     bf16 *q_out, *kdst, *vdst;
     int slots, nh, hd;
+    long lo;
 };
 // RMSNorm folded into a pair of decode GEMMs (the norm's per-row scale
 // commutes with the projection that follows it):
 //   producer (an H-output GEMM, EPI_STORE / EPI_ADD): besides Y = x, writes
-//     xg[m][o] = bf16(x[m][o] * g[o]) and ss[m][tile] = sum over the tile's 128
-//     rows of x[m][o]^2 (fixed order), ld = row stride of ss;
+//     xg[m][o] = x[m][o] * g[o] (split bf16, lo plane at xg + lo) and
+//     ss[m][tile] = sum over the tile's 128 rows of x[m][o]^2 (fixed order),
+//     ld = row stride of ss;
 //   consumer (EPI_ROPE_KV / EPI_SWIGLU on X = xg): scales its accumulator row m
 //     by 1 / sqrt(sum_{j < parts} ss[m][j] / H + eps) (summed in j order) before
 //     the rotation or the SwiGLU.
@@ -69,12 +75,14 @@ struct GemmNorm {
     const bf16 *g;
     int parts, H;
     float eps;
+    long lo;
 };
 
 // Runs the fused GEMM and returns true when the shape takes the decode path;
 // returns false (nothing launched) otherwise.
-bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
-                     const GemmFused &fx, int *status, cudaStream_t s, const GemmNorm *norm_in = nullptr);
+bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, int M, int K, const GemmW &W,
+                     int O, const GemmFused &fx, int *status, cudaStream_t s,
+                     const GemmNorm *norm_in = nullptr);
 
 // Profiling: while enabled, every launch is bracketed by CUDA events on its
 // stream; gemm_profile_read synchronises on them and returns the launches,

@@ -17,24 +17,24 @@ template <typename T>
 void launch_embed_rows(const T *E, const T *vis, const int *src, int R, int H,
                        float *x, T *emb_out, int V, int *status, cudaStream_t s);
 
-// out[r] = T(x[r] / sqrt(mean(x[r]^2) + eps) * g)
+// out[r] = x[r] / sqrt(mean(x[r]^2) + eps) * g, split (lo plane at out + lo)
 template <typename T>
-void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
+void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out, long lo,
                     cudaStream_t s);
 
 // act[r][j] = T(silu(g) * u) with g = gu[r][j], u = gu[r][F + j], or, for
 // glu-packed gate/up products (glu = true, rows of 128 * ceil(F / 64)),
 // g = gu[r][128 (j / 64) + j % 64] and u 64 columns further.
 template <typename T>
-void launch_swiglu(const float *gu, int R, int F, bool glu, T *act, cudaStream_t s);
+void launch_swiglu(const float *gu, int R, int F, bool glu, T *act, long lo, cudaStream_t s);
 
 // RoPE (rotate-half, table of (cos, sin) per position and pair) on q and k of
 // qkv [R][3H]; q -> q_out [R][H]; k, v -> kdst/vdst at slot rows[r].dst of
-// request rows[r].req: [B][nh][slots][hd].
+// request rows[r].req: [B][nh][slots][hd]; all outputs split (lo planes at +lo).
 template <typename T>
 void launch_rope_kv(const float *qkv, const RowDesc *rows, int R, int nh, int hd,
                     const float2 *rope_tab, int max_pos, T *q_out, T *kdst,
-                    T *vdst, int slots, int *status, cudaStream_t s);
+                    T *vdst, int slots, long lo, int *status, cudaStream_t s);
 
 // Row r attends to cache[req][h][0 .. plen) and to the tree slots j of
 // request req with bit j of mask[r] set.
@@ -53,6 +53,7 @@ struct AttnArgs {
     float scale;
     T *out;                     // [R][nh*hd]
     bool cache_fresh;           // the kernel launched just before may have written cache_k/v
+    long lo;                    // split bf16: lo planes of q, K/V and out sit lo elements on (0: none)
 };
 template <typename T>
 void launch_attention(const AttnArgs<T> &a, cudaStream_t s);

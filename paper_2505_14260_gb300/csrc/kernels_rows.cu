@@ -52,7 +52,7 @@ constexpr int RMS_VEC = 8;
 template <typename T>
 __global__ void __launch_bounds__(RMS_THREADS) rmsnorm_kernel(const float *__restrict__ x,
                                                               const T *__restrict__ g, int H,
-                                                              float eps, T *__restrict__ out) {
+                                                              float eps, T *__restrict__ out, long lo) {
     wait_prior();
     allow_dependents();
     __shared__ float red[32];
@@ -73,25 +73,25 @@ __global__ void __launch_bounds__(RMS_THREADS) rmsnorm_kernel(const float *__res
         const int j = threadIdx.x + i * RMS_THREADS;
         if (j < n4) {
             const float4 gg = Vec4<T>::load(g + 4 * j);
-            Vec4<T>::store(out + (size_t)r * H + 4 * j,
-                           make_float4(v[i].x * inv * gg.x, v[i].y * inv * gg.y,
-                                       v[i].z * inv * gg.z, v[i].w * inv * gg.w));
+            Split<T>::store4(out + (size_t)r * H + 4 * j, lo,
+                             make_float4(v[i].x * inv * gg.x, v[i].y * inv * gg.y,
+                                         v[i].z * inv * gg.z, v[i].w * inv * gg.w));
         }
     }
 }
 
 template <typename T>
-void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out,
+void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out, long lo,
                     cudaStream_t s) {
     if (R <= 0) return;
-    launch_pdl(rmsnorm_kernel<T>, R, RMS_THREADS, 0, s, x, g, H, eps, out); note_launch();
+    launch_pdl(rmsnorm_kernel<T>, R, RMS_THREADS, 0, s, x, g, H, eps, out, lo); note_launch();
 }
 
 // ---------------------------------------------------------------------------
 // SwiGLU: silu(gate) * up
 // ---------------------------------------------------------------------------
 template <typename T>
-__global__ void swiglu_kernel(const float *__restrict__ gu, int F, int glu, T *__restrict__ act) {
+__global__ void swiglu_kernel(const float *__restrict__ gu, int F, int glu, T *__restrict__ act, long lo) {
     wait_prior();
     allow_dependents();
     const int r = blockIdx.y;
@@ -101,15 +101,15 @@ __global__ void swiglu_kernel(const float *__restrict__ gu, int F, int glu, T *_
         const int gi = glu ? ((j >> 6) << 7) + (j & 63) : j;
         const float g = row[gi], u = row[gi + (glu ? 64 : F)];
         const float sg = g / (1.f + __expf(-g));
-        act[(size_t)r * F + j] = from_f<T>(sg * u);
+        Split<T>::store(act + (size_t)r * F + j, lo, sg * u);
     }
 }
 
 template <typename T>
-void launch_swiglu(const float *gu, int R, int F, bool glu, T *act, cudaStream_t s) {
+void launch_swiglu(const float *gu, int R, int F, bool glu, T *act, long lo, cudaStream_t s) {
     if (R <= 0) return;
     dim3 grid((F + 255) / 256, R);
-    launch_pdl(swiglu_kernel<T>, grid, 256, 0, s, gu, F, glu ? 1 : 0, act); note_launch();
+    launch_pdl(swiglu_kernel<T>, grid, 256, 0, s, gu, F, glu ? 1 : 0, act, lo); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -119,7 +119,7 @@ template <typename T>
 __global__ void rope_kv_kernel(const float *__restrict__ qkv, const RowDesc *__restrict__ rows,
                                int nh, int hd, const float2 *__restrict__ tab, int max_pos,
                                T *__restrict__ q_out, T *__restrict__ kdst, T *__restrict__ vdst,
-                               int slots, int *status) {
+                               int slots, long lo, int *status) {
     wait_prior();
     allow_dependents();
     const int r = blockIdx.x;
@@ -141,15 +141,15 @@ __global__ void rope_kv_kernel(const float *__restrict__ qkv, const RowDesc *__r
         const float2 c = cs[i];
         const int a = h * hd + i, b = a + half;
         const float qa = q[a], qb = q[b];
-        q_out[(size_t)r * H + a] = from_f<T>(qa * c.x - qb * c.y);
-        q_out[(size_t)r * H + b] = from_f<T>(qb * c.x + qa * c.y);
+        Split<T>::store(q_out + (size_t)r * H + a, lo, qa * c.x - qb * c.y);
+        Split<T>::store(q_out + (size_t)r * H + b, lo, qb * c.x + qa * c.y);
         if (write_kv) {
             const float ka = k[a], kb = k[b];
             const size_t base = ((size_t)(d.req * nh + h) * slots + d.dst) * hd;
-            kdst[base + i] = from_f<T>(ka * c.x - kb * c.y);
-            kdst[base + i + half] = from_f<T>(kb * c.x + ka * c.y);
-            vdst[base + i] = from_f<T>(v[a]);
-            vdst[base + i + half] = from_f<T>(v[b]);
+            Split<T>::store(kdst + base + i, lo, ka * c.x - kb * c.y);
+            Split<T>::store(kdst + base + i + half, lo, kb * c.x + ka * c.y);
+            Split<T>::store(vdst + base + i, lo, v[a]);
+            Split<T>::store(vdst + base + i + half, lo, v[b]);
         }
     }
 }
@@ -157,10 +157,10 @@ __global__ void rope_kv_kernel(const float *__restrict__ qkv, const RowDesc *__r
 template <typename T>
 void launch_rope_kv(const float *qkv, const RowDesc *rows, int R, int nh, int hd,
                     const float2 *rope_tab, int max_pos, T *q_out, T *kdst, T *vdst,
-                    int slots, int *status, cudaStream_t s) {
+                    int slots, long lo, int *status, cudaStream_t s) {
     if (R <= 0) return;
     launch_pdl(rope_kv_kernel<T>, R, 256, 0, s, qkv, rows, nh, hd, rope_tab, max_pos, q_out, kdst,
-                                        vdst, slots, status); note_launch();
+                                        vdst, slots, lo, status); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -453,11 +453,11 @@ void launch_flag(int *status, int code, cudaStream_t s) {
 #define MSD_INST(T)                                                                          \
     template void launch_embed_rows<T>(const T *, const T *, const int *, int, int, float *,  \
                                        T *, int, int *, cudaStream_t);                       \
-    template void launch_rmsnorm<T>(const float *, const T *, int, int, float, T *,          \
+    template void launch_rmsnorm<T>(const float *, const T *, int, int, float, T *, long,    \
                                     cudaStream_t);                                           \
-    template void launch_swiglu<T>(const float *, int, int, bool, T *, cudaStream_t);              \
+    template void launch_swiglu<T>(const float *, int, int, bool, T *, long, cudaStream_t);  \
     template void launch_rope_kv<T>(const float *, const RowDesc *, int, int, int,           \
-                                    const float2 *, int, T *, T *, T *, int, int *,          \
+                                    const float2 *, int, T *, T *, T *, int, long, int *,    \
                                     cudaStream_t);                                           \
     template void launch_convert<T>(const float *, T *, long, cudaStream_t);
 MSD_INST(float)

@@ -15,7 +15,7 @@ template <typename T>
 __global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int *__restrict__ n_pend,
                                      const T *__restrict__ pend_h, const int *__restrict__ pend_next,
                                      const T *__restrict__ E, int H, int D1, int V,
-                                     T *__restrict__ xfc, RowDesc *__restrict__ rows, int *status) {
+                                     T *__restrict__ xfc, long lo, RowDesc *__restrict__ rows, int *status) {
     wait_prior();
     allow_dependents();
     const int r = blockIdx.x, b = r / D1, j = r - b * D1;
@@ -36,29 +36,31 @@ __global__ void catchup_setup_kernel(const int *__restrict__ seq_len, const int 
         tok = 0;
     }
     T *dst = xfc + (size_t)r * 2 * H;
-    copy_rows2(dst, valid ? pend_h + (size_t)(b * D1 + j) * H : nullptr, dst + H, E + (size_t)tok * H, H);
+    copy_rows2_split(dst, valid ? pend_h + (size_t)(b * D1 + j) * H : nullptr, lo, dst + H, E + (size_t)tok * H,
+                     H, lo);
 }
 
 // h_hat of the root slot = draft output of the last pending row.
 template <typename T>
 __global__ void root_gather_kernel(const float *__restrict__ x, const int *__restrict__ n_pend, int D1,
-                                   int H, float *__restrict__ hhat_root, T *__restrict__ xr) {
+                                   int H, float *__restrict__ hhat_root, T *__restrict__ xr, long lo) {
     wait_prior();
     allow_dependents();
     const int b = blockIdx.x;
     const int r = b * D1 + max(n_pend[b] - 1, 0);
-    copy_row_2dst(hhat_root + (size_t)b * H, xr + (size_t)b * H, x + (size_t)r * H, H);
+    copy_row_2dst_split(hhat_root + (size_t)b * H, xr + (size_t)b * H, lo, x + (size_t)r * H, H);
 }
 
 // Store h_hat of a tree pass's rows by slot, and a T copy for the LM head.
 template <typename T>
 __global__ void hhat_store_kernel(const float *__restrict__ x, const RowDesc *__restrict__ rows,
-                                  int Td, int H, float *__restrict__ hhat_slot, T *__restrict__ xb) {
+                                  int Td, int H, float *__restrict__ hhat_slot, T *__restrict__ xb, long lo) {
     wait_prior();
     allow_dependents();
     const int r = blockIdx.x;
     const RowDesc d = rows[r];
-    copy_row_2dst(hhat_slot + ((size_t)d.req * Td + d.dst) * H, xb + (size_t)r * H, x + (size_t)r * H, H);
+    copy_row_2dst_split(hhat_slot + ((size_t)d.req * Td + d.dst) * H, xb + (size_t)r * H, lo,
+                        x + (size_t)r * H, H);
 }
 
 // Assemble the draft-pass row j of request b for a frontier node with token
@@ -86,7 +88,7 @@ __device__ void emit_frontier_row(const DraftArgs<T> &a, int b, int j, int tok, 
     }
     if (tok < 0 || tok >= a.V) tok = 0;
     T *dst = a.xfc + (size_t)r * 2 * H;
-    copy_rows2(dst, parent_h, dst + H, a.E + (size_t)tok * H, H);
+    copy_rows2_split(dst, parent_h, 0, dst + H, a.E + (size_t)tok * H, H, a.lo);
 }
 
 // Depth-1 candidates from the root slot's top-k; the frontier of pass 2 is all
@@ -754,7 +756,7 @@ accept_sample_kernel(TreeIn t, const float *__restrict__ logits, const float *__
 __global__ void compact_kv_kernel(const uint4 *__restrict__ tree_kv, uint4 *__restrict__ cache,
                                   const int *__restrict__ acc_path, const int *__restrict__ acc_L0,
                                   const int *__restrict__ acc_a, int B, int nh, int N, int S,
-                                  int D1, int vec_per_row, int *status) {
+                                  int D1, int vec_per_row, long tree_lo, long cache_lo, int *status) {
     wait_prior();
     allow_dependents();
     const int lkh = blockIdx.x, b = blockIdx.y;
@@ -770,7 +772,13 @@ __global__ void compact_kv_kernel(const uint4 *__restrict__ tree_kv, uint4 *__re
     for (int idx = threadIdx.x; idx < total; idx += blockDim.x) {
         const int j = idx / vec_per_row, v = idx - j * vec_per_row;
         const int node = acc_path[b * D1 + j];
-        cache[(cb + L0 + j) * vec_per_row + v] = tree_kv[(tb + node) * vec_per_row + v];
+        const size_t dst = (cb + L0 + j) * vec_per_row + v, src = (tb + node) * vec_per_row + v;
+        const uint4 hi = tree_kv[src];
+        if (tree_lo) {
+            const uint4 lo = tree_kv[src + tree_lo];
+            cache[dst + cache_lo] = lo;
+        }
+        cache[dst] = hi;
     }
 }
 
@@ -778,14 +786,14 @@ __global__ void compact_kv_kernel(const uint4 *__restrict__ tree_kv, uint4 *__re
 template <typename T>
 __global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ acc_path,
                               const int *__restrict__ acc_a, int N, int D1, int H,
-                              T *__restrict__ pend_h) {
+                              T *__restrict__ pend_h, long lo) {
     wait_prior();
     allow_dependents();
     const int b = blockIdx.x / D1, j = blockIdx.x - b * D1;
     if (j > acc_a[b]) return;
     const int node = acc_path[b * D1 + j];
     const T *s = hT + ((size_t)b * N + node) * H;
-    copy_row(pend_h + ((size_t)b * D1 + j) * H, s, H);
+    copy_row_split(pend_h + ((size_t)b * D1 + j) * H, lo, s, lo, H);
 }
 
 // ---------------------------------------------------------------------------
@@ -793,31 +801,32 @@ __global__ void pend_h_kernel(const T *__restrict__ hT, const int *__restrict__ 
 // ---------------------------------------------------------------------------
 // Decoupled draft input (Eq. 7): visual rows take the raw embedding.
 template <typename T>
-__global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict__ emb,
+__global__ void select_visual_kernel(float *__restrict__ x, const T *__restrict__ emb, long slo,
                                      const int *__restrict__ src, int H) {
     wait_prior();
     allow_dependents();
     const int r = blockIdx.x;
     if (src[r] >= 0) return;
-    copy_row(x + (size_t)r * H, emb + (size_t)r * H, H);
+    copy_row_split(x + (size_t)r * H, 0, emb + (size_t)r * H, slo, H);
 }
 
 // Concat(h_i, e_{i+1}) rows for the draft prefill (text positions; visual rows
 // are overwritten after f_down by select_visual_kernel).
 template <typename T>
 __global__ void concat_next_kernel(const T *__restrict__ h, const T *__restrict__ emb, int H,
-                                   T *__restrict__ xfc) {
+                                   T *__restrict__ xfc, long lo) {
     wait_prior();
     allow_dependents();
     const int r = blockIdx.x;
-    copy_rows2(xfc + (size_t)r * 2 * H, h + (size_t)r * H, xfc + (size_t)r * 2 * H + H, emb + (size_t)(r + 1) * H, H);
+    copy_rows2_split(xfc + (size_t)r * 2 * H, h + (size_t)r * H, lo, xfc + (size_t)r * 2 * H + H,
+                     emb + (size_t)(r + 1) * H, H, lo);
 }
 
 template <typename T>
 __global__ void prefill_finish_kernel(const int *__restrict__ argmax1, const T *__restrict__ h_last,
                                       int b, int L, int D1, int H, int *__restrict__ seq_len,
                                       int *__restrict__ n_pend, int *__restrict__ root,
-                                      int *__restrict__ pend_next, T *__restrict__ pend_h,
+                                      int *__restrict__ pend_next, T *__restrict__ pend_h, long lo,
                                       int *__restrict__ root_out) {
     wait_prior();
     const int x = argmax1[0];
@@ -828,7 +837,7 @@ __global__ void prefill_finish_kernel(const int *__restrict__ argmax1, const T *
         pend_next[b * D1] = x;
         if (root_out) root_out[b] = x;
     }
-    copy_row(pend_h + (size_t)b * D1 * H, h_last, H);
+    copy_row_split(pend_h + (size_t)b * D1 * H, lo, h_last, lo, H);
 }
 
 // ---------------------------------------------------------------------------
@@ -837,21 +846,21 @@ __global__ void prefill_finish_kernel(const int *__restrict__ argmax1, const T *
 template <typename T>
 void launch_catchup_setup(const int *seq_len, const int *n_pend, const T *pend_h,
                           const int *pend_next, const T *E, int B, int H, int D1, int V, T *xfc,
-                          RowDesc *rows, int *status, cudaStream_t s) {
+                          long lo, RowDesc *rows, int *status, cudaStream_t s) {
     launch_pdl(catchup_setup_kernel<T>, B * D1, 256, 0, s, seq_len, n_pend, pend_h, pend_next, E, H, D1,
-                                                   V, xfc, rows, status); note_launch();
+                                                   V, xfc, lo, rows, status); note_launch();
 }
 
 template <typename T>
 void launch_root_gather(const float *x, const int *n_pend, int B, int D1, int H, float *hhat_root,
-                        T *xr, cudaStream_t s) {
-    launch_pdl(root_gather_kernel<T>, B, 256, 0, s, x, n_pend, D1, H, hhat_root, xr); note_launch();
+                        T *xr, long lo, cudaStream_t s) {
+    launch_pdl(root_gather_kernel<T>, B, 256, 0, s, x, n_pend, D1, H, hhat_root, xr, lo); note_launch();
 }
 
 template <typename T>
 void launch_hhat_store(const float *x, const RowDesc *rows, int R, int Td, int H,
-                       float *hhat_slot, T *xb, cudaStream_t s) {
-    launch_pdl(hhat_store_kernel<T>, R, 256, 0, s, x, rows, Td, H, hhat_slot, xb); note_launch();
+                       float *hhat_slot, T *xb, long lo, cudaStream_t s) {
+    launch_pdl(hhat_store_kernel<T>, R, 256, 0, s, x, rows, Td, H, hhat_slot, xb, lo); note_launch();
 }
 
 template <typename T>
@@ -935,56 +944,57 @@ bool launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, in
 
 void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, const int *acc_L0,
                        const int *acc_a, int n_layers, int B, int nh, int N, int S, int D1,
-                       int row_bytes, int *status, cudaStream_t s) {
+                       int row_bytes, long lo_bytes, int *status, cudaStream_t s) {
     dim3 grid(n_layers * 2 * nh, B);
+    const long lo_vec = lo_bytes / 16;      // both lo planes sit lo_bytes after their hi planes
     launch_pdl(compact_kv_kernel, grid, 128, 0, s, static_cast<const uint4 *>(tree_kv),
                                            static_cast<uint4 *>(cache), acc_path, acc_L0, acc_a,
-                                           B, nh, N, S, D1, row_bytes / 16, status); note_launch();
+                                           B, nh, N, S, D1, row_bytes / 16, lo_vec, lo_vec, status); note_launch();
 }
 
 template <typename T>
 void launch_pend_h(const T *hT, const int *acc_path, const int *acc_a, int B, int N, int D1,
-                   int H, T *pend_h, cudaStream_t s) {
-    launch_pdl(pend_h_kernel<T>, B * D1, 256, 0, s, hT, acc_path, acc_a, N, D1, H, pend_h); note_launch();
+                   int H, T *pend_h, long lo, cudaStream_t s) {
+    launch_pdl(pend_h_kernel<T>, B * D1, 256, 0, s, hT, acc_path, acc_a, N, D1, H, pend_h, lo); note_launch();
 }
 
 template <typename T>
-void launch_select_visual(float *x, const T *emb, const int *src, int R, int H, cudaStream_t s) {
+void launch_select_visual(float *x, const T *emb, long slo, const int *src, int R, int H, cudaStream_t s) {
     if (R <= 0) return;
-    launch_pdl(select_visual_kernel<T>, R, 256, 0, s, x, emb, src, H); note_launch();
+    launch_pdl(select_visual_kernel<T>, R, 256, 0, s, x, emb, slo, src, H); note_launch();
 }
 
 template <typename T>
-void launch_concat_next(const T *h, const T *emb, int R, int H, T *xfc, cudaStream_t s) {
+void launch_concat_next(const T *h, const T *emb, int R, int H, T *xfc, long lo, cudaStream_t s) {
     if (R <= 0) return;
-    launch_pdl(concat_next_kernel<T>, R, 256, 0, s, h, emb, H, xfc); note_launch();
+    launch_pdl(concat_next_kernel<T>, R, 256, 0, s, h, emb, H, xfc, lo); note_launch();
 }
 
 template <typename T>
 void launch_prefill_finish(const int *argmax1, const T *h_last, int b, int L, int D1, int H,
-                           int *seq_len, int *n_pend, int *root, int *pend_next, T *pend_h,
+                           int *seq_len, int *n_pend, int *root, int *pend_next, T *pend_h, long lo,
                            int *root_out, cudaStream_t s) {
     launch_pdl(prefill_finish_kernel<T>, 1, 256, 0, s, argmax1, h_last, b, L, D1, H, seq_len, n_pend,
-                                               root, pend_next, pend_h, root_out); note_launch();
+                                               root, pend_next, pend_h, lo, root_out); note_launch();
 }
 
 #define MSD_INST(T)                                                                             \
     template void launch_catchup_setup<T>(const int *, const int *, const T *, const int *,     \
-                                          const T *, int, int, int, int, T *, RowDesc *, int *, \
-                                          cudaStream_t);                                        \
+                                          const T *, int, int, int, int, T *, long, RowDesc *,  \
+                                          int *, cudaStream_t);                                 \
     template void launch_root_gather<T>(const float *, const int *, int, int, int, float *, T *, \
-                                        cudaStream_t);                                          \
+                                        long, cudaStream_t);                                    \
     template void launch_hhat_store<T>(const float *, const RowDesc *, int, int, int, float *,  \
-                                       T *, cudaStream_t);                                      \
+                                       T *, long, cudaStream_t);                                \
     template void launch_tree_init<T>(const DraftArgs<T> &, int, cudaStream_t);                 \
     template void launch_tree_step<T>(const DraftArgs<T> &, int, int, cudaStream_t);            \
     template void launch_pend_h<T>(const T *, const int *, const int *, int, int, int, int, T *, \
-                                   cudaStream_t);                                               \
-    template void launch_select_visual<T>(float *, const T *, const int *, int, int,            \
+                                   long, cudaStream_t);                                         \
+    template void launch_select_visual<T>(float *, const T *, long, const int *, int, int,      \
                                           cudaStream_t);                                        \
-    template void launch_concat_next<T>(const T *, const T *, int, int, T *, cudaStream_t);     \
+    template void launch_concat_next<T>(const T *, const T *, int, int, T *, long, cudaStream_t); \
     template void launch_prefill_finish<T>(const int *, const T *, int, int, int, int, int *,   \
-                                           int *, int *, int *, T *, int *, cudaStream_t);
+                                           int *, int *, int *, T *, long, int *, cudaStream_t);
 MSD_INST(float)
 MSD_INST(bf16)
 #undef MSD_INST

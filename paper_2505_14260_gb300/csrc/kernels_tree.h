@@ -22,7 +22,8 @@ struct DraftArgs {
     const float *hhat_slot;                  // [B][Td][H]
     const T *E;
     const int *seq_len;
-    T *xfc;                     // next pass input rows [B*k][2H]
+    T *xfc;                     // next pass input rows [B*k][2H] (split: lo plane at +lo)
+    long lo;
     RowDesc *rows;              // next pass row descriptors [B*k]
     uint64_t *slot_mask;        // [B][Td][Wd]
     uint64_t *row_mask;         // [B*k][Wd]
@@ -40,16 +41,17 @@ struct TreeIn {
     const int *n_nodes;
 };
 
+// `lo`: the lo-plane offset of the split bf16 buffers (0 for fp32 contexts).
 template <typename T>
 void launch_catchup_setup(const int *seq_len, const int *n_pend, const T *pend_h,
                           const int *pend_next, const T *E, int B, int H, int D1, int V, T *xfc,
-                          RowDesc *rows, int *status, cudaStream_t s);
+                          long lo, RowDesc *rows, int *status, cudaStream_t s);
 template <typename T>
 void launch_root_gather(const float *x, const int *n_pend, int B, int D1, int H, float *hhat_root,
-                        T *xr, cudaStream_t s);
+                        T *xr, long lo, cudaStream_t s);
 template <typename T>
 void launch_hhat_store(const float *x, const RowDesc *rows, int R, int Td, int H,
-                       float *hhat_slot, T *xb, cudaStream_t s);
+                       float *hhat_slot, T *xb, long lo, cudaStream_t s);
 template <typename T>
 void launch_tree_init(const DraftArgs<T> &a, int B, cudaStream_t s);
 template <typename T>
@@ -88,19 +90,21 @@ bool launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, in
                           int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
                           int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,
                           int *status, cudaStream_t s);
+// KV compaction; lo_bytes (0: none) = the lo planes' byte offset from their hi planes.
 void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, const int *acc_L0,
                        const int *acc_a, int n_layers, int B, int nh, int N, int S, int D1,
-                       int row_bytes, int *status, cudaStream_t s);
+                       int row_bytes, long lo_bytes, int *status, cudaStream_t s);
 template <typename T>
 void launch_pend_h(const T *hT, const int *acc_path, const int *acc_a, int B, int N, int D1,
-                   int H, T *pend_h, cudaStream_t s);
+                   int H, T *pend_h, long lo, cudaStream_t s);
+// slo: lo plane of emb (0: emb is exact, e.g. the embedding rows)
 template <typename T>
-void launch_select_visual(float *x, const T *emb, const int *src, int R, int H, cudaStream_t s);
+void launch_select_visual(float *x, const T *emb, long slo, const int *src, int R, int H, cudaStream_t s);
 template <typename T>
-void launch_concat_next(const T *h, const T *emb, int R, int H, T *xfc, cudaStream_t s);
+void launch_concat_next(const T *h, const T *emb, int R, int H, T *xfc, long lo, cudaStream_t s);
 template <typename T>
 void launch_prefill_finish(const int *argmax1, const T *h_last, int b, int L, int D1, int H,
-                           int *seq_len, int *n_pend, int *root, int *pend_next, T *pend_h,
+                           int *seq_len, int *n_pend, int *root, int *pend_next, T *pend_h, long lo,
                            int *root_out, cudaStream_t s);
 
 }  // namespace msd

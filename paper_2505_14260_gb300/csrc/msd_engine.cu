@@ -61,6 +61,10 @@ struct msd_ctx {
     bool draft_stale = false;   // msd_ar_step ran: the draft cache no longer follows the target's
     float2 *rope_tab = nullptr;
     void *h_all = nullptr, *emb_all = nullptr;
+    // bf16 contexts: every bf16 buffer that feeds a tensor-core product (and the
+    // KV caches) is carved from one arena whose upper half holds the lo planes
+    // of the split pairs; lo = that half's size in elements (0: fp32 context)
+    long lo = 0;
     int *status = nullptr;
     int *status_host = nullptr;
     cudaEvent_t status_ev = nullptr;
@@ -169,20 +173,27 @@ T *tkv(const msd_ctx *c, void *base, int layer, int kv, int slots) {
 
 // Y (=|+=) X W^T on the dtype's GEMM: tcgen05 tensor cores for bf16, the
 // CUDA-core kernel for fp32.
+// X is a context buffer (its lo plane, if any, sits c->lo elements on) unless
+// `own` is false (a caller-owned operand: hi values only).
 template <typename T>
 void gemm(msd_ctx *c, const T *X, int ldx, int M, int K, const GemmW &W, int O, float *Y,
-          int ldy, int epi, cudaStream_t s);
+          int ldy, int epi, cudaStream_t s, bool own = true);
 
 template <>
 void gemm<float>(msd_ctx *c, const float *X, int ldx, int M, int K, const GemmW &W, int O,
-                 float *Y, int ldy, int epi, cudaStream_t s) {
+                 float *Y, int ldy, int epi, cudaStream_t s, bool) {
     launch_gemm_simt<float>(X, ldx, M, K, W, O, Y, ldy, epi, s);
 }
 
 template <>
 void gemm<bf16>(msd_ctx *c, const bf16 *X, int ldx, int M, int K, const GemmW &W, int O,
-                float *Y, int ldy, int epi, cudaStream_t s) {
-    gemm_bf16(c->gplan, X, ldx, M, K, W, O, Y, ldy, epi, c->status, s);
+                float *Y, int ldy, int epi, cudaStream_t s, bool own) {
+    gemm_bf16(c->gplan, X, own && c->lo ? X + c->lo : nullptr, ldx, M, K, W, O, Y, ldy, epi, c->status, s);
+}
+
+// The lo plane of a context buffer (null for fp32 contexts).
+const bf16 *lo_of(const msd_ctx *c, const void *hi) {
+    return c->lo ? static_cast<const bf16 *>(hi) + c->lo : nullptr;
 }
 
 // One pre-norm decoder layer over R rows (target or draft).
@@ -234,13 +245,14 @@ void qkv_rope(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int
         fx.slots = dst_slots;
         fx.nh = c->nh;
         fx.hd = c->hd;
-        if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), H, R, H, wqkv, 3 * H, fx,
-                            c->status, s, norm_in))
+        fx.lo = c->lo;
+        if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), lo_of(c, c->xn), H, R, H, wqkv, 3 * H,
+                            fx, c->status, s, norm_in))
             return;
     }
     gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wqkv, 3 * H, c->qkv, 3 * H, EPI_STORE, s);
     launch_rope_kv<T>(c->qkv, rows, R, c->nh, c->hd, c->rope_tab, c->S, static_cast<T *>(c->q),
-                      kdst, vdst, dst_slots, c->status, s);
+                      kdst, vdst, dst_slots, c->lo, c->status, s);
 }
 
 // act = silu(xn wg^T) * (xn wu^T). bf16 contexts hold gate/up glu-packed; the
@@ -257,15 +269,16 @@ void gate_up_swiglu(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &l
         fx.epi = EPI_SWIGLU;
         fx.act = static_cast<bf16 *>(c->act);
         fx.F = F;
-        if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), H, R, H, wgu, O, fx, c->status, s,
-                            norm_in))
+        fx.lo = c->lo;
+        if (gemm_bf16_fused(c->gplan, static_cast<const bf16 *>(c->xn), lo_of(c, c->xn), H, R, H, wgu, O, fx,
+                            c->status, s, norm_in))
             return;
         gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wgu, O, c->gu, O, EPI_STORE, s);
-        launch_swiglu<T>(c->gu, R, F, true, static_cast<T *>(c->act), s);
+        launch_swiglu<T>(c->gu, R, F, true, static_cast<T *>(c->act), c->lo, s);
     } else {
         GemmW wgu = {{lw.w_gate, lw.w_up, nullptr}, {F, F, 0}, 2, nullptr};
         gemm<T>(c, static_cast<const T *>(c->xn), H, R, H, wgu, 2 * F, c->gu, 2 * F, EPI_STORE, s);
-        launch_swiglu<T>(c->gu, R, F, false, static_cast<T *>(c->act), s);
+        launch_swiglu<T>(c->gu, R, F, false, static_cast<T *>(c->act), c->lo, s);
     }
 }
 
@@ -279,11 +292,11 @@ bool folds(const msd_ctx *c, int R, const void *packed) {
 
 GemmNorm norm_out(msd_ctx *c, const void *g) {
     return GemmNorm{c->ss_part, c->ss_ld, static_cast<bf16 *>(c->xn), static_cast<const bf16 *>(g),
-                    0, c->H, c->cfg.rms_eps};
+                    0, c->H, c->cfg.rms_eps, c->lo};
 }
 
 GemmNorm norm_in(msd_ctx *c) {
-    return GemmNorm{c->ss_part, c->ss_ld, nullptr, nullptr, c->ss_ld, c->H, c->cfg.rms_eps};
+    return GemmNorm{c->ss_part, c->ss_ld, nullptr, nullptr, c->ss_ld, c->H, c->cfg.rms_eps, c->lo};
 }
 
 // One pre-norm decoder layer over R rows (target or draft). Rows come in
@@ -303,7 +316,7 @@ bool run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, in
     const GemmNorm nin = norm_in(c);
     if (!(fold && in_folded))
         launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.attn_norm), R, H, eps,
-                          static_cast<T *>(c->xn), s);
+                          static_cast<T *>(c->xn), c->lo, s);
     qkv_rope<T>(c, lw, lp, R, rows, kdst, vdst, dst_slots, s, fold && in_folded ? &nin : nullptr);
     AttnArgs<T> a;
     a.q = static_cast<const T *>(c->q);
@@ -322,19 +335,20 @@ bool run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, in
     a.scale = 1.0f / sqrtf((float)c->hd);
     a.out = static_cast<T *>(c->attn);
     a.cache_fresh = kdst == ck;         // this layer's own K/V go into the cache it reads
+    a.lo = c->lo;
     attention<T>(c, a, rows_per_req, p_bound, s);
     GemmW wo = {{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1, lp.o};
     GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, lp.down};
     if constexpr (std::is_same<T, bf16>::value) {
         if (fold) {
             const GemmNorm no = norm_out(c, lw.mlp_norm);
-            gemm_bf16(c->gplan, static_cast<const bf16 *>(c->attn), H, R, H, wo, H, c->x, H, EPI_ADD,
-                      c->status, s, &no);
+            gemm_bf16(c->gplan, static_cast<const bf16 *>(c->attn), lo_of(c, c->attn), H, R, H, wo, H, c->x, H,
+                      EPI_ADD, c->status, s, &no);
             gate_up_swiglu<T>(c, lw, lp, R, s, &nin);
             if (out_norm_g) {
                 const GemmNorm nd = norm_out(c, out_norm_g);
-                gemm_bf16(c->gplan, static_cast<const bf16 *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD,
-                          c->status, s, &nd);
+                gemm_bf16(c->gplan, static_cast<const bf16 *>(c->act), lo_of(c, c->act), F, R, F, wd, H, c->x, H,
+                          EPI_ADD, c->status, s, &nd);
                 return true;
             }
             gemm<T>(c, static_cast<const T *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD, s);
@@ -343,7 +357,7 @@ bool run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, in
     }
     gemm<T>(c, static_cast<const T *>(c->attn), H, R, H, wo, H, c->x, H, EPI_ADD, s);
     launch_rmsnorm<T>(c->x, static_cast<const T *>(lw.mlp_norm), R, H, eps,
-                      static_cast<T *>(c->xn), s);
+                      static_cast<T *>(c->xn), c->lo, s);
     gate_up_swiglu<T>(c, lw, lp, R, s);
     gemm<T>(c, static_cast<const T *>(c->act), F, R, F, wd, H, c->x, H, EPI_ADD, s);
     return false;
@@ -362,8 +376,8 @@ bool draft_fc(msd_ctx *c, int R, cudaStream_t s) {
     if constexpr (std::is_same<T, bf16>::value) {
         if (folds(c, R, c->pk_fc) && c->dpack.o) {
             const GemmNorm no = norm_out(c, c->w.draft.attn_norm);
-            return gemm_bf16(c->gplan, static_cast<const bf16 *>(c->xfc), 2 * H, R, 2 * H, W, H, c->x, H,
-                             EPI_STORE, c->status, s, &no);
+            return gemm_bf16(c->gplan, static_cast<const bf16 *>(c->xfc), lo_of(c, c->xfc), 2 * H, R, 2 * H, W,
+                             H, c->x, H, EPI_STORE, c->status, s, &no);
         }
     }
     gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, R, 2 * H, W, H, c->x, H, EPI_STORE, s);
@@ -415,7 +429,7 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
                              nullptr, 0, nullptr, 0, n, r0 + n, s);
             }
             launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), n, H, c->cfg.rms_eps,
-                              static_cast<T *>(c->h_all) + (size_t)r0 * H, s);
+                              static_cast<T *>(c->h_all) + (size_t)r0 * H, c->lo, s);
             CU(cudaStreamSynchronize(s));   // rd/src host vectors are reused
         }
         const T *h_last = static_cast<const T *>(c->h_all) + (size_t)(L - 1) * H;
@@ -431,12 +445,13 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
             CU(cudaMemcpyAsync(c->rows, rd.data(), sizeof(RowDesc) * n, cudaMemcpyHostToDevice, s));
             launch_concat_next<T>(static_cast<const T *>(c->h_all) + (size_t)r0 * H,
                                   static_cast<const T *>(c->emb_all) + (size_t)r0 * H, n, H,
-                                  static_cast<T *>(c->xfc), s);
+                                  static_cast<T *>(c->xfc), c->lo, s);
             gemm<T>(c, static_cast<const T *>(c->xfc), 2 * H, n, 2 * H, one(c->w.draft_fc, H, c->pk_fc), H,
                     c->x, H, EPI_STORE, s);
             if (c->cfg.draft_input != MSD_DRAFT_CONCAT) {
-                const void *vis_rows = c->cfg.draft_input == MSD_DRAFT_FEATURE ? c->h_all : c->emb_all;
-                launch_select_visual<T>(c->x, static_cast<const T *>(vis_rows) + (size_t)r0 * H,
+                const bool feat = c->cfg.draft_input == MSD_DRAFT_FEATURE;
+                const void *vis_rows = feat ? c->h_all : c->emb_all;
+                launch_select_visual<T>(c->x, static_cast<const T *>(vis_rows) + (size_t)r0 * H, feat ? c->lo : 0,
                                         c->src + r0, n, H, s);
             }
             T *K = tkv<T>(c, c->draft_kv, 0, 0, c->S), *Vv = tkv<T>(c, c->draft_kv, 0, 1, c->S);
@@ -445,7 +460,7 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
             CU(cudaStreamSynchronize(s));
         }
         launch_prefill_finish<T>(c->argmax_tmp, h_last, b, L, D1, H, c->seq_len, c->n_pend, c->root,
-                                 c->pend_next, static_cast<T *>(c->pend_h), root_out, s);
+                                 c->pend_next, static_cast<T *>(c->pend_h), c->lo, root_out, s);
         c->L_bound[b] = L;
     }
     c->prefilled = true;
@@ -469,6 +484,7 @@ DraftArgs<T> draft_args(msd_ctx *c) {
     a.E = static_cast<const T *>(c->w.embed);
     a.seq_len = c->seq_len;
     a.xfc = static_cast<T *>(c->xfc);
+    a.lo = c->lo;
     a.rows = c->rows;
     a.slot_mask = c->slot_mask;
     a.row_mask = c->row_mask;
@@ -504,12 +520,12 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
     // pass 1: catch-up rows + root slot
     const int R1 = B * D1;
     launch_catchup_setup<T>(c->seq_len, c->n_pend, static_cast<const T *>(c->pend_h), c->pend_next,
-                            E, B, H, D1, V, static_cast<T *>(c->xfc), c->rows, c->status, s);
+                            E, B, H, D1, V, static_cast<T *>(c->xfc), c->lo, c->rows, c->status, s);
     bool folded = draft_fc<T>(c, R1, s);
     const int pb = max_L_bound(c);
     run_layer<T>(c, c->w.draft, c->dpack, R1, c->rows, dK, dV, S, dK, dV, S, nullptr, nullptr, 0, nullptr, 0,
                  D1, pb, s, folded);
-    launch_root_gather<T>(c->x, c->n_pend, B, D1, H, c->hhat_root, static_cast<T *>(c->xr), s);
+    launch_root_gather<T>(c->x, c->n_pend, B, D1, H, c->hhat_root, static_cast<T *>(c->xr), c->lo, s);
     gemm<T>(c, static_cast<const T *>(c->xr), H, B, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V,
             EPI_STORE, s);
     launch_topk_logp(c->logits, B, V, k, c->topk_ids, c->topk_logp, c->tks, s);
@@ -523,7 +539,7 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
         folded = draft_fc<T>(c, Rk, s);
         run_layer<T>(c, c->w.draft, c->dpack, Rk, c->rows, tK, tV, c->Td, dK, dV, S, tK, tV, c->Td,
                      c->row_mask, c->Wd, k, pb, s, folded);
-        launch_hhat_store<T>(c->x, c->rows, Rk, c->Td, H, c->hhat_slot, static_cast<T *>(c->xr), s);
+        launch_hhat_store<T>(c->x, c->rows, Rk, c->Td, H, c->hhat_slot, static_cast<T *>(c->xr), c->lo, s);
         gemm<T>(c, static_cast<const T *>(c->xr), H, Rk, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V,
                 EPI_STORE, s);
         launch_topk_logp(c->logits, Rk, V, k, c->topk_ids, c->topk_logp, c->tks, s);
@@ -558,7 +574,7 @@ msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, fl
                               c->vmask, c->W, N, pb, s, folded, next_g);
     }
     launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), R, H, c->cfg.rms_eps,
-                      static_cast<T *>(c->hT), s);
+                      static_cast<T *>(c->hT), c->lo, s);
     float *lg = logits_dev ? logits_dev : c->logits;
     gemm<T>(c, static_cast<const T *>(c->hT), H, R, H, one(c->w.lm_head, V, c->pk_lm), V, lg, V, EPI_STORE,
             s);
@@ -572,9 +588,9 @@ msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, fl
 template <typename T>
 msd_status compact_impl(msd_ctx *c, cudaStream_t s, int grow) {
     launch_compact_kv(c->tree_kv, c->target_kv, c->acc_path, c->acc_L0, c->acc_a, c->NL, c->B, c->nh,
-                      c->N, c->S, c->D1, (int)(c->hd * c->esz), c->status, s);
+                      c->N, c->S, c->D1, (int)(c->hd * c->esz), c->lo * (long)c->esz, c->status, s);
     launch_pend_h<T>(static_cast<const T *>(c->hT), c->acc_path, c->acc_a, c->B, c->N, c->D1, c->H,
-                     static_cast<T *>(c->pend_h), s);
+                     static_cast<T *>(c->pend_h), c->lo, s);
     if (!c->capturing)
         for (int b = 0; b < c->B; ++b) c->L_bound[b] += grow < 0 ? c->D1 : grow;
     return post_status(c, s);
@@ -772,26 +788,51 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     c->L_bound.assign(c->B, 0);
     const size_t e = c->esz, H = c->H, F = c->F, R = c->Rmax;
     bool ok = true;
-    ok &= dalloc(c, &c->target_kv, (size_t)c->NL * 2 * kv_layer_elems(c, c->S) * e);
-    ok &= dalloc(c, &c->draft_kv, 2 * kv_layer_elems(c, c->S) * e);
-    ok &= dalloc(c, &c->tree_kv, (size_t)c->NL * 2 * kv_layer_elems(c, c->N) * e);
-    ok &= dalloc(c, &c->dtree_kv, 2 * kv_layer_elems(c, c->Td) * e);
+    // Buffers in the model dtype. In bf16 contexts they are split pairs: one
+    // arena holds them all, and its upper half (lo elements on) their lo planes.
+    struct Carve { void **p; size_t elems; };
+    const Carve split_bufs[] = {
+        {&c->target_kv, (size_t)c->NL * 2 * kv_layer_elems(c, c->S)},
+        {&c->draft_kv, 2 * kv_layer_elems(c, c->S)},
+        {&c->tree_kv, (size_t)c->NL * 2 * kv_layer_elems(c, c->N)},
+        {&c->dtree_kv, 2 * kv_layer_elems(c, c->Td)},
+        {&c->pend_h, (size_t)c->B * c->D1 * H},
+        {&c->xn, R * H},
+        {&c->q, R * H},
+        {&c->attn, R * H},
+        {&c->act, R * F},
+        {&c->xfc, R * 2 * H},
+        {&c->xr, R * H},
+        {&c->hT, (size_t)c->B * c->N * H},
+        {&c->h_all, (size_t)c->S * H},
+    };
+    if (cfg->dtype == MSD_BF16) {
+        size_t total = 0;
+        for (const Carve &b : split_bufs) total += (b.elems + 127) / 128 * 128;     // 256-byte pieces
+        const size_t quantum = H * 64;      // the lo offset is a whole number of rows of any buffer
+        total = (total + quantum - 1) / quantum * quantum;
+        void *arena = nullptr;
+        ok &= dalloc(c, &arena, 2 * total * e);
+        if (ok) {
+            size_t off = 0;
+            for (const Carve &b : split_bufs) {
+                *b.p = static_cast<bf16 *>(arena) + off;
+                off += (b.elems + 127) / 128 * 128;
+            }
+            c->lo = (long)total;
+        }
+    } else {
+        for (const Carve &b : split_bufs) ok &= dalloc(c, b.p, b.elems * e);
+    }
     ok &= dalloc(c, &c->seq_len, sizeof(int) * c->B);
     ok &= dalloc(c, &c->n_pend, sizeof(int) * c->B);
     ok &= dalloc(c, &c->root, sizeof(int) * c->B);
     ok &= dalloc(c, &c->pend_next, sizeof(int) * c->B * c->D1);
-    ok &= dalloc(c, &c->pend_h, (size_t)c->B * c->D1 * H * e);
     ok &= dalloc(c, &c->x, R * H * 4);
-    ok &= dalloc(c, &c->xn, R * H * e);
     ok &= dalloc(c, &c->qkv, R * 3 * H * 4);
-    ok &= dalloc(c, &c->q, R * H * e);
-    ok &= dalloc(c, &c->attn, R * H * e);
     c->ss_ld = (H + 127) / 128;
     ok &= dalloc(c, &c->ss_part, R * (size_t)c->ss_ld * 4);
     ok &= dalloc(c, &c->gu, R * std::max<size_t>(2 * F, glu_rows(c->F)) * 4);
-    ok &= dalloc(c, &c->act, R * F * e);
-    ok &= dalloc(c, &c->xfc, R * 2 * H * e);
-    ok &= dalloc(c, &c->xr, R * H * e);
     ok &= dalloc(c, &c->logits, (size_t)c->Rlog * c->V * 4);
     ok &= dalloc(c, &c->argmax_tmp, sizeof(int) * 4);
     ok &= dalloc(c, &c->rows, sizeof(RowDesc) * R);
@@ -811,7 +852,6 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     ok &= dalloc(c, &c->topk_logp, sizeof(float) * c->Rlog * c->k);
     ok &= dalloc(c, &c->tks.ws, sizeof(float) * topk_scratch_floats(c->Rlog, c->V));
     ok &= dalloc(c, &c->tks.counters, sizeof(int) * c->Rlog);
-    ok &= dalloc(c, &c->hT, (size_t)c->B * c->N * H * e);
     ok &= dalloc(c, &c->acc_path, sizeof(int) * c->B * c->D1);
     ok &= dalloc(c, &c->acc_L0, sizeof(int) * c->B);
     ok &= dalloc(c, &c->acc_a, sizeof(int) * c->B);
@@ -824,13 +864,15 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     ok &= dalloc(c, &c->ar_tree.n_nodes, sizeof(int) * c->B);
     ok &= dalloc(c, &c->ar_argmax, sizeof(int) * c->B * c->N);
     ok &= dalloc(c, &c->rope_tab, sizeof(float2) * (size_t)c->S * (c->hd / 2));
-    ok &= dalloc(c, &c->h_all, (size_t)c->S * H * e);
     ok &= dalloc(c, &c->emb_all, (size_t)c->S * H * e);
     ok &= dalloc(c, &c->status, sizeof(int));
     if (ok) ok = cudaMallocHost(&c->status_host, sizeof(int)) == cudaSuccess;
     if (ok) ok = cudaEventCreateWithFlags(&c->status_ev, cudaEventDisableTiming) == cudaSuccess;
     if (ok && cfg->dtype == MSD_BF16) ok = gemm_plan_create(&c->gplan, c->Rmax, c->H, c->F, c->V);
-    if (ok && cfg->dtype == MSD_BF16) ok = attn_tc_plan_create(&c->aplan, c->S);
+    if (ok && cfg->dtype == MSD_BF16) {
+        const int decode_rows = std::max(c->N, std::max(c->k, c->D1));
+        ok = attn_tc_plan_create(&c->aplan, c->S, c->B * ((decode_rows + 63) / 64) * c->nh);
+    }
     c->lpack.assign(c->NL, msd_ctx::LayerPack());
     if (ok && cfg->dtype == MSD_BF16) ok = pack_weights(c);
     if (!ok) {
@@ -1195,7 +1237,7 @@ msd_status msd_linear(msd_ctx *c, const void *x, int32_t ldx, int32_t m, int32_t
         }
         gemm_pack(W, k, c->pk_scratch, s);
         W.packed = c->pk_scratch;
-        gemm<bf16>(c, static_cast<const bf16 *>(x), ldx, m, k, W, o, y, ldy, epi, s);
+        gemm<bf16>(c, static_cast<const bf16 *>(x), ldx, m, k, W, o, y, ldy, epi, s, false);
     } else
         gemm<float>(c, static_cast<const float *>(x), ldx, m, k, W, o, y, ldy, epi, s);
     return post_status(c, s);
@@ -1255,6 +1297,7 @@ msd_status msd_state(msd_ctx *c, msd_state_view *out) {
     out->n_pending = c->n_pend;
     out->root = c->root;
     out->elem_bytes = (int64_t)c->esz;
+    out->lo_offset = (int64_t)c->lo;
     return MSD_OK;
 }
 

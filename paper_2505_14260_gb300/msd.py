@@ -53,7 +53,8 @@ class msd_draft_record(ctypes.Structure):
 
 class msd_state_view(ctypes.Structure):
     _fields_ = [("target_kv", c_void_p), ("draft_kv", c_void_p), ("seq_len", c_void_p),
-                ("n_pending", c_void_p), ("root", c_void_p), ("elem_bytes", c_int64)]
+                ("n_pending", c_void_p), ("root", c_void_p), ("elem_bytes", c_int64),
+                ("lo_offset", c_int64)]
 
 
 class msd_profile(ctypes.Structure):
@@ -332,13 +333,19 @@ class Engine:
         c = self.cfg
         dt = torch.bfloat16 if c.dtype == MSD_BF16 else torch.float32
         B, nh, S, hd = c.max_batch, c.n_heads, c.max_seq, c.head_dim
-        return {
+        out = {
             "target_kv": device_view(v.target_kv, (c.n_layers, 2, B, nh, S, hd), dt),
             "draft_kv": device_view(v.draft_kv, (2, B, nh, S, hd), dt),
             "seq_len": device_view(v.seq_len, (B,), torch.int32),
             "n_pending": device_view(v.n_pending, (B,), torch.int32),
             "root": device_view(v.root, (B,), torch.int32),
+            "lo_offset": int(v.lo_offset),
         }
+        if v.lo_offset:     # bf16: the lo planes of the split cache entries
+            eb = int(v.elem_bytes)
+            out["target_kv_lo"] = device_view(v.target_kv + v.lo_offset * eb, (c.n_layers, 2, B, nh, S, hd), dt)
+            out["draft_kv_lo"] = device_view(v.draft_kv + v.lo_offset * eb, (2, B, nh, S, hd), dt)
+        return out
 
 
 def make_config(wl, max_seq: int, batch: int | None = None) -> msd_config:

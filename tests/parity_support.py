@@ -19,17 +19,25 @@ from tests.gpu_support import (KV_REL_L2, TOL, abs_bound, assert_close, open_eng
 from tests.oracle_support import oracle_model, prompt_numpy
 
 
+def cache_values(s, name, idx):
+    """The cached values at idx: fp32 entries, or hi + lo of bf16 split pairs."""
+    v = s[name][idx].double()
+    if s.get("lo_offset"):
+        v = v + s[name + "_lo"][idx].double()
+    return v.cpu().numpy()
+
+
 def kv_compare(eng, st, wl, b, L, kv_tol, what):
     s = eng.state()
     nh, hd = wl.n_heads, wl.head_dim
     for l in range(wl.n_layers):
         for kv, ref in ((0, st.K[l]), (1, st.V[l])):
-            g = s["target_kv"][l, kv, b, :, :L, :].float().cpu().numpy()      # [nh, L, hd]
+            g = cache_values(s, "target_kv", (l, kv, b, slice(None), slice(0, L), slice(None)))   # [nh, L, hd]
             r = np.asarray(ref[:L]).reshape(L, nh, hd).transpose(1, 0, 2)
             assert rel_l2(g, r) <= kv_tol, f"{what} layer {l} kv {kv}: {rel_l2(g, r)}"
     Ld = st.dK.shape[0]
     for kv, ref in ((0, st.dK), (1, st.dV)):
-        g = s["draft_kv"][kv, b, :, :Ld, :].float().cpu().numpy()
+        g = cache_values(s, "draft_kv", (kv, b, slice(None), slice(0, Ld), slice(None)))
         r = np.asarray(ref).reshape(Ld, nh, hd).transpose(1, 0, 2)
         assert rel_l2(g, r) <= kv_tol, f"{what} draft kv {kv}: {rel_l2(g, r)}"
 

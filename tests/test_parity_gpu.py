@@ -232,6 +232,8 @@ def test_step_graph_matches_separate_calls():
     sa, sb = ea.state(), eb.state()
     assert torch.equal(sa["seq_len"], sb["seq_len"]) and int(sa["seq_len"][0]) > 512
     L = int(sa["seq_len"][0])
-    assert torch.equal(sa["target_kv"][..., :L, :], sb["target_kv"][..., :L, :])
-    assert torch.equal(sa["draft_kv"][..., :L - 8, :], sb["draft_kv"][..., :L - 8, :])
+    for name in [n for n in ("target_kv", "target_kv_lo") if n in sa]:   # hi and lo planes
+        assert torch.equal(sa[name][..., :L, :], sb[name][..., :L, :]), name
+    for name in [n for n in ("draft_kv", "draft_kv_lo") if n in sa]:
+        assert torch.equal(sa[name][..., :L - 8, :], sb[name][..., :L - 8, :]), name
     ea.close(); eb.close()

@@ -212,7 +212,8 @@ def test_step_sample_graph_matches_separate_calls():
     sa, sb = ea.state(), eb.state()
     L = int(sa["seq_len"][0])
     assert torch.equal(sa["seq_len"], sb["seq_len"]) and torch.equal(sa["root"], sb["root"])
-    assert torch.equal(sa["target_kv"][..., :L, :], sb["target_kv"][..., :L, :])
+    for name in [n for n in ("target_kv", "target_kv_lo") if n in sa]:   # hi and lo planes
+        assert torch.equal(sa[name][..., :L, :], sb[name][..., :L, :]), name
     ea.close(); eb.close()
 
 
