@@ -5,25 +5,14 @@ import torch
 
 from paper_2505_14260_gb300 import msd, synth
 
-# Tolerances. bf16 against the float64 oracle: the stated bound for the
-# logits (max |d| <= 3e-2 and relative L2 <= 1e-2). fp32: float32 rounding of
-# a float64 computation over two layers.
+# Tolerances against the float64 oracle. bf16 workloads: the stated bound for
+# the logits, max |d| <= 3e-2 and relative L2 <= 1e-2, at every width (the
+# split-bf16 activations and caches carry each value to about 2^-17, so the
+# measured errors sit orders of magnitude below it). fp32: float32 rounding of
+# a float64 computation over two layers. KV caches (hi + lo of each entry for
+# bf16): relative L2 <= 1e-3 -- a check of our own, not a stated bound.
 TOL = {"f32": dict(max_abs=2e-4, rel_l2=1e-5), "bf16": dict(max_abs=3e-2, rel_l2=1e-2)}
-KV_REL_L2 = {"f32": 1e-5, "bf16": 1e-2}
-
-# Full-width bf16 (hidden 4096-5120, vocabulary 32000): the stated absolute
-# bound does not hold there. Every activation that enters a tensor-core
-# operation is rounded to bf16 (relative error <= 2^-8, RMS about 2.3e-3): the
-# normalised input, q/k/v and the KV cache, the softmax weights, the attention
-# and MLP outputs, the LM head and f_down inputs, about 15 roundings over a
-# two-layer pass, which combine to ~9e-3 (relative L2 of the logits). The draft
-# feeds its own un-normalised feature back at every pass, so pass p carries
-# the errors of p + 1 passes (x sqrt(6) ~ 2.4 at the sixth), and its logits
-# reach magnitudes of 15 .. 70. Bound, with a 1.5x margin: relative L2 <=
-# 3e-2 and max |d| <= 4e-2 of the block's largest reference logit (measured
-# at 7B: 1.1e-2 verify, 1.6e-2 .. 2.1e-2 draft; 13B up to 2.5e-2).
-TOL_FULL = dict(max_abs=4e-2, rel_l2=3e-2, relative=True)
-KV_REL_L2_FULL = 3e-2
+KV_REL_L2 = {"f32": 1e-5, "bf16": 1e-3}
 
 
 def to_device(w: dict, device="cuda") -> dict:
@@ -51,10 +40,7 @@ def rel_l2(a, b) -> float:
 
 
 def abs_bound(ref, tol) -> float:
-    """The max |d| bound for a reference block: absolute, or (full width)
-    relative to the block's largest magnitude."""
-    if tol.get("relative"):
-        return tol["max_abs"] * max(1.0, float(np.max(np.abs(ref))) if np.size(ref) else 1.0)
+    """The max |d| bound of a block (absolute)."""
     return tol["max_abs"]
 
 
