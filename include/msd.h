@@ -11,7 +11,14 @@
  * - Weight matrices are [out, in] row-major (in contiguous), in the dtype of
  *   msd_config.dtype; norm gains are [hidden] vectors of the same dtype.
  *   Weights are BORROWED: the caller keeps them alive and unchanged for the
- *   lifetime of the context.
+ *   lifetime of the context. Exception: a bf16 context (MSD_BF16) packs every
+ *   projection matrix -- the target layers' and the draft layer's wq, wk, wv,
+ *   wo, w_gate, w_up and w_down, plus lm_head and draft_fc -- into
+ *   context-owned tile-contiguous copies during msd_create and never reads
+ *   those borrowed matrices again, so the caller may free them once
+ *   msd_create has returned (the copies take as many bytes as the matrices).
+ *   embed and the norm gains stay borrowed. An fp32 context reads every
+ *   borrowed weight on every call.
  * - The context OWNS its KV caches, tree scratch and activations (allocated
  *   once in msd_create; no call allocates afterwards).
  * - Output buffers are caller-owned device memory.
@@ -336,21 +343,45 @@ msd_status msd_test_wait_timeout(msd_ctx *ctx, int64_t limit_ns, void *stream);
 
 /* Profiling counters (tracing subsystem). kernel_launches counts every kernel
  * the library has run in this process (kernels executed by step graphs
- * included, kernels merely recorded into graphs excluded). While profiling is enabled on a
- * context, each tensor-core GEMM launch (bf16 contexts) is bracketed by CUDA
- * events on its own stream; msd_profile_read synchronises on them and returns
- * the number of timed launches, their summed durations, and their algorithmic
- * bytes (every weight element once + activations read + fp32 output written,
- * read too when accumulating), then starts a new window. */
+ * included, kernels merely recorded into graphs excluded).
+ *
+ * msd_profile_enable(ctx, mode) times the tensor-core GEMM launches of a bf16
+ * context:
+ *   mode 0  off.
+ *   mode 1  each GEMM launch is bracketed by CUDA events on its own stream;
+ *           step calls run as separate launches instead of their graphs.
+ *           gemm_ms = the events' summed durations.
+ *   mode 2  step calls replay graphs recorded with launch stamps: each CTA of
+ *           a GEMM launch stamps a device slot with %globaltimer (earliest
+ *           entry, earliest return from the wait on the previous kernel,
+ *           latest exit) and the graph's last kernel adds the step's spans to
+ *           a device sum, so the step runs as it does unprofiled (the same
+ *           graph, programmatic dependent launches included) plus those atomics.
+ *           gemm_ms = sum of exit - entry over launches; gemm_critical_ms =
+ *           sum of exit - wait (these intervals are disjoint for the kernels of
+ *           one stream, so their sum never exceeds the steps' time); windows =
+ *           steps measured. Stamped graphs are cached apart from the others.
+ * msd_profile_read synchronises the device, returns the launches timed since
+ * the last read, their time and their algorithmic bytes (every weight element
+ * once + activations read + output written, read too when accumulating), and
+ * starts a new window. Enabling either mode also starts a new window.
+ * Errors: MSD_ERR_INVALID (mode out of range), MSD_ERR_CUDA (mode 2 buffers). */
 typedef struct {
     int64_t kernel_launches;
     int64_t gemm_launches;
     double gemm_ms;
     double gemm_bytes;
     double gemm_weight_bytes;
+    double gemm_critical_ms;
+    int64_t windows;
+    double gemm_flops;       /* 2 x rows x outputs x inner size, summed */
+    double gemm_mma_flops;   /* as issued to the tensor cores: twice gemm_flops
+                                for launches whose token operand is a split pair */
+    double gemm_prefetch_bytes; /* weight bytes the launches request before they
+                                   wait for the previous kernel (part of gemm_bytes) */
 } msd_profile;
 
-msd_status msd_profile_enable(msd_ctx *ctx, int32_t on);
+msd_status msd_profile_enable(msd_ctx *ctx, int32_t mode);
 msd_status msd_profile_read(msd_ctx *ctx, msd_profile *out);
 
 /* Device pointers of the context state (see msd_state_view). */

@@ -69,6 +69,16 @@ __device__ __forceinline__ unsigned long long gtimer() {
     return t;
 }
 
+// Launch stamps (profiling): [0] the earliest CTA entry, [1] the earliest
+// return from griddepcontrol.wait (the previous kernel's results are visible),
+// [2] the latest CTA exit, in %globaltimer nanoseconds.
+__device__ __forceinline__ void stamp_min(unsigned long long *st, int i) {
+    if (st) atomicMin(st + i, gtimer());
+}
+__device__ __forceinline__ void stamp_max(unsigned long long *st, int i) {
+    if (st) atomicMax(st + i, gtimer());
+}
+
 __device__ __forceinline__ void mbar_init(uint32_t bar, uint32_t count) {
     asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count));
 }
@@ -401,6 +411,7 @@ struct PkParams {
     uint32_t stg_off;       // EPI_SWIGLU: byte offset of the 16 KB staging tile
     int has_lo;             // X is a split pair: its lo plane comes through the second map
     long lo;                // lo-plane offset of act (elements)
+    unsigned long long *stamp;   // launch stamps (entry, wait, exit ns) or null
 };
 
 // silu(g) * u, the SwiGLU product of the fused epilogues.
@@ -466,6 +477,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
     const uint32_t drain = smem_u32(&bars[2 * P_MAX_STAGES + 4]);
 
     if (threadIdx.x == 0) {
+        stamp_min(p.stamp, 0);
         for (int s = 0; s < stages; ++s) {
             mbar_init(full0 + 8 * s, 1);
             mbar_init(empty0 + 8 * s, 1);
@@ -523,6 +535,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
                 }
             }
             pdl_wait();
+            stamp_min(p.stamp, 1);
             pdl_trigger();
             ItemIter it = items0;
             int t, kb_b, kb_e, s = 0, i = 0;
@@ -775,6 +788,7 @@ __global__ void __launch_bounds__(P_THREADS, 1)
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
+    if (threadIdx.x == 0) stamp_max(p.stamp, 2);
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
@@ -812,6 +826,7 @@ struct CkParams {
     int *status;
     GemmFused fx;           // EPI_SWIGLU / EPI_ROPE_KV operands
     GemmNorm nout, nin;     // folded RMSNorm: producer / consumer side (ss null: off)
+    unsigned long long *stamp;   // launch stamps (entry, wait, exit ns) or null
 };
 
 __device__ __forceinline__ void c_cluster_sync() {
@@ -1165,6 +1180,7 @@ __global__ void __launch_bounds__(C_THREADS)
     const uint32_t recv_bar = smem_u32(&bars[2 * C_STAGES + 1]);   // the other ranks' slices have landed
 
     if (threadIdx.x == 0) {
+        stamp_min(p.stamp, 0);
         for (int s = 0; s < stages; ++s) {
             mbar_init(full0 + 8 * s, 1);
             mbar_init(empty0 + 8 * s, 1);
@@ -1197,6 +1213,7 @@ __global__ void __launch_bounds__(C_THREADS)
                 bulk_load(a_base + j * A_BYTES, wblk + (size_t)j * blk_elems, A_BYTES, full0 + 8 * j);
             }
             pdl_wait();
+            stamp_min(p.stamp, 1);
             pdl_trigger();
             int s = 0;
             uint32_t ph = 0;
@@ -1408,6 +1425,7 @@ __global__ void __launch_bounds__(C_THREADS)
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
+    if (threadIdx.x == 0) stamp_max(p.stamp, 2);
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
@@ -1475,6 +1493,63 @@ struct MapKeyHash {
 
 }  // namespace
 
+constexpr int MAX_STAMPS = 2048;   // launches per stamping window
+
+// Sums of the closed stamping windows (device memory).
+struct StampAcc {
+    unsigned long long span_ns;   // sum over launches of exit - entry
+    unsigned long long crit_ns;   // sum over launches of exit - wait
+    unsigned long long launches, windows;
+    double bytes, wbytes;         // algorithmic bytes of those launches
+    double flops, mma_flops;      // 2 M O K of those launches; as issued (x2 for split operands)
+    double pre_bytes;             // weight bytes requested before the wait on the previous kernel
+};
+
+__global__ void stamp_init_kernel(unsigned long long *st, int n, StampAcc *acc) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
+        st[3 * i] = ~0ull;
+        st[3 * i + 1] = ~0ull;
+        st[3 * i + 2] = 0ull;
+    }
+    if (blockIdx.x == 0 && threadIdx.x == 0) *acc = StampAcc{0, 0, 0, 0, 0.0, 0.0, 0.0, 0.0, 0.0};
+}
+
+// Closes a window of n launches: adds their spans to acc and clears their
+// slots for the next window (one block; runs after the window's launches).
+__global__ void stamp_collect_kernel(unsigned long long *st, int n, double bytes, double wbytes, double flops,
+                                     double mma_flops, double pre_bytes, StampAcc *acc) {
+    __shared__ unsigned long long s_span, s_crit, s_cnt;
+    if (threadIdx.x == 0) s_span = s_crit = s_cnt = 0;
+    __syncthreads();
+    unsigned long long span = 0, crit = 0, cnt = 0;
+    for (int i = threadIdx.x; i < n; i += blockDim.x) {
+        const unsigned long long e0 = st[3 * i], w0 = st[3 * i + 1], e1 = st[3 * i + 2];
+        if (e0 != ~0ull && e1 >= e0) {
+            span += e1 - e0;
+            crit += e1 - (w0 <= e1 ? (w0 > e0 ? w0 : e0) : e0);
+            ++cnt;
+        }
+        st[3 * i] = ~0ull;
+        st[3 * i + 1] = ~0ull;
+        st[3 * i + 2] = 0ull;
+    }
+    atomicAdd(&s_span, span);
+    atomicAdd(&s_crit, crit);
+    atomicAdd(&s_cnt, cnt);
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        acc->span_ns += s_span;
+        acc->crit_ns += s_crit;
+        acc->launches += s_cnt;
+        acc->windows += 1;
+        acc->bytes += bytes;
+        acc->wbytes += wbytes;
+        acc->flops += flops;
+        acc->mma_flops += mma_flops;
+        acc->pre_bytes += pre_bytes;
+    }
+}
+
 struct GemmPlan {
     float *ws = nullptr;
     int *counters = nullptr;
@@ -1486,7 +1561,13 @@ struct GemmPlan {
     bool profile = false;
     std::vector<cudaEvent_t> ev;
     size_t ev_used = 0;
-    double prof_bytes = 0.0, prof_wbytes = 0.0;
+    double prof_bytes = 0.0, prof_wbytes = 0.0, prof_flops = 0.0, prof_mma = 0.0, prof_pre = 0.0;
+    // launch stamps: one slot of 3 per launch of a stamping window
+    bool stamp_mode = false, stamp_active = false;
+    int stamp_next = 0;
+    double stamp_bytes = 0.0, stamp_wbytes = 0.0, stamp_flops = 0.0, stamp_mma = 0.0, stamp_pre = 0.0;
+    unsigned long long *stamps = nullptr;
+    StampAcc *stamp_acc = nullptr;
 };
 
 bool gemm_plan_create(GemmPlan **out, int, int, int, int) {
@@ -1517,20 +1598,102 @@ void gemm_plan_destroy(GemmPlan *p) {
     if (!p) return;
     if (p->ws) cudaFree(p->ws);
     if (p->counters) cudaFree(p->counters);
+    if (p->stamps) cudaFree(p->stamps);
+    if (p->stamp_acc) cudaFree(p->stamp_acc);
     for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
     delete p;
 }
 
-void gemm_profile_enable(GemmPlan *p, bool on) {
-    p->profile = on;
+bool gemm_profile_enable(GemmPlan *p, int mode) {
+    if (mode == 2 && !p->stamps) {
+        if (cudaMalloc(&p->stamps, sizeof(unsigned long long) * 3 * MAX_STAMPS) != cudaSuccess ||
+            cudaMalloc(&p->stamp_acc, sizeof(StampAcc)) != cudaSuccess) {
+            cudaGetLastError();
+            return false;
+        }
+    }
+    p->profile = mode == 1;
+    p->stamp_mode = mode == 2;
+    p->stamp_active = false;
     p->ev_used = 0;
-    p->prof_bytes = p->prof_wbytes = 0.0;
+    p->prof_bytes = p->prof_wbytes = p->prof_flops = p->prof_mma = p->prof_pre = 0.0;
+    if (p->stamp_mode) {
+        stamp_init_kernel<<<8, 256>>>(p->stamps, MAX_STAMPS, p->stamp_acc);
+        if (cudaDeviceSynchronize() != cudaSuccess) return false;
+    }
+    return true;
 }
 
 bool gemm_profile_on(const GemmPlan *p) { return p->profile; }
+bool gemm_stamp_on(const GemmPlan *p) { return p->stamp_mode; }
+
+void gemm_stamp_begin(GemmPlan *p) {
+    if (!p->stamp_mode) return;
+    p->stamp_active = true;
+    p->stamp_next = 0;
+    p->stamp_bytes = p->stamp_wbytes = p->stamp_flops = p->stamp_mma = p->stamp_pre = 0.0;
+}
+
+void gemm_stamp_end(GemmPlan *p, cudaStream_t s) {
+    if (!p->stamp_active) return;
+    p->stamp_active = false;
+    stamp_collect_kernel<<<1, 256, 0, s>>>(p->stamps, p->stamp_next, p->stamp_bytes, p->stamp_wbytes,
+                                           p->stamp_flops, p->stamp_mma, p->stamp_pre, p->stamp_acc);
+    note_launch();
+}
+
+// The stamp slot of the next launch (null outside a window or when full).
+static unsigned long long *stamp_slot(GemmPlan *p) {
+    if (!p->stamp_active || p->stamp_next >= MAX_STAMPS) return nullptr;
+    return p->stamps + 3 * (p->stamp_next++);
+}
+
+// Algorithmic bytes and flops of a launch of M token rows x O outputs x K for
+// the open profile (events or stamps); nb = 2 for split token operands (two
+// MMAs per tile); pre = weight bytes its CTAs request before they wait for
+// the previous kernel.
+static void account(GemmPlan *p, double weight_bytes, double total_bytes, int M, int O, int K, int nb,
+                    double pre) {
+    const double fl = 2.0 * M * O * K;
+    if (p->profile) {
+        p->prof_wbytes += weight_bytes;
+        p->prof_bytes += total_bytes;
+        p->prof_flops += fl;
+        p->prof_mma += fl * nb;
+        p->prof_pre += pre;
+    }
+    if (p->stamp_active) {
+        p->stamp_wbytes += weight_bytes;
+        p->stamp_bytes += total_bytes;
+        p->stamp_flops += fl;
+        p->stamp_mma += fl * nb;
+        p->stamp_pre += pre;
+    }
+}
 
 GemmProfile gemm_profile_read(GemmPlan *p) {
-    GemmProfile r{0, 0.0, p->prof_bytes, p->prof_wbytes};
+    GemmProfile r{};
+    if (p->stamp_mode) {
+        StampAcc a{};
+        cudaDeviceSynchronize();
+        cudaMemcpy(&a, p->stamp_acc, sizeof a, cudaMemcpyDeviceToHost);
+        cudaMemset(p->stamp_acc, 0, sizeof a);
+        r.launches = (long)a.launches;
+        r.ms = a.span_ns * 1e-6;
+        r.critical_ms = a.crit_ns * 1e-6;
+        r.windows = (long)a.windows;
+        r.bytes = a.bytes;
+        r.weight_bytes = a.wbytes;
+        r.flops = a.flops;
+        r.mma_flops = a.mma_flops;
+        r.prefetch_bytes = a.pre_bytes;
+        return r;
+    }
+    r.bytes = p->prof_bytes;
+    r.weight_bytes = p->prof_wbytes;
+    r.flops = p->prof_flops;
+    r.mma_flops = p->prof_mma;
+    r.prefetch_bytes = p->prof_pre;
     for (size_t i = 0; i + 1 < p->ev_used; i += 2) {
         float ms = 0.f;
         cudaEventSynchronize(p->ev[i + 1]);
@@ -1538,7 +1701,7 @@ GemmProfile gemm_profile_read(GemmPlan *p) {
         r.launches += 1;
     }
     p->ev_used = 0;
-    p->prof_bytes = p->prof_wbytes = 0.0;
+    p->prof_bytes = p->prof_wbytes = p->prof_flops = p->prof_mma = p->prof_pre = 0.0;
     return r;
 }
 
@@ -1639,6 +1802,7 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     ck.epi = epi;
     ck.status = status;
     const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
+    ck.stamp = stamp_slot(p);
     const CUtensorMap *mxl = X_lo ? get_map(p, X_lo, M, K, ldx, BN, status) : mx;
     if (!mx || !mxl) return;
     const size_t smem = 1024 + (size_t)stages * stage;
@@ -1680,13 +1844,14 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     if (prof) {
         cudaEventRecord(p->ev[p->ev_used + 1], s);
         p->ev_used += 2;
-        const double wb = (double)O * K * 2.0;
-        p->prof_wbytes += wb;
-        double yb = (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
-        if (epi == EPI_SWIGLU) yb = (double)M * fx->F * 2.0 * nb;
-        if (epi == EPI_ROPE_KV) yb = (double)M * O * 2.0 * nb;
-        p->prof_bytes += wb + (double)M * K * 2.0 * nb + yb;
     }
+    const double wb = (double)O * K * 2.0;
+    double yb = (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
+    if (epi == EPI_SWIGLU) yb = (double)M * fx->F * 2.0 * nb;
+    if (epi == EPI_ROPE_KV) yb = (double)M * O * 2.0 * nb;
+    const int nk_split = (kblocks + S - 1) / S;
+    account(p, wb, wb + (double)M * K * 2.0 * nb + yb, M, O, K, nb,
+            (double)tiles * S * std::min(stages, nk_split) * A_BYTES);
 }
 
 // The persistent stream-K GEMM (many token rows). fx: EPI_SWIGLU writes
@@ -1821,6 +1986,7 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
     const CUtensorMap *mxl = X_lo ? get_map(p, X_lo, M, K, ldx, BN, status) : mx;
     if (!mx || !mxl) return;
+    pk.stamp = stamp_slot(p);
     if (!p->smem_set) {
         cudaFuncSetAttribute(gemm_persist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)(BUDGET + 1024));
@@ -1854,11 +2020,11 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     if (prof) {
         cudaEventRecord(p->ev[p->ev_used + 1], s);
         p->ev_used += 2;
-        const double wb = (double)O * K * 2.0;
-        p->prof_wbytes += wb;
-        p->prof_bytes += wb + (double)M * K * 2.0 * nb +
-                         (glu ? (double)M * fx->F * 2.0 * nb : (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1));
     }
+    const double wb = (double)O * K * 2.0;
+    account(p, wb, wb + (double)M * K * 2.0 * nb +
+                       (glu ? (double)M * fx->F * 2.0 * nb : (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1)),
+            M, O, K, nb, (double)G * std::min<long long>(stages, all_units / G) * A_BYTES);
 }
 
 }  // namespace msd

@@ -84,15 +84,26 @@ bool gemm_bf16_fused(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, int 
                      int O, const GemmFused &fx, int *status, cudaStream_t s,
                      const GemmNorm *norm_in = nullptr);
 
-// Profiling: while enabled, every launch is bracketed by CUDA events on its
-// stream; gemm_profile_read synchronises on them and returns the launches,
-// their summed durations and their algorithmic bytes (weights + X + Y),
-// then starts a new window.
+// Profiling. Mode 1: every launch is bracketed by CUDA events on its stream;
+// gemm_profile_read synchronises on them and returns the launches, their
+// summed durations and their algorithmic bytes (weights + X + Y), then starts
+// a new window. Mode 2: launches between gemm_stamp_begin and gemm_stamp_end
+// (a window, e.g. one captured step graph) carry a device slot that their CTAs
+// stamp with %globaltimer (earliest entry, earliest return from
+// griddepcontrol.wait, latest exit); gemm_stamp_end enqueues a kernel that
+// adds the window's spans and bytes to a device sum, so a replayed graph
+// measures itself. gemm_profile_read then returns those sums: ms = entry to
+// exit, critical_ms = wait to exit (disjoint between kernels of one stream).
 struct GemmProfile {
     long launches;
     double ms;
     double bytes;
     double weight_bytes;
+    double critical_ms;
+    long windows;
+    double flops;       // 2 M O K summed over the launches
+    double mma_flops;   // as issued: x2 where the token operand is a split pair
+    double prefetch_bytes;   // weight bytes requested before the wait on the previous kernel
 };
 // Device address of msd_linear_noalloc's status word on the current device
 // (first use sets the device up); null if that failed.
@@ -103,8 +114,12 @@ int *noalloc_status_word();
 // *status. Returns false if the launch failed.
 bool launch_wait_probe(int *status, long long limit_ns, cudaStream_t s);
 
-void gemm_profile_enable(GemmPlan *p, bool on);
-bool gemm_profile_on(const GemmPlan *p);
+// mode 0 off, 1 events, 2 stamps; false if the stamp buffers cannot be made.
+bool gemm_profile_enable(GemmPlan *p, int mode);
+bool gemm_profile_on(const GemmPlan *p);     // mode 1
+bool gemm_stamp_on(const GemmPlan *p);       // mode 2
+void gemm_stamp_begin(GemmPlan *p);
+void gemm_stamp_end(GemmPlan *p, cudaStream_t s);
 GemmProfile gemm_profile_read(GemmPlan *p);
 
 }  // namespace msd

@@ -96,6 +96,7 @@ struct msd_ctx {
         float temp = 0.f;
         long kernels = 0;
         long uses = 0;
+        bool stamped = false;       // recorded with GEMM launch stamps (profile mode 2)
     };
     std::vector<StepGraph> graphs;
     cudaStream_t cap_stream = nullptr;
@@ -1045,10 +1046,11 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
         return st == MSD_OK ? post_status(c, s) : st;
     }
     int need = max_L_bound(c);
+    const bool stamped = c->gplan && gemm_stamp_on(c->gplan);
     msd_ctx::StepGraph *g = nullptr;
     bool rollover = false;
     for (auto &x : c->graphs)
-        if (same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa)) {
+        if (x.stamped == stamped && same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa)) {
             if (x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi)) g = &x;
             else rollover = true;
         }
@@ -1060,7 +1062,8 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
             for (int b = 0; b < c->B; ++b) c->L_bound[b] = L[b];
             need = max_L_bound(c);
             for (auto &x : c->graphs)
-                if (same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa) &&
+                if (x.stamped == stamped &&
+                    same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa) &&
                     x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi))
                     g = &x;
         }
@@ -1068,6 +1071,7 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
     if (!g) {
         msd_ctx::StepGraph ng;
         ng.kind = kind;
+        ng.stamped = stamped;
         ng.bucket_hi = std::min(c->S, ((need + c->D + 511) / 512) * 512);
         ng.tree = *tree;
         ng.argmax = argmax_dev; ng.path = path_dev; ng.alen = accept_len_dev; ng.bonus = bonus_dev;
@@ -1080,8 +1084,10 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
         cudaGraph_t graph = nullptr;
         cudaError_t ce = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
         if (ce == cudaSuccess) {
+            if (stamped) gemm_stamp_begin(c->gplan);    // the graph closes its own window
             st = step_kind_eager(c, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa,
                                  c->cap_stream);
+            if (stamped) gemm_stamp_end(c->gplan, c->cap_stream);
             ce = cudaStreamEndCapture(c->cap_stream, &graph);
         } else {
             st = MSD_OK;
@@ -1243,9 +1249,11 @@ msd_status msd_linear(msd_ctx *c, const void *x, int32_t ldx, int32_t m, int32_t
     return post_status(c, s);
 }
 
-msd_status msd_profile_enable(msd_ctx *c, int32_t on) {
-    if (!c) return MSD_ERR_INVALID;
-    if (c->gplan) gemm_profile_enable(c->gplan, on != 0);
+msd_status msd_profile_enable(msd_ctx *c, int32_t mode) {
+    if (!c || mode < 0 || mode > 2) return MSD_ERR_INVALID;
+    c->err.clear();
+    if (c->gplan && !gemm_profile_enable(c->gplan, mode))
+        return fail(c, MSD_ERR_CUDA, "GEMM launch stamps: device buffers or reset failed");
     return MSD_OK;
 }
 
@@ -1259,6 +1267,11 @@ msd_status msd_profile_read(msd_ctx *c, msd_profile *out) {
         out->gemm_ms = g.ms;
         out->gemm_bytes = g.bytes;
         out->gemm_weight_bytes = g.weight_bytes;
+        out->gemm_critical_ms = g.critical_ms;
+        out->windows = g.windows;
+        out->gemm_flops = g.flops;
+        out->gemm_mma_flops = g.mma_flops;
+        out->gemm_prefetch_bytes = g.prefetch_bytes;
     }
     return MSD_OK;
 }

@@ -59,7 +59,10 @@ class msd_state_view(ctypes.Structure):
 
 class msd_profile(ctypes.Structure):
     _fields_ = [("kernel_launches", c_int64), ("gemm_launches", c_int64), ("gemm_ms", ctypes.c_double),
-                ("gemm_bytes", ctypes.c_double), ("gemm_weight_bytes", ctypes.c_double)]
+                ("gemm_bytes", ctypes.c_double), ("gemm_weight_bytes", ctypes.c_double),
+                ("gemm_critical_ms", ctypes.c_double), ("windows", c_int64),
+                ("gemm_flops", ctypes.c_double), ("gemm_mma_flops", ctypes.c_double),
+                ("gemm_prefetch_bytes", ctypes.c_double)]
 
 
 _SIGNATURES = {
@@ -318,8 +321,10 @@ class Engine:
         st = lib().msd_test_wait_timeout(self.ctx, int(limit_ns), _stream(stream))
         self._check(st, "msd_test_wait_timeout")
 
-    def profile_enable(self, on: bool = True):
-        self._check(lib().msd_profile_enable(self.ctx, int(on)), "msd_profile_enable")
+    def profile_enable(self, mode=True):
+        """0/False off, 1/True CUDA events around separate launches, 2 launch
+        stamps inside the replayed step graphs."""
+        self._check(lib().msd_profile_enable(self.ctx, int(mode)), "msd_profile_enable")
 
     def profile_read(self) -> dict:
         p = msd_profile()

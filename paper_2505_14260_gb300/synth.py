@@ -112,12 +112,14 @@ def layer_shapes(wl: Workload) -> dict:
             "w_gate": (F, H), "w_up": (F, H), "w_down": (H, F)}
 
 
-def make_weights(wl: Workload, device="cpu") -> dict:
+def make_weights(wl: Workload, device="cpu", layers: int | None = None) -> dict:
     """All model weights as tensors of the workload dtype on ``device``.
 
     Returns {"embed", "lm_head", "final_norm", "draft_fc",
              "layers": [ {name: tensor} * n_layers ], "draft": {name: tensor}}.
-    Matrices are [out, in] row-major.
+    Matrices are [out, in] row-major. With ``layers`` set, only the first
+    ``layers`` decoder layers are kept (the others are still drawn, so every
+    kept tensor equals its value in the full set).
     """
     device = torch.device(device)
     g = torch.Generator(device=device)
@@ -135,15 +137,20 @@ def make_weights(wl: Workload, device="cpu") -> dict:
         return (1.0 + NORM_JITTER * t).to(dt)
 
     shapes = layer_shapes(wl)
+    keep = wl.n_layers if layers is None else min(layers, wl.n_layers)
     w = {"embed": mat((V, H)), "layers": []}
-    for _ in range(wl.n_layers):
-        w["layers"].append({n: mat(shapes[n]) for n in LAYER_MATS})
+    for i in range(wl.n_layers):
+        lw = {n: mat(shapes[n]) for n in LAYER_MATS}
+        if i < keep:
+            w["layers"].append(lw)
+        del lw
     w["lm_head"] = mat((V, H))
     w["draft"] = {n: mat(shapes[n]) for n in LAYER_MATS}
     w["draft_fc"] = mat((H, 2 * H))
-    for lw in w["layers"]:
-        for n in LAYER_NORMS:
-            lw[n] = gain()
+    for i in range(wl.n_layers):
+        g_ = {n: gain() for n in LAYER_NORMS}
+        if i < keep:
+            w["layers"][i].update(g_)
     w["final_norm"] = gain()
     for n in LAYER_NORMS:
         w["draft"][n] = gain()

@@ -124,3 +124,35 @@ def test_bounded_wait_that_runs_out_is_reported():
         eng.draft_tree()
     assert e.value.status == msd.MSD_ERR_DEVICE
     eng.close()
+
+
+def test_bf16_context_never_reads_its_borrowed_projection_matrices():
+    """A bf16 context packs every projection matrix (the target's and the
+    draft's wq, wk, wv, wo, w_gate, w_up, w_down, plus lm_head and draft_fc)
+    into copies of its own in msd_create and reads the caller's matrices no
+    more: overwriting them with NaN afterwards changes no output of the step."""
+    from tests.gpu_support import to_device
+    wl = synth.WORKLOADS["tiny"].with_(dtype="bf16")
+    w = synth.make_weights(wl)
+    ids, lens, vis, offs = msd.upload_prompts(synth.make_prompts(wl))
+    runs = []
+    for poison in (False, True):
+        wd = to_device(w)
+        eng = msd.Engine(msd.make_config(wl, wl.max_seq(4)), wd)
+        if poison:
+            for lw in wd["layers"] + [wd["draft"]]:
+                for n in synth.LAYER_MATS:
+                    lw[n].fill_(float("nan"))
+            wd["lm_head"].fill_(float("nan"))
+            wd["draft_fc"].fill_(float("nan"))
+        eng.prefill(ids, lens, vis, offs)
+        out = []
+        for _ in range(3):
+            path, a, bonus = eng.step()
+            out.append([t.clone() for t in (path, a, bonus, eng.tree.tokens, eng.argmax)])
+        torch.cuda.synchronize()
+        eng.close()
+        runs.append(out)
+    for s, (x, y) in enumerate(zip(*runs)):
+        for p, q in zip(x, y):
+            assert torch.equal(p, q), f"step {s}"

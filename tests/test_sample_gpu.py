@@ -280,3 +280,54 @@ def test_many_walks_match_oracle():
             walks += 1
     eng.close()
     assert walks == 96 and near <= 2
+
+
+def test_sampling_at_the_vocabulary_limit_matches_oracle():
+    """msd_accept_sample at the largest vocabulary it accepts (393216 tokens:
+    one removed-candidate bit per token fills its 48 KB of shared memory),
+    on caller-supplied logits, against the oracle's accept_sample. In the
+    middle step request 0 verifies a planted tree whose candidates are the
+    vocabulary's last three tokens and draws uniforms that reject both root
+    children, so the residual draw runs with the top bits of the mask set."""
+    V = 48 * 1024 * 8
+    wl = synth.WORKLOADS["tiny"].with_(dtype="bf16", vocab=V, topk=2, tree_nodes=5, tree_depth=2,
+                                       batch=2, steps=3)
+    B, N, D, k = wl.batch, wl.tree_nodes, wl.tree_depth, wl.topk
+    eng, _ = open_engine(wl, steps=wl.steps)
+    ids, lens, vis, offs = msd.upload_prompts(synth.make_prompts(wl))
+    eng.prefill(ids, lens, vis, offs)
+    logits = torch.zeros(B * N, V, device="cuda")
+    gen = torch.Generator().manual_seed(31)
+    near = 0
+    for step in range(wl.steps):
+        eng.draft_tree()
+        tree = eng.tree
+        u = torch.rand(B, D + 1, k + 1, generator=gen)
+        if step == 1:
+            tree = msd.Tree(B, N)
+            roots = eng.state()["root"].cpu().numpy()
+            plant(eng, tree, 0, [int(roots[0]), V - 1, V - 2, V - 3], [-1, 0, 0, 1])
+            plant(eng, tree, 1, [int(roots[1])], [-1])
+        eng.verify(tree=tree, logits=logits)
+        if step == 1:
+            z = torch.randn(N, V, generator=gen) * 0.5
+            z[:, V - 4:] += torch.tensor([13.0, 13.0, 13.5, 14.0])  # about 86% of the mass
+            logits[:N] = z.cuda()
+            u[0, 0, :k] = 0.999                                     # reject both root children
+        eng.accept_sample(1.0, u.cuda(), logits=logits, tree=tree)
+        torch.cuda.synchronize()
+        g_all = logits.cpu().numpy().astype(np.float64)
+        path_all, alen, bonus = eng.path.cpu().numpy(), eng.accept_len.cpu().numpy(), eng.bonus.cpu().numpy()
+        n_nodes = tree.n_nodes.cpu().numpy()
+        for b in range(B):
+            toks, par, dep, _ = tree_numpy(tree, b)
+            n = int(n_nodes[b])
+            otree = O.Tree(tokens=toks[:n], parent=par[:n], depth=dep[:n])
+            a = int(alen[b])
+            gpu = ([int(x) for x in path_all[b * (D + 1):b * (D + 1) + a + 1]], a, int(bonus[b]))
+            near += check_walk(gpu, otree, g_all[b * N:(b + 1) * N], 1.0, u[b].numpy().astype(np.float64), k,
+                               f"request {b} step {step}")
+            if step == 1 and b == 0:
+                assert a == 0 and gpu[2] not in (V - 1, V - 2), gpu
+    eng.close()
+    assert near <= 1
