@@ -248,19 +248,19 @@ msd_status msd_accept_sample(msd_ctx *ctx, const msd_tree *tree, const float *lo
  * sequence (Sec. 3.2; Eq. 6 at T = 0), with the same arguments and outputs as
  * those calls (the drafted tree is written to *tree and then verified). The
  * context records the sequence once into a CUDA graph per set of output
- * buffers and per bucket of cache lengths (512 positions) and replays it, so a
- * step is one graph launch; the first step in a new bucket records a new graph
- * (host work of a few milliseconds, and one host-device synchronisation to
- * refresh the bound on L). While GEMM profiling is enabled the calls run
- * without a graph. Errors: as for the three calls, and MSD_ERR_CUDA if the
- * graph cannot be recorded. */
+ * buffers and replays it, so a step is one graph launch (every kernel reads
+ * the lengths it needs from device state; the first step with new buffers
+ * records the graph, host work of a few milliseconds). While GEMM profiling
+ * mode 1 is enabled the calls run without a graph; mode 2 replays graphs
+ * recorded with launch stamps (msd_profile_enable). Errors: as for the three
+ * calls, and MSD_ERR_CUDA if the graph cannot be recorded. */
 msd_status msd_step(msd_ctx *ctx, const msd_tree *tree, int32_t *argmax_dev, int32_t *path_dev,
                     int32_t *accept_len_dev, int32_t *bonus_dev, void *stream);
 
 /* One whole decode step at temperature T > 0: msd_draft_tree, msd_verify (its
  * logits kept in the context) and msd_accept_sample, recorded and replayed as a
  * CUDA graph exactly as msd_step (one graph per set of buffers, u_dev pointer,
- * temperature and bucket of cache lengths). The caller refills u_dev
+ * and temperature). The caller refills u_dev
  * ([B][D+1][k+1] uniforms in [0, 1)) before each step; the graph reads it when
  * it runs. Errors: as msd_step, and MSD_ERR_INVALID for a null u_dev, a
  * temperature that is not finite and > 0, or vocab > 393216 (as
@@ -276,7 +276,7 @@ msd_status msd_step_sample(msd_ctx *ctx, const msd_tree *tree, float temperature
  * (ties: lower id) becomes the new root and is written to token_dev[b] (B int32,
  * device). The same kernels as msd_verify and msd_accept_compact run it (a
  * tree of the root alone), recorded once into a CUDA graph per token_dev and
- * bucket of cache lengths and replayed, as msd_step. A context created with
+ * replayed, as msd_step. A context created with
  * tree_nodes = 1 runs it on B token rows; with more tree nodes the other rows
  * are computed and ignored. The draft is not run, so after this call the draft
  * cache no longer follows the target's: msd_draft_tree and msd_step return

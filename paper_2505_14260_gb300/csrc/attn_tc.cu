@@ -75,7 +75,8 @@ struct AttnTcParams {
     int lo_rows;
     int *status;
     int R, rows_per_req, tiles_per_req, nh, cache_slots, tree_slots, mask_words;
-    int nsplit_cache, has_tree, chunk;
+    int nsplit_cache, has_tree;
+    int tree_merged;          // the tree keys follow the cache keys in the one cache split (no tree split)
     int cache_early;          // cache K/V may be requested before the wait (not written by the previous kernel)
     float scale_log2;
 };
@@ -276,7 +277,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int blk = tile / p.tiles_per_req;
     const int r0 = blk * p.rows_per_req + (tile - blk * p.tiles_per_req) * ROWS;
     const int r_end = min(r0 + ROWS, (blk + 1) * p.rows_per_req);
-    const bool is_tree = p.has_tree && split == p.nsplit_cache;
+    const bool is_tree = p.has_tree && !p.tree_merged && split == p.nsplit_cache;
     const int H = p.nh * HD;
 
     const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
@@ -329,30 +330,32 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_base;
 
-    // Key range of this split.
-    int k_lo, k_hi, row_base;
-    const CUtensorMap *mk, *mv;
-    if (is_tree) {
-        k_lo = 0;
-        k_hi = p.tree_slots;
-        row_base = (req * p.nh + h) * p.tree_slots;
-        mk = &mkt;
-        mv = &mvt;
-    } else {
-        k_lo = split * p.chunk;
-        k_hi = min(k_lo + p.chunk, min(s_pmax, p.cache_slots));
-        row_base = (req * p.nh + h) * p.cache_slots;
-        mk = &mkc;
-        mv = &mvc;
+    // Key range of this split. The request's live prefix is cut into
+    // nsplit_cache equal runs of whole 64-key tiles (the count is fixed per
+    // context, so a result depends on L alone, never on the launch's bound of
+    // L); a tree split, or the tree tiles after the cache tiles of a merged
+    // CTA, covers the tree slots.
+    const int live = min(s_pmax, p.cache_slots);
+    const int per_split = ((live + KT - 1) / KT + p.nsplit_cache - 1) / p.nsplit_cache * KT;
+    int k_lo = 0, k_hi = 0;
+    if (!is_tree) {
+        k_lo = split * per_split;
+        k_hi = min(k_lo + per_split, live);
     }
-    const int ntiles = k_hi > k_lo ? (k_hi - k_lo + KT - 1) / KT : 0;
+    const int nc = k_hi > k_lo ? (k_hi - k_lo + KT - 1) / KT : 0;      // cache tiles
+    const bool has_tree_tiles = is_tree || (p.has_tree && p.tree_merged);
+    const int ntiles = nc + (has_tree_tiles ? (p.tree_slots + KT - 1) / KT : 0);
+    const int row_base_c = (req * p.nh + h) * p.cache_slots;
+    const int row_base_t = (req * p.nh + h) * p.tree_slots;
 
     auto issue = [&](int i) {
         const int s = i % STAGES;
         const uint32_t bar = full0 + 8 * s;
         const uint32_t kd = base + s * L::STAGE;
         bar_expect_tx(bar, L::STAGE);
-        const int y = row_base + k_lo + i * KT;
+        const bool cache = i < nc;
+        const CUtensorMap *mk = cache ? &mkc : &mkt, *mv = cache ? &mvc : &mvt;
+        const int y = cache ? row_base_c + k_lo + i * KT : row_base_t + (i - nc) * KT;
 #pragma unroll
         for (int b = 0; b < L::NB; ++b) {
             tma2d(kd + b * L::BOX, mk, b * 64, y, bar);
@@ -361,10 +364,12 @@ __global__ void __launch_bounds__(THREADS, 1)
             tma2d(kd + 3 * L::TILE + b * L::BOX, mv, b * 64, y + p.lo_rows, bar);
         }
     };
-    const bool early = !is_tree && p.cache_early;
+    // the cache tiles of the first stages may go out before the wait; tree
+    // K/V is the previous kernel's output
     const int n_pre = min(STAGES, ntiles);
-    if (threadIdx.x == 0 && early)
-        for (int i = 0; i < n_pre; ++i) issue(i);
+    const int n_early = p.cache_early ? min(n_pre, nc) : 0;
+    if (threadIdx.x == 0)
+        for (int i = 0; i < n_early; ++i) issue(i);
     wait_prior();
     allow_dependents();
 
@@ -374,8 +379,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 0) {
         // ---- producer ------------------------------------------------------
         if (lane == 0) {
-            if (!early)
-                for (int i = 0; i < n_pre; ++i) issue(i);
+            for (int i = n_early; i < n_pre; ++i) issue(i);
             int i = n_pre;
             for (; i < ntiles; ++i) {
                 const int s = i % STAGES;
@@ -481,20 +485,22 @@ __global__ void __launch_bounds__(THREADS, 1)
             asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
             bar_arrive(q_ready);
         }
-        const uint64_t *mrow = (is_tree && valid) ? p.mask + (size_t)row * p.mask_words : nullptr;
-        const int klim = valid ? (is_tree ? k_hi : min(k_hi, plen)) : 0;     // keys visible by position
+        const uint64_t *mrow = (has_tree_tiles && valid) ? p.mask + (size_t)row * p.mask_words : nullptr;
+        const int klim = valid ? min(k_hi, plen) : 0;        // cache keys visible by position
+        const int tlim = valid ? p.tree_slots : 0;           // tree keys: by the ancestor mask
         for (int j = 0; j < ntiles; ++j) {
             if (!dead && !wwait(s_full0 + 8 * (j & 1), (uint32_t)(j >> 1) & 1u)) dead = true;
             asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
             const uint32_t sd = tq + L::T_S + (j & 1) * KT;
             uint32_t sr[32];
             tmem_ld32(sd + 32 * hf, sr);
-            const int key0 = k_lo + j * KT + 32 * hf;
-            const int lim = klim - key0;                  // columns c < lim are inside the range
+            const bool tree_tile = j >= nc;
+            const int key0 = (tree_tile ? (j - nc) * KT : k_lo + j * KT) + 32 * hf;
+            const int lim = (tree_tile ? tlim : klim) - key0;   // columns c < lim are inside the range
             uint32_t bits = 0xffffffffu;
-            if (mrow) {
-                const int w = (k_lo + j * KT) >> 6;
-                bits = w < p.mask_words ? (uint32_t)(mrow[w] >> (32 * hf)) : 0u;
+            if (tree_tile) {
+                const int w = j - nc;                           // one mask word per 64 tree keys
+                bits = (mrow && w < p.mask_words) ? (uint32_t)(mrow[w] >> (32 * hf)) : 0u;
             }
             float v[32];
             float mx = -INFINITY;
@@ -565,7 +571,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     const bool ok = !dead && !abort_flag;
 
-    const int nsplit = p.nsplit_cache + p.has_tree;
+    const int nsplit = p.nsplit_cache + (p.has_tree && !p.tree_merged);
     if (nsplit == 1) {
         if (valid && ok) {
             const float inv = l_sum > 0.f ? 1.f / l_sum : 0.f;
@@ -668,25 +674,22 @@ struct MapKeyHash {
 
 struct AttnTcPlan {
     int num_sms = 148;
-    int chunk_tiles = 1;       // keys per cache split / 64: fixed per context
+    int splits = 1;            // cache splits of a decode launch: fixed per context
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     std::unordered_map<MapKey, CUtensorMap, MapKeyHash> maps;
     bool attr_set = false;
 };
 
-bool attn_tc_plan_create(AttnTcPlan **out, int max_keys, int decode_ctas) {
+bool attn_tc_plan_create(AttnTcPlan **out, int decode_ctas) {
     AttnTcPlan *p = new AttnTcPlan();
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev);
-    // The cache range is cut at fixed multiples of chunk_tiles * 64 keys, a
-    // function of the capacity only, so results never depend on how many
-    // (possibly empty) splits a launch covers. A CTA fills an SM (one per SM):
-    // a decode launch of decode_ctas (row tile, head) pairs takes as many cache
-    // splits as keep it, with the tree split, within one wave.
-    const int tiles = (max_keys + KT - 1) / KT;
-    const int splits = std::max(1, std::min(MAX_SPLITS - 1, p->num_sms / std::max(1, decode_ctas) - 1));
-    p->chunk_tiles = std::max(2, (tiles + splits - 1) / splits);
+    // A CTA fills an SM (one per SM): a decode launch of decode_ctas (row
+    // tile, head) pairs takes as many cache splits as keep it, with the tree
+    // split, within one wave. The count is fixed for the context, so a result
+    // never depends on which launch (eager call or graph bucket) computed it.
+    p->splits = std::max(1, std::min(MAX_SPLITS - 1, p->num_sms / std::max(1, decode_ctas) - 1));
     cudaDriverEntryPointQueryResult q;
     void *fn = nullptr;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
@@ -720,8 +723,8 @@ static const CUtensorMap *kv_map(AttnTcPlan *p, const void *ptr, long rows, int 
     return &p->maps.emplace(key, m).first->second;
 }
 
-bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, int p_bound,
-                         int *status, cudaStream_t s) {
+bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, int *status,
+                         cudaStream_t s) {
     if (a.R <= 0) return true;
     if (a.hd != 64 && a.hd != 128) return false;
     if (a.lo % a.hd) return false;
@@ -730,13 +733,13 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     const int row_tiles = n_blocks * tiles_per_req;
     const long base = (long)row_tiles * a.nh;
     const int has_tree = a.mask != nullptr;
-    const int pb = std::max(1, std::min(p_bound, a.cache_slots));
-    const int cache_tiles = (pb + KT - 1) / KT;
-    // enough (row tile, head) CTAs already: one split over the whole range;
-    // otherwise fixed-size splits (the count only covers [0, p_bound))
-    const int chunk_tiles = base * (1 + has_tree) >= p->num_sms ? cache_tiles : p->chunk_tiles;
-    const int nsplit = (cache_tiles + chunk_tiles - 1) / chunk_tiles;
-    const int tot = nsplit + has_tree;
+    // Enough (row tile, head) CTAs already: one cache split per CTA, and when
+    // they fill a wave by themselves the tree keys join it (no tree split);
+    // otherwise the context's fixed split count.
+    const bool single = base * (1 + has_tree) >= p->num_sms;
+    const int nsplit = single ? 1 : p->splits;
+    const int tree_merged = has_tree && single && base >= p->num_sms;
+    const int tot = nsplit + (has_tree && !tree_merged);
     if (tot > MAX_SPLITS) return false;
     const long lo_rows = a.lo / a.hd;
     const long kc_rows = (long)B * a.nh * a.cache_slots + lo_rows;
@@ -767,7 +770,7 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.mask_words = a.mask_words;
     tp.nsplit_cache = nsplit;
     tp.has_tree = has_tree;
-    tp.chunk = chunk_tiles * KT;
+    tp.tree_merged = tree_merged;
     tp.cache_early = a.cache_fresh ? 0 : 1;
     tp.scale_log2 = a.scale * 1.4426950408889634f;
     const size_t smem = 1024 + (a.hd == 128 ? (size_t)STAGES * Lay<128>::STAGE : (size_t)STAGES * Lay<64>::STAGE);

@@ -8,16 +8,16 @@ namespace msd {
 
 struct AttnTcPlan;
 
-// Per-context plan (tensor-map cache, split size); max_keys = cache capacity,
-// decode_ctas = the (row tile of 64, head) pairs of a decode launch.
-bool attn_tc_plan_create(AttnTcPlan **out, int max_keys, int decode_ctas);
+// Per-context plan (tensor-map cache, split count); decode_ctas = the (row
+// tile of 64, head) pairs of a decode launch.
+bool attn_tc_plan_create(AttnTcPlan **out, int decode_ctas);
 void attn_tc_plan_destroy(AttnTcPlan *p);
 
-// a.R rows grouped by request in blocks of rows_per_req; every row's plen is
-// at most p_bound (used to size the split of the cache range). B is the
-// number of requests the cache buffers hold. Returns false if the shape is not
-// supported (the caller reports it).
-bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req,
-                         int p_bound, int *status, cudaStream_t s);
+// a.R rows grouped by request in blocks of rows_per_req; each row's visible
+// prefix length comes from its row descriptor. B is the number of requests
+// the cache buffers hold. Returns false if the shape is not supported (the
+// caller reports it).
+bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, int *status,
+                         cudaStream_t s);
 
 }  // namespace msd

@@ -1849,9 +1849,11 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     double yb = (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1);
     if (epi == EPI_SWIGLU) yb = (double)M * fx->F * 2.0 * nb;
     if (epi == EPI_ROPE_KV) yb = (double)M * O * 2.0 * nb;
-    const int nk_split = (kblocks + S - 1) / S;
-    account(p, wb, wb + (double)M * K * 2.0 * nb + yb, M, O, K, nb,
-            (double)tiles * S * std::min(stages, nk_split) * A_BYTES);
+    double pre = 0.0;      // the blocks each split requests before its wait (padded rows included)
+    for (int z = 0; z < S; ++z)
+        pre += (double)tiles * std::min(stages, (int)((long long)(z + 1) * kblocks / S - (long long)z * kblocks / S)) *
+               A_BYTES;
+    account(p, wb, wb + (double)M * K * 2.0 * nb + yb, M, O, K, nb, std::min(pre, wb));
 }
 
 // The persistent stream-K GEMM (many token rows). fx: EPI_SWIGLU writes
@@ -2024,7 +2026,7 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     const double wb = (double)O * K * 2.0;
     account(p, wb, wb + (double)M * K * 2.0 * nb +
                        (glu ? (double)M * fx->F * 2.0 * nb : (double)M * O * 4.0 * (epi == EPI_ADD ? 2 : 1)),
-            M, O, K, nb, (double)G * std::min<long long>(stages, all_units / G) * A_BYTES);
+            M, O, K, nb, std::min(wb, (double)G * std::min<long long>(stages, all_units / G) * A_BYTES));
 }
 
 }  // namespace msd

@@ -84,12 +84,11 @@ struct msd_ctx {
     std::vector<long> L_bound;
     bool prefilled = false;
     std::string err;
-    // whole-step CUDA graphs (msd_step), one per L bucket and buffer set
+    // whole-step CUDA graphs (msd_step), one per buffer set
     struct StepGraph {
         cudaGraphExec_t exec = nullptr;
         int kind = 0;               // 0: draft-verify-accept step, 1: plain greedy step,
                                     // 2: draft-verify-sample step
-        int bucket_hi = 0;
         msd_tree tree{};
         const void *argmax = nullptr, *path = nullptr, *alen = nullptr, *bonus = nullptr;
         const void *u = nullptr;    // kind 2: the uniforms' buffer and the temperature
@@ -100,7 +99,6 @@ struct msd_ctx {
     };
     std::vector<StepGraph> graphs;
     cudaStream_t cap_stream = nullptr;
-    int pb_override = 0;        // attention p_bound while capturing a graph
     bool capturing = false;
     long captured_launches = 0; // launches recorded into graphs (not executed then)
     long graph_kernels = 0;     // kernels executed by graph replays
@@ -199,29 +197,19 @@ const bf16 *lo_of(const msd_ctx *c, const void *hi) {
 
 // One pre-norm decoder layer over R rows (target or draft).
 template <typename T>
-void attention(msd_ctx *c, const AttnArgs<T> &a, int rows_per_req, int p_bound, cudaStream_t s);
+void attention(msd_ctx *c, const AttnArgs<T> &a, int rows_per_req, cudaStream_t s);
 
 template <>
-void attention<float>(msd_ctx *c, const AttnArgs<float> &a, int, int, cudaStream_t s) {
+void attention<float>(msd_ctx *c, const AttnArgs<float> &a, int, cudaStream_t s) {
     launch_attention<float>(a, s);
 }
 
 template <>
-void attention<bf16>(msd_ctx *c, const AttnArgs<bf16> &a, int rows_per_req, int p_bound,
-                     cudaStream_t s) {
-    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, p_bound, c->status, s)) {
+void attention<bf16>(msd_ctx *c, const AttnArgs<bf16> &a, int rows_per_req, cudaStream_t s) {
+    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, c->status, s)) {
         c->err = "tensor-core attention: unsupported shape or launch failure";
         launch_flag(c->status, ST_RANGE, s);     // reported by the next call
     }
-}
-
-// Largest L any request may have now (host-side upper bound); while a step
-// graph is being captured, the upper end of its L bucket.
-int max_L_bound(const msd_ctx *c) {
-    if (c->pb_override > 0) return c->pb_override;
-    long m = 1;
-    for (long v : c->L_bound) m = std::max(m, v);
-    return (int)std::min<long>(m, c->S);
 }
 
 // qkv = xn [wq;wk;wv]^T, then RoPE on q and k (Sec. 3.1 backbone), q to c->q
@@ -301,7 +289,7 @@ GemmNorm norm_in(msd_ctx *c) {
 }
 
 // One pre-norm decoder layer over R rows (target or draft). Rows come in
-// blocks of rows_per_req per request; every row attends to at most p_bound
+// blocks of rows_per_req per request.
 // cache positions. in_folded: the layer's input norm was folded into the GEMM
 // that produced x; out_norm_g (nullable): the next layer's input-norm gain,
 // to fold into this layer's last GEMM. Returns whether it did.
@@ -309,7 +297,7 @@ template <typename T>
 bool run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, int R,
                const RowDesc *rows, T *kdst, T *vdst, int dst_slots, const T *ck, const T *cv,
                int cslots, const T *tk, const T *tv, int tslots, const uint64_t *mask, int mw,
-               int rows_per_req, int p_bound, cudaStream_t s, bool in_folded = false,
+               int rows_per_req, cudaStream_t s, bool in_folded = false,
                const void *out_norm_g = nullptr) {
     const int H = c->H, F = c->F;
     const float eps = c->cfg.rms_eps;
@@ -337,7 +325,7 @@ bool run_layer(msd_ctx *c, const msd_layer &lw, const msd_ctx::LayerPack &lp, in
     a.out = static_cast<T *>(c->attn);
     a.cache_fresh = kdst == ck;         // this layer's own K/V go into the cache it reads
     a.lo = c->lo;
-    attention<T>(c, a, rows_per_req, p_bound, s);
+    attention<T>(c, a, rows_per_req, s);
     GemmW wo = {{lw.wo, nullptr, nullptr}, {H, 0, 0}, 1, lp.o};
     GemmW wd = {{lw.w_down, nullptr, nullptr}, {H, 0, 0}, 1, lp.down};
     if constexpr (std::is_same<T, bf16>::value) {
@@ -427,7 +415,7 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
             for (int l = 0; l < c->NL; ++l) {
                 T *K = tkv<T>(c, c->target_kv, l, 0, c->S), *Vv = tkv<T>(c, c->target_kv, l, 1, c->S);
                 run_layer<T>(c, c->layers[l], c->lpack[l], n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr,
-                             nullptr, 0, nullptr, 0, n, r0 + n, s);
+                             nullptr, 0, nullptr, 0, n, s);
             }
             launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), n, H, c->cfg.rms_eps,
                               static_cast<T *>(c->h_all) + (size_t)r0 * H, c->lo, s);
@@ -457,7 +445,7 @@ msd_status prefill_impl(msd_ctx *c, int batch, const int32_t *seq_len_host, cons
             }
             T *K = tkv<T>(c, c->draft_kv, 0, 0, c->S), *Vv = tkv<T>(c, c->draft_kv, 0, 1, c->S);
             run_layer<T>(c, c->w.draft, c->dpack, n, c->rows, K, Vv, c->S, K, Vv, c->S, nullptr, nullptr, 0,
-                         nullptr, 0, n, r0 + n, s);
+                         nullptr, 0, n, s);
             CU(cudaStreamSynchronize(s));
         }
         launch_prefill_finish<T>(c->argmax_tmp, h_last, b, L, D1, H, c->seq_len, c->n_pend, c->root,
@@ -523,9 +511,8 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
     launch_catchup_setup<T>(c->seq_len, c->n_pend, static_cast<const T *>(c->pend_h), c->pend_next,
                             E, B, H, D1, V, static_cast<T *>(c->xfc), c->lo, c->rows, c->status, s);
     bool folded = draft_fc<T>(c, R1, s);
-    const int pb = max_L_bound(c);
     run_layer<T>(c, c->w.draft, c->dpack, R1, c->rows, dK, dV, S, dK, dV, S, nullptr, nullptr, 0, nullptr, 0,
-                 D1, pb, s, folded);
+                 D1, s, folded);
     launch_root_gather<T>(c->x, c->n_pend, B, D1, H, c->hhat_root, static_cast<T *>(c->xr), c->lo, s);
     gemm<T>(c, static_cast<const T *>(c->xr), H, B, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V,
             EPI_STORE, s);
@@ -539,7 +526,7 @@ msd_status draft_impl(msd_ctx *c, const msd_tree *out, const msd_draft_record *r
     for (int d = 2; d <= c->D; ++d) {
         folded = draft_fc<T>(c, Rk, s);
         run_layer<T>(c, c->w.draft, c->dpack, Rk, c->rows, tK, tV, c->Td, dK, dV, S, tK, tV, c->Td,
-                     c->row_mask, c->Wd, k, pb, s, folded);
+                     c->row_mask, c->Wd, k, s, folded);
         launch_hhat_store<T>(c->x, c->rows, Rk, c->Td, H, c->hhat_slot, static_cast<T *>(c->xr), c->lo, s);
         gemm<T>(c, static_cast<const T *>(c->xr), H, Rk, H, one(c->w.lm_head, V, c->pk_lm), V, c->logits, V,
                 EPI_STORE, s);
@@ -561,7 +548,6 @@ template <typename T>
 msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, float *logits_dev,
                        cudaStream_t s) {
     const int B = c->B, N = c->N, H = c->H, V = c->V, R = B * N;
-    const int pb = max_L_bound(c);
     TreeIn t{tree->tokens, tree->parent, tree->depth, tree->mask, tree->n_nodes};
     launch_verify_setup(t, c->seq_len, c->root, B, N, V, c->rows, c->src, c->vmask, c->status, s);
     launch_embed_rows<T>(static_cast<const T *>(c->w.embed), nullptr, c->src, R, H, c->x, nullptr,
@@ -572,7 +558,7 @@ msd_status verify_impl(msd_ctx *c, const msd_tree *tree, int32_t *argmax_dev, fl
         T *tK = tkv<T>(c, c->tree_kv, l, 0, N), *tV = tkv<T>(c, c->tree_kv, l, 1, N);
         const void *next_g = l + 1 < c->NL ? c->layers[l + 1].attn_norm : nullptr;
         folded = run_layer<T>(c, c->layers[l], c->lpack[l], R, c->rows, tK, tV, N, K, Vv, c->S, tK, tV, N,
-                              c->vmask, c->W, N, pb, s, folded, next_g);
+                              c->vmask, c->W, N, s, folded, next_g);
     }
     launch_rmsnorm<T>(c->x, static_cast<const T *>(c->w.final_norm), R, H, c->cfg.rms_eps,
                       static_cast<T *>(c->hT), c->lo, s);
@@ -872,7 +858,7 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     if (ok && cfg->dtype == MSD_BF16) ok = gemm_plan_create(&c->gplan, c->Rmax, c->H, c->F, c->V);
     if (ok && cfg->dtype == MSD_BF16) {
         const int decode_rows = std::max(c->N, std::max(c->k, c->D1));
-        ok = attn_tc_plan_create(&c->aplan, c->S, c->B * ((decode_rows + 63) / 64) * c->nh);
+        ok = attn_tc_plan_create(&c->aplan, c->B * ((decode_rows + 63) / 64) * c->nh);
     }
     c->lpack.assign(c->NL, msd_ctx::LayerPack());
     if (ok && cfg->dtype == MSD_BF16) ok = pack_weights(c);
@@ -1018,9 +1004,9 @@ msd_status msd_accept_compact(msd_ctx *c, const msd_tree *tree, const int32_t *a
 
 namespace {
 
-// One step (kind 0: draft, verify, accept; kind 1: plain greedy) recorded once
-// into a CUDA graph per set of buffers and per bucket of cache lengths, then
-// replayed.
+// One step (kind 0: draft, verify, accept; kind 1: plain greedy; kind 2:
+// draft, verify, sample) recorded once into a CUDA graph per set of buffers,
+// then replayed: every kernel reads the lengths it needs from device state.
 msd_status step_kind_eager(msd_ctx *c, int kind, const msd_tree *tree, int32_t *argmax_dev,
                            int32_t *path_dev, int32_t *accept_len_dev, int32_t *bonus_dev,
                            const SampleArgs *sa, cudaStream_t s) {
@@ -1045,41 +1031,21 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
         st = step_kind_eager(c, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa, s);
         return st == MSD_OK ? post_status(c, s) : st;
     }
-    int need = max_L_bound(c);
     const bool stamped = c->gplan && gemm_stamp_on(c->gplan);
     msd_ctx::StepGraph *g = nullptr;
-    bool rollover = false;
     for (auto &x : c->graphs)
-        if (x.stamped == stamped && same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa)) {
-            if (x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi)) g = &x;
-            else rollover = true;
-        }
-    if (!g) {
-        if (rollover) {   // refresh the bound of L from the device before a new bucket
-            std::vector<int> L(c->B);
-            CU(cudaStreamSynchronize(s));
-            CU(cudaMemcpy(L.data(), c->seq_len, sizeof(int) * c->B, cudaMemcpyDeviceToHost));
-            for (int b = 0; b < c->B; ++b) c->L_bound[b] = L[b];
-            need = max_L_bound(c);
-            for (auto &x : c->graphs)
-                if (x.stamped == stamped &&
-                    same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa) &&
-                    x.bucket_hi >= need && (!g || x.bucket_hi < g->bucket_hi))
-                    g = &x;
-        }
-    }
+        if (x.stamped == stamped && same_buffers(x, kind, tree, argmax_dev, path_dev, accept_len_dev, bonus_dev, sa))
+            g = &x;
     if (!g) {
         msd_ctx::StepGraph ng;
         ng.kind = kind;
         ng.stamped = stamped;
-        ng.bucket_hi = std::min(c->S, ((need + c->D + 511) / 512) * 512);
         ng.tree = *tree;
         ng.argmax = argmax_dev; ng.path = path_dev; ng.alen = accept_len_dev; ng.bonus = bonus_dev;
         if (sa) { ng.u = sa->u; ng.temp = sa->temp; }
         if (!c->cap_stream)   // graphs are recorded on a stream of the context's own
             CU(cudaStreamCreateWithFlags(&c->cap_stream, cudaStreamNonBlocking));
         const long l0 = launch_count();
-        c->pb_override = ng.bucket_hi;
         c->capturing = true;
         cudaGraph_t graph = nullptr;
         cudaError_t ce = cudaStreamBeginCapture(c->cap_stream, cudaStreamCaptureModeThreadLocal);
@@ -1093,7 +1059,6 @@ msd_status run_step_graph(msd_ctx *c, int kind, const msd_tree *tree, int32_t *a
             st = MSD_OK;
         }
         c->capturing = false;
-        c->pb_override = 0;
         ng.kernels = launch_count() - l0;
         c->captured_launches += ng.kernels;
         if (ce != cudaSuccess || st != MSD_OK || !graph) {

@@ -209,8 +209,9 @@ def test_capacity_is_refused_on_the_host():
 
 
 def test_step_graph_matches_separate_calls():
-    """msd_step (replayed CUDA graphs, re-recorded when L crosses a 512-position
-    bucket) gives bit-identical steps to msd_draft_tree + msd_verify +
+    """msd_step (one CUDA graph, recorded once and replayed while the cache
+    grows past 512 positions, so attention's split boundaries move between
+    replays) gives bit-identical steps to msd_draft_tree + msd_verify +
     msd_accept_compact."""
     wl = synth.WORKLOADS["tiny"].with_(dtype="bf16", n_text=(440, 440), steps=24)
     w = synth.make_weights(wl)

@@ -58,4 +58,4 @@ def test_stamped_step_graph_times_its_gemms(nodes, depth, k):
     assert prof["gemm_critical_ms"] <= ms, (prof["gemm_critical_ms"], ms)
     assert prof["gemm_bytes"] > prof["gemm_weight_bytes"] > 0
     assert prof["gemm_flops"] <= prof["gemm_mma_flops"] <= 2 * prof["gemm_flops"]
-    assert 0 < prof["gemm_prefetch_bytes"] <= prof["gemm_weight_bytes"]
+    assert 0 < prof["gemm_prefetch_bytes"] <= prof["gemm_weight_bytes"]   # (capped per launch)
