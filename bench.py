@@ -85,15 +85,18 @@ def parse():
     return ap.parse_args()
 
 
-# DRAM traffic of the decode GEMM: ncu dram__bytes_read.sum + dram__bytes_write.sum
-# over the 45 GEMM launches of one 2-layer 7B-width step, divided by the same
-# launches' algorithmic bytes (0.996: no re-reads); per launch of the full
-# workload it is this ratio times its algorithmic bytes per launch. Valid for
-# the GEMM source with this SHA-1 only.
-GEMM_TRAFFIC = {"source_sha1": "193c26f55d2a60d169edb4ddfdc3b5a6a13e3e64", "ratio": 0.9958}
+# DRAM traffic of the GEMMs: ncu dram__bytes_read.sum + dram__bytes_write.sum
+# per launch divided by the same launches' algorithmic bytes. Decode
+# (gemm_cluster_kernel): the 90 launches of two 2-layer 7B-width steps, 0.9946
+# (no re-reads). Many rows (gemm_persist_kernel): two batch-16 draft launches
+# (f_down, q/k/v; 160 token rows), 0.998. Per launch of a full workload it is
+# the ratio times its algorithmic bytes per launch. Valid for the GEMM source
+# with this SHA-1 only.
+GEMM_TRAFFIC = {"source_sha1": "dfb428b4e1511ccd672769040ad5bb0af94a62e1",
+                "ratio": {"hbm": 0.9946, "tensor": 0.998}}
 
 
-def gemm_traffic(bytes_per_launch):
+def gemm_traffic(bytes_per_launch, bound="hbm"):
     import hashlib
     src = os.path.join(ROOT, "paper_2505_14260_gb300", "csrc", "gemm_tc.cu")
     try:
@@ -103,7 +106,7 @@ def gemm_traffic(bytes_per_launch):
         return None
     if sha != GEMM_TRAFFIC["source_sha1"] or not bytes_per_launch:
         return None
-    return GEMM_TRAFFIC["ratio"] * bytes_per_launch
+    return GEMM_TRAFFIC["ratio"][bound] * bytes_per_launch
 
 
 # Output length and average acceptance lengths the paper reports (Sec. 4): the
@@ -755,7 +758,7 @@ def run_msd(args, rank, world, local_rank):
             "tokens_per_s": world * tokens / (ms / 1e3),
             "tau": tokens / (K * B),
             "roofline": dict(roof, **{
-                "traffic": gemm_traffic(roof["bytes_per_launch"]),
+                "traffic": gemm_traffic(roof["bytes_per_launch"], roof["bound"]),
                 "kernel": "gemm_cluster_kernel / gemm_persist_kernel (tcgen05 bf16 GEMMs: 128-row weight "
                           "tiles x token rows, TMA-staged, TMEM accumulators, fused epilogues; all "
                           "projections and LM heads of the step)",

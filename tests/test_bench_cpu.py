@@ -40,7 +40,54 @@ def test_aggregate_rate_is_whole_job_throughput():
 
 def test_gemm_traffic_only_for_the_captured_source(monkeypatch):
     assert bench.gemm_traffic(0) is None
-    v = bench.gemm_traffic(100.0)
-    assert v is None or v == pytest.approx(bench.GEMM_TRAFFIC["ratio"] * 100.0)
+    for bound in ("hbm", "tensor"):
+        v = bench.gemm_traffic(100.0, bound)
+        assert v is None or v == pytest.approx(bench.GEMM_TRAFFIC["ratio"][bound] * 100.0)
     monkeypatch.setitem(bench.GEMM_TRAFFIC, "source_sha1", "0" * 40)
     assert bench.gemm_traffic(100.0) is None
+
+
+def _prof(windows, crit_ms, entry_ms, byts, flops, launches, pre=0.0):
+    return {"windows": windows, "gemm_critical_ms": crit_ms, "gemm_ms": entry_ms, "gemm_bytes": byts,
+            "gemm_flops": flops, "gemm_mma_flops": 2 * flops, "gemm_launches": launches,
+            "gemm_prefetch_bytes": pre, "gemm_weight_bytes": byts}
+
+
+def test_gemm_roofline_is_per_step_from_the_critical_spans():
+    """Per step: the wait-to-exit spans (not the entry spans) divide the bytes;
+    a decode mix (60 flops per byte) is HBM-bound against the copy bandwidth."""
+    r = bench.gemm_roofline(_prof(4, 4 * 3.0, 4 * 4.5, 4 * 18e9, 4 * 60 * 18e9, 4 * 165, 4 * 2e9), 6000.0, "m")
+    assert r["bound"] == "hbm" and r["unit"] == "GB/s"
+    assert r["gemm_ms_per_step"] == pytest.approx(3.0)
+    assert r["gemm_ms_per_step_from_entry"] == pytest.approx(4.5)
+    assert r["achieved"] == pytest.approx(18e9 / 3e-3 / 1e9)
+    assert r["frac"] == pytest.approx(r["achieved"] / 6000.0)
+    assert r["frac_nominal"] == pytest.approx(r["achieved"] / bench.NOMINAL_HBM_GBS)
+    assert r["achieved_after_wait"] == pytest.approx(16e9 / 3e-3 / 1e9)
+    assert r["launches_per_step"] == 165
+
+
+def test_gemm_roofline_past_the_ridge_is_tensor_bound():
+    """A many-row mix (500 flops per byte, above the sustained-bf16 / HBM ridge
+    of about 250) reports TFLOP/s against the sustained bf16 rate."""
+    tf, _ = bench.tensor_peak()
+    r = bench.gemm_roofline(_prof(2, 2 * 18.0, 2 * 20.0, 2 * 27e9, 2 * 500 * 27e9, 2 * 165), 6767.1, "m")
+    assert r["bound"] == "tensor" and r["unit"] == "TFLOP/s"
+    assert r["achieved"] == pytest.approx(500 * 27e9 / 18e-3 / 1e12)
+    assert r["frac"] == pytest.approx(r["achieved"] / tf)
+    assert r["frac_issued"] == pytest.approx(2 * r["frac"])
+
+
+def test_oracle_sample_runs_every_layer_with_two_held():
+    """The CPU baseline's oracle step covers all of the target's layers (two
+    layers' weights held and alternated, their prefilled caches laid down for
+    every layer); nothing is scaled."""
+    wl = synth.WORKLOADS["tiny"].with_(n_layers=5)
+    w = synth.make_weights(wl, layers=bench.OracleSample.HELD)
+    sample = bench.OracleSample(wl, w, synth.make_prompts(wl))
+    assert len(sample.m.w["layers"]) == 5 and len(sample.st.K) == 5
+    assert sample.m.w["layers"][4] is sample.m.w["layers"][0]
+    L0 = sample.st.L
+    assert sample.step_seconds() > 0
+    assert sample.st.L > L0 and all(k.shape[0] == sample.st.L for k in sample.st.K)
+    assert "scaled" not in sample.describe().replace("nothing scaled", "")
