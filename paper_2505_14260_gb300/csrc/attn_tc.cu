@@ -28,8 +28,9 @@
 //
 // Visible keys of a row (Sec. 3.2: a candidate is conditioned on its prefix
 // only): cache positions [0, plen) of its request, and tree slots whose bit is
-// set in its mask. The cache range is cut into splits (a function of the
-// capacity only, so results never depend on L) plus one tree split; the splits
+// set in its mask. The live prefix is cut into splits of whole key tiles (their
+// count a function of the launch's shape, so a result depends on L alone), the
+// last split also taking the tree slots; the splits
 // of a (row tile, head) form a thread-block cluster and combine their
 // partials (O, max, sum) through distributed shared memory in split order:
 // deterministic. Every mbarrier wait is bounded.
@@ -50,7 +51,7 @@ constexpr int ROWS = 64;          // query rows per CTA (MMA M)
 constexpr int KT = 64;            // keys per tile (N of Q K^T, K of P V)
 constexpr int THREADS = 320;      // warp 0 TMA, warp 1 MMA, warps 2-9 softmax
 constexpr int STAGES = 3;
-constexpr int MAX_SPLITS = 9;     // cache splits + the tree split = cluster size
+constexpr int MAX_SPLITS = 9;     // splits of a (row tile, head) = cluster size
 constexpr unsigned long long ATTN_TIMEOUT_NS = 2000000000ull;
 constexpr float RESCALE_LOG2 = 8.f;
 
@@ -75,8 +76,7 @@ struct AttnTcParams {
     int lo_rows;
     int *status;
     int R, rows_per_req, tiles_per_req, nh, cache_slots, tree_slots, mask_words;
-    int nsplit_cache, has_tree;
-    int tree_merged;          // the tree keys follow the cache keys in the one cache split (no tree split)
+    int nsplit, has_tree;     // splits of the live prefix; the tree keys follow in the last one
     int cache_early;          // cache K/V may be requested before the wait (not written by the previous kernel)
     float scale_log2;
 };
@@ -277,7 +277,6 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int blk = tile / p.tiles_per_req;
     const int r0 = blk * p.rows_per_req + (tile - blk * p.tiles_per_req) * ROWS;
     const int r_end = min(r0 + ROWS, (blk + 1) * p.rows_per_req);
-    const bool is_tree = p.has_tree && !p.tree_merged && split == p.nsplit_cache;
     const int H = p.nh * HD;
 
     const uint32_t base = (su32(smem_raw) + 1023u) & ~1023u;
@@ -330,20 +329,15 @@ __global__ void __launch_bounds__(THREADS, 1)
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_base;
 
-    // Key range of this split. The request's live prefix is cut into
-    // nsplit_cache equal runs of whole 64-key tiles (the count is fixed per
-    // context, so a result depends on L alone, never on the launch's bound of
-    // L); a tree split, or the tree tiles after the cache tiles of a merged
-    // CTA, covers the tree slots.
+    // Key range of this split. The request's live prefix is cut into nsplit
+    // equal runs of whole 64-key tiles (nsplit depends only on the launch's
+    // shape, so a result depends on L alone); the last split, whose run is the
+    // shortest, takes the tree keys after its cache keys.
     const int live = min(s_pmax, p.cache_slots);
-    const int per_split = ((live + KT - 1) / KT + p.nsplit_cache - 1) / p.nsplit_cache * KT;
-    int k_lo = 0, k_hi = 0;
-    if (!is_tree) {
-        k_lo = split * per_split;
-        k_hi = min(k_lo + per_split, live);
-    }
+    const int per_split = ((live + KT - 1) / KT + p.nsplit - 1) / p.nsplit * KT;
+    const int k_lo = split * per_split, k_hi = min(k_lo + per_split, live);
     const int nc = k_hi > k_lo ? (k_hi - k_lo + KT - 1) / KT : 0;      // cache tiles
-    const bool has_tree_tiles = is_tree || (p.has_tree && p.tree_merged);
+    const bool has_tree_tiles = p.has_tree && split == p.nsplit - 1;
     const int ntiles = nc + (has_tree_tiles ? (p.tree_slots + KT - 1) / KT : 0);
     const int row_base_c = (req * p.nh + h) * p.cache_slots;
     const int row_base_t = (req * p.nh + h) * p.tree_slots;
@@ -571,7 +565,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     const bool ok = !dead && !abort_flag;
 
-    const int nsplit = p.nsplit_cache + (p.has_tree && !p.tree_merged);
+    const int nsplit = p.nsplit;
     if (nsplit == 1) {
         if (valid && ok) {
             const float inv = l_sum > 0.f ? 1.f / l_sum : 0.f;
@@ -674,22 +668,16 @@ struct MapKeyHash {
 
 struct AttnTcPlan {
     int num_sms = 148;
-    int splits = 1;            // cache splits of a decode launch: fixed per context
     PFN_cuTensorMapEncodeTiled_v12000 encode = nullptr;
     std::unordered_map<MapKey, CUtensorMap, MapKeyHash> maps;
     bool attr_set = false;
 };
 
-bool attn_tc_plan_create(AttnTcPlan **out, int decode_ctas) {
+bool attn_tc_plan_create(AttnTcPlan **out) {
     AttnTcPlan *p = new AttnTcPlan();
     int dev = 0;
     cudaGetDevice(&dev);
     cudaDeviceGetAttribute(&p->num_sms, cudaDevAttrMultiProcessorCount, dev);
-    // A CTA fills an SM (one per SM): a decode launch of decode_ctas (row
-    // tile, head) pairs takes as many cache splits as keep it, with the tree
-    // split, within one wave. The count is fixed for the context, so a result
-    // never depends on which launch (eager call or graph bucket) computed it.
-    p->splits = std::max(1, std::min(MAX_SPLITS - 1, p->num_sms / std::max(1, decode_ctas) - 1));
     cudaDriverEntryPointQueryResult q;
     void *fn = nullptr;
     if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) !=
@@ -733,14 +721,9 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     const int row_tiles = n_blocks * tiles_per_req;
     const long base = (long)row_tiles * a.nh;
     const int has_tree = a.mask != nullptr;
-    // Enough (row tile, head) CTAs already: one cache split per CTA, and when
-    // they fill a wave by themselves the tree keys join it (no tree split);
-    // otherwise the context's fixed split count.
-    const bool single = base * (1 + has_tree) >= p->num_sms;
-    const int nsplit = single ? 1 : p->splits;
-    const int tree_merged = has_tree && single && base >= p->num_sms;
-    const int tot = nsplit + (has_tree && !tree_merged);
-    if (tot > MAX_SPLITS) return false;
+    // One CTA fills an SM: as many splits per (row tile, head) as keep the
+    // launch within one wave (a function of the launch's shape alone).
+    const int nsplit = (int)std::max<long>(1, std::min<long>(MAX_SPLITS, p->num_sms / base));
     const long lo_rows = a.lo / a.hd;
     const long kc_rows = (long)B * a.nh * a.cache_slots + lo_rows;
     const CUtensorMap *mkc = kv_map(p, a.cache_k, kc_rows, a.hd);
@@ -768,9 +751,8 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.cache_slots = a.cache_slots;
     tp.tree_slots = a.tree_slots;
     tp.mask_words = a.mask_words;
-    tp.nsplit_cache = nsplit;
     tp.has_tree = has_tree;
-    tp.tree_merged = tree_merged;
+    tp.nsplit = nsplit;
     tp.cache_early = a.cache_fresh ? 0 : 1;
     tp.scale_log2 = a.scale * 1.4426950408889634f;
     const size_t smem = 1024 + (a.hd == 128 ? (size_t)STAGES * Lay<128>::STAGE : (size_t)STAGES * Lay<64>::STAGE);
@@ -786,7 +768,7 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     // the splits of one (row tile, head) run as one cluster (z = splits)
     cudaLaunchConfig_t lc;
     memset(&lc, 0, sizeof lc);
-    lc.gridDim = dim3(row_tiles, a.nh, tot);
+    lc.gridDim = dim3(row_tiles, a.nh, nsplit);
     lc.blockDim = dim3(THREADS);
     lc.dynamicSmemBytes = smem;
     lc.stream = s;
@@ -794,7 +776,7 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = 1;
     at[0].val.clusterDim.y = 1;
-    at[0].val.clusterDim.z = tot;
+    at[0].val.clusterDim.z = nsplit;
     at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     at[1].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = at;

@@ -8,9 +8,8 @@ namespace msd {
 
 struct AttnTcPlan;
 
-// Per-context plan (tensor-map cache, split count); decode_ctas = the (row
-// tile of 64, head) pairs of a decode launch.
-bool attn_tc_plan_create(AttnTcPlan **out, int decode_ctas);
+// Per-context plan (tensor-map cache, SM count).
+bool attn_tc_plan_create(AttnTcPlan **out);
 void attn_tc_plan_destroy(AttnTcPlan *p);
 
 // a.R rows grouped by request in blocks of rows_per_req; each row's visible

@@ -856,10 +856,7 @@ msd_status msd_create(const msd_config *cfg, const msd_weights *w, msd_ctx **out
     if (ok) ok = cudaMallocHost(&c->status_host, sizeof(int)) == cudaSuccess;
     if (ok) ok = cudaEventCreateWithFlags(&c->status_ev, cudaEventDisableTiming) == cudaSuccess;
     if (ok && cfg->dtype == MSD_BF16) ok = gemm_plan_create(&c->gplan, c->Rmax, c->H, c->F, c->V);
-    if (ok && cfg->dtype == MSD_BF16) {
-        const int decode_rows = std::max(c->N, std::max(c->k, c->D1));
-        ok = attn_tc_plan_create(&c->aplan, c->B * ((decode_rows + 63) / 64) * c->nh);
-    }
+    if (ok && cfg->dtype == MSD_BF16) ok = attn_tc_plan_create(&c->aplan);
     c->lpack.assign(c->NL, msd_ctx::LayerPack());
     if (ok && cfg->dtype == MSD_BF16) ok = pack_weights(c);
     if (!ok) {

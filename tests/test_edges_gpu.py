@@ -158,10 +158,11 @@ def test_bf16_context_never_reads_its_borrowed_projection_matrices():
             assert torch.equal(p, q), f"step {s}"
 
 
-def test_tree_keys_merged_into_single_split_matches_oracle():
+def test_single_split_attention_matches_oracle():
     """When the (row tile, head) CTAs of a launch fill a wave by themselves
     (40 requests x 4 heads on the tiny model), attention takes each request's
-    whole cache in one CTA and the tree keys follow in the same CTA (no
-    separate tree split); a ragged batch against the oracle."""
+    whole cache and then its tree keys in one CTA (no cluster, no combine); a
+    ragged batch against the oracle. (Batch 1 on the tiny model runs nine
+    splits per head, the last one with the tree keys.)"""
     wl = synth.WORKLOADS["tiny"].with_(dtype="bf16", batch=40, n_text=(8, 90), steps=2)
     run_parity(wl, wl.steps, (0, 17, 39))
