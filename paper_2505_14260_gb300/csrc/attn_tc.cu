@@ -202,13 +202,15 @@ __device__ __forceinline__ void tmem_st16(uint32_t taddr, const uint32_t *r) {
         : "memory");
 }
 
-// Barrier of the 256 softmax threads (named barrier 1; the TMA and MMA warps
-// never join it). The warp reconverges first: the barrier's aligned form needs
-// every lane of a warp to reach it together.
-__device__ __forceinline__ void softmax_sync() {
+// Barrier of the two softmax warps that share TMEM lane quarter q (named
+// barrier 1 + q, 64 threads; no other warp joins it): they exchange their
+// rows' tile maxima and sums through shared memory. The warp reconverges
+// first: the barrier's aligned form needs every lane of a warp to reach it
+// together.
+__device__ __forceinline__ void softmax_sync(int quarter) {
     __syncwarp();
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
-    asm volatile("barrier.sync.aligned 1, 256;" ::: "memory");
+    asm volatile("barrier.sync.aligned %0, 64;" ::"r"(1 + quarter) : "memory");
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
 }
 
@@ -507,7 +509,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             // the row's tile maximum over both halves
             float *xm = s_xmax + ((j & 1) * 2 + hf) * ROWS;
             if (lane < 16) xm[row_local] = mx;
-            softmax_sync();
+            softmax_sync(quarter);
             if (lane < 16) mx = fmaxf(mx, s_xmax[((j & 1) * 2 + (hf ^ 1)) * ROWS + row_local]);
             // move the reference maximum only when the tile's exceeds it by > 2^8
             // (and O already holds visible keys: otherwise O is exactly 0). The
@@ -560,7 +562,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         // the row's sum over both halves
         if (lane < 16) s_xmax[(4 + hf) * ROWS + row_local] = l_sum;
-        softmax_sync();
+        softmax_sync(quarter);
         if (lane < 16) l_sum += s_xmax[(4 + (hf ^ 1)) * ROWS + row_local];
     }
     const bool ok = !dead && !abort_flag;
@@ -604,41 +606,54 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int per = (nrows + nsplit - 1) / nsplit;
         const int row_lo = (int)rank * per, row_hi = min(nrows, row_lo + per);
         const uint32_t o_local = su32(s_o), ml_local = su32(s_ml);
-        constexpr int C4 = HD / 4, NWARP = THREADS / 32;
-        for (int rr = row_lo + warp; rr < row_hi; rr += NWARP) {
+        // a half-warp per row (16 lanes, HD/64 float4 each): every row of the
+        // slice in one pass at the decode shapes
+        constexpr int C4 = HD / 4, NHALF = THREADS / 16, PER_LANE = C4 / 16;
+        const int hl = lane & 15;
+        for (int r2 = row_lo + (threadIdx.x >> 4); r2 - (int)(lane >> 4) < row_hi; r2 += NHALF) {
+            const bool live = r2 < row_hi;
+            const int rr = live ? r2 : row_lo;
             float2 ml = make_float2(-INFINITY, 0.f);
-            if (lane < nsplit) ml = dsmem_ld_f2(dsmem_addr(ml_local + rr * 8, lane));
-            float4 v[MAX_SPLITS];
+            if (live && hl < nsplit) ml = dsmem_ld_f2(dsmem_addr(ml_local + rr * 8, hl));
+            float4 v[MAX_SPLITS][PER_LANE];
 #pragma unroll
             for (int sp = 0; sp < MAX_SPLITS; ++sp)
-                if (lane < C4 && sp < nsplit) v[sp] = dsmem_ld_f4(dsmem_addr(o_local + (rr * L::LD + 4 * lane) * 4, sp));
-            // lane sp holds split sp's (m, l); warp shuffles give the max and the sum
-            const float M = warp_max(ml.x);
-            const float w = (lane < nsplit && M != -INFINITY) ? exp2f(ml.x - M) : 0.f;
+#pragma unroll
+                for (int e = 0; e < PER_LANE; ++e)
+                    if (live && sp < nsplit)
+                        v[sp][e] = dsmem_ld_f4(dsmem_addr(o_local + (rr * L::LD + 4 * (hl + 16 * e)) * 4, sp));
+            // lane sp of the half holds split sp's (m, l); shuffles within the
+            // half give the max and the sum
+            float M = ml.x;
+#pragma unroll
+            for (int o = 8; o > 0; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o, 16));
+            const float w = (hl < nsplit && M != -INFINITY) ? exp2f(ml.x - M) : 0.f;
             // the normaliser summed in split order (empty splits add exact zeros),
             // so a launch's result never depends on how many empty splits it has
             const float wl = w * ml.y;
             float den = 0.f;
 #pragma unroll
             for (int sp = 0; sp < MAX_SPLITS; ++sp) {
-                const float t = __shfl_sync(0xffffffffu, wl, sp);
+                const float t = __shfl_sync(0xffffffffu, wl, sp, 16);
                 if (sp < nsplit) den += t;
             }
             const float inv = den > 0.f ? 1.f / den : 0.f;
             const float wn = w * inv;
             float wsp[MAX_SPLITS];
 #pragma unroll
-            for (int sp = 0; sp < MAX_SPLITS; ++sp) wsp[sp] = __shfl_sync(0xffffffffu, wn, sp);
-            if (lane < C4) {
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (int sp = 0; sp < MAX_SPLITS; ++sp) wsp[sp] = __shfl_sync(0xffffffffu, wn, sp, 16);
+            if (live && !abort_flag) {
 #pragma unroll
-                for (int sp = 0; sp < MAX_SPLITS; ++sp)
-                    if (sp < nsplit) {
-                        acc.x += wsp[sp] * v[sp].x; acc.y += wsp[sp] * v[sp].y;
-                        acc.z += wsp[sp] * v[sp].z; acc.w += wsp[sp] * v[sp].w;
-                    }
-                if (!abort_flag)
-                    Split<bf16>::store4(p.out + (size_t)(r0 + rr) * H + h * HD + 4 * lane, p.lo, acc);
+                for (int e = 0; e < PER_LANE; ++e) {
+                    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+                    for (int sp = 0; sp < MAX_SPLITS; ++sp)
+                        if (sp < nsplit) {
+                            acc.x += wsp[sp] * v[sp][e].x; acc.y += wsp[sp] * v[sp][e].y;
+                            acc.z += wsp[sp] * v[sp][e].z; acc.w += wsp[sp] * v[sp][e].w;
+                        }
+                    Split<bf16>::store4(p.out + (size_t)(r0 + rr) * H + h * HD + 4 * (hl + 16 * e), p.lo, acc);
+                }
             }
         }
         cluster_sync();                    // partials stay readable until all are done
