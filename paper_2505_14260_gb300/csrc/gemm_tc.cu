@@ -845,27 +845,6 @@ __device__ __forceinline__ uint32_t c_mapa(uint32_t local, uint32_t rank) {
     return a;
 }
 
-__device__ __forceinline__ float4 c_dsmem_ld4(uint32_t local, uint32_t rank) {
-    uint32_t a;
-    asm volatile("mapa.shared::cluster.u32 %0, %1, %2;" : "=r"(a) : "r"(local), "r"(rank));
-    float4 v;
-    asm volatile("ld.shared::cluster.v4.f32 {%0,%1,%2,%3}, [%4];"
-                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(a));
-    return v;
-}
-
-// (no memory clobber: the partials are read only after a barrier, which is
-// itself a compiler barrier, and the loads may overlap one another)
-__device__ __forceinline__ float4 c_smem_ld4(uint32_t local) {
-    float4 v;
-    asm volatile("ld.shared.v4.f32 {%0,%1,%2,%3}, [%4];"
-                 : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w)
-                 : "r"(local));
-    return v;
-}
-
-
 // Where a CTA finds the S partials of the token columns it owns, [c_lo,
 // c_hi) = [rank * BN / S, (rank + 1) * BN / S): its own partial ([BN][128]
 // fp32, all columns) and, for S > 1, the other ranks' slices of its columns,
