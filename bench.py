@@ -92,7 +92,7 @@ def parse():
 # (f_down, q/k/v; 160 token rows), 0.998. Per launch of a full workload it is
 # the ratio times its algorithmic bytes per launch. Valid for the GEMM source
 # with this SHA-1 only.
-GEMM_TRAFFIC = {"source_sha1": "e4b0f48a05431d6c0635e98a3220dcb6de291f20",
+GEMM_TRAFFIC = {"source_sha1": "80a506e7c16b4583bef1213803dd6fc2f915ad89",
                 "ratio": {"hbm": 0.9946, "tensor": 0.998}}
 
 

@@ -365,7 +365,8 @@ msd_status msd_test_wait_timeout(msd_ctx *ctx, int64_t limit_ns, void *stream);
  * the last read, their time and their algorithmic bytes (every weight element
  * once + activations read + output written, read too when accumulating), and
  * starts a new window. Enabling either mode also starts a new window.
- * Errors: MSD_ERR_INVALID (mode out of range), MSD_ERR_CUDA (mode 2 buffers). */
+ * The stamp buffers are made with the context; enabling allocates nothing.
+ * Errors: MSD_ERR_INVALID (mode out of range), MSD_ERR_CUDA (the stamp reset failed). */
 typedef struct {
     int64_t kernel_launches;
     int64_t gemm_launches;

@@ -1564,7 +1564,9 @@ bool gemm_plan_create(GemmPlan **out, int, int, int, int) {
     }
     p->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     if (cudaMalloc(&p->ws, WS_BYTES) != cudaSuccess ||
-        cudaMalloc(&p->counters, sizeof(int) * N_COUNTERS) != cudaSuccess) {
+        cudaMalloc(&p->counters, sizeof(int) * N_COUNTERS) != cudaSuccess ||
+        cudaMalloc(&p->stamps, sizeof(unsigned long long) * 3 * MAX_STAMPS) != cudaSuccess ||
+        cudaMalloc(&p->stamp_acc, sizeof(StampAcc)) != cudaSuccess) {
         gemm_plan_destroy(p);
         return false;
     }
@@ -1584,13 +1586,6 @@ void gemm_plan_destroy(GemmPlan *p) {
 }
 
 bool gemm_profile_enable(GemmPlan *p, int mode) {
-    if (mode == 2 && !p->stamps) {
-        if (cudaMalloc(&p->stamps, sizeof(unsigned long long) * 3 * MAX_STAMPS) != cudaSuccess ||
-            cudaMalloc(&p->stamp_acc, sizeof(StampAcc)) != cudaSuccess) {
-            cudaGetLastError();
-            return false;
-        }
-    }
     p->profile = mode == 1;
     p->stamp_mode = mode == 2;
     p->stamp_active = false;

@@ -114,7 +114,8 @@ int *noalloc_status_word();
 // *status. Returns false if the launch failed.
 bool launch_wait_probe(int *status, long long limit_ns, cudaStream_t s);
 
-// mode 0 off, 1 events, 2 stamps; false if the stamp buffers cannot be made.
+// mode 0 off, 1 events, 2 stamps (buffers made with the plan); false if the
+// stamp reset fails.
 bool gemm_profile_enable(GemmPlan *p, int mode);
 bool gemm_profile_on(const GemmPlan *p);     // mode 1
 bool gemm_stamp_on(const GemmPlan *p);       // mode 2

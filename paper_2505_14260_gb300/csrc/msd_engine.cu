@@ -1215,7 +1215,7 @@ msd_status msd_profile_enable(msd_ctx *c, int32_t mode) {
     if (!c || mode < 0 || mode > 2) return MSD_ERR_INVALID;
     c->err.clear();
     if (c->gplan && !gemm_profile_enable(c->gplan, mode))
-        return fail(c, MSD_ERR_CUDA, "GEMM launch stamps: device buffers or reset failed");
+        return fail(c, MSD_ERR_CUDA, "GEMM launch stamps: reset failed");
     return MSD_OK;
 }
 
