@@ -90,3 +90,29 @@ def test_tree_set_nodes_copies_tokens_and_parents_only():
         t.set_nodes(0, [1, 2], [-1])                      # one parent entry per node
     with pytest.raises(ValueError):
         t.set_nodes(0, list(range(N + 1)), [-1] * (N + 1))
+
+
+def _header_struct_fields(name):
+    import re
+    text = open(os.path.join(ROOT, "include", "msd.h")).read()
+    text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+    body = re.search(r"typedef struct\s*\{([^}]*)\}\s*" + name + r"\s*;", text, flags=re.S).group(1)
+    fields = []
+    for decl in body.split(";"):
+        decl = decl.strip()
+        if decl:
+            fields += [n.strip().lstrip("*") for n in decl.split(None, 1)[1].split(",")]
+    return fields
+
+
+@pytest.mark.parametrize("cname,pyname", [("msd_profile", "msd_profile"), ("msd_state_view", "msd_state_view")])
+def test_binding_structs_match_the_header(cname, pyname):
+    """The ctypes mirrors of the header's output structs list the same fields
+    in the same order (the library writes them by position)."""
+    from paper_2505_14260_gb300 import msd
+    assert [f for f, _ in getattr(msd, pyname)._fields_] == _header_struct_fields(cname)
+
+
+def test_profile_enable_rejects_a_null_context(libmsd):
+    from paper_2505_14260_gb300 import msd
+    assert libmsd.msd_profile_enable(None, 2) == msd.MSD_ERR_INVALID

@@ -91,3 +91,21 @@ def test_oracle_sample_runs_every_layer_with_two_held():
     assert sample.step_seconds() > 0
     assert sample.st.L > L0 and all(k.shape[0] == sample.st.L for k in sample.st.K)
     assert "scaled" not in sample.describe().replace("nothing scaled", "")
+
+
+def test_weights_with_layers_kept_equal_the_full_set():
+    """make_weights(layers=n) draws the whole random stream and keeps the first
+    n decoder layers: every kept tensor equals its value in the full set (the
+    reference arm's held layers are the workload's own)."""
+    import torch
+    wl = synth.WORKLOADS["tiny"].with_(n_layers=3)
+    full, part = synth.make_weights(wl), synth.make_weights(wl, layers=2)
+    assert len(part["layers"]) == 2
+    for k, v in full.items():
+        if k == "layers":
+            for a, b in zip(v[:2], part["layers"]):
+                assert a.keys() == b.keys() and all(torch.equal(a[n], b[n]) for n in a)
+        elif k == "draft":
+            assert all(torch.equal(v[n], part[k][n]) for n in v)
+        else:
+            assert torch.equal(v, part[k]), k
