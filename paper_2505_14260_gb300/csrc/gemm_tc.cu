@@ -147,10 +147,10 @@ __device__ __forceinline__ uint64_t smem_desc(uint32_t saddr) {
 }
 
 // Instruction descriptor, kind::f16: fp32 accumulate, bf16 A and B, both
-// K-major, N = BN, M = 128.
-__device__ __forceinline__ uint32_t instr_desc(int BN) {
+// K-major, N = BN, M = 128 (256 for a two-SM tile).
+__device__ __forceinline__ uint32_t instr_desc(int BN, int M = BM) {
     return (1u << 4) | (1u << 7) | (1u << 10) | ((uint32_t)(BN >> 3) << 17) |
-           ((uint32_t)(BM >> 4) << 24);
+           ((uint32_t)(M >> 4) << 24);
 }
 
 __device__ __forceinline__ void mma_bf16(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc,
@@ -166,6 +166,73 @@ __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile(
         "tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar)
         : "memory");
+}
+
+// Two-SM tiles (tcgen05 cta_group::2; CTAs 2j and 2j+1 of a cluster are a
+// pair). The even CTA issues M = 256 MMAs: each CTA's own 128 weight rows are A,
+// at the same shared-memory offset in both; each CTA holds BN/2 token columns
+// of B (the even CTA the first half); each CTA's TMEM receives its own 128 rows
+// x BN. Both CTAs' copies complete on the even CTA's stage barrier.
+__device__ __forceinline__ void mma_bf16_pair(uint32_t tmem_d, uint64_t a, uint64_t b, uint32_t idesc,
+                                              uint32_t accumulate) {
+    asm volatile(
+        "{\n.reg .pred p;\n"
+        "setp.ne.b32 p, %4, 0;\n"
+        "tcgen05.mma.cta_group::2.kind::f16 [%0], %1, %2, %3, p;\n}" ::"r"(tmem_d),
+        "l"(a), "l"(b), "r"(idesc), "r"(accumulate));
+}
+
+// Arrives, once the pair's MMAs issued so far complete, on the mbarrier at the
+// same offset in each CTA of cta_mask (cluster ranks).
+__device__ __forceinline__ void mma_commit_pair(uint32_t bar, uint16_t cta_mask) {
+    asm volatile(
+        "tcgen05.commit.cta_group::2.mbarrier::arrive::one.shared::cluster.multicast::cluster.b64 [%0], %1;" ::"r"(
+            bar),
+        "h"(cta_mask)
+        : "memory");
+}
+
+// 2-D tensor copy into this CTA's shared memory completing on an mbarrier of
+// either CTA of the pair (a shared::cluster address).
+__device__ __forceinline__ void tma_load_2d_pair(uint32_t dst, const CUtensorMap *map, int x, int y,
+                                                 uint32_t cluster_bar) {
+    asm volatile(
+        "cp.async.bulk.tensor.2d.shared::cluster.global.mbarrier::complete_tx::bytes.cta_group::2"
+        " [%0], [%1, {%2, %3}], [%4];" ::"r"(dst),
+        "l"(map), "r"(x), "r"(y), "r"(cluster_bar)
+        : "memory");
+}
+
+// Arrive (release, cluster scope) on an mbarrier of another CTA of the cluster.
+__device__ __forceinline__ void mbar_arrive_remote(uint32_t cluster_addr) {
+    asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(cluster_addr) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_cluster(uint32_t bar, uint32_t parity) {
+    uint32_t ok;
+    asm volatile(
+        "{\n.reg .pred p;\n"
+        "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n"
+        "selp.b32 %0, 1, 0, p;\n}"
+        : "=r"(ok)
+        : "r"(bar), "r"(parity)
+        : "memory");
+    return ok != 0;
+}
+
+// Bounded wait on a barrier another CTA of the cluster arrives on.
+__device__ bool mbar_wait_cluster(uint32_t bar, uint32_t parity, volatile int *abort_flag, int *status) {
+    if (mbar_try_cluster(bar, parity)) return true;
+    const unsigned long long t0 = gtimer();
+    while (true) {
+        if (mbar_try_cluster(bar, parity)) return true;
+        if (*abort_flag) return false;
+        if (gtimer() - t0 > TIMEOUT_NS) {
+            *abort_flag = 1;
+            set_status(status, ST_TIMEOUT);
+            return false;
+        }
+    }
 }
 
 // TMEM loads of this warp's 32 lanes, 16 or 32 columns, each waited for in
@@ -1122,11 +1189,12 @@ __device__ __forceinline__ void c_reduce_norm(const CkParams &p, const PartSrc &
     }
 }
 
+template <bool PAIR>
 __global__ void __launch_bounds__(C_THREADS)
     gemm_cluster_kernel(const __grid_constant__ CUtensorMap mx, const __grid_constant__ CUtensorMap mxl,
-                        const CkParams p) {
+                        const __grid_constant__ CUtensorMap mw, const CkParams p) {
     extern __shared__ uint8_t smem_raw[];
-    __shared__ __align__(8) uint64_t bars[2 * C_STAGES + 2];
+    __shared__ __align__(8) uint64_t bars[2 * C_STAGES + 3];
     __shared__ uint32_t tmem_base;
     __shared__ volatile int abort_flag;
     __shared__ float s_rinv[128];     // folded RMSNorm (consumer): 1/rms of each token column
@@ -1147,7 +1215,12 @@ __global__ void __launch_bounds__(C_THREADS)
     const int BN = p.BN;
     const int stages = p.stages;
     const bool has_lo = p.has_lo != 0;
-    const uint32_t b_bytes = (uint32_t)BN * BK * 2;          // one plane of a token stage
+    // Two-SM mode (one K split only): CTAs 2j and 2j+1 run one M = 256 tile;
+    // each holds its own weight rows and half of the token columns.
+    constexpr bool pair = PAIR;
+    const uint32_t half = pair ? (blockIdx.x & 1u) : 0u;       // 1: the odd CTA of a pair
+    const int BNs = pair ? BN / 2 : BN;                        // token columns in this CTA's stages
+    const uint32_t b_bytes = (uint32_t)BNs * BK * 2;         // one plane of a token stage
     const uint32_t bs_bytes = has_lo ? 2 * b_bytes : b_bytes; // hi, then lo
     const size_t blk_elems = A_BYTES / 2;
     const bf16 *wblk = p.wpacked + ((size_t)blockIdx.x * KB + kb0) * blk_elems;
@@ -1157,6 +1230,7 @@ __global__ void __launch_bounds__(C_THREADS)
     const uint32_t full0 = smem_u32(&bars[0]), empty0 = smem_u32(&bars[C_STAGES]);
     const uint32_t done = smem_u32(&bars[2 * C_STAGES]);
     const uint32_t recv_bar = smem_u32(&bars[2 * C_STAGES + 1]);   // the other ranks' slices have landed
+    const uint32_t pexit = smem_u32(&bars[2 * C_STAGES + 2]);      // (pair) the other CTA is done with its TMEM
 
     if (threadIdx.x == 0) {
         stamp_min(p.stamp, 0);
@@ -1166,31 +1240,56 @@ __global__ void __launch_bounds__(C_THREADS)
         }
         mbar_init(done, 1);
         mbar_init(recv_bar, 1);
+        mbar_init(pexit, 1);
         abort_flag = 0;
         asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
     }
     if (warp == 1) {
-        asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
-                         smem_u32(&tmem_base)),
-                     "r"(p.tmem_cols)
-                     : "memory");
-        asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        if constexpr (pair) {   // both CTAs of the pair allocate together (the same columns in each)
+            asm volatile("tcgen05.alloc.cta_group::2.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             smem_u32(&tmem_base)),
+                         "r"(p.tmem_cols)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::2.sync.aligned;" ::: "memory");
+        } else {
+            asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(
+                             smem_u32(&tmem_base)),
+                         "r"(p.tmem_cols)
+                         : "memory");
+            asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+        }
     }
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const uint32_t tmem = tmem_base;
+    const uint32_t my_rank = pair ? c_cluster_rank() : 0u;
+    const uint32_t lead_rank = my_rank & ~1u;                 // (pair) the even CTA
+    const uint16_t pair_mask = (uint16_t)(3u << lead_rank);
+    // where this CTA's copies complete: its own barriers, or (pair) the even CTA's
+    const uint32_t sig0 = pair ? c_mapa(full0, lead_rank) : full0;
+    const uint32_t stage_tx = (pair ? 2u : 1u) * (A_BYTES + bs_bytes);
+    // (pair) both CTAs' barriers are initialised before either signals the other's
+    if constexpr (pair) c_cluster_sync();
 
     if (warp == 0) {
         if (lane == 0) {
             asm volatile("prefetch.tensormap [%0];" ::"l"(&mx) : "memory");
             if (has_lo) asm volatile("prefetch.tensormap [%0];" ::"l"(&mxl) : "memory");
+            if (pair) asm volatile("prefetch.tensormap [%0];" ::"l"(&mw) : "memory");
+            // the weight block of pipeline step i: a bulk copy, or (pair) a tensor
+            // copy of its 128 rows that completes on the even CTA's barrier
+            auto load_w = [&](int i, int st) {
+                if (!pair || half == 0) mbar_expect_tx(full0 + 8 * st, stage_tx);
+                if constexpr (pair)
+                    tma_load_2d_pair(a_base + st * A_BYTES, &mw, 0, (int)(((size_t)blockIdx.x * KB + kb0 + i) * BM),
+                                     sig0 + 8 * st);
+                else
+                    bulk_load(a_base + st * A_BYTES, wblk + (size_t)i * blk_elems, A_BYTES, full0 + 8 * st);
+            };
             // weights first (they never depend on the previous kernel), then wait
             const int n_pre = min(stages, nk);
-            for (int j = 0; j < n_pre; ++j) {
-                mbar_expect_tx(full0 + 8 * j, A_BYTES + bs_bytes);
-                bulk_load(a_base + j * A_BYTES, wblk + (size_t)j * blk_elems, A_BYTES, full0 + 8 * j);
-            }
+            for (int j = 0; j < n_pre; ++j) load_w(j, j);
             pdl_wait();
             stamp_min(p.stamp, 1);
             pdl_trigger();
@@ -1200,17 +1299,22 @@ __global__ void __launch_bounds__(C_THREADS)
             for (; i < nk; ++i) {
                 if (i >= n_pre) {
                     if (!mbar_wait(empty0 + 8 * s, ph ^ 1u, &abort_flag, p.status)) break;
-                    mbar_expect_tx(full0 + 8 * s, A_BYTES + bs_bytes);
-                    bulk_load(a_base + s * A_BYTES, wblk + (size_t)i * blk_elems, A_BYTES, full0 + 8 * s);
+                    load_w(i, s);
                 }
-                tma_load_2d(b_base + s * bs_bytes, &mx, (kb0 + i) * BK, n0, full0 + 8 * s);
-                if (has_lo) tma_load_2d(b_base + s * bs_bytes + b_bytes, &mxl, (kb0 + i) * BK, n0, full0 + 8 * s);
+                if constexpr (pair) {
+                    const int ny = n0 + (int)half * BNs;
+                    tma_load_2d_pair(b_base + s * bs_bytes, &mx, (kb0 + i) * BK, ny, sig0 + 8 * s);
+                    if (has_lo) tma_load_2d_pair(b_base + s * bs_bytes + b_bytes, &mxl, (kb0 + i) * BK, ny, sig0 + 8 * s);
+                } else {
+                    tma_load_2d(b_base + s * bs_bytes, &mx, (kb0 + i) * BK, n0, full0 + 8 * s);
+                    if (has_lo) tma_load_2d(b_base + s * bs_bytes + b_bytes, &mxl, (kb0 + i) * BK, n0, full0 + 8 * s);
+                }
                 if (++s == stages) {
                     s = 0;
                     ph ^= 1u;
                 }
             }
-            if (abort_flag) {
+            if (abort_flag && (!pair || half == 0)) {   // (pair: the even CTA's barriers count both CTAs' copies)
                 volatile int never = 0;
                 for (int j = (i > stages ? i - stages : 0); j < i; ++j)
                     mbar_wait(full0 + 8 * (j % stages), (uint32_t)(j / stages) & 1u, &never, p.status);
@@ -1219,28 +1323,40 @@ __global__ void __launch_bounds__(C_THREADS)
         __syncwarp();
     } else if (warp == 1) {
         pdl_wait();
-        if (lane == 0) {
-            const uint32_t idesc = instr_desc(BN);
+        if (lane == 0 && (!pair || half == 0)) {      // (pair: the even CTA issues for both)
+            const uint32_t idesc = instr_desc(BN, pair ? 2 * BM : BM);
             int s = 0;
             uint32_t ph = 0;
             for (int i = 0; i < nk; ++i) {
-                if (!mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status)) break;
+                if (pair ? !mbar_wait_cluster(full0 + 8 * s, ph, &abort_flag, p.status)
+                         : !mbar_wait(full0 + 8 * s, ph, &abort_flag, p.status))
+                    break;
                 asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
                 const uint64_t ad = smem_desc(a_base + s * A_BYTES);
                 const uint64_t bd = smem_desc(b_base + s * bs_bytes);
                 const uint64_t bl = smem_desc(b_base + s * bs_bytes + b_bytes);
+                if constexpr (pair) {
 #pragma unroll
-                for (int kk = 0; kk < BK / 16; ++kk) {
-                    mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (i != 0) || (kk != 0));
-                    if (has_lo) mma_bf16(tmem, ad + 2 * kk, bl + 2 * kk, idesc, 1u);
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        mma_bf16_pair(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (i != 0) || (kk != 0));
+                        if (has_lo) mma_bf16_pair(tmem, ad + 2 * kk, bl + 2 * kk, idesc, 1u);
+                    }
+                    mma_commit_pair(empty0 + 8 * s, pair_mask);
+                } else {
+#pragma unroll
+                    for (int kk = 0; kk < BK / 16; ++kk) {
+                        mma_bf16(tmem, ad + 2 * kk, bd + 2 * kk, idesc, (i != 0) || (kk != 0));
+                        if (has_lo) mma_bf16(tmem, ad + 2 * kk, bl + 2 * kk, idesc, 1u);
+                    }
+                    mma_commit(empty0 + 8 * s);
                 }
-                mma_commit(empty0 + 8 * s);
                 if (++s == stages) {
                     s = 0;
                     ph ^= 1u;
                 }
             }
-            mma_commit(done);
+            if constexpr (pair) mma_commit_pair(done, pair_mask);
+            else mma_commit(done);
             volatile int never = 0;     // (as gemm_tc_kernel: no MMA outlives the CTA's TMEM)
             mbar_wait(done, 0, &never, p.status);
         }
@@ -1405,7 +1521,22 @@ __global__ void __launch_bounds__(C_THREADS)
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
     if (threadIdx.x == 0) stamp_max(p.stamp, 2);
-    if (warp == 1) {
+    if constexpr (pair) {
+        // the pair frees its tensor memory together, once both CTAs have read
+        // theirs (and, for the odd CTA, once the even one has seen every copy land)
+        if (warp == 1) {
+            if (lane == 0) {
+                mbar_arrive_remote(c_mapa(pexit, my_rank ^ 1u));
+                volatile int never = 0;
+                mbar_wait_cluster(pexit, 0, &never, p.status);
+            }
+            __syncwarp();
+            asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+            asm volatile("tcgen05.dealloc.cta_group::2.sync.aligned.b32 %0, %1;" ::"r"(tmem),
+                         "r"(p.tmem_cols)
+                         : "memory");
+        }
+    } else if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem),
                      "r"(p.tmem_cols)
@@ -1702,6 +1833,27 @@ static const CUtensorMap *get_map(GemmPlan *p, const void *ptr, long rows, long 
     return &p->maps.emplace(key, m).first->second;
 }
 
+// Tensor map over a packed weight buffer as rows of 64 bf16 (blocks of 128 rows
+// are the 16 KB pipeline blocks, already in shared-memory order: no swizzle).
+static const CUtensorMap *get_wmap(GemmPlan *p, const void *packed, long rows) {
+    MapKey key{packed, rows, BK, -1, BM};
+    auto it = p->maps.find(key);
+    if (it != p->maps.end()) return &it->second;
+    CUtensorMap m;
+    memset(&m, 0, sizeof m);
+    cuuint64_t dims[2] = {(cuuint64_t)BK, (cuuint64_t)rows};
+    cuuint64_t strides[1] = {(cuuint64_t)BK * 2};
+    cuuint32_t box[2] = {(cuuint32_t)BK, (cuuint32_t)BM};
+    cuuint32_t estr[2] = {1, 1};
+    if (p->encode(&m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(packed), dims, strides, box, estr,
+                  CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_NONE, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+                  CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) != CUDA_SUCCESS) {
+        fprintf(stderr, "msd: cuTensorMapEncodeTiled failed for packed weights (%ld rows)\n", rows);
+        return nullptr;
+    }
+    return &p->maps.emplace(key, m).first->second;
+}
+
 size_t gemm_pack_bytes(const GemmW &W, int K) {
     long long tiles = 0;
     for (int i = 0; i < W.nseg; ++i) tiles += (W.rows[i] + BM - 1) / BM;
@@ -1752,7 +1904,7 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
         out_off += W.rows[i];
     }
     const int nb = X_lo ? 2 : 1;
-    const size_t stage = A_BYTES + (size_t)nb * BN * BK * 2;
+    size_t stage = A_BYTES + (size_t)nb * BN * BK * 2;
     constexpr size_t HALF_SM = 104u * 1024u, FULL_SM = 200u * 1024u;
     const int per_sm = 3 * stage <= HALF_SM ? 2 : 1;
     int stages = (int)((per_sm == 2 ? HALF_SM : FULL_SM) / stage);
@@ -1762,6 +1914,15 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     while (S > 1 && kblocks / S < 2) --S;
     // own partial [BN][128] fp32 plus the other ranks' slices of this rank's columns
     while (S > 1 && (size_t)BN * BM * 4 + (size_t)(S - 1) * ((BN + S - 1) / S) * BM * 4 > stages * stage) --S;
+    // Two-SM tiles for unsplit launches whose token stage is as large as the
+    // weight block (split token rows, 32 or more): each CTA of a pair holds
+    // half the token columns, so the ring gets a fourth stage.
+    const bool pair = S == 1 && nb == 2 && BN >= 32 && tiles % 2 == 0 && per_sm == 2;
+    const int BNs = pair ? BN / 2 : BN;
+    if (pair) {
+        stage = A_BYTES + (size_t)nb * BNs * BK * 2;
+        stages = std::max(2, std::min((int)(HALF_SM / stage), C_STAGES));
+    }
     ck.M = M;
     ck.kblocks = kblocks;
     ck.BN = BN;
@@ -1775,13 +1936,16 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     ck.ldy = ldy;
     ck.epi = epi;
     ck.status = status;
-    const CUtensorMap *mx = get_map(p, X, M, K, ldx, BN, status);
+    const CUtensorMap *mx = get_map(p, X, M, K, ldx, BNs, status);
     ck.stamp = stamp_slot(p);
-    const CUtensorMap *mxl = X_lo ? get_map(p, X_lo, M, K, ldx, BN, status) : mx;
-    if (!mx || !mxl) return;
+    const CUtensorMap *mxl = X_lo ? get_map(p, X_lo, M, K, ldx, BNs, status) : mx;
+    const CUtensorMap *mw = pair ? get_wmap(p, W.packed, (long)tiles * kblocks * BM) : mx;
+    if (!mx || !mxl || !mw) return;
     const size_t smem = 1024 + (size_t)stages * stage;
     if (!p->cluster_attr_set) {
-        cudaFuncSetAttribute(gemm_cluster_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        cudaFuncSetAttribute(gemm_cluster_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             (int)(1024 + FULL_SM));
+        cudaFuncSetAttribute(gemm_cluster_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              (int)(1024 + FULL_SM));
         p->cluster_attr_set = true;
     }
@@ -1804,12 +1968,13 @@ static void gemm_cluster(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     at[0].val.programmaticStreamSerializationAllowed = 1;
     at[1].id = cudaLaunchAttributeClusterDimension;
-    at[1].val.clusterDim.x = 1;
+    at[1].val.clusterDim.x = pair ? 2u : 1u;
     at[1].val.clusterDim.y = 1;
     at[1].val.clusterDim.z = (unsigned)S;
     lc.attrs = at;
     lc.numAttrs = 2;
-    if (cudaLaunchKernelEx(&lc, gemm_cluster_kernel, *mx, *mxl, ck) != cudaSuccess) {
+    if ((pair ? cudaLaunchKernelEx(&lc, gemm_cluster_kernel<true>, *mx, *mxl, *mw, ck)
+              : cudaLaunchKernelEx(&lc, gemm_cluster_kernel<false>, *mx, *mxl, *mw, ck)) != cudaSuccess) {
         cudaGetLastError();
         flag_kernel<<<1, 1, 0, s>>>(status, ST_RANGE);
         fprintf(stderr, "msd: cluster GEMM launch failed (M=%d K=%d O=%d S=%d)\n", M, K, O, S);
