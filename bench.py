@@ -87,13 +87,13 @@ def parse():
 
 # DRAM traffic of the GEMMs: ncu dram__bytes_read.sum + dram__bytes_write.sum
 # per launch divided by the same launches' algorithmic bytes. Decode
-# (gemm_cluster_kernel): the 90 launches of two 2-layer 7B-width steps, 0.9946
+# (gemm_cluster_kernel): the 90 launches of two 2-layer 7B-width steps, 0.9945
 # (no re-reads). Many rows (gemm_persist_kernel): two batch-16 draft launches
 # (f_down, q/k/v; 160 token rows), 0.998. Per launch of a full workload it is
 # the ratio times its algorithmic bytes per launch. Valid for the GEMM source
 # with this SHA-1 only.
-GEMM_TRAFFIC = {"source_sha1": "80a506e7c16b4583bef1213803dd6fc2f915ad89",
-                "ratio": {"hbm": 0.9946, "tensor": 0.998}}
+GEMM_TRAFFIC = {"source_sha1": "0abc8b22ad69491c3dabc7fc4ce335eb05760889",
+                "ratio": {"hbm": 0.9945, "tensor": 0.998}}
 
 
 def gemm_traffic(bytes_per_launch, bound="hbm"):
