@@ -36,6 +36,14 @@ def test_full_width_two_layers_match_oracle(name, requests):
     run_parity(wl, 2, requests)
 
 
+def test_llava7b_40_node_tree_two_layers_match_oracle():
+    """A 40-node tree at the 7B width (48 token columns: the unsplit gate/up and
+    LM-head GEMMs run as two-SM tiles of 24 columns per CTA, a shape the 60-node
+    workloads do not take), cut to 2 layers."""
+    wl = synth.WORKLOADS["llava7b"].with_(n_layers=2, tree_nodes=40)
+    run_parity(wl, 2, None)
+
+
 def test_llava7b_chain_drafts_two_layers_match_oracle():
     """Chain drafts at the 7B width (top-1 at every depth, N = D + 1 = 7), the
     drafting mode of the paper's n-alpha measurement and of the bench's chain
