@@ -52,6 +52,7 @@ constexpr int KT = 64;            // keys per tile (N of Q K^T, K of P V)
 constexpr int THREADS = 320;      // warp 0 TMA, warp 1 MMA, warps 2-9 softmax
 constexpr int STAGES = 3;
 constexpr int MAX_SPLITS = 9;     // splits of a (row tile, head) = cluster size
+constexpr int ORDER_MAX = 64;     // request blocks a launch can reorder
 constexpr unsigned long long ATTN_TIMEOUT_NS = 2000000000ull;
 constexpr float RESCALE_LOG2 = 8.f;
 
@@ -79,6 +80,8 @@ struct AttnTcParams {
     int nsplit, has_tree;     // splits of the live prefix; the tree keys follow in the last one
     int cache_early;          // cache K/V may be requested before the wait (not written by the previous kernel)
     float scale_log2;
+    int n_order;              // > 0: row-tile blocks launch in this order (longest request first)
+    uint8_t order[ORDER_MAX];
 };
 
 __device__ __forceinline__ uint32_t su32(const void *p) { return (uint32_t)__cvta_generic_to_shared(p); }
@@ -275,9 +278,12 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ float s_xmax[6 * ROWS];     // tile maxima [tile parity][half][row], then row sums [half][row]
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int tile = blockIdx.x, h = blockIdx.y, split = blockIdx.z;
-    const int blk = tile / p.tiles_per_req;
-    const int r0 = blk * p.rows_per_req + (tile - blk * p.tiles_per_req) * ROWS;
+    // heads vary fastest in the launch order, then row tiles, request blocks in
+    // p.order (the CTAs of the longest requests start first)
+    const int h = blockIdx.x, tile = blockIdx.y, split = blockIdx.z;
+    const int pos = tile / p.tiles_per_req;
+    const int blk = p.n_order > 0 ? (int)p.order[pos] : pos;
+    const int r0 = blk * p.rows_per_req + (tile - pos * p.tiles_per_req) * ROWS;
     const int r_end = min(r0 + ROWS, (blk + 1) * p.rows_per_req);
     const int H = p.nh * HD;
 
@@ -726,14 +732,15 @@ static const CUtensorMap *kv_map(AttnTcPlan *p, const void *ptr, long rows, int 
     return &p->maps.emplace(key, m).first->second;
 }
 
-bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, int *status,
-                         cudaStream_t s) {
+bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, const int *order,
+                         int *status, cudaStream_t s) {
     if (a.R <= 0) return true;
     if (a.hd != 64 && a.hd != 128) return false;
     if (a.lo % a.hd) return false;
     const int tiles_per_req = (rows_per_req + ROWS - 1) / ROWS;
     const int n_blocks = a.R / rows_per_req;
     const int row_tiles = n_blocks * tiles_per_req;
+    if (row_tiles > 65535 || a.nh > 65535) return false;   // grid (heads, row tiles, splits)
     const long base = (long)row_tiles * a.nh;
     const int has_tree = a.mask != nullptr;
     // One CTA fills an SM: as many splits per (row tile, head) as keep the
@@ -770,6 +777,16 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.nsplit = nsplit;
     tp.cache_early = a.cache_fresh ? 0 : 1;
     tp.scale_log2 = a.scale * 1.4426950408889634f;
+    if (order && n_blocks > 1 && n_blocks <= ORDER_MAX) {
+        // the kernel indexes rows through it: only a permutation is taken
+        uint64_t seen = 0;
+        for (int i = 0; i < n_blocks; ++i) {
+            if (order[i] < 0 || order[i] >= n_blocks || (seen >> order[i] & 1)) return false;
+            seen |= 1ull << order[i];
+            tp.order[i] = (uint8_t)order[i];
+        }
+        tp.n_order = n_blocks;
+    }
     const size_t smem = 1024 + (a.hd == 128 ? (size_t)STAGES * Lay<128>::STAGE : (size_t)STAGES * Lay<64>::STAGE);
     if (!p->attr_set) {
         cudaFuncSetAttribute(attn_tc_kernel<128>, cudaFuncAttributeMaxDynamicSharedMemorySize,
@@ -783,7 +800,7 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     // the splits of one (row tile, head) run as one cluster (z = splits)
     cudaLaunchConfig_t lc;
     memset(&lc, 0, sizeof lc);
-    lc.gridDim = dim3(row_tiles, a.nh, nsplit);
+    lc.gridDim = dim3(a.nh, row_tiles, nsplit);
     lc.blockDim = dim3(THREADS);
     lc.dynamicSmemBytes = smem;
     lc.stream = s;

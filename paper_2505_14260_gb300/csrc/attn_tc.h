@@ -14,9 +14,12 @@ void attn_tc_plan_destroy(AttnTcPlan *p);
 
 // a.R rows grouped by request in blocks of rows_per_req; each row's visible
 // prefix length comes from its row descriptor. B is the number of requests
-// the cache buffers hold. Returns false if the shape is not supported (the
-// caller reports it).
-bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, int *status,
-                         cudaStream_t s);
+// the cache buffers hold. order (nullable, a permutation of the a.R /
+// rows_per_req blocks, used when there are at most 64): the blocks' launch
+// order, longest first, so that the last wave holds the shortest CTAs (it
+// changes no result). Returns false if the shape is not supported (the caller
+// reports it).
+bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, const int *order,
+                         int *status, cudaStream_t s);
 
 }  // namespace msd

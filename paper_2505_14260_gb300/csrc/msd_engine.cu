@@ -206,7 +206,16 @@ void attention<float>(msd_ctx *c, const AttnArgs<float> &a, int, cudaStream_t s)
 
 template <>
 void attention<bf16>(msd_ctx *c, const AttnArgs<bf16> &a, int rows_per_req, cudaStream_t s) {
-    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, c->status, s)) {
+    // one block per request: launch the longest requests' CTAs first (the host's
+    // bound of each request's L orders them; only scheduling depends on it)
+    int order[64];
+    const int *ord = nullptr;
+    if (a.R == c->B * rows_per_req && c->B > 1 && c->B <= 64) {
+        for (int b = 0; b < c->B; ++b) order[b] = b;
+        std::stable_sort(order, order + c->B, [&](int x, int y) { return c->L_bound[x] > c->L_bound[y]; });
+        ord = order;
+    }
+    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, ord, c->status, s)) {
         c->err = "tensor-core attention: unsupported shape or launch failure";
         launch_flag(c->status, ST_RANGE, s);     // reported by the next call
     }
