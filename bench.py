@@ -87,13 +87,13 @@ def parse():
 
 # DRAM traffic of the GEMMs: ncu dram__bytes_read.sum + dram__bytes_write.sum
 # per launch divided by the same launches' algorithmic bytes. Decode
-# (gemm_cluster_kernel): the 90 launches of two 2-layer 7B-width steps, 0.9945
+# (gemm_cluster_kernel): the 90 launches of two 2-layer 7B-width steps, 0.9947
 # (no re-reads). Many rows (gemm_persist_kernel): two batch-16 draft launches
 # (f_down, q/k/v; 160 token rows), 0.998. Per launch of a full workload it is
 # the ratio times its algorithmic bytes per launch. Valid for the GEMM source
 # with this SHA-1 only.
-GEMM_TRAFFIC = {"source_sha1": "0abc8b22ad69491c3dabc7fc4ce335eb05760889",
-                "ratio": {"hbm": 0.9945, "tensor": 0.998}}
+GEMM_TRAFFIC = {"source_sha1": "4d36367b4ffed3305403572d726f67c9ae4e59be",
+                "ratio": {"hbm": 0.9947, "tensor": 0.998}}
 
 
 def gemm_traffic(bytes_per_launch, bound="hbm"):
@@ -188,6 +188,54 @@ def gemm_roofline(prof, hbm, hbm_kind):
                   "nominal_peak": NOMINAL_HBM_GBS,
                   "achieved_after_wait": after, "frac_after_wait": after / hbm if after else None})
     return r
+
+
+def kernel_breakdown(slots, wl, L_mean_per_req, hbm, windows):
+    """Per-projection (and attention) breakdown of the replayed step from the
+    per-launch stamp slots (msd_profile_slots): launches per step, wait-to-exit
+    time per launch and per step, and the achieved rate against the measured
+    copy bandwidth. GEMM bytes are each launch's algorithmic bytes; verify
+    attention reads every request's visible prefix and tree keys (K and V, 2
+    bytes an element, the stamped steps' mean prefix); the draft passes'
+    attention is timed only."""
+    H, F, V, B, N = wl.hidden, wl.ffn, wl.vocab, wl.batch, wl.tree_nodes
+    glu = 128 * ((F + 63) // 64)
+    names = {(3 * H, H): "q/k/v + RoPE", (H, H): "O + residual", (glu, H): "gate/up + SwiGLU",
+             (H, F): "down + residual", (V, H): "LM head", (H, 2 * H): "input projection"}
+    groups = {}
+    w = max(windows, 1)
+    for sl in slots:
+        if sl["launches"] <= 0:
+            continue
+        phase = "verify" if sl["rows"] == B * N else "draft"
+        flops = None
+        if sl["kind"] == 0:
+            name = f"{phase} {names.get((sl['outputs'], sl['inner']), 'GEMM %dx%d' % (sl['outputs'], sl['inner']))}"
+            byts = sl["bytes"]
+            flops = 2.0 * sl["rows"] * sl["outputs"] * sl["inner"]
+        else:
+            name = f"{phase} tree attention"
+            byts = sum(2 * (L + N) * H * 2 for L in L_mean_per_req) if phase == "verify" else None
+        g = groups.setdefault(name, {"name": name, "launches_per_step": 0.0, "ms_per_step": 0.0,
+                                     "bytes_per_step": None if byts is None else 0.0,
+                                     "flops_per_step": None if flops is None else 0.0})
+        g["launches_per_step"] += sl["launches"] / w
+        g["ms_per_step"] += sl["critical_ms"] / w
+        if byts is not None:
+            g["bytes_per_step"] += byts * sl["launches"] / w
+        if flops is not None:
+            g["flops_per_step"] += flops * sl["launches"] / w
+    out = []
+    for g in groups.values():
+        sec = g["ms_per_step"] / 1e3
+        g["us_per_launch"] = g["ms_per_step"] * 1e3 / g["launches_per_step"]
+        if g["bytes_per_step"] is not None and sec > 0:
+            g["achieved_gbs"] = g["bytes_per_step"] / sec / 1e9
+            g["frac_hbm"] = g["achieved_gbs"] / hbm
+        if g["flops_per_step"] is not None and sec > 0:
+            g["achieved_tflops"] = g["flops_per_step"] / sec / 1e12
+        out.append(g)
+    return sorted(out, key=lambda g: -g["ms_per_step"])
 
 
 # ----------------------------------------------------------------------------
@@ -494,6 +542,8 @@ def run_msd(args, rank, world, local_rank):
         eng.step()
     torch.cuda.synchronize()
     eng.profile_read()
+    eng.profile_slots()
+    Ls0 = eng.state()["seq_len"].cpu().numpy().astype(np.int64)
     e0.record(stream)
     for _ in range(K_prof):
         eng.step()
@@ -501,6 +551,8 @@ def run_msd(args, rank, world, local_rank):
     torch.cuda.synchronize()
     ms_stamped = e0.elapsed_time(e1) / K_prof
     prof = eng.profile_read()
+    slots = eng.profile_slots()
+    Ls1 = eng.state()["seq_len"].cpu().numpy().astype(np.int64)
     eng.profile_enable(0)
     if world > 1:
         dist.barrier()
@@ -509,6 +561,8 @@ def run_msd(args, rank, world, local_rank):
 
     hbm, peak_kind = peaks()
     roof = gemm_roofline(prof, hbm, peak_kind)
+    roof["by_kernel"] = kernel_breakdown(slots, wl, [(a + b) / 2 for a, b in zip(Ls0, Ls1)], hbm,
+                                         prof["windows"])
     sb, parts = step_bytes(wl, [(a + b) / 2 for a, b in zip(L0, L1)])
     step_gbs = sb / (ms / 1e3 / K) / 1e9
 

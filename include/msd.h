@@ -385,6 +385,32 @@ typedef struct {
 msd_status msd_profile_enable(msd_ctx *ctx, int32_t mode);
 msd_status msd_profile_read(msd_ctx *ctx, msd_profile *out);
 
+/* Per-launch breakdown of mode 2 (the tracing subsystem's timeline of the
+ * replayed step). Every launch of a stamped step graph owns a slot: its
+ * tensor-core GEMMs in launch order, then its tree-attention launches (whose
+ * CTAs stamp entry, wait and exit the same way). msd_profile_slots copies, for
+ * each slot of the last stamped graph recorded, the sums over the steps
+ * replayed since the last call of exit - wait (critical_ms) and exit - entry
+ * (span_ms), with the launch's shape, then clears the sums. Slot i describes
+ * the i-th stamped launch of that graph; graphs recorded with another launch
+ * sequence (the sampling step) sum into the same slots, so read once per kind
+ * of step. *n = slots written (at most max). Outside mode 2, *n = 0.
+ * Errors: MSD_ERR_INVALID (null ctx or n, max < 0, null out with max > 0),
+ * MSD_ERR_CUDA. */
+typedef struct {
+    int32_t kind;         /* 0 tensor-core GEMM, 1 tree attention */
+    int32_t rows;         /* GEMM: token rows M; attention: query rows */
+    int32_t outputs;      /* GEMM: output features O; attention: heads */
+    int32_t inner;        /* GEMM: inner size K; attention: head dim */
+    int64_t launches;     /* stamped launches summed (steps replayed) */
+    double bytes;         /* GEMM: algorithmic bytes of one launch; attention: 0
+                             (its bytes follow the visible prefix of each step) */
+    double critical_ms;   /* sum of exit - wait */
+    double span_ms;       /* sum of exit - entry */
+} msd_kernel_slot;
+
+msd_status msd_profile_slots(msd_ctx *ctx, msd_kernel_slot *out, int32_t max, int32_t *n);
+
 /* Device pointers of the context state (see msd_state_view). */
 msd_status msd_state(msd_ctx *ctx, msd_state_view *out);
 

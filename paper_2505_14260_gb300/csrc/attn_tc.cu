@@ -80,6 +80,7 @@ struct AttnTcParams {
     int nsplit, has_tree;     // splits of the live prefix; the tree keys follow in the last one
     int cache_early;          // cache K/V may be requested before the wait (not written by the previous kernel)
     float scale_log2;
+    unsigned long long *stamp;   // profiling: earliest entry, earliest return from the wait, latest exit (ns)
     int n_order;              // > 0: row-tile blocks launch in this order (longest request first)
     uint8_t order[ORDER_MAX];
 };
@@ -278,6 +279,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     __shared__ float s_xmax[6 * ROWS];     // tile maxima [tile parity][half][row], then row sums [half][row]
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    if (threadIdx.x == 0 && p.stamp) atomicMin(p.stamp, gtime());
     // heads vary fastest in the launch order, then row tiles, request blocks in
     // p.order (the CTAs of the longest requests start first)
     const int h = blockIdx.x, tile = blockIdx.y, split = blockIdx.z;
@@ -373,6 +375,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (threadIdx.x == 0)
         for (int i = 0; i < n_early; ++i) issue(i);
     wait_prior();
+    if (threadIdx.x == 0 && p.stamp) atomicMin(p.stamp + 1, gtime());
     allow_dependents();
 
     // TMEM addresses of this warp's lane quarter
@@ -667,6 +670,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
     __syncthreads();
+    if (threadIdx.x == 0 && p.stamp) atomicMax(p.stamp + 2, gtime());
     if (warp == 1) {
         asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
         asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(L::T_COLS)
@@ -733,7 +737,7 @@ static const CUtensorMap *kv_map(AttnTcPlan *p, const void *ptr, long rows, int 
 }
 
 bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, const int *order,
-                         int *status, cudaStream_t s) {
+                         int *status, cudaStream_t s, unsigned long long *stamp) {
     if (a.R <= 0) return true;
     if (a.hd != 64 && a.hd != 128) return false;
     if (a.lo % a.hd) return false;
@@ -777,6 +781,7 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     tp.nsplit = nsplit;
     tp.cache_early = a.cache_fresh ? 0 : 1;
     tp.scale_log2 = a.scale * 1.4426950408889634f;
+    tp.stamp = stamp;
     if (order && n_blocks > 1 && n_blocks <= ORDER_MAX) {
         // the kernel indexes rows through it: only a permutation is taken
         uint64_t seen = 0;

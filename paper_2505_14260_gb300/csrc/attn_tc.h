@@ -17,9 +17,11 @@ void attn_tc_plan_destroy(AttnTcPlan *p);
 // the cache buffers hold. order (nullable, a permutation of the a.R /
 // rows_per_req blocks, used when there are at most 64): the blocks' launch
 // order, longest first, so that the last wave holds the shortest CTAs (it
-// changes no result). Returns false if the shape is not supported (the caller
-// reports it).
+// changes no result). stamp (nullable): a profiling slot of three
+// %globaltimer values (earliest entry, earliest return from the wait on the
+// previous kernel, latest exit), min/min/max-updated by the CTAs. Returns false
+// if the shape is not supported (the caller reports it).
 bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows_per_req, const int *order,
-                         int *status, cudaStream_t s);
+                         int *status, cudaStream_t s, unsigned long long *stamp = nullptr);
 
 }  // namespace msd

@@ -920,24 +920,41 @@ __device__ __forceinline__ uint32_t c_mapa(uint32_t local, uint32_t rank) {
 struct PartSrc {
     const float *own, *recv;
     int rank, S, c_lo, c_hi, span;
-    __device__ __forceinline__ const float4 *at(int q, int col, int row) const {
+    // shared-window address of a float4 (read with ld.shared)
+    __device__ __forceinline__ uint32_t at(int q, int col, int row) const {
         const float *b = q == rank ? own + col * BM : recv + ((q < rank ? q : q - 1) * span + (col - c_lo)) * BM;
-        return reinterpret_cast<const float4 *>(b + row);
+        return (uint32_t)__cvta_generic_to_shared(b + row);
     }
 };
+
+__device__ __forceinline__ float4 lds4(uint32_t a) {
+    float4 v;
+    asm volatile("ld.shared.v4.f32 {%0, %1, %2, %3}, [%4];" : "=f"(v.x), "=f"(v.y), "=f"(v.z), "=f"(v.w) : "r"(a));
+    return v;
+}
+__device__ __forceinline__ float lds1(const float *p) {
+    float v;
+    asm volatile("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"((uint32_t)__cvta_generic_to_shared(p)));
+    return v;
+}
 
 // Sums, in rank order, of the S partials' float4 at K (column, row) places
 // (all in this CTA's shared memory); every load is issued before the first sum.
 template <int K>
 __device__ __forceinline__ void c_part_sums(const PartSrc &ps, const int (&col)[K], const int (&row)[K],
                                             const bool (&use)[K], float4 (&out)[K]) {
+    if (ps.S == 1) {                 // one partial: plain loads (no unrolled rank loop)
+#pragma unroll
+        for (int k = 0; k < K; ++k) out[k] = use[k] ? lds4(ps.at(0, col[k], row[k])) : make_float4(0.f, 0.f, 0.f, 0.f);
+        return;
+    }
     float4 v[K][8];
 #pragma unroll
     for (int q = 0; q < 8; ++q) {
         if (q >= ps.S) break;
 #pragma unroll
         for (int k = 0; k < K; ++k)
-            if (use[k]) v[k][q] = *ps.at(q, col[k], row[k]);
+            if (use[k]) v[k][q] = lds4(ps.at(q, col[k], row[k]));
     }
 #pragma unroll
     for (int k = 0; k < K; ++k) {
@@ -962,9 +979,25 @@ __device__ __forceinline__ void c_part_sums(const PartSrc &ps, const int (&col)[
 // act[m][64 t + i] = bf16(silu(g) * u), scaled first by the folded-norm 1/rms.
 __device__ __forceinline__ void c_epi_swiglu(const CkParams &p, const PartSrc &ps, bool ok, int wt, int n0,
                                              const float *rinv) {
+    // the parameters the loop uses, read once before its stores
     bf16 *const act = p.fx.act;
     const int F = p.fx.F, M = p.M;
+    const long lo = p.fx.lo;
     const int n = (ps.c_hi - ps.c_lo) * 16;         // groups of this CTA's columns
+    auto emit = [&](float4 a, float4 b, int c, int j) {
+        const int m = n0 + c;
+        if (!ok || m >= M || j >= F) return;          // F % 4 == 0: whole groups
+        if (rinv) {
+            const float sc = lds1(rinv + c);
+            a.x *= sc; a.y *= sc; a.z *= sc; a.w *= sc;
+            b.x *= sc; b.y *= sc; b.z *= sc; b.w *= sc;
+        }
+        const float o0 = __fdividef(a.x, 1.f + __expf(-a.x)) * b.x;
+        const float o1 = __fdividef(a.y, 1.f + __expf(-a.y)) * b.y;
+        const float o2 = __fdividef(a.z, 1.f + __expf(-a.z)) * b.z;
+        const float o3 = __fdividef(a.w, 1.f + __expf(-a.w)) * b.w;
+        Split<bf16>::store4(act + (size_t)m * F + j, lo, make_float4(o0, o1, o2, o3));
+    };
     for (int e0 = threadIdx.x; e0 < n; e0 += 2 * C_THREADS) {
         int col[4], row[4];
         bool use[4];
@@ -979,21 +1012,8 @@ __device__ __forceinline__ void c_epi_swiglu(const CkParams &p, const PartSrc &p
         float4 v[4];
         c_part_sums<4>(ps, col, row, use, v);
 #pragma unroll
-        for (int u = 0; u < 2; ++u) {
-            float4 a = v[2 * u], b = v[2 * u + 1];
-            const int c = col[2 * u], m = n0 + c, j = wt * 64 + row[2 * u];
-            if (!use[2 * u] || !ok || m >= M || j >= F) continue;     // F % 4 == 0: whole groups
-            if (rinv) {
-                const float sc = rinv[c];
-                a.x *= sc; a.y *= sc; a.z *= sc; a.w *= sc;
-                b.x *= sc; b.y *= sc; b.z *= sc; b.w *= sc;
-            }
-            const float o0 = __fdividef(a.x, 1.f + __expf(-a.x)) * b.x;
-            const float o1 = __fdividef(a.y, 1.f + __expf(-a.y)) * b.y;
-            const float o2 = __fdividef(a.z, 1.f + __expf(-a.z)) * b.z;
-            const float o3 = __fdividef(a.w, 1.f + __expf(-a.w)) * b.w;
-            Split<bf16>::store4(act + (size_t)m * F + j, p.fx.lo, make_float4(o0, o1, o2, o3));
-        }
+        for (int u = 0; u < 2; ++u)
+            if (use[2 * u]) emit(v[2 * u], v[2 * u + 1], col[2 * u], wt * 64 + row[2 * u]);
     }
 }
 
@@ -1057,6 +1077,8 @@ __device__ __forceinline__ void c_epi_rope(const CkParams &p, const PartSrc &ps,
     const RopeGeom g(p.fx.hd, ps);
     const int slots = p.fx.slots, nh = p.fx.nh, M = p.M, hd = g.hd, half = g.half;
     bf16 *const qo = p.fx.q_out, *const kvd = seg == 1 ? p.fx.kdst : p.fx.vdst;
+    const long lo = p.fx.lo;
+    int *const status = p.status;
     for (int k = 0;; ++k) {
         const int e = threadIdx.x + k * C_THREADS;
         if (e >= g.n) break;
@@ -1080,7 +1102,7 @@ __device__ __forceinline__ void c_epi_rope(const CkParams &p, const PartSrc &ps,
         c_part_sums<2>(ps, col, row, use, v);
         float4 a = v[0], b = v[1];
         if (rinv) {
-            const float sc = rinv[c];
+            const float sc = lds1(rinv + c);
             a.x *= sc; a.y *= sc; a.z *= sc; a.w *= sc;
             b.x *= sc; b.y *= sc; b.z *= sc; b.w *= sc;
         }
@@ -1096,12 +1118,12 @@ __device__ __forceinline__ void c_epi_rope(const CkParams &p, const PartSrc &ps,
         if (seg == 0) {
             dst = qo + (size_t)m * (nh * hd) + o;
         } else {
-            if (d.dst >= slots) set_status(p.status, ST_RANGE);
+            if (d.dst >= slots) set_status(status, ST_RANGE);
             if (d.dst < 0 || d.dst >= slots) continue;
             dst = kvd + ((size_t)(d.req * nh + h) * slots + d.dst) * hd + i;
         }
-        Split<bf16>::store4(dst, p.fx.lo, a);
-        Split<bf16>::store4(dst + half, p.fx.lo, b);
+        Split<bf16>::store4(dst, lo, a);
+        Split<bf16>::store4(dst + half, lo, b);
     }
 }
 
@@ -1142,6 +1164,10 @@ __device__ __forceinline__ void c_reduce_norm(const CkParams &p, const PartSrc &
     float *const Y = p.Y;
     bf16 *const XG = p.nout.xg;
     const int ldy = p.ldy, M = p.M;
+    const long xlo = p.nout.lo;
+    float *const ssd = p.nout.ss;
+    const int ssld = p.nout.ld;
+    const bf16 *const gn = p.nout.g;
     for (int k = 0;; ++k) {
         const int c = ps.c_lo + warp + k * NW;
         if (c >= ps.c_hi) break;                         // warp-uniform
@@ -1169,23 +1195,22 @@ __device__ __forceinline__ void c_reduce_norm(const CkParams &p, const PartSrc &
                     a[0] += yi.x; a[1] += yi.y; a[2] += yi.z; a[3] += yi.w;
                 }
                 *reinterpret_cast<float4 *>(y) = make_float4(a[0], a[1], a[2], a[3]);
-                Split<bf16>::store4(xg, p.nout.lo,
-                                    make_float4(a[0] * g4[0], a[1] * g4[1], a[2] * g4[2], a[3] * g4[3]));
+                Split<bf16>::store4(xg, xlo, make_float4(a[0] * g4[0], a[1] * g4[1], a[2] * g4[2], a[3] * g4[3]));
                 ss = a[0] * a[0] + a[1] * a[1] + a[2] * a[2] + a[3] * a[3];
             } else {
-                const bf16 *g = p.nout.g + o_base + r4;
+                const bf16 *g = gn + o_base + r4;
 #pragma unroll
                 for (int e = 0; e < 4; ++e)
                     if (r4 + e < rows_here) {
                         const float ye = add ? y[e] + a[e] : a[e];
                         y[e] = ye;
-                        Split<bf16>::store(xg + e, p.nout.lo, ye * __bfloat162float(g[e]));
+                        Split<bf16>::store(xg + e, xlo, ye * __bfloat162float(g[e]));
                         ss += ye * ye;
                     }
             }
         }
         ss = warp_sum(ss);
-        if (live && lane == 0) p.nout.ss[(size_t)m * p.nout.ld + tile] = ss;
+        if (live && lane == 0) ssd[(size_t)m * ssld + tile] = ss;
     }
 }
 
@@ -1441,11 +1466,15 @@ __global__ void __launch_bounds__(C_THREADS)
         ps.c_hi = ((int)rank + 1) * BN / S;
         ps.span = span;
         bool okr = ok;
-        __syncthreads();                 // the staged row descriptors, for every warp
+        __syncthreads();                 // the staged row descriptors and the partial, for every warp
         RopePre rpre;
         float4 yv[EPI_PRE];
-        if (paired && p.epi == EPI_ROPE_KV) c_rope_pre(p, ps, ok, seg, row0, n0, rows_here, s_rows, rpre);
-        if (norm_out) c_norm_pre(p, ps, ok, o_base, rows_here, n0, yv);
+        // the global operands of the first groups are requested after the
+        // cluster barrier, so that they arrive while the slices are exchanged
+        auto pre_loads = [&]() {
+            if (paired && p.epi == EPI_ROPE_KV) c_rope_pre(p, ps, ok, seg, row0, n0, rows_here, s_rows, rpre);
+            if (norm_out) c_norm_pre(p, ps, ok, o_base, rows_here, n0, yv);
+        };
         if (S > 1) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");    // part, for the bulk copies
             c_cluster_sync();
@@ -1465,9 +1494,10 @@ __global__ void __launch_bounds__(C_THREADS)
                 }
                 asm volatile("cp.async.bulk.commit_group;" ::: "memory");
             }
+            pre_loads();
             okr = mbar_wait(recv_bar, 0, &abort_flag, p.status) && ok;
         } else {
-            __syncthreads();
+            pre_loads();
         }
         if (p.epi == EPI_SWIGLU)
             c_epi_swiglu(p, ps, okr, wt, n0, p.nin.ss ? s_rinv : nullptr);
@@ -1603,7 +1633,9 @@ struct MapKeyHash {
 
 }  // namespace
 
-constexpr int MAX_STAMPS = 2048;   // launches per stamping window
+constexpr int MAX_STAMPS = 2048;   // GEMM launches per stamping window
+constexpr int MAX_XSTAMPS = 512;   // other stamped launches (attention) per window, slots after the GEMMs'
+constexpr int ALL_STAMPS = MAX_STAMPS + MAX_XSTAMPS;
 
 // Sums of the closed stamping windows (device memory).
 struct StampAcc {
@@ -1615,29 +1647,57 @@ struct StampAcc {
     double pre_bytes;             // weight bytes requested before the wait on the previous kernel
 };
 
-__global__ void stamp_init_kernel(unsigned long long *st, int n, StampAcc *acc) {
+__global__ void stamp_init_kernel(unsigned long long *st, int n, StampAcc *acc, unsigned long long *slot_acc) {
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < n; i += gridDim.x * blockDim.x) {
         st[3 * i] = ~0ull;
         st[3 * i + 1] = ~0ull;
         st[3 * i + 2] = 0ull;
+        slot_acc[3 * i] = slot_acc[3 * i + 1] = slot_acc[3 * i + 2] = 0ull;
     }
     if (blockIdx.x == 0 && threadIdx.x == 0) *acc = StampAcc{0, 0, 0, 0, 0.0, 0.0, 0.0, 0.0, 0.0};
 }
 
-// Closes a window of n launches: adds their spans to acc and clears their
-// slots for the next window (one block; runs after the window's launches).
-__global__ void stamp_collect_kernel(unsigned long long *st, int n, double bytes, double wbytes, double flops,
-                                     double mma_flops, double pre_bytes, StampAcc *acc) {
+// A stamp's spans: exit - max(wait, entry) and exit - entry (0, 0 if unused).
+__device__ __forceinline__ bool stamp_spans(const unsigned long long *st, unsigned long long &crit,
+                                            unsigned long long &span) {
+    const unsigned long long e0 = st[0], w0 = st[1], e1 = st[2];
+    if (e0 == ~0ull || e1 < e0) return false;
+    span = e1 - e0;
+    crit = e1 - (w0 <= e1 ? (w0 > e0 ? w0 : e0) : e0);
+    return true;
+}
+
+// Closes a window of n GEMM launches and xn other launches: adds the GEMMs'
+// spans to acc, every launch's spans to its slot's sums in slot_acc, and
+// clears the slots for the next window (one block; runs after the window's
+// launches).
+__global__ void stamp_collect_kernel(unsigned long long *st, int n, int xn, double bytes, double wbytes, double flops,
+                                     double mma_flops, double pre_bytes, StampAcc *acc, unsigned long long *slot_acc) {
     __shared__ unsigned long long s_span, s_crit, s_cnt;
     if (threadIdx.x == 0) s_span = s_crit = s_cnt = 0;
     __syncthreads();
     unsigned long long span = 0, crit = 0, cnt = 0;
     for (int i = threadIdx.x; i < n; i += blockDim.x) {
-        const unsigned long long e0 = st[3 * i], w0 = st[3 * i + 1], e1 = st[3 * i + 2];
-        if (e0 != ~0ull && e1 >= e0) {
-            span += e1 - e0;
-            crit += e1 - (w0 <= e1 ? (w0 > e0 ? w0 : e0) : e0);
+        unsigned long long c1, s1;
+        if (stamp_spans(st + 3 * i, c1, s1)) {
+            span += s1;
+            crit += c1;
             ++cnt;
+            slot_acc[3 * i] += c1;
+            slot_acc[3 * i + 1] += s1;
+            slot_acc[3 * i + 2] += 1;
+        }
+        st[3 * i] = ~0ull;
+        st[3 * i + 1] = ~0ull;
+        st[3 * i + 2] = 0ull;
+    }
+    for (int j = threadIdx.x; j < xn; j += blockDim.x) {
+        const int i = MAX_STAMPS + j;
+        unsigned long long c1, s1;
+        if (stamp_spans(st + 3 * i, c1, s1)) {
+            slot_acc[3 * i] += c1;
+            slot_acc[3 * i + 1] += s1;
+            slot_acc[3 * i + 2] += 1;
         }
         st[3 * i] = ~0ull;
         st[3 * i + 1] = ~0ull;
@@ -1674,10 +1734,15 @@ struct GemmPlan {
     double prof_bytes = 0.0, prof_wbytes = 0.0, prof_flops = 0.0, prof_mma = 0.0, prof_pre = 0.0;
     // launch stamps: one slot of 3 per launch of a stamping window
     bool stamp_mode = false, stamp_active = false;
-    int stamp_next = 0;
+    int stamp_next = 0, xstamp_next = 0, cur_slot = -1;
     double stamp_bytes = 0.0, stamp_wbytes = 0.0, stamp_flops = 0.0, stamp_mma = 0.0, stamp_pre = 0.0;
     unsigned long long *stamps = nullptr;
     StampAcc *stamp_acc = nullptr;
+    // per slot: sums of exit - wait, exit - entry and the stamped launches
+    // ([ALL_STAMPS][3]); what each slot of the last closed window held
+    unsigned long long *slot_acc = nullptr;
+    std::vector<GemmSlot> slot_info = std::vector<GemmSlot>(ALL_STAMPS);
+    int slot_n = 0, xslot_n = 0;
 };
 
 bool gemm_plan_create(GemmPlan **out, int, int, int, int) {
@@ -1696,7 +1761,8 @@ bool gemm_plan_create(GemmPlan **out, int, int, int, int) {
     p->encode = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(fn);
     if (cudaMalloc(&p->ws, WS_BYTES) != cudaSuccess ||
         cudaMalloc(&p->counters, sizeof(int) * N_COUNTERS) != cudaSuccess ||
-        cudaMalloc(&p->stamps, sizeof(unsigned long long) * 3 * MAX_STAMPS) != cudaSuccess ||
+        cudaMalloc(&p->stamps, sizeof(unsigned long long) * 3 * ALL_STAMPS) != cudaSuccess ||
+        cudaMalloc(&p->slot_acc, sizeof(unsigned long long) * 3 * ALL_STAMPS) != cudaSuccess ||
         cudaMalloc(&p->stamp_acc, sizeof(StampAcc)) != cudaSuccess) {
         gemm_plan_destroy(p);
         return false;
@@ -1712,6 +1778,7 @@ void gemm_plan_destroy(GemmPlan *p) {
     if (p->counters) cudaFree(p->counters);
     if (p->stamps) cudaFree(p->stamps);
     if (p->stamp_acc) cudaFree(p->stamp_acc);
+    if (p->slot_acc) cudaFree(p->slot_acc);
     for (cudaEvent_t e : p->ev) cudaEventDestroy(e);
     delete p;
 }
@@ -1723,7 +1790,7 @@ bool gemm_profile_enable(GemmPlan *p, int mode) {
     p->ev_used = 0;
     p->prof_bytes = p->prof_wbytes = p->prof_flops = p->prof_mma = p->prof_pre = 0.0;
     if (p->stamp_mode) {
-        stamp_init_kernel<<<8, 256>>>(p->stamps, MAX_STAMPS, p->stamp_acc);
+        stamp_init_kernel<<<8, 256>>>(p->stamps, ALL_STAMPS, p->stamp_acc, p->slot_acc);
         if (cudaDeviceSynchronize() != cudaSuccess) return false;
     }
     return true;
@@ -1736,21 +1803,55 @@ void gemm_stamp_begin(GemmPlan *p) {
     if (!p->stamp_mode) return;
     p->stamp_active = true;
     p->stamp_next = 0;
+    p->xstamp_next = 0;
+    p->cur_slot = -1;
     p->stamp_bytes = p->stamp_wbytes = p->stamp_flops = p->stamp_mma = p->stamp_pre = 0.0;
 }
 
 void gemm_stamp_end(GemmPlan *p, cudaStream_t s) {
     if (!p->stamp_active) return;
     p->stamp_active = false;
-    stamp_collect_kernel<<<1, 256, 0, s>>>(p->stamps, p->stamp_next, p->stamp_bytes, p->stamp_wbytes,
-                                           p->stamp_flops, p->stamp_mma, p->stamp_pre, p->stamp_acc);
+    p->slot_n = p->stamp_next;
+    p->xslot_n = p->xstamp_next;
+    stamp_collect_kernel<<<1, 256, 0, s>>>(p->stamps, p->stamp_next, p->xstamp_next, p->stamp_bytes, p->stamp_wbytes,
+                                           p->stamp_flops, p->stamp_mma, p->stamp_pre, p->stamp_acc, p->slot_acc);
     note_launch();
 }
 
 // The stamp slot of the next launch (null outside a window or when full).
 static unsigned long long *stamp_slot(GemmPlan *p) {
     if (!p->stamp_active || p->stamp_next >= MAX_STAMPS) return nullptr;
+    p->cur_slot = p->stamp_next;
     return p->stamps + 3 * (p->stamp_next++);
+}
+
+unsigned long long *gemm_stamp_external(GemmPlan *p, int kind, int rows, int outputs, int inner) {
+    if (!p || !p->stamp_active || p->xstamp_next >= MAX_XSTAMPS) return nullptr;
+    const int i = MAX_STAMPS + p->xstamp_next++;
+    p->slot_info[i] = GemmSlot{kind, rows, outputs, inner, 0, 0.0, 0.0, 0.0};
+    return p->stamps + 3 * i;
+}
+
+int gemm_profile_slots(GemmPlan *p, GemmSlot *out, int max) {
+    if (!p->stamp_mode) return 0;
+    std::vector<unsigned long long> acc(3 * (size_t)ALL_STAMPS);
+    cudaDeviceSynchronize();
+    if (cudaMemcpy(acc.data(), p->slot_acc, acc.size() * sizeof(unsigned long long), cudaMemcpyDeviceToHost) !=
+        cudaSuccess)
+        return -1;
+    cudaMemset(p->slot_acc, 0, acc.size() * sizeof(unsigned long long));
+    int n = 0;
+    auto put = [&](int i) {
+        if (n >= max) return;
+        GemmSlot g = p->slot_info[i];
+        g.launches = (long)acc[3 * i + 2];
+        g.critical_ms = acc[3 * i] * 1e-6;
+        g.ms = acc[3 * i + 1] * 1e-6;
+        out[n++] = g;
+    };
+    for (int i = 0; i < p->slot_n; ++i) put(i);
+    for (int j = 0; j < p->xslot_n; ++j) put(MAX_STAMPS + j);
+    return n;
 }
 
 // Algorithmic bytes and flops of a launch of M token rows x O outputs x K for
@@ -1760,6 +1861,10 @@ static unsigned long long *stamp_slot(GemmPlan *p) {
 static void account(GemmPlan *p, double weight_bytes, double total_bytes, int M, int O, int K, int nb,
                     double pre) {
     const double fl = 2.0 * M * O * K;
+    if (p->cur_slot >= 0) {          // the launch that just took a stamp slot
+        p->slot_info[p->cur_slot] = GemmSlot{0, M, O, K, 0, total_bytes, 0.0, 0.0};
+        p->cur_slot = -1;
+    }
     if (p->profile) {
         p->prof_wbytes += weight_bytes;
         p->prof_bytes += total_bytes;

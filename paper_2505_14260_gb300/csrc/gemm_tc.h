@@ -105,6 +105,15 @@ struct GemmProfile {
     double mma_flops;   // as issued: x2 where the token operand is a split pair
     double prefetch_bytes;   // weight bytes requested before the wait on the previous kernel
 };
+// One stamp slot of the last closed window (mode 2), summed over the windows
+// since the last read: kind 0 a GEMM launch (rows M, outputs O, inner K,
+// algorithmic bytes per launch), kind 1 an attention launch (query rows,
+// heads, head dim; bytes 0).
+struct GemmSlot {
+    int kind, rows, outputs, inner;
+    long launches;
+    double bytes, critical_ms, ms;
+};
 // Device address of msd_linear_noalloc's status word on the current device
 // (first use sets the device up); null if that failed.
 int *noalloc_status_word();
@@ -122,5 +131,12 @@ bool gemm_stamp_on(const GemmPlan *p);       // mode 2
 void gemm_stamp_begin(GemmPlan *p);
 void gemm_stamp_end(GemmPlan *p, cudaStream_t s);
 GemmProfile gemm_profile_read(GemmPlan *p);
+// A stamp slot for another kernel of the open window (null when none is open
+// or the slots are used up); its spans are summed per slot, apart from the GEMMs'.
+unsigned long long *gemm_stamp_external(GemmPlan *p, int kind, int rows, int outputs, int inner);
+// Per-slot sums since the last call (which it clears): GEMM slots in launch
+// order, then the other kernels'. Returns the count written, -1 on a copy
+// error, 0 outside mode 2.
+int gemm_profile_slots(GemmPlan *p, GemmSlot *out, int max);
 
 }  // namespace msd

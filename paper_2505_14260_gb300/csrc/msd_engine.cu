@@ -215,7 +215,8 @@ void attention<bf16>(msd_ctx *c, const AttnArgs<bf16> &a, int rows_per_req, cuda
         std::stable_sort(order, order + c->B, [&](int x, int y) { return c->L_bound[x] > c->L_bound[y]; });
         ord = order;
     }
-    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, ord, c->status, s)) {
+    unsigned long long *st = gemm_stamp_external(c->gplan, 1, a.R, a.nh, a.hd);
+    if (!launch_attention_tc(c->aplan, a, c->B, rows_per_req, ord, c->status, s, st)) {
         c->err = "tensor-core attention: unsupported shape or launch failure";
         launch_flag(c->status, ST_RANGE, s);     // reported by the next call
     }
@@ -1244,6 +1245,27 @@ msd_status msd_profile_read(msd_ctx *c, msd_profile *out) {
         out->gemm_mma_flops = g.mma_flops;
         out->gemm_prefetch_bytes = g.prefetch_bytes;
     }
+    return MSD_OK;
+}
+
+msd_status msd_profile_slots(msd_ctx *c, msd_kernel_slot *out, int32_t max, int32_t *n) {
+    if (!c || !n || max < 0 || (max > 0 && !out)) return MSD_ERR_INVALID;
+    *n = 0;
+    if (!c->gplan || max == 0) return MSD_OK;
+    std::vector<GemmSlot> g((size_t)max);
+    const int k = gemm_profile_slots(c->gplan, g.data(), max);
+    if (k < 0) return fail(c, MSD_ERR_CUDA, "reading the stamp slots failed");
+    for (int i = 0; i < k; ++i) {
+        out[i].kind = g[i].kind;
+        out[i].rows = g[i].rows;
+        out[i].outputs = g[i].outputs;
+        out[i].inner = g[i].inner;
+        out[i].launches = g[i].launches;
+        out[i].bytes = g[i].bytes;
+        out[i].critical_ms = g[i].critical_ms;
+        out[i].span_ms = g[i].ms;
+    }
+    *n = k;
     return MSD_OK;
 }
 

@@ -65,6 +65,12 @@ class msd_profile(ctypes.Structure):
                 ("gemm_prefetch_bytes", ctypes.c_double)]
 
 
+class msd_kernel_slot(ctypes.Structure):
+    _fields_ = [("kind", c_int32), ("rows", c_int32), ("outputs", c_int32), ("inner", c_int32),
+                ("launches", c_int64), ("bytes", ctypes.c_double), ("critical_ms", ctypes.c_double),
+                ("span_ms", ctypes.c_double)]
+
+
 _SIGNATURES = {
     "msd_create": (c_int32, [POINTER(msd_config), POINTER(msd_weights), POINTER(c_void_p)]),
     "msd_destroy": (c_int32, [c_void_p]),
@@ -89,6 +95,7 @@ _SIGNATURES = {
     "msd_test_wait_timeout": (c_int32, [c_void_p, c_int64, c_void_p]),
     "msd_profile_enable": (c_int32, [c_void_p, c_int32]),
     "msd_profile_read": (c_int32, [c_void_p, POINTER(msd_profile)]),
+    "msd_profile_slots": (c_int32, [c_void_p, POINTER(msd_kernel_slot), c_int32, POINTER(c_int32)]),
     "msd_state": (c_int32, [c_void_p, POINTER(msd_state_view)]),
     "msd_last_error": (c_char_p, [c_void_p]),
 }
@@ -330,6 +337,14 @@ class Engine:
         p = msd_profile()
         self._check(lib().msd_profile_read(self.ctx, ctypes.byref(p)), "msd_profile_read")
         return {n: getattr(p, n) for n, _ in msd_profile._fields_}
+
+    def profile_slots(self, max_slots: int = 4096) -> list:
+        """Per-launch sums of the stamped step graphs since the last call
+        (mode 2): GEMM slots in launch order, then the attention launches."""
+        buf = (msd_kernel_slot * max_slots)()
+        n = c_int32(0)
+        self._check(lib().msd_profile_slots(self.ctx, buf, max_slots, ctypes.byref(n)), "msd_profile_slots")
+        return [{f: getattr(buf[i], f) for f, _ in msd_kernel_slot._fields_} for i in range(n.value)]
 
     # -- state ---------------------------------------------------------------
     def state(self) -> dict:

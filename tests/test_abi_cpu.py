@@ -105,7 +105,8 @@ def _header_struct_fields(name):
     return fields
 
 
-@pytest.mark.parametrize("cname,pyname", [("msd_profile", "msd_profile"), ("msd_state_view", "msd_state_view")])
+@pytest.mark.parametrize("cname,pyname", [("msd_profile", "msd_profile"), ("msd_state_view", "msd_state_view"),
+                                          ("msd_kernel_slot", "msd_kernel_slot")])
 def test_binding_structs_match_the_header(cname, pyname):
     """The ctypes mirrors of the header's output structs list the same fields
     in the same order (the library writes them by position)."""
@@ -116,3 +117,10 @@ def test_binding_structs_match_the_header(cname, pyname):
 def test_profile_enable_rejects_a_null_context(libmsd):
     from paper_2505_14260_gb300 import msd
     assert libmsd.msd_profile_enable(None, 2) == msd.MSD_ERR_INVALID
+
+
+def test_profile_slots_rejects_bad_arguments(libmsd):
+    import ctypes
+    from paper_2505_14260_gb300 import msd
+    n = ctypes.c_int32(7)
+    assert libmsd.msd_profile_slots(None, None, 0, ctypes.byref(n)) == msd.MSD_ERR_INVALID

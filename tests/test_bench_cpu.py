@@ -109,3 +109,29 @@ def test_weights_with_layers_kept_equal_the_full_set():
             assert all(torch.equal(v[n], part[k][n]) for n in v)
         else:
             assert torch.equal(v, part[k]), k
+
+
+def test_kernel_breakdown_groups_slots_by_projection():
+    """Stamp slots of two steps: the verify q/k/v slots of both layers form one
+    group, rates come from the summed wait-to-exit spans, and verify attention
+    is charged its requests' prefix and tree keys."""
+    wl = synth.WORKLOADS["llava7b"].with_(n_layers=2)
+    H, N = wl.hidden, wl.tree_nodes
+    R = wl.batch * N
+
+    def slot(kind, rows, outputs, inner, byts, ms):
+        return {"kind": kind, "rows": rows, "outputs": outputs, "inner": inner, "launches": 2,
+                "bytes": byts, "critical_ms": 2 * ms, "span_ms": 3 * ms}
+
+    qkv = 3 * H * H * 2.0
+    slots = [slot(0, R, 3 * H, H, qkv, 0.02), slot(1, R, wl.n_heads, wl.head_dim, 0.0, 0.01),
+             slot(0, R, 3 * H, H, qkv, 0.02), slot(0, 10, 3 * H, H, qkv, 0.015)]
+    rows = {g["name"]: g for g in bench.kernel_breakdown(slots, wl, [1000.0], 6767.1, 2)}
+    v = rows["verify q/k/v + RoPE"]
+    assert v["launches_per_step"] == 2 and v["ms_per_step"] == pytest.approx(0.04)
+    assert v["us_per_launch"] == pytest.approx(20.0)
+    assert v["achieved_gbs"] == pytest.approx(2 * qkv / 0.04e-3 / 1e9)
+    assert v["achieved_tflops"] == pytest.approx(2 * 2.0 * R * 3 * H * H / 0.04e-3 / 1e12)
+    a = rows["verify tree attention"]
+    assert a["bytes_per_step"] == pytest.approx(2 * (1000 + N) * H * 2)
+    assert rows["draft q/k/v + RoPE"]["launches_per_step"] == 1

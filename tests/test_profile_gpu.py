@@ -1,7 +1,8 @@
-"""The GEMM launch stamps of profile mode 2: replayed step graphs that time
-their own tensor-core GEMMs with %globaltimer leave every output of the step
-unchanged, measure each step once, and report spans that fit inside the steps'
-elapsed time (the wait-to-exit spans of one stream's kernels are disjoint)."""
+"""The launch stamps of profile mode 2: replayed step graphs that time their
+own tensor-core GEMMs and tree-attention launches with %globaltimer leave every
+output of the step unchanged, measure each step once, and report spans that fit
+inside the steps' elapsed time (the wait-to-exit spans of one stream's kernels
+are disjoint); the per-slot breakdown adds up to the totals."""
 import pytest
 import torch
 
@@ -32,6 +33,7 @@ def run_steps(wl, w, mode):
     torch.cuda.synchronize()
     prof = eng.profile_read() if mode else None
     if mode:
+        prof["slots"] = eng.profile_slots()
         with pytest.raises(msd.MsdError) as e:
             eng.profile_enable(3)
         assert e.value.status == msd.MSD_ERR_INVALID
@@ -59,3 +61,12 @@ def test_stamped_step_graph_times_its_gemms(nodes, depth, k):
     assert prof["gemm_bytes"] > prof["gemm_weight_bytes"] > 0
     assert prof["gemm_flops"] <= prof["gemm_mma_flops"] <= 2 * prof["gemm_flops"]
     assert 0 < prof["gemm_prefetch_bytes"] <= prof["gemm_weight_bytes"]   # (capped per launch)
+    gemm = [s for s in prof["slots"] if s["kind"] == 0]
+    attn = [s for s in prof["slots"] if s["kind"] == 1]
+    assert len(gemm) == n // STEPS and len(attn) > 0
+    assert all(s["launches"] == STEPS for s in prof["slots"])
+    assert all(0.0 < s["critical_ms"] <= s["span_ms"] for s in prof["slots"])
+    assert sum(s["critical_ms"] for s in gemm) == pytest.approx(prof["gemm_critical_ms"], rel=1e-9)
+    assert sum(s["bytes"] * s["launches"] for s in gemm) == pytest.approx(prof["gemm_bytes"], rel=1e-9)
+    assert sum(s["critical_ms"] for s in prof["slots"]) <= ms
+    assert all(s["outputs"] == wl.n_heads and s["inner"] == wl.head_dim for s in attn)
