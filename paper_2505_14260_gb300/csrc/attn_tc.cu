@@ -809,15 +809,18 @@ bool launch_attention_tc(AttnTcPlan *p, const AttnArgs<bf16> &a, int B, int rows
     lc.blockDim = dim3(THREADS);
     lc.dynamicSmemBytes = smem;
     lc.stream = s;
-    cudaLaunchAttribute at[2];
+    // Plain stream order behind the previous kernel (no programmatic
+    // serialisation: its CTAs could not start before that kernel's CTAs left
+    // the SMs anyway, and its griddepcontrol.wait then returned 3-4 us after
+    // their exit where a plain launch starts 1.3 us after it); the kernel still
+    // releases its own dependents early.
+    cudaLaunchAttribute at[1];
     at[0].id = cudaLaunchAttributeClusterDimension;
     at[0].val.clusterDim.x = 1;
     at[0].val.clusterDim.y = 1;
     at[0].val.clusterDim.z = nsplit;
-    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    at[1].val.programmaticStreamSerializationAllowed = 1;
     lc.attrs = at;
-    lc.numAttrs = 2;
+    lc.numAttrs = 1;
     cudaError_t e = a.hd == 128 ? cudaLaunchKernelEx(&lc, attn_tc_kernel<128>, *mkc, *mvc, *mkt, *mvt, tp)
                                 : cudaLaunchKernelEx(&lc, attn_tc_kernel<64>, *mkc, *mvc, *mkt, *mvt, tp);
     note_launch();
