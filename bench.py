@@ -88,12 +88,14 @@ def parse():
 # DRAM traffic of the GEMMs: ncu dram__bytes_read.sum + dram__bytes_write.sum
 # per launch divided by the same launches' algorithmic bytes. Decode
 # (gemm_cluster_kernel): the 90 launches of two 2-layer 7B-width steps, 0.9947
-# (no re-reads). Many rows (gemm_persist_kernel): two batch-16 draft launches
-# (f_down, q/k/v; 160 token rows), 0.998. Per launch of a full workload it is
-# the ratio times its algorithmic bytes per launch. Valid for the GEMM source
-# with this SHA-1 only.
+# (no re-reads). Many rows (gemm_persist_kernel): the first two many-row
+# launches of a 2-layer batch-16 step (the draft's input projection and q/k/v at
+# 160 token rows), 0.975 (0.997 and 0.960: part of q/k/v's fp32 output is still
+# in L2 when the launch ends). Per launch of a full workload it is the ratio
+# times its algorithmic bytes per launch. Valid for the GEMM source with this
+# SHA-1 only.
 GEMM_TRAFFIC = {"source_sha1": "4d36367b4ffed3305403572d726f67c9ae4e59be",
-                "ratio": {"hbm": 0.9947, "tensor": 0.998}}
+                "ratio": {"hbm": 0.9947, "tensor": 0.975}}
 
 
 def gemm_traffic(bytes_per_launch, bound="hbm"):
