@@ -2187,8 +2187,18 @@ static void gemm_persist(GemmPlan *p, const bf16 *X, const bf16 *X_lo, int ldx, 
     if (G > p->num_sms) G = p->num_sms;
     if (G < 1) G = 1;
     // whole tiles in rounds of G, the remainder split stream-K across all CTAs
-    const int dp_rounds = (int)(tiles_total / G);
-    const int T_sk = (int)(tiles_total - (long long)dp_rounds * G);
+    // (its fix-ups overlap the whole tiles that follow). A remainder of a few
+    // short-K tiles would cut each into more than eight pieces, summed by one
+    // CTA: there one round of whole tiles joins it (every tile in two or three
+    // pieces, fixed up at the end). Measured on the 960-row verify GEMMs: O
+    // (K = 4096) 89 -> 75 us; down (K = 11008) 106 -> 140 us and the SwiGLU
+    // launches slower, so those keep the rounds.
+    int dp_rounds = (int)(tiles_total / G);
+    int T_sk = (int)(tiles_total - (long long)dp_rounds * G);
+    if (T_sk > 0 && dp_rounds > 0 && G > 8LL * T_sk && kblocks <= 64 && !glu) {
+        --dp_rounds;
+        T_sk += (int)G;
+    }
     const long long units = (long long)T_sk * kblocks;
     const size_t ws_need = 2ull * G * BN * BM * sizeof(float);
     if (ws_need > WS_BYTES || tiles_total > N_COUNTERS) {
