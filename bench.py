@@ -94,7 +94,7 @@ def parse():
 # in L2 when the launch ends). Per launch of a full workload it is the ratio
 # times its algorithmic bytes per launch. Valid for the GEMM source with this
 # SHA-1 only.
-GEMM_TRAFFIC = {"source_sha1": "4d36367b4ffed3305403572d726f67c9ae4e59be",
+GEMM_TRAFFIC = {"source_sha1": "b06a5a07809661b97a8943189afe56ae80fc02fb",
                 "ratio": {"hbm": 0.9947, "tensor": 0.975}}
 
 
