@@ -1406,6 +1406,14 @@ __global__ void __launch_bounds__(C_THREADS)
 
     // ---- epilogue: all 4 warps, TMEM lane quarter = warp -------------------
     const bool ok = mbar_wait(done, 0, &abort_flag, p.status) && !abort_flag;
+    // K split over the cluster: this CTA's MMAs are done, so its ring may now
+    // receive the other ranks' slices. It arrives on the cluster barrier here
+    // and waits on it only after storing its own partial, which hides the
+    // barrier's round trip behind that store.
+    if (S > 1) {
+        __syncwarp();
+        asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+    }
     pdl_wait();                       // (every thread) before reading Y, rows or the table
     asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
     const int row = warp * 32 + lane;
@@ -1477,7 +1485,7 @@ __global__ void __launch_bounds__(C_THREADS)
         };
         if (S > 1) {
             asm volatile("fence.proxy.async.shared::cta;" ::: "memory");    // part, for the bulk copies
-            c_cluster_sync();
+            asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory");
             if (threadIdx.x == 0) {
                 mbar_expect_tx(recv_bar, (uint32_t)((S - 1) * (ps.c_hi - ps.c_lo) * BM * 4));
                 for (int t = 0; t < S; ++t) {
