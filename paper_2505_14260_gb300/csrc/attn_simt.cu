@@ -70,9 +70,9 @@ void launch_attention(const AttnArgs<T> &a, cudaStream_t s) {
     const int threads = 128;
     const int blocks = (int)((warps * 32 + threads - 1) / threads);
     if (a.hd == 128)
-        launch_pdl(attn_simt_kernel<T, 128>, blocks, threads, 0, s, a);
+        launch_chain(attn_simt_kernel<T, 128>, blocks, threads, 0, s, a);
     else
-        launch_pdl(attn_simt_kernel<T, 64>, blocks, threads, 0, s, a);
+        launch_chain(attn_simt_kernel<T, 64>, blocks, threads, 0, s, a);
     note_launch();
 }
 

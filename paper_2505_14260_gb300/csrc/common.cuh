@@ -49,29 +49,26 @@ __device__ __forceinline__ void allow_dependents() {
 }
 
 // Waits until the grids this one depends on have completed and their writes
-// are visible. Every kernel launched by launch_pdl calls it before it reads
-// anything the previous kernel may have written, so that completion stays
-// transitive along the stream.
+// are visible (after a programmatic launch; a no-op after a plain one). Every
+// kernel calls it before it reads anything the previous kernel may have
+// written, so that the order holds however it was launched.
 __device__ __forceinline__ void wait_prior() {
     asm volatile("griddepcontrol.wait;" ::: "memory");
 }
 
-// Launches `kernel` with programmatic stream serialization: its CTAs may be
-// scheduled while the previous kernel on `s` finishes (its launch latency
-// overlaps that kernel's tail); the kernel orders itself with wait_prior().
+// Launches a short kernel in plain stream order behind the previous one. (With
+// programmatic serialization these kernels' griddepcontrol.wait returned
+// later than a plain launch starts: measured slower.) The kernel still calls
+// wait_prior(), a no-op here, and allow_dependents(), which lets a following
+// programmatic launch (the tensor-core GEMMs) start early.
 template <typename... KArgs, typename... Args>
-inline cudaError_t launch_pdl(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
-                              cudaStream_t s, Args &&...args) {
+inline cudaError_t launch_chain(void (*kernel)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                cudaStream_t s, Args &&...args) {
     cudaLaunchConfig_t lc = {};
     lc.gridDim = grid;
     lc.blockDim = block;
     lc.dynamicSmemBytes = smem;
     lc.stream = s;
-    cudaLaunchAttribute at[1];
-    at[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    at[0].val.programmaticStreamSerializationAllowed = 1;
-    lc.attrs = at;
-    lc.numAttrs = 1;
     return cudaLaunchKernelEx(&lc, kernel, std::forward<Args>(args)...);
 }
 

@@ -73,7 +73,7 @@ void launch_gemm_simt(const T *X, int ldx, int M, int K, const GemmW &W, int O, 
                       int ldy, int epi, cudaStream_t s) {
     if (M <= 0 || O <= 0) return;
     dim3 grid((O + SG_BO - 1) / SG_BO, (M + SG_BM - 1) / SG_BM);
-    launch_pdl(gemm_simt_kernel<T>, grid, 256, 0, s, X, ldx, M, K, W, O, Y, ldy, epi); note_launch();
+    launch_chain(gemm_simt_kernel<T>, grid, 256, 0, s, X, ldx, M, K, W, O, Y, ldy, epi); note_launch();
 }
 
 template void launch_gemm_simt<float>(const float *, int, int, int, const GemmW &, int, float *,

@@ -39,7 +39,7 @@ template <typename T>
 void launch_embed_rows(const T *E, const T *vis, const int *src, int R, int H, float *x,
                        T *emb_out, int V, int *status, cudaStream_t s) {
     if (R <= 0) return;
-    launch_pdl(embed_rows_kernel<T>, R, 256, 0, s, E, vis, src, H, x, emb_out, V, status); note_launch();
+    launch_chain(embed_rows_kernel<T>, R, 256, 0, s, E, vis, src, H, x, emb_out, V, status); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -84,7 +84,7 @@ template <typename T>
 void launch_rmsnorm(const float *x, const T *g, int R, int H, float eps, T *out, long lo,
                     cudaStream_t s) {
     if (R <= 0) return;
-    launch_pdl(rmsnorm_kernel<T>, R, RMS_THREADS, 0, s, x, g, H, eps, out, lo); note_launch();
+    launch_chain(rmsnorm_kernel<T>, R, RMS_THREADS, 0, s, x, g, H, eps, out, lo); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -109,7 +109,7 @@ template <typename T>
 void launch_swiglu(const float *gu, int R, int F, bool glu, T *act, long lo, cudaStream_t s) {
     if (R <= 0) return;
     dim3 grid((F + 255) / 256, R);
-    launch_pdl(swiglu_kernel<T>, grid, 256, 0, s, gu, F, glu ? 1 : 0, act, lo); note_launch();
+    launch_chain(swiglu_kernel<T>, grid, 256, 0, s, gu, F, glu ? 1 : 0, act, lo); note_launch();
 }
 
 // ---------------------------------------------------------------------------
@@ -159,7 +159,7 @@ void launch_rope_kv(const float *qkv, const RowDesc *rows, int R, int nh, int hd
                     const float2 *rope_tab, int max_pos, T *q_out, T *kdst, T *vdst,
                     int slots, long lo, int *status, cudaStream_t s) {
     if (R <= 0) return;
-    launch_pdl(rope_kv_kernel<T>, R, 256, 0, s, qkv, rows, nh, hd, rope_tab, max_pos, q_out, kdst,
+    launch_chain(rope_kv_kernel<T>, R, 256, 0, s, qkv, rows, nh, hd, rope_tab, max_pos, q_out, kdst,
                                         vdst, slots, lo, status); note_launch();
 }
 
@@ -412,7 +412,7 @@ void launch_topk_logp(const float *logits, int R, int V, int k, int *ids, float 
     if (R <= 0 || k < 1 || k > TOPK_MAX) return;
     const int nc = topk_chunks(V);
     if (nc * k > 32 * TK_MERGE_SLOTS) return;            // refused at msd_create
-    launch_pdl(topk_rows_kernel, dim3(nc, R), TK_THREADS, 0, s, logits, V, k, ids, logp, sc.ws,
+    launch_chain(topk_rows_kernel, dim3(nc, R), TK_THREADS, 0, s, logits, V, k, ids, logp, sc.ws,
                sc.counters);
     note_launch();
 }
@@ -439,14 +439,14 @@ void launch_convert(const float *x, T *y, long n, cudaStream_t s) {
     if (n <= 0) return;
     long blocks = (n + 255) / 256;
     if (blocks > 4096) blocks = 4096;
-    launch_pdl(convert_kernel<T>, (int)blocks, 256, 0, s, x, y, n); note_launch();
+    launch_chain(convert_kernel<T>, (int)blocks, 256, 0, s, x, y, n); note_launch();
 }
 
 __global__ void flag_status_kernel(int *status, int code) { wait_prior(); set_status(status, code); }
 
 void launch_flag(int *status, int code, cudaStream_t s) {
     cudaGetLastError();
-    launch_pdl(flag_status_kernel, 1, 1, 0, s, status, code);
+    launch_chain(flag_status_kernel, 1, 1, 0, s, status, code);
     note_launch();
 }
 

@@ -847,32 +847,32 @@ template <typename T>
 void launch_catchup_setup(const int *seq_len, const int *n_pend, const T *pend_h,
                           const int *pend_next, const T *E, int B, int H, int D1, int V, T *xfc,
                           long lo, RowDesc *rows, int *status, cudaStream_t s) {
-    launch_pdl(catchup_setup_kernel<T>, B * D1, 256, 0, s, seq_len, n_pend, pend_h, pend_next, E, H, D1,
+    launch_chain(catchup_setup_kernel<T>, B * D1, 256, 0, s, seq_len, n_pend, pend_h, pend_next, E, H, D1,
                                                    V, xfc, lo, rows, status); note_launch();
 }
 
 template <typename T>
 void launch_root_gather(const float *x, const int *n_pend, int B, int D1, int H, float *hhat_root,
                         T *xr, long lo, cudaStream_t s) {
-    launch_pdl(root_gather_kernel<T>, B, 256, 0, s, x, n_pend, D1, H, hhat_root, xr, lo); note_launch();
+    launch_chain(root_gather_kernel<T>, B, 256, 0, s, x, n_pend, D1, H, hhat_root, xr, lo); note_launch();
 }
 
 template <typename T>
 void launch_hhat_store(const float *x, const RowDesc *rows, int R, int Td, int H,
                        float *hhat_slot, T *xb, long lo, cudaStream_t s) {
-    launch_pdl(hhat_store_kernel<T>, R, 256, 0, s, x, rows, Td, H, hhat_slot, xb, lo); note_launch();
+    launch_chain(hhat_store_kernel<T>, R, 256, 0, s, x, rows, Td, H, hhat_slot, xb, lo); note_launch();
 }
 
 template <typename T>
 void launch_tree_init(const DraftArgs<T> &a, int B, cudaStream_t s) {
-    launch_pdl(tree_init_kernel<T>, dim3(a.k, B), 256, 0, s, a);
+    launch_chain(tree_init_kernel<T>, dim3(a.k, B), 256, 0, s, a);
     note_launch();
 }
 
 template <typename T>
 void launch_tree_step(const DraftArgs<T> &a, int B, int d, cudaStream_t s) {
     const size_t sm = (size_t)a.k * a.k * sizeof(float) + (size_t)a.k * sizeof(int);
-    launch_pdl(tree_step_kernel<T>, dim3(a.k, B), 256, sm, s, a, d);
+    launch_chain(tree_step_kernel<T>, dim3(a.k, B), 256, sm, s, a, d);
     note_launch();
 }
 
@@ -882,7 +882,7 @@ void launch_tree_finalize(const TreeOut &t, const int *cand_tok, const int *cand
     const size_t smem = (size_t)C * 3 * sizeof(float);
     // candidate arrays beyond 48 KB (deep, wide trees); the attribute is per device
     cudaFuncSetAttribute(tree_finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, 227 * 1024);
-    launch_pdl(tree_finalize_kernel, B, 512, smem, s, t, cand_tok, cand_par, cand_depth, cand_score, node_of,
+    launch_chain(tree_finalize_kernel, B, 512, smem, s, t, cand_tok, cand_par, cand_depth, cand_score, node_of,
                root, C, N, status);
     note_launch();
 }
@@ -891,19 +891,19 @@ void launch_verify_setup(const TreeIn &t, const int *seq_len, const int *root, i
                          int V, RowDesc *rows, int *src, uint64_t *vmask, int *status,
                          cudaStream_t s) {
     const int R = B * N;
-    launch_pdl(verify_setup_kernel, (R + 127) / 128, 128, 0, s, t, seq_len, root, B, N, V, rows, src,
+    launch_chain(verify_setup_kernel, (R + 127) / 128, 128, 0, s, t, seq_len, root, B, N, V, rows, src,
                                                           vmask, status); note_launch();
 }
 
 void launch_tree_complete(const int *parent, int *depth, uint64_t *mask, const int *n_nodes, int b0, int nb,
                           int N, int *status, cudaStream_t s) {
-    launch_pdl(tree_complete_kernel, nb, 256, 0, s, parent, depth, mask, n_nodes, N, (N + 63) / 64, b0, status);
+    launch_chain(tree_complete_kernel, nb, 256, 0, s, parent, depth, mask, n_nodes, N, (N + 63) / 64, b0, status);
     note_launch();
 }
 
 void launch_root_tree(const int *root, int B, int N, int W, int *tokens, int *parent, int *depth,
                       uint64_t *mask, int *n_nodes, cudaStream_t s) {
-    launch_pdl(root_tree_kernel, (B + 127) / 128, 128, 0, s, root, B, N, W, tokens, parent, depth, mask, n_nodes);
+    launch_chain(root_tree_kernel, (B + 127) / 128, 128, 0, s, root, B, N, W, tokens, parent, depth, mask, n_nodes);
     note_launch();
 }
 
@@ -911,7 +911,7 @@ void launch_accept(const TreeIn &t, const int *argmax, int B, int N, int D, int 
                    int *n_pend, int *root, int *pend_next, int *acc_path, int *acc_L0, int *acc_a,
                    int *path_out, int *accept_len_out, int *bonus_out, int *index_map_out,
                    cudaStream_t s) {
-    launch_pdl(accept_kernel, B, 32, 0, s, t, argmax, N, D, seq_len, n_pend, root, pend_next, acc_path,
+    launch_chain(accept_kernel, B, 32, 0, s, t, argmax, N, D, seq_len, n_pend, root, pend_next, acc_path,
                                    acc_L0, acc_a, path_out, accept_len_out, bonus_out,
                                    index_map_out); note_launch();
 }
@@ -929,12 +929,12 @@ bool launch_accept_sample(const TreeIn &t, const float *logits, int B, int N, in
                              (int)(sizeof(unsigned) * (SAMPLE_MAX_VOCAB / 32))) != cudaSuccess)
         return false;
     const float scale = (float)(1.4426950408889634 * (double)inv_temp);     // log2(e) / T
-    if (launch_pdl(sample_stats_kernel, B * N, STATS_THREADS, 0, s, logits, V, scale, row_max, row_sum) !=
+    if (launch_chain(sample_stats_kernel, B * N, STATS_THREADS, 0, s, logits, V, scale, row_max, row_sum) !=
         cudaSuccess)
         return false;
     note_launch();
     const size_t smem = sizeof(unsigned) * (size_t)((V + 31) / 32);
-    if (launch_pdl(accept_sample_kernel, B, SAMPLE_THREADS, smem, s, t, logits, (const float *)row_max,
+    if (launch_chain(accept_sample_kernel, B, SAMPLE_THREADS, smem, s, t, logits, (const float *)row_max,
                    (const double *)row_sum, N, D, k, V, scale, u, seq_len, n_pend, root, pend_next, acc_path,
                    acc_L0, acc_a, path_out, accept_len_out, bonus_out, index_map_out, status) != cudaSuccess)
         return false;
@@ -947,7 +947,7 @@ void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, co
                        int row_bytes, long lo_bytes, int *status, cudaStream_t s) {
     dim3 grid(n_layers * 2 * nh, B);
     const long lo_vec = lo_bytes / 16;      // both lo planes sit lo_bytes after their hi planes
-    launch_pdl(compact_kv_kernel, grid, 128, 0, s, static_cast<const uint4 *>(tree_kv),
+    launch_chain(compact_kv_kernel, grid, 128, 0, s, static_cast<const uint4 *>(tree_kv),
                                            static_cast<uint4 *>(cache), acc_path, acc_L0, acc_a,
                                            B, nh, N, S, D1, row_bytes / 16, lo_vec, lo_vec, status); note_launch();
 }
@@ -955,26 +955,26 @@ void launch_compact_kv(const void *tree_kv, void *cache, const int *acc_path, co
 template <typename T>
 void launch_pend_h(const T *hT, const int *acc_path, const int *acc_a, int B, int N, int D1,
                    int H, T *pend_h, long lo, cudaStream_t s) {
-    launch_pdl(pend_h_kernel<T>, B * D1, 256, 0, s, hT, acc_path, acc_a, N, D1, H, pend_h, lo); note_launch();
+    launch_chain(pend_h_kernel<T>, B * D1, 256, 0, s, hT, acc_path, acc_a, N, D1, H, pend_h, lo); note_launch();
 }
 
 template <typename T>
 void launch_select_visual(float *x, const T *emb, long slo, const int *src, int R, int H, cudaStream_t s) {
     if (R <= 0) return;
-    launch_pdl(select_visual_kernel<T>, R, 256, 0, s, x, emb, slo, src, H); note_launch();
+    launch_chain(select_visual_kernel<T>, R, 256, 0, s, x, emb, slo, src, H); note_launch();
 }
 
 template <typename T>
 void launch_concat_next(const T *h, const T *emb, int R, int H, T *xfc, long lo, cudaStream_t s) {
     if (R <= 0) return;
-    launch_pdl(concat_next_kernel<T>, R, 256, 0, s, h, emb, H, xfc, lo); note_launch();
+    launch_chain(concat_next_kernel<T>, R, 256, 0, s, h, emb, H, xfc, lo); note_launch();
 }
 
 template <typename T>
 void launch_prefill_finish(const int *argmax1, const T *h_last, int b, int L, int D1, int H,
                            int *seq_len, int *n_pend, int *root, int *pend_next, T *pend_h, long lo,
                            int *root_out, cudaStream_t s) {
-    launch_pdl(prefill_finish_kernel<T>, 1, 256, 0, s, argmax1, h_last, b, L, D1, H, seq_len, n_pend,
+    launch_chain(prefill_finish_kernel<T>, 1, 256, 0, s, argmax1, h_last, b, L, D1, H, seq_len, n_pend,
                                                root, pend_next, pend_h, lo, root_out); note_launch();
 }
 
