@@ -87,15 +87,15 @@ def parse():
 
 # DRAM traffic of the GEMMs: ncu dram__bytes_read.sum + dram__bytes_write.sum
 # per launch divided by the same launches' algorithmic bytes. Decode
-# (gemm_cluster_kernel): the 90 launches of two 2-layer 7B-width steps, 0.9947
+# (gemm_cluster_kernel): the 90 launches of two 2-layer 7B-width steps, 0.9945
 # (no re-reads). Many rows (gemm_persist_kernel): the first two many-row
 # launches of a 2-layer batch-16 step (the draft's input projection and q/k/v at
 # 160 token rows), 0.975 (0.997 and 0.960: part of q/k/v's fp32 output is still
 # in L2 when the launch ends). Per launch of a full workload it is the ratio
 # times its algorithmic bytes per launch. Valid for the GEMM source with this
 # SHA-1 only.
-GEMM_TRAFFIC = {"source_sha1": "b06a5a07809661b97a8943189afe56ae80fc02fb",
-                "ratio": {"hbm": 0.9947, "tensor": 0.975}}
+GEMM_TRAFFIC = {"source_sha1": "af8b12bbe0baebb332dc96e69230605bb01a881e",
+                "ratio": {"hbm": 0.9945, "tensor": 0.975}}
 
 
 def gemm_traffic(bytes_per_launch, bound="hbm"):
