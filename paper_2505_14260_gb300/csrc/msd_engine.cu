@@ -1252,8 +1252,10 @@ msd_status msd_profile_slots(msd_ctx *c, msd_kernel_slot *out, int32_t max, int3
     if (!c || !n || max < 0 || (max > 0 && !out)) return MSD_ERR_INVALID;
     *n = 0;
     if (!c->gplan || max == 0) return MSD_OK;
-    std::vector<GemmSlot> g((size_t)max);
-    const int k = gemm_profile_slots(c->gplan, g.data(), max);
+    // (a window holds at most 2560 stamped launches)
+    const int cap = std::min<int32_t>(max, 4096);
+    std::vector<GemmSlot> g((size_t)cap);
+    const int k = gemm_profile_slots(c->gplan, g.data(), cap);
     if (k < 0) return fail(c, MSD_ERR_CUDA, "reading the stamp slots failed");
     for (int i = 0; i < k; ++i) {
         out[i].kind = g[i].kind;
